@@ -1,0 +1,214 @@
+"""QuantEase fp64 CPU oracle (Behdin et al., arXiv 2309.01885).
+
+TEST INFRASTRUCTURE ONLY.  Only the tests, ``__graft_entry__.smoke()`` and the
+CPU-baseline leg of ``bench.py`` import this package.  It shares no code with the
+CUDA library (``paper_2309_01885_gb300``) and never imports it.
+
+The arithmetic lives in ``qe_oracle.c`` (plain C, binary64, OpenMP over the
+independent rows of Sec. 3.2); this module compiles it with gcc and marshals
+numpy arrays through ctypes.  Parity pins: ``tests/test_oracle_*.py``.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+SRC = os.path.join(_HERE, "qe_oracle.c")
+LIB = os.path.join(_HERE, "_build", "libqe_oracle.so")
+CFLAGS = ["-O2", "-fopenmp", "-ffp-contract=off", "-fPIC", "-shared", "-std=c11"]
+
+
+def build(src: str = SRC, out: str = LIB, force: bool = False) -> str:
+    """Compile the oracle shared library with gcc; returns its path."""
+    if not force and os.path.exists(out) and os.path.getmtime(out) >= os.path.getmtime(src):
+        return out
+    os.makedirs(os.path.dirname(out), exist_ok=True)
+    tmp = out + f".tmp{os.getpid()}"
+    subprocess.check_call(["gcc", *CFLAGS, "-o", tmp, src, "-lm"])
+    os.replace(tmp, out)
+    return out
+
+
+_u8p = ctypes.POINTER(ctypes.c_uint8)
+_f32p = ctypes.POINTER(ctypes.c_float)
+_f64p = ctypes.POINTER(ctypes.c_double)
+_i64p = ctypes.POINTER(ctypes.c_int64)
+_i64 = ctypes.c_int64
+_int = ctypes.c_int
+
+
+def _ptr(a, typ):
+    if a is None:
+        return None
+    return a.ctypes.data_as(typ)
+
+
+def _f64(a):
+    return np.ascontiguousarray(a, dtype=np.float64)
+
+
+class Oracle:
+    """ctypes front end over one build of ``qe_oracle.c``."""
+
+    def __init__(self, path: str | None = None):
+        self.path = path or build()
+        lib = ctypes.CDLL(self.path)
+        lib.qo_grid.argtypes = [_f64p, _i64, _i64, _int, _u8p, _f32p, _f32p]
+        lib.qo_grid.restype = None
+        lib.qo_rtn.argtypes = [_f64p, _i64, _i64, _f32p, _f32p, _int, _u8p]
+        lib.qo_rtn.restype = None
+        lib.qo_sigma.argtypes = [_f64p, _i64, _i64, _f64p]
+        lib.qo_sigma.restype = None
+        lib.qo_objective_rows.argtypes = [_f64p, _f64p, _u8p, _f32p, _f32p, _i64, _i64, _f64p, _f64p]
+        lib.qo_objective_rows.restype = None
+        lib.qo_quantease_alg1.argtypes = [_f64p, _i64, _i64, _f64p, _f32p, _f32p, _int, _int,
+                                          _u8p, _u8p, _u8p, _f64p, _u8p, _f64p]
+        lib.qo_quantease_alg1.restype = _int
+        lib.qo_quantease_alg3.argtypes = [_f64p, _i64, _i64, _f64p, _f32p, _f32p, _int, _int,
+                                          _u8p, _f64p]
+        lib.qo_quantease_alg3.restype = _int
+        lib.qo_power_lambda.argtypes = [_f64p, _i64, _int]
+        lib.qo_power_lambda.restype = ctypes.c_double
+        lib.qo_topk.argtypes = [_f64p, _i64, _i64, _i64p]
+        lib.qo_topk.restype = _i64
+        lib.qo_quantease_outlier.argtypes = [_f64p, _i64, _i64, _f64p, _int, _int, _i64, _int,
+                                             _u8p, _f32p, _f32p, _f64p, _f64p, _f64p, _f64p, _i64p]
+        lib.qo_quantease_outlier.restype = _int
+        self.lib = lib
+
+    # -- grid ---------------------------------------------------------------
+    def grid(self, W, bits, excl=None):
+        """Per-row (scale, zero) of the asymmetric min/max grid (binary32)."""
+        W = _f64(W)
+        q, p = W.shape
+        scale = np.empty(q, np.float32)
+        zero = np.empty(q, np.float32)
+        ex = None if excl is None else np.ascontiguousarray(excl, dtype=np.uint8)
+        self.lib.qo_grid(_ptr(W, _f64p), q, p, bits, _ptr(ex, _u8p),
+                         _ptr(scale, _f32p), _ptr(zero, _f32p))
+        return scale, zero
+
+    def rtn(self, W, scale, zero, bits):
+        W = _f64(W)
+        q, p = W.shape
+        codes = np.empty((q, p), np.uint8)
+        self.lib.qo_rtn(_ptr(W, _f64p), q, p, _ptr(np.ascontiguousarray(scale, np.float32), _f32p),
+                        _ptr(np.ascontiguousarray(zero, np.float32), _f32p), bits, _ptr(codes, _u8p))
+        return codes
+
+    # -- Sigma / objective --------------------------------------------------
+    def sigma(self, X):
+        X = _f64(X)
+        p, n = X.shape
+        S = np.empty((p, p), np.float64)
+        self.lib.qo_sigma(_ptr(X, _f64p), p, n, _ptr(S, _f64p))
+        return S
+
+    def objective_rows(self, W, codes, scale, zero, S, H=None):
+        W = _f64(W)
+        q, p = W.shape
+        out = np.empty(q, np.float64)
+        Hc = None if H is None else _f64(H)
+        self.lib.qo_objective_rows(_ptr(W, _f64p), _ptr(Hc, _f64p),
+                                   _ptr(np.ascontiguousarray(codes, np.uint8), _u8p),
+                                   _ptr(np.ascontiguousarray(scale, np.float32), _f32p),
+                                   _ptr(np.ascontiguousarray(zero, np.float32), _f32p),
+                                   q, p, _ptr(_f64(S), _f64p), _ptr(out, _f64p))
+        return out
+
+    # -- Algorithm 1 / 3 ----------------------------------------------------
+    def alg1(self, W, S, scale, zero, bits, iters, init_codes=None, forced=None,
+             record=False, want_beta=False):
+        """Algorithm 1.  Returns dict(codes, obj_rows[iters, q], obj[iters],
+        sweep_codes[iters, q, p] if record, beta[iters, q, p] if want_beta)."""
+        W = _f64(W)
+        S = _f64(S)
+        q, p = W.shape
+        codes = np.empty((q, p), np.uint8)
+        obj_rows = np.empty((iters, q), np.float64)
+        sweep = np.empty((iters, q, p), np.uint8) if record else None
+        beta = np.empty((iters, q, p), np.float64) if want_beta else None
+        ic = None if init_codes is None else np.ascontiguousarray(init_codes, np.uint8)
+        fc = None if forced is None else np.ascontiguousarray(forced, np.uint8)
+        rc = self.lib.qo_quantease_alg1(
+            _ptr(W, _f64p), q, p, _ptr(S, _f64p),
+            _ptr(np.ascontiguousarray(scale, np.float32), _f32p),
+            _ptr(np.ascontiguousarray(zero, np.float32), _f32p), bits, iters,
+            _ptr(ic, _u8p), _ptr(fc, _u8p), _ptr(codes, _u8p), _ptr(obj_rows, _f64p),
+            _ptr(sweep, _u8p), _ptr(beta, _f64p))
+        if rc:
+            raise MemoryError("oracle alg1 allocation failed")
+        out = dict(codes=codes, obj_rows=obj_rows, obj=obj_rows.sum(axis=1))
+        if record:
+            out["sweep_codes"] = sweep
+        if want_beta:
+            out["beta"] = beta
+        return out
+
+    def alg3(self, W, S, scale, zero, bits, iters):
+        W = _f64(W)
+        S = _f64(S)
+        q, p = W.shape
+        codes = np.empty((q, p), np.uint8)
+        obj_rows = np.empty((iters, q), np.float64)
+        rc = self.lib.qo_quantease_alg3(
+            _ptr(W, _f64p), q, p, _ptr(S, _f64p),
+            _ptr(np.ascontiguousarray(scale, np.float32), _f32p),
+            _ptr(np.ascontiguousarray(zero, np.float32), _f32p), bits, iters,
+            _ptr(codes, _u8p), _ptr(obj_rows, _f64p))
+        if rc:
+            raise MemoryError("oracle alg3 allocation failed")
+        return dict(codes=codes, obj_rows=obj_rows, obj=obj_rows.sum(axis=1))
+
+    # -- outlier-aware (Algorithm 4) ----------------------------------------
+    def power_lambda(self, S, iters):
+        S = _f64(S)
+        return float(self.lib.qo_power_lambda(_ptr(S, _f64p), S.shape[0], iters))
+
+    def topk(self, T, s):
+        T = _f64(T).ravel()
+        idx = np.empty(max(int(s), 1), np.int64)
+        cnt = self.lib.qo_topk(_ptr(T, _f64p), T.size, int(s), _ptr(idx, _i64p))
+        return idx[:cnt].copy()
+
+    def outlier(self, W, S, bits, iters, s_budget, power_iters):
+        W = _f64(W)
+        S = _f64(S)
+        q, p = W.shape
+        codes = np.empty((q, p), np.uint8)
+        scale = np.empty(q, np.float32)
+        zero = np.empty(q, np.float32)
+        H = np.empty((q, p), np.float64)
+        obj = np.empty(iters, np.float64)
+        obj_cd = np.empty(iters, np.float64)
+        eta = np.zeros(1, np.float64)
+        nnz = np.zeros(1, np.int64)
+        rc = self.lib.qo_quantease_outlier(
+            _ptr(W, _f64p), q, p, _ptr(S, _f64p), bits, iters, int(s_budget), power_iters,
+            _ptr(codes, _u8p), _ptr(scale, _f32p), _ptr(zero, _f32p), _ptr(H, _f64p),
+            _ptr(obj, _f64p), _ptr(obj_cd, _f64p), _ptr(eta, _f64p), _ptr(nnz, _i64p))
+        if rc:
+            raise MemoryError("oracle outlier allocation failed")
+        return dict(codes=codes, scale=scale, zero=zero, H=H, obj=obj, obj_cd=obj_cd,
+                    eta=float(eta[0]), nnz=int(nnz[0]))
+
+
+_default: Oracle | None = None
+
+
+def get() -> Oracle:
+    """The oracle built from ``qe_oracle.c`` (compiled on first use)."""
+    global _default
+    if _default is None:
+        _default = Oracle()
+    return _default
+
+
+def levels(codes, scale, zero):
+    """Dequantised values s_i (c - z_i) in binary64."""
+    return np.asarray(scale, np.float64)[:, None] * (np.asarray(codes, np.float64)
+                                                     - np.asarray(zero, np.float64)[:, None])

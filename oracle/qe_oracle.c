@@ -1,0 +1,529 @@
+/*
+ * QuantEase oracle: a plain, slow, binary64 CPU restatement of the layer-wise
+ * quantization method of Behdin et al., "QuantEase: Optimization-based
+ * Quantization for Language Models" (arXiv 2309.01885).
+ *
+ * TEST INFRASTRUCTURE ONLY. This file is compiled into its own shared library
+ * (oracle/_build/libqe_oracle.so) that only the test-suite, the smoke check and
+ * the CPU-baseline leg of bench.py load. It shares no code, header, table or
+ * constant with the CUDA library, and the product path never calls it.
+ *
+ * Conventions (Sec. 2.1): matrices are row-major; W is q x p (q output channels,
+ * p input features), X is p x n, Sigma = X X^T is p x p.  All arithmetic is
+ * binary64, except the per-row grid (scale, zero-point): its zero-point is an
+ * integer decided by a division, and that decision is taken in binary32 here as
+ * in the GPU path, so that both sides decide it identically.
+ *
+ * Every function below is pinned by the CPU tests in tests/test_oracle_*.py
+ * (brute-force 1-D argmin, exhaustive search on tiny layers, monotone
+ * objective, Algorithm 1 == Algorithm 3, diagonal Sigma == round-to-nearest,
+ * direct ||WX - W^X||^2, eigvalsh for lambda_max, a full sort for P_s, and
+ * the IHT descent of Lemma 3).  The relax-every-third-iteration heuristic of
+ * Sec. 3.2 is not implemented here (parity unpinned, not on the hot path).
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+/* ------------------------------------------------------------------------- */
+/* Quantization grid and operator                                            */
+/* ------------------------------------------------------------------------- */
+
+/*
+ * Per-channel uniform grid Q_i (Sec. 2.1, "uniformly spaced, following GPTQ"):
+ * levels s_i * (c - z_i), c = 0 .. 2^b - 1, asymmetric min/max over row i with
+ * 0 always inside the range; an all-zero row gets the range [-1, 1].
+ * excl (q*p bytes, may be NULL) removes entries from the pool; with 0 always in
+ * the range this is the same as setting them to 0 (Sec. 4.3, outliers removed
+ * from the quantization pool).  Evaluated in binary32 (see file header).
+ */
+void qo_grid(const double *W, int64_t q, int64_t p, int bits,
+             const uint8_t *excl, float *scale, float *zero)
+{
+    const float maxq = (float)((1 << bits) - 1);
+    for (int64_t i = 0; i < q; ++i) {
+        float lo = 0.0f, hi = 0.0f;
+        for (int64_t j = 0; j < p; ++j) {
+            if (excl && excl[i * p + j])
+                continue;
+            float w = (float)W[i * p + j];
+            if (w < lo) lo = w;
+            if (w > hi) hi = w;
+        }
+        if (lo == 0.0f && hi == 0.0f) {
+            lo = -1.0f;
+            hi = 1.0f;
+        }
+        float s = (hi - lo) / maxq;
+        float z = nearbyintf(-lo / s);
+        scale[i] = s;
+        zero[i] = z;
+    }
+}
+
+/*
+ * q_i of Eq. (eq:quant): the nearest level to x.  With levels s (c - z) and
+ * s > 0, |x - s (c - z)| is minimised over integers c by the integer nearest
+ * to x / s + z, clamped to [0, 2^b - 1] (a convex 1-D distance).  Exact ties
+ * go to the even integer (round-half-to-even).  Returns the code c.
+ */
+static int qo_code(double x, double s, double z, int maxq)
+{
+    double c = nearbyint(x / s + z);
+    if (c < 0.0) c = 0.0;
+    if (c > (double)maxq) c = (double)maxq;
+    return (int)c;
+}
+
+static double qo_level(int c, double s, double z)
+{
+    return s * ((double)c - z);
+}
+
+/* Round-to-nearest of a whole matrix on the grid (used for dead columns). */
+void qo_rtn(const double *W, int64_t q, int64_t p, const float *scale,
+            const float *zero, int bits, uint8_t *codes)
+{
+    const int maxq = (1 << bits) - 1;
+    for (int64_t i = 0; i < q; ++i)
+        for (int64_t j = 0; j < p; ++j)
+            codes[i * p + j] = (uint8_t)qo_code(W[i * p + j], scale[i], zero[i], maxq);
+}
+
+/* ------------------------------------------------------------------------- */
+/* Sigma and objective                                                       */
+/* ------------------------------------------------------------------------- */
+
+/* Sigma = X X^T (Lemma 1), X p x n row-major, Sigma p x p. */
+void qo_sigma(const double *X, int64_t p, int64_t n, double *S)
+{
+#pragma omp parallel for schedule(dynamic)
+    for (int64_t a = 0; a < p; ++a) {
+        for (int64_t b = a; b < p; ++b) {
+            double acc = 0.0;
+            for (int64_t k = 0; k < n; ++k)
+                acc += X[a * n + k] * X[b * n + k];
+            S[a * p + b] = acc;
+            S[b * p + a] = acc;
+        }
+    }
+}
+
+/* d^T Sigma d for one row d (the per-row term of f = tr(D Sigma D^T), proof of Lemma 1). */
+static double qo_quad(const double *d, const double *S, int64_t p)
+{
+    double f = 0.0;
+    for (int64_t a = 0; a < p; ++a) {
+        if (d[a] == 0.0)
+            continue;
+        double t = 0.0;
+        for (int64_t b = 0; b < p; ++b)
+            t += S[a * p + b] * d[b];
+        f += d[a] * t;
+    }
+    return f;
+}
+
+/*
+ * Per-row objective f_i = (T_i - What_i) Sigma (T_i - What_i)^T of Eq.
+ * (layerwise-main), What = s (codes - z) plus the optional dense H (Eq.
+ * main-outlier: g = ||W X - (What + H) X||^2).  rows_out[i] = f_i.
+ */
+void qo_objective_rows(const double *W, const double *H, const uint8_t *codes,
+                       const float *scale, const float *zero, int64_t q, int64_t p,
+                       const double *S, double *rows_out)
+{
+#pragma omp parallel for schedule(dynamic)
+    for (int64_t i = 0; i < q; ++i) {
+        double *d = (double *)malloc((size_t)p * sizeof(double));
+        for (int64_t j = 0; j < p; ++j) {
+            double wh = qo_level(codes[i * p + j], scale[i], zero[i]);
+            d[j] = W[i * p + j] - wh - (H ? H[i * p + j] : 0.0);
+        }
+        rows_out[i] = qo_quad(d, S, p);
+        free(d);
+    }
+}
+
+/* ------------------------------------------------------------------------- */
+/* Algorithm 1 (basic QuantEase, rank-1 bookkeeping of What Sigma)           */
+/* ------------------------------------------------------------------------- */
+
+/*
+ * One cyclic sweep j = 1..p of Algorithm 1 on one row (rows are independent,
+ * Sec. 3.2 "Parallelization over i").
+ *   Wh   : current row of What (in/out)
+ *   WS   : (What Sigma)_i,:  kept current by the rank-1 updates of Eq. (rank1-update)
+ *   TS   : (T Sigma)_i,: for the fixed target T (T = W, or W - H in Algorithm 4)
+ *   tgt  : the target row T_i (used for dead columns only)
+ * For each column j: u = [(What Sigma)_ij - Sigma_jj What_ij - (T Sigma)_ij] / Sigma_jj
+ * (so -u is beta~ of Lemma 1), remove the old column (part A), set
+ * What_ij = q_i(-u), add the new column (part B).
+ * A dead column (Sigma_jj <= 0, i.e. X_j,: = 0, footnote of Lemma 1) drops out
+ * of the objective; it is set to the nearest level of the target and fixed.
+ * forced (p codes, may be NULL): use these codes instead of q_i(-u) (teacher
+ * forcing; beta~ is still recorded).  beta (p, may be NULL) receives beta~.
+ */
+static void qo_sweep_row(const double *S, int64_t p, double s, double z, int maxq,
+                         const double *tgt, const double *TS, double *Wh, double *WS,
+                         const uint8_t *forced, uint8_t *codes, double *beta)
+{
+    for (int64_t j = 0; j < p; ++j) {
+        const double *Sj = S + j * p;
+        const double djj = Sj[j];
+        int c;
+        if (djj > 0.0) {
+            double u = (WS[j] - djj * Wh[j] - TS[j]) / djj;
+            double b = -u;
+            double old = Wh[j];
+            for (int64_t k = 0; k < p; ++k)          /* part (A) */
+                WS[k] -= old * Sj[k];
+            c = forced ? (int)forced[j] : qo_code(b, s, z, maxq);
+            Wh[j] = qo_level(c, s, z);
+            for (int64_t k = 0; k < p; ++k)          /* part (B) */
+                WS[k] += Wh[j] * Sj[k];
+            if (beta) beta[j] = b;
+        } else {
+            c = forced ? (int)forced[j] : qo_code(tgt[j], s, z, maxq);
+            Wh[j] = qo_level(c, s, z);
+            if (beta) beta[j] = tgt[j];
+        }
+        codes[j] = (uint8_t)c;
+    }
+}
+
+/* y = x Sigma for a row vector x. */
+static void qo_row_times_sigma(const double *x, const double *S, int64_t p, double *y)
+{
+    for (int64_t k = 0; k < p; ++k)
+        y[k] = 0.0;
+    for (int64_t l = 0; l < p; ++l) {
+        if (x[l] == 0.0)
+            continue;
+        const double *Sl = S + l * p;
+        for (int64_t k = 0; k < p; ++k)
+            y[k] += x[l] * Sl[k];
+    }
+}
+
+/*
+ * Algorithm 1.  Start: What = W (Sec. 3.1), or the levels of init_codes.
+ *   codes       q*p   out: codes after the last sweep
+ *   obj_rows    iters*q out (may be NULL): f_i after each sweep
+ *   sweep_codes iters*q*p out (may be NULL): codes after each sweep
+ *   forced      iters*q*p in (may be NULL): teacher-forced codes per sweep
+ *   beta        iters*q*p out (may be NULL): beta~ of every update
+ */
+int qo_quantease_alg1(const double *W, int64_t q, int64_t p, const double *S,
+                      const float *scale, const float *zero, int bits, int iters,
+                      const uint8_t *init_codes, const uint8_t *forced,
+                      uint8_t *codes, double *obj_rows, uint8_t *sweep_codes,
+                      double *beta)
+{
+    const int maxq = (1 << bits) - 1;
+    int err = 0;
+#pragma omp parallel for schedule(dynamic)
+    for (int64_t i = 0; i < q; ++i) {
+        double *Wh = (double *)malloc((size_t)p * sizeof(double));
+        double *WS = (double *)malloc((size_t)p * sizeof(double));
+        double *TS = (double *)malloc((size_t)p * sizeof(double));
+        double *d = (double *)malloc((size_t)p * sizeof(double));
+        if (!Wh || !WS || !TS || !d) {
+            err = 1;
+        } else {
+            const double *Wi = W + i * p;
+            const double s = scale[i], z = zero[i];
+            for (int64_t j = 0; j < p; ++j)
+                Wh[j] = init_codes ? qo_level(init_codes[i * p + j], s, z) : Wi[j];
+            qo_row_times_sigma(Wh, S, p, WS);
+            qo_row_times_sigma(Wi, S, p, TS);
+            for (int t = 0; t < iters; ++t) {
+                const size_t off = ((size_t)t * (size_t)q + (size_t)i) * (size_t)p;
+                qo_sweep_row(S, p, s, z, maxq, Wi, TS, Wh, WS,
+                             forced ? forced + off : NULL, codes + i * p,
+                             beta ? beta + off : NULL);
+                if (sweep_codes)
+                    memcpy(sweep_codes + off, codes + i * p, (size_t)p);
+                if (obj_rows) {
+                    for (int64_t j = 0; j < p; ++j)
+                        d[j] = Wi[j] - Wh[j];
+                    obj_rows[(size_t)t * (size_t)q + (size_t)i] = qo_quad(d, S, p);
+                }
+            }
+        }
+        free(Wh); free(WS); free(TS); free(d);
+    }
+    return err;
+}
+
+/* ------------------------------------------------------------------------- */
+/* Algorithm 3 (accelerated QuantEase with partial update)                   */
+/* ------------------------------------------------------------------------- */
+
+/*
+ * Algorithm 3, written independently of Algorithm 1 as a second form that must
+ * agree with it in exact arithmetic (Sec. 3.2, Eq. cd-update-closed-2):
+ *   Sn_:,j = Sigma_:,j / Sigma_jj;  P = W Sn (diagonal still 1);  then Sn_jj = 0.
+ *   per sweep: dW = What;  Ph = What Sn;
+ *     per column j: beta = P_:,j - Ph_:,j + dW_:,1:j Sn_1:j,j;  What_:,j = q(beta);
+ *                   dW_:,j -= What_:,j.
+ * Dead columns (Sigma_jj <= 0) are set to the nearest level of W and fixed.
+ */
+int qo_quantease_alg3(const double *W, int64_t q, int64_t p, const double *S,
+                      const float *scale, const float *zero, int bits, int iters,
+                      uint8_t *codes, double *obj_rows)
+{
+    const int maxq = (1 << bits) - 1;
+    double *Sn = (double *)malloc((size_t)p * (size_t)p * sizeof(double));
+    if (!Sn)
+        return 1;
+    for (int64_t k = 0; k < p; ++k)
+        for (int64_t j = 0; j < p; ++j) {
+            double djj = S[j * p + j];
+            Sn[k * p + j] = djj > 0.0 ? S[k * p + j] / djj : 0.0;
+        }
+    int err = 0;
+#pragma omp parallel for schedule(dynamic)
+    for (int64_t i = 0; i < q; ++i) {
+        double *P = (double *)malloc((size_t)p * sizeof(double));
+        double *Ph = (double *)malloc((size_t)p * sizeof(double));
+        double *Wh = (double *)malloc((size_t)p * sizeof(double));
+        double *dW = (double *)malloc((size_t)p * sizeof(double));
+        if (!P || !Ph || !Wh || !dW) {
+            err = 1;
+        } else {
+            const double *Wi = W + i * p;
+            const double s = scale[i], z = zero[i];
+            /* P = W Sn with the unit diagonal, before the diagonal is zeroed */
+            for (int64_t j = 0; j < p; ++j) {
+                double acc = 0.0;
+                for (int64_t k = 0; k < p; ++k)
+                    acc += Wi[k] * Sn[k * p + j];
+                P[j] = acc;
+            }
+            for (int64_t j = 0; j < p; ++j)
+                Wh[j] = Wi[j];
+            for (int t = 0; t < iters; ++t) {
+                for (int64_t j = 0; j < p; ++j)
+                    dW[j] = Wh[j];
+                /* Ph = What Sn with Sn_jj = 0 */
+                for (int64_t j = 0; j < p; ++j) {
+                    double acc = 0.0;
+                    for (int64_t k = 0; k < p; ++k)
+                        if (k != j)
+                            acc += Wh[k] * Sn[k * p + j];
+                    Ph[j] = acc;
+                }
+                for (int64_t j = 0; j < p; ++j) {
+                    int c;
+                    if (S[j * p + j] > 0.0) {
+                        double b = P[j] - Ph[j];
+                        for (int64_t k = 0; k < j; ++k)   /* k = j adds Sn_jj = 0 */
+                            b += dW[k] * Sn[k * p + j];
+                        c = qo_code(b, s, z, maxq);
+                    } else {
+                        c = qo_code(Wi[j], s, z, maxq);
+                    }
+                    Wh[j] = qo_level(c, s, z);
+                    dW[j] -= Wh[j];
+                    codes[i * p + j] = (uint8_t)c;
+                }
+                if (obj_rows) {
+                    double *d = Ph; /* reuse */
+                    for (int64_t j = 0; j < p; ++j)
+                        d[j] = Wi[j] - Wh[j];
+                    obj_rows[(size_t)t * (size_t)q + (size_t)i] = qo_quad(d, S, p);
+                }
+            }
+        }
+        free(P); free(Ph); free(Wh); free(dW);
+    }
+    free(Sn);
+    return err;
+}
+
+/* ------------------------------------------------------------------------- */
+/* Outlier-aware QuantEase (Sec. 4, Algorithm 4)                             */
+/* ------------------------------------------------------------------------- */
+
+/*
+ * lambda_max(Sigma) by the power method (Sec. 4.3, "iterative power method"):
+ * v0 = 1/sqrt(p) * ones;  iters times: v <- Sigma v / ||Sigma v||;
+ * return the Rayleigh quotient v^T Sigma v.
+ */
+double qo_power_lambda(const double *S, int64_t p, int iters)
+{
+    double *v = (double *)malloc((size_t)p * sizeof(double));
+    double *w = (double *)malloc((size_t)p * sizeof(double));
+    for (int64_t k = 0; k < p; ++k)
+        v[k] = 1.0 / sqrt((double)p);
+    double lam = 0.0;
+    for (int it = 0; it <= iters; ++it) {
+        for (int64_t a = 0; a < p; ++a) {
+            double acc = 0.0;
+            for (int64_t b = 0; b < p; ++b)
+                acc += S[a * p + b] * v[b];
+            w[a] = acc;
+        }
+        if (it == iters) {
+            lam = 0.0;
+            for (int64_t a = 0; a < p; ++a)
+                lam += v[a] * w[a];
+            break;
+        }
+        double nrm = 0.0;
+        for (int64_t a = 0; a < p; ++a)
+            nrm += w[a] * w[a];
+        nrm = sqrt(nrm);
+        if (nrm == 0.0)
+            break;
+        for (int64_t a = 0; a < p; ++a)
+            v[a] = w[a] / nrm;
+    }
+    free(v);
+    free(w);
+    return lam;
+}
+
+typedef struct {
+    double key;
+    int64_t idx;
+} qo_kv;
+
+static int qo_kv_cmp(const void *a, const void *b)
+{
+    const qo_kv *x = (const qo_kv *)a, *y = (const qo_kv *)b;
+    if (x->key > y->key) return -1;      /* larger magnitude first */
+    if (x->key < y->key) return 1;
+    if (x->idx < y->idx) return -1;      /* tie: smaller linear index first */
+    if (x->idx > y->idx) return 1;
+    return 0;
+}
+
+static int qo_i64_cmp(const void *a, const void *b)
+{
+    int64_t x = *(const int64_t *)a, y = *(const int64_t *)b;
+    return (x > y) - (x < y);
+}
+
+/*
+ * P_s of Eq. (iht-update): keep the s entries of largest |T| (over all q*p
+ * entries), zero the rest.  Ties at the threshold go to the smaller row-major
+ * index; exact zeros are never kept.  idx_out receives the kept linear indices
+ * in ascending order; returns their count (<= s).
+ */
+int64_t qo_topk(const double *T, int64_t N, int64_t s, int64_t *idx_out)
+{
+    qo_kv *kv = (qo_kv *)malloc((size_t)(N > 0 ? N : 1) * sizeof(qo_kv));
+    int64_t m = 0;
+    for (int64_t k = 0; k < N; ++k) {
+        double a = fabs(T[k]);
+        if (a > 0.0) {
+            kv[m].key = a;
+            kv[m].idx = k;
+            ++m;
+        }
+    }
+    qsort(kv, (size_t)m, sizeof(qo_kv), qo_kv_cmp);
+    int64_t cnt = m < s ? m : s;
+    for (int64_t k = 0; k < cnt; ++k)
+        idx_out[k] = kv[k].idx;
+    qsort(idx_out, (size_t)cnt, sizeof(int64_t), qo_i64_cmp);
+    free(kv);
+    return cnt;
+}
+
+/*
+ * Algorithm 4 (outlier-aware QuantEase), block coordinate descent between What
+ * and H (Sec. 4.3):
+ *   H = P_s(W); grid from W without the support of H; What = W - H;
+ *   eta = 1 / (2 lambda_max(Sigma));
+ *   per iteration t:
+ *     one sweep of Algorithm 1 on every row with target W - H;   obj_cd[t] = g
+ *     G = 2 (H + What - W) Sigma;  H = P_s(H - eta G);           obj[t]    = g
+ * Outputs: codes, scale, zero, dense H (q*p), obj, obj_cd (iters each), eta.
+ */
+int qo_quantease_outlier(const double *W, int64_t q, int64_t p, const double *S,
+                         int bits, int iters, int64_t s_budget, int power_iters,
+                         uint8_t *codes, float *scale, float *zero, double *H,
+                         double *obj, double *obj_cd, double *eta_out,
+                         int64_t *nnz_out)
+{
+    const int maxq = (1 << bits) - 1;
+    const int64_t N = q * p;
+    int64_t *idx = (int64_t *)malloc((size_t)(s_budget > 0 ? s_budget : 1) * sizeof(int64_t));
+    uint8_t *excl = (uint8_t *)calloc((size_t)N, 1);
+    double *Wh = (double *)malloc((size_t)N * sizeof(double));
+    double *T = (double *)malloc((size_t)N * sizeof(double));
+    double *rows = (double *)malloc((size_t)q * sizeof(double));
+    if (!idx || !excl || !Wh || !T || !rows)
+        return 1;
+
+    /* H = P_s(W), grid without the support of H, What = W - H */
+    int64_t nnz = qo_topk(W, N, s_budget, idx);
+    memset(H, 0, (size_t)N * sizeof(double));
+    for (int64_t k = 0; k < nnz; ++k) {
+        H[idx[k]] = W[idx[k]];
+        excl[idx[k]] = 1;
+    }
+    qo_grid(W, q, p, bits, excl, scale, zero);
+    for (int64_t k = 0; k < N; ++k)
+        Wh[k] = W[k] - H[k];
+
+    double lam = qo_power_lambda(S, p, power_iters);
+    double eta = 1.0 / (2.0 * lam);
+    if (eta_out)
+        *eta_out = eta;
+
+    for (int t = 0; t < iters; ++t) {
+        /* CD sweep with W replaced by W - H */
+#pragma omp parallel for schedule(dynamic)
+        for (int64_t i = 0; i < q; ++i) {
+            double *tgt = (double *)malloc((size_t)p * sizeof(double));
+            double *TS = (double *)malloc((size_t)p * sizeof(double));
+            double *WS = (double *)malloc((size_t)p * sizeof(double));
+            for (int64_t j = 0; j < p; ++j)
+                tgt[j] = W[i * p + j] - H[i * p + j];
+            qo_row_times_sigma(tgt, S, p, TS);
+            qo_row_times_sigma(Wh + i * p, S, p, WS);
+            qo_sweep_row(S, p, scale[i], zero[i], maxq, tgt, TS, Wh + i * p, WS,
+                         NULL, codes + i * p, NULL);
+            free(tgt); free(TS); free(WS);
+        }
+        qo_objective_rows(W, H, codes, scale, zero, q, p, S, rows);
+        double g = 0.0;
+        for (int64_t i = 0; i < q; ++i)
+            g += rows[i];
+        if (obj_cd)
+            obj_cd[t] = g;
+
+        /* gradient step and hard thresholding */
+#pragma omp parallel for schedule(dynamic)
+        for (int64_t i = 0; i < q; ++i) {
+            double *D = (double *)malloc((size_t)p * sizeof(double));
+            double *G = (double *)malloc((size_t)p * sizeof(double));
+            for (int64_t j = 0; j < p; ++j)
+                D[j] = H[i * p + j] + Wh[i * p + j] - W[i * p + j];
+            qo_row_times_sigma(D, S, p, G);          /* G/2 = (H + What - W) Sigma */
+            for (int64_t j = 0; j < p; ++j)
+                T[i * p + j] = H[i * p + j] - eta * 2.0 * G[j];
+            free(D); free(G);
+        }
+        nnz = qo_topk(T, N, s_budget, idx);
+        memset(H, 0, (size_t)N * sizeof(double));
+        for (int64_t k = 0; k < nnz; ++k)
+            H[idx[k]] = T[idx[k]];
+
+        qo_objective_rows(W, H, codes, scale, zero, q, p, S, rows);
+        g = 0.0;
+        for (int64_t i = 0; i < q; ++i)
+            g += rows[i];
+        if (obj)
+            obj[t] = g;
+    }
+    if (nnz_out)
+        *nnz_out = nnz;
+    free(idx); free(excl); free(Wh); free(T); free(rows);
+    return 0;
+}

@@ -1,0 +1,326 @@
+"""Pins of the fp64 oracle against what the paper and the mathematics fix.
+
+None of these compares the oracle with itself: each one checks it against a
+brute force, an exhaustive search, a closed form, an invariant, an algebraic
+identity between two independently written forms, or a textbook special case.
+"""
+import itertools
+
+import numpy as np
+import pytest
+
+import oracle
+from oracle import levels
+
+O = oracle.get()
+
+
+def _rand_layer(rng, q, p, n, heavy=(), heavy_mult=8.0, zero_rows=(), corr=False):
+    W = rng.normal(0.0, 0.02, size=(q, p))
+    X = rng.normal(0.0, 1.0, size=(p, n))
+    if corr:
+        U = rng.normal(size=(p, 2)) / np.sqrt(p)
+        V = rng.normal(size=(p, 2)) * 2.0
+        X = X + U @ (V.T @ X)
+    for r in heavy:
+        X[r] *= heavy_mult
+    for r in zero_rows:
+        X[r] = 0.0
+    # exact binary32 values, as the layers fed to the GPU path
+    return W.astype(np.float32).astype(np.float64), X.astype(np.float32).astype(np.float64)
+
+
+def _f_direct(W, What, X):
+    """||W X - What X||_F^2 of Eq. (layerwise-main), from X itself."""
+    R = (W - What) @ X
+    return float(np.sum(R * R))
+
+
+# --------------------------------------------------------------------------
+# grid and quantization operator (Sec. 2.1, Eq. eq:quant)
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("bits", [2, 3, 4, 8])
+def test_quantizer_returns_nearest_level(bits):
+    rng = np.random.default_rng(bits)
+    W = rng.normal(0, 0.05, size=(6, 300)).astype(np.float32).astype(np.float64)
+    W[1] = np.abs(W[1])          # all non-negative row
+    W[2] = -np.abs(W[2])         # all non-positive row
+    W[3] = 0.0                   # all-zero row -> range [-1, 1]
+    W[4, :3] = [4.0, -0.5, 0.25]  # one dominant entry
+    s, z = O.grid(W, bits)
+    maxq = 2 ** bits - 1
+    assert np.all(s > 0) and np.all(z == np.round(z)) and np.all((z >= 0) & (z <= maxq))
+    codes = O.rtn(W, s, z, bits)
+    lev = s.astype(np.float64)[:, None] * (np.arange(maxq + 1)[None, :] - z.astype(np.float64)[:, None])
+    dist = (W[:, :, None] - lev[:, None, :]) ** 2
+    chosen = np.take_along_axis(dist, codes[:, :, None].astype(np.int64), axis=2)[..., 0]
+    assert np.all(chosen <= dist.min(axis=2) * (1 + 1e-12) + 1e-300)
+
+
+@pytest.mark.parametrize("bits", [2, 3, 4])
+def test_grid_covers_row_range_and_zero(bits):
+    rng = np.random.default_rng(10 + bits)
+    W = rng.normal(0, 0.02, size=(20, 64)).astype(np.float32).astype(np.float64)
+    W[5] = np.abs(W[5])
+    W[6] = 0.0
+    s, z = O.grid(W, bits)
+    maxq = 2 ** bits - 1
+    lo = np.minimum(W.min(axis=1), 0.0)
+    hi = np.maximum(W.max(axis=1), 0.0)
+    lo[6], hi[6] = -1.0, 1.0
+    s64, z64 = s.astype(np.float64), z.astype(np.float64)
+    # 2^b distinct levels, zero is one of them exactly, the extremes are within half a step
+    assert np.all(s64 * (0 - z64) <= lo + 0.5 * s64 * (1 + 1e-6))
+    assert np.all(s64 * (maxq - z64) >= hi - 0.5 * s64 * (1 + 1e-6))
+    assert np.all(s64 * (z64 - z64) == 0.0)
+    assert np.allclose(s64 * maxq, hi - lo, rtol=1e-6)
+
+
+def test_grid_excluded_entries_leave_the_pool():
+    rng = np.random.default_rng(3)
+    W = rng.normal(0, 0.02, size=(4, 50))
+    W[0, 7] = 1.5
+    W[2, 3] = -2.0
+    excl = np.zeros(W.shape, np.uint8)
+    excl[0, 7] = excl[2, 3] = 1
+    s1, z1 = O.grid(W, 3, excl)
+    W2 = W.copy()
+    W2[0, 7] = W2[2, 3] = 0.0
+    s2, z2 = O.grid(W2, 3)
+    assert np.array_equal(s1, s2) and np.array_equal(z1, z2)
+
+
+# --------------------------------------------------------------------------
+# Lemma 1: every CD update is the exact 1-D minimiser over the grid
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("bits", [2, 3, 4])
+def test_every_update_is_bruteforce_argmin(bits):
+    rng = np.random.default_rng(100 + bits)
+    q, p, n, iters = 3, 7, 40, 3
+    W, X = _rand_layer(rng, q, p, n, heavy=(2,), zero_rows=(5,), corr=True)
+    S = O.sigma(X)
+    s, z = O.grid(W, bits)
+    r = O.alg1(W, S, s, z, bits, iters, record=True)
+    sc = r["sweep_codes"]
+    maxq = 2 ** bits - 1
+    cand = np.arange(maxq + 1)
+    for t in range(iters):
+        before = W.copy() if t == 0 else levels(sc[t - 1], s, z)
+        after = levels(sc[t], s, z)
+        for i in range(q):
+            for j in range(p):
+                state = np.concatenate([after[i, :j], before[i, j:]])
+                if j == 5:  # dead column: nearest level of W, fixed
+                    assert sc[t, i, j] == O.rtn(W[i:i + 1, j:j + 1], s[i:i + 1], z[i:i + 1], bits)[0, 0]
+                    continue
+                f = []
+                for c in cand:
+                    row = state.copy()
+                    row[j] = float(s[i]) * (c - float(z[i]))
+                    f.append(_f_direct(W[i:i + 1], row[None, :], X))
+                f = np.array(f)
+                assert f[sc[t, i, j]] <= f.min() + 1e-12 * max(1.0, abs(f.min())), (t, i, j)
+
+
+# --------------------------------------------------------------------------
+# exhaustive search on tiny layers: CD ends at a coordinate-wise minimum
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("p", [2, 3, 4])
+def test_exhaustive_tiny_layer_cw_minimum(p):
+    bits = 2
+    rng = np.random.default_rng(200 + p)
+    for trial in range(5):
+        W, X = _rand_layer(rng, 1, p, 12, corr=True)
+        S = O.sigma(X)
+        s, z = O.grid(W, bits)
+        r = O.alg1(W, S, s, z, bits, iters=40)
+        lev = lambda c: float(s[0]) * (np.asarray(c, np.float64) - float(z[0]))
+        allf = {c: _f_direct(W, lev(c)[None, :], X)
+                for c in itertools.product(range(4), repeat=p)}
+        fstar = min(allf.values())
+        c_cd = tuple(int(v) for v in r["codes"][0])
+        f_cd = allf[c_cd]
+        # the reported objective is f of the returned codes, and no code vector beats f*
+        assert np.isclose(r["obj"][-1], f_cd, rtol=1e-10, atol=1e-300)
+        assert f_cd >= fstar - 1e-15
+        # coordinate-wise minimum (Sec. 3.3, Definition): no single coordinate change improves f
+        for j in range(p):
+            for c in range(4):
+                alt = list(c_cd)
+                alt[j] = c
+                assert allf[tuple(alt)] >= f_cd - 1e-12 * max(1.0, f_cd)
+
+
+# --------------------------------------------------------------------------
+# monotone objective after the first (feasible) sweep (Sec. 3.1, Lemma 2)
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("seed,corr", [(0, False), (1, True), (2, True)])
+def test_objective_non_increasing(seed, corr):
+    rng = np.random.default_rng(300 + seed)
+    W, X = _rand_layer(rng, 16, 48, 200, heavy=(3, 11), heavy_mult=20.0, corr=corr)
+    S = O.sigma(X)
+    for bits in (3, 4):
+        s, z = O.grid(W, bits)
+        obj = O.alg1(W, S, s, z, bits, iters=8)["obj"]
+        assert np.all(np.diff(obj) <= 1e-12 * obj[:-1])
+
+
+# --------------------------------------------------------------------------
+# Algorithm 1 == Algorithm 3 (Sec. 3.2: an exact reassociation)
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("bits", [3, 4])
+def test_algorithm1_equals_algorithm3(bits):
+    rng = np.random.default_rng(400 + bits)
+    W, X = _rand_layer(rng, 24, 40, 160, heavy=(1,), heavy_mult=30.0, zero_rows=(7,), corr=True)
+    S = O.sigma(X)
+    s, z = O.grid(W, bits)
+    a1 = O.alg1(W, S, s, z, bits, iters=5)
+    a3 = O.alg3(W, S, s, z, bits, iters=5)
+    assert np.array_equal(a1["codes"], a3["codes"])
+    assert np.allclose(a1["obj_rows"], a3["obj_rows"], rtol=1e-10, atol=0)
+
+
+# --------------------------------------------------------------------------
+# textbook special case: orthogonal input channels -> round-to-nearest
+# --------------------------------------------------------------------------
+def test_diagonal_sigma_gives_round_to_nearest():
+    rng = np.random.default_rng(5)
+    q, p, n = 10, 32, 64
+    Qm, _ = np.linalg.qr(rng.normal(size=(n, p)))
+    X = (Qm.T * rng.uniform(0.5, 3.0, size=(p, 1)))        # rows orthogonal
+    W = rng.normal(0, 0.02, size=(q, p))
+    S = X @ X.T
+    S = np.diag(np.diag(S))                                  # exactly diagonal
+    for bits in (2, 4):
+        s, z = O.grid(W, bits)
+        r = O.alg1(W, S, s, z, bits, iters=3, record=True)
+        rtn = O.rtn(W, s, z, bits)
+        for t in range(3):
+            assert np.array_equal(r["sweep_codes"][t], rtn)
+
+
+# --------------------------------------------------------------------------
+# objective identity: tr(D Sigma D^T) == ||W X - What X||^2 (proof of Lemma 1)
+# --------------------------------------------------------------------------
+def test_objective_matches_direct_residual():
+    rng = np.random.default_rng(6)
+    W, X = _rand_layer(rng, 12, 30, 90, heavy=(4,), corr=True)
+    S = O.sigma(X)
+    s, z = O.grid(W, 3)
+    r = O.alg1(W, S, s, z, 3, iters=2)
+    What = levels(r["codes"], s, z)
+    direct = np.sum(((W - What) @ X) ** 2, axis=1)
+    assert np.allclose(r["obj_rows"][-1], direct, rtol=1e-10)
+
+
+# --------------------------------------------------------------------------
+# Sigma: symmetric PSD, diagonal = squared row norms, X (X^T v) association
+# --------------------------------------------------------------------------
+def test_sigma_properties():
+    rng = np.random.default_rng(7)
+    X = rng.normal(size=(37, 111))
+    X[3] *= 25.0
+    X[9] = 0.0
+    S = O.sigma(X)
+    assert np.array_equal(S, S.T)
+    assert np.allclose(np.diag(S), np.einsum("ij,ij->i", X, X), rtol=1e-13)
+    assert S[9, 9] == 0.0 and np.all(S[9] == 0.0)
+    ev = np.linalg.eigvalsh(S)
+    assert ev.min() >= -1e-10 * ev.max()
+    v = rng.normal(size=37)
+    assert np.allclose(S @ v, X @ (X.T @ v), rtol=1e-10)
+
+
+# --------------------------------------------------------------------------
+# invariances: scaling X, permuting / sub-setting rows (Sec. 3.2, rows independent)
+# --------------------------------------------------------------------------
+def test_invariances():
+    rng = np.random.default_rng(8)
+    W, X = _rand_layer(rng, 9, 20, 70, heavy=(2,), corr=True)
+    S = O.sigma(X)
+    s, z = O.grid(W, 3)
+    base = O.alg1(W, S, s, z, 3, iters=4)
+    S2 = O.sigma(2.0 * X)            # power-of-two scale: bit-identical trajectory
+    assert np.array_equal(O.alg1(W, S2, s, z, 3, iters=4)["codes"], base["codes"])
+    S3 = O.sigma(3.0 * X)
+    assert np.mean(O.alg1(W, S3, s, z, 3, iters=4)["codes"] == base["codes"]) > 0.99
+    perm = rng.permutation(9)
+    rp = O.alg1(W[perm], S, s[perm], z[perm], 3, iters=4)
+    assert np.array_equal(rp["codes"], base["codes"][perm])
+    assert np.allclose(rp["obj_rows"], base["obj_rows"][:, perm], rtol=1e-13)
+    sub = [1, 4, 7]
+    rs = O.alg1(W[sub], S, s[sub], z[sub], 3, iters=4)
+    assert np.array_equal(rs["codes"], base["codes"][sub])
+
+
+def test_warm_start_from_fixed_point_is_stationary():
+    """Sec. 3.1: CD can refine any feasible What; a converged state stays put."""
+    rng = np.random.default_rng(9)
+    W, X = _rand_layer(rng, 6, 16, 60, corr=True)
+    S = O.sigma(X)
+    s, z = O.grid(W, 3)
+    conv = O.alg1(W, S, s, z, 3, iters=60)["codes"]
+    again = O.alg1(W, S, s, z, 3, iters=2, init_codes=conv)
+    assert np.array_equal(again["codes"], conv)
+
+
+# --------------------------------------------------------------------------
+# outlier-aware pieces (Sec. 4.3): lambda_max, P_s, Lemma 3, s = 0 reduction
+# --------------------------------------------------------------------------
+def test_power_lambda_matches_eigvalsh():
+    rng = np.random.default_rng(11)
+    A = rng.normal(size=(40, 80))
+    A[0] *= 6.0
+    S = A @ A.T
+    lam = O.power_lambda(S, 800)
+    ev = np.linalg.eigvalsh(S)
+    assert abs(lam - ev[-1]) <= 1e-10 * ev[-1]
+    for it in (0, 1, 3):                 # a Rayleigh quotient never exceeds lambda_max
+        assert O.power_lambda(S, it) <= ev[-1] * (1 + 1e-12)
+
+
+def test_topk_matches_full_sort_with_ties():
+    rng = np.random.default_rng(12)
+    T = rng.integers(-5, 6, size=(7, 31)).astype(np.float64) * 0.25   # many ties and zeros
+    for s in (0, 1, 5, 40, 150, 217, 400):
+        got = O.topk(T, s)
+        flat = T.ravel()
+        nz = np.nonzero(flat)[0]
+        order = nz[np.lexsort((nz, -np.abs(flat[nz])))]
+        want = np.sort(order[:s])
+        assert np.array_equal(got, want), s
+
+
+def test_outlier_iht_descent_and_budget():
+    rng = np.random.default_rng(13)
+    q, p, n, s_budget = 12, 24, 80, 20
+    W, X = _rand_layer(rng, q, p, n, heavy=(5,), heavy_mult=10.0, corr=True)
+    W[rng.integers(0, q, 8), rng.integers(0, p, 8)] += rng.normal(0, 0.3, 8)
+    S = O.sigma(X)
+    r = O.outlier(W, S, 3, 8, s_budget, 600)
+    assert r["nnz"] <= s_budget and np.count_nonzero(r["H"]) <= s_budget
+    # Lemma 3: each IHT step does not increase g; CD halves do not either once feasible
+    assert np.all(r["obj"] <= r["obj_cd"] * (1 + 1e-10))
+    assert np.all(r["obj_cd"][1:] <= r["obj"][:-1] * (1 + 1e-10))
+    # the grid ignores the s largest |W| (Sec. 4.3)
+    excl = np.zeros(q * p, np.uint8)
+    excl[O.topk(W, s_budget)] = 1
+    s_, z_ = O.grid(W, 3, excl.reshape(q, p))
+    assert np.array_equal(s_, r["scale"]) and np.array_equal(z_, r["zero"])
+    # eta = 1 / (2 lambda_max)
+    assert np.isclose(r["eta"], 1.0 / (2.0 * np.linalg.eigvalsh(S)[-1]), rtol=1e-8)
+    # reported g equals ||W X - (What + H) X||^2 from X
+    What = levels(r["codes"], r["scale"], r["zero"])
+    assert np.isclose(r["obj"][-1], _f_direct(W, What + r["H"], X), rtol=1e-10)
+
+
+def test_outlier_with_zero_budget_reduces_to_algorithm1():
+    rng = np.random.default_rng(14)
+    W, X = _rand_layer(rng, 8, 20, 50, corr=True)
+    S = O.sigma(X)
+    r = O.outlier(W, S, 3, 4, 0, 50)
+    s, z = O.grid(W, 3)
+    a1 = O.alg1(W, S, s, z, 3, iters=4)
+    assert np.array_equal(r["codes"], a1["codes"])
+    assert np.allclose(r["obj"], a1["obj"], rtol=1e-12) and np.allclose(r["obj_cd"], a1["obj"], rtol=1e-12)
+    assert not np.any(r["H"])
