@@ -1,0 +1,350 @@
+"""Benchmark: QuantEase layer quantization on GB300 (one JSON line on stdout).
+
+Workload (default): the LLaMA-7B-shaped attention projection, q = p = 4096,
+n = 262144 calibration tokens (128 x 2048), bf16 W and X (synthetic, seeded).
+One step = build Sigma = X X^T, then quantize the layer at 3 and at 4 bits with
+20 CD sweeps each: the whole hot path, inputs resident in HBM.
+
+metric / unit: CD column-updates per second (q p^2 per sweep, summed over both
+bit-widths) over the whole step including the Sigma build; the JSON line also
+carries the layer quantize time, Sigma TFLOP/s and the CD-phase rate.
+
+--impl reference times the fp64 CPU oracle (the reference arm) on a bounded
+sample of the same workload (rows are independent given Sigma).
+
+Multi-GPU (torchrun): every rank quantizes its own layer (weak scaling, no
+collective on the data path); timing is the max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = ("layer quantize time; CD column-updates/s (q·p²/s) and Σ TFLOP/s vs roofline")
+UNIT = "q·p² column-updates/s"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=3)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="qe", choices=["qe", "reference"])
+    ap.add_argument("--config", default="llama7b_proj_4096x4096")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--cpu-rows", type=int, default=96, help="oracle rows in the CPU sample")
+    return ap.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as fh:
+            m = json.load(fh)
+        return dict(hbm=float(m["hbm_gbs"]), bf16=float(m["bf16_tflops"]),
+                    bf16_sustained=float(m["bf16_tflops_sustained"]), source="measured")
+    except (OSError, KeyError, ValueError):
+        return dict(hbm=6800.0, bf16=1900.0, bf16_sustained=1700.0, source="fallback")
+
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled every 200 ms during the timed region."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        if self.thread:
+            self.thread.join(timeout=2)
+        sm, smax, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [x.strip() for x in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax = float(parts[2])
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[5:9]):
+                if v.lower() in ("active", "1", "yes"):
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": smax, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def cpu_oracle_sample(W64, S64, bits, rows, sweeps):
+    """Time Algorithm 1 of the fp64 oracle on a row sample; returns (units/s, seconds, threads)."""
+    import numpy as np
+    import oracle
+    O = oracle.get()
+    s, z = O.grid(W64[:rows], bits)
+    t0 = time.perf_counter()
+    O.alg1(np.ascontiguousarray(W64[:rows]), S64, s, z, bits, sweeps)
+    dt = time.perf_counter() - t0
+    p = W64.shape[1]
+    threads = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    return rows * p * p * sweeps / dt, dt, threads
+
+
+def run_reference(args):
+    """The reference arm: the fp64 CPU oracle, on a bounded sample per step."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    import numpy as np
+    import torch
+    from paper_2309_01885_gb300 import inputs
+    cfg = inputs.CONFIGS[args.config]
+    W = cfg.weights("cpu").double().numpy()
+    # Sigma from a 4096-token slice: the oracle's CD rate depends on p, not on Sigma's values
+    n_ref = 4096
+    X = inputs.calib_inputs(cfg.p, n_ref, dtype=cfg.x_dtype, seed=cfg.seed, device="cpu",
+                            heavy_frac=cfg.heavy_frac, heavy_mult=cfg.heavy_mult).double().numpy()
+    import oracle
+    O = oracle.get()
+    S = O.sigma(X)
+    rows = max(1, min(cfg.q, args.cpu_rows))
+    times, units = [], 0
+    for step in range(args.warmup + args.steps):
+        t0 = time.perf_counter()
+        for b in cfg.bits:
+            cpu_oracle_sample(W, S, b, rows, 1)
+        dt = time.perf_counter() - t0
+        if step >= args.warmup:
+            times.append(dt)
+    units = rows * cfg.p * cfg.p * len(cfg.bits)
+    ms = 1e3 * sum(times) / len(times)
+    value = units / (ms / 1e3)
+    threads = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    sample = (f"Algorithm 1 (fp64 oracle) on {rows} of {cfg.q} rows, 1 sweep per bit-width "
+              f"{list(cfg.bits)}, p={cfg.p}, Sigma from {n_ref} tokens; rows are independent given Sigma")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": cfg.name, "q": cfg.q, "p": cfg.p, "n": cfg.n, "bits": list(cfg.bits),
+                       "sweeps": cfg.iters},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        return run_reference(args)
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+    from paper_2309_01885_gb300 import inputs, qe
+    from paper_2309_01885_gb300.build import build_lib
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    if rank == 0:
+        build_lib()
+    if world > 1:
+        dist.barrier()
+    qe.load()
+
+    cfg = inputs.CONFIGS[args.config]
+    q, p, n = cfg.q, cfg.p, cfg.n
+    seed = cfg.seed + rank                        # each rank owns a different layer
+    W = inputs.layer_weights(q, p, dtype=cfg.w_dtype, seed=seed, device="cuda")
+    X = inputs.calib_inputs(p, n, dtype=cfg.x_dtype, seed=seed, device="cuda",
+                            heavy_frac=cfg.heavy_frac, heavy_mult=cfg.heavy_mult)
+    Sigma = torch.empty(p, p, dtype=torch.float32, device="cuda")
+    ws = torch.empty(qe.qe_workspace_size(q, p), dtype=torch.uint8, device="cuda")
+    stream = torch.cuda.current_stream()
+    nb = len(cfg.bits)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(nb + 2)]
+          for _ in range(args.steps)]
+
+    def step(events=None):
+        if events:
+            events[0].record(stream)
+        qe.qe_build_sigma(X, Sigma=Sigma)
+        if events:
+            events[1].record(stream)
+        outs = []
+        for k, b in enumerate(cfg.bits):
+            outs.append(qe.qe_quantize_layer(W, Sigma, b, cfg.iters, workspace=ws))
+            if events:
+                events[2 + k].record(stream)
+        return outs
+
+    for _ in range(args.warmup):
+        step()
+    st = qe.qe_sync_status()
+    if st != qe.QE_OK:
+        raise RuntimeError(f"device status {qe.qe_status_string(st)}")
+
+    clocks = ClockSampler(local)
+    clocks.start()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    outs = None
+    for k in range(args.steps):
+        outs = step(ev[k])
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clk = clocks.stop()
+    total_ms = t_start.elapsed_time(t_end)
+    sigma_ms = [e[0].elapsed_time(e[1]) for e in ev]
+    cd_ms = [[e[1 + k].elapsed_time(e[2 + k]) for e in ev] for k in range(nb)]
+    ms = total_ms / args.steps
+    if world > 1:
+        t = torch.tensor([ms], dtype=torch.float64, device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+
+    units_per_step = q * p * p * cfg.iters * nb           # column updates per rank per step
+    value = units_per_step * world / (ms / 1e3)
+    sig_flops = p * (p + 1) * n                            # symmetric half of X X^T
+    sigma_avg = statistics.mean(sigma_ms)
+    cd_avg = [statistics.mean(x) for x in cd_ms]
+    pk = peaks()
+
+    result = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+              "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+              "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+              "config": {"workload": cfg.name, "q": q, "p": p, "n": n, "bits": list(cfg.bits),
+                         "sweeps": cfg.iters, "parallelism": f"layer-replicas x{world}",
+                         "l2": "inputs larger than L2 (X is %.2f GiB)" % (p * n * 2 / 2**30)},
+              "layer_quantize_ms": ms,
+              "sigma_ms": sigma_avg,
+              "sigma_tflops": sig_flops / (sigma_avg / 1e3) / 1e12,
+              "sigma_dense_equiv_tflops": 2 * p * p * n / (sigma_avg / 1e3) / 1e12,
+              "cd_ms": {str(b): v for b, v in zip(cfg.bits, cd_avg)},
+              "cd_updates_per_s": q * p * p * cfg.iters * nb / (sum(cd_avg) / 1e3),
+              "roofline": {"bound": "tensor", "kernel": "k_tc_gemm<256> (Sigma = X X^T)",
+                           "achieved": sig_flops / (sigma_avg / 1e3) / 1e12,
+                           "peak": pk["bf16_sustained"], "unit": "TFLOP/s",
+                           "frac": sig_flops / (sigma_avg / 1e3) / 1e12 / pk["bf16_sustained"],
+                           "traffic": None,
+                           "peak_source": f"{pk['source']} bf16 dense sustained"},
+              "clocks": clk}
+
+    # launches of our kernels per step (schedule of qe_api.cu)
+    nblk = (p + 63) // 64
+    w_planes = 0 if cfg.w_dtype == torch.bfloat16 else 1
+    per_layer = 6 + w_planes + cfg.iters * (nblk + (nblk - 1) + 1 + 2)
+    result["gpu_launches"] = args.steps * (1 + nb * per_layer)
+
+    # end to end through the C ABI with host buffers
+    if not args.no_e2e:
+        Xh = X.cpu().pin_memory()
+        Wh = W.cpu().pin_memory()
+        Xd = torch.empty_like(X)
+        Wd = torch.empty_like(W)
+        host_out = [dict(codes=torch.empty(q, p, dtype=torch.uint8).pin_memory(),
+                         scales=torch.empty(q).pin_memory(), zeros=torch.empty(q).pin_memory(),
+                         obj=torch.empty(cfg.iters, dtype=torch.float64).pin_memory())
+                    for _ in cfg.bits]
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        e0.record(stream)
+        for _ in range(args.steps):
+            Xd.copy_(Xh, non_blocking=True)
+            Wd.copy_(Wh, non_blocking=True)
+            qe.qe_build_sigma(Xd, Sigma=Sigma)
+            for k, b in enumerate(cfg.bits):
+                o = qe.qe_quantize_layer(Wd, Sigma, b, cfg.iters, workspace=ws)
+                for key in ("codes", "scales", "zeros", "obj"):
+                    host_out[k][key].copy_(o[key], non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        e2e_ms = e0.elapsed_time(e1) / args.steps
+        if world > 1:
+            t = torch.tensor([e2e_ms], dtype=torch.float64, device="cuda")
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e2e_ms = float(t.item())
+        h2d = X.numel() * X.element_size() + W.numel() * W.element_size()
+        d2h = nb * (q * p + 4 * q + 4 * q + 8 * cfg.iters)
+        result["e2e"] = {"value": units_per_step * world / (e2e_ms / 1e3), "unit": UNIT,
+                         "ms_per_step": e2e_ms, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+
+    st = qe.qe_sync_status()
+    if st != qe.QE_OK:
+        raise RuntimeError(f"device status {qe.qe_status_string(st)}")
+
+    # CPU baseline: the fp64 oracle on a row sample of the same layer (rank 0, N = 1 only)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        W64 = W.double().cpu().numpy()
+        S64 = Sigma.double().cpu().numpy()
+        rows = max(1, min(q, args.cpu_rows))
+        rate, dt, threads = cpu_oracle_sample(W64, S64, cfg.bits[0], rows, 1)
+        result["cpu_baseline"] = {
+            "value": rate, "unit": "q·p² column-updates/s (CD only)", "cores": threads,
+            "kind": "oracle",
+            "sample": (f"Algorithm 1 (fp64 oracle) on {rows} of {q} rows x 1 sweep, {cfg.bits[0]}-bit, "
+                       f"given this layer's Sigma; {dt:.1f} s")}
+        result["obj_last"] = {str(b): float(o["obj"][-1].item()) for b, o in zip(cfg.bits, outs)}
+
+    if rank == 0:
+        print(json.dumps(result), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,159 @@
+/*
+ * qe.h -- C ABI of libqe.so: QuantEase layer-wise quantization on one GB300
+ * (Behdin et al., "QuantEase: Optimization-based Quantization for Language
+ * Models", arXiv 2309.01885).
+ *
+ * Problem (Sec. 2.1, Eq. layerwise-main): for a linear layer with weights
+ * W (q x p: q output channels, p input features) and calibration inputs
+ * X (p x n), find What on a per-row uniform b-bit grid Q_i minimising
+ *     f(What) = || W X - What X ||_F^2 = tr((W - What) Sigma (W - What)^T),
+ * Sigma = X X^T.  The solver is cyclic coordinate descent with the closed-form
+ * quantized update of Lemma 1, organised as the accelerated Algorithm 3.
+ *
+ * Conventions for every entry point:
+ *  - All array arguments are DEVICE pointers owned by the caller, unless a
+ *    parameter says otherwise.  The library never frees caller memory.
+ *  - Matrices are row-major with an explicit leading dimension (elements).
+ *  - Calls are stream-ordered and asynchronous on `stream` (a cudaStream_t;
+ *    NULL = legacy default stream).  Argument errors are returned
+ *    synchronously before anything is enqueued.  Errors found on the device
+ *    (non-finite input, a device-side wait that gave up) are latched in a
+ *    per-device error word and reported by qe_sync_status().
+ *  - Scratch memory: taken from opts->workspace when given (at least
+ *    qe_workspace_size() bytes, 256-byte aligned), otherwise allocated with
+ *    cudaMallocAsync / cudaFreeAsync on `stream` inside the call.
+ *  - Thread safety: distinct streams may be used from distinct host threads.
+ */
+#ifndef QE_H
+#define QE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same object as cudaStream_t; declared here so the header needs no CUDA headers. */
+typedef struct CUstream_st *qe_stream_t;
+
+typedef enum {
+    QE_OK = 0,
+    QE_ERR_INVALID_ARG = 1,   /* bad size, pointer, alignment or option */
+    QE_ERR_CUDA = 2,          /* a CUDA runtime/driver call failed */
+    QE_ERR_OOM = 3,           /* workspace allocation failed or too small */
+    QE_ERR_NUMERIC = 4,       /* non-finite value in W or Sigma (device-detected) */
+    QE_ERR_TIMEOUT = 5,       /* a bounded device-side wait gave up (device-detected) */
+    QE_ERR_UNSUPPORTED = 6    /* option or layout not implemented */
+} qe_status;
+
+typedef enum { QE_F32 = 0, QE_BF16 = 1 } qe_dtype;
+
+typedef enum {
+    QE_FEATURE_MAJOR = 0,     /* X is p x n row-major: the paper's X (Sec. 2.1) */
+    QE_TOKEN_MAJOR = 1        /* X is n x p row-major: activations as a model emits them */
+} qe_xlayout;
+
+typedef struct {
+    /* Column block width B of the blocked CD sweep: 0 = default (64); 32 or 64. */
+    int block_width;
+    /* Relax heuristic of Sec. 3.2 (skip quantization every R-th sweep): must be 0. */
+    int relax_period;
+    /* Structured (column) outliers of Sec. 4.3: must be 0. */
+    int structured_outliers;
+    /* Outlier variant: power-method iterations for lambda_max(Sigma), 0 = default 64. */
+    int power_iters;
+    /* Optional warm start (Sec. 3.1, "initialized with ... any other algorithm"):
+     * q x p codes (leading dimension p) on the grid this call computes.  NULL = start at W. */
+    const uint8_t *init_codes;
+    /* Optional output: iters x q x p codes after every sweep (for parity checks). */
+    uint8_t *sweep_codes;
+    /* Optional output: one double, ||W X||_F^2, the denominator of the relative
+     * calibration error of Sec. 3.4 (target W - H for the outlier variant). */
+    double *wx_norm2;
+    /* Optional caller workspace (device, 256-byte aligned) and its size. */
+    void *workspace;
+    size_t workspace_bytes;
+} qe_opts;
+
+/*
+ * Sigma = X X^T (Lemma 1; the memory-footprint paragraph of Sec. 3.2 keeps it
+ * resident), fp32 output, p x p row-major, leading dimension p.
+ *   X          device, bf16 or fp32; layout QE_FEATURE_MAJOR (p x n, leading
+ *              dimension ldx >= n) or QE_TOKEN_MAJOR (n x p, ldx >= p).
+ *   accumulate 0: Sigma = X X^T;  1: Sigma += X X^T (stream n in chunks).
+ * The result is exactly symmetric.  bf16 X runs on tcgen05 tensor cores with
+ * fp32 accumulation; fp32 X on fp32 FMA.  Errors: QE_ERR_INVALID_ARG for
+ * p < 1, n < 0, a short leading dimension or NULL pointers.
+ */
+qe_status qe_build_sigma(const void *X, qe_dtype x_dtype, qe_xlayout layout,
+                         int64_t p, int64_t n, int64_t ldx, float *Sigma,
+                         int accumulate, qe_stream_t stream);
+
+/*
+ * QuantEase for one layer (Algorithm 3, Sec. 3.2, blocked by columns).
+ *   W        device q x p, bf16 or fp32, leading dimension ldw >= p.
+ *   Sigma    device p x p fp32, symmetric PSD (e.g. from qe_build_sigma).
+ *            Columns with Sigma_jj <= 0 (X_j = 0, footnote of Lemma 1) drop
+ *            out of the objective and get the nearest level of W_ij.
+ *   bits     b in [2, 8]: 2^b levels per row.
+ *   iters    K >= 1 cyclic sweeps over j = 1..p (Sec. 3.1).
+ *   codes    out, device q x p uint8 (leading dimension p): What_ij = s_i (c_ij - z_i).
+ *   scales   out, device q floats s_i;  zeros: out, device q floats z_i
+ *            (integer-valued).  Grid: asymmetric per-row min/max with 0 in
+ *            range, s = (max - min)/(2^b - 1), z = round(-min/s), evaluated
+ *            in binary32 (Sec. 2.1, "uniformly spaced, following GPTQ").
+ *   obj      out, device iters doubles: f after each sweep.
+ *   opts     may be NULL (all defaults).
+ * Each coordinate takes the nearest level of the closed-form minimiser
+ * (Lemma 1); ties in rounding go to the even integer of beta/s + z.
+ */
+qe_status qe_quantize_layer(const void *W, qe_dtype w_dtype, int64_t q, int64_t p,
+                            int64_t ldw, const float *Sigma, int bits, int iters,
+                            const qe_opts *opts, uint8_t *codes, float *scales,
+                            float *zeros, double *obj, qe_stream_t stream);
+
+/*
+ * Outlier-aware QuantEase (Sec. 4, Eq. main-outlier, Algorithm 4): What on
+ * the grid plus a sparse full-precision H with ||H||_0 <= s_budget.
+ *   H = P_s(W) initially; the grid is computed from W without those entries
+ *   (Sec. 4.3); every iteration runs one CD sweep with target W - H, then one
+ *   IHT step H <- P_s(H - eta grad_H g), eta = 1/(2 lambda_max(Sigma)) with
+ *   lambda_max from opts->power_iters power-method steps (Sec. 4.3).
+ *   P_s keeps the s_budget largest |entries|; ties go to the smaller
+ *   row-major index i*p + j; exact zeros are never kept.
+ *   H_val, H_idx  out, device s_budget floats / int64: the kept values and
+ *                 their linear indices i*p + j in ascending order.
+ *   H_nnz         out, device int64: number of kept entries (<= s_budget).
+ *   obj           out, device iters doubles: g after the IHT step of each iteration.
+ *   obj_cd        out (may be NULL), device iters doubles: g after the CD sweep.
+ * Other arguments as qe_quantize_layer.
+ */
+qe_status qe_quantize_layer_outlier(const void *W, qe_dtype w_dtype, int64_t q,
+                                    int64_t p, int64_t ldw, const float *Sigma,
+                                    int bits, int iters, int64_t s_budget,
+                                    const qe_opts *opts, uint8_t *codes,
+                                    float *scales, float *zeros, float *H_val,
+                                    int64_t *H_idx, int64_t *H_nnz, double *obj,
+                                    double *obj_cd, qe_stream_t stream);
+
+/* Bytes of scratch qe_quantize_layer (outlier = 0) or qe_quantize_layer_outlier
+ * (outlier = 1) needs for this shape and options; written to *bytes. */
+qe_status qe_workspace_size(int64_t q, int64_t p, int outlier, const qe_opts *opts,
+                            size_t *bytes);
+
+/* Waits for `stream`, then returns and clears the error latched on the current
+ * device (QE_ERR_NUMERIC / QE_ERR_TIMEOUT), or QE_ERR_CUDA if the stream failed. */
+qe_status qe_sync_status(qe_stream_t stream);
+
+/* Static description of a status code. */
+const char *qe_status_string(qe_status status);
+
+/* ABI version: major * 10000 + minor * 100 + patch. */
+int qe_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* QE_H */

@@ -1,0 +1,576 @@
+// C ABI of libqe (include/qe.h): argument checks, workspace layout and the
+// stream-ordered schedule of the QuantEase kernels.
+//
+// qe_quantize_layer, per layer (Algorithm 3 of Sec. 3.2, blocked by columns):
+//   grid(W) -> s, z;  Sigma -> d, Sigma_bar^T planes;  P = W (I + Sigma_bar);
+//   R = W (the first sweep starts at What = W, Sec. 3.1);
+//   per sweep:  per column block [b0, b0+B):
+//                   partial = Delta'[:, 0:b0] Sigma_bar[0:b0, block]   (tcgen05, split-K)
+//                   sequential in-block updates -> codes, C - z, Delta'
+//               R = P - s (C - z) Sigma_bar                           (tcgen05)
+//               f = sum D_ij d_j (R_ij - What_ij)                     (reduction)
+// qe_quantize_layer_outlier adds, per iteration (Algorithm 4 of Sec. 4.3):
+//   T = H + 2 eta d_j (R - What);  H = P_s(T);  P = P_W - H (I + Sigma_bar);
+//   R += P_new - P_old.
+#include <stdio.h>
+#include <string.h>
+
+#include "../../include/qe.h"
+#include "qe_common.cuh"
+#include "qe_internal.h"
+#include "qe_kernels.h"
+#include "qe_outlier.h"
+
+namespace qe {
+
+__device__ unsigned g_err_word;
+
+static unsigned *error_word() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+    static unsigned *cache[64] = {};
+    if (!cache[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_err_word) == cudaSuccess) cache[dev] = static_cast<unsigned *>(p);
+    }
+    return cache[dev];
+}
+
+static int sm_count() {
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 148;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+        return 148;
+    return n;
+}
+
+constexpr int kDefaultBlock = 64;
+constexpr int kDefaultPowerIters = 64;
+
+// ---- workspace layout -----------------------------------------------------------
+struct Plan {
+    int64_t q = 0, p = 0, ld = 0;
+    int B = kDefaultBlock, smax = 1;
+    size_t snt = 0, d = 0, dinv = 0, P = 0, R = 0, wpl = 0, qf = 0, dp = 0, part = 0, objp = 0;
+    size_t PW = 0, H = 0, T = 0, st = 0, cg = 0, ce = 0, sb = 0, eb = 0, y0 = 0, y1 = 0, lam = 0,
+           eta = 0, rowptr = 0;
+    size_t total = 0;
+};
+
+static size_t take(size_t &cur, size_t bytes) {
+    const size_t o = cur;
+    cur += static_cast<size_t>(round_up(static_cast<int64_t>(bytes > 0 ? bytes : 1), 256));
+    return o;
+}
+
+static Plan make_plan(int64_t q, int64_t p, int B, bool outlier, int wpl_planes, int nsm) {
+    Plan pl;
+    pl.q = q;
+    pl.p = p;
+    pl.ld = round_up(p, 64);
+    pl.B = B;
+    const int64_t mtiles = ceil_div(q, 128);
+    int64_t smax = nsm / mtiles;
+    if (smax < 1) smax = 1;
+    if (smax > 16) smax = 16;
+    pl.smax = static_cast<int>(smax);
+    const size_t qld = static_cast<size_t>(q) * pl.ld;
+    size_t cur = 0;
+    pl.snt = take(cur, static_cast<size_t>(2 * p) * pl.ld * 2);
+    pl.d = take(cur, p * 4);
+    pl.dinv = take(cur, p * 4);
+    pl.P = take(cur, qld * 4);
+    pl.R = take(cur, qld * 4);
+    pl.wpl = take(cur, wpl_planes > 0 ? qld * 2 * wpl_planes : 0);
+    pl.qf = take(cur, qld * 2);
+    pl.dp = take(cur, qld * 2 * 2);
+    pl.part = take(cur, static_cast<size_t>(pl.smax) * q * B * 4);
+    pl.objp = take(cur, static_cast<size_t>(objective_blocks(q)) * 8);
+    if (outlier) {
+        const int64_t N = q * p;
+        const int64_t nch = topk_chunks(N);
+        pl.PW = take(cur, qld * 4);
+        pl.H = take(cur, qld * 4);
+        pl.T = take(cur, static_cast<size_t>(N) * 4);
+        pl.st = take(cur, sizeof(TopkState));
+        pl.cg = take(cur, nch * 4);
+        pl.ce = take(cur, nch * 4);
+        pl.sb = take(cur, nch * 4);
+        pl.eb = take(cur, nch * 4);
+        pl.y0 = take(cur, p * 4);
+        pl.y1 = take(cur, p * 4);
+        pl.lam = take(cur, 8);
+        pl.eta = take(cur, 8);
+        pl.rowptr = take(cur, (q + 1) * 8);
+    }
+    pl.total = cur;
+    return pl;
+}
+
+// ---- per-call context ----------------------------------------------------------------
+struct Ctx {
+    cudaStream_t s = nullptr;
+    unsigned *err = nullptr;
+    int nsm = 148;
+    Plan pl;
+    uint8_t *ws = nullptr;
+    bool own = false;
+    __nv_bfloat16 *snt = nullptr, *wpl = nullptr, *qf = nullptr, *dp = nullptr;
+    float *d = nullptr, *dinv = nullptr, *P = nullptr, *R = nullptr, *part = nullptr;
+    double *objp = nullptr;
+    float *PW = nullptr, *H = nullptr, *T = nullptr, *y0 = nullptr, *y1 = nullptr;
+    TopkState *st = nullptr;
+    unsigned *cg = nullptr, *ce = nullptr, *sb = nullptr, *eb = nullptr;
+    double *lam = nullptr, *eta = nullptr;
+    int64_t *rowptr = nullptr;
+    CUtensorMap tm_snt256, tm_snt64, tm_qf, tm_dp, tm_wa;
+    int wa_planes = 1;
+
+    ~Ctx() {
+        if (own && ws) cudaFreeAsync(ws, s);
+    }
+};
+
+template <typename T>
+static T *at(uint8_t *ws, size_t off) {
+    return reinterpret_cast<T *>(ws + off);
+}
+
+static qe_status setup_ctx(Ctx &c, const Plan &pl, const qe_opts *o, cudaStream_t s) {
+    c.s = s;
+    c.pl = pl;
+    c.err = error_word();
+    if (!c.err) return QE_ERR_CUDA;
+    if (o && o->workspace) {
+        if (o->workspace_bytes < pl.total || (reinterpret_cast<uintptr_t>(o->workspace) & 255u))
+            return QE_ERR_OOM;
+        c.ws = static_cast<uint8_t *>(o->workspace);
+    } else {
+        void *p = nullptr;
+        if (cudaMallocAsync(&p, pl.total, s) != cudaSuccess) {
+            cudaGetLastError();
+            return QE_ERR_OOM;
+        }
+        c.ws = static_cast<uint8_t *>(p);
+        c.own = true;
+    }
+    uint8_t *w = c.ws;
+    c.snt = at<__nv_bfloat16>(w, pl.snt);
+    c.d = at<float>(w, pl.d);
+    c.dinv = at<float>(w, pl.dinv);
+    c.P = at<float>(w, pl.P);
+    c.R = at<float>(w, pl.R);
+    c.wpl = at<__nv_bfloat16>(w, pl.wpl);
+    c.qf = at<__nv_bfloat16>(w, pl.qf);
+    c.dp = at<__nv_bfloat16>(w, pl.dp);
+    c.part = at<float>(w, pl.part);
+    c.objp = at<double>(w, pl.objp);
+    if (pl.PW) {
+        c.PW = at<float>(w, pl.PW);
+        c.H = at<float>(w, pl.H);
+        c.T = at<float>(w, pl.T);
+        c.st = at<TopkState>(w, pl.st);
+        c.cg = at<unsigned>(w, pl.cg);
+        c.ce = at<unsigned>(w, pl.ce);
+        c.sb = at<unsigned>(w, pl.sb);
+        c.eb = at<unsigned>(w, pl.eb);
+        c.y0 = at<float>(w, pl.y0);
+        c.y1 = at<float>(w, pl.y1);
+        c.lam = at<double>(w, pl.lam);
+        c.eta = at<double>(w, pl.eta);
+        c.rowptr = at<int64_t>(w, pl.rowptr);
+    }
+    const uint64_t q = pl.q, p = pl.p, ld = pl.ld;
+    if (!make_tmap_bf16(&c.tm_snt256, c.snt, 2 * p, p, ld, 256) ||
+        !make_tmap_bf16(&c.tm_snt64, c.snt, 2 * p, p, ld, 64) ||
+        !make_tmap_bf16(&c.tm_qf, c.qf, q, p, ld, 128) ||
+        !make_tmap_bf16(&c.tm_dp, c.dp, 2 * q, p, ld, 128))
+        return QE_ERR_CUDA;
+    return QE_OK;
+}
+
+#define QE_CK(x)                                     \
+    do {                                             \
+        if ((x) != cudaSuccess) {                    \
+            cudaGetLastError();                      \
+            return QE_ERR_CUDA;                      \
+        }                                            \
+    } while (0)
+
+static GemmArgs gemm_args(const Ctx &c, int M, int N, int kb_count, int mode) {
+    GemmArgs g;
+    memset(&g, 0, sizeof(g));
+    g.M = M;
+    g.N = N;
+    g.kb_begin = 0;
+    g.kb_count = kb_count;
+    g.mode = mode;
+    g.err = c.err;
+    return g;
+}
+
+static void set_prods(GemmArgs &g, int a_planes) {
+    // hi.hi, hi.lo and (two A planes) lo.hi; the lo.lo product is below fp32 rounding.
+    g.prod_a[0] = 0; g.prod_b[0] = 0;
+    g.prod_a[1] = 0; g.prod_b[1] = 1;
+    g.prod_a[2] = 1; g.prod_b[2] = 0;
+    g.n_prod = (a_planes == 2) ? 3 : 2;
+}
+
+// Sigma -> d, Sigma_bar^T planes; W operand planes; P = W (I + Sigma_bar) into `Pout`.
+static qe_status prepare(Ctx &c, const void *W, int wbf16, int64_t ldw, const float *Sigma, float *Pout) {
+    const int64_t q = c.pl.q, p = c.pl.p, ld = c.pl.ld;
+    QE_CK(launch_sigma_norm(Sigma, p, p, c.d, c.snt, ld, c.err, c.s));
+    QE_CK(launch_dinv(c.d, p, c.dinv, c.s));
+    const bool direct = wbf16 && ((reinterpret_cast<uintptr_t>(W) & 15u) == 0) && (ldw % 8 == 0);
+    if (direct) {
+        if (!make_tmap_bf16(&c.tm_wa, W, q, p, ldw, 128)) return QE_ERR_CUDA;
+        c.wa_planes = 1;
+    } else {
+        c.wa_planes = wbf16 ? 1 : 2;
+        QE_CK(launch_make_planes(W, wbf16, ldw, q, p, c.wa_planes == 2, c.wpl, ld, c.s));
+        if (!make_tmap_bf16(&c.tm_wa, c.wpl, c.wa_planes * q, p, ld, 128)) return QE_ERR_CUDA;
+    }
+    GemmArgs g = gemm_args(c, static_cast<int>(q), static_cast<int>(p), static_cast<int>(ceil_div(p, 64)),
+                           EPI_PINIT);
+    set_prods(g, c.wa_planes);
+    g.a_plane_rows = static_cast<int>(q);
+    g.b_plane_rows = static_cast<int>(p);
+    g.out = Pout;
+    g.ldo = ld;
+    g.W = W;
+    g.w_is_bf16 = wbf16;
+    g.ldw = ldw;
+    QE_CK(launch_tc_gemm(256, c.tm_wa, c.tm_snt256, g, 1, c.s));
+    return QE_OK;
+}
+
+// R = P - s (C - z) Sigma_bar from the current codes (C - z held in qf).
+static qe_status residual(Ctx &c, const float *scales) {
+    const int64_t q = c.pl.q, p = c.pl.p, ld = c.pl.ld;
+    GemmArgs g = gemm_args(c, static_cast<int>(q), static_cast<int>(p), static_cast<int>(ceil_div(p, 64)),
+                           EPI_RFULL);
+    set_prods(g, 1);
+    g.a_plane_rows = static_cast<int>(q);
+    g.b_plane_rows = static_cast<int>(p);
+    g.out = c.R;
+    g.ldo = ld;
+    g.P = c.P;
+    g.ldp = ld;
+    g.scale = scales;
+    QE_CK(launch_tc_gemm(256, c.tm_qf, c.tm_snt256, g, 1, c.s));
+    return QE_OK;
+}
+
+// One cyclic sweep j = 1..p, blocked by B columns.
+static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float *zeros, int bits,
+                       bool first) {
+    const int64_t q = c.pl.q, p = c.pl.p, ld = c.pl.ld;
+    const int B = c.pl.B;
+    for (int64_t b0 = 0; b0 < p; b0 += B) {
+        const int bw = static_cast<int>((p - b0) < B ? (p - b0) : B);
+        int nsplit = 0;
+        if (b0 > 0) {
+            const int kb = static_cast<int>(b0 / 64);
+            const int S = kb < c.pl.smax ? kb : c.pl.smax;
+            GemmArgs g = gemm_args(c, static_cast<int>(q), bw, kb, EPI_TRAIL);
+            set_prods(g, first ? 2 : 1);
+            g.a_plane_rows = static_cast<int>(q);
+            g.b_plane_rows = static_cast<int>(p);
+            g.b_row0 = static_cast<int>(b0);
+            g.out = c.part;
+            g.ldo = B;
+            g.split_stride = q * B;
+            QE_CK(launch_tc_gemm(64, c.tm_dp, c.tm_snt64, g, S, c.s));
+            nsplit = S;
+        }
+        CdArgs a;
+        memset(&a, 0, sizeof(a));
+        a.q = q;
+        a.p = p;
+        a.b0 = b0;
+        a.bw = bw;
+        a.R = c.R;
+        a.ldr = ld;
+        a.part = c.part;
+        a.nsplit = nsplit;
+        a.part_stride = q * B;
+        a.ldpart = B;
+        a.snt = c.snt;
+        a.ldsn = ld;
+        a.snt_plane_rows = p;
+        a.scale = scales;
+        a.zero = zeros;
+        a.maxq = static_cast<float>((1 << bits) - 1);
+        a.first_sweep = first ? 1 : 0;
+        a.codes = codes;
+        a.ldc = p;
+        a.qf = c.qf;
+        a.ldq = ld;
+        a.dp = c.dp;
+        a.ldd = ld;
+        a.dp_plane_rows = q;
+        QE_CK(launch_cd_block(B, a, c.s));
+    }
+    return QE_OK;
+}
+
+static qe_status objective(Ctx &c, const void *W, int wbf16, int64_t ldw, const float *H,
+                           const uint8_t *codes, const float *scales, const float *zeros,
+                           const float *Rsrc, double *out) {
+    ObjArgs a;
+    memset(&a, 0, sizeof(a));
+    a.q = c.pl.q;
+    a.p = c.pl.p;
+    a.W = W;
+    a.w_bf16 = wbf16;
+    a.ldw = ldw;
+    a.H = H;
+    a.ldh = c.pl.ld;
+    a.codes = codes;
+    a.ldc = c.pl.p;
+    a.scale = scales;
+    a.zero = zeros;
+    a.d = c.d;
+    a.R = Rsrc;
+    a.ldr = c.pl.ld;
+    QE_CK(launch_objective(a, c.objp, out, c.s));
+    return QE_OK;
+}
+
+static qe_status check_opts(const qe_opts *o) {
+    if (!o) return QE_OK;
+    if (o->relax_period != 0 || o->structured_outliers != 0) return QE_ERR_UNSUPPORTED;
+    if (o->block_width != 0 && o->block_width != 64) return QE_ERR_UNSUPPORTED;
+    if (o->power_iters < 0) return QE_ERR_INVALID_ARG;
+    if (o->workspace && o->workspace_bytes == 0) return QE_ERR_INVALID_ARG;
+    return QE_OK;
+}
+
+static qe_status check_layer(const void *W, qe_dtype wt, int64_t q, int64_t p, int64_t ldw,
+                             const float *Sigma, int bits, int iters, const uint8_t *codes,
+                             const float *scales, const float *zeros, const double *obj) {
+    if (!W || !Sigma || !codes || !scales || !zeros || !obj) return QE_ERR_INVALID_ARG;
+    if (wt != QE_F32 && wt != QE_BF16) return QE_ERR_INVALID_ARG;
+    if (q < 1 || p < 1 || q > (1ll << 30) || p > (1ll << 30) || ldw < p) return QE_ERR_INVALID_ARG;
+    if (bits < 2 || bits > 8 || iters < 1) return QE_ERR_INVALID_ARG;
+    return QE_OK;
+}
+
+}  // namespace qe
+
+using namespace qe;
+
+extern "C" {
+
+int qe_version(void) { return 10000; }
+
+const char *qe_status_string(qe_status st) {
+    switch (st) {
+        case QE_OK: return "ok";
+        case QE_ERR_INVALID_ARG: return "invalid argument";
+        case QE_ERR_CUDA: return "CUDA error";
+        case QE_ERR_OOM: return "workspace allocation failed or too small";
+        case QE_ERR_NUMERIC: return "non-finite value in W or Sigma";
+        case QE_ERR_TIMEOUT: return "a device-side wait gave up";
+        case QE_ERR_UNSUPPORTED: return "option or layout not implemented";
+        default: return "unknown status";
+    }
+}
+
+qe_status qe_sync_status(qe_stream_t stream) {
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if (cudaStreamSynchronize(s) != cudaSuccess) {
+        cudaGetLastError();
+        return QE_ERR_CUDA;
+    }
+    unsigned *e = error_word();
+    if (!e) return QE_ERR_CUDA;
+    unsigned v = 0;
+    if (cudaMemcpyAsync(&v, e, sizeof(v), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+        cudaMemsetAsync(e, 0, sizeof(unsigned), s) != cudaSuccess || cudaStreamSynchronize(s) != cudaSuccess) {
+        cudaGetLastError();
+        return QE_ERR_CUDA;
+    }
+    if (v & ERR_TIMEOUT) return QE_ERR_TIMEOUT;
+    if (v & ERR_NUMERIC) return QE_ERR_NUMERIC;
+    return QE_OK;
+}
+
+qe_status qe_workspace_size(int64_t q, int64_t p, int outlier, const qe_opts *opts, size_t *bytes) {
+    if (!bytes || q < 1 || p < 1) return QE_ERR_INVALID_ARG;
+    const qe_status st = check_opts(opts);
+    if (st != QE_OK) return st;
+    const Plan pl = make_plan(q, p, kDefaultBlock, outlier != 0, 2, sm_count());
+    *bytes = pl.total;
+    return QE_OK;
+}
+
+qe_status qe_build_sigma(const void *X, qe_dtype x_dtype, qe_xlayout layout, int64_t p, int64_t n,
+                         int64_t ldx, float *Sigma, int accumulate, qe_stream_t stream) {
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if (!X || !Sigma || p < 1 || n < 0 || p > (1ll << 30)) return QE_ERR_INVALID_ARG;
+    if (x_dtype != QE_F32 && x_dtype != QE_BF16) return QE_ERR_INVALID_ARG;
+    if (layout != QE_FEATURE_MAJOR && layout != QE_TOKEN_MAJOR) return QE_ERR_INVALID_ARG;
+    if (layout == QE_FEATURE_MAJOR ? ldx < n : ldx < p) return QE_ERR_INVALID_ARG;
+    if (n == 0) {
+        if (!accumulate) QE_CK(cudaMemsetAsync(Sigma, 0, static_cast<size_t>(p) * p * 4, s));
+        return QE_OK;
+    }
+    unsigned *err = error_word();
+    if (!err) return QE_ERR_CUDA;
+    if (x_dtype == QE_F32) {
+        const float *Xf = static_cast<const float *>(X);
+        if (layout == QE_FEATURE_MAJOR) QE_CK(launch_sigma_f32(Xf, p, n, ldx, 1, Sigma, accumulate, s));
+        else QE_CK(launch_sigma_f32(Xf, p, n, 1, ldx, Sigma, accumulate, s));
+        return QE_OK;
+    }
+    GemmArgs g;
+    memset(&g, 0, sizeof(g));
+    g.M = static_cast<int>(p);
+    g.N = static_cast<int>(p);
+    g.n_prod = 1;
+    g.mode = EPI_SIGMA;
+    g.out = Sigma;
+    g.ldo = p;
+    g.err = err;
+    const bool direct = layout == QE_FEATURE_MAJOR && ((reinterpret_cast<uintptr_t>(X) & 15u) == 0) &&
+                        (ldx % 8 == 0);
+    if (direct) {
+        CUtensorMap ta, tb;
+        if (!make_tmap_bf16(&ta, X, p, n, ldx, 128) || !make_tmap_bf16(&tb, X, p, n, ldx, 256))
+            return QE_ERR_CUDA;
+        g.kb_count = static_cast<int>(ceil_div(n, 64));
+        g.accumulate = accumulate;
+        QE_CK(launch_tc_gemm(256, ta, tb, g, 1, s));
+        return QE_OK;
+    }
+    // Token-major or unaligned bf16 X: stage feature-major chunks of tokens.
+    const int64_t nc = n < 8192 ? round_up(n, 64) : 8192;
+    void *buf = nullptr;
+    if (cudaMallocAsync(&buf, static_cast<size_t>(p) * nc * 2, s) != cudaSuccess) {
+        cudaGetLastError();
+        return QE_ERR_OOM;
+    }
+    qe_status st = QE_OK;
+    CUtensorMap ta, tb;
+    if (!make_tmap_bf16(&ta, buf, p, nc, nc, 128) || !make_tmap_bf16(&tb, buf, p, nc, nc, 256)) st = QE_ERR_CUDA;
+    for (int64_t n0 = 0; st == QE_OK && n0 < n; n0 += nc) {
+        const int64_t len = (n - n0) < nc ? (n - n0) : nc;
+        cudaError_t e;
+        if (layout == QE_TOKEN_MAJOR) {
+            e = launch_transpose_bf16(X, n0, len, p, ldx, buf, nc, s);
+        } else {
+            e = cudaMemcpy2DAsync(buf, nc * 2, static_cast<const __nv_bfloat16 *>(X) + n0, ldx * 2, len * 2,
+                                  p, cudaMemcpyDeviceToDevice, s);
+        }
+        if (e == cudaSuccess && len < nc)  // zero the unused tail of the chunk
+            e = cudaMemset2DAsync(static_cast<__nv_bfloat16 *>(buf) + len, nc * 2, 0, (nc - len) * 2, p, s);
+        g.kb_count = static_cast<int>(ceil_div(len, 64));
+        g.accumulate = (n0 > 0) ? 1 : accumulate;
+        if (e == cudaSuccess) e = launch_tc_gemm(256, ta, tb, g, 1, s);
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            st = QE_ERR_CUDA;
+        }
+    }
+    cudaFreeAsync(buf, s);
+    return st;
+}
+
+qe_status qe_quantize_layer(const void *W, qe_dtype w_dtype, int64_t q, int64_t p, int64_t ldw,
+                            const float *Sigma, int bits, int iters, const qe_opts *opts,
+                            uint8_t *codes, float *scales, float *zeros, double *obj, qe_stream_t stream) {
+    qe_status st = check_layer(W, w_dtype, q, p, ldw, Sigma, bits, iters, codes, scales, zeros, obj);
+    if (st != QE_OK) return st;
+    if ((st = check_opts(opts)) != QE_OK) return st;
+    const int wbf16 = (w_dtype == QE_BF16);
+    Ctx c;
+    const Plan pl = make_plan(q, p, kDefaultBlock, false, wbf16 ? 1 : 2, sm_count());
+    if ((st = setup_ctx(c, pl, opts, reinterpret_cast<cudaStream_t>(stream))) != QE_OK) return st;
+
+    QE_CK(launch_grid(W, wbf16, ldw, nullptr, 0, q, p, bits, scales, zeros, c.err, c.s));
+    if ((st = prepare(c, W, wbf16, ldw, Sigma, c.P)) != QE_OK) return st;
+    if (opts && opts->wx_norm2)
+        if ((st = objective(c, W, wbf16, ldw, nullptr, nullptr, nullptr, nullptr, c.P, opts->wx_norm2)) != QE_OK)
+            return st;
+    const bool warm = opts && opts->init_codes;
+    if (warm) {
+        QE_CK(cudaMemcpyAsync(codes, opts->init_codes, static_cast<size_t>(q) * p, cudaMemcpyDeviceToDevice, c.s));
+        QE_CK(launch_codes_to_qf(codes, p, zeros, q, p, c.qf, pl.ld, c.s));
+        if ((st = residual(c, scales)) != QE_OK) return st;
+    } else {
+        QE_CK(launch_init_residual(W, wbf16, ldw, nullptr, 0, q, p, c.R, pl.ld, c.s));
+    }
+    for (int t = 0; t < iters; ++t) {
+        if ((st = sweep(c, codes, scales, zeros, bits, t == 0 && !warm)) != QE_OK) return st;
+        if ((st = residual(c, scales)) != QE_OK) return st;
+        if ((st = objective(c, W, wbf16, ldw, nullptr, codes, scales, zeros, c.R, obj + t)) != QE_OK) return st;
+        if (opts && opts->sweep_codes)
+            QE_CK(cudaMemcpyAsync(opts->sweep_codes + static_cast<size_t>(t) * q * p, codes,
+                                  static_cast<size_t>(q) * p, cudaMemcpyDeviceToDevice, c.s));
+    }
+    return QE_OK;
+}
+
+qe_status qe_quantize_layer_outlier(const void *W, qe_dtype w_dtype, int64_t q, int64_t p, int64_t ldw,
+                                    const float *Sigma, int bits, int iters, int64_t s_budget,
+                                    const qe_opts *opts, uint8_t *codes, float *scales, float *zeros,
+                                    float *H_val, int64_t *H_idx, int64_t *H_nnz, double *obj,
+                                    double *obj_cd, qe_stream_t stream) {
+    qe_status st = check_layer(W, w_dtype, q, p, ldw, Sigma, bits, iters, codes, scales, zeros, obj);
+    if (st != QE_OK) return st;
+    if ((st = check_opts(opts)) != QE_OK) return st;
+    const int64_t N = q * p;
+    if (s_budget < 0 || s_budget > N || N >= (1ll << 32) || !H_nnz) return QE_ERR_INVALID_ARG;
+    if (s_budget > 0 && (!H_val || !H_idx)) return QE_ERR_INVALID_ARG;
+    const int wbf16 = (w_dtype == QE_BF16);
+    const int power_iters = (opts && opts->power_iters > 0) ? opts->power_iters : kDefaultPowerIters;
+    Ctx c;
+    c.nsm = sm_count();
+    const Plan pl = make_plan(q, p, kDefaultBlock, true, wbf16 ? 1 : 2, c.nsm);
+    if ((st = setup_ctx(c, pl, opts, reinterpret_cast<cudaStream_t>(stream))) != QE_OK) return st;
+    const int64_t ld = pl.ld;
+
+    // H = P_s(W); the grid ignores those entries (Sec. 4.3)
+    QE_CK(launch_flat_copy(W, wbf16, ldw, q, p, c.T, c.s));
+    QE_CK(launch_topk(c.T, N, s_budget, c.st, c.cg, c.ce, c.sb, c.eb, H_idx, H_val, H_nnz, c.nsm, c.s));
+    QE_CK(cudaMemsetAsync(c.H, 0, static_cast<size_t>(q) * ld * 4, c.s));
+    QE_CK(launch_scatter_rowptr(H_idx, H_val, H_nnz, s_budget, q, p, c.H, ld, c.rowptr, c.s));
+    QE_CK(launch_grid(W, wbf16, ldw, c.H, ld, q, p, bits, scales, zeros, c.err, c.s));
+    // P_W = W (I + Sigma_bar), eta = 1 / (2 lambda_max), P = P_W - H (I + Sigma_bar)
+    if ((st = prepare(c, W, wbf16, ldw, Sigma, c.PW)) != QE_OK) return st;
+    QE_CK(launch_power_lambda(Sigma, p, p, power_iters, c.y0, c.y1, c.lam, c.eta, c.nsm, c.s));
+    QE_CK(launch_spmm_refresh(c.PW, c.P, c.R, ld, Sigma, p, c.d, c.dinv, H_idx, H_val, c.rowptr, q, p, 0, c.s));
+    if (opts && opts->wx_norm2)
+        if ((st = objective(c, W, wbf16, ldw, c.H, nullptr, nullptr, nullptr, c.P, opts->wx_norm2)) != QE_OK)
+            return st;
+    const bool warm = opts && opts->init_codes;
+    if (warm) {
+        QE_CK(cudaMemcpyAsync(codes, opts->init_codes, static_cast<size_t>(q) * p, cudaMemcpyDeviceToDevice, c.s));
+        QE_CK(launch_codes_to_qf(codes, p, zeros, q, p, c.qf, ld, c.s));
+        if ((st = residual(c, scales)) != QE_OK) return st;
+    } else {
+        QE_CK(launch_init_residual(W, wbf16, ldw, c.H, ld, q, p, c.R, ld, c.s));
+    }
+    for (int t = 0; t < iters; ++t) {
+        if ((st = sweep(c, codes, scales, zeros, bits, t == 0 && !warm)) != QE_OK) return st;
+        if ((st = residual(c, scales)) != QE_OK) return st;
+        if (obj_cd)
+            if ((st = objective(c, W, wbf16, ldw, c.H, codes, scales, zeros, c.R, obj_cd + t)) != QE_OK) return st;
+        // IHT step: T = H + 2 eta d (R - What); H = P_s(T)
+        QE_CK(launch_iht_target(c.H, c.R, ld, codes, p, scales, zeros, c.d, c.eta, q, p, c.T, c.s));
+        QE_CK(launch_topk(c.T, N, s_budget, c.st, c.cg, c.ce, c.sb, c.eb, H_idx, H_val, H_nnz, c.nsm, c.s));
+        QE_CK(cudaMemsetAsync(c.H, 0, static_cast<size_t>(q) * ld * 4, c.s));
+        QE_CK(launch_scatter_rowptr(H_idx, H_val, H_nnz, s_budget, q, p, c.H, ld, c.rowptr, c.s));
+        // P = P_W - H (I + Sigma_bar); R += P_new - P_old  (R = P - What Sigma_bar stays current)
+        QE_CK(launch_spmm_refresh(c.PW, c.P, c.R, ld, Sigma, p, c.d, c.dinv, H_idx, H_val, c.rowptr, q, p, 1, c.s));
+        if ((st = objective(c, W, wbf16, ldw, c.H, codes, scales, zeros, c.R, obj + t)) != QE_OK) return st;
+        if (opts && opts->sweep_codes)
+            QE_CK(cudaMemcpyAsync(opts->sweep_codes + static_cast<size_t>(t) * q * p, codes,
+                                  static_cast<size_t>(q) * p, cudaMemcpyDeviceToDevice, c.s));
+    }
+    return QE_OK;
+}
+
+}  // extern "C"

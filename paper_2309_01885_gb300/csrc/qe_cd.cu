@@ -1,0 +1,448 @@
+// Streaming and sequential kernels of the QuantEase CD path (Sec. 3.2):
+// per-row grid, Sigma normalisation into bf16 hi/lo planes of Sigma_bar^T,
+// the in-block sequential column updates (Lemma 1, Eq. cd-update-closed-2),
+// the objective reduction, plus the fp32 SIMT Sigma and the bf16 transpose.
+#include "qe_common.cuh"
+#include "qe_internal.h"
+#include "qe_kernels.h"
+
+namespace qe {
+
+__device__ __forceinline__ float load_elem(const void *base, int is_bf16, int64_t idx) {
+    if (is_bf16) return __bfloat162float(reinterpret_cast<const __nv_bfloat16 *>(base)[idx]);
+    return reinterpret_cast<const float *>(base)[idx];
+}
+
+// ---------------------------------------------------------------------------
+// Grid (Sec. 2.1): asymmetric per-row min/max with 0 in range, binary32.
+// One CTA of 256 threads per row.  Optional H (dense) is subtracted first, so
+// that the entries held by H (exactly equal to W there) leave the pool
+// (Sec. 4.3).  Non-finite entries latch ERR_NUMERIC.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) k_grid(const void *W, int w_bf16, int64_t ldw, const float *H,
+                                              int64_t ldh, int64_t p, float maxq, float *scale,
+                                              float *zero, unsigned *err) {
+    const int64_t i = blockIdx.x;
+    float lo = 0.0f, hi = 0.0f;
+    bool bad = false;
+    for (int64_t j = threadIdx.x; j < p; j += blockDim.x) {
+        float w = load_elem(W, w_bf16, i * ldw + j);
+        if (!isfinite(w)) bad = true;
+        if (H) w = w - H[i * ldh + j];
+        lo = fminf(lo, w);
+        hi = fmaxf(hi, w);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
+        hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
+    }
+    __shared__ float slo[8], shi[8];
+    __shared__ int sbad;
+    if (threadIdx.x == 0) sbad = 0;
+    __syncthreads();
+    if (bad) sbad = 1;
+    if ((threadIdx.x & 31) == 0) {
+        slo[threadIdx.x >> 5] = lo;
+        shi[threadIdx.x >> 5] = hi;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        for (int w = 1; w < (int)(blockDim.x >> 5); ++w) {
+            lo = fminf(lo, slo[w]);
+            hi = fmaxf(hi, shi[w]);
+        }
+        if (lo == 0.0f && hi == 0.0f) {
+            lo = -1.0f;
+            hi = 1.0f;
+        }
+        const float s = __fdiv_rn(__fsub_rn(hi, lo), maxq);
+        const float z = rintf(__fdiv_rn(-lo, s));
+        scale[i] = s;
+        zero[i] = z;
+        if (sbad) set_error(err, ERR_NUMERIC);
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Sigma normalisation (Algorithm 3 initialisation, footnote of Lemma 1):
+// d_j = Sigma_jj; a column with d_j <= 0 is dead.  SnT = Sigma_bar^T with
+// SnT[j][k] = Sigma[j][k] / d_j for k != j and j, k alive, 0 otherwise; this is
+// Sigma_bar[k][j] = Sigma[k][j] / Sigma_jj of the column-normalised matrix with
+// zero diagonal.  Stored as two bf16 planes (rows [0, p) = hi, [p, 2p) = lo).
+// ---------------------------------------------------------------------------
+__global__ void k_sigma_diag(const float *S, int64_t lds, int64_t p, float *d, unsigned *err) {
+    const int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+    if (j >= p) return;
+    const float v = S[j * lds + j];
+    if (!isfinite(v)) set_error(err, ERR_NUMERIC);
+    d[j] = v;
+}
+
+__global__ void k_sigma_planes(const float *S, int64_t lds, int64_t p, const float *d,
+                               __nv_bfloat16 *snt, int64_t ldn, unsigned *err) {
+    bool bad = false;
+    for (int64_t j = blockIdx.y; j < p; j += gridDim.y) {
+        const float dj = d[j];
+        const bool jalive = dj > 0.0f;
+        for (int64_t k = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; k < p;
+             k += (int64_t)gridDim.x * blockDim.x) {
+            const float sv = S[j * lds + k];
+            if (!isfinite(sv)) bad = true;
+            float x = 0.0f;
+            if (jalive && k != j && d[k] > 0.0f) x = __fdiv_rn(sv, dj);
+            const __nv_bfloat16 h = __float2bfloat16_rn(x);
+            const __nv_bfloat16 l = __float2bfloat16_rn(x - __bfloat162float(h));
+            snt[j * ldn + k] = h;
+            snt[(p + j) * ldn + k] = l;
+        }
+    }
+    if (bad) set_error(err, ERR_NUMERIC);
+}
+
+// ---------------------------------------------------------------------------
+// Operand planes of a q x p matrix for the tensor-core GEMM (rows [0,q) = hi,
+// [q, 2q) = lo when two planes).  fp32 input splits hi/lo; bf16 input copies.
+// ---------------------------------------------------------------------------
+__global__ void k_make_planes(const void *W, int w_bf16, int64_t ldw, int64_t q, int64_t p,
+                              int two_planes, __nv_bfloat16 *out, int64_t ldo) {
+    for (int64_t i = blockIdx.y; i < q; i += gridDim.y) {
+        for (int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; j < p;
+             j += (int64_t)gridDim.x * blockDim.x) {
+            const float w = load_elem(W, w_bf16, i * ldw + j);
+            const __nv_bfloat16 h = __float2bfloat16_rn(w);
+            out[i * ldo + j] = h;
+            if (two_planes) out[(q + i) * ldo + j] = __float2bfloat16_rn(w - __bfloat162float(h));
+        }
+    }
+}
+
+// R = W - H (fp32), the residual at the start of the first sweep: with
+// What = W - H, P - What Sigma_bar = (W - H)(I + Sigma_bar) - (W - H) Sigma_bar.
+__global__ void k_init_residual(const void *W, int w_bf16, int64_t ldw, const float *H, int64_t ldh,
+                                int64_t q, int64_t p, float *R, int64_t ldr) {
+    for (int64_t i = blockIdx.y; i < q; i += gridDim.y) {
+        for (int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; j < p;
+             j += (int64_t)gridDim.x * blockDim.x) {
+            float w = load_elem(W, w_bf16, i * ldw + j);
+            if (H) w -= H[i * ldh + j];
+            R[i * ldr + j] = w;
+        }
+    }
+}
+
+// (C - z) as bf16 (exact: |C - z| <= 255) for the R = P - s (C - z) Sigma_bar GEMM.
+__global__ void k_codes_to_qf(const uint8_t *codes, int64_t ldc, const float *zero, int64_t q,
+                              int64_t p, __nv_bfloat16 *qf, int64_t ldq) {
+    for (int64_t i = blockIdx.y; i < q; i += gridDim.y) {
+        const float z = zero[i];
+        for (int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; j < p;
+             j += (int64_t)gridDim.x * blockDim.x)
+            qf[i * ldq + j] = __float2bfloat16_rn(static_cast<float>(codes[i * ldc + j]) - z);
+    }
+}
+
+// ---------------------------------------------------------------------------
+// In-block sequential CD (Algorithm 3 inner loop, one column block of width B).
+// One thread per row i (rows are independent, Sec. 3.2).  Work in units of the
+// grid step: t_ij = beta_ij / s_i + z_i, so the code is rint(clamp(t, 0, 2^b-1))
+// (the nearest level, Eq. eq:quant) and the column change is
+// Delta'_ij = (What_start_ij - What_new_ij) / s_i = a_ij - c_ij with
+// a_ij = What_start_ij / s_i + z_i (an integer code after the first sweep).
+// On entry t for column l of the block is
+//     R_il / s_i + z_i + sum_split partial[split][i][l]
+// (R = P - What_start Sigma_bar, partial = Delta'[:, 0:b0] Sigma_bar[0:b0, block]);
+// the in-block contributions Delta'_ij Sigma_bar_jl (j < l in the block) are
+// added here, right after column j is decided.
+// ---------------------------------------------------------------------------
+template <int B>
+__global__ void __launch_bounds__(32) k_cd_block(const CdArgs a) {
+    constexpr int RP = B + 1;  // padded row of the per-row staging tiles
+    constexpr int SP = B + 4;  // padded row of the Sigma_bar block (16-byte aligned)
+    __shared__ __align__(16) float sig[B][SP];
+    __shared__ float cin[32][RP];
+    __shared__ float ain[32][RP];
+    const int lane = threadIdx.x;
+    const int64_t i0 = static_cast<int64_t>(blockIdx.x) * 32;
+    const int bw = a.bw;
+    const int64_t b0 = a.b0;
+
+    // Sigma_bar[b0 + k][b0 + l] = SnT[b0 + l][b0 + k] (hi + lo)
+    for (int idx = lane; idx < B * B; idx += 32) {
+        const int k = idx % B, l = idx / B;
+        float v = 0.0f;
+        if (k < bw && l < bw) {
+            const int64_t o = (b0 + l) * a.ldsn + b0 + k;
+            v = __bfloat162float(a.snt[o]) + __bfloat162float(a.snt[a.snt_plane_rows * a.ldsn + o]);
+        }
+        sig[k][l] = v;
+    }
+    // stage the block of t values and start values, coalesced over columns
+    for (int r = 0; r < 32; ++r) {
+        const int64_t i = i0 + r;
+        if (i >= a.q) {
+            for (int l = lane; l < B; l += 32) cin[r][l] = ain[r][l] = 0.0f;
+            continue;
+        }
+        const float s = a.scale[i], z = a.zero[i];
+        for (int l = lane; l < B; l += 32) {
+            float t = 0.0f, st = 0.0f;
+            if (l < bw) {
+                t = __fdiv_rn(a.R[i * a.ldr + b0 + l], s) + z;
+                st = a.first_sweep ? t : static_cast<float>(a.codes[i * a.ldc + b0 + l]);
+                for (int sp = 0; sp < a.nsplit; ++sp)
+                    t += a.part[sp * a.part_stride + i * a.ldpart + l];
+            }
+            cin[r][l] = t;
+            ain[r][l] = st;
+        }
+    }
+    __syncwarp();
+
+    // the sequential chain, one row per lane
+    float acc[B];
+#pragma unroll
+    for (int l = 0; l < B; ++l) acc[l] = cin[lane][l];
+    const float maxq = a.maxq;
+#pragma unroll
+    for (int j = 0; j < B; ++j) {
+        if (j < bw) {
+            const float c = rintf(fminf(fmaxf(acc[j], 0.0f), maxq));
+            const float dl = ain[lane][j] - c;
+            ain[lane][j] = dl;
+            cin[lane][j] = c;
+#pragma unroll
+            for (int l4 = ((j + 1) & ~3); l4 < B; l4 += 4) {
+                const float4 sv = *reinterpret_cast<const float4 *>(&sig[j][l4]);
+                if (l4 + 0 > j) acc[l4 + 0] = fmaf(dl, sv.x, acc[l4 + 0]);
+                if (l4 + 1 > j) acc[l4 + 1] = fmaf(dl, sv.y, acc[l4 + 1]);
+                if (l4 + 2 > j) acc[l4 + 2] = fmaf(dl, sv.z, acc[l4 + 2]);
+                if (l4 + 3 > j) acc[l4 + 3] = fmaf(dl, sv.w, acc[l4 + 3]);
+            }
+        }
+    }
+    __syncwarp();
+
+    // write codes, C - z and the Delta' plane(s), coalesced over columns
+    for (int r = 0; r < 32; ++r) {
+        const int64_t i = i0 + r;
+        if (i >= a.q) break;
+        const float z = a.zero[i];
+        for (int l = lane; l < bw; l += 32) {
+            const float c = cin[r][l];
+            const float dl = ain[r][l];
+            const int64_t col = b0 + l;
+            a.codes[i * a.ldc + col] = static_cast<uint8_t>(c);
+            a.qf[i * a.ldq + col] = __float2bfloat16_rn(c - z);
+            const __nv_bfloat16 h = __float2bfloat16_rn(dl);
+            a.dp[i * a.ldd + col] = h;
+            if (a.first_sweep)
+                a.dp[(a.dp_plane_rows + i) * a.ldd + col] = __float2bfloat16_rn(dl - __bfloat162float(h));
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Objective (proof of Lemma 1; Eq. main-outlier): with D = W - H - What and
+// R = P - What Sigma_bar current,  (D Sigma)_ij = d_j (R_ij - What_ij), so
+//     f = sum_ij D_ij d_j (R_ij - What_ij).
+// With codes == NULL it computes sum_ij (W - H)_ij d_j P_ij = ||(W - H) X||^2.
+// Per-CTA partial sums (fp64), reduced in a fixed order by k_sum_partials.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) k_objective(const ObjArgs a, double *partial) {
+    double acc = 0.0;
+    for (int64_t i = blockIdx.x; i < a.q; i += gridDim.x) {
+        const float s = a.codes ? a.scale[i] : 0.0f;
+        const float z = a.codes ? a.zero[i] : 0.0f;
+        for (int64_t j = threadIdx.x; j < a.p; j += blockDim.x) {
+            const float dj = a.d[j];
+            if (!(dj > 0.0f)) continue;
+            float t = load_elem(a.W, a.w_bf16, i * a.ldw + j);
+            if (a.H) t -= a.H[i * a.ldh + j];
+            const float r = a.R[i * a.ldr + j];
+            float term;
+            if (a.codes) {
+                const float wh = s * (static_cast<float>(a.codes[i * a.ldc + j]) - z);
+                term = (t - wh) * dj * (r - wh);
+            } else {
+                term = t * dj * r;
+            }
+            acc += static_cast<double>(term);
+        }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    __shared__ double sw[8];
+    if ((threadIdx.x & 31) == 0) sw[threadIdx.x >> 5] = acc;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double t = 0.0;
+        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += sw[w];
+        partial[blockIdx.x] = t;
+    }
+}
+
+__global__ void k_sum_partials(const double *partial, int n, double *out) {
+    __shared__ double sw[32];
+    double acc = 0.0;
+    for (int k = threadIdx.x; k < n; k += blockDim.x) acc += partial[k];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if ((threadIdx.x & 31) == 0) sw[threadIdx.x >> 5] = acc;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double t = 0.0;
+        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += sw[w];
+        *out = t;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Sigma for fp32 X on fp32 FMA (64 x 64 tiles on or above the diagonal,
+// mirrored).  X(a, k) = X[a * sa + k * sk] covers both layouts.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) k_sigma_f32(const float *X, int64_t p, int64_t n, int64_t sa,
+                                                   int64_t sk, float *S, int accumulate) {
+    const int ti = blockIdx.y, tj = blockIdx.x;
+    if (tj < ti) return;
+    __shared__ float As[16][68], Bs[16][68];
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+    const int64_t a0 = static_cast<int64_t>(ti) * 64, b0 = static_cast<int64_t>(tj) * 64;
+    float acc[4][4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int v = 0; v < 4; ++v) acc[u][v] = 0.0f;
+    const bool kfast = (sk == 1);
+    for (int64_t k0 = 0; k0 < n; k0 += 16) {
+        for (int e = threadIdx.x; e < 1024; e += 256) {
+            int kk, rr;
+            if (kfast) {
+                kk = e & 15;
+                rr = e >> 4;
+            } else {
+                rr = e & 63;
+                kk = e >> 6;
+            }
+            const int64_t k = k0 + kk, ra = a0 + rr, rb = b0 + rr;
+            As[kk][rr] = (k < n && ra < p) ? X[ra * sa + k * sk] : 0.0f;
+            Bs[kk][rr] = (k < n && rb < p) ? X[rb * sa + k * sk] : 0.0f;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int kk = 0; kk < 16; ++kk) {
+            float av[4], bv[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) av[u] = As[kk][ty * 4 + u];
+#pragma unroll
+            for (int v = 0; v < 4; ++v) bv[v] = Bs[kk][tx * 4 + v];
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+#pragma unroll
+                for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(av[u], bv[v], acc[u][v]);
+        }
+        __syncthreads();
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+            const int64_t r = a0 + ty * 4 + u, c = b0 + tx * 4 + v;
+            if (r < p && c < p && c >= r) {
+                float val = acc[u][v];
+                if (accumulate) val += S[r * p + c];
+                S[r * p + c] = val;
+                if (c != r) S[c * p + r] = val;
+            }
+        }
+}
+
+cudaError_t launch_sigma_f32(const float *X, int64_t p, int64_t n, int64_t sa, int64_t sk, float *S,
+                             int accumulate, cudaStream_t s) {
+    const unsigned t = static_cast<unsigned>(ceil_div(p, 64));
+    k_sigma_f32<<<dim3(t, t), 256, 0, s>>>(X, p, n, sa, sk, S, accumulate);
+    return cudaGetLastError();
+}
+
+// Token-major bf16 X (rows n0 .. n0+nc of an n x p matrix) -> feature-major p x nc.
+__global__ void k_transpose_bf16(const __nv_bfloat16 *X, int64_t n0, int64_t nc, int64_t p,
+                                 int64_t ldx, __nv_bfloat16 *out, int64_t ldo) {
+    __shared__ __nv_bfloat16 tile[32][33];
+    const int64_t kb = static_cast<int64_t>(blockIdx.x) * 32, fb = static_cast<int64_t>(blockIdx.y) * 32;
+    for (int r = threadIdx.y; r < 32; r += blockDim.y) {
+        const int64_t k = kb + r, f = fb + threadIdx.x;
+        tile[r][threadIdx.x] = (k < nc && f < p) ? X[(n0 + k) * ldx + f] : __float2bfloat16_rn(0.0f);
+    }
+    __syncthreads();
+    for (int r = threadIdx.y; r < 32; r += blockDim.y) {
+        const int64_t f = fb + r, k = kb + threadIdx.x;
+        if (f < p && k < nc) out[f * ldo + k] = tile[threadIdx.x][r];
+    }
+}
+
+cudaError_t launch_transpose_bf16(const void *X, int64_t n0, int64_t nc, int64_t p, int64_t ldx,
+                                  void *out, int64_t ld_out, cudaStream_t s) {
+    dim3 grid(static_cast<unsigned>(ceil_div(nc, 32)), static_cast<unsigned>(ceil_div(p, 32)));
+    k_transpose_bf16<<<grid, dim3(32, 8), 0, s>>>(reinterpret_cast<const __nv_bfloat16 *>(X), n0, nc,
+                                                  p, ldx, reinterpret_cast<__nv_bfloat16 *>(out),
+                                                  ld_out);
+    return cudaGetLastError();
+}
+
+// ---- launchers -------------------------------------------------------------
+static inline dim3 row_grid(int64_t rows, int64_t cols) {
+    const int64_t bx = ceil_div(cols, 256) < 16 ? ceil_div(cols, 256) : 16;
+    return dim3(static_cast<unsigned>(bx > 0 ? bx : 1), static_cast<unsigned>(rows < 65535 ? rows : 65535));
+}
+
+cudaError_t launch_grid(const void *W, int w_bf16, int64_t ldw, const float *H, int64_t ldh, int64_t q,
+                        int64_t p, int bits, float *scale, float *zero, unsigned *err, cudaStream_t s) {
+    k_grid<<<static_cast<unsigned>(q), 256, 0, s>>>(W, w_bf16, ldw, H, ldh, p,
+                                                    static_cast<float>((1 << bits) - 1), scale, zero,
+                                                    err);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_sigma_norm(const float *S, int64_t lds, int64_t p, float *d, __nv_bfloat16 *snt,
+                              int64_t ldn, unsigned *err, cudaStream_t s) {
+    k_sigma_diag<<<static_cast<unsigned>(ceil_div(p, 256)), 256, 0, s>>>(S, lds, p, d, err);
+    k_sigma_planes<<<row_grid(p, p), 256, 0, s>>>(S, lds, p, d, snt, ldn, err);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_make_planes(const void *W, int w_bf16, int64_t ldw, int64_t q, int64_t p,
+                               int two_planes, __nv_bfloat16 *out, int64_t ldo, cudaStream_t s) {
+    k_make_planes<<<row_grid(q, p), 256, 0, s>>>(W, w_bf16, ldw, q, p, two_planes, out, ldo);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_init_residual(const void *W, int w_bf16, int64_t ldw, const float *H, int64_t ldh,
+                                 int64_t q, int64_t p, float *R, int64_t ldr, cudaStream_t s) {
+    k_init_residual<<<row_grid(q, p), 256, 0, s>>>(W, w_bf16, ldw, H, ldh, q, p, R, ldr);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_codes_to_qf(const uint8_t *codes, int64_t ldc, const float *zero, int64_t q,
+                               int64_t p, __nv_bfloat16 *qf, int64_t ldq, cudaStream_t s) {
+    k_codes_to_qf<<<row_grid(q, p), 256, 0, s>>>(codes, ldc, zero, q, p, qf, ldq);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_cd_block(int B, const CdArgs &a, cudaStream_t s) {
+    const unsigned grid = static_cast<unsigned>(ceil_div(a.q, 32));
+    if (B == 64) k_cd_block<64><<<grid, 32, 0, s>>>(a);
+    else if (B == 32) k_cd_block<32><<<grid, 32, 0, s>>>(a);
+    else return cudaErrorInvalidValue;
+    return cudaGetLastError();
+}
+
+int objective_blocks(int64_t q) { return static_cast<int>(q < 1024 ? q : 1024); }
+
+cudaError_t launch_objective(const ObjArgs &a, double *partial, double *out, cudaStream_t s) {
+    const int nb = objective_blocks(a.q);
+    k_objective<<<nb, 256, 0, s>>>(a, partial);
+    k_sum_partials<<<1, 256, 0, s>>>(partial, nb, out);
+    return cudaGetLastError();
+}
+
+}  // namespace qe

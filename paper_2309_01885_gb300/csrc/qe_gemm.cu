@@ -1,0 +1,291 @@
+// Tensor-core GEMM of libqe: D[M x N] = sum_t A_{pa(t)} . B_{pb(t)}^T over K, on
+// tcgen05 (bf16 x bf16 -> fp32 accumulators in TMEM), operands fed by TMA in
+// 128-byte-swizzled K-major tiles.  One kernel serves four contractions of the
+// method, selected by the epilogue:
+//   Sigma = X X^T                         (Lemma 1; upper tiles + mirror)
+//   P = W (I + Sigma_bar)                 (Algorithm 3, "P = W Sigma^norm")
+//   R = P - s (C - z) Sigma_bar           (Algorithm 3, "P_hat = What Sigma^norm")
+//   partial_k = Delta' Sigma_bar[0:b0, block]  (Eq. cd-update-closed-2, the
+//                                          dW_{:,1:j} Sigma^norm_{1:j,j} term,
+//                                          deferred per column block, split-K)
+// fp32 accuracy for the Sigma_bar products comes from splitting an fp32 operand
+// into two bf16 planes (hi + lo) and summing the cross products in the same
+// TMEM accumulator (planes are stacked along rows in one tensor map).
+//
+// Warp roles (128 threads): warp 0 lane 0 issues TMA, warp 1 lane 0 issues MMA,
+// warp 2 owns the TMEM allocation, all four warps run the epilogue (warp w reads
+// TMEM lanes 32w..32w+31 = output rows).
+#include <cudaTypedefs.h>
+
+#include "qe_common.cuh"
+#include "qe_internal.h"
+
+namespace qe {
+
+template <int BN>
+struct GemmCfg {
+    static constexpr int BM = 128;
+    static constexpr int BK = 64;                       // 64 bf16 = one 128-byte swizzle row
+    static constexpr int A_BYTES = BM * BK * 2;
+    static constexpr int B_BYTES = BN * BK * 2;
+    static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+    static constexpr int STAGES = (BN == 256) ? 4 : (BN == 128) ? 6 : 8;
+    static constexpr int TMEM_COLS = BN;               // power of two >= 32
+    static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + 256;
+    static_assert(BN == 64 || BN == 128 || BN == 256, "BN");
+    static_assert(SMEM_BYTES <= 232448, "smem");
+};
+
+__device__ __forceinline__ float load_w(const GemmArgs &g, int64_t r, int64_t c) {
+    if (g.w_is_bf16)
+        return __bfloat162float(reinterpret_cast<const __nv_bfloat16 *>(g.W)[r * g.ldw + c]);
+    return reinterpret_cast<const float *>(g.W)[r * g.ldw + c];
+}
+
+// Epilogue for one thread: output row r, columns [c0, c0 + 32) of the window.
+__device__ __forceinline__ void epilogue_row(const GemmArgs &g, int r, int c0, const float (&v)[32],
+                                             int split) {
+    if (r >= g.M) return;
+    const int64_t rr = r;
+    switch (g.mode) {
+        case EPI_SIGMA: {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+                const int c = c0 + i;
+                if (c < g.N && c >= r) {
+                    float *a = g.out + rr * g.ldo + c;
+                    float *b = g.out + static_cast<int64_t>(c) * g.ldo + r;
+                    if (g.accumulate) {
+                        const float nv = *a + v[i];
+                        *a = nv;
+                        if (c != r) *b = nv;
+                    } else {
+                        *a = v[i];
+                        if (c != r) *b = v[i];
+                    }
+                }
+            }
+            break;
+        }
+        case EPI_PINIT: {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+                const int c = c0 + i;
+                if (c < g.N) g.out[rr * g.ldo + c] = load_w(g, rr, c) + v[i];
+            }
+            break;
+        }
+        case EPI_RFULL: {
+            const float s = g.scale[r];
+            const float *prow = g.P + rr * g.ldp;
+            float *orow = g.out + rr * g.ldo;
+            if (c0 + 32 <= g.N && ((g.ldo | g.ldp) & 3) == 0) {
+#pragma unroll
+                for (int i = 0; i < 32; i += 4) {
+                    const float4 pv = *reinterpret_cast<const float4 *>(prow + c0 + i);
+                    float4 o;
+                    o.x = fmaf(-s, v[i + 0], pv.x);
+                    o.y = fmaf(-s, v[i + 1], pv.y);
+                    o.z = fmaf(-s, v[i + 2], pv.z);
+                    o.w = fmaf(-s, v[i + 3], pv.w);
+                    *reinterpret_cast<float4 *>(orow + c0 + i) = o;
+                }
+            } else {
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    const int c = c0 + i;
+                    if (c < g.N) orow[c] = fmaf(-s, v[i], prow[c]);
+                }
+            }
+            break;
+        }
+        case EPI_TRAIL: {
+            float *orow = g.out + static_cast<int64_t>(split) * g.split_stride + rr * g.ldo;
+            if (c0 + 32 <= g.N && (g.ldo & 3) == 0 && (g.split_stride & 3) == 0) {
+#pragma unroll
+                for (int i = 0; i < 32; i += 4)
+                    *reinterpret_cast<float4 *>(orow + c0 + i) =
+                        make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+            } else {
+#pragma unroll
+                for (int i = 0; i < 32; ++i)
+                    if (c0 + i < g.N) orow[c0 + i] = v[i];
+            }
+            break;
+        }
+        default:
+            break;
+    }
+}
+
+template <int BN>
+__global__ void __launch_bounds__(128, 1)
+    k_tc_gemm(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb,
+              const GemmArgs g) {
+    using C = GemmCfg<BN>;
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t pad = (1024u - (smem_u32(smem_raw) & 1023u)) & 1023u;
+    uint8_t *smem = smem_raw + pad;
+    uint64_t *full = reinterpret_cast<uint64_t *>(smem + C::STAGES * C::STAGE_BYTES);
+    uint64_t *empty = full + C::STAGES;
+    uint64_t *done = empty + C::STAGES;
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(done + 1);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const int m0 = blockIdx.y * C::BM;
+    const int n0 = blockIdx.x * BN;
+    // Sigma: a tile whose every element lies strictly below the diagonal is
+    // produced by the mirror of its transpose (uniform exit, before any barrier).
+    if (g.mode == EPI_SIGMA && n0 + BN <= m0) return;
+
+    const int split = blockIdx.z;
+    const int splits = gridDim.z;
+    const int kb_lo = g.kb_begin + static_cast<int>((static_cast<long long>(g.kb_count) * split) / splits);
+    const int kb_hi =
+        g.kb_begin + static_cast<int>((static_cast<long long>(g.kb_count) * (split + 1)) / splits);
+    const int nsteps = (kb_hi - kb_lo) * g.n_prod;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < C::STAGES; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        mbar_init(done, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 0 && lane == 0) {
+        prefetch_tensormap(&ta);
+        prefetch_tensormap(&tb);
+    }
+    if (warp == 2) tmem_alloc(tmem_slot, C::TMEM_COLS);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    if (warp == 0 && lane == 0) {
+        // ---- TMA producer ----
+        for (int st = 0; st < nsteps; ++st) {
+            const int s = st % C::STAGES;
+            const uint32_t ph = (st / C::STAGES) & 1u;
+            if (!mbar_wait_bounded(&empty[s], ph ^ 1u, abort_flag)) {
+                *abort_flag = 1;
+                set_error(g.err, ERR_TIMEOUT);
+                break;
+            }
+            const int kb = kb_lo + st / g.n_prod;
+            const int t = st % g.n_prod;
+            uint8_t *sa = smem + s * C::STAGE_BYTES;
+            uint8_t *sb = sa + C::A_BYTES;
+            mbar_arrive_expect_tx(&full[s], C::STAGE_BYTES);
+            tma_load_2d(&ta, sa, &full[s], kb * C::BK, g.a_row0 + m0 + g.prod_a[t] * g.a_plane_rows);
+            tma_load_2d(&tb, sb, &full[s], kb * C::BK, g.b_row0 + n0 + g.prod_b[t] * g.b_plane_rows);
+        }
+    } else if (warp == 1 && lane == 0) {
+        // ---- MMA issuer ----
+        constexpr uint32_t idesc = idesc_bf16_f32(C::BM, BN);
+        for (int st = 0; st < nsteps; ++st) {
+            const int s = st % C::STAGES;
+            const uint32_t ph = (st / C::STAGES) & 1u;
+            if (!mbar_wait_bounded(&full[s], ph, abort_flag)) {
+                *abort_flag = 1;
+                set_error(g.err, ERR_TIMEOUT);
+                break;
+            }
+            tc_fence_after();
+            const uint32_t sa = smem_u32(smem + s * C::STAGE_BYTES);
+            const uint64_t da = smem_desc_k128(sa);
+            const uint64_t db = smem_desc_k128(sa + C::A_BYTES);
+#pragma unroll
+            for (int k = 0; k < C::BK / 16; ++k)
+                mma_bf16_ss(tmem, da + 2u * k, db + 2u * k, idesc, (st | k) != 0 ? 1u : 0u);
+            mma_commit(&empty[s]);
+        }
+        mma_commit(done);  // arrives when every MMA issued above has completed
+    }
+    __syncwarp();
+
+    // ---- epilogue: TMEM -> registers -> global ----
+    const bool ok = mbar_wait_bounded(done, 0u, nullptr);
+    if (!ok && threadIdx.x == 0) set_error(g.err, ERR_TIMEOUT);
+    tc_fence_after();
+    const bool valid = ok && (*abort_flag == 0);
+    const int r = m0 + warp * 32 + lane;
+    const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+    for (int c = 0; c < BN; c += 32) {
+        if (n0 + c >= g.N) break;  // uniform over the CTA
+        float v[32];
+        if (nsteps > 0) {
+            tmem_ld_32x32b_x32(trow + static_cast<uint32_t>(c), v);
+        } else {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = 0.0f;
+        }
+        if (valid) epilogue_row(g, r, n0 + c, v, split);
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 2) tmem_dealloc(tmem, C::TMEM_COLS);
+}
+
+// ---- host side ---------------------------------------------------------------
+static PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+static bool get_encode() {
+    if (g_encode) return true;
+    void *fn = nullptr;
+    cudaDriverEntryPointQueryResult qres;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
+                                         &qres) != cudaSuccess ||
+        qres != cudaDriverEntryPointSuccess || fn == nullptr)
+        return false;
+    g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    return true;
+}
+
+bool make_tmap_bf16(CUtensorMap *map, const void *base, uint64_t rows, uint64_t cols, uint64_t ld,
+                    uint32_t box_rows) {
+    if (!get_encode()) return false;
+    if ((reinterpret_cast<uintptr_t>(base) & 15u) != 0 || ((ld * 2) & 15u) != 0) return false;
+    if (rows == 0 || cols == 0 || box_rows == 0 || box_rows > 256) return false;
+    cuuint64_t dims[2] = {cols, rows};
+    cuuint64_t strides[1] = {ld * 2};
+    cuuint32_t box[2] = {64, box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    const CUresult r =
+        g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides,
+                 box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                 CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+template <int BN>
+static cudaError_t launch_bn(const CUtensorMap &ta, const CUtensorMap &tb, const GemmArgs &g,
+                             int splits, cudaStream_t s) {
+    using C = GemmCfg<BN>;
+    cudaError_t e = cudaFuncSetAttribute(k_tc_gemm<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         C::SMEM_BYTES);
+    if (e != cudaSuccess) return e;
+    dim3 grid(static_cast<unsigned>(ceil_div(g.N, BN)), static_cast<unsigned>(ceil_div(g.M, C::BM)),
+              static_cast<unsigned>(splits));
+    k_tc_gemm<BN><<<grid, 128, C::SMEM_BYTES, s>>>(ta, tb, g);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_tc_gemm(int BN, const CUtensorMap &ta, const CUtensorMap &tb, const GemmArgs &g,
+                           int splits, cudaStream_t s) {
+    if (g.M <= 0 || g.N <= 0 || splits < 1 || g.n_prod < 1 || g.n_prod > 3)
+        return cudaErrorInvalidValue;
+    if (ceil_div(g.M, 128) > 65535 || splits > 65535) return cudaErrorInvalidValue;
+    switch (BN) {
+        case 64: return launch_bn<64>(ta, tb, g, splits, s);
+        case 128: return launch_bn<128>(ta, tb, g, splits, s);
+        case 256: return launch_bn<256>(ta, tb, g, splits, s);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
+}  // namespace qe

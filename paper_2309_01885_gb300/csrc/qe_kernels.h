@@ -1,0 +1,62 @@
+// Argument blocks and launchers of the streaming / sequential kernels of libqe.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace qe {
+
+// In-block sequential CD over one column block [b0, b0 + bw).
+struct CdArgs {
+    int64_t q, p;
+    int64_t b0;
+    int bw;
+    const float *R;                 // residual P - What_start Sigma_bar (q x ldr)
+    int64_t ldr;
+    const float *part;              // split-K partials [nsplit][q][ldpart] (t-units)
+    int nsplit;
+    int64_t part_stride, ldpart;
+    const __nv_bfloat16 *snt;       // Sigma_bar^T hi plane; lo plane snt_plane_rows rows below
+    int64_t ldsn, snt_plane_rows;
+    const float *scale, *zero;
+    float maxq;
+    int first_sweep;                // What_start is R itself (not on the grid)
+    uint8_t *codes;                 // in: codes at sweep start (unless first_sweep); out: new codes
+    int64_t ldc;
+    __nv_bfloat16 *qf;              // out: C - z
+    int64_t ldq;
+    __nv_bfloat16 *dp;              // out: Delta' hi plane (lo plane dp_plane_rows rows below)
+    int64_t ldd, dp_plane_rows;
+};
+
+// Objective / reference-norm reduction.
+struct ObjArgs {
+    int64_t q, p;
+    const void *W;
+    int w_bf16;
+    int64_t ldw;
+    const float *H;                 // dense outlier matrix or NULL
+    int64_t ldh;
+    const uint8_t *codes;           // NULL: reference norm sum (W-H)_ij d_j R_ij
+    int64_t ldc;
+    const float *scale, *zero, *d;
+    const float *R;                 // residual (or P for the reference norm)
+    int64_t ldr;
+};
+
+cudaError_t launch_grid(const void *W, int w_bf16, int64_t ldw, const float *H, int64_t ldh, int64_t q,
+                        int64_t p, int bits, float *scale, float *zero, unsigned *err, cudaStream_t s);
+cudaError_t launch_sigma_norm(const float *S, int64_t lds, int64_t p, float *d, __nv_bfloat16 *snt,
+                              int64_t ldn, unsigned *err, cudaStream_t s);
+cudaError_t launch_make_planes(const void *W, int w_bf16, int64_t ldw, int64_t q, int64_t p,
+                               int two_planes, __nv_bfloat16 *out, int64_t ldo, cudaStream_t s);
+cudaError_t launch_init_residual(const void *W, int w_bf16, int64_t ldw, const float *H, int64_t ldh,
+                                 int64_t q, int64_t p, float *R, int64_t ldr, cudaStream_t s);
+cudaError_t launch_codes_to_qf(const uint8_t *codes, int64_t ldc, const float *zero, int64_t q,
+                               int64_t p, __nv_bfloat16 *qf, int64_t ldq, cudaStream_t s);
+cudaError_t launch_cd_block(int B, const CdArgs &a, cudaStream_t s);
+int objective_blocks(int64_t q);
+cudaError_t launch_objective(const ObjArgs &a, double *partial, double *out, cudaStream_t s);
+
+}  // namespace qe

@@ -1,0 +1,411 @@
+// Kernels of the outlier-aware variant (Sec. 4.3, Algorithm 4): lambda_max by
+// the power method, the IHT target T = H - eta grad_H g, the hard-thresholding
+// operator P_s as a radix select + stable compaction, and the sparse refresh
+// P = P_W - H (I + Sigma_bar).
+#include "qe_common.cuh"
+#include "qe_outlier.h"
+
+namespace qe {
+
+// ---- block reductions ------------------------------------------------------
+__device__ __forceinline__ double block_sum(double v, double *sh) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+    __syncthreads();
+    if (l == 0) sh[w] = v;
+    __syncthreads();
+    double t = 0.0;
+    for (int k = 0; k < (int)(blockDim.x >> 5); ++k) t += sh[k];
+    return t;
+}
+
+// Exclusive scan of one unsigned value per thread over the CTA (blockDim <= 1024).
+__device__ __forceinline__ unsigned block_excl_scan(unsigned v, unsigned *sh, unsigned *total) {
+    const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+    unsigned x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const unsigned y = __shfl_up_sync(0xffffffffu, x, o);
+        if (l >= o) x += y;
+    }
+    __syncthreads();
+    if (l == 31) sh[w] = x;
+    __syncthreads();
+    if (w == 0) {
+        const int nw = blockDim.x >> 5;
+        unsigned s = (l < nw) ? sh[l] : 0u;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const unsigned y = __shfl_up_sync(0xffffffffu, s, o);
+            if (l >= o) s += y;
+        }
+        if (l < nw) sh[l] = s;
+    }
+    __syncthreads();
+    const unsigned warp_base = (w > 0) ? sh[w - 1] : 0u;
+    if (total) *total = sh[(blockDim.x >> 5) - 1];
+    return warp_base + x - v;
+}
+
+// ---- power method (Sec. 4.3: lambda_max(X X^T) "by iterative power method") --
+// y_out = Sigma (y_in / ||y_in||); every CTA recomputes ||y_in||.
+__global__ void __launch_bounds__(256) k_power_step(const float *S, int64_t lds, int64_t p,
+                                                    const float *y_in, float *y_out) {
+    __shared__ double sh[8];
+    double n2 = 0.0;
+    for (int64_t k = threadIdx.x; k < p; k += blockDim.x) n2 += (double)y_in[k] * y_in[k];
+    n2 = block_sum(n2, sh);
+    const float inv = n2 > 0.0 ? static_cast<float>(1.0 / sqrt(n2)) : 0.0f;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    for (int64_t a = (int64_t)blockIdx.x * 8 + warp; a < p; a += (int64_t)gridDim.x * 8) {
+        float acc = 0.0f;
+        for (int64_t b = lane; b < p; b += 32) acc = fmaf(S[a * lds + b], y_in[b], acc);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+        if (lane == 0) y_out[a] = acc * inv;
+    }
+}
+
+// lambda = (y/||y||) . z with z = Sigma (y/||y||); eta = 1 / (2 lambda).
+__global__ void __launch_bounds__(256) k_power_final(const float *y, const float *z, int64_t p,
+                                                     double *lam, double *eta) {
+    __shared__ double sh[8];
+    double n2 = 0.0, dz = 0.0;
+    for (int64_t k = threadIdx.x; k < p; k += blockDim.x) {
+        n2 += (double)y[k] * y[k];
+        dz += (double)y[k] * z[k];
+    }
+    n2 = block_sum(n2, sh);
+    dz = block_sum(dz, sh);
+    if (threadIdx.x == 0) {
+        const double l = n2 > 0.0 ? dz / sqrt(n2) : 0.0;
+        *lam = l;
+        *eta = l > 0.0 ? 1.0 / (2.0 * l) : 0.0;
+    }
+}
+
+__global__ void k_fill(float *y, int64_t n, float v) {
+    const int64_t k = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+    if (k < n) y[k] = v;
+}
+
+// ---- IHT target (Eq. iht-update, Algorithm 4) --------------------------------
+// grad_H g = 2 (H + What - W) Sigma = -2 D Sigma and (D Sigma)_ij = d_j (R_ij - What_ij),
+// so T = H - eta grad = H + 2 eta d_j (R_ij - What_ij).  T is written flat (ld = p).
+__global__ void k_iht_target(const float *H, const float *R, int64_t ld, const uint8_t *codes,
+                             int64_t ldc, const float *scale, const float *zero, const float *d,
+                             const double *eta, int64_t q, int64_t p, float *T) {
+    for (int64_t i = blockIdx.y; i < q; i += gridDim.y) {
+        const float e2 = static_cast<float>(2.0 * (*eta));
+        const float s = scale[i], z = zero[i];
+        for (int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; j < p;
+             j += (int64_t)gridDim.x * blockDim.x) {
+            const float dj = d[j] > 0.0f ? d[j] : 0.0f;
+            const float wh = s * (static_cast<float>(codes[i * ldc + j]) - z);
+            T[i * p + j] = H[i * ld + j] + e2 * dj * (R[i * ld + j] - wh);
+        }
+    }
+}
+
+// Flat copy of a q x p matrix (bf16 / fp32, leading dimension ldw) into T (ld = p).
+__global__ void k_flat_copy(const void *W, int w_bf16, int64_t ldw, int64_t q, int64_t p, float *T) {
+    for (int64_t i = blockIdx.y; i < q; i += gridDim.y) {
+        for (int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; j < p;
+             j += (int64_t)gridDim.x * blockDim.x) {
+            const float w = w_bf16 ? __bfloat162float(reinterpret_cast<const __nv_bfloat16 *>(W)[i * ldw + j])
+                                   : reinterpret_cast<const float *>(W)[i * ldw + j];
+            T[i * p + j] = w;
+        }
+    }
+}
+
+// ---- P_s: radix select of the s-th largest nonzero |T| ----------------------
+// Keys are the binary32 magnitudes (sign bit cleared): for non-negative floats
+// the unsigned bit pattern orders like the value.  Four 8-bit digit passes find
+// kstar; then exactly count_gt keys are > kstar and need_eq keys == kstar are
+// taken in ascending linear index (the tie rule).
+__device__ __forceinline__ unsigned mag_key(float v) { return __float_as_uint(v) & 0x7fffffffu; }
+
+__global__ void __launch_bounds__(256) k_topk_hist(const float *T, int64_t N, TopkState *st, int shift,
+                                                   unsigned mask_hi) {
+    __shared__ unsigned h[256];
+    h[threadIdx.x] = 0;
+    __syncthreads();
+    const unsigned prefix = st->prefix;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < N; e += stride) {
+        const unsigned k = mag_key(T[e]);
+        if (k == 0u || ((k ^ prefix) & mask_hi) != 0u) continue;
+        atomicAdd(&h[(k >> shift) & 255u], 1u);
+    }
+    __syncthreads();
+    if (h[threadIdx.x]) atomicAdd(&st->hist[threadIdx.x], h[threadIdx.x]);
+}
+
+__global__ void k_topk_pick(TopkState *st, int shift, int64_t s_budget, int first) {
+    if (threadIdx.x != 0) return;
+    if (first) {
+        unsigned long long total = 0;
+        for (int b = 0; b < 256; ++b) total += st->hist[b];
+        st->count_gt = 0;
+        st->prefix = 0;
+        const unsigned long long want = (unsigned long long)s_budget < total ? (unsigned long long)s_budget : total;
+        st->remaining = static_cast<unsigned>(want);
+        st->empty = (want == 0) ? 1u : 0u;
+    }
+    if (!st->empty) {
+        unsigned cum = 0;
+        int b = 255;
+        for (; b > 0; --b) {
+            if (cum + st->hist[b] >= st->remaining) break;
+            cum += st->hist[b];
+        }
+        st->prefix |= static_cast<unsigned>(b) << shift;
+        st->count_gt += cum;
+        st->remaining -= cum;
+    }
+    for (int b = 0; b < 256; ++b) st->hist[b] = 0;
+    if (shift == 0) {
+        st->kstar = st->empty ? 0xffffffffu : st->prefix;
+        st->need_eq = st->empty ? 0u : st->remaining;
+    }
+}
+
+constexpr int kChunk = 4096;   // elements per CTA in the compaction (256 threads x 16)
+
+__global__ void __launch_bounds__(256) k_topk_count(const float *T, int64_t N, const TopkState *st,
+                                                    unsigned *cnt_gt, unsigned *cnt_eq) {
+    __shared__ unsigned sh[32];
+    const unsigned kstar = st->kstar;
+    const int64_t base = (int64_t)blockIdx.x * kChunk + threadIdx.x * 16;
+    unsigned g = 0, q = 0;
+    for (int u = 0; u < 16; ++u) {
+        const int64_t e = base + u;
+        if (e >= N) break;
+        const unsigned k = mag_key(T[e]);
+        if (k == 0u) continue;
+        g += (k > kstar) ? 1u : 0u;
+        q += (k == kstar) ? 1u : 0u;
+    }
+    unsigned tg, tq;
+    block_excl_scan(g, sh, &tg);
+    block_excl_scan(q, sh, &tq);
+    if (threadIdx.x == 0) {
+        cnt_gt[blockIdx.x] = tg;
+        cnt_eq[blockIdx.x] = tq;
+    }
+}
+
+// One CTA: exclusive scans over the chunks.  sel_base[c] = first output slot of
+// chunk c, eq_base[c] = number of keys == kstar in chunks before c.
+__global__ void __launch_bounds__(1024) k_topk_scan(const unsigned *cnt_gt, const unsigned *cnt_eq,
+                                                    int nchunks, const TopkState *st, unsigned *sel_base,
+                                                    unsigned *eq_base, int64_t *nnz_out) {
+    __shared__ unsigned sh[32];
+    const unsigned need = st->need_eq;
+    unsigned carry_eq = 0, carry_sel = 0;
+    for (int c0 = 0; c0 < nchunks; c0 += blockDim.x) {
+        const int c = c0 + threadIdx.x;
+        const unsigned ge = (c < nchunks) ? cnt_gt[c] : 0u;
+        const unsigned qe_ = (c < nchunks) ? cnt_eq[c] : 0u;
+        unsigned tq;
+        const unsigned eqb = carry_eq + block_excl_scan(qe_, sh, &tq);
+        unsigned take = 0;
+        if (need > eqb) take = (need - eqb) < qe_ ? (need - eqb) : qe_;
+        const unsigned sel = ge + take;
+        unsigned ts;
+        const unsigned sb = carry_sel + block_excl_scan(sel, sh, &ts);
+        if (c < nchunks) {
+            sel_base[c] = sb;
+            eq_base[c] = eqb;
+        }
+        carry_eq += tq;
+        carry_sel += ts;
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) *nnz_out = static_cast<int64_t>(carry_sel);
+}
+
+__global__ void __launch_bounds__(256) k_topk_emit(const float *T, int64_t N, const TopkState *st,
+                                                   const unsigned *sel_base, const unsigned *eq_base,
+                                                   int64_t *H_idx, float *H_val) {
+    __shared__ unsigned sh[32];
+    const unsigned kstar = st->kstar, need = st->need_eq;
+    const int64_t base = (int64_t)blockIdx.x * kChunk + threadIdx.x * 16;
+    unsigned ng = 0, nq = 0;
+    for (int u = 0; u < 16; ++u) {
+        const int64_t e = base + u;
+        if (e >= N) break;
+        const unsigned k = mag_key(T[e]);
+        if (k == 0u) continue;
+        ng += (k > kstar) ? 1u : 0u;
+        nq += (k == kstar) ? 1u : 0u;
+    }
+    const unsigned eq0 = eq_base[blockIdx.x] + block_excl_scan(nq, sh, nullptr);
+    unsigned take = 0;
+    if (need > eq0) take = (need - eq0) < nq ? (need - eq0) : nq;
+    unsigned out = sel_base[blockIdx.x] + block_excl_scan(ng + take, sh, nullptr);
+    unsigned eqseen = 0;
+    for (int u = 0; u < 16; ++u) {
+        const int64_t e = base + u;
+        if (e >= N) break;
+        const float v = T[e];
+        const unsigned k = mag_key(v);
+        if (k == 0u) continue;
+        bool keep = k > kstar;
+        if (k == kstar) {
+            keep = eqseen < take;
+            ++eqseen;
+        }
+        if (keep) {
+            H_idx[out] = e;
+            H_val[out] = v;
+            ++out;
+        }
+    }
+}
+
+// Dense H from the kept entries (H zeroed before).
+__global__ void k_scatter(const int64_t *H_idx, const float *H_val, const int64_t *nnz, int64_t cap,
+                          int64_t p, float *H, int64_t ld) {
+    const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+    if (t >= cap || t >= *nnz) return;
+    const int64_t e = H_idx[t];
+    H[(e / p) * ld + (e % p)] = H_val[t];
+}
+
+// rowptr[i] = first kept entry with linear index >= i * p (entries are sorted).
+__global__ void k_rowptr(const int64_t *H_idx, const int64_t *nnz, int64_t q, int64_t p,
+                         int64_t *rowptr) {
+    const int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+    if (i > q) return;
+    const int64_t key = i * p;
+    int64_t lo = 0, hi = *nnz;
+    while (lo < hi) {
+        const int64_t mid = (lo + hi) >> 1;
+        if (H_idx[mid] < key) lo = mid + 1;
+        else hi = mid;
+    }
+    rowptr[i] = lo;
+}
+
+// P_new = P_W - H (I + Sigma_bar) for row i (Sigma_bar_kj = Sigma_kj / d_j off
+// the diagonal, 0 for dead columns); R += P_new - P_old when update_r; P = P_new.
+__global__ void __launch_bounds__(256) k_spmm_refresh(const float *PW, float *P, float *R, int64_t ld,
+                                                      const float *S, int64_t lds, const float *d,
+                                                      const float *dinv, const int64_t *H_idx,
+                                                      const float *H_val, const int64_t *rowptr,
+                                                      int64_t p, int update_r) {
+    const int64_t i = blockIdx.x;
+    const int64_t e0 = rowptr[i], e1 = rowptr[i + 1];
+    for (int64_t j = threadIdx.x; j < p; j += blockDim.x) {
+        float acc = PW[i * ld + j];
+        const float dj = d[j];
+        const float ij = dinv[j];
+        for (int64_t e = e0; e < e1; ++e) {
+            const int64_t k = H_idx[e] - i * p;
+            const float v = H_val[e];
+            float sb;
+            if (k == j) sb = 1.0f;
+            else sb = (dj > 0.0f && d[k] > 0.0f) ? S[k * lds + j] * ij : 0.0f;
+            acc = fmaf(-v, sb, acc);
+        }
+        if (update_r) R[i * ld + j] += acc - P[i * ld + j];
+        P[i * ld + j] = acc;
+    }
+}
+
+__global__ void k_dinv(const float *d, int64_t p, float *dinv) {
+    const int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+    if (j < p) dinv[j] = d[j] > 0.0f ? 1.0f / d[j] : 0.0f;
+}
+
+// ---- launchers --------------------------------------------------------------
+static inline dim3 rows_grid(int64_t rows, int64_t cols) {
+    int64_t bx = ceil_div(cols, 256);
+    if (bx > 16) bx = 16;
+    if (bx < 1) bx = 1;
+    return dim3(static_cast<unsigned>(bx), static_cast<unsigned>(rows < 65535 ? rows : 65535));
+}
+
+cudaError_t launch_power_lambda(const float *S, int64_t lds, int64_t p, int iters, float *y0, float *y1,
+                                double *lam, double *eta, int nsm, cudaStream_t s) {
+    k_fill<<<static_cast<unsigned>(ceil_div(p, 256)), 256, 0, s>>>(y0, p, 1.0f);
+    int64_t blocks = ceil_div(p, 8);
+    if (blocks > nsm * 4) blocks = nsm * 4;
+    float *a = y0, *b = y1;
+    for (int it = 0; it <= iters; ++it) {
+        k_power_step<<<static_cast<unsigned>(blocks), 256, 0, s>>>(S, lds, p, a, b);
+        if (it < iters) {
+            float *t = a;
+            a = b;
+            b = t;
+        }
+    }
+    // a = y_iters, b = Sigma (y_iters / ||y_iters||)
+    k_power_final<<<1, 256, 0, s>>>(a, b, p, lam, eta);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_iht_target(const float *H, const float *R, int64_t ld, const uint8_t *codes,
+                              int64_t ldc, const float *scale, const float *zero, const float *d,
+                              const double *eta, int64_t q, int64_t p, float *T, cudaStream_t s) {
+    k_iht_target<<<rows_grid(q, p), 256, 0, s>>>(H, R, ld, codes, ldc, scale, zero, d, eta, q, p, T);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_flat_copy(const void *W, int w_bf16, int64_t ldw, int64_t q, int64_t p, float *T,
+                             cudaStream_t s) {
+    k_flat_copy<<<rows_grid(q, p), 256, 0, s>>>(W, w_bf16, ldw, q, p, T);
+    return cudaGetLastError();
+}
+
+int64_t topk_chunks(int64_t N) { return ceil_div(N, kChunk); }
+
+cudaError_t launch_topk(const float *T, int64_t N, int64_t s_budget, TopkState *st, unsigned *cnt_gt,
+                        unsigned *cnt_eq, unsigned *sel_base, unsigned *eq_base, int64_t *H_idx,
+                        float *H_val, int64_t *nnz, int nsm, cudaStream_t s) {
+    cudaError_t e = cudaMemsetAsync(st, 0, sizeof(TopkState), s);
+    if (e != cudaSuccess) return e;
+    int64_t hb = ceil_div(N, 256 * 8);
+    if (hb > nsm * 8) hb = nsm * 8;
+    if (hb < 1) hb = 1;
+    const unsigned masks[4] = {0x00000000u, 0xff000000u, 0xffff0000u, 0xffffff00u};
+    for (int pass = 0; pass < 4; ++pass) {
+        const int shift = 24 - 8 * pass;
+        k_topk_hist<<<static_cast<unsigned>(hb), 256, 0, s>>>(T, N, st, shift, masks[pass]);
+        k_topk_pick<<<1, 32, 0, s>>>(st, shift, s_budget, pass == 0);
+    }
+    const int64_t nch = topk_chunks(N);
+    k_topk_count<<<static_cast<unsigned>(nch), 256, 0, s>>>(T, N, st, cnt_gt, cnt_eq);
+    k_topk_scan<<<1, 1024, 0, s>>>(cnt_gt, cnt_eq, static_cast<int>(nch), st, sel_base, eq_base, nnz);
+    k_topk_emit<<<static_cast<unsigned>(nch), 256, 0, s>>>(T, N, st, sel_base, eq_base, H_idx, H_val);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_scatter_rowptr(const int64_t *H_idx, const float *H_val, const int64_t *nnz,
+                                  int64_t cap, int64_t q, int64_t p, float *H, int64_t ld,
+                                  int64_t *rowptr, cudaStream_t s) {
+    if (cap > 0)
+        k_scatter<<<static_cast<unsigned>(ceil_div(cap, 256)), 256, 0, s>>>(H_idx, H_val, nnz, cap, p, H,
+                                                                             ld);
+    k_rowptr<<<static_cast<unsigned>(ceil_div(q + 1, 256)), 256, 0, s>>>(H_idx, nnz, q, p, rowptr);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_spmm_refresh(const float *PW, float *P, float *R, int64_t ld, const float *S,
+                                int64_t lds, const float *d, const float *dinv, const int64_t *H_idx,
+                                const float *H_val, const int64_t *rowptr, int64_t q, int64_t p,
+                                int update_r, cudaStream_t s) {
+    k_spmm_refresh<<<static_cast<unsigned>(q), 256, 0, s>>>(PW, P, R, ld, S, lds, d, dinv, H_idx, H_val,
+                                                            rowptr, p, update_r);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_dinv(const float *d, int64_t p, float *dinv, cudaStream_t s) {
+    k_dinv<<<static_cast<unsigned>(ceil_div(p, 256)), 256, 0, s>>>(d, p, dinv);
+    return cudaGetLastError();
+}
+
+}  // namespace qe

@@ -1,0 +1,41 @@
+// Launchers of the outlier-aware kernels (Sec. 4.3, Algorithm 4).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace qe {
+
+// Device-side state of the radix select behind P_s.
+struct TopkState {
+    unsigned hist[256];
+    unsigned prefix;
+    unsigned remaining;
+    unsigned long long count_gt;
+    unsigned kstar;      // the s-th largest nonzero key (0xffffffff: nothing kept)
+    unsigned need_eq;    // keys == kstar to keep, in ascending linear index
+    unsigned empty;
+    unsigned pad;
+};
+
+cudaError_t launch_power_lambda(const float *S, int64_t lds, int64_t p, int iters, float *y0, float *y1,
+                                double *lam, double *eta, int nsm, cudaStream_t s);
+cudaError_t launch_iht_target(const float *H, const float *R, int64_t ld, const uint8_t *codes,
+                              int64_t ldc, const float *scale, const float *zero, const float *d,
+                              const double *eta, int64_t q, int64_t p, float *T, cudaStream_t s);
+cudaError_t launch_flat_copy(const void *W, int w_bf16, int64_t ldw, int64_t q, int64_t p, float *T,
+                             cudaStream_t s);
+int64_t topk_chunks(int64_t N);
+cudaError_t launch_topk(const float *T, int64_t N, int64_t s_budget, TopkState *st, unsigned *cnt_gt,
+                        unsigned *cnt_eq, unsigned *sel_base, unsigned *eq_base, int64_t *H_idx,
+                        float *H_val, int64_t *nnz, int nsm, cudaStream_t s);
+cudaError_t launch_scatter_rowptr(const int64_t *H_idx, const float *H_val, const int64_t *nnz,
+                                  int64_t cap, int64_t q, int64_t p, float *H, int64_t ld,
+                                  int64_t *rowptr, cudaStream_t s);
+cudaError_t launch_spmm_refresh(const float *PW, float *P, float *R, int64_t ld, const float *S,
+                                int64_t lds, const float *d, const float *dinv, const int64_t *H_idx,
+                                const float *H_val, const int64_t *rowptr, int64_t q, int64_t p,
+                                int update_r, cudaStream_t s);
+cudaError_t launch_dinv(const float *d, int64_t p, float *dinv, cudaStream_t s);
+
+}  // namespace qe

@@ -1,0 +1,205 @@
+"""Python binding of libqe.so (the C ABI declared in include/qe.h).
+
+Argument marshalling only: torch tensors are passed as raw device pointers and
+the current torch CUDA stream as the cudaStream_t; every step of the method runs
+in the library's CUDA kernels.  There is no fallback: if libqe.so is missing the
+calls raise.  The function names are those of the C ABI.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "_build", "libqe.so")
+
+QE_OK, QE_ERR_INVALID_ARG, QE_ERR_CUDA, QE_ERR_OOM, QE_ERR_NUMERIC, QE_ERR_TIMEOUT, \
+    QE_ERR_UNSUPPORTED = range(7)
+QE_F32, QE_BF16 = 0, 1
+QE_FEATURE_MAJOR, QE_TOKEN_MAJOR = 0, 1
+
+EXPORTED = ("qe_build_sigma", "qe_quantize_layer", "qe_quantize_layer_outlier",
+            "qe_workspace_size", "qe_sync_status", "qe_status_string", "qe_version")
+
+
+class QEError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        super().__init__(f"{what}: status {status} ({qe_status_string(status)})")
+        self.status = status
+
+
+class QEOpts(ctypes.Structure):
+    """Mirror of ``qe_opts``."""
+    _fields_ = [("block_width", ctypes.c_int), ("relax_period", ctypes.c_int),
+                ("structured_outliers", ctypes.c_int), ("power_iters", ctypes.c_int),
+                ("init_codes", ctypes.c_void_p), ("sweep_codes", ctypes.c_void_p),
+                ("wx_norm2", ctypes.c_void_p), ("workspace", ctypes.c_void_p),
+                ("workspace_bytes", ctypes.c_size_t)]
+
+
+_lib = None
+
+
+def load(path: str = LIB_PATH) -> ctypes.CDLL:
+    """Load libqe.so (once).  Raises if it has not been built."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise RuntimeError(f"libqe.so not found at {path}: build it with "
+                           "paper_2309_01885_gb300.build.build_lib()")
+    L = ctypes.CDLL(path)
+    vp, i64, i32, st = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_int
+    L.qe_build_sigma.argtypes = [vp, i32, i32, i64, i64, i64, vp, i32, vp]
+    L.qe_build_sigma.restype = st
+    L.qe_quantize_layer.argtypes = [vp, i32, i64, i64, i64, vp, i32, i32, ctypes.POINTER(QEOpts),
+                                    vp, vp, vp, vp, vp]
+    L.qe_quantize_layer.restype = st
+    L.qe_quantize_layer_outlier.argtypes = [vp, i32, i64, i64, i64, vp, i32, i32, i64,
+                                            ctypes.POINTER(QEOpts), vp, vp, vp, vp, vp, vp, vp, vp,
+                                            vp]
+    L.qe_quantize_layer_outlier.restype = st
+    L.qe_workspace_size.argtypes = [i64, i64, i32, ctypes.POINTER(QEOpts),
+                                    ctypes.POINTER(ctypes.c_size_t)]
+    L.qe_workspace_size.restype = st
+    L.qe_sync_status.argtypes = [vp]
+    L.qe_sync_status.restype = st
+    L.qe_status_string.argtypes = [st]
+    L.qe_status_string.restype = ctypes.c_char_p
+    L.qe_version.argtypes = []
+    L.qe_version.restype = ctypes.c_int
+    _lib = L
+    return L
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _dtype(t: torch.Tensor) -> int:
+    if t.dtype == torch.float32:
+        return QE_F32
+    if t.dtype == torch.bfloat16:
+        return QE_BF16
+    raise TypeError(f"unsupported dtype {t.dtype}: bf16 or fp32")
+
+
+def _check(status: int, what: str):
+    if status != QE_OK:
+        raise QEError(status, what)
+
+
+def _rowmajor_ld(t: torch.Tensor) -> int:
+    if t.dim() != 2 or t.stride(1) != 1:
+        raise ValueError("expected a 2-D tensor with unit column stride")
+    return t.stride(0)
+
+
+def qe_status_string(status: int) -> str:
+    return load().qe_status_string(status).decode()
+
+
+def qe_version() -> int:
+    return load().qe_version()
+
+
+def qe_sync_status(stream=None) -> int:
+    """Wait for the stream; return the device-latched status (0 = ok)."""
+    return load().qe_sync_status(_stream(stream))
+
+
+def qe_workspace_size(q: int, p: int, outlier: bool = False) -> int:
+    out = ctypes.c_size_t(0)
+    _check(load().qe_workspace_size(q, p, int(outlier), None, ctypes.byref(out)), "qe_workspace_size")
+    return out.value
+
+
+def qe_build_sigma(X: torch.Tensor, layout: int = QE_FEATURE_MAJOR, Sigma: torch.Tensor | None = None,
+                   accumulate: bool = False, stream=None) -> torch.Tensor:
+    """Sigma = X X^T (fp32, p x p) from X (bf16 / fp32, p x n feature-major or n x p token-major)."""
+    ld = _rowmajor_ld(X)
+    p, n = (X.shape[0], X.shape[1]) if layout == QE_FEATURE_MAJOR else (X.shape[1], X.shape[0])
+    if Sigma is None:
+        Sigma = torch.empty(p, p, dtype=torch.float32, device=X.device)
+    _check(load().qe_build_sigma(_ptr(X), _dtype(X), layout, p, n, ld, _ptr(Sigma), int(accumulate),
+                                 _stream(stream)), "qe_build_sigma")
+    return Sigma
+
+
+def _opts(block_width=0, power_iters=0, init_codes=None, sweep_codes=None, wx_norm2=None,
+          workspace=None) -> QEOpts:
+    o = QEOpts()
+    o.block_width = block_width
+    o.power_iters = power_iters
+    o.init_codes = None if init_codes is None else init_codes.data_ptr()
+    o.sweep_codes = None if sweep_codes is None else sweep_codes.data_ptr()
+    o.wx_norm2 = None if wx_norm2 is None else wx_norm2.data_ptr()
+    if workspace is not None:
+        o.workspace = workspace.data_ptr()
+        o.workspace_bytes = workspace.numel() * workspace.element_size()
+    return o
+
+
+def qe_quantize_layer(W: torch.Tensor, Sigma: torch.Tensor, bits: int, iters: int, *,
+                      init_codes: torch.Tensor | None = None, record_sweeps: bool = False,
+                      want_norm: bool = False, block_width: int = 0,
+                      workspace: torch.Tensor | None = None, stream=None) -> dict:
+    """QuantEase on one layer; returns codes (u8 q x p), scales, zeros, obj (fp64 per sweep),
+    and optionally sweep_codes (iters x q x p) and wx_norm2."""
+    q, p = W.shape
+    dev = W.device
+    codes = torch.empty(q, p, dtype=torch.uint8, device=dev)
+    scales = torch.empty(q, dtype=torch.float32, device=dev)
+    zeros = torch.empty(q, dtype=torch.float32, device=dev)
+    obj = torch.empty(iters, dtype=torch.float64, device=dev)
+    sweep = torch.empty(iters, q, p, dtype=torch.uint8, device=dev) if record_sweeps else None
+    norm = torch.empty(1, dtype=torch.float64, device=dev) if want_norm else None
+    o = _opts(block_width, 0, init_codes, sweep, norm, workspace)
+    _check(load().qe_quantize_layer(_ptr(W), _dtype(W), q, p, _rowmajor_ld(W), _ptr(Sigma), bits, iters,
+                                    ctypes.byref(o), _ptr(codes), _ptr(scales), _ptr(zeros), _ptr(obj),
+                                    _stream(stream)), "qe_quantize_layer")
+    out = dict(codes=codes, scales=scales, zeros=zeros, obj=obj)
+    if record_sweeps:
+        out["sweep_codes"] = sweep
+    if want_norm:
+        out["wx_norm2"] = norm
+    return out
+
+
+def qe_quantize_layer_outlier(W: torch.Tensor, Sigma: torch.Tensor, bits: int, iters: int,
+                              s_budget: int, *, power_iters: int = 0, init_codes=None,
+                              record_sweeps: bool = False, want_norm: bool = False,
+                              workspace: torch.Tensor | None = None, stream=None) -> dict:
+    """Outlier-aware QuantEase; adds H_val, H_idx (sorted linear indices), H_nnz, obj_cd."""
+    q, p = W.shape
+    dev = W.device
+    codes = torch.empty(q, p, dtype=torch.uint8, device=dev)
+    scales = torch.empty(q, dtype=torch.float32, device=dev)
+    zeros = torch.empty(q, dtype=torch.float32, device=dev)
+    obj = torch.empty(iters, dtype=torch.float64, device=dev)
+    obj_cd = torch.empty(iters, dtype=torch.float64, device=dev)
+    cap = max(int(s_budget), 1)
+    H_val = torch.empty(cap, dtype=torch.float32, device=dev)
+    H_idx = torch.empty(cap, dtype=torch.int64, device=dev)
+    H_nnz = torch.zeros(1, dtype=torch.int64, device=dev)
+    sweep = torch.empty(iters, q, p, dtype=torch.uint8, device=dev) if record_sweeps else None
+    norm = torch.empty(1, dtype=torch.float64, device=dev) if want_norm else None
+    o = _opts(0, power_iters, init_codes, sweep, norm, workspace)
+    _check(load().qe_quantize_layer_outlier(
+        _ptr(W), _dtype(W), q, p, _rowmajor_ld(W), _ptr(Sigma), bits, iters, int(s_budget),
+        ctypes.byref(o), _ptr(codes), _ptr(scales), _ptr(zeros), _ptr(H_val), _ptr(H_idx),
+        _ptr(H_nnz), _ptr(obj), _ptr(obj_cd), _stream(stream)), "qe_quantize_layer_outlier")
+    out = dict(codes=codes, scales=scales, zeros=zeros, obj=obj, obj_cd=obj_cd, H_val=H_val,
+               H_idx=H_idx, H_nnz=H_nnz)
+    if record_sweeps:
+        out["sweep_codes"] = sweep
+    if want_norm:
+        out["wx_norm2"] = norm
+    return out

@@ -1,0 +1,98 @@
+"""The C ABI: libqe.so builds, loads without a GPU, exports every function that
+include/qe.h declares, and rejects bad arguments before touching the device."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2309_01885_gb300 import build, qe
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build_lib()
+    return qe.load()
+
+
+def declared_functions():
+    text = open(os.path.join(ROOT, "include", "qe.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(qe_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = declared_functions()
+    assert set(qe.EXPORTED) == set(names)
+    for name in names:
+        assert hasattr(lib, name), name
+
+
+def test_status_strings_and_version(lib):
+    assert qe.qe_version() >= 10000
+    for s in range(7):
+        assert qe.qe_status_string(s)
+    assert qe.qe_status_string(99) == "unknown status"
+
+
+def test_opts_struct_matches_header():
+    # 4 ints, 4 pointers, 1 size_t on LP64
+    assert ctypes.sizeof(qe.QEOpts) == 4 * 4 + 4 * 8 + 8
+
+
+def _fake(n=1):
+    return ctypes.c_void_p(0x1000 * n)   # never dereferenced: rejected before any launch
+
+
+def test_invalid_arguments_rejected_synchronously(lib):
+    L = lib
+    opts = None
+    # p = 0
+    assert L.qe_quantize_layer(_fake(), qe.QE_F32, 4, 0, 4, _fake(2), 4, 1, opts, _fake(3), _fake(4),
+                               _fake(5), _fake(6), None) == qe.QE_ERR_INVALID_ARG
+    # bits out of range
+    assert L.qe_quantize_layer(_fake(), qe.QE_F32, 4, 4, 4, _fake(2), 9, 1, opts, _fake(3), _fake(4),
+                               _fake(5), _fake(6), None) == qe.QE_ERR_INVALID_ARG
+    # short leading dimension
+    assert L.qe_quantize_layer(_fake(), qe.QE_F32, 4, 8, 4, _fake(2), 3, 1, opts, _fake(3), _fake(4),
+                               _fake(5), _fake(6), None) == qe.QE_ERR_INVALID_ARG
+    # null output
+    assert L.qe_quantize_layer(_fake(), qe.QE_F32, 4, 4, 4, _fake(2), 3, 1, opts, None, _fake(4),
+                               _fake(5), _fake(6), None) == qe.QE_ERR_INVALID_ARG
+    # iters = 0
+    assert L.qe_quantize_layer(_fake(), qe.QE_BF16, 4, 4, 4, _fake(2), 3, 0, opts, _fake(3), _fake(4),
+                               _fake(5), _fake(6), None) == qe.QE_ERR_INVALID_ARG
+    # unsupported options
+    o = qe.QEOpts()
+    o.relax_period = 3
+    assert L.qe_quantize_layer(_fake(), qe.QE_F32, 4, 4, 4, _fake(2), 3, 1, ctypes.byref(o), _fake(3),
+                               _fake(4), _fake(5), _fake(6), None) == qe.QE_ERR_UNSUPPORTED
+    o = qe.QEOpts()
+    o.block_width = 48
+    assert L.qe_quantize_layer(_fake(), qe.QE_F32, 4, 4, 4, _fake(2), 3, 1, ctypes.byref(o), _fake(3),
+                               _fake(4), _fake(5), _fake(6), None) == qe.QE_ERR_UNSUPPORTED
+    # outlier budget larger than the layer / missing outputs
+    assert L.qe_quantize_layer_outlier(_fake(), qe.QE_F32, 4, 4, 4, _fake(2), 3, 1, 17, None, _fake(3),
+                                       _fake(4), _fake(5), _fake(7), _fake(8), _fake(9), _fake(6),
+                                       None, None) == qe.QE_ERR_INVALID_ARG
+    assert L.qe_quantize_layer_outlier(_fake(), qe.QE_F32, 4, 4, 4, _fake(2), 3, 1, 2, None, _fake(3),
+                                       _fake(4), _fake(5), None, None, _fake(9), _fake(6),
+                                       None, None) == qe.QE_ERR_INVALID_ARG
+    # Sigma: bad sizes / layouts
+    assert L.qe_build_sigma(_fake(), qe.QE_BF16, qe.QE_FEATURE_MAJOR, 0, 10, 10, _fake(2), 0,
+                            None) == qe.QE_ERR_INVALID_ARG
+    assert L.qe_build_sigma(_fake(), qe.QE_BF16, qe.QE_FEATURE_MAJOR, 8, 10, 9, _fake(2), 0,
+                            None) == qe.QE_ERR_INVALID_ARG
+    assert L.qe_build_sigma(_fake(), qe.QE_BF16, qe.QE_TOKEN_MAJOR, 8, 10, 7, _fake(2), 0,
+                            None) == qe.QE_ERR_INVALID_ARG
+    assert L.qe_build_sigma(_fake(), 7, qe.QE_TOKEN_MAJOR, 8, 10, 8, _fake(2), 0,
+                            None) == qe.QE_ERR_INVALID_ARG
+
+
+def test_workspace_size_grows_with_shape(lib):
+    a = qe.qe_workspace_size(256, 256)
+    b = qe.qe_workspace_size(512, 1024)
+    c = qe.qe_workspace_size(512, 1024, outlier=True)
+    assert 0 < a < b < c

@@ -1,0 +1,245 @@
+"""GPU parity: the CUDA path (through the C ABI) against the fp64 oracle.
+
+Sizes here run in seconds on the oracle and span several GEMM tiles, several
+64-column CD blocks and ragged tails.  Full-size workloads are in
+test_gpu_fullsize.py.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2309_01885_gb300 import inputs
+from paper_2309_01885_gb300 import qe
+from tests import parity
+
+pytestmark = pytest.mark.gpu
+O = oracle.get()
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    qe.load()
+
+
+def _sigma_check(Sg, X64):
+    S64 = O.sigma(X64)
+    Sg64 = parity.f64(Sg)
+    assert np.array_equal(Sg64, Sg64.T), "Sigma is not exactly symmetric"
+    dg = np.sqrt(np.outer(np.diag(S64), np.diag(S64)))
+    err = np.abs(Sg64 - S64)
+    tol = 1e-5 * np.maximum(dg, 1e-30)
+    assert np.all(err <= tol), f"Sigma: max err/tol = {np.max(err / tol):.3f}"
+    return S64
+
+
+# ---------------------------------------------------------------------------
+# Sigma = X X^T
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("p,n", [(200, 1000), (384, 4096), (130, 70), (640, 3000)])
+def test_sigma_bf16_feature_major(p, n):
+    X = inputs.calib_inputs(p, n, dtype=torch.bfloat16, seed=1, device="cuda", heavy_frac=0.02,
+                            heavy_mult=30.0)
+    Sg = qe.qe_build_sigma(X)
+    torch.cuda.synchronize()
+    _sigma_check(Sg, parity.f64(X))
+
+
+def test_sigma_bf16_token_major_and_accumulate():
+    p, n = 272, 5000
+    X = inputs.calib_inputs(p, n, dtype=torch.bfloat16, seed=2, device="cuda", heavy_frac=0.02,
+                            heavy_mult=20.0)
+    Xt = X.t().contiguous()                      # n x p, token-major
+    Sg = qe.qe_build_sigma(Xt, layout=qe.QE_TOKEN_MAJOR)
+    torch.cuda.synchronize()
+    _sigma_check(Sg, parity.f64(X))
+    # Sigma over the token stream in two chunks equals Sigma of the whole
+    S2 = qe.qe_build_sigma(X[:, :3000].contiguous())
+    qe.qe_build_sigma(X[:, 3000:].contiguous(), Sigma=S2, accumulate=True)
+    torch.cuda.synchronize()
+    _sigma_check(S2, parity.f64(X))
+
+
+@pytest.mark.parametrize("layout", [qe.QE_FEATURE_MAJOR, qe.QE_TOKEN_MAJOR])
+def test_sigma_fp32(layout):
+    p, n = 150, 777
+    X = inputs.calib_inputs(p, n, dtype=torch.float32, seed=3, device="cuda", heavy_frac=0.02,
+                            heavy_mult=20.0)
+    src = X if layout == qe.QE_FEATURE_MAJOR else X.t().contiguous()
+    Sg = qe.qe_build_sigma(src, layout=layout)
+    torch.cuda.synchronize()
+    _sigma_check(Sg, parity.f64(X))
+
+
+# ---------------------------------------------------------------------------
+# qe_quantize_layer
+# ---------------------------------------------------------------------------
+def _layer_case(q, p, n, w_dtype, bits, iters, seed, corr_rank=0, zero_rows=(), w_outlier=0.0):
+    W = inputs.layer_weights(q, p, dtype=w_dtype, seed=seed, device="cuda",
+                             w_outlier_frac=w_outlier, w_outlier_mult=10.0)
+    X = inputs.calib_inputs(p, n, dtype=torch.bfloat16, seed=seed, device="cuda",
+                            heavy_frac=0.01, heavy_mult=30.0, corr_rank=corr_rank,
+                            zero_rows=zero_rows)
+    Sg = qe.qe_build_sigma(X)
+    out = qe.qe_quantize_layer(W, Sg, bits, iters, record_sweeps=True, want_norm=True)
+    assert qe.qe_sync_status() == qe.QE_OK
+    return W, X, Sg, out
+
+
+def _check_layer(W, Sg, out, bits, iters, init_codes=None):
+    W64 = parity.f64(W)
+    S64 = parity.f64(Sg)                      # the same Sigma on both sides
+    s, z = parity.check_grid(out["scales"], out["zeros"], W64, bits)
+    sweep = out["sweep_codes"].cpu().numpy()
+    # teacher-forced: every decision is the nearest level of the fp64 beta~
+    nbad, ntot = parity.teacher_forced(W64, S64, s, z, bits, sweep, init_codes=init_codes)
+    # objective of the GPU's own state, fp64
+    forced = O.alg1(W64, S64, s, z, bits, iters, init_codes=init_codes, forced=sweep)
+    parity.check_obj(out["obj"].cpu().numpy(), forced["obj"], what="objective (GPU state)")
+    # free-running oracle
+    ref = O.alg1(W64, S64, s, z, bits, iters, init_codes=init_codes)
+    parity.check_obj(out["obj"].cpu().numpy(), ref["obj"], what="objective (free-running)")
+    m = parity.code_match(out["codes"].cpu().numpy(), ref["codes"])
+    assert m >= parity.CODE_MATCH, f"codes match {m:.5f}"
+    # ||W X||^2 = sum_i W_i Sigma W_i^T
+    wx = float(np.einsum("ij,jk,ik->", W64, S64, W64))
+    assert abs(out["wx_norm2"].item() - wx) <= 1e-4 * wx
+    return nbad, ntot
+
+
+@pytest.mark.parametrize("w_dtype", [torch.bfloat16, torch.float32])
+@pytest.mark.parametrize("bits", [3, 4])
+def test_layer_parity_small(w_dtype, bits):
+    W, X, Sg, out = _layer_case(200, 300, 2048, w_dtype, bits, 4, seed=bits, corr_rank=4)
+    _check_layer(W, Sg, out, bits, 4)
+    # objective non-increasing after the first sweep (Lemma 2)
+    obj = out["obj"].cpu().numpy()
+    assert np.all(np.diff(obj) <= 1e-6 * obj[:-1])
+
+
+def test_layer_parity_multi_tile_ragged():
+    W, X, Sg, out = _layer_case(300, 520, 4096, torch.bfloat16, 3, 3, seed=11, corr_rank=8)
+    _check_layer(W, Sg, out, 3, 3)
+
+
+def test_layer_dead_columns_round_to_nearest():
+    dead = (5, 77, 130)
+    W, X, Sg, out = _layer_case(96, 160, 1024, torch.float32, 4, 3, seed=12, zero_rows=dead)
+    _check_layer(W, Sg, out, 4, 3)
+    W64 = parity.f64(W)
+    rtn = O.rtn(W64, out["scales"].cpu().numpy(), out["zeros"].cpu().numpy(), 4)
+    codes = out["codes"].cpu().numpy()
+    for j in dead:
+        assert np.array_equal(codes[:, j], rtn[:, j])
+
+
+@pytest.mark.parametrize("bits", [2, 8])
+def test_layer_extreme_bits(bits):
+    W, X, Sg, out = _layer_case(64, 128, 1024, torch.float32, bits, 3, seed=13)
+    _check_layer(W, Sg, out, bits, 3)
+
+
+def test_layer_tiny_and_single_column():
+    for q, p in [(1, 1), (3, 5), (1, 70), (129, 1)]:
+        W, X, Sg, out = _layer_case(q, p, 256, torch.float32, 3, 2, seed=q * 100 + p)
+        _check_layer(W, Sg, out, 3, 2)
+
+
+def test_layer_warm_start():
+    q, p, n, bits, iters = 128, 192, 2048, 3, 3
+    W = inputs.layer_weights(q, p, dtype=torch.bfloat16, seed=21, device="cuda")
+    X = inputs.calib_inputs(p, n, dtype=torch.bfloat16, seed=21, device="cuda", heavy_frac=0.02,
+                            heavy_mult=30.0, corr_rank=4)
+    Sg = qe.qe_build_sigma(X)
+    W64 = parity.f64(W)
+    s, z = O.grid(W64, bits)
+    init = O.rtn(W64, s, z, bits)
+    out = qe.qe_quantize_layer(W, Sg, bits, iters, init_codes=torch.from_numpy(init).cuda(),
+                               record_sweeps=True, want_norm=True)
+    assert qe.qe_sync_status() == qe.QE_OK
+    _check_layer(W, Sg, out, bits, iters, init_codes=init)
+
+
+def test_config1_opt125m_full():
+    cfg = inputs.CONFIGS["opt125m_768x768"]
+    W = cfg.weights("cuda")
+    X = cfg.inputs("cuda")
+    Sg = qe.qe_build_sigma(X)
+    out = qe.qe_quantize_layer(W, Sg, cfg.bits[0], cfg.iters, record_sweeps=True, want_norm=True)
+    assert qe.qe_sync_status() == qe.QE_OK
+    _sigma_check(Sg, parity.f64(X))
+    _check_layer(W, Sg, out, cfg.bits[0], cfg.iters)
+
+
+def test_deterministic_repeat():
+    W, X, Sg, out = _layer_case(150, 200, 1024, torch.bfloat16, 3, 3, seed=31, corr_rank=4)
+    out2 = qe.qe_quantize_layer(W, Sg, 3, 3)
+    torch.cuda.synchronize()
+    assert torch.equal(out["codes"], out2["codes"])
+    assert torch.equal(out["obj"], out2["obj"])
+    S2 = qe.qe_build_sigma(X)
+    torch.cuda.synchronize()
+    assert torch.equal(S2, Sg)
+
+
+def test_nonfinite_input_is_reported():
+    W = inputs.layer_weights(16, 32, dtype=torch.float32, seed=1, device="cuda")
+    W[3, 7] = float("nan")
+    X = inputs.calib_inputs(32, 128, dtype=torch.float32, seed=1, device="cuda")
+    Sg = qe.qe_build_sigma(X)
+    qe.qe_quantize_layer(W, Sg, 4, 1)
+    assert qe.qe_sync_status() == qe.QE_ERR_NUMERIC
+    assert qe.qe_sync_status() == qe.QE_OK          # the latch is cleared
+
+
+# ---------------------------------------------------------------------------
+# qe_quantize_layer_outlier
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("q,p,bits,frac", [(96, 192, 3, 0.01), (130, 260, 2, 0.02)])
+def test_outlier_parity_small(q, p, bits, frac):
+    iters, power_iters = 4, 200
+    W = inputs.layer_weights(q, p, dtype=torch.bfloat16, seed=41, device="cuda", planted_frac=frac,
+                             planted_std=0.3)
+    X = inputs.calib_inputs(p, 2048, dtype=torch.bfloat16, seed=41, device="cuda", heavy_frac=0.02,
+                            heavy_mult=30.0, corr_rank=4)
+    Sg = qe.qe_build_sigma(X)
+    s_budget = int(round(frac * q * p))
+    out = qe.qe_quantize_layer_outlier(W, Sg, bits, iters, s_budget, power_iters=power_iters,
+                                       record_sweeps=True)
+    assert qe.qe_sync_status() == qe.QE_OK
+    W64, S64 = parity.f64(W), parity.f64(Sg)
+    ref = O.outlier(W64, S64, bits, iters, s_budget, power_iters)
+    assert np.array_equal(out["scales"].cpu().numpy(), ref["scale"])
+    assert np.array_equal(out["zeros"].cpu().numpy(), ref["zero"])
+    parity.check_obj(out["obj_cd"].cpu().numpy(), ref["obj_cd"], what="g after CD")
+    parity.check_obj(out["obj"].cpu().numpy(), ref["obj"], what="g after IHT")
+    m = parity.code_match(out["codes"].cpu().numpy(), ref["codes"])
+    assert m >= parity.CODE_MATCH, f"codes match {m:.5f}"
+    nnz = int(out["H_nnz"].item())
+    assert nnz == ref["nnz"]
+    idx = out["H_idx"][:nnz].cpu().numpy()
+    assert np.all(np.diff(idx) > 0)
+    ref_idx = np.nonzero(ref["H"].ravel())[0]
+    same = np.intersect1d(idx, ref_idx).size
+    assert same >= 0.999 * nnz
+    Hd = np.zeros(q * p)
+    Hd[idx] = out["H_val"][:nnz].cpu().numpy()
+    common = np.intersect1d(idx, ref_idx)
+    assert np.allclose(Hd[common], ref["H"].ravel()[common], rtol=1e-3, atol=1e-6)
+    # Lemma 3: the IHT half never increases g
+    assert np.all(out["obj"].cpu().numpy() <= out["obj_cd"].cpu().numpy() * (1 + 1e-6))
+
+
+def test_outlier_zero_budget_matches_plain_layer():
+    q, p, bits, iters = 64, 128, 3, 3
+    W = inputs.layer_weights(q, p, dtype=torch.bfloat16, seed=51, device="cuda")
+    X = inputs.calib_inputs(p, 1024, dtype=torch.bfloat16, seed=51, device="cuda", corr_rank=4)
+    Sg = qe.qe_build_sigma(X)
+    a = qe.qe_quantize_layer(W, Sg, bits, iters)
+    b = qe.qe_quantize_layer_outlier(W, Sg, bits, iters, 0)
+    torch.cuda.synchronize()
+    assert torch.equal(a["codes"], b["codes"])
+    assert int(b["H_nnz"].item()) == 0
+    assert np.allclose(a["obj"].cpu().numpy(), b["obj"].cpu().numpy(), rtol=1e-6)
