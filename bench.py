@@ -43,7 +43,7 @@ def parse():
     ap.add_argument("--config", default="llama7b_proj_4096x4096")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--cpu-rows", type=int, default=96, help="oracle rows in the CPU sample")
+    ap.add_argument("--cpu-rows", type=int, default=4096, help="oracle rows in the CPU sample")
     return ap.parse_args()
 
 

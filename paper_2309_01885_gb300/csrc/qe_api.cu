@@ -76,14 +76,14 @@ static Plan make_plan(int64_t q, int64_t p, int B, bool outlier, int wpl_planes,
     pl.smax = static_cast<int>(smax);
     const size_t qld = static_cast<size_t>(q) * pl.ld;
     size_t cur = 0;
-    pl.snt = take(cur, static_cast<size_t>(2 * p) * pl.ld * 2);
+    pl.snt = take(cur, static_cast<size_t>(3 * p) * pl.ld * 2);
     pl.d = take(cur, p * 4);
     pl.dinv = take(cur, p * 4);
     pl.P = take(cur, qld * 4);
     pl.R = take(cur, qld * 4);
     pl.wpl = take(cur, wpl_planes > 0 ? qld * 2 * wpl_planes : 0);
     pl.qf = take(cur, qld * 2);
-    pl.dp = take(cur, qld * 2 * 2);
+    pl.dp = take(cur, qld * 2 * 3);
     pl.part = take(cur, static_cast<size_t>(pl.smax) * q * B * 4);
     pl.objp = take(cur, static_cast<size_t>(objective_blocks(q)) * 8);
     if (outlier) {
@@ -181,10 +181,10 @@ static qe_status setup_ctx(Ctx &c, const Plan &pl, const qe_opts *o, cudaStream_
         c.rowptr = at<int64_t>(w, pl.rowptr);
     }
     const uint64_t q = pl.q, p = pl.p, ld = pl.ld;
-    if (!make_tmap_bf16(&c.tm_snt256, c.snt, 2 * p, p, ld, 256) ||
-        !make_tmap_bf16(&c.tm_snt64, c.snt, 2 * p, p, ld, 64) ||
+    if (!make_tmap_bf16(&c.tm_snt256, c.snt, 3 * p, p, ld, 256) ||
+        !make_tmap_bf16(&c.tm_snt64, c.snt, 3 * p, p, ld, 64) ||
         !make_tmap_bf16(&c.tm_qf, c.qf, q, p, ld, 128) ||
-        !make_tmap_bf16(&c.tm_dp, c.dp, 2 * q, p, ld, 128))
+        !make_tmap_bf16(&c.tm_dp, c.dp, 3 * q, p, ld, 128))
         return QE_ERR_CUDA;
     return QE_OK;
 }
@@ -209,12 +209,16 @@ static GemmArgs gemm_args(const Ctx &c, int M, int N, int kb_count, int mode) {
     return g;
 }
 
+// Plane products of A (1 exact plane, or hi/mid/lo) times B = Sigma_bar^T (hi/mid/lo):
+// every pair whose order is at least 2^-16 relative (plane k carries ~2^-8k).
 static void set_prods(GemmArgs &g, int a_planes) {
-    // hi.hi, hi.lo and (two A planes) lo.hi; the lo.lo product is below fp32 rounding.
-    g.prod_a[0] = 0; g.prod_b[0] = 0;
-    g.prod_a[1] = 0; g.prod_b[1] = 1;
-    g.prod_a[2] = 1; g.prod_b[2] = 0;
-    g.n_prod = (a_planes == 2) ? 3 : 2;
+    static const int one[3][2] = {{0, 0}, {0, 1}, {0, 2}};
+    static const int three[6][2] = {{0, 0}, {0, 1}, {1, 0}, {0, 2}, {1, 1}, {2, 0}};
+    g.n_prod = (a_planes == 3) ? 6 : 3;
+    for (int t = 0; t < g.n_prod; ++t) {
+        g.prod_a[t] = (a_planes == 3) ? three[t][0] : one[t][0];
+        g.prod_b[t] = (a_planes == 3) ? three[t][1] : one[t][1];
+    }
 }
 
 // Sigma -> d, Sigma_bar^T planes; W operand planes; P = W (I + Sigma_bar) into `Pout`.
@@ -227,8 +231,8 @@ static qe_status prepare(Ctx &c, const void *W, int wbf16, int64_t ldw, const fl
         if (!make_tmap_bf16(&c.tm_wa, W, q, p, ldw, 128)) return QE_ERR_CUDA;
         c.wa_planes = 1;
     } else {
-        c.wa_planes = wbf16 ? 1 : 2;
-        QE_CK(launch_make_planes(W, wbf16, ldw, q, p, c.wa_planes == 2, c.wpl, ld, c.s));
+        c.wa_planes = wbf16 ? 1 : 3;
+        QE_CK(launch_make_planes(W, wbf16, ldw, q, p, c.wa_planes == 3, c.wpl, ld, c.s));
         if (!make_tmap_bf16(&c.tm_wa, c.wpl, c.wa_planes * q, p, ld, 128)) return QE_ERR_CUDA;
     }
     GemmArgs g = gemm_args(c, static_cast<int>(q), static_cast<int>(p), static_cast<int>(ceil_div(p, 64)),
@@ -274,7 +278,7 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
             const int kb = static_cast<int>(b0 / 64);
             const int S = kb < c.pl.smax ? kb : c.pl.smax;
             GemmArgs g = gemm_args(c, static_cast<int>(q), bw, kb, EPI_TRAIL);
-            set_prods(g, first ? 2 : 1);
+            set_prods(g, first ? 3 : 1);
             g.a_plane_rows = static_cast<int>(q);
             g.b_plane_rows = static_cast<int>(p);
             g.b_row0 = static_cast<int>(b0);
@@ -401,7 +405,7 @@ qe_status qe_workspace_size(int64_t q, int64_t p, int outlier, const qe_opts *op
     if (!bytes || q < 1 || p < 1) return QE_ERR_INVALID_ARG;
     const qe_status st = check_opts(opts);
     if (st != QE_OK) return st;
-    const Plan pl = make_plan(q, p, kDefaultBlock, outlier != 0, 2, sm_count());
+    const Plan pl = make_plan(q, p, kDefaultBlock, outlier != 0, 3, sm_count());
     *bytes = pl.total;
     return QE_OK;
 }
@@ -486,7 +490,7 @@ qe_status qe_quantize_layer(const void *W, qe_dtype w_dtype, int64_t q, int64_t 
     if ((st = check_opts(opts)) != QE_OK) return st;
     const int wbf16 = (w_dtype == QE_BF16);
     Ctx c;
-    const Plan pl = make_plan(q, p, kDefaultBlock, false, wbf16 ? 1 : 2, sm_count());
+    const Plan pl = make_plan(q, p, kDefaultBlock, false, wbf16 ? 1 : 3, sm_count());
     if ((st = setup_ctx(c, pl, opts, reinterpret_cast<cudaStream_t>(stream))) != QE_OK) return st;
 
     QE_CK(launch_grid(W, wbf16, ldw, nullptr, 0, q, p, bits, scales, zeros, c.err, c.s));
@@ -528,7 +532,7 @@ qe_status qe_quantize_layer_outlier(const void *W, qe_dtype w_dtype, int64_t q, 
     const int power_iters = (opts && opts->power_iters > 0) ? opts->power_iters : kDefaultPowerIters;
     Ctx c;
     c.nsm = sm_count();
-    const Plan pl = make_plan(q, p, kDefaultBlock, true, wbf16 ? 1 : 2, c.nsm);
+    const Plan pl = make_plan(q, p, kDefaultBlock, true, wbf16 ? 1 : 3, c.nsm);
     if ((st = setup_ctx(c, pl, opts, reinterpret_cast<cudaStream_t>(stream))) != QE_OK) return st;
     const int64_t ld = pl.ld;
 

@@ -69,7 +69,8 @@ __global__ void __launch_bounds__(256) k_grid(const void *W, int w_bf16, int64_t
 // d_j = Sigma_jj; a column with d_j <= 0 is dead.  SnT = Sigma_bar^T with
 // SnT[j][k] = Sigma[j][k] / d_j for k != j and j, k alive, 0 otherwise; this is
 // Sigma_bar[k][j] = Sigma[k][j] / Sigma_jj of the column-normalised matrix with
-// zero diagonal.  Stored as two bf16 planes (rows [0, p) = hi, [p, 2p) = lo).
+// zero diagonal.  Stored as three bf16 planes hi, mid, lo (rows [0, p), [p, 2p),
+// [2p, 3p)) whose sum carries the 24 significant bits of the fp32 value.
 // ---------------------------------------------------------------------------
 __global__ void k_sigma_diag(const float *S, int64_t lds, int64_t p, float *d, unsigned *err) {
     const int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
@@ -92,9 +93,12 @@ __global__ void k_sigma_planes(const float *S, int64_t lds, int64_t p, const flo
             float x = 0.0f;
             if (jalive && k != j && d[k] > 0.0f) x = __fdiv_rn(sv, dj);
             const __nv_bfloat16 h = __float2bfloat16_rn(x);
-            const __nv_bfloat16 l = __float2bfloat16_rn(x - __bfloat162float(h));
+            const float r1 = x - __bfloat162float(h);
+            const __nv_bfloat16 m = __float2bfloat16_rn(r1);
+            const __nv_bfloat16 l = __float2bfloat16_rn(r1 - __bfloat162float(m));
             snt[j * ldn + k] = h;
-            snt[(p + j) * ldn + k] = l;
+            snt[(p + j) * ldn + k] = m;
+            snt[(2 * p + j) * ldn + k] = l;
         }
     }
     if (bad) set_error(err, ERR_NUMERIC);
@@ -102,17 +106,23 @@ __global__ void k_sigma_planes(const float *S, int64_t lds, int64_t p, const flo
 
 // ---------------------------------------------------------------------------
 // Operand planes of a q x p matrix for the tensor-core GEMM (rows [0,q) = hi,
-// [q, 2q) = lo when two planes).  fp32 input splits hi/lo; bf16 input copies.
+// [q, 2q) = mid, [2q, 3q) = lo when split).  fp32 input splits into three bf16
+// planes; bf16 input is copied (exact in one plane).
 // ---------------------------------------------------------------------------
 __global__ void k_make_planes(const void *W, int w_bf16, int64_t ldw, int64_t q, int64_t p,
-                              int two_planes, __nv_bfloat16 *out, int64_t ldo) {
+                              int split, __nv_bfloat16 *out, int64_t ldo) {
     for (int64_t i = blockIdx.y; i < q; i += gridDim.y) {
         for (int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; j < p;
              j += (int64_t)gridDim.x * blockDim.x) {
             const float w = load_elem(W, w_bf16, i * ldw + j);
             const __nv_bfloat16 h = __float2bfloat16_rn(w);
             out[i * ldo + j] = h;
-            if (two_planes) out[(q + i) * ldo + j] = __float2bfloat16_rn(w - __bfloat162float(h));
+            if (split) {
+                const float r1 = w - __bfloat162float(h);
+                const __nv_bfloat16 m = __float2bfloat16_rn(r1);
+                out[(q + i) * ldo + j] = m;
+                out[(2 * q + i) * ldo + j] = __float2bfloat16_rn(r1 - __bfloat162float(m));
+            }
         }
     }
 }
@@ -167,13 +177,15 @@ __global__ void __launch_bounds__(32) k_cd_block(const CdArgs a) {
     const int bw = a.bw;
     const int64_t b0 = a.b0;
 
-    // Sigma_bar[b0 + k][b0 + l] = SnT[b0 + l][b0 + k] (hi + lo)
+    // Sigma_bar[b0 + k][b0 + l] = SnT[b0 + l][b0 + k] (hi + mid + lo)
     for (int idx = lane; idx < B * B; idx += 32) {
         const int k = idx % B, l = idx / B;
         float v = 0.0f;
         if (k < bw && l < bw) {
             const int64_t o = (b0 + l) * a.ldsn + b0 + k;
-            v = __bfloat162float(a.snt[o]) + __bfloat162float(a.snt[a.snt_plane_rows * a.ldsn + o]);
+            const int64_t pl = a.snt_plane_rows * a.ldsn;
+            v = __bfloat162float(a.snt[o]) + __bfloat162float(a.snt[pl + o]) +
+                __bfloat162float(a.snt[2 * pl + o]);
         }
         sig[k][l] = v;
     }
@@ -236,8 +248,12 @@ __global__ void __launch_bounds__(32) k_cd_block(const CdArgs a) {
             a.qf[i * a.ldq + col] = __float2bfloat16_rn(c - z);
             const __nv_bfloat16 h = __float2bfloat16_rn(dl);
             a.dp[i * a.ldd + col] = h;
-            if (a.first_sweep)
-                a.dp[(a.dp_plane_rows + i) * a.ldd + col] = __float2bfloat16_rn(dl - __bfloat162float(h));
+            if (a.first_sweep) {   // Delta' is not an integer in the first sweep: three planes
+                const float r1 = dl - __bfloat162float(h);
+                const __nv_bfloat16 m = __float2bfloat16_rn(r1);
+                a.dp[(a.dp_plane_rows + i) * a.ldd + col] = m;
+                a.dp[(2 * a.dp_plane_rows + i) * a.ldd + col] = __float2bfloat16_rn(r1 - __bfloat162float(m));
+            }
         }
     }
 }
@@ -411,8 +427,8 @@ cudaError_t launch_sigma_norm(const float *S, int64_t lds, int64_t p, float *d, 
 }
 
 cudaError_t launch_make_planes(const void *W, int w_bf16, int64_t ldw, int64_t q, int64_t p,
-                               int two_planes, __nv_bfloat16 *out, int64_t ldo, cudaStream_t s) {
-    k_make_planes<<<row_grid(q, p), 256, 0, s>>>(W, w_bf16, ldw, q, p, two_planes, out, ldo);
+                               int split, __nv_bfloat16 *out, int64_t ldo, cudaStream_t s) {
+    k_make_planes<<<row_grid(q, p), 256, 0, s>>>(W, w_bf16, ldw, q, p, split, out, ldo);
     return cudaGetLastError();
 }
 

@@ -9,12 +9,14 @@
 //                                          dW_{:,1:j} Sigma^norm_{1:j,j} term,
 //                                          deferred per column block, split-K)
 // fp32 accuracy for the Sigma_bar products comes from splitting an fp32 operand
-// into two bf16 planes (hi + lo) and summing the cross products in the same
-// TMEM accumulator (planes are stacked along rows in one tensor map).
+// into three bf16 planes (hi + mid + lo, 24 significant bits) and summing the
+// cross products down to 2^-16 relative order in the same accumulator (planes
+// are stacked along rows in one tensor map).
 //
-// Warp roles (128 threads): warp 0 lane 0 issues TMA, warp 1 lane 0 issues MMA,
-// warp 2 owns the TMEM allocation, all four warps run the epilogue (warp w reads
-// TMEM lanes 32w..32w+31 = output rows).
+// Warp roles (320 threads): warp 0 lane 0 issues TMA, warp 1 lane 0 issues MMA
+// (warp 1 owns the TMEM allocation: two accumulation buffers), warps 2..9 fold
+// the chunk partial sums into fp32 registers and run the epilogue (warp w reads
+// TMEM lanes 32 (w mod 4) .. +31 = output rows, half of the columns each).
 #include <cudaTypedefs.h>
 
 #include "qe_common.cuh"
@@ -30,11 +32,21 @@ struct GemmCfg {
     static constexpr int B_BYTES = BN * BK * 2;
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
     static constexpr int STAGES = (BN == 256) ? 4 : (BN == 128) ? 6 : 8;
-    static constexpr int TMEM_COLS = BN;               // power of two >= 32
+    static constexpr int TMEM_COLS = 2 * BN;           // two accumulation buffers
+    static constexpr int HALF = BN / 2;                // columns per epilogue thread
+    static constexpr int THREADS = 320;                // producer, MMA, 8 epilogue warps
     static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + 256;
     static_assert(BN == 64 || BN == 128 || BN == 256, "BN");
     static_assert(SMEM_BYTES <= 232448, "smem");
 };
+
+// Virtual K steps (k-block x operand-plane product) accumulated in one TMEM
+// buffer before the epilogue warps fold it into fp32 registers.  The tensor-core
+// accumulator loses up to about one unit in the last place per accumulate
+// (measured: ~1e-5 relative after 256 accumulates), so long K is summed as
+// short chunks (4 MMA per step -> 8 accumulates per chunk) whose partial
+// sums are added with round-to-nearest fp32 on the CUDA cores.
+constexpr int kChunkSteps = 2;
 
 __device__ __forceinline__ float load_w(const GemmArgs &g, int64_t r, int64_t c) {
     if (g.w_is_bf16)
@@ -119,7 +131,7 @@ __device__ __forceinline__ void epilogue_row(const GemmArgs &g, int r, int c0, c
 }
 
 template <int BN>
-__global__ void __launch_bounds__(128, 1)
+__global__ void __launch_bounds__(320, 1)
     k_tc_gemm(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb,
               const GemmArgs g) {
     using C = GemmCfg<BN>;
@@ -128,8 +140,9 @@ __global__ void __launch_bounds__(128, 1)
     uint8_t *smem = smem_raw + pad;
     uint64_t *full = reinterpret_cast<uint64_t *>(smem + C::STAGES * C::STAGE_BYTES);
     uint64_t *empty = full + C::STAGES;
-    uint64_t *done = empty + C::STAGES;
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(done + 1);
+    uint64_t *acc_full = empty + C::STAGES;   // [2]: chunk accumulated in buffer b
+    uint64_t *acc_empty = acc_full + 2;       // [2]: buffer b drained by the epilogue
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(acc_empty + 2);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5;
@@ -146,13 +159,17 @@ __global__ void __launch_bounds__(128, 1)
     const int kb_hi =
         g.kb_begin + static_cast<int>((static_cast<long long>(g.kb_count) * (split + 1)) / splits);
     const int nsteps = (kb_hi - kb_lo) * g.n_prod;
+    const int nchunks = (nsteps + kChunkSteps - 1) / kChunkSteps;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < C::STAGES; ++s) {
             mbar_init(&full[s], 1);
             mbar_init(&empty[s], 1);
         }
-        mbar_init(done, 1);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&acc_full[b], 1);
+            mbar_init(&acc_empty[b], 256);
+        }
         *abort_flag = 0;
         fence_mbar_init();
     }
@@ -160,75 +177,113 @@ __global__ void __launch_bounds__(128, 1)
         prefetch_tensormap(&ta);
         prefetch_tensormap(&tb);
     }
-    if (warp == 2) tmem_alloc(tmem_slot, C::TMEM_COLS);
+    if (warp == 1) tmem_alloc(tmem_slot, C::TMEM_COLS);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
-    if (warp == 0 && lane == 0) {
-        // ---- TMA producer ----
-        for (int st = 0; st < nsteps; ++st) {
-            const int s = st % C::STAGES;
-            const uint32_t ph = (st / C::STAGES) & 1u;
-            if (!mbar_wait_bounded(&empty[s], ph ^ 1u, abort_flag)) {
-                *abort_flag = 1;
-                set_error(g.err, ERR_TIMEOUT);
-                break;
+    if (warp == 0) {
+        if (lane == 0) {
+            // ---- TMA producer ----
+            for (int st = 0; st < nsteps; ++st) {
+                const int s = st % C::STAGES;
+                const uint32_t ph = (st / C::STAGES) & 1u;
+                if (!mbar_wait_bounded(&empty[s], ph ^ 1u, abort_flag)) {
+                    *abort_flag = 1;
+                    set_error(g.err, ERR_TIMEOUT);
+                    break;
+                }
+                const int kb = kb_lo + st / g.n_prod;
+                const int t = st % g.n_prod;
+                uint8_t *sa = smem + s * C::STAGE_BYTES;
+                uint8_t *sb = sa + C::A_BYTES;
+                mbar_arrive_expect_tx(&full[s], C::STAGE_BYTES);
+                tma_load_2d(&ta, sa, &full[s], kb * C::BK, g.a_row0 + m0 + g.prod_a[t] * g.a_plane_rows);
+                tma_load_2d(&tb, sb, &full[s], kb * C::BK, g.b_row0 + n0 + g.prod_b[t] * g.b_plane_rows);
             }
-            const int kb = kb_lo + st / g.n_prod;
-            const int t = st % g.n_prod;
-            uint8_t *sa = smem + s * C::STAGE_BYTES;
-            uint8_t *sb = sa + C::A_BYTES;
-            mbar_arrive_expect_tx(&full[s], C::STAGE_BYTES);
-            tma_load_2d(&ta, sa, &full[s], kb * C::BK, g.a_row0 + m0 + g.prod_a[t] * g.a_plane_rows);
-            tma_load_2d(&tb, sb, &full[s], kb * C::BK, g.b_row0 + n0 + g.prod_b[t] * g.b_plane_rows);
         }
-    } else if (warp == 1 && lane == 0) {
-        // ---- MMA issuer ----
-        constexpr uint32_t idesc = idesc_bf16_f32(C::BM, BN);
-        for (int st = 0; st < nsteps; ++st) {
-            const int s = st % C::STAGES;
-            const uint32_t ph = (st / C::STAGES) & 1u;
-            if (!mbar_wait_bounded(&full[s], ph, abort_flag)) {
+    } else if (warp == 1) {
+        if (lane == 0) {
+            // ---- MMA issuer: chunk c accumulates into TMEM buffer c & 1 ----
+            constexpr uint32_t idesc = idesc_bf16_f32(C::BM, BN);
+            int st = 0;
+            for (int c = 0; c < nchunks && !*abort_flag; ++c) {
+                const int buf = c & 1;
+                if (c >= 2 && !mbar_wait_bounded(&acc_empty[buf], ((c >> 1) - 1) & 1u, abort_flag)) {
+                    *abort_flag = 1;
+                    set_error(g.err, ERR_TIMEOUT);
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t dst = tmem + static_cast<uint32_t>(buf * BN);
+                const int st_end = (st + kChunkSteps < nsteps) ? st + kChunkSteps : nsteps;
+                for (int first = 1; st < st_end; ++st, first = 0) {
+                    const int s = st % C::STAGES;
+                    const uint32_t ph = (st / C::STAGES) & 1u;
+                    if (!mbar_wait_bounded(&full[s], ph, abort_flag)) {
+                        *abort_flag = 1;
+                        set_error(g.err, ERR_TIMEOUT);
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t sa = smem_u32(smem + s * C::STAGE_BYTES);
+                    const uint64_t da = smem_desc_k128(sa);
+                    const uint64_t db = smem_desc_k128(sa + C::A_BYTES);
+#pragma unroll
+                    for (int k = 0; k < C::BK / 16; ++k)
+                        mma_bf16_ss(dst, da + 2u * k, db + 2u * k, idesc, (first && k == 0) ? 0u : 1u);
+                    mma_commit(&empty[s]);
+                }
+                mma_commit(&acc_full[buf]);   // arrives when this chunk's MMAs complete
+            }
+        }
+    } else {
+        // ---- epilogue warps 2..9: fold chunks into fp32 registers, then store ----
+        const int quad = warp & 3;                    // TMEM lanes 32*quad .. +31
+        const int half = (warp - 2) >> 2;             // columns [half*BN/2, +BN/2)
+        const uint32_t tl = tmem + (static_cast<uint32_t>(quad * 32) << 16) +
+                            static_cast<uint32_t>(half * C::HALF);
+        float acc[C::HALF];
+#pragma unroll
+        for (int i = 0; i < C::HALF; ++i) acc[i] = 0.0f;
+        bool ok = true;
+        for (int c = 0; c < nchunks; ++c) {
+            const int buf = c & 1;
+            if (!mbar_wait_bounded(&acc_full[buf], (c >> 1) & 1u, abort_flag)) {
+                ok = false;
+                if (lane == 0) set_error(g.err, ERR_TIMEOUT);
                 *abort_flag = 1;
-                set_error(g.err, ERR_TIMEOUT);
                 break;
             }
             tc_fence_after();
-            const uint32_t sa = smem_u32(smem + s * C::STAGE_BYTES);
-            const uint64_t da = smem_desc_k128(sa);
-            const uint64_t db = smem_desc_k128(sa + C::A_BYTES);
 #pragma unroll
-            for (int k = 0; k < C::BK / 16; ++k)
-                mma_bf16_ss(tmem, da + 2u * k, db + 2u * k, idesc, (st | k) != 0 ? 1u : 0u);
-            mma_commit(&empty[s]);
-        }
-        mma_commit(done);  // arrives when every MMA issued above has completed
-    }
-    __syncwarp();
-
-    // ---- epilogue: TMEM -> registers -> global ----
-    const bool ok = mbar_wait_bounded(done, 0u, nullptr);
-    if (!ok && threadIdx.x == 0) set_error(g.err, ERR_TIMEOUT);
-    tc_fence_after();
-    const bool valid = ok && (*abort_flag == 0);
-    const int r = m0 + warp * 32 + lane;
-    const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
-    for (int c = 0; c < BN; c += 32) {
-        if (n0 + c >= g.N) break;  // uniform over the CTA
-        float v[32];
-        if (nsteps > 0) {
-            tmem_ld_32x32b_x32(trow + static_cast<uint32_t>(c), v);
-        } else {
+            for (int q = 0; q < C::HALF / 32; ++q) {
+                float v[32];
+                tmem_ld_32x32b_x32(tl + static_cast<uint32_t>(buf * BN + q * 32), v);
 #pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] = 0.0f;
+                for (int i = 0; i < 32; ++i) acc[q * 32 + i] += v[i];
+            }
+            tc_fence_before();
+            mbar_arrive(&acc_empty[buf]);
         }
-        if (valid) epilogue_row(g, r, n0 + c, v, split);
+        if (ok && *abort_flag == 0) {
+            const int r = m0 + quad * 32 + lane;
+#pragma unroll
+            for (int q = 0; q < C::HALF / 32; ++q) {
+                const int c0 = n0 + half * C::HALF + q * 32;
+                if (c0 < g.N) {
+                    float v[32];
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) v[i] = acc[q * 32 + i];
+                    epilogue_row(g, r, c0, v, split);
+                }
+            }
+        }
     }
     tc_fence_before();
     __syncthreads();
-    if (warp == 2) tmem_dealloc(tmem, C::TMEM_COLS);
+    if (warp == 1) tmem_dealloc(tmem, C::TMEM_COLS);
 }
 
 // ---- host side ---------------------------------------------------------------
@@ -271,13 +326,13 @@ static cudaError_t launch_bn(const CUtensorMap &ta, const CUtensorMap &tb, const
     if (e != cudaSuccess) return e;
     dim3 grid(static_cast<unsigned>(ceil_div(g.N, BN)), static_cast<unsigned>(ceil_div(g.M, C::BM)),
               static_cast<unsigned>(splits));
-    k_tc_gemm<BN><<<grid, 128, C::SMEM_BYTES, s>>>(ta, tb, g);
+    k_tc_gemm<BN><<<grid, C::THREADS, C::SMEM_BYTES, s>>>(ta, tb, g);
     return cudaGetLastError();
 }
 
 cudaError_t launch_tc_gemm(int BN, const CUtensorMap &ta, const CUtensorMap &tb, const GemmArgs &g,
                            int splits, cudaStream_t s) {
-    if (g.M <= 0 || g.N <= 0 || splits < 1 || g.n_prod < 1 || g.n_prod > 3)
+    if (g.M <= 0 || g.N <= 0 || splits < 1 || g.n_prod < 1 || g.n_prod > 6)
         return cudaErrorInvalidValue;
     if (ceil_div(g.M, 128) > 65535 || splits > 65535) return cudaErrorInvalidValue;
     switch (BN) {

@@ -19,8 +19,8 @@ enum EpiMode : int {
 struct GemmArgs {
     int M, N;                 // extent of the output window
     int kb_begin, kb_count;   // 64-wide k-blocks covered (split evenly over gridDim.z)
-    int n_prod;               // products per k-block (1..3)
-    int prod_a[3], prod_b[3]; // operand plane of each product
+    int n_prod;               // products per k-block (1..6)
+    int prod_a[6], prod_b[6]; // operand plane of each product
     int a_plane_rows, b_plane_rows;  // row distance between stacked planes in the maps
     int a_row0, b_row0;       // row offsets of the operand windows
     int mode;

@@ -17,7 +17,7 @@ struct CdArgs {
     const float *part;              // split-K partials [nsplit][q][ldpart] (t-units)
     int nsplit;
     int64_t part_stride, ldpart;
-    const __nv_bfloat16 *snt;       // Sigma_bar^T hi plane; lo plane snt_plane_rows rows below
+    const __nv_bfloat16 *snt;       // Sigma_bar^T hi plane; mid / lo planes snt_plane_rows apart
     int64_t ldsn, snt_plane_rows;
     const float *scale, *zero;
     float maxq;
@@ -26,7 +26,7 @@ struct CdArgs {
     int64_t ldc;
     __nv_bfloat16 *qf;              // out: C - z
     int64_t ldq;
-    __nv_bfloat16 *dp;              // out: Delta' hi plane (lo plane dp_plane_rows rows below)
+    __nv_bfloat16 *dp;              // out: Delta' hi plane (mid / lo planes dp_plane_rows apart)
     int64_t ldd, dp_plane_rows;
 };
 
@@ -50,7 +50,7 @@ cudaError_t launch_grid(const void *W, int w_bf16, int64_t ldw, const float *H, 
 cudaError_t launch_sigma_norm(const float *S, int64_t lds, int64_t p, float *d, __nv_bfloat16 *snt,
                               int64_t ldn, unsigned *err, cudaStream_t s);
 cudaError_t launch_make_planes(const void *W, int w_bf16, int64_t ldw, int64_t q, int64_t p,
-                               int two_planes, __nv_bfloat16 *out, int64_t ldo, cudaStream_t s);
+                               int split, __nv_bfloat16 *out, int64_t ldo, cudaStream_t s);
 cudaError_t launch_init_residual(const void *W, int w_bf16, int64_t ldw, const float *H, int64_t ldh,
                                  int64_t q, int64_t p, float *R, int64_t ldr, cudaStream_t s);
 cudaError_t launch_codes_to_qf(const uint8_t *codes, int64_t ldc, const float *zero, int64_t q,
