@@ -55,7 +55,7 @@ typedef enum {
 } qe_xlayout;
 
 typedef struct {
-    /* Column block width B of the blocked CD sweep: 0 = default (64); 32 or 64. */
+    /* Column block width B of the blocked CD sweep: 0 = default (256); 64, 128 or 256. */
     int block_width;
     /* Relax heuristic of Sec. 3.2 (skip quantization every R-th sweep): must be 0. */
     int relax_period;

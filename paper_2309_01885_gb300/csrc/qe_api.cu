@@ -44,14 +44,14 @@ static int sm_count() {
     return n;
 }
 
-constexpr int kDefaultBlock = 64;
+constexpr int kDefaultBlock = 256;
 constexpr int kDefaultPowerIters = 64;
 
 // ---- workspace layout -----------------------------------------------------------
 struct Plan {
     int64_t q = 0, p = 0, ld = 0;
     int B = kDefaultBlock, smax = 1;
-    size_t snt = 0, d = 0, dinv = 0, P = 0, R = 0, wpl = 0, qf = 0, dp = 0, part = 0, objp = 0;
+    size_t snt = 0, d = 0, dinv = 0, tri = 0, P = 0, R = 0, wpl = 0, qf = 0, dp = 0, part = 0, objp = 0;
     size_t PW = 0, H = 0, T = 0, st = 0, cg = 0, ce = 0, sb = 0, eb = 0, y0 = 0, y1 = 0, lam = 0,
            eta = 0, rowptr = 0;
     size_t total = 0;
@@ -79,6 +79,7 @@ static Plan make_plan(int64_t q, int64_t p, int B, bool outlier, int wpl_planes,
     pl.snt = take(cur, static_cast<size_t>(3 * p) * pl.ld * 2);
     pl.d = take(cur, p * 4);
     pl.dinv = take(cur, p * 4);
+    pl.tri = take(cur, static_cast<size_t>(packed_diag_floats(p, B)) * 4);
     pl.P = take(cur, qld * 4);
     pl.R = take(cur, qld * 4);
     pl.wpl = take(cur, wpl_planes > 0 ? qld * 2 * wpl_planes : 0);
@@ -116,14 +117,14 @@ struct Ctx {
     uint8_t *ws = nullptr;
     bool own = false;
     __nv_bfloat16 *snt = nullptr, *wpl = nullptr, *qf = nullptr, *dp = nullptr;
-    float *d = nullptr, *dinv = nullptr, *P = nullptr, *R = nullptr, *part = nullptr;
+    float *d = nullptr, *dinv = nullptr, *tri = nullptr, *P = nullptr, *R = nullptr, *part = nullptr;
     double *objp = nullptr;
     float *PW = nullptr, *H = nullptr, *T = nullptr, *y0 = nullptr, *y1 = nullptr;
     TopkState *st = nullptr;
     unsigned *cg = nullptr, *ce = nullptr, *sb = nullptr, *eb = nullptr;
     double *lam = nullptr, *eta = nullptr;
     int64_t *rowptr = nullptr;
-    CUtensorMap tm_snt256, tm_snt64, tm_qf, tm_dp, tm_wa;
+    CUtensorMap tm_snt256, tm_snt64, tm_snt128, tm_qf, tm_dp, tm_wa;
     int wa_planes = 1;
 
     ~Ctx() {
@@ -158,6 +159,7 @@ static qe_status setup_ctx(Ctx &c, const Plan &pl, const qe_opts *o, cudaStream_
     c.snt = at<__nv_bfloat16>(w, pl.snt);
     c.d = at<float>(w, pl.d);
     c.dinv = at<float>(w, pl.dinv);
+    c.tri = at<float>(w, pl.tri);
     c.P = at<float>(w, pl.P);
     c.R = at<float>(w, pl.R);
     c.wpl = at<__nv_bfloat16>(w, pl.wpl);
@@ -183,6 +185,7 @@ static qe_status setup_ctx(Ctx &c, const Plan &pl, const qe_opts *o, cudaStream_
     const uint64_t q = pl.q, p = pl.p, ld = pl.ld;
     if (!make_tmap_bf16(&c.tm_snt256, c.snt, 3 * p, p, ld, 256) ||
         !make_tmap_bf16(&c.tm_snt64, c.snt, 3 * p, p, ld, 64) ||
+        !make_tmap_bf16(&c.tm_snt128, c.snt, 3 * p, p, ld, 128) ||
         !make_tmap_bf16(&c.tm_qf, c.qf, q, p, ld, 128) ||
         !make_tmap_bf16(&c.tm_dp, c.dp, 3 * q, p, ld, 128))
         return QE_ERR_CUDA;
@@ -226,6 +229,7 @@ static qe_status prepare(Ctx &c, const void *W, int wbf16, int64_t ldw, const fl
     const int64_t q = c.pl.q, p = c.pl.p, ld = c.pl.ld;
     QE_CK(launch_sigma_norm(Sigma, p, p, c.d, c.snt, ld, c.err, c.s));
     QE_CK(launch_dinv(c.d, p, c.dinv, c.s));
+    QE_CK(launch_pack_diag(c.snt, ld, p, c.pl.B, c.tri, c.s));
     const bool direct = wbf16 && ((reinterpret_cast<uintptr_t>(W) & 15u) == 0) && (ldw % 8 == 0);
     if (direct) {
         if (!make_tmap_bf16(&c.tm_wa, W, q, p, ldw, 128)) return QE_ERR_CUDA;
@@ -285,7 +289,8 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
             g.out = c.part;
             g.ldo = B;
             g.split_stride = q * B;
-            QE_CK(launch_tc_gemm(64, c.tm_dp, c.tm_snt64, g, S, c.s));
+            QE_CK(launch_tc_gemm(B, c.tm_dp, B == 64 ? c.tm_snt64 : (B == 128 ? c.tm_snt128 : c.tm_snt256), g,
+                                 S, c.s));
             nsplit = S;
         }
         CdArgs a;
@@ -300,9 +305,7 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
         a.nsplit = nsplit;
         a.part_stride = q * B;
         a.ldpart = B;
-        a.snt = c.snt;
-        a.ldsn = ld;
-        a.snt_plane_rows = p;
+        a.tri = c.tri;
         a.scale = scales;
         a.zero = zeros;
         a.maxq = static_cast<float>((1 << bits) - 1);
@@ -342,10 +345,15 @@ static qe_status objective(Ctx &c, const void *W, int wbf16, int64_t ldw, const 
     return QE_OK;
 }
 
+static int block_width(const qe_opts *o) {
+    return (o && o->block_width) ? o->block_width : kDefaultBlock;
+}
+
 static qe_status check_opts(const qe_opts *o) {
     if (!o) return QE_OK;
     if (o->relax_period != 0 || o->structured_outliers != 0) return QE_ERR_UNSUPPORTED;
-    if (o->block_width != 0 && o->block_width != 64) return QE_ERR_UNSUPPORTED;
+    if (o->block_width != 0 && o->block_width != 64 && o->block_width != 128 && o->block_width != 256)
+        return QE_ERR_UNSUPPORTED;
     if (o->power_iters < 0) return QE_ERR_INVALID_ARG;
     if (o->workspace && o->workspace_bytes == 0) return QE_ERR_INVALID_ARG;
     return QE_OK;
@@ -405,7 +413,7 @@ qe_status qe_workspace_size(int64_t q, int64_t p, int outlier, const qe_opts *op
     if (!bytes || q < 1 || p < 1) return QE_ERR_INVALID_ARG;
     const qe_status st = check_opts(opts);
     if (st != QE_OK) return st;
-    const Plan pl = make_plan(q, p, kDefaultBlock, outlier != 0, 3, sm_count());
+    const Plan pl = make_plan(q, p, block_width(opts), outlier != 0, 3, sm_count());
     *bytes = pl.total;
     return QE_OK;
 }
@@ -490,7 +498,7 @@ qe_status qe_quantize_layer(const void *W, qe_dtype w_dtype, int64_t q, int64_t 
     if ((st = check_opts(opts)) != QE_OK) return st;
     const int wbf16 = (w_dtype == QE_BF16);
     Ctx c;
-    const Plan pl = make_plan(q, p, kDefaultBlock, false, wbf16 ? 1 : 3, sm_count());
+    const Plan pl = make_plan(q, p, block_width(opts), false, wbf16 ? 1 : 3, sm_count());
     if ((st = setup_ctx(c, pl, opts, reinterpret_cast<cudaStream_t>(stream))) != QE_OK) return st;
 
     QE_CK(launch_grid(W, wbf16, ldw, nullptr, 0, q, p, bits, scales, zeros, c.err, c.s));
@@ -532,7 +540,7 @@ qe_status qe_quantize_layer_outlier(const void *W, qe_dtype w_dtype, int64_t q, 
     const int power_iters = (opts && opts->power_iters > 0) ? opts->power_iters : kDefaultPowerIters;
     Ctx c;
     c.nsm = sm_count();
-    const Plan pl = make_plan(q, p, kDefaultBlock, true, wbf16 ? 1 : 3, c.nsm);
+    const Plan pl = make_plan(q, p, block_width(opts), true, wbf16 ? 1 : 3, c.nsm);
     if ((st = setup_ctx(c, pl, opts, reinterpret_cast<cudaStream_t>(stream))) != QE_OK) return st;
     const int64_t ld = pl.ld;
 

@@ -154,7 +154,8 @@ __global__ void k_codes_to_qf(const uint8_t *codes, int64_t ldc, const float *ze
 
 // ---------------------------------------------------------------------------
 // In-block sequential CD (Algorithm 3 inner loop, one column block of width B).
-// One thread per row i (rows are independent, Sec. 3.2).  Work in units of the
+// One warp per row i (rows are independent, Sec. 3.2); the lanes hold the
+// block's columns and the decisions travel by warp shuffles.  Work in units of the
 // grid step: t_ij = beta_ij / s_i + z_i, so the code is rint(clamp(t, 0, 2^b-1))
 // (the nearest level, Eq. eq:quant) and the column change is
 // Delta'_ij = (What_start_ij - What_new_ij) / s_i = a_ij - c_ij with
@@ -165,95 +166,132 @@ __global__ void k_codes_to_qf(const uint8_t *codes, int64_t ldc, const float *ze
 // the in-block contributions Delta'_ij Sigma_bar_jl (j < l in the block) are
 // added here, right after column j is decided.
 // ---------------------------------------------------------------------------
+// Packed strict upper triangle of a diagonal B x B block of Sigma_bar:
+// row j holds columns j+1 .. B-1 at kPackPad + tri_off(j) + (l - j - 1).  The
+// kPackPad floats in front keep the harmless reads of already-decided lanes
+// (l <= j, see the chain below) inside the array.
+constexpr int kPackPad = 32;
+__host__ __device__ constexpr int tri_off(int B, int j) { return j * B - (j * (j + 1)) / 2; }
+__host__ __device__ constexpr int packed_block_floats(int B) {
+    return static_cast<int>(round_up(kPackPad + B * (B - 1) / 2, 4));
+}
+
+// One diagonal block per CTA row of the grid: Sigma_bar[b0 + j][b0 + l] for l > j,
+// from the hi + mid + lo planes (the same values the tensor-core GEMMs use).
+__global__ void k_pack_diag(const __nv_bfloat16 *snt, int64_t ldn, int64_t plane_rows, int64_t p, int B,
+                            float *out) {
+    const int bi = blockIdx.x, j = blockIdx.y;
+    const int64_t b0 = static_cast<int64_t>(bi) * B;
+    float *blk = out + static_cast<int64_t>(bi) * packed_block_floats(B);
+    const int64_t pl = plane_rows * ldn;
+    if (j == 0 && threadIdx.x < kPackPad) blk[threadIdx.x] = 0.0f;
+    for (int l = j + 1 + threadIdx.x; l < B; l += blockDim.x) {
+        float v = 0.0f;
+        if (b0 + j < p && b0 + l < p) {
+            const int64_t o = (b0 + l) * ldn + b0 + j;
+            v = __bfloat162float(snt[o]) + __bfloat162float(snt[pl + o]) + __bfloat162float(snt[2 * pl + o]);
+        }
+        blk[kPackPad + tri_off(B, j) + (l - j - 1)] = v;
+    }
+}
+
 template <int B>
-__global__ void __launch_bounds__(32) k_cd_block(const CdArgs a) {
-    constexpr int RP = B + 1;  // padded row of the per-row staging tiles
-    constexpr int SP = B + 4;  // padded row of the Sigma_bar block (16-byte aligned)
-    __shared__ __align__(16) float sig[B][SP];
-    __shared__ float cin[32][RP];
-    __shared__ float ain[32][RP];
-    const int lane = threadIdx.x;
-    const int64_t i0 = static_cast<int64_t>(blockIdx.x) * 32;
-    const int bw = a.bw;
+struct CdCfg {
+    static constexpr int CPL = B / 32;                    // columns owned by each lane
+    static constexpr int WARPS = (B == 256) ? 32 : 16;    // rows per CTA (one row per warp)
+    static constexpr int PACK = packed_block_floats(B);
+    static constexpr int SMEM = (PACK + WARPS * 2 * B) * 4;
+};
+
+template <int B, bool FULL>
+__global__ void __launch_bounds__(32 * CdCfg<B>::WARPS) k_cd_block(const CdArgs a) {
+    using C = CdCfg<B>;
+    constexpr int CPL = C::CPL, NT = 32 * C::WARPS;
+    extern __shared__ __align__(16) float cd_smem[];
+    float *tri = cd_smem;                                  // packed Sigma_bar block
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    float *rec = cd_smem + C::PACK + warp * 2 * B;         // this warp's Delta' and code record
+    const int bw = FULL ? B : a.bw;
     const int64_t b0 = a.b0;
 
-    // Sigma_bar[b0 + k][b0 + l] = SnT[b0 + l][b0 + k] (hi + mid + lo)
-    for (int idx = lane; idx < B * B; idx += 32) {
-        const int k = idx % B, l = idx / B;
-        float v = 0.0f;
-        if (k < bw && l < bw) {
-            const int64_t o = (b0 + l) * a.ldsn + b0 + k;
-            const int64_t pl = a.snt_plane_rows * a.ldsn;
-            v = __bfloat162float(a.snt[o]) + __bfloat162float(a.snt[pl + o]) +
-                __bfloat162float(a.snt[2 * pl + o]);
-        }
-        sig[k][l] = v;
+    {
+        const float4 *src = reinterpret_cast<const float4 *>(a.tri + (b0 / B) * C::PACK);
+        float4 *dst = reinterpret_cast<float4 *>(tri);
+        for (int e = tid; e < C::PACK / 4; e += NT) dst[e] = src[e];
     }
-    // stage the block of t values and start values, coalesced over columns
-    for (int r = 0; r < 32; ++r) {
-        const int64_t i = i0 + r;
-        if (i >= a.q) {
-            for (int l = lane; l < B; l += 32) cin[r][l] = ain[r][l] = 0.0f;
-            continue;
-        }
-        const float s = a.scale[i], z = a.zero[i];
-        for (int l = lane; l < B; l += 32) {
-            float t = 0.0f, st = 0.0f;
-            if (l < bw) {
-                t = __fdiv_rn(a.R[i * a.ldr + b0 + l], s) + z;
-                st = a.first_sweep ? t : static_cast<float>(a.codes[i * a.ldc + b0 + l]);
-                for (int sp = 0; sp < a.nsplit; ++sp)
-                    t += a.part[sp * a.part_stride + i * a.ldpart + l];
-            }
-            cin[r][l] = t;
-            ain[r][l] = st;
-        }
-    }
-    __syncwarp();
+    __syncthreads();
 
-    // the sequential chain, one row per lane
-    float acc[B];
+    const int64_t i = static_cast<int64_t>(blockIdx.x) * C::WARPS + warp;
+    if (i >= a.q) return;
+    const float s = a.scale[i], z = a.zero[i];
+
+    // t = R / s + z + sum of split partials (grid-step units); st = start value
+    float t[CPL], st[CPL];
 #pragma unroll
-    for (int l = 0; l < B; ++l) acc[l] = cin[lane][l];
+    for (int h = 0; h < CPL; ++h) {
+        const int l = 32 * h + lane;
+        t[h] = 0.0f;
+        st[h] = 0.0f;
+        if (FULL || l < bw) {
+            t[h] = __fdiv_rn(a.R[i * a.ldr + b0 + l], s) + z;
+            st[h] = a.first_sweep ? t[h] : static_cast<float>(a.codes[i * a.ldc + b0 + l]);
+        }
+    }
+    for (int sp = 0; sp < a.nsplit; ++sp) {
+        const float *prow = a.part + sp * a.part_stride + i * a.ldpart;
+#pragma unroll
+        for (int h = 0; h < CPL; ++h)
+            if (FULL || 32 * h + lane < bw) t[h] += prow[32 * h + lane];
+    }
+
+    // The chain: column j = 32 h + jj is decided by lane jj; its code and change
+    // Delta' (db, the same in every lane after the shuffle) are recorded, and db,
+    // times
+    // Sigma_bar[j][l], to every later column l.  Lanes whose column is already
+    // decided (l <= j) absorb harmless updates, so no lane test is needed; an
+    // unchanged column (db == 0, the common case once the codes settle) skips
+    // the updates altogether.
     const float maxq = a.maxq;
+    const bool writer = lane == 0;
 #pragma unroll
-    for (int j = 0; j < B; ++j) {
-        if (j < bw) {
-            const float c = rintf(fminf(fmaxf(acc[j], 0.0f), maxq));
-            const float dl = ain[lane][j] - c;
-            ain[lane][j] = dl;
-            cin[lane][j] = c;
+    for (int h = 0; h < CPL; ++h) {
 #pragma unroll
-            for (int l4 = ((j + 1) & ~3); l4 < B; l4 += 4) {
-                const float4 sv = *reinterpret_cast<const float4 *>(&sig[j][l4]);
-                if (l4 + 0 > j) acc[l4 + 0] = fmaf(dl, sv.x, acc[l4 + 0]);
-                if (l4 + 1 > j) acc[l4 + 1] = fmaf(dl, sv.y, acc[l4 + 1]);
-                if (l4 + 2 > j) acc[l4 + 2] = fmaf(dl, sv.z, acc[l4 + 2]);
-                if (l4 + 3 > j) acc[l4 + 3] = fmaf(dl, sv.w, acc[l4 + 3]);
+        for (int jj = 0; jj < 32; ++jj) {
+            const int j = 32 * h + jj;
+            if (!FULL && j >= bw) break;
+            const float c = rintf(fminf(fmaxf(t[h], 0.0f), maxq));
+            const float db = __shfl_sync(0xffffffffu, st[h] - c, jj);
+            const float cb = __shfl_sync(0xffffffffu, c, jj);
+            if (writer) {
+                rec[j] = db;
+                rec[B + j] = cb;
+            }
+            if (db != 0.0f) {
+                const float *row = tri + kPackPad + tri_off(B, j) - (j + 1);
+#pragma unroll
+                for (int g = h; g < CPL; ++g) t[g] = fmaf(db, row[32 * g + lane], t[g]);
             }
         }
     }
     __syncwarp();
 
-    // write codes, C - z and the Delta' plane(s), coalesced over columns
-    for (int r = 0; r < 32; ++r) {
-        const int64_t i = i0 + r;
-        if (i >= a.q) break;
-        const float z = a.zero[i];
-        for (int l = lane; l < bw; l += 32) {
-            const float c = cin[r][l];
-            const float dl = ain[r][l];
-            const int64_t col = b0 + l;
-            a.codes[i * a.ldc + col] = static_cast<uint8_t>(c);
-            a.qf[i * a.ldq + col] = __float2bfloat16_rn(c - z);
-            const __nv_bfloat16 h = __float2bfloat16_rn(dl);
-            a.dp[i * a.ldd + col] = h;
-            if (a.first_sweep) {   // Delta' is not an integer in the first sweep: three planes
-                const float r1 = dl - __bfloat162float(h);
-                const __nv_bfloat16 m = __float2bfloat16_rn(r1);
-                a.dp[(a.dp_plane_rows + i) * a.ldd + col] = m;
-                a.dp[(2 * a.dp_plane_rows + i) * a.ldd + col] = __float2bfloat16_rn(r1 - __bfloat162float(m));
-            }
+    // codes, C - z and the Delta' plane(s)
+#pragma unroll
+    for (int h = 0; h < CPL; ++h) {
+        const int l = 32 * h + lane;
+        if (!FULL && l >= bw) continue;
+        const float dl = rec[l];
+        const float code = rec[B + l];
+        const int64_t col = b0 + l;
+        a.codes[i * a.ldc + col] = static_cast<uint8_t>(code);
+        a.qf[i * a.ldq + col] = __float2bfloat16_rn(code - z);
+        const __nv_bfloat16 hi = __float2bfloat16_rn(dl);
+        a.dp[i * a.ldd + col] = hi;
+        if (a.first_sweep) {   // Delta' is not an integer in the first sweep: three planes
+            const float r1 = dl - __bfloat162float(hi);
+            const __nv_bfloat16 mid = __float2bfloat16_rn(r1);
+            a.dp[(a.dp_plane_rows + i) * a.ldd + col] = mid;
+            a.dp[(2 * a.dp_plane_rows + i) * a.ldd + col] = __float2bfloat16_rn(r1 - __bfloat162float(mid));
         }
     }
 }
@@ -444,11 +482,33 @@ cudaError_t launch_codes_to_qf(const uint8_t *codes, int64_t ldc, const float *z
     return cudaGetLastError();
 }
 
+template <int B, bool FULL>
+static cudaError_t launch_cd_block_b(const CdArgs &a, cudaStream_t s) {
+    using C = CdCfg<B>;
+    cudaError_t e = cudaFuncSetAttribute(k_cd_block<B, FULL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         C::SMEM);
+    if (e != cudaSuccess) return e;
+    const unsigned grid = static_cast<unsigned>(ceil_div(a.q, C::WARPS));
+    k_cd_block<B, FULL><<<grid, 32 * C::WARPS, C::SMEM, s>>>(a);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_cd_block(int B, const CdArgs &a, cudaStream_t s) {
-    const unsigned grid = static_cast<unsigned>(ceil_div(a.q, 32));
-    if (B == 64) k_cd_block<64><<<grid, 32, 0, s>>>(a);
-    else if (B == 32) k_cd_block<32><<<grid, 32, 0, s>>>(a);
-    else return cudaErrorInvalidValue;
+    const bool full = a.bw == B;
+    switch (B) {
+        case 64: return full ? launch_cd_block_b<64, true>(a, s) : launch_cd_block_b<64, false>(a, s);
+        case 128: return full ? launch_cd_block_b<128, true>(a, s) : launch_cd_block_b<128, false>(a, s);
+        case 256: return full ? launch_cd_block_b<256, true>(a, s) : launch_cd_block_b<256, false>(a, s);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
+int64_t packed_diag_floats(int64_t p, int B) { return ceil_div(p, B) * packed_block_floats(B); }
+
+cudaError_t launch_pack_diag(const __nv_bfloat16 *snt, int64_t ldn, int64_t p, int B, float *out,
+                             cudaStream_t s) {
+    dim3 grid(static_cast<unsigned>(ceil_div(p, B)), static_cast<unsigned>(B));
+    k_pack_diag<<<grid, 128, 0, s>>>(snt, ldn, p, p, B, out);
     return cudaGetLastError();
 }
 

@@ -17,8 +17,7 @@ struct CdArgs {
     const float *part;              // split-K partials [nsplit][q][ldpart] (t-units)
     int nsplit;
     int64_t part_stride, ldpart;
-    const __nv_bfloat16 *snt;       // Sigma_bar^T hi plane; mid / lo planes snt_plane_rows apart
-    int64_t ldsn, snt_plane_rows;
+    const float *tri;               // packed diagonal blocks of Sigma_bar (launch_pack_diag)
     const float *scale, *zero;
     float maxq;
     int first_sweep;                // What_start is R itself (not on the grid)
@@ -56,6 +55,9 @@ cudaError_t launch_init_residual(const void *W, int w_bf16, int64_t ldw, const f
 cudaError_t launch_codes_to_qf(const uint8_t *codes, int64_t ldc, const float *zero, int64_t q,
                                int64_t p, __nv_bfloat16 *qf, int64_t ldq, cudaStream_t s);
 cudaError_t launch_cd_block(int B, const CdArgs &a, cudaStream_t s);
+int64_t packed_diag_floats(int64_t p, int B);
+cudaError_t launch_pack_diag(const __nv_bfloat16 *snt, int64_t ldn, int64_t p, int B, float *out,
+                             cudaStream_t s);
 int objective_blocks(int64_t q);
 cudaError_t launch_objective(const ObjArgs &a, double *partial, double *out, cudaStream_t s);
 
