@@ -283,7 +283,7 @@ def main():
     # launches of our kernels per step (schedule of qe_api.cu)
     nblk = (p + 255) // 256                    # default column block width 256
     w_planes = 0 if cfg.w_dtype == torch.bfloat16 else 1
-    per_layer = 7 + w_planes + cfg.iters * (nblk + (nblk - 1) + 1 + 2)
+    per_layer = 7 + w_planes + cfg.iters * (nblk + (nblk - 1) + 1 + 1)
     result["gpu_launches"] = args.steps * (1 + nb * per_layer)
 
     # end to end through the C ABI with host buffers

@@ -86,7 +86,8 @@ static Plan make_plan(int64_t q, int64_t p, int B, bool outlier, int wpl_planes,
     pl.qf = take(cur, qld * 2);
     pl.dp = take(cur, qld * 2 * 3);
     pl.part = take(cur, static_cast<size_t>(pl.smax) * q * B * 4);
-    pl.objp = take(cur, static_cast<size_t>(objective_blocks(q)) * 8);
+    pl.objp = take(cur, static_cast<size_t>(rfull_partials(q, p) > objective_blocks(q) ? rfull_partials(q, p)
+                                                                                    : objective_blocks(q)) * 8);
     if (outlier) {
         const int64_t N = q * p;
         const int64_t nch = topk_chunks(N);
@@ -253,8 +254,20 @@ static qe_status prepare(Ctx &c, const void *W, int wbf16, int64_t ldw, const fl
     return QE_OK;
 }
 
-// R = P - s (C - z) Sigma_bar from the current codes (C - z held in qf).
-static qe_status residual(Ctx &c, const float *scales) {
+// R = P - s (C - z) Sigma_bar from the current codes (C - z held in qf).  With
+// `obj`, the epilogue also reduces f = sum D_ij d_j (R_ij - What_ij) for the
+// codes in `codes` (D = W - What - H) and k_sum_partials writes it to *obj.
+struct ObjFuse {
+    double *obj;
+    const void *W;
+    int wbf16;
+    int64_t ldw;
+    const uint8_t *codes;
+    const float *zeros;
+    const float *H;
+};
+
+static qe_status residual(Ctx &c, const float *scales, const ObjFuse *f = nullptr) {
     const int64_t q = c.pl.q, p = c.pl.p, ld = c.pl.ld;
     GemmArgs g = gemm_args(c, static_cast<int>(q), static_cast<int>(p), static_cast<int>(ceil_div(p, 64)),
                            EPI_RFULL);
@@ -266,7 +279,20 @@ static qe_status residual(Ctx &c, const float *scales) {
     g.P = c.P;
     g.ldp = ld;
     g.scale = scales;
+    if (f) {
+        g.obj_part = c.objp;
+        g.W = f->W;
+        g.w_is_bf16 = f->wbf16;
+        g.ldw = f->ldw;
+        g.codes = f->codes;
+        g.ldc = p;
+        g.zero = f->zeros;
+        g.dvec = c.d;
+        g.Hd = f->H;
+        g.ldh = ld;
+    }
     QE_CK(launch_tc_gemm(256, c.tm_qf, c.tm_snt256, g, 1, c.s));
+    if (f) QE_CK(launch_sum_partials(c.objp, static_cast<int>(rfull_partials(q, p)), f->obj, c.s));
     return QE_OK;
 }
 
@@ -317,7 +343,8 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
         a.dp = c.dp;
         a.ldd = ld;
         a.dp_plane_rows = q;
-        QE_CK(launch_cd_block(B, a, c.s));
+        a.err = c.err;
+        QE_CK(launch_cd_block(B, a, c.nsm, c.s));
     }
     return QE_OK;
 }
@@ -498,7 +525,8 @@ qe_status qe_quantize_layer(const void *W, qe_dtype w_dtype, int64_t q, int64_t 
     if ((st = check_opts(opts)) != QE_OK) return st;
     const int wbf16 = (w_dtype == QE_BF16);
     Ctx c;
-    const Plan pl = make_plan(q, p, block_width(opts), false, wbf16 ? 1 : 3, sm_count());
+    c.nsm = sm_count();
+    const Plan pl = make_plan(q, p, block_width(opts), false, wbf16 ? 1 : 3, c.nsm);
     if ((st = setup_ctx(c, pl, opts, reinterpret_cast<cudaStream_t>(stream))) != QE_OK) return st;
 
     QE_CK(launch_grid(W, wbf16, ldw, nullptr, 0, q, p, bits, scales, zeros, c.err, c.s));
@@ -516,8 +544,8 @@ qe_status qe_quantize_layer(const void *W, qe_dtype w_dtype, int64_t q, int64_t 
     }
     for (int t = 0; t < iters; ++t) {
         if ((st = sweep(c, codes, scales, zeros, bits, t == 0 && !warm)) != QE_OK) return st;
-        if ((st = residual(c, scales)) != QE_OK) return st;
-        if ((st = objective(c, W, wbf16, ldw, nullptr, codes, scales, zeros, c.R, obj + t)) != QE_OK) return st;
+        const ObjFuse f{obj + t, W, wbf16, ldw, codes, zeros, nullptr};
+        if ((st = residual(c, scales, &f)) != QE_OK) return st;
         if (opts && opts->sweep_codes)
             QE_CK(cudaMemcpyAsync(opts->sweep_codes + static_cast<size_t>(t) * q * p, codes,
                                   static_cast<size_t>(q) * p, cudaMemcpyDeviceToDevice, c.s));
@@ -567,9 +595,8 @@ qe_status qe_quantize_layer_outlier(const void *W, qe_dtype w_dtype, int64_t q, 
     }
     for (int t = 0; t < iters; ++t) {
         if ((st = sweep(c, codes, scales, zeros, bits, t == 0 && !warm)) != QE_OK) return st;
-        if ((st = residual(c, scales)) != QE_OK) return st;
-        if (obj_cd)
-            if ((st = objective(c, W, wbf16, ldw, c.H, codes, scales, zeros, c.R, obj_cd + t)) != QE_OK) return st;
+        const ObjFuse f{obj_cd ? obj_cd + t : nullptr, W, wbf16, ldw, codes, zeros, c.H};
+        if ((st = residual(c, scales, obj_cd ? &f : nullptr)) != QE_OK) return st;
         // IHT step: T = H + 2 eta d (R - What); H = P_s(T)
         QE_CK(launch_iht_target(c.H, c.R, ld, codes, p, scales, zeros, c.d, c.eta, q, p, c.T, c.s));
         QE_CK(launch_topk(c.T, N, s_budget, c.st, c.cg, c.ce, c.sb, c.eb, H_idx, H_val, H_nnz, c.nsm, c.s));

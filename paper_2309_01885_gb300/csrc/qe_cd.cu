@@ -168,16 +168,16 @@ __global__ void k_codes_to_qf(const uint8_t *codes, int64_t ldc, const float *ze
 // ---------------------------------------------------------------------------
 // Packed strict upper triangle of a diagonal B x B block of Sigma_bar:
 // row j holds columns j+1 .. B-1 at kPackPad + tri_off(j) + (l - j - 1).  The
-// kPackPad floats in front keep the harmless reads of already-decided lanes
-// (l <= j, see the chain below) inside the array.
+// kPackPad floats in front keep the harmless reads of already-decided columns
+// (l <= j, see the kernels below) inside the array.
 constexpr int kPackPad = 32;
 __host__ __device__ constexpr int tri_off(int B, int j) { return j * B - (j * (j + 1)) / 2; }
 __host__ __device__ constexpr int packed_block_floats(int B) {
     return static_cast<int>(round_up(kPackPad + B * (B - 1) / 2, 4));
 }
 
-// One diagonal block per CTA row of the grid: Sigma_bar[b0 + j][b0 + l] for l > j,
-// from the hi + mid + lo planes (the same values the tensor-core GEMMs use).
+// One diagonal block per grid row: Sigma_bar[b0 + j][b0 + l] (l > j) from the
+// hi + mid + lo planes (the same values the tensor-core GEMMs use).
 __global__ void k_pack_diag(const __nv_bfloat16 *snt, int64_t ldn, int64_t plane_rows, int64_t p, int B,
                             float *out) {
     const int bi = blockIdx.x, j = blockIdx.y;
@@ -198,61 +198,121 @@ __global__ void k_pack_diag(const __nv_bfloat16 *snt, int64_t ldn, int64_t plane
 template <int B>
 struct CdCfg {
     static constexpr int CPL = B / 32;                    // columns owned by each lane
-    static constexpr int WARPS = (B == 256) ? 32 : 16;    // rows per CTA (one row per warp)
+    static constexpr int MAX_WARPS = 32;                  // rows per CTA (one row per warp)
     static constexpr int PACK = packed_block_floats(B);
-    static constexpr int SMEM = (PACK + WARPS * 2 * B) * 4;
+    static constexpr int SMEM = PACK * 4 + 16;            // packed block + its mbarrier
+    static constexpr int MAX_SPLITS = 16;
 };
 
+// Common prologue of both in-block kernels: start the bulk copy of the packed
+// block, stage the row (t = R / s + z + sum of split partials, in grid steps;
+// st = start value: t before the partials in the first sweep, else the old
+// code), then wait for the block.  Lane l holds columns 32 h + l.
 template <int B, bool FULL>
-__global__ void __launch_bounds__(32 * CdCfg<B>::WARPS) k_cd_block(const CdArgs a) {
+__device__ __forceinline__ bool cd_prologue(const CdArgs &a, float *tri, uint64_t *bar, int64_t i,
+                                            bool row_ok, int lane, float (&t)[B / 32], float (&st)[B / 32]) {
     using C = CdCfg<B>;
-    constexpr int CPL = C::CPL, NT = 32 * C::WARPS;
-    extern __shared__ __align__(16) float cd_smem[];
-    float *tri = cd_smem;                                  // packed Sigma_bar block
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    float *rec = cd_smem + C::PACK + warp * 2 * B;         // this warp's Delta' and code record
+    constexpr int CPL = C::CPL;
     const int bw = FULL ? B : a.bw;
     const int64_t b0 = a.b0;
-
-    {
-        const float4 *src = reinterpret_cast<const float4 *>(a.tri + (b0 / B) * C::PACK);
-        float4 *dst = reinterpret_cast<float4 *>(tri);
-        for (int e = tid; e < C::PACK / 4; e += NT) dst[e] = src[e];
+    if (threadIdx.x == 0) {
+        mbar_init(bar, 1);
+        fence_mbar_init();
     }
     __syncthreads();
-
-    const int64_t i = static_cast<int64_t>(blockIdx.x) * C::WARPS + warp;
-    if (i >= a.q) return;
-    const float s = a.scale[i], z = a.zero[i];
-
-    // t = R / s + z + sum of split partials (grid-step units); st = start value
-    float t[CPL], st[CPL];
+    if (threadIdx.x == 0) {
+        constexpr uint32_t bytes = C::PACK * 4;
+        mbar_arrive_expect_tx(bar, bytes);
+        bulk_load(tri, a.tri + (b0 / B) * C::PACK, bytes, bar);
+    }
+    const int64_t ii = row_ok ? i : 0;
+    const float s = a.scale[ii], z = a.zero[ii];
+    float r_[CPL], ps[CPL];
+    uint32_t cd_[CPL];
 #pragma unroll
     for (int h = 0; h < CPL; ++h) {
         const int l = 32 * h + lane;
-        t[h] = 0.0f;
-        st[h] = 0.0f;
-        if (FULL || l < bw) {
-            t[h] = __fdiv_rn(a.R[i * a.ldr + b0 + l], s) + z;
-            st[h] = a.first_sweep ? t[h] : static_cast<float>(a.codes[i * a.ldc + b0 + l]);
-        }
+        const bool ok = row_ok && (FULL || l < bw);
+        r_[h] = ok ? a.R[ii * a.ldr + b0 + l] : 0.0f;
+        cd_[h] = (ok && !a.first_sweep) ? a.codes[ii * a.ldc + b0 + l] : 0u;
+        ps[h] = 0.0f;
     }
-    for (int sp = 0; sp < a.nsplit; ++sp) {
-        const float *prow = a.part + sp * a.part_stride + i * a.ldpart;
+#pragma unroll
+    for (int sp = 0; sp < C::MAX_SPLITS; ++sp) {
+        if (sp >= a.nsplit) break;
+        const float *prow = a.part + sp * a.part_stride + ii * a.ldpart;
 #pragma unroll
         for (int h = 0; h < CPL; ++h)
-            if (FULL || 32 * h + lane < bw) t[h] += prow[32 * h + lane];
+            if (row_ok && (FULL || 32 * h + lane < bw)) ps[h] += prow[32 * h + lane];
     }
+#pragma unroll
+    for (int h = 0; h < CPL; ++h) {
+        const float t0 = __fdiv_rn(r_[h], s) + z;
+        st[h] = a.first_sweep ? t0 : static_cast<float>(cd_[h]);
+        t[h] = t0 + ps[h];
+    }
+    if (!mbar_wait_bounded(bar, 0u, nullptr)) {
+        if (lane == 0) set_error(a.err, ERR_TIMEOUT);
+        return false;
+    }
+    return true;
+}
 
-    // The chain: column j = 32 h + jj is decided by lane jj; its code and change
-    // Delta' (db, the same in every lane after the shuffle) are recorded, and db,
-    // times
-    // Sigma_bar[j][l], to every later column l.  Lanes whose column is already
-    // decided (l <= j) absorb harmless updates, so no lane test is needed; an
-    // unchanged column (db == 0, the common case once the codes settle) skips
-    // the updates altogether.
+// Common epilogue: codes, C - z (both skipped for unchanged columns when
+// skip_same) and the Delta' plane(s).
+template <int B, bool FULL>
+__device__ __forceinline__ void cd_epilogue(const CdArgs &a, int64_t i, int lane, const float (&code)[B / 32],
+                                            const float (&dlt)[B / 32], bool skip_same) {
+    constexpr int CPL = B / 32;
+    const int bw = FULL ? B : a.bw;
+    const float z = a.zero[i];
+#pragma unroll
+    for (int h = 0; h < CPL; ++h) {
+        const int l = 32 * h + lane;
+        if (!FULL && l >= bw) continue;
+        const int64_t col = a.b0 + l;
+        if (!skip_same || dlt[h] != 0.0f) {
+            a.codes[i * a.ldc + col] = static_cast<uint8_t>(code[h]);
+            a.qf[i * a.ldq + col] = __float2bfloat16_rn(code[h] - z);
+        }
+        const __nv_bfloat16 hi = __float2bfloat16_rn(dlt[h]);
+        a.dp[i * a.ldd + col] = hi;
+        if (a.first_sweep) {   // Delta' is not an integer in the first sweep: three planes
+            const float r1 = dlt[h] - __bfloat162float(hi);
+            const __nv_bfloat16 mid = __float2bfloat16_rn(r1);
+            a.dp[(a.dp_plane_rows + i) * a.ldd + col] = mid;
+            a.dp[(2 * a.dp_plane_rows + i) * a.ldd + col] = __float2bfloat16_rn(r1 - __bfloat162float(mid));
+        }
+    }
+}
+
+// Sequential in-block kernel (the first sweep, where every column changes).
+// One warp per row; column j = 32 h + jj is decided by lane jj, which keeps
+// its code and change Delta'; the change (db, the same in every lane after the
+// shuffle) times Sigma_bar[j][l] is added to every later column l.  Lanes whose
+// column is already decided (l <= j) absorb harmless updates, so no lane test
+// is needed; an unchanged column (db == 0) skips the updates.
+template <int B, bool FULL>
+__global__ void __launch_bounds__(1024) k_cd_block_seq(const CdArgs a) {
+    using C = CdCfg<B>;
+    constexpr int CPL = C::CPL;
+    extern __shared__ __align__(16) float cd_smem[];
+    float *tri = cd_smem;
+    uint64_t *bar = reinterpret_cast<uint64_t *>(cd_smem + C::PACK);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t i = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + warp;
+    const bool row_ok = i < a.q;
+    float t[CPL], st[CPL];
+    if (!cd_prologue<B, FULL>(a, tri, bar, i, row_ok, lane, t, st)) return;
+    if (!row_ok) return;
+    const int bw = FULL ? B : a.bw;
     const float maxq = a.maxq;
-    const bool writer = lane == 0;
+    float code[CPL], dlt[CPL];
+#pragma unroll
+    for (int h = 0; h < CPL; ++h) {
+        code[h] = 0.0f;
+        dlt[h] = 0.0f;
+    }
 #pragma unroll
     for (int h = 0; h < CPL; ++h) {
 #pragma unroll
@@ -260,12 +320,12 @@ __global__ void __launch_bounds__(32 * CdCfg<B>::WARPS) k_cd_block(const CdArgs 
             const int j = 32 * h + jj;
             if (!FULL && j >= bw) break;
             const float c = rintf(fminf(fmaxf(t[h], 0.0f), maxq));
-            const float db = __shfl_sync(0xffffffffu, st[h] - c, jj);
-            const float cb = __shfl_sync(0xffffffffu, c, jj);
-            if (writer) {
-                rec[j] = db;
-                rec[B + j] = cb;
+            const float dl = st[h] - c;
+            if (lane == jj) {
+                code[h] = c;
+                dlt[h] = dl;
             }
+            const float db = __shfl_sync(0xffffffffu, dl, jj);
             if (db != 0.0f) {
                 const float *row = tri + kPackPad + tri_off(B, j) - (j + 1);
 #pragma unroll
@@ -273,27 +333,106 @@ __global__ void __launch_bounds__(32 * CdCfg<B>::WARPS) k_cd_block(const CdArgs 
             }
         }
     }
-    __syncwarp();
+    cd_epilogue<B, FULL>(a, i, lane, code, dlt, false);
+}
 
-    // codes, C - z and the Delta' plane(s)
+// Change-driven in-block kernel (every sweep after the first), exactly
+// equivalent to the sequential order: a column whose code does not change
+// alters no other column, so all remaining columns are quantized at once, the
+// first one that changes is found by a warp ballot, its change is applied to
+// the columns after it, and the pass resumes right after it.  The cost is
+// (number of changed columns + 1) data-parallel passes.
+template <int B, bool FULL>
+__global__ void __launch_bounds__(1024) k_cd_block_chg(const CdArgs a) {
+    using C = CdCfg<B>;
+    constexpr int CPL = C::CPL;
+    extern __shared__ __align__(16) float cd_smem[];
+    float *tri = cd_smem;
+    uint64_t *bar = reinterpret_cast<uint64_t *>(cd_smem + C::PACK);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t i = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + warp;
+    const bool row_ok = i < a.q;
+    float t[CPL], st[CPL];
+    if (!cd_prologue<B, FULL>(a, tri, bar, i, row_ok, lane, t, st)) return;
+    if (!row_ok) return;
+    const int bw = FULL ? B : a.bw;
+    const float maxq = a.maxq;
+    float code[CPL], dlt[CPL];
 #pragma unroll
     for (int h = 0; h < CPL; ++h) {
-        const int l = 32 * h + lane;
-        if (!FULL && l >= bw) continue;
-        const float dl = rec[l];
-        const float code = rec[B + l];
-        const int64_t col = b0 + l;
-        a.codes[i * a.ldc + col] = static_cast<uint8_t>(code);
-        a.qf[i * a.ldq + col] = __float2bfloat16_rn(code - z);
-        const __nv_bfloat16 hi = __float2bfloat16_rn(dl);
-        a.dp[i * a.ldd + col] = hi;
-        if (a.first_sweep) {   // Delta' is not an integer in the first sweep: three planes
-            const float r1 = dl - __bfloat162float(hi);
-            const __nv_bfloat16 mid = __float2bfloat16_rn(r1);
-            a.dp[(a.dp_plane_rows + i) * a.ldd + col] = mid;
-            a.dp[(2 * a.dp_plane_rows + i) * a.ldd + col] = __float2bfloat16_rn(r1 - __bfloat162float(mid));
-        }
+        code[h] = st[h];
+        dlt[h] = 0.0f;
     }
+    int pos = 0;                                       // first column not yet final
+    while (pos < bw) {
+        int jstar = -1;
+#pragma unroll
+        for (int h = 0; h < CPL; ++h) {
+            const int l = 32 * h + lane;
+            const bool active = l >= pos && (FULL || l < bw);
+            const float c = rintf(fminf(fmaxf(t[h], 0.0f), maxq));
+            const float dl = st[h] - c;
+            if (active) {
+                code[h] = c;
+                dlt[h] = dl;
+            }
+            const unsigned m = __ballot_sync(0xffffffffu, active && dl != 0.0f);
+            if (jstar < 0 && m != 0u) jstar = 32 * h + (__ffs(m) - 1);
+        }
+        if (jstar < 0) break;
+        // the change of column jstar, from its lane
+        float v = dlt[0];
+#pragma unroll
+        for (int h = 1; h < CPL; ++h)
+            if (h == (jstar >> 5)) v = dlt[h];
+        const float db = __shfl_sync(0xffffffffu, v, jstar & 31);
+        const float *row = tri + kPackPad + tri_off(B, jstar) - (jstar + 1);
+#pragma unroll
+        for (int g = 0; g < CPL; ++g) t[g] = fmaf(db, row[32 * g + lane], t[g]);
+        pos = jstar + 1;
+    }
+    cd_epilogue<B, FULL>(a, i, lane, code, dlt, true);
+}
+
+template <int B, bool FULL, bool SEQ>
+static cudaError_t launch_cd_block_b(const CdArgs &a, int nsm, cudaStream_t s) {
+    using C = CdCfg<B>;
+    if (a.nsplit > C::MAX_SPLITS) return cudaErrorInvalidValue;
+    auto kern = SEQ ? k_cd_block_seq<B, FULL> : k_cd_block_chg<B, FULL>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+    if (e != cudaSuccess) return e;
+    // one CTA per SM when the rows allow it (the packed block is shared by the CTA's rows)
+    int64_t warps = ceil_div(a.q, nsm);
+    if (warps > C::MAX_WARPS) warps = C::MAX_WARPS;
+    if (warps < 1) warps = 1;
+    const unsigned grid = static_cast<unsigned>(ceil_div(a.q, warps));
+    kern<<<grid, static_cast<unsigned>(32 * warps), C::SMEM, s>>>(a);
+    return cudaGetLastError();
+}
+
+template <int B>
+static cudaError_t launch_cd_block_w(const CdArgs &a, int nsm, cudaStream_t s) {
+    const bool full = a.bw == B, seq = a.first_sweep != 0;
+    if (full) return seq ? launch_cd_block_b<B, true, true>(a, nsm, s) : launch_cd_block_b<B, true, false>(a, nsm, s);
+    return seq ? launch_cd_block_b<B, false, true>(a, nsm, s) : launch_cd_block_b<B, false, false>(a, nsm, s);
+}
+
+cudaError_t launch_cd_block(int B, const CdArgs &a, int nsm, cudaStream_t s) {
+    switch (B) {
+        case 64: return launch_cd_block_w<64>(a, nsm, s);
+        case 128: return launch_cd_block_w<128>(a, nsm, s);
+        case 256: return launch_cd_block_w<256>(a, nsm, s);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
+int64_t packed_diag_floats(int64_t p, int B) { return ceil_div(p, B) * packed_block_floats(B); }
+
+cudaError_t launch_pack_diag(const __nv_bfloat16 *snt, int64_t ldn, int64_t p, int B, float *out,
+                             cudaStream_t s) {
+    dim3 grid(static_cast<unsigned>(ceil_div(p, B)), static_cast<unsigned>(B));
+    k_pack_diag<<<grid, 128, 0, s>>>(snt, ldn, p, p, B, out);
+    return cudaGetLastError();
 }
 
 // ---------------------------------------------------------------------------
@@ -482,37 +621,15 @@ cudaError_t launch_codes_to_qf(const uint8_t *codes, int64_t ldc, const float *z
     return cudaGetLastError();
 }
 
-template <int B, bool FULL>
-static cudaError_t launch_cd_block_b(const CdArgs &a, cudaStream_t s) {
-    using C = CdCfg<B>;
-    cudaError_t e = cudaFuncSetAttribute(k_cd_block<B, FULL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         C::SMEM);
-    if (e != cudaSuccess) return e;
-    const unsigned grid = static_cast<unsigned>(ceil_div(a.q, C::WARPS));
-    k_cd_block<B, FULL><<<grid, 32 * C::WARPS, C::SMEM, s>>>(a);
-    return cudaGetLastError();
-}
 
-cudaError_t launch_cd_block(int B, const CdArgs &a, cudaStream_t s) {
-    const bool full = a.bw == B;
-    switch (B) {
-        case 64: return full ? launch_cd_block_b<64, true>(a, s) : launch_cd_block_b<64, false>(a, s);
-        case 128: return full ? launch_cd_block_b<128, true>(a, s) : launch_cd_block_b<128, false>(a, s);
-        case 256: return full ? launch_cd_block_b<256, true>(a, s) : launch_cd_block_b<256, false>(a, s);
-        default: return cudaErrorInvalidValue;
-    }
-}
 
-int64_t packed_diag_floats(int64_t p, int B) { return ceil_div(p, B) * packed_block_floats(B); }
-
-cudaError_t launch_pack_diag(const __nv_bfloat16 *snt, int64_t ldn, int64_t p, int B, float *out,
-                             cudaStream_t s) {
-    dim3 grid(static_cast<unsigned>(ceil_div(p, B)), static_cast<unsigned>(B));
-    k_pack_diag<<<grid, 128, 0, s>>>(snt, ldn, p, p, B, out);
-    return cudaGetLastError();
-}
 
 int objective_blocks(int64_t q) { return static_cast<int>(q < 1024 ? q : 1024); }
+
+cudaError_t launch_sum_partials(const double *partial, int n, double *out, cudaStream_t s) {
+    k_sum_partials<<<1, 256, 0, s>>>(partial, n, out);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_objective(const ObjArgs &a, double *partial, double *out, cudaStream_t s) {
     const int nb = objective_blocks(a.q);

@@ -55,8 +55,9 @@ __device__ __forceinline__ float load_w(const GemmArgs &g, int64_t r, int64_t c)
 }
 
 // Epilogue for one thread: output row r, columns [c0, c0 + 32) of the window.
+// `objacc` collects the fused objective terms of EPI_RFULL (when requested).
 __device__ __forceinline__ void epilogue_row(const GemmArgs &g, int r, int c0, const float (&v)[32],
-                                             int split) {
+                                             int split, double &objacc) {
     if (r >= g.M) return;
     const int64_t rr = r;
     switch (g.mode) {
@@ -91,23 +92,75 @@ __device__ __forceinline__ void epilogue_row(const GemmArgs &g, int r, int c0, c
             const float s = g.scale[r];
             const float *prow = g.P + rr * g.ldp;
             float *orow = g.out + rr * g.ldo;
-            if (c0 + 32 <= g.N && ((g.ldo | g.ldp) & 3) == 0) {
+            float o[32];
+            const bool full = c0 + 32 <= g.N;
+            if (full && ((g.ldo | g.ldp) & 3) == 0) {
 #pragma unroll
                 for (int i = 0; i < 32; i += 4) {
                     const float4 pv = *reinterpret_cast<const float4 *>(prow + c0 + i);
-                    float4 o;
-                    o.x = fmaf(-s, v[i + 0], pv.x);
-                    o.y = fmaf(-s, v[i + 1], pv.y);
-                    o.z = fmaf(-s, v[i + 2], pv.z);
-                    o.w = fmaf(-s, v[i + 3], pv.w);
-                    *reinterpret_cast<float4 *>(orow + c0 + i) = o;
+                    o[i] = fmaf(-s, v[i + 0], pv.x);
+                    o[i + 1] = fmaf(-s, v[i + 1], pv.y);
+                    o[i + 2] = fmaf(-s, v[i + 2], pv.z);
+                    o[i + 3] = fmaf(-s, v[i + 3], pv.w);
+                    *reinterpret_cast<float4 *>(orow + c0 + i) = make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]);
                 }
             } else {
 #pragma unroll
                 for (int i = 0; i < 32; ++i) {
                     const int c = c0 + i;
-                    if (c < g.N) orow[c] = fmaf(-s, v[i], prow[c]);
+                    o[i] = 0.0f;
+                    if (c < g.N) orow[c] = o[i] = fmaf(-s, v[i], prow[c]);
                 }
+            }
+            if (g.obj_part) {
+                // (D Sigma)_ij = d_j (R_ij - What_ij) with the new R: f = sum D_ij d_j (R_ij - What_ij)
+                const float z = g.zero[r];
+                float part = 0.0f;
+                const bool vec = full && g.w_is_bf16 && (g.ldw % 8) == 0 && (g.ldc % 16) == 0 && g.Hd == nullptr;
+                if (vec) {
+                    const uint4 *wp = reinterpret_cast<const uint4 *>(
+                        reinterpret_cast<const __nv_bfloat16 *>(g.W) + rr * g.ldw + c0);
+                    const uint4 *cp = reinterpret_cast<const uint4 *>(g.codes + rr * g.ldc + c0);
+                    const float4 *dp = reinterpret_cast<const float4 *>(g.dvec + c0);
+#pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        union { uint4 v; uint8_t b[16]; } cu;
+                        cu.v = cp[h];
+#pragma unroll
+                        for (int w8 = 0; w8 < 2; ++w8) {
+                            union { uint4 v; __nv_bfloat16 e[8]; } wu;
+                            wu.v = wp[2 * h + w8];
+#pragma unroll
+                            for (int q4 = 0; q4 < 2; ++q4) {
+                                const float4 d4 = dp[4 * h + 2 * w8 + q4];
+                                const float dd[4] = {d4.x, d4.y, d4.z, d4.w};
+#pragma unroll
+                                for (int e = 0; e < 4; ++e) {
+                                    const int i = 16 * h + 8 * w8 + 4 * q4 + e;
+                                    const float wh = s * (static_cast<float>(cu.b[i - 16 * h]) - z);
+                                    const float t = __bfloat162float(wu.e[4 * q4 + e]) - wh;
+                                    const float dj = dd[e] > 0.0f ? dd[e] : 0.0f;
+                                    part += t * dj * (o[i] - wh);
+                                }
+                            }
+                        }
+                    }
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) {
+                        const int c = c0 + i;
+                        if (c < g.N) {
+                            const float dj = g.dvec[c];
+                            if (dj > 0.0f) {
+                                const float wh = s * (static_cast<float>(g.codes[rr * g.ldc + c]) - z);
+                                float t = load_w(g, rr, c) - wh;
+                                if (g.Hd) t -= g.Hd[rr * g.ldh + c];
+                                part += t * dj * (o[i] - wh);
+                            }
+                        }
+                    }
+                }
+                objacc += static_cast<double>(part);
             }
             break;
         }
@@ -267,6 +320,7 @@ __global__ void __launch_bounds__(320, 1)
             tc_fence_before();
             mbar_arrive(&acc_empty[buf]);
         }
+        double objacc = 0.0;
         if (ok && *abort_flag == 0) {
             const int r = m0 + quad * 32 + lane;
 #pragma unroll
@@ -276,9 +330,15 @@ __global__ void __launch_bounds__(320, 1)
                     float v[32];
 #pragma unroll
                     for (int i = 0; i < 32; ++i) v[i] = acc[q * 32 + i];
-                    epilogue_row(g, r, c0, v, split);
+                    epilogue_row(g, r, c0, v, split, objacc);
                 }
             }
+        }
+        if (g.obj_part) {   // one fp64 partial per epilogue warp, reduced later in a fixed order
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) objacc += __shfl_xor_sync(0xffffffffu, objacc, o);
+            if (lane == 0)
+                g.obj_part[(static_cast<int64_t>(blockIdx.y) * gridDim.x + blockIdx.x) * 8 + (warp - 2)] = objacc;
         }
     }
     tc_fence_before();

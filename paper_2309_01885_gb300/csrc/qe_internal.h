@@ -34,6 +34,16 @@ struct GemmArgs {
     int w_is_bf16;
     int64_t ldw;
     int accumulate;           // EPI_SIGMA
+    // EPI_RFULL, optional fused objective f = sum D_ij d_j (R_ij - What_ij) with
+    // What = s (codes - z) and D = W - What (- H): one fp64 partial per epilogue
+    // warp and tile, at obj_part[(tile * 8) + warp - 2].
+    double *obj_part;
+    const uint8_t *codes;
+    int64_t ldc;
+    const float *zero;
+    const float *dvec;
+    const float *Hd;
+    int64_t ldh;
     unsigned *err;
 };
 

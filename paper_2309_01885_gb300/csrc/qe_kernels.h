@@ -27,6 +27,7 @@ struct CdArgs {
     int64_t ldq;
     __nv_bfloat16 *dp;              // out: Delta' hi plane (mid / lo planes dp_plane_rows apart)
     int64_t ldd, dp_plane_rows;
+    unsigned *err;
 };
 
 // Objective / reference-norm reduction.
@@ -54,11 +55,14 @@ cudaError_t launch_init_residual(const void *W, int w_bf16, int64_t ldw, const f
                                  int64_t q, int64_t p, float *R, int64_t ldr, cudaStream_t s);
 cudaError_t launch_codes_to_qf(const uint8_t *codes, int64_t ldc, const float *zero, int64_t q,
                                int64_t p, __nv_bfloat16 *qf, int64_t ldq, cudaStream_t s);
-cudaError_t launch_cd_block(int B, const CdArgs &a, cudaStream_t s);
+cudaError_t launch_cd_block(int B, const CdArgs &a, int nsm, cudaStream_t s);
 int64_t packed_diag_floats(int64_t p, int B);
 cudaError_t launch_pack_diag(const __nv_bfloat16 *snt, int64_t ldn, int64_t p, int B, float *out,
                              cudaStream_t s);
 int objective_blocks(int64_t q);
+// fp64 partials written by the residual GEMM's fused objective (8 per 128 x 256 tile)
+inline int64_t rfull_partials(int64_t q, int64_t p) { return ((q + 127) / 128) * ((p + 255) / 256) * 8; }
+cudaError_t launch_sum_partials(const double *partial, int n, double *out, cudaStream_t s);
 cudaError_t launch_objective(const ObjArgs &a, double *partial, double *out, cudaStream_t s);
 
 }  // namespace qe
