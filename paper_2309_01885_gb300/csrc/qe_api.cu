@@ -51,7 +51,8 @@ constexpr int kDefaultPowerIters = 64;
 struct Plan {
     int64_t q = 0, p = 0, ld = 0;
     int B = kDefaultBlock, smax = 1;
-    size_t snt = 0, d = 0, dinv = 0, tri = 0, P = 0, R = 0, wpl = 0, qf = 0, dp = 0, part = 0, objp = 0;
+    size_t snt = 0, d = 0, dinv = 0, tri = 0, P = 0, R = 0, wpl = 0, qf = 0, dp = 0, part = 0, objp = 0,
+           rowdf = 0, objbase = 0;
     size_t PW = 0, H = 0, T = 0, st = 0, cg = 0, ce = 0, sb = 0, eb = 0, y0 = 0, y1 = 0, lam = 0,
            eta = 0, rowptr = 0;
     size_t total = 0;
@@ -88,6 +89,8 @@ static Plan make_plan(int64_t q, int64_t p, int B, bool outlier, int wpl_planes,
     pl.part = take(cur, static_cast<size_t>(pl.smax) * q * B * 4);
     pl.objp = take(cur, static_cast<size_t>(rfull_partials(q, p) > objective_blocks(q) ? rfull_partials(q, p)
                                                                                     : objective_blocks(q)) * 8);
+    pl.rowdf = take(cur, static_cast<size_t>(q) * 8);
+    pl.objbase = take(cur, 8);
     if (outlier) {
         const int64_t N = q * p;
         const int64_t nch = topk_chunks(N);
@@ -119,7 +122,7 @@ struct Ctx {
     bool own = false;
     __nv_bfloat16 *snt = nullptr, *wpl = nullptr, *qf = nullptr, *dp = nullptr;
     float *d = nullptr, *dinv = nullptr, *tri = nullptr, *P = nullptr, *R = nullptr, *part = nullptr;
-    double *objp = nullptr;
+    double *objp = nullptr, *rowdf = nullptr, *objbase = nullptr;
     float *PW = nullptr, *H = nullptr, *T = nullptr, *y0 = nullptr, *y1 = nullptr;
     TopkState *st = nullptr;
     unsigned *cg = nullptr, *ce = nullptr, *sb = nullptr, *eb = nullptr;
@@ -168,6 +171,8 @@ static qe_status setup_ctx(Ctx &c, const Plan &pl, const qe_opts *o, cudaStream_
     c.dp = at<__nv_bfloat16>(w, pl.dp);
     c.part = at<float>(w, pl.part);
     c.objp = at<double>(w, pl.objp);
+    c.rowdf = at<double>(w, pl.rowdf);
+    c.objbase = at<double>(w, pl.objbase);
     if (pl.PW) {
         c.PW = at<float>(w, pl.PW);
         c.H = at<float>(w, pl.H);
@@ -297,15 +302,25 @@ static qe_status residual(Ctx &c, const float *scales, const ObjFuse *f = nullpt
 }
 
 // One cyclic sweep j = 1..p, blocked by B columns.
+//   classic (window == 0): block b gets the deferred correction
+//       Delta'[:, 0:b0] Sigma_bar[0:b0, block] on top of R (the sweep-start
+//       residual), which a residual GEMM refreshes after the sweep.
+//   rolling window (window > 0): R holds each block's value from its last
+//       visit; the correction covers the `window` most recent column changes
+//       (this sweep's for columns < b0, the previous sweep's for columns >= b0,
+//       all of them in dp), the staged values become the new base, and the
+//       objective changes of the decisions accumulate in rowdf.  window = -1
+//       means the first window sweep after a residual refresh: only columns < b0.
 static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float *zeros, int bits,
-                       bool first) {
+                       bool first, int window) {
     const int64_t q = c.pl.q, p = c.pl.p, ld = c.pl.ld;
     const int B = c.pl.B;
     for (int64_t b0 = 0; b0 < p; b0 += B) {
         const int bw = static_cast<int>((p - b0) < B ? (p - b0) : B);
+        const int64_t kcols = (window > 0) ? p : b0;
         int nsplit = 0;
-        if (b0 > 0) {
-            const int kb = static_cast<int>(b0 / 64);
+        if (kcols > 0) {
+            const int kb = static_cast<int>(ceil_div(kcols, 64));
             const int S = kb < c.pl.smax ? kb : c.pl.smax;
             GemmArgs g = gemm_args(c, static_cast<int>(q), bw, kb, EPI_TRAIL);
             set_prods(g, first ? 3 : 1);
@@ -327,6 +342,7 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
         a.bw = bw;
         a.R = c.R;
         a.ldr = ld;
+        a.store_base = window != 0 ? 1 : 0;
         a.part = c.part;
         a.nsplit = nsplit;
         a.part_stride = q * B;
@@ -334,8 +350,11 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
         a.tri = c.tri;
         a.scale = scales;
         a.zero = zeros;
+        a.d = c.d;
+        a.rowdf = window != 0 ? c.rowdf : nullptr;
         a.maxq = static_cast<float>((1 << bits) - 1);
         a.first_sweep = first ? 1 : 0;
+        a.write_qf = window != 0 ? 0 : 1;
         a.codes = codes;
         a.ldc = p;
         a.qf = c.qf;
@@ -534,18 +553,33 @@ qe_status qe_quantize_layer(const void *W, qe_dtype w_dtype, int64_t q, int64_t 
     if (opts && opts->wx_norm2)
         if ((st = objective(c, W, wbf16, ldw, nullptr, nullptr, nullptr, nullptr, c.P, opts->wx_norm2)) != QE_OK)
             return st;
+    // Sweep 1 starts at What = W (Sec. 3.1) and changes every coordinate by a
+    // real amount: the classic schedule with a residual refresh (which also
+    // yields obj[0]).  Later sweeps change few codes, by integers: the rolling
+    // window schedule with the objective updated decision by decision.
     const bool warm = opts && opts->init_codes;
+    const size_t plane0 = static_cast<size_t>(q) * pl.ld * 2;
+    int t0 = 0;
     if (warm) {
         QE_CK(cudaMemcpyAsync(codes, opts->init_codes, static_cast<size_t>(q) * p, cudaMemcpyDeviceToDevice, c.s));
         QE_CK(launch_codes_to_qf(codes, p, zeros, q, p, c.qf, pl.ld, c.s));
-        if ((st = residual(c, scales)) != QE_OK) return st;
-    } else {
-        QE_CK(launch_init_residual(W, wbf16, ldw, nullptr, 0, q, p, c.R, pl.ld, c.s));
-    }
-    for (int t = 0; t < iters; ++t) {
-        if ((st = sweep(c, codes, scales, zeros, bits, t == 0 && !warm)) != QE_OK) return st;
-        const ObjFuse f{obj + t, W, wbf16, ldw, codes, zeros, nullptr};
+        const ObjFuse f{c.objbase, W, wbf16, ldw, codes, zeros, nullptr};
         if ((st = residual(c, scales, &f)) != QE_OK) return st;
+    } else {
+        QE_CK(launch_init_residual(W, wbf16, ldw, nullptr, 0, q, p, scales, zeros, c.R, pl.ld, c.s));
+        if ((st = sweep(c, codes, scales, zeros, bits, true, 0)) != QE_OK) return st;
+        const ObjFuse f{obj, W, wbf16, ldw, codes, zeros, nullptr};
+        if ((st = residual(c, scales, &f)) != QE_OK) return st;
+        if (opts && opts->sweep_codes)
+            QE_CK(cudaMemcpyAsync(opts->sweep_codes, codes, static_cast<size_t>(q) * p, cudaMemcpyDeviceToDevice, c.s));
+        t0 = 1;
+    }
+    // the refreshed residual already holds every change so far: start the window empty
+    QE_CK(cudaMemsetAsync(c.dp, 0, plane0, c.s));
+    QE_CK(cudaMemsetAsync(c.rowdf, 0, static_cast<size_t>(q) * 8, c.s));
+    for (int t = t0; t < iters; ++t) {
+        if ((st = sweep(c, codes, scales, zeros, bits, false, t == t0 ? -1 : 1)) != QE_OK) return st;
+        QE_CK(launch_obj_step(c.rowdf, q, t == 0 ? c.objbase : obj + t - 1, obj + t, c.s));
         if (opts && opts->sweep_codes)
             QE_CK(cudaMemcpyAsync(opts->sweep_codes + static_cast<size_t>(t) * q * p, codes,
                                   static_cast<size_t>(q) * p, cudaMemcpyDeviceToDevice, c.s));
@@ -581,7 +615,8 @@ qe_status qe_quantize_layer_outlier(const void *W, qe_dtype w_dtype, int64_t q, 
     // P_W = W (I + Sigma_bar), eta = 1 / (2 lambda_max), P = P_W - H (I + Sigma_bar)
     if ((st = prepare(c, W, wbf16, ldw, Sigma, c.PW)) != QE_OK) return st;
     QE_CK(launch_power_lambda(Sigma, p, p, power_iters, c.y0, c.y1, c.lam, c.eta, c.nsm, c.s));
-    QE_CK(launch_spmm_refresh(c.PW, c.P, c.R, ld, Sigma, p, c.d, c.dinv, H_idx, H_val, c.rowptr, q, p, 0, c.s));
+    QE_CK(launch_spmm_refresh(c.PW, c.P, c.R, ld, Sigma, p, c.d, c.dinv, H_idx, H_val, c.rowptr, q, p, 0, scales,
+                              c.s));
     if (opts && opts->wx_norm2)
         if ((st = objective(c, W, wbf16, ldw, c.H, nullptr, nullptr, nullptr, c.P, opts->wx_norm2)) != QE_OK)
             return st;
@@ -591,10 +626,10 @@ qe_status qe_quantize_layer_outlier(const void *W, qe_dtype w_dtype, int64_t q, 
         QE_CK(launch_codes_to_qf(codes, p, zeros, q, p, c.qf, ld, c.s));
         if ((st = residual(c, scales)) != QE_OK) return st;
     } else {
-        QE_CK(launch_init_residual(W, wbf16, ldw, c.H, ld, q, p, c.R, ld, c.s));
+        QE_CK(launch_init_residual(W, wbf16, ldw, c.H, ld, q, p, scales, zeros, c.R, ld, c.s));
     }
     for (int t = 0; t < iters; ++t) {
-        if ((st = sweep(c, codes, scales, zeros, bits, t == 0 && !warm)) != QE_OK) return st;
+        if ((st = sweep(c, codes, scales, zeros, bits, t == 0 && !warm, 0)) != QE_OK) return st;
         const ObjFuse f{obj_cd ? obj_cd + t : nullptr, W, wbf16, ldw, codes, zeros, c.H};
         if ((st = residual(c, scales, obj_cd ? &f : nullptr)) != QE_OK) return st;
         // IHT step: T = H + 2 eta d (R - What); H = P_s(T)
@@ -603,7 +638,8 @@ qe_status qe_quantize_layer_outlier(const void *W, qe_dtype w_dtype, int64_t q, 
         QE_CK(cudaMemsetAsync(c.H, 0, static_cast<size_t>(q) * ld * 4, c.s));
         QE_CK(launch_scatter_rowptr(H_idx, H_val, H_nnz, s_budget, q, p, c.H, ld, c.rowptr, c.s));
         // P = P_W - H (I + Sigma_bar); R += P_new - P_old  (R = P - What Sigma_bar stays current)
-        QE_CK(launch_spmm_refresh(c.PW, c.P, c.R, ld, Sigma, p, c.d, c.dinv, H_idx, H_val, c.rowptr, q, p, 1, c.s));
+        QE_CK(launch_spmm_refresh(c.PW, c.P, c.R, ld, Sigma, p, c.d, c.dinv, H_idx, H_val, c.rowptr, q, p, 1, scales,
+                                  c.s));
         if ((st = objective(c, W, wbf16, ldw, c.H, codes, scales, zeros, c.R, obj + t)) != QE_OK) return st;
         if (opts && opts->sweep_codes)
             QE_CK(cudaMemcpyAsync(opts->sweep_codes + static_cast<size_t>(t) * q * p, codes,

@@ -127,17 +127,39 @@ __global__ void k_make_planes(const void *W, int w_bf16, int64_t ldw, int64_t q,
     }
 }
 
-// R = W - H (fp32), the residual at the start of the first sweep: with
-// What = W - H, P - What Sigma_bar = (W - H)(I + Sigma_bar) - (W - H) Sigma_bar.
+// The residual at the start of the first sweep, in grid-step units: with
+// What = W - H, P - What Sigma_bar = (W - H)(I + Sigma_bar) - (W - H) Sigma_bar
+// = W - H, stored as (W - H) / s + z.
 __global__ void k_init_residual(const void *W, int w_bf16, int64_t ldw, const float *H, int64_t ldh,
-                                int64_t q, int64_t p, float *R, int64_t ldr) {
+                                int64_t q, int64_t p, const float *scale, const float *zero, float *R,
+                                int64_t ldr) {
     for (int64_t i = blockIdx.y; i < q; i += gridDim.y) {
+        const float s = scale[i], z = zero[i];
         for (int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; j < p;
              j += (int64_t)gridDim.x * blockDim.x) {
             float w = load_elem(W, w_bf16, i * ldw + j);
             if (H) w -= H[i * ldh + j];
-            R[i * ldr + j] = w;
+            R[i * ldr + j] = __fdiv_rn(w, s) + z;
         }
+    }
+}
+
+// obj_out = obj_prev + sum_i rowdf[i] (fixed order); rowdf is cleared.
+__global__ void k_obj_step(double *rowdf, int64_t q, const double *prev, double *out) {
+    __shared__ double sw[32];
+    double acc = 0.0;
+    for (int64_t k = threadIdx.x; k < q; k += blockDim.x) {
+        acc += rowdf[k];
+        rowdf[k] = 0.0;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if ((threadIdx.x & 31) == 0) sw[threadIdx.x >> 5] = acc;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double t = prev ? *prev : 0.0;
+        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += sw[w];
+        *out = t;
     }
 }
 
@@ -205,9 +227,10 @@ struct CdCfg {
 };
 
 // Common prologue of both in-block kernels: start the bulk copy of the packed
-// block, stage the row (t = R / s + z + sum of split partials, in grid steps;
-// st = start value: t before the partials in the first sweep, else the old
-// code), then wait for the block.  Lane l holds columns 32 h + l.
+// block, stage the row (t = R + sum of split partials, R already in grid-step
+// units; st = start value: R itself in the first sweep, else the old code),
+// optionally store t back as the block's new base (rolling window), then wait
+// for the block.  Lane l holds columns 32 h + l.
 template <int B, bool FULL>
 __device__ __forceinline__ bool cd_prologue(const CdArgs &a, float *tri, uint64_t *bar, int64_t i,
                                             bool row_ok, int lane, float (&t)[B / 32], float (&st)[B / 32]) {
@@ -226,7 +249,6 @@ __device__ __forceinline__ bool cd_prologue(const CdArgs &a, float *tri, uint64_
         bulk_load(tri, a.tri + (b0 / B) * C::PACK, bytes, bar);
     }
     const int64_t ii = row_ok ? i : 0;
-    const float s = a.scale[ii], z = a.zero[ii];
     float r_[CPL], ps[CPL];
     uint32_t cd_[CPL];
 #pragma unroll
@@ -247,9 +269,15 @@ __device__ __forceinline__ bool cd_prologue(const CdArgs &a, float *tri, uint64_
     }
 #pragma unroll
     for (int h = 0; h < CPL; ++h) {
-        const float t0 = __fdiv_rn(r_[h], s) + z;
-        st[h] = a.first_sweep ? t0 : static_cast<float>(cd_[h]);
-        t[h] = t0 + ps[h];
+        st[h] = a.first_sweep ? r_[h] : static_cast<float>(cd_[h]);
+        t[h] = r_[h] + ps[h];
+    }
+    if (a.store_base && a.nsplit > 0) {
+#pragma unroll
+        for (int h = 0; h < CPL; ++h) {
+            const int l = 32 * h + lane;
+            if (row_ok && (FULL || l < bw)) a.R[ii * a.ldr + b0 + l] = t[h];
+        }
     }
     if (!mbar_wait_bounded(bar, 0u, nullptr)) {
         if (lane == 0) set_error(a.err, ERR_TIMEOUT);
@@ -273,7 +301,7 @@ __device__ __forceinline__ void cd_epilogue(const CdArgs &a, int64_t i, int lane
         const int64_t col = a.b0 + l;
         if (!skip_same || dlt[h] != 0.0f) {
             a.codes[i * a.ldc + col] = static_cast<uint8_t>(code[h]);
-            a.qf[i * a.ldq + col] = __float2bfloat16_rn(code[h] - z);
+            if (a.write_qf) a.qf[i * a.ldq + col] = __float2bfloat16_rn(code[h] - z);
         }
         const __nv_bfloat16 hi = __float2bfloat16_rn(dlt[h]);
         a.dp[i * a.ldd + col] = hi;
@@ -363,6 +391,11 @@ __global__ void __launch_bounds__(1024) k_cd_block_chg(const CdArgs a) {
         code[h] = st[h];
         dlt[h] = 0.0f;
     }
+    // objective change of the decisions (Lemma 1: f(u) = Sigma_jj (u - beta)^2 + const
+    // along one coordinate), in units where u = s (code - z) and beta = s (t - z)
+    const float s = a.scale[i];
+    const float s2 = s * s;
+    double dfacc = 0.0;
     int pos = 0;                                       // first column not yet final
     while (pos < bw) {
         int jstar = -1;
@@ -381,15 +414,32 @@ __global__ void __launch_bounds__(1024) k_cd_block_chg(const CdArgs a) {
         }
         if (jstar < 0) break;
         // the change of column jstar, from its lane
-        float v = dlt[0];
+        float v = dlt[0], tv = t[0], cv = code[0], sv = st[0];
 #pragma unroll
         for (int h = 1; h < CPL; ++h)
-            if (h == (jstar >> 5)) v = dlt[h];
+            if (h == (jstar >> 5)) {
+                v = dlt[h];
+                tv = t[h];
+                cv = code[h];
+                sv = st[h];
+            }
+        if (a.rowdf && lane == (jstar & 31)) {
+            const float dj = a.d[a.b0 + jstar];
+            if (dj > 0.0f) {
+                const float e1 = cv - tv, e0 = sv - tv;
+                dfacc += static_cast<double>(dj * s2 * (e1 * e1 - e0 * e0));
+            }
+        }
         const float db = __shfl_sync(0xffffffffu, v, jstar & 31);
         const float *row = tri + kPackPad + tri_off(B, jstar) - (jstar + 1);
 #pragma unroll
         for (int g = 0; g < CPL; ++g) t[g] = fmaf(db, row[32 * g + lane], t[g]);
         pos = jstar + 1;
+    }
+    if (a.rowdf) {
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) dfacc += __shfl_xor_sync(0xffffffffu, dfacc, o);
+        if (lane == 0) a.rowdf[i] += dfacc;
     }
     cd_epilogue<B, FULL>(a, i, lane, code, dlt, true);
 }
@@ -454,9 +504,10 @@ __global__ void __launch_bounds__(256) k_objective(const ObjArgs a, double *part
             if (a.H) t -= a.H[i * a.ldh + j];
             const float r = a.R[i * a.ldr + j];
             float term;
-            if (a.codes) {
-                const float wh = s * (static_cast<float>(a.codes[i * a.ldc + j]) - z);
-                term = (t - wh) * dj * (r - wh);
+            if (a.codes) {   // R in grid-step units: R_abs - What = s (R - code)
+                const float cj = static_cast<float>(a.codes[i * a.ldc + j]);
+                const float wh = s * (cj - z);
+                term = (t - wh) * dj * (s * (r - cj));
             } else {
                 term = t * dj * r;
             }
@@ -610,8 +661,14 @@ cudaError_t launch_make_planes(const void *W, int w_bf16, int64_t ldw, int64_t q
 }
 
 cudaError_t launch_init_residual(const void *W, int w_bf16, int64_t ldw, const float *H, int64_t ldh,
-                                 int64_t q, int64_t p, float *R, int64_t ldr, cudaStream_t s) {
-    k_init_residual<<<row_grid(q, p), 256, 0, s>>>(W, w_bf16, ldw, H, ldh, q, p, R, ldr);
+                                 int64_t q, int64_t p, const float *scale, const float *zero, float *R,
+                                 int64_t ldr, cudaStream_t s) {
+    k_init_residual<<<row_grid(q, p), 256, 0, s>>>(W, w_bf16, ldw, H, ldh, q, p, scale, zero, R, ldr);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_obj_step(double *rowdf, int64_t q, const double *prev, double *out, cudaStream_t s) {
+    k_obj_step<<<1, 1024, 0, s>>>(rowdf, q, prev, out);
     return cudaGetLastError();
 }
 

@@ -4,7 +4,7 @@
 // method, selected by the epilogue:
 //   Sigma = X X^T                         (Lemma 1; upper tiles + mirror)
 //   P = W (I + Sigma_bar)                 (Algorithm 3, "P = W Sigma^norm")
-//   R = P - s (C - z) Sigma_bar           (Algorithm 3, "P_hat = What Sigma^norm")
+//   R = (P - s (C - z) Sigma_bar) / s + z  (Algorithm 3, "P_hat = What Sigma^norm"), grid steps
 //   partial_k = Delta' Sigma_bar[0:b0, block]  (Eq. cd-update-closed-2, the
 //                                          dW_{:,1:j} Sigma^norm_{1:j,j} term,
 //                                          deferred per column block, split-K)
@@ -89,7 +89,9 @@ __device__ __forceinline__ void epilogue_row(const GemmArgs &g, int r, int c0, c
             break;
         }
         case EPI_RFULL: {
+            // R in grid-step units: (P - s (C - z) Sigma_bar) / s + z = P / s - acc + z
             const float s = g.scale[r];
+            const float zz = g.zero[r];
             const float *prow = g.P + rr * g.ldp;
             float *orow = g.out + rr * g.ldo;
             float o[32];
@@ -98,10 +100,10 @@ __device__ __forceinline__ void epilogue_row(const GemmArgs &g, int r, int c0, c
 #pragma unroll
                 for (int i = 0; i < 32; i += 4) {
                     const float4 pv = *reinterpret_cast<const float4 *>(prow + c0 + i);
-                    o[i] = fmaf(-s, v[i + 0], pv.x);
-                    o[i + 1] = fmaf(-s, v[i + 1], pv.y);
-                    o[i + 2] = fmaf(-s, v[i + 2], pv.z);
-                    o[i + 3] = fmaf(-s, v[i + 3], pv.w);
+                    o[i] = (__fdiv_rn(pv.x, s) - v[i + 0]) + zz;
+                    o[i + 1] = (__fdiv_rn(pv.y, s) - v[i + 1]) + zz;
+                    o[i + 2] = (__fdiv_rn(pv.z, s) - v[i + 2]) + zz;
+                    o[i + 3] = (__fdiv_rn(pv.w, s) - v[i + 3]) + zz;
                     *reinterpret_cast<float4 *>(orow + c0 + i) = make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]);
                 }
             } else {
@@ -109,12 +111,13 @@ __device__ __forceinline__ void epilogue_row(const GemmArgs &g, int r, int c0, c
                 for (int i = 0; i < 32; ++i) {
                     const int c = c0 + i;
                     o[i] = 0.0f;
-                    if (c < g.N) orow[c] = o[i] = fmaf(-s, v[i], prow[c]);
+                    if (c < g.N) orow[c] = o[i] = (__fdiv_rn(prow[c], s) - v[i]) + zz;
                 }
             }
             if (g.obj_part) {
-                // (D Sigma)_ij = d_j (R_ij - What_ij) with the new R: f = sum D_ij d_j (R_ij - What_ij)
-                const float z = g.zero[r];
+                // (D Sigma)_ij = d_j (R_ij - What_ij) = d_j s (R'_ij - C_ij) with R' = R / s + z:
+                // f = sum D_ij d_j s (R'_ij - C_ij)
+                const float z = zz;
                 float part = 0.0f;
                 const bool vec = full && g.w_is_bf16 && (g.ldw % 8) == 0 && (g.ldc % 16) == 0 && g.Hd == nullptr;
                 if (vec) {
@@ -137,10 +140,11 @@ __device__ __forceinline__ void epilogue_row(const GemmArgs &g, int r, int c0, c
 #pragma unroll
                                 for (int e = 0; e < 4; ++e) {
                                     const int i = 16 * h + 8 * w8 + 4 * q4 + e;
-                                    const float wh = s * (static_cast<float>(cu.b[i - 16 * h]) - z);
+                                    const float cj = static_cast<float>(cu.b[i - 16 * h]);
+                                    const float wh = s * (cj - z);
                                     const float t = __bfloat162float(wu.e[4 * q4 + e]) - wh;
                                     const float dj = dd[e] > 0.0f ? dd[e] : 0.0f;
-                                    part += t * dj * (o[i] - wh);
+                                    part += t * dj * (s * (o[i] - cj));
                                 }
                             }
                         }
@@ -152,10 +156,11 @@ __device__ __forceinline__ void epilogue_row(const GemmArgs &g, int r, int c0, c
                         if (c < g.N) {
                             const float dj = g.dvec[c];
                             if (dj > 0.0f) {
-                                const float wh = s * (static_cast<float>(g.codes[rr * g.ldc + c]) - z);
+                                const float cj = static_cast<float>(g.codes[rr * g.ldc + c]);
+                                const float wh = s * (cj - z);
                                 float t = load_w(g, rr, c) - wh;
                                 if (g.Hd) t -= g.Hd[rr * g.ldh + c];
-                                part += t * dj * (o[i] - wh);
+                                part += t * dj * (s * (o[i] - cj));
                             }
                         }
                     }

@@ -12,7 +12,7 @@ namespace qe {
 enum EpiMode : int {
     EPI_SIGMA = 0,  // out[r][c] (=|+=) D, only c >= r, mirrored to out[c][r]
     EPI_PINIT = 1,  // out[r][c] = W[r][c] + D            (P = W (I + Sigma_bar))
-    EPI_RFULL = 2,  // out[r][c] = P[r][c] - scale[r] * D (R = P - What Sigma_bar)
+    EPI_RFULL = 2,  // out[r][c] = P[r][c] / s_r - D + z_r  (R = P - What Sigma_bar in grid steps)
     EPI_TRAIL = 3   // out[split][r][c] = D               (split-K partial sums)
 };
 

@@ -12,15 +12,19 @@ struct CdArgs {
     int64_t q, p;
     int64_t b0;
     int bw;
-    const float *R;                 // residual P - What_start Sigma_bar (q x ldr)
+    float *R;                       // residual in grid-step units: (P - What Sigma_bar) / s + z
     int64_t ldr;
+    int store_base;                 // write the staged block values back to R (rolling window)
     const float *part;              // split-K partials [nsplit][q][ldpart] (t-units)
     int nsplit;
     int64_t part_stride, ldpart;
     const float *tri;               // packed diagonal blocks of Sigma_bar (launch_pack_diag)
     const float *scale, *zero;
+    const float *d;                 // Sigma_jj (objective change of each decision)
+    double *rowdf;                  // per-row objective change accumulator, or NULL
     float maxq;
     int first_sweep;                // What_start is R itself (not on the grid)
+    int write_qf;                   // also write C - z (needed by the residual GEMM)
     uint8_t *codes;                 // in: codes at sweep start (unless first_sweep); out: new codes
     int64_t ldc;
     __nv_bfloat16 *qf;              // out: C - z
@@ -52,7 +56,10 @@ cudaError_t launch_sigma_norm(const float *S, int64_t lds, int64_t p, float *d, 
 cudaError_t launch_make_planes(const void *W, int w_bf16, int64_t ldw, int64_t q, int64_t p,
                                int split, __nv_bfloat16 *out, int64_t ldo, cudaStream_t s);
 cudaError_t launch_init_residual(const void *W, int w_bf16, int64_t ldw, const float *H, int64_t ldh,
-                                 int64_t q, int64_t p, float *R, int64_t ldr, cudaStream_t s);
+                                 int64_t q, int64_t p, const float *scale, const float *zero, float *R,
+                                 int64_t ldr, cudaStream_t s);
+// obj[out] = obj[prev] + sum_i rowdf[i]; rowdf is zeroed.  prev may be NULL (0).
+cudaError_t launch_obj_step(double *rowdf, int64_t q, const double *prev, double *out, cudaStream_t s);
 cudaError_t launch_codes_to_qf(const uint8_t *codes, int64_t ldc, const float *zero, int64_t q,
                                int64_t p, __nv_bfloat16 *qf, int64_t ldq, cudaStream_t s);
 cudaError_t launch_cd_block(int B, const CdArgs &a, int nsm, cudaStream_t s);

@@ -98,12 +98,13 @@ __global__ void k_iht_target(const float *H, const float *R, int64_t ld, const u
                              const double *eta, int64_t q, int64_t p, float *T) {
     for (int64_t i = blockIdx.y; i < q; i += gridDim.y) {
         const float e2 = static_cast<float>(2.0 * (*eta));
-        const float s = scale[i], z = zero[i];
+        const float s = scale[i];
         for (int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; j < p;
              j += (int64_t)gridDim.x * blockDim.x) {
             const float dj = d[j] > 0.0f ? d[j] : 0.0f;
-            const float wh = s * (static_cast<float>(codes[i * ldc + j]) - z);
-            T[i * p + j] = H[i * ld + j] + e2 * dj * (R[i * ld + j] - wh);
+            // R in grid-step units: R_abs - What = s (R - code)
+            const float cj = static_cast<float>(codes[i * ldc + j]);
+            T[i * p + j] = H[i * ld + j] + e2 * dj * (s * (R[i * ld + j] - cj));
         }
     }
 }
@@ -291,13 +292,15 @@ __global__ void k_rowptr(const int64_t *H_idx, const int64_t *nnz, int64_t q, in
 }
 
 // P_new = P_W - H (I + Sigma_bar) for row i (Sigma_bar_kj = Sigma_kj / d_j off
-// the diagonal, 0 for dead columns); R += P_new - P_old when update_r; P = P_new.
+// the diagonal, 0 for dead columns); R += (P_new - P_old) / s_i when update_r
+// (R in grid-step units); P = P_new.
 __global__ void __launch_bounds__(256) k_spmm_refresh(const float *PW, float *P, float *R, int64_t ld,
                                                       const float *S, int64_t lds, const float *d,
                                                       const float *dinv, const int64_t *H_idx,
                                                       const float *H_val, const int64_t *rowptr,
-                                                      int64_t p, int update_r) {
+                                                      int64_t p, int update_r, const float *scale) {
     const int64_t i = blockIdx.x;
+    const float s = update_r ? scale[i] : 1.0f;
     const int64_t e0 = rowptr[i], e1 = rowptr[i + 1];
     for (int64_t j = threadIdx.x; j < p; j += blockDim.x) {
         float acc = PW[i * ld + j];
@@ -311,7 +314,7 @@ __global__ void __launch_bounds__(256) k_spmm_refresh(const float *PW, float *P,
             else sb = (dj > 0.0f && d[k] > 0.0f) ? S[k * lds + j] * ij : 0.0f;
             acc = fmaf(-v, sb, acc);
         }
-        if (update_r) R[i * ld + j] += acc - P[i * ld + j];
+        if (update_r) R[i * ld + j] += __fdiv_rn(acc - P[i * ld + j], s);
         P[i * ld + j] = acc;
     }
 }
@@ -397,9 +400,9 @@ cudaError_t launch_scatter_rowptr(const int64_t *H_idx, const float *H_val, cons
 cudaError_t launch_spmm_refresh(const float *PW, float *P, float *R, int64_t ld, const float *S,
                                 int64_t lds, const float *d, const float *dinv, const int64_t *H_idx,
                                 const float *H_val, const int64_t *rowptr, int64_t q, int64_t p,
-                                int update_r, cudaStream_t s) {
+                                int update_r, const float *scale, cudaStream_t s) {
     k_spmm_refresh<<<static_cast<unsigned>(q), 256, 0, s>>>(PW, P, R, ld, S, lds, d, dinv, H_idx, H_val,
-                                                            rowptr, p, update_r);
+                                                            rowptr, p, update_r, scale);
     return cudaGetLastError();
 }
 

@@ -35,7 +35,7 @@ cudaError_t launch_scatter_rowptr(const int64_t *H_idx, const float *H_val, cons
 cudaError_t launch_spmm_refresh(const float *PW, float *P, float *R, int64_t ld, const float *S,
                                 int64_t lds, const float *d, const float *dinv, const int64_t *H_idx,
                                 const float *H_val, const int64_t *rowptr, int64_t q, int64_t p,
-                                int update_r, cudaStream_t s);
+                                int update_r, const float *scale, cudaStream_t s);
 cudaError_t launch_dinv(const float *d, int64_t p, float *dinv, cudaStream_t s);
 
 }  // namespace qe
