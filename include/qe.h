@@ -137,6 +137,35 @@ qe_status qe_quantize_layer_outlier(const void *W, qe_dtype w_dtype, int64_t q,
                                     int64_t *H_idx, int64_t *H_nnz, double *obj,
                                     double *obj_cd, qe_stream_t stream);
 
+/*
+ * Sigma = X X^T like qe_build_sigma, but the call never allocates device
+ * memory.  (The paper has no counterpart: this is a deployment variant.)
+ *
+ * For callers that cannot let a library allocate: processes whose device
+ * memory is handed out entirely by their own allocator, latency-critical
+ * loops that must stay off the allocator, and platforms without
+ * stream-ordered allocation.  Where qe_build_sigma allocates a staging buffer
+ * (bf16 X that is token-major, or feature-major with an unaligned base or a
+ * leading dimension that is not a multiple of 8), this entry point stages
+ * through a fixed array of QE_STATIC_SCRATCH_BYTES that belongs to the
+ * library's device image: every GPU that loads the library holds it until the
+ * process exits.  Other inputs need no staging and run as in qe_build_sigma.
+ *
+ *   Arguments, layouts and the result are those of qe_build_sigma.
+ *   Limit: a staged X needs p <= QE_STATIC_SCRATCH_BYTES / 128 (= 65536 for
+ *   8 MiB); larger p returns QE_ERR_INVALID_ARG before anything is enqueued.
+ *   First call per device: looks up the array's device address (with that
+ *   device current) and caches it; make that first call before any stream
+ *   capture.
+ *   Every call shares the array: calls that overlap on the GPU (other streams,
+ *   other host threads) race.  Each call clears the part of the array it relies
+ *   on being zero.
+ */
+#define QE_STATIC_SCRATCH_BYTES (8u << 20)
+qe_status qe_build_sigma_static(const void *X, qe_dtype x_dtype, qe_xlayout layout,
+                                int64_t p, int64_t n, int64_t ldx, float *Sigma,
+                                int accumulate, qe_stream_t stream);
+
 /* Bytes of scratch qe_quantize_layer (outlier = 0) or qe_quantize_layer_outlier
  * (outlier = 1) needs for this shape and options; written to *bytes. */
 qe_status qe_workspace_size(int64_t q, int64_t p, int outlier, const qe_opts *opts,

@@ -36,6 +36,8 @@ static unsigned *error_word() {
     return cache[dev];
 }
 
+unsigned *device_error_word() { return error_word(); }
+
 static int sm_count() {
     int dev = 0, n = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return 148;

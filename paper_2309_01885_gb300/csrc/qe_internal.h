@@ -47,6 +47,9 @@ struct GemmArgs {
     unsigned *err;
 };
 
+// The per-device error word that qe_sync_status reads and clears.
+unsigned *device_error_word();
+
 // Builds a 2-D bf16 tensor map (rows x cols, leading dimension ld elements) with
 // a box of 64 columns x box_rows rows and 128-byte swizzle.  false on failure.
 bool make_tmap_bf16(CUtensorMap *map, const void *base, uint64_t rows, uint64_t cols,

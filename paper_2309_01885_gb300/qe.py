@@ -21,7 +21,8 @@ QE_F32, QE_BF16 = 0, 1
 QE_FEATURE_MAJOR, QE_TOKEN_MAJOR = 0, 1
 
 EXPORTED = ("qe_build_sigma", "qe_quantize_layer", "qe_quantize_layer_outlier",
-            "qe_workspace_size", "qe_sync_status", "qe_status_string", "qe_version")
+            "qe_workspace_size", "qe_sync_status", "qe_status_string", "qe_version",
+            "qe_build_sigma_static")
 
 
 class QEError(RuntimeError):
@@ -70,6 +71,8 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     L.qe_status_string.restype = ctypes.c_char_p
     L.qe_version.argtypes = []
     L.qe_version.restype = ctypes.c_int
+    L.qe_build_sigma_static.argtypes = [vp, i32, i32, i64, i64, i64, vp, i32, vp]
+    L.qe_build_sigma_static.restype = st
     _lib = L
     return L
 
@@ -130,6 +133,20 @@ def qe_build_sigma(X: torch.Tensor, layout: int = QE_FEATURE_MAJOR, Sigma: torch
         Sigma = torch.empty(p, p, dtype=torch.float32, device=X.device)
     _check(load().qe_build_sigma(_ptr(X), _dtype(X), layout, p, n, ld, _ptr(Sigma), int(accumulate),
                                  _stream(stream)), "qe_build_sigma")
+    return Sigma
+
+
+def qe_build_sigma_static(X: torch.Tensor, layout: int = QE_FEATURE_MAJOR, Sigma: torch.Tensor | None = None,
+                          accumulate: bool = False, stream=None) -> torch.Tensor:
+    """As qe_build_sigma, but the library call allocates no device memory: staged
+    inputs go through the library's fixed scratch array (see include/qe.h).  The
+    output tensor, when not given, is still allocated here by torch."""
+    ld = _rowmajor_ld(X)
+    p, n = (X.shape[0], X.shape[1]) if layout == QE_FEATURE_MAJOR else (X.shape[1], X.shape[0])
+    if Sigma is None:
+        Sigma = torch.empty(p, p, dtype=torch.float32, device=X.device)
+    _check(load().qe_build_sigma_static(_ptr(X), _dtype(X), layout, p, n, ld, _ptr(Sigma), int(accumulate),
+                                        _stream(stream)), "qe_build_sigma_static")
     return Sigma
 
 
