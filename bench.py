@@ -44,6 +44,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-rows", type=int, default=4096, help="oracle rows in the CPU sample")
+    ap.add_argument("--tokens", type=int, default=0,
+                    help="override n (calibration tokens), for small profiling captures only")
     return ap.parse_args()
 
 
@@ -114,6 +116,43 @@ class ClockSampler:
             return None
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": smax, "reasons": sorted(reasons),
                 "samples": len(sm)}
+
+
+def traffic_per_launch(kernel: str):
+    """DRAM bytes per launch of `kernel` from the committed ncu summary, if the
+    kernel sources are unchanged since it was taken (else None)."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", "roofline_traffic.json")
+    try:
+        with open(path) as fh:
+            rec = json.load(fh)
+    except (OSError, ValueError):
+        return None
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2309_01885_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, name), "rb") as fh:
+            h.update(name.encode() + b"\0" + fh.read())
+    entry = rec.get(kernel)
+    if not entry or entry.get("csrc_sha256") != h.hexdigest():
+        return None
+    return entry.get("dram_bytes_per_launch")
+
+
+def roofline_entry(launches, total_ms, total_flops, expected_launches, pk):
+    """The dominant kernel (per-block trailing GEMM) against the bf16 tensor roofline.
+    achieved = algorithmic flops (2 per deferred column update) / measured time; the
+    kernel executes 3 bf16 MMAs per product (hi/mid/lo planes of Sigma_bar)."""
+    if launches == 0 or total_ms <= 0:
+        return None
+    achieved = total_flops * (launches / expected_launches) / (total_ms / 1e3) / 1e12
+    return {"bound": "tensor", "kernel": "k_tc_gemm<256> trailing block correction",
+            "achieved": achieved, "peak": pk["bf16_sustained"], "unit": "TFLOP/s",
+            "frac": achieved / pk["bf16_sustained"],
+            "traffic": traffic_per_launch("trail_gemm"),
+            "launches_timed": launches, "avg_launch_us": 1e3 * total_ms / launches,
+            "executed_tflops": 3 * achieved, "split_products": 3,
+            "peak_source": f"{pk['source']} bf16 dense sustained (MEASURED_PEAKS.json)"}
 
 
 def cpu_oracle_sample(W64, S64, bits, rows, sweeps):
@@ -197,6 +236,9 @@ def main():
     qe.load()
 
     cfg = inputs.CONFIGS[args.config]
+    if args.tokens:
+        import dataclasses
+        cfg = dataclasses.replace(cfg, n=args.tokens)
     q, p, n = cfg.q, cfg.p, cfg.n
     seed = cfg.seed + rank                        # each rank owns a different layer
     W = inputs.layer_weights(q, p, dtype=cfg.w_dtype, seed=seed, device="cuda")
@@ -209,7 +251,7 @@ def main():
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(nb + 2)]
           for _ in range(args.steps)]
 
-    def step(events=None):
+    def step(events=None, timer=None):
         if events:
             events[0].record(stream)
         qe.qe_build_sigma(X, Sigma=Sigma)
@@ -217,7 +259,7 @@ def main():
             events[1].record(stream)
         outs = []
         for k, b in enumerate(cfg.bits):
-            outs.append(qe.qe_quantize_layer(W, Sigma, b, cfg.iters, workspace=ws))
+            outs.append(qe.qe_quantize_layer(W, Sigma, b, cfg.iters, workspace=ws, timer=timer))
             if events:
                 events[2 + k].record(stream)
         return outs
@@ -235,10 +277,14 @@ def main():
         dist.barrier()
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
+    # the dominant kernel (the per-block trailing GEMM) is timed by CUDA events that the
+    # library records around each of its launches on this stream
+    nblk = (p + 255) // 256                    # default column block width 256
+    dom = qe.Timer([qe.QE_KERNEL_TRAIL_GEMM], capacity=args.steps * nb * cfg.iters * nblk + 16)
     t_start.record(stream)
     outs = None
     for k in range(args.steps):
-        outs = step(ev[k])
+        outs = step(ev[k], dom)
     t_end.record(stream)
     torch.cuda.synchronize()
     if world > 1:
@@ -252,6 +298,18 @@ def main():
         t = torch.tensor([ms], dtype=torch.float64, device="cuda")
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         ms = float(t.item())
+
+    dom_launches, dom_ms = dom.read(qe.QE_KERNEL_TRAIL_GEMM)
+    dom.close()
+
+    # algorithmic flops of the trailing GEMMs of one quantize call (block width 256):
+    # sweep 1 and the first window sweep correct block b with its b0 predecessors,
+    # later sweeps with the p most recent column changes (2 flops per update)
+    blocks = [(b0, min(256, p - b0)) for b0 in range(0, p, 256)]
+    tri_flops = sum(2 * q * bw * b0 for b0, bw in blocks)
+    win_flops = sum(2 * q * bw * p for b0, bw in blocks)
+    trail_flops = 2 * tri_flops + max(cfg.iters - 2, 0) * win_flops if cfg.iters >= 2 else tri_flops
+    trail_launches = (2 * (nblk - 1) + max(cfg.iters - 2, 0) * nblk) if cfg.iters >= 2 else nblk - 1
 
     units_per_step = q * p * p * cfg.iters * nb           # column updates per rank per step
     value = units_per_step * world / (ms / 1e3)
@@ -272,18 +330,36 @@ def main():
               "sigma_dense_equiv_tflops": 2 * p * p * n / (sigma_avg / 1e3) / 1e12,
               "cd_ms": {str(b): v for b, v in zip(cfg.bits, cd_avg)},
               "cd_updates_per_s": q * p * p * cfg.iters * nb / (sum(cd_avg) / 1e3),
-              "roofline": {"bound": "tensor", "kernel": "k_tc_gemm<256> (Sigma = X X^T)",
-                           "achieved": sig_flops / (sigma_avg / 1e3) / 1e12,
-                           "peak": pk["bf16_sustained"], "unit": "TFLOP/s",
-                           "frac": sig_flops / (sigma_avg / 1e3) / 1e12 / pk["bf16_sustained"],
-                           "traffic": None,
-                           "peak_source": f"{pk['source']} bf16 dense sustained"},
+              "roofline": roofline_entry(dom_launches, dom_ms, trail_flops * nb * args.steps,
+                                         trail_launches * nb * args.steps, pk),
               "clocks": clk}
 
+    # per-class breakdown of one extra, untimed step (events around every launch)
+    brk = qe.Timer([qe.QE_KERNEL_PINIT_GEMM, qe.QE_KERNEL_RESIDUAL_GEMM, qe.QE_KERNEL_TRAIL_GEMM,
+                    qe.QE_KERNEL_CD_BLOCK], capacity=nb * (2 + cfg.iters * (2 * nblk + 1)) + 16)
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    qe.qe_build_sigma(X, Sigma=Sigma)
+    e1.record(stream)
+    for b in cfg.bits:
+        qe.qe_quantize_layer(W, Sigma, b, cfg.iters, workspace=ws, timer=brk)
+    torch.cuda.synchronize()
+    names = {qe.QE_KERNEL_PINIT_GEMM: "pinit_gemm", qe.QE_KERNEL_RESIDUAL_GEMM: "residual_gemm",
+             qe.QE_KERNEL_TRAIL_GEMM: "trail_gemm", qe.QE_KERNEL_CD_BLOCK: "cd_block"}
+    breakdown = {"sigma_gemm": {"launches": 1, "ms": e0.elapsed_time(e1)}}
+    for k, nm in names.items():
+        n_, ms_ = brk.read(k)
+        breakdown[nm] = {"launches": n_, "ms": ms_}
+    brk.close()
+    result["kernel_ms_per_step"] = breakdown
+
     # launches of our kernels per step (schedule of qe_api.cu)
-    nblk = (p + 255) // 256                    # default column block width 256
     w_planes = 0 if cfg.w_dtype == torch.bfloat16 else 1
-    per_layer = 7 + w_planes + cfg.iters * (nblk + (nblk - 1) + 1 + 1)
+    # set-up: grid, Sigma diagonal, planes, 1/d, packed blocks, P, initial residual;
+    # sweep 1: 15 trailing GEMMs + 16 in-block + residual GEMM + objective sum;
+    # later sweeps: trailing GEMMs (15 in the first window sweep, 16 after) + 16 in-block + objective step
+    per_layer = 7 + w_planes + ((nblk - 1) + nblk + 2) + (cfg.iters - 1) * (2 * nblk + 1) - 1
     result["gpu_launches"] = args.steps * (1 + nb * per_layer)
 
     # end to end through the C ABI with host buffers

@@ -54,6 +54,18 @@ typedef enum {
     QE_TOKEN_MAJOR = 1        /* X is n x p row-major: activations as a model emits them */
 } qe_xlayout;
 
+/* Kernel classes an optional qe_timer can time (bit k of its mask = class k). */
+typedef enum {
+    QE_KERNEL_PINIT_GEMM = 0,     /* P = W (I + Sigma_bar), once per call */
+    QE_KERNEL_RESIDUAL_GEMM = 1,  /* R = P - What Sigma_bar (+ the fused objective) */
+    QE_KERNEL_TRAIL_GEMM = 2,     /* per column block: Delta' Sigma_bar correction (split-K) */
+    QE_KERNEL_CD_BLOCK = 3,       /* per column block: the in-block coordinate updates */
+    QE_KERNEL_COUNT = 4
+} qe_kernel;
+
+/* Opaque set of CUDA event pairs; see qe_timer_create. */
+typedef struct qe_timer qe_timer;
+
 typedef struct {
     /* Column block width B of the blocked CD sweep: 0 = default (256); 64, 128 or 256. */
     int block_width;
@@ -74,6 +86,8 @@ typedef struct {
     /* Optional caller workspace (device, 256-byte aligned) and its size. */
     void *workspace;
     size_t workspace_bytes;
+    /* Optional: record CUDA events around the launches of the timed kernel classes. */
+    qe_timer *timer;
 } qe_opts;
 
 /*
@@ -170,6 +184,21 @@ qe_status qe_build_sigma_static(const void *X, qe_dtype x_dtype, qe_xlayout layo
  * (outlier = 1) needs for this shape and options; written to *bytes. */
 qe_status qe_workspace_size(int64_t q, int64_t p, int outlier, const qe_opts *opts,
                             size_t *bytes);
+
+/*
+ * Kernel timing (profiling aid; the paper has no counterpart).  A timer holds
+ * `capacity` pairs of CUDA events created on the current device.  Passed in
+ * qe_opts, it makes the call record one pair on the call's stream around each
+ * launch whose class bit is set in `kernel_mask`, until the pairs run out
+ * (later launches go untimed).  Recording adds no synchronisation;
+ * qe_timer_read waits for the recorded events and returns the number of timed
+ * launches of `kernel` and their summed duration in milliseconds.  Not
+ * thread-safe: one timer per host thread.
+ */
+qe_status qe_timer_create(unsigned kernel_mask, int capacity, qe_timer **timer);
+qe_status qe_timer_read(qe_timer *timer, int kernel, int *launches, double *total_ms);
+qe_status qe_timer_reset(qe_timer *timer);
+qe_status qe_timer_destroy(qe_timer *timer);
 
 /* Waits for `stream`, then returns and clears the error latched on the current
  * device (QE_ERR_NUMERIC / QE_ERR_TIMEOUT), or QE_ERR_CUDA if the stream failed. */

@@ -15,6 +15,8 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <vector>
+
 #include "../../include/qe.h"
 #include "qe_common.cuh"
 #include "qe_internal.h"
@@ -114,9 +116,43 @@ static Plan make_plan(int64_t q, int64_t p, int B, bool outlier, int wpl_planes,
     return pl;
 }
 
+}  // namespace qe
+
+// ---- kernel timer (C ABI type) ----------------------------------------------------------
+struct qe_timer {
+    unsigned mask = 0;
+    int used = 0;
+    std::vector<cudaEvent_t> start, stop;
+    std::vector<int> kind;
+};
+
+namespace qe {
+
+// Records an event pair around one launch of class `k` when the timer asks for it.
+class Timed {
+  public:
+    Timed(qe_timer *t, int k, cudaStream_t s) : t_(nullptr), s_(s) {
+        if (t && (t->mask & (1u << k)) && t->used < static_cast<int>(t->start.size())) {
+            t_ = t;
+            idx_ = t->used++;
+            t->kind[idx_] = k;
+            cudaEventRecord(t->start[idx_], s);
+        }
+    }
+    ~Timed() {
+        if (t_) cudaEventRecord(t_->stop[idx_], s_);
+    }
+
+  private:
+    qe_timer *t_;
+    cudaStream_t s_;
+    int idx_ = 0;
+};
+
 // ---- per-call context ----------------------------------------------------------------
 struct Ctx {
     cudaStream_t s = nullptr;
+    qe_timer *timer = nullptr;
     unsigned *err = nullptr;
     int nsm = 148;
     Plan pl;
@@ -145,6 +181,7 @@ static T *at(uint8_t *ws, size_t off) {
 
 static qe_status setup_ctx(Ctx &c, const Plan &pl, const qe_opts *o, cudaStream_t s) {
     c.s = s;
+    c.timer = o ? o->timer : nullptr;
     c.pl = pl;
     c.err = error_word();
     if (!c.err) return QE_ERR_CUDA;
@@ -257,7 +294,10 @@ static qe_status prepare(Ctx &c, const void *W, int wbf16, int64_t ldw, const fl
     g.W = W;
     g.w_is_bf16 = wbf16;
     g.ldw = ldw;
-    QE_CK(launch_tc_gemm(256, c.tm_wa, c.tm_snt256, g, 1, c.s));
+    {
+        Timed tm(c.timer, QE_KERNEL_PINIT_GEMM, c.s);
+        QE_CK(launch_tc_gemm(256, c.tm_wa, c.tm_snt256, g, 1, c.s));
+    }
     return QE_OK;
 }
 
@@ -298,7 +338,10 @@ static qe_status residual(Ctx &c, const float *scales, const ObjFuse *f = nullpt
         g.Hd = f->H;
         g.ldh = ld;
     }
-    QE_CK(launch_tc_gemm(256, c.tm_qf, c.tm_snt256, g, 1, c.s));
+    {
+        Timed tm(c.timer, QE_KERNEL_RESIDUAL_GEMM, c.s);
+        QE_CK(launch_tc_gemm(256, c.tm_qf, c.tm_snt256, g, 1, c.s));
+    }
     if (f) QE_CK(launch_sum_partials(c.objp, static_cast<int>(rfull_partials(q, p)), f->obj, c.s));
     return QE_OK;
 }
@@ -332,6 +375,7 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
             g.out = c.part;
             g.ldo = B;
             g.split_stride = q * B;
+            Timed tm(c.timer, QE_KERNEL_TRAIL_GEMM, c.s);
             QE_CK(launch_tc_gemm(B, c.tm_dp, B == 64 ? c.tm_snt64 : (B == 128 ? c.tm_snt128 : c.tm_snt256), g,
                                  S, c.s));
             nsplit = S;
@@ -365,6 +409,7 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
         a.ldd = ld;
         a.dp_plane_rows = q;
         a.err = c.err;
+        Timed tm(c.timer, QE_KERNEL_CD_BLOCK, c.s);
         QE_CK(launch_cd_block(B, a, c.nsm, c.s));
     }
     return QE_OK;
@@ -436,6 +481,60 @@ const char *qe_status_string(qe_status st) {
         case QE_ERR_UNSUPPORTED: return "option or layout not implemented";
         default: return "unknown status";
     }
+}
+
+qe_status qe_timer_create(unsigned kernel_mask, int capacity, qe_timer **timer) {
+    if (!timer || capacity < 1 || capacity > (1 << 20)) return QE_ERR_INVALID_ARG;
+    qe_timer *t = new qe_timer();
+    t->mask = kernel_mask;
+    t->start.assign(capacity, nullptr);
+    t->stop.assign(capacity, nullptr);
+    t->kind.assign(capacity, -1);
+    for (int k = 0; k < capacity; ++k) {
+        if (cudaEventCreate(&t->start[k]) != cudaSuccess || cudaEventCreate(&t->stop[k]) != cudaSuccess) {
+            cudaGetLastError();
+            qe_timer_destroy(t);
+            return QE_ERR_CUDA;
+        }
+    }
+    *timer = t;
+    return QE_OK;
+}
+
+qe_status qe_timer_read(qe_timer *timer, int kernel, int *launches, double *total_ms) {
+    if (!timer || !launches || !total_ms || kernel < 0 || kernel >= QE_KERNEL_COUNT) return QE_ERR_INVALID_ARG;
+    int n = 0;
+    double ms = 0.0;
+    for (int k = 0; k < timer->used; ++k) {
+        if (timer->kind[k] != kernel) continue;
+        float e = 0.0f;
+        if (cudaEventSynchronize(timer->stop[k]) != cudaSuccess ||
+            cudaEventElapsedTime(&e, timer->start[k], timer->stop[k]) != cudaSuccess) {
+            cudaGetLastError();
+            return QE_ERR_CUDA;
+        }
+        ms += e;
+        ++n;
+    }
+    *launches = n;
+    *total_ms = ms;
+    return QE_OK;
+}
+
+qe_status qe_timer_reset(qe_timer *timer) {
+    if (!timer) return QE_ERR_INVALID_ARG;
+    timer->used = 0;
+    return QE_OK;
+}
+
+qe_status qe_timer_destroy(qe_timer *timer) {
+    if (!timer) return QE_ERR_INVALID_ARG;
+    for (size_t k = 0; k < timer->start.size(); ++k) {
+        if (timer->start[k]) cudaEventDestroy(timer->start[k]);
+        if (timer->stop[k]) cudaEventDestroy(timer->stop[k]);
+    }
+    delete timer;
+    return QE_OK;
 }
 
 qe_status qe_sync_status(qe_stream_t stream) {

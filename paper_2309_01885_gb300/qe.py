@@ -22,7 +22,10 @@ QE_FEATURE_MAJOR, QE_TOKEN_MAJOR = 0, 1
 
 EXPORTED = ("qe_build_sigma", "qe_quantize_layer", "qe_quantize_layer_outlier",
             "qe_workspace_size", "qe_sync_status", "qe_status_string", "qe_version",
-            "qe_build_sigma_static")
+            "qe_build_sigma_static", "qe_timer_create", "qe_timer_read", "qe_timer_reset",
+            "qe_timer_destroy")
+QE_KERNEL_PINIT_GEMM, QE_KERNEL_RESIDUAL_GEMM, QE_KERNEL_TRAIL_GEMM, QE_KERNEL_CD_BLOCK, \
+    QE_KERNEL_COUNT = range(5)
 
 
 class QEError(RuntimeError):
@@ -37,7 +40,7 @@ class QEOpts(ctypes.Structure):
                 ("structured_outliers", ctypes.c_int), ("power_iters", ctypes.c_int),
                 ("init_codes", ctypes.c_void_p), ("sweep_codes", ctypes.c_void_p),
                 ("wx_norm2", ctypes.c_void_p), ("workspace", ctypes.c_void_p),
-                ("workspace_bytes", ctypes.c_size_t)]
+                ("workspace_bytes", ctypes.c_size_t), ("timer", ctypes.c_void_p)]
 
 
 _lib = None
@@ -73,6 +76,14 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     L.qe_version.restype = ctypes.c_int
     L.qe_build_sigma_static.argtypes = [vp, i32, i32, i64, i64, i64, vp, i32, vp]
     L.qe_build_sigma_static.restype = st
+    L.qe_timer_create.argtypes = [ctypes.c_uint, i32, ctypes.POINTER(vp)]
+    L.qe_timer_create.restype = st
+    L.qe_timer_read.argtypes = [vp, i32, ctypes.POINTER(ctypes.c_int), ctypes.POINTER(ctypes.c_double)]
+    L.qe_timer_read.restype = st
+    L.qe_timer_reset.argtypes = [vp]
+    L.qe_timer_reset.restype = st
+    L.qe_timer_destroy.argtypes = [vp]
+    L.qe_timer_destroy.restype = st
     _lib = L
     return L
 
@@ -150,9 +161,43 @@ def qe_build_sigma_static(X: torch.Tensor, layout: int = QE_FEATURE_MAJOR, Sigma
     return Sigma
 
 
+class Timer:
+    """CUDA-event timing of selected kernel classes inside the library's calls."""
+
+    def __init__(self, kernels, capacity: int = 4096):
+        mask = 0
+        for k in kernels:
+            mask |= 1 << k
+        h = ctypes.c_void_p()
+        _check(load().qe_timer_create(mask, capacity, ctypes.byref(h)), "qe_timer_create")
+        self.handle = h
+
+    def read(self, kernel: int):
+        """(launches, total milliseconds) of the timed launches of `kernel`."""
+        n = ctypes.c_int(0)
+        ms = ctypes.c_double(0.0)
+        _check(load().qe_timer_read(self.handle, kernel, ctypes.byref(n), ctypes.byref(ms)), "qe_timer_read")
+        return n.value, ms.value
+
+    def reset(self):
+        _check(load().qe_timer_reset(self.handle), "qe_timer_reset")
+
+    def close(self):
+        if self.handle:
+            load().qe_timer_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
 def _opts(block_width=0, power_iters=0, init_codes=None, sweep_codes=None, wx_norm2=None,
-          workspace=None) -> QEOpts:
+          workspace=None, timer=None) -> QEOpts:
     o = QEOpts()
+    o.timer = None if timer is None else timer.handle.value
     o.block_width = block_width
     o.power_iters = power_iters
     o.init_codes = None if init_codes is None else init_codes.data_ptr()
@@ -167,7 +212,8 @@ def _opts(block_width=0, power_iters=0, init_codes=None, sweep_codes=None, wx_no
 def qe_quantize_layer(W: torch.Tensor, Sigma: torch.Tensor, bits: int, iters: int, *,
                       init_codes: torch.Tensor | None = None, record_sweeps: bool = False,
                       want_norm: bool = False, block_width: int = 0,
-                      workspace: torch.Tensor | None = None, stream=None) -> dict:
+                      workspace: torch.Tensor | None = None, timer: Timer | None = None,
+                      stream=None) -> dict:
     """QuantEase on one layer; returns codes (u8 q x p), scales, zeros, obj (fp64 per sweep),
     and optionally sweep_codes (iters x q x p) and wx_norm2."""
     q, p = W.shape
@@ -178,7 +224,7 @@ def qe_quantize_layer(W: torch.Tensor, Sigma: torch.Tensor, bits: int, iters: in
     obj = torch.empty(iters, dtype=torch.float64, device=dev)
     sweep = torch.empty(iters, q, p, dtype=torch.uint8, device=dev) if record_sweeps else None
     norm = torch.empty(1, dtype=torch.float64, device=dev) if want_norm else None
-    o = _opts(block_width, 0, init_codes, sweep, norm, workspace)
+    o = _opts(block_width, 0, init_codes, sweep, norm, workspace, timer)
     _check(load().qe_quantize_layer(_ptr(W), _dtype(W), q, p, _rowmajor_ld(W), _ptr(Sigma), bits, iters,
                                     ctypes.byref(o), _ptr(codes), _ptr(scales), _ptr(zeros), _ptr(obj),
                                     _stream(stream)), "qe_quantize_layer")

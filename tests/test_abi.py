@@ -38,8 +38,8 @@ def test_status_strings_and_version(lib):
 
 
 def test_opts_struct_matches_header():
-    # 4 ints, 4 pointers, 1 size_t on LP64
-    assert ctypes.sizeof(qe.QEOpts) == 4 * 4 + 4 * 8 + 8
+    # 4 ints, 4 pointers, 1 size_t, 1 pointer on LP64
+    assert ctypes.sizeof(qe.QEOpts) == 4 * 4 + 4 * 8 + 8 + 8
 
 
 def _fake(n=1):
