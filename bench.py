@@ -32,6 +32,7 @@ if ROOT not in sys.path:
 
 METRIC = ("layer quantize time; CD column-updates/s (q·p²/s) and Σ TFLOP/s vs roofline")
 UNIT = "q·p² column-updates/s"
+DEFAULT_DENSE_SWEEPS = 1      # the library's default for qe_opts.dense_sweeps
 
 
 def parse():
@@ -44,6 +45,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-rows", type=int, default=4096, help="oracle rows in the CPU sample")
+    ap.add_argument("--dense-sweeps", type=int, default=0,
+                    help="sweeps whose cross-block term uses the tensor-core GEMM (0 = library default)")
     ap.add_argument("--tokens", type=int, default=0,
                     help="override n (calibration tokens), for small profiling captures only")
     return ap.parse_args()
@@ -259,7 +262,8 @@ def main():
             events[1].record(stream)
         outs = []
         for k, b in enumerate(cfg.bits):
-            outs.append(qe.qe_quantize_layer(W, Sigma, b, cfg.iters, workspace=ws, timer=timer))
+            outs.append(qe.qe_quantize_layer(W, Sigma, b, cfg.iters, workspace=ws, timer=timer,
+                                             dense_sweeps=args.dense_sweeps))
             if events:
                 events[2 + k].record(stream)
         return outs
@@ -308,8 +312,12 @@ def main():
     blocks = [(b0, min(256, p - b0)) for b0 in range(0, p, 256)]
     tri_flops = sum(2 * q * bw * b0 for b0, bw in blocks)
     win_flops = sum(2 * q * bw * p for b0, bw in blocks)
-    trail_flops = 2 * tri_flops + max(cfg.iters - 2, 0) * win_flops if cfg.iters >= 2 else tri_flops
-    trail_launches = (2 * (nblk - 1) + max(cfg.iters - 2, 0) * nblk) if cfg.iters >= 2 else nblk - 1
+    dense = args.dense_sweeps or DEFAULT_DENSE_SWEEPS
+    trail_flops, trail_launches = tri_flops, nblk - 1
+    for t in range(1, cfg.iters):
+        if t < dense:   # later sweeps take the cross-block term from the change lists
+            trail_flops += tri_flops if t == 1 else win_flops
+            trail_launches += nblk - 1 if t == 1 else nblk
 
     units_per_step = q * p * p * cfg.iters * nb           # column updates per rank per step
     value = units_per_step * world / (ms / 1e3)
@@ -343,7 +351,7 @@ def main():
     qe.qe_build_sigma(X, Sigma=Sigma)
     e1.record(stream)
     for b in cfg.bits:
-        qe.qe_quantize_layer(W, Sigma, b, cfg.iters, workspace=ws, timer=brk)
+        qe.qe_quantize_layer(W, Sigma, b, cfg.iters, workspace=ws, timer=brk, dense_sweeps=args.dense_sweeps)
     torch.cuda.synchronize()
     names = {qe.QE_KERNEL_PINIT_GEMM: "pinit_gemm", qe.QE_KERNEL_RESIDUAL_GEMM: "residual_gemm",
              qe.QE_KERNEL_TRAIL_GEMM: "trail_gemm", qe.QE_KERNEL_CD_BLOCK: "cd_block"}
@@ -354,12 +362,17 @@ def main():
     brk.close()
     result["kernel_ms_per_step"] = breakdown
 
-    # launches of our kernels per step (schedule of qe_api.cu)
+    # launches of our kernels per step (the schedule of qe_quantize_layer)
     w_planes = 0 if cfg.w_dtype == torch.bfloat16 else 1
-    # set-up: grid, Sigma diagonal, planes, 1/d, packed blocks, P, initial residual;
-    # sweep 1: 15 trailing GEMMs + 16 in-block + residual GEMM + objective sum;
-    # later sweeps: trailing GEMMs (15 in the first window sweep, 16 after) + 16 in-block + objective step
-    per_layer = 7 + w_planes + ((nblk - 1) + nblk + 2) + (cfg.iters - 1) * (2 * nblk + 1) - 1
+    # set-up: grid, Sigma diagonal, Sigma_bar planes, 1/d, packed blocks, Sigma_bar rows,
+    # [W planes], P, initial residual; sweep 1: nblk - 1 trailing GEMMs + nblk in-block +
+    # residual GEMM + objective sum; dense window sweeps: trailing GEMMs (nblk - 1 in the
+    # first) + nblk in-block + objective step; list sweeps: one persistent launch and one
+    # objective prefix per 32 sweeps
+    per_layer = 8 + w_planes + (nblk - 1) + nblk + 2
+    for t in range(1, min(dense, cfg.iters)):
+        per_layer += (nblk - 1 if t == 1 else nblk) + nblk + 1
+    per_layer += 2 * -(-max(cfg.iters - max(dense, 1), 0) // 32)
     result["gpu_launches"] = args.steps * (1 + nb * per_layer)
 
     # end to end through the C ABI with host buffers
@@ -383,7 +396,8 @@ def main():
             Wd.copy_(Wh, non_blocking=True)
             qe.qe_build_sigma(Xd, Sigma=Sigma)
             for k, b in enumerate(cfg.bits):
-                o = qe.qe_quantize_layer(Wd, Sigma, b, cfg.iters, workspace=ws)
+                o = qe.qe_quantize_layer(Wd, Sigma, b, cfg.iters, workspace=ws,
+                                         dense_sweeps=args.dense_sweeps)
                 for key in ("codes", "scales", "zeros", "obj"):
                     host_out[k][key].copy_(o[key], non_blocking=True)
         e1.record(stream)

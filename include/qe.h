@@ -75,6 +75,15 @@ typedef struct {
     int structured_outliers;
     /* Outlier variant: power-method iterations for lambda_max(Sigma), 0 = default 64. */
     int power_iters;
+    /* How the cross-block term Delta'[:, other blocks] Sigma_bar[:, block] of a
+     * sweep is formed (no paper counterpart: both forms compute the same sums of
+     * Eq. cd-update-closed-2).  Sweeps 1 .. dense_sweeps multiply the dense
+     * change matrix on the tensor cores; later sweeps, where few codes change,
+     * walk per-row lists of the changed columns and add their fp32 Sigma_bar
+     * rows.  0 = default (1: lists from sweep 2 on); a value >= iters keeps the
+     * dense form throughout;
+     * negative is QE_ERR_INVALID_ARG.  Ignored by the outlier variant. */
+    int dense_sweeps;
     /* Optional warm start (Sec. 3.1, "initialized with ... any other algorithm"):
      * q x p codes (leading dimension p) on the grid this call computes.  NULL = start at W. */
     const uint8_t *init_codes;

@@ -50,13 +50,17 @@ static int sm_count() {
 
 constexpr int kDefaultBlock = 256;
 constexpr int kDefaultPowerIters = 64;
+constexpr int kDefaultDenseSweeps = 1;
+constexpr int kSweepChunk = 32;          // list-mode sweeps per persistent launch
+constexpr int kFreeMaxChanges = 16;      // changes per row in the previous sweep below which a CTA runs free
 
 // ---- workspace layout -----------------------------------------------------------
 struct Plan {
     int64_t q = 0, p = 0, ld = 0;
     int B = kDefaultBlock, smax = 1;
     size_t snt = 0, d = 0, dinv = 0, tri = 0, P = 0, R = 0, wpl = 0, qf = 0, dp = 0, part = 0, objp = 0,
-           rowdf = 0, objbase = 0;
+           rowdf = 0, objbase = 0, sbar = 0, lcnt = 0, lent = 0, rowdft = 0;
+    int64_t nblk = 0;
     size_t PW = 0, H = 0, T = 0, st = 0, cg = 0, ce = 0, sb = 0, eb = 0, y0 = 0, y1 = 0, lam = 0,
            eta = 0, rowptr = 0;
     size_t total = 0;
@@ -74,6 +78,7 @@ static Plan make_plan(int64_t q, int64_t p, int B, bool outlier, int wpl_planes,
     pl.p = p;
     pl.ld = round_up(p, 64);
     pl.B = B;
+    pl.nblk = ceil_div(p, B);
     const int64_t mtiles = ceil_div(q, 128);
     int64_t smax = nsm / mtiles;
     if (smax < 1) smax = 1;
@@ -95,6 +100,12 @@ static Plan make_plan(int64_t q, int64_t p, int B, bool outlier, int wpl_planes,
                                                                                     : objective_blocks(q)) * 8);
     pl.rowdf = take(cur, static_cast<size_t>(q) * 8);
     pl.objbase = take(cur, 8);
+    if (!outlier) {   // change lists and fp32 Sigma_bar rows of the rolling-window sweeps
+        pl.sbar = take(cur, static_cast<size_t>(p) * pl.ld * 4);
+        pl.lcnt = take(cur, static_cast<size_t>(q) * pl.nblk * 4);
+        pl.lent = take(cur, static_cast<size_t>(q) * pl.nblk * B * 4);
+        pl.rowdft = take(cur, static_cast<size_t>(q) * kSweepChunk * 8);
+    }
     if (outlier) {
         const int64_t N = q * p;
         const int64_t nch = topk_chunks(N);
@@ -161,6 +172,10 @@ struct Ctx {
     __nv_bfloat16 *snt = nullptr, *wpl = nullptr, *qf = nullptr, *dp = nullptr;
     float *d = nullptr, *dinv = nullptr, *tri = nullptr, *P = nullptr, *R = nullptr, *part = nullptr;
     double *objp = nullptr, *rowdf = nullptr, *objbase = nullptr;
+    float *sbar = nullptr;
+    int *lcnt = nullptr;
+    uint32_t *lent = nullptr;
+    double *rowdft = nullptr;
     float *PW = nullptr, *H = nullptr, *T = nullptr, *y0 = nullptr, *y1 = nullptr;
     TopkState *st = nullptr;
     unsigned *cg = nullptr, *ce = nullptr, *sb = nullptr, *eb = nullptr;
@@ -212,6 +227,12 @@ static qe_status setup_ctx(Ctx &c, const Plan &pl, const qe_opts *o, cudaStream_
     c.objp = at<double>(w, pl.objp);
     c.rowdf = at<double>(w, pl.rowdf);
     c.objbase = at<double>(w, pl.objbase);
+    if (pl.sbar) {
+        c.sbar = at<float>(w, pl.sbar);
+        c.lcnt = at<int>(w, pl.lcnt);
+        c.lent = at<uint32_t>(w, pl.lent);
+        c.rowdft = at<double>(w, pl.rowdft);
+    }
     if (pl.PW) {
         c.PW = at<float>(w, pl.PW);
         c.H = at<float>(w, pl.H);
@@ -275,6 +296,7 @@ static qe_status prepare(Ctx &c, const void *W, int wbf16, int64_t ldw, const fl
     QE_CK(launch_sigma_norm(Sigma, p, p, c.d, c.snt, ld, c.err, c.s));
     QE_CK(launch_dinv(c.d, p, c.dinv, c.s));
     QE_CK(launch_pack_diag(c.snt, ld, p, c.pl.B, c.tri, c.s));
+    if (c.sbar) QE_CK(launch_sigma_bar_rows(Sigma, p, p, c.d, c.sbar, ld, c.s));
     const bool direct = wbf16 && ((reinterpret_cast<uintptr_t>(W) & 15u) == 0) && (ldw % 8 == 0);
     if (direct) {
         if (!make_tmap_bf16(&c.tm_wa, W, q, p, ldw, 128)) return QE_ERR_CUDA;
@@ -356,6 +378,8 @@ static qe_status residual(Ctx &c, const float *scales, const ObjFuse *f = nullpt
 //       all of them in dp), the staged values become the new base, and the
 //       objective changes of the decisions accumulate in rowdf.  window = -1
 //       means the first window sweep after a residual refresh: only columns < b0.
+//       Every window visit also records its changes in the block's change list,
+//       from which the later sweeps (k_cd_rows_lists) take the correction.
 static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float *zeros, int bits,
                        bool first, int window) {
     const int64_t q = c.pl.q, p = c.pl.p, ld = c.pl.ld;
@@ -406,6 +430,9 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
         a.qf = c.qf;
         a.ldq = ld;
         a.dp = c.dp;
+        a.nblk = static_cast<int>(c.pl.nblk);
+        a.lcnt = c.lcnt;
+        if (window != 0) a.lent = c.lent;
         a.ldd = ld;
         a.dp_plane_rows = q;
         a.err = c.err;
@@ -413,6 +440,32 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
         QE_CK(launch_cd_block(B, a, c.nsm, c.s));
     }
     return QE_OK;
+}
+
+// Arguments of the persistent change-list kernel (block fields unused).
+static CdArgs list_args(const Ctx &c, uint8_t *codes, const float *scales, const float *zeros, int bits) {
+    CdArgs a;
+    memset(&a, 0, sizeof(a));
+    a.q = c.pl.q;
+    a.p = c.pl.p;
+    a.R = c.R;
+    a.ldr = c.pl.ld;
+    a.tri = c.tri;
+    a.scale = scales;
+    a.zero = zeros;
+    a.d = c.d;
+    a.maxq = static_cast<float>((1 << bits) - 1);
+    a.codes = codes;
+    a.ldc = c.pl.p;
+    a.qf = c.qf;
+    a.ldq = c.pl.ld;
+    a.sbar = c.sbar;
+    a.lds = c.pl.ld;
+    a.nblk = static_cast<int>(c.pl.nblk);
+    a.lcnt = c.lcnt;
+    a.lent = c.lent;
+    a.err = c.err;
+    return a;
 }
 
 static qe_status objective(Ctx &c, const void *W, int wbf16, int64_t ldw, const float *H,
@@ -442,12 +495,16 @@ static int block_width(const qe_opts *o) {
     return (o && o->block_width) ? o->block_width : kDefaultBlock;
 }
 
+static int dense_sweeps(const qe_opts *o) {
+    return (o && o->dense_sweeps) ? o->dense_sweeps : kDefaultDenseSweeps;
+}
+
 static qe_status check_opts(const qe_opts *o) {
     if (!o) return QE_OK;
     if (o->relax_period != 0 || o->structured_outliers != 0) return QE_ERR_UNSUPPORTED;
     if (o->block_width != 0 && o->block_width != 64 && o->block_width != 128 && o->block_width != 256)
         return QE_ERR_UNSUPPORTED;
-    if (o->power_iters < 0) return QE_ERR_INVALID_ARG;
+    if (o->power_iters < 0 || o->dense_sweeps < 0) return QE_ERR_INVALID_ARG;
     if (o->workspace && o->workspace_bytes == 0) return QE_ERR_INVALID_ARG;
     return QE_OK;
 }
@@ -677,13 +734,30 @@ qe_status qe_quantize_layer(const void *W, qe_dtype w_dtype, int64_t q, int64_t 
     }
     // the refreshed residual already holds every change so far: start the window empty
     QE_CK(cudaMemsetAsync(c.dp, 0, plane0, c.s));
+    QE_CK(cudaMemsetAsync(c.lcnt, 0, static_cast<size_t>(q) * pl.nblk * 4, c.s));
     QE_CK(cudaMemsetAsync(c.rowdf, 0, static_cast<size_t>(q) * 8, c.s));
-    for (int t = t0; t < iters; ++t) {
+    // sweeps 1 .. dense use the tensor-core correction, one launch pair per block
+    const int dense = dense_sweeps(opts);
+    int t = t0;
+    for (; t < iters && t < dense; ++t) {
         if ((st = sweep(c, codes, scales, zeros, bits, false, t == t0 ? -1 : 1)) != QE_OK) return st;
         QE_CK(launch_obj_step(c.rowdf, q, t == 0 ? c.objbase : obj + t - 1, obj + t, c.s));
         if (opts && opts->sweep_codes)
             QE_CK(cudaMemcpyAsync(opts->sweep_codes + static_cast<size_t>(t) * q * p, codes,
                                   static_cast<size_t>(q) * p, cudaMemcpyDeviceToDevice, c.s));
+    }
+    // later sweeps: the change lists, persistent over blocks and sweeps
+    while (t < iters) {
+        const int te = (iters - t) < kSweepChunk ? iters : t + kSweepChunk;
+        CdArgs a = list_args(c, codes, scales, zeros, bits);
+        {
+            Timed tm(c.timer, QE_KERNEL_CD_BLOCK, c.s);
+            // the lists are empty at the window start (t0): that sweep steps in lockstep
+            QE_CK(launch_cd_rows_lists(pl.B, a, t, te, c.rowdft, opts ? opts->sweep_codes : nullptr, t == t0,
+                                       kFreeMaxChanges, c.nsm, c.s));
+        }
+        QE_CK(launch_obj_prefix(c.rowdft, q, te - t, t == 0 ? c.objbase : obj + t - 1, obj + t, c.s));
+        t = te;
     }
     return QE_OK;
 }

@@ -104,6 +104,35 @@ __global__ void k_sigma_planes(const float *S, int64_t lds, int64_t p, const flo
     if (bad) set_error(err, ERR_NUMERIC);
 }
 
+// Sigma_bar in fp32, row-major (row k, column j): Sigma_bar[k][j] =
+// Sigma[j][k] / d_j, the same binary32 value whose hi + mid + lo planes
+// k_sigma_planes writes (so the change-list correction and the tensor-core
+// correction multiply the same matrix).  Row k holds what a change of column k
+// adds to the other columns, contiguous over j.  Columns [p, ld) are zero.
+// 32 x 32 tiles transposed through shared memory; grid (ld / 32, p / 32).
+__global__ void __launch_bounds__(256) k_sigma_bar_rows(const float *S, int64_t lds, int64_t p, const float *d,
+                                                        float *sbar, int64_t ld) {
+    __shared__ float tile[32][33];
+    const int64_t j0 = static_cast<int64_t>(blockIdx.x) * 32, k0 = static_cast<int64_t>(blockIdx.y) * 32;
+    const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+    // load: S[j][k] for j in [j0, j0+32) (rows), k = k0 + tx (coalesced)
+    for (int r = ty; r < 32; r += 8) {
+        const int64_t j = j0 + r, k = k0 + tx;
+        float x = 0.0f;
+        if (j < p && k < p) {
+            const float dj = d[j];
+            if (dj > 0.0f && k != j && d[k] > 0.0f) x = __fdiv_rn(S[j * lds + k], dj);
+        }
+        tile[r][tx] = x;
+    }
+    __syncthreads();
+    // store: sbar[k][j] for k in [k0, k0+32), j = j0 + tx (coalesced)
+    for (int r = ty; r < 32; r += 8) {
+        const int64_t k = k0 + r, j = j0 + tx;
+        if (k < p && j < ld) sbar[k * ld + j] = tile[tx][r];
+    }
+}
+
 // ---------------------------------------------------------------------------
 // Operand planes of a q x p matrix for the tensor-core GEMM (rows [0,q) = hi,
 // [q, 2q) = mid, [2q, 3q) = lo when split).  fp32 input splits into three bf16
@@ -226,6 +255,66 @@ struct CdCfg {
     static constexpr int MAX_SPLITS = 16;
 };
 
+// Cross-block correction from the change lists (the sparse form of the
+// trailing GEMM, used once few codes change per sweep): for every column block
+// (this one included) the changes of its most recent visit, each adding
+// Delta'_ik Sigma_bar[k][block] to the row; Sigma_bar rows are fp32 and
+// contiguous over the block, so each change is one coalesced read of B floats
+// per warp.  Returns whether the row had any change in the window.
+template <int B, bool FULL>
+__device__ __forceinline__ bool list_correction(const CdArgs &a, int64_t b0, int bw_, int64_t ii, bool row_ok,
+                                                int lane, float (&ps)[B / 32]) {
+    constexpr int CPL = B / 32;
+    const int bw = FULL ? B : bw_;
+    const int64_t rb = ii * a.nblk;
+    const float *sb0 = a.sbar + b0 + lane;
+    bool any = false;
+    for (int c0 = 0; c0 < a.nblk; c0 += 32) {
+        const int cnt = (row_ok && c0 + lane < a.nblk) ? a.lcnt[rb + c0 + lane] : 0;
+        unsigned m = __ballot_sync(0xffffffffu, cnt > 0);
+        any = any || m != 0u;
+        while (m != 0u) {
+            const int sl = __ffs(m) - 1;
+            m &= m - 1u;
+            const int c = __shfl_sync(0xffffffffu, cnt, sl);
+            const int64_t blk2 = c0 + sl;
+            const uint32_t *seg = a.lent + (rb + blk2) * B;
+            const float *sbk = sb0 + blk2 * B * a.lds;
+            for (int e0 = 0; e0 < c; e0 += 32) {
+                const uint32_t mine = (e0 + lane < c) ? seg[e0 + lane] : 0u;
+                const int ne = (c - e0) < 32 ? (c - e0) : 32;
+                int u = 0;
+                for (; u + 2 <= ne; u += 2) {
+                    const uint32_t e1 = __shfl_sync(0xffffffffu, mine, u);
+                    const uint32_t e2 = __shfl_sync(0xffffffffu, mine, u + 1);
+                    const float *r1 = sbk + static_cast<int64_t>(e1 & 0xffffu) * a.lds;
+                    const float *r2 = sbk + static_cast<int64_t>(e2 & 0xffffu) * a.lds;
+                    const float d1 = static_cast<float>(static_cast<int16_t>(e1 >> 16));
+                    const float d2 = static_cast<float>(static_cast<int16_t>(e2 >> 16));
+                    float v1[CPL], v2[CPL];
+#pragma unroll
+                    for (int h = 0; h < CPL; ++h) {
+                        const bool ok = FULL || 32 * h + lane < bw;
+                        v1[h] = ok ? __ldg(r1 + 32 * h) : 0.0f;
+                        v2[h] = ok ? __ldg(r2 + 32 * h) : 0.0f;
+                    }
+#pragma unroll
+                    for (int h = 0; h < CPL; ++h) ps[h] = fmaf(d2, v2[h], fmaf(d1, v1[h], ps[h]));
+                }
+                if (u < ne) {
+                    const uint32_t e1 = __shfl_sync(0xffffffffu, mine, u);
+                    const float *r1 = sbk + static_cast<int64_t>(e1 & 0xffffu) * a.lds;
+                    const float d1 = static_cast<float>(static_cast<int16_t>(e1 >> 16));
+#pragma unroll
+                    for (int h = 0; h < CPL; ++h)
+                        if (FULL || 32 * h + lane < bw) ps[h] = fmaf(d1, __ldg(r1 + 32 * h), ps[h]);
+                }
+            }
+        }
+    }
+    return any;
+}
+
 // Common prologue of both in-block kernels: start the bulk copy of the packed
 // block, stage the row (t = R + sum of split partials, R already in grid-step
 // units; st = start value: R itself in the first sweep, else the old code),
@@ -267,12 +356,13 @@ __device__ __forceinline__ bool cd_prologue(const CdArgs &a, float *tri, uint64_
         for (int h = 0; h < CPL; ++h)
             if (row_ok && (FULL || 32 * h + lane < bw)) ps[h] += prow[32 * h + lane];
     }
+    const bool changed = a.nsplit > 0;
 #pragma unroll
     for (int h = 0; h < CPL; ++h) {
         st[h] = a.first_sweep ? r_[h] : static_cast<float>(cd_[h]);
         t[h] = r_[h] + ps[h];
     }
-    if (a.store_base && a.nsplit > 0) {
+    if (a.store_base && changed) {
 #pragma unroll
         for (int h = 0; h < CPL; ++h) {
             const int l = 32 * h + lane;
@@ -288,21 +378,23 @@ __device__ __forceinline__ bool cd_prologue(const CdArgs &a, float *tri, uint64_
 
 // Common epilogue: codes, C - z (both skipped for unchanged columns when
 // skip_same) and the Delta' plane(s).
-template <int B, bool FULL>
-__device__ __forceinline__ void cd_epilogue(const CdArgs &a, int64_t i, int lane, const float (&code)[B / 32],
-                                            const float (&dlt)[B / 32], bool skip_same) {
+template <int B, bool FULL, bool RECORD>
+__device__ __forceinline__ void cd_epilogue(const CdArgs &a, int64_t b0, int bw_, int64_t i, int lane,
+                                            const float (&code)[B / 32], const float (&dlt)[B / 32],
+                                            bool skip_same) {
     constexpr int CPL = B / 32;
-    const int bw = FULL ? B : a.bw;
+    const int bw = FULL ? B : bw_;
     const float z = a.zero[i];
 #pragma unroll
     for (int h = 0; h < CPL; ++h) {
         const int l = 32 * h + lane;
         if (!FULL && l >= bw) continue;
-        const int64_t col = a.b0 + l;
+        const int64_t col = b0 + l;
         if (!skip_same || dlt[h] != 0.0f) {
             a.codes[i * a.ldc + col] = static_cast<uint8_t>(code[h]);
             if (a.write_qf) a.qf[i * a.ldq + col] = __float2bfloat16_rn(code[h] - z);
         }
+        if (!a.dp) continue;
         const __nv_bfloat16 hi = __float2bfloat16_rn(dlt[h]);
         a.dp[i * a.ldd + col] = hi;
         if (a.first_sweep) {   // Delta' is not an integer in the first sweep: three planes
@@ -311,6 +403,25 @@ __device__ __forceinline__ void cd_epilogue(const CdArgs &a, int64_t i, int lane
             a.dp[(a.dp_plane_rows + i) * a.ldd + col] = mid;
             a.dp[(2 * a.dp_plane_rows + i) * a.ldd + col] = __float2bfloat16_rn(r1 - __bfloat162float(mid));
         }
+    }
+    if (RECORD) {   // this visit's changes replace the block's list (ascending columns)
+        __syncwarp();
+        const int64_t seg = i * a.nblk + b0 / B;
+        uint32_t *ent = a.lent + seg * B;
+        int n = 0;
+#pragma unroll
+        for (int h = 0; h < CPL; ++h) {
+            const int l = 32 * h + lane;
+            const bool ch = (FULL || l < bw) && dlt[h] != 0.0f;
+            const unsigned m = __ballot_sync(0xffffffffu, ch);
+            if (ch) {
+                const int16_t dv = static_cast<int16_t>(__float2int_rn(dlt[h]));
+                ent[n + __popc(m & ((1u << lane) - 1u))] =
+                    static_cast<uint32_t>(l) | (static_cast<uint32_t>(static_cast<uint16_t>(dv)) << 16);
+            }
+            n += __popc(m);
+        }
+        if (lane == 0) a.lcnt[seg] = n;
     }
 }
 
@@ -361,7 +472,7 @@ __global__ void __launch_bounds__(1024) k_cd_block_seq(const CdArgs a) {
             }
         }
     }
-    cd_epilogue<B, FULL>(a, i, lane, code, dlt, false);
+    cd_epilogue<B, FULL, false>(a, a.b0, a.bw, i, lane, code, dlt, false);
 }
 
 // Change-driven in-block kernel (every sweep after the first), exactly
@@ -370,35 +481,35 @@ __global__ void __launch_bounds__(1024) k_cd_block_seq(const CdArgs a) {
 // first one that changes is found by a warp ballot, its change is applied to
 // the columns after it, and the pass resumes right after it.  The cost is
 // (number of changed columns + 1) data-parallel passes.
-template <int B, bool FULL>
-__global__ void __launch_bounds__(1024) k_cd_block_chg(const CdArgs a) {
-    using C = CdCfg<B>;
-    constexpr int CPL = C::CPL;
-    extern __shared__ __align__(16) float cd_smem[];
-    float *tri = cd_smem;
-    uint64_t *bar = reinterpret_cast<uint64_t *>(cd_smem + C::PACK);
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int64_t i = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + warp;
-    const bool row_ok = i < a.q;
-    float t[CPL], st[CPL];
-    if (!cd_prologue<B, FULL>(a, tri, bar, i, row_ok, lane, t, st)) return;
-    if (!row_ok) return;
-    const int bw = FULL ? B : a.bw;
-    const float maxq = a.maxq;
-    float code[CPL], dlt[CPL];
+// The change-driven decisions of one row over one block (shared by the
+// per-block and the persistent kernels): quantize every column not yet final,
+// find the first one whose code changes (warp ballot), add its change times
+// its row of the block's Sigma_bar (packed triangle `tri`) to the columns
+// after it, and resume right after it.  dfacc (per lane) collects the exact
+// objective change of each applied decision (Lemma 1: along one coordinate
+// f(u) = Sigma_jj (u - beta)^2 + const, here u = s (code - z), beta = s (t - z)).
+//   GROWS = false: the coupling rows come from the packed triangle in shared
+//   memory; GROWS = true: from the fp32 Sigma_bar rows in global memory
+//   (`grow` = &Sigma_bar[b0][b0], leading dimension lds; the same values).
+template <int B, bool FULL, bool GROWS = false>
+__device__ __forceinline__ int chg_decide(const float *tri, const float *d_blk, int bw_, float maxq, float s2,
+                                          bool want_df, int lane, float (&t)[B / 32], const float (&st)[B / 32],
+                                          float (&code)[B / 32], float (&dlt)[B / 32], double &dfacc,
+                                          const float *grow = nullptr, int64_t lds = 0) {
+    constexpr int CPL = B / 32;
+    const int bw = FULL ? B : bw_;
 #pragma unroll
     for (int h = 0; h < CPL; ++h) {
         code[h] = st[h];
         dlt[h] = 0.0f;
     }
-    // objective change of the decisions (Lemma 1: f(u) = Sigma_jj (u - beta)^2 + const
-    // along one coordinate), in units where u = s (code - z) and beta = s (t - z)
-    const float s = a.scale[i];
-    const float s2 = s * s;
-    double dfacc = 0.0;
     int pos = 0;                                       // first column not yet final
+    int nchg = 0;
     while (pos < bw) {
         int jstar = -1;
+        // values of this lane's column in the word that holds the first change
+        // (captured with a compile-time h, so the arrays stay in registers)
+        float v = 0.0f, tv = 0.0f, cv = 0.0f, sv = 0.0f;
 #pragma unroll
         for (int h = 0; h < CPL; ++h) {
             const int l = 32 * h + lane;
@@ -410,38 +521,233 @@ __global__ void __launch_bounds__(1024) k_cd_block_chg(const CdArgs a) {
                 dlt[h] = dl;
             }
             const unsigned m = __ballot_sync(0xffffffffu, active && dl != 0.0f);
-            if (jstar < 0 && m != 0u) jstar = 32 * h + (__ffs(m) - 1);
-        }
-        if (jstar < 0) break;
-        // the change of column jstar, from its lane
-        float v = dlt[0], tv = t[0], cv = code[0], sv = st[0];
-#pragma unroll
-        for (int h = 1; h < CPL; ++h)
-            if (h == (jstar >> 5)) {
-                v = dlt[h];
+            if (jstar < 0 && m != 0u) {
+                jstar = 32 * h + (__ffs(m) - 1);
+                v = dl;
                 tv = t[h];
-                cv = code[h];
+                cv = c;
                 sv = st[h];
             }
-        if (a.rowdf && lane == (jstar & 31)) {
-            const float dj = a.d[a.b0 + jstar];
+        }
+        if (jstar < 0) break;
+        if (want_df && lane == (jstar & 31)) {
+            const float dj = d_blk[jstar];
             if (dj > 0.0f) {
                 const float e1 = cv - tv, e0 = sv - tv;
                 dfacc += static_cast<double>(dj * s2 * (e1 * e1 - e0 * e0));
             }
         }
         const float db = __shfl_sync(0xffffffffu, v, jstar & 31);
-        const float *row = tri + kPackPad + tri_off(B, jstar) - (jstar + 1);
+        if (GROWS) {
+            const float *row = grow + jstar * lds + lane;
+            float rv[CPL];
 #pragma unroll
-        for (int g = 0; g < CPL; ++g) t[g] = fmaf(db, row[32 * g + lane], t[g]);
+            for (int g = 0; g < CPL; ++g) rv[g] = (FULL || 32 * g + lane < bw) ? __ldg(row + 32 * g) : 0.0f;
+#pragma unroll
+            for (int g = 0; g < CPL; ++g) t[g] = fmaf(db, rv[g], t[g]);
+        } else {
+            const float *row = tri + kPackPad + tri_off(B, jstar) - (jstar + 1);
+#pragma unroll
+            for (int g = 0; g < CPL; ++g) t[g] = fmaf(db, row[32 * g + lane], t[g]);
+        }
         pos = jstar + 1;
+        ++nchg;
     }
-    if (a.rowdf) {
+    return nchg;
+}
+
+__device__ __forceinline__ double warp_sum(double x) {
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) dfacc += __shfl_xor_sync(0xffffffffu, dfacc, o);
+    for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+    return x;
+}
+
+// Change-driven in-block kernel (every sweep after the first), exactly
+// equivalent to the sequential order: a column whose code does not change
+// alters no other column, so the cost is (number of changed columns + 1)
+// data-parallel passes (chg_decide).
+template <int B, bool FULL>
+__global__ void __launch_bounds__(1024, 1) k_cd_block_chg(const CdArgs a) {
+    using C = CdCfg<B>;
+    constexpr int CPL = C::CPL;
+    extern __shared__ __align__(16) float cd_smem[];
+    float *tri = cd_smem;
+    uint64_t *bar = reinterpret_cast<uint64_t *>(cd_smem + C::PACK);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t i = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + warp;
+    const bool row_ok = i < a.q;
+    float t[CPL], st[CPL];
+    if (!cd_prologue<B, FULL>(a, tri, bar, i, row_ok, lane, t, st)) return;
+    if (!row_ok) return;
+    float code[CPL], dlt[CPL];
+    const float s = a.scale[i];
+    double dfacc = 0.0;
+    chg_decide<B, FULL>(tri, a.d + a.b0, a.bw, a.maxq, s * s, a.rowdf != nullptr, lane, t, st, code, dlt, dfacc);
+    if (a.rowdf) {
+        dfacc = warp_sum(dfacc);
         if (lane == 0) a.rowdf[i] += dfacc;
     }
-    cd_epilogue<B, FULL>(a, i, lane, code, dlt, true);
+    if (a.lent)
+        cd_epilogue<B, FULL, true>(a, a.b0, a.bw, i, lane, code, dlt, true);
+    else
+        cd_epilogue<B, FULL, false>(a, a.b0, a.bw, i, lane, code, dlt, true);
+}
+
+// One block of one row in the persistent list kernel: stage t = R + the
+// change-list correction (storing it back as the block's base when the window
+// held a change), wait for the block's packed Sigma_bar, decide, write back.
+// Returns false when the wait gave up.
+template <int B, bool FULL, bool LATE>
+__device__ __forceinline__ bool rows_block(const CdArgs &a, int64_t b0, int bw_, const float *tri, uint64_t *bar,
+                                           uint32_t parity, int64_t i, bool row_ok, int lane, float s2,
+                                           double &dfacc, int &nchg) {
+    constexpr int CPL = B / 32;
+    const int bw = FULL ? B : bw_;
+    const int64_t ii = row_ok ? i : 0;
+    float r_[CPL], ps[CPL], st[CPL], t[CPL];
+#pragma unroll
+    for (int h = 0; h < CPL; ++h) {
+        const int l = 32 * h + lane;
+        const bool ok = row_ok && (FULL || l < bw);
+        r_[h] = ok ? a.R[ii * a.ldr + b0 + l] : 0.0f;
+        st[h] = ok ? static_cast<float>(a.codes[ii * a.ldc + b0 + l]) : 0.0f;
+        ps[h] = 0.0f;
+    }
+    const bool changed = list_correction<B, FULL>(a, b0, bw, ii, row_ok, lane, ps);
+#pragma unroll
+    for (int h = 0; h < CPL; ++h) t[h] = r_[h] + ps[h];
+    if (changed) {
+#pragma unroll
+        for (int h = 0; h < CPL; ++h) {
+            const int l = 32 * h + lane;
+            if (row_ok && (FULL || l < bw)) a.R[ii * a.ldr + b0 + l] = t[h];
+        }
+    }
+    if (!LATE && !mbar_wait_bounded(bar, parity, nullptr)) return false;
+    if (!row_ok) return true;
+    float code[CPL], dlt[CPL];
+    nchg += chg_decide<B, FULL, LATE>(tri, a.d + b0, bw, a.maxq, s2, true, lane, t, st, code, dlt, dfacc,
+                                      a.sbar + b0 * a.lds + b0, a.lds);
+    cd_epilogue<B, FULL, true>(a, b0, bw, i, lane, code, dlt, true);
+    return true;
+}
+
+// Rolling-window sweeps t_begin .. t_end-1 with the change-list correction,
+// persistent over column blocks and sweeps.  With the correction taken from
+// each row's own change lists, rows need nothing from one another (rows are
+// independent given Sigma, Sec. 3.2), so a CTA keeps its rows (one per warp)
+// for all its sweeps.  Each sweep, a CTA picks one of two modes from the
+// number of changes its rows made in the previous sweep (the entries of the
+// lists at sweep start):
+//   lockstep: the warps step through the blocks together to share the packed
+//     Sigma_bar block in shared memory, whose bulk copy overlaps the gathers
+//     (many in-block changes per row: early sweeps);
+//   free: every warp runs through the blocks on its own and reads the coupling
+//     row of each in-block change from the fp32 Sigma_bar in global memory
+//     (few changes: no block barriers, no copies).
+// first_lockstep forces lockstep for the first sweep (its lists are empty
+// after a residual refresh although many codes are about to change).
+// Per sweep and row the objective change goes to rowdf_t[t - t_begin][i]; with
+// sweep_codes the row's codes after each sweep are copied out.
+template <int B>
+__global__ void __launch_bounds__(1024, 1) k_cd_rows_lists(const CdArgs a, int t_begin, int t_end,
+                                                           double *rowdf_t, uint8_t *sweep_codes,
+                                                           int first_lockstep, int free_max_changes) {
+    using C = CdCfg<B>;
+    extern __shared__ __align__(16) float cd_smem[];
+    float *tri = cd_smem;
+    uint64_t *bar = reinterpret_cast<uint64_t *>(cd_smem + C::PACK);
+    __shared__ int s_bad;
+    __shared__ int s_chg[C::MAX_WARPS];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int nwarps = static_cast<int>(blockDim.x >> 5);
+    const int64_t i = static_cast<int64_t>(blockIdx.x) * nwarps + warp;
+    const bool row_ok = i < a.q;
+    if (threadIdx.x == 0) {
+        mbar_init(bar, 1);
+        fence_mbar_init();
+        s_bad = 0;
+    }
+    const float s = row_ok ? a.scale[i] : 1.0f;
+    const float s2 = s * s;
+    // changes of this row in the previous sweep = entries of its lists now
+    int prev = 0;
+    if (row_ok) {
+        for (int c0 = 0; c0 < a.nblk; c0 += 32) {
+            int cnt = (c0 + lane < a.nblk) ? a.lcnt[i * a.nblk + c0 + lane] : 0;
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, o);
+            prev += cnt;
+        }
+    }
+    uint32_t use = 0;
+    for (int t = t_begin; t < t_end; ++t) {
+        if (lane == 0) s_chg[warp] = prev;
+        __syncthreads();
+        int cta = 0;
+        for (int w = 0; w < nwarps; ++w) cta += s_chg[w];
+        const bool lockstep = (first_lockstep && t == t_begin) ||
+                              static_cast<int64_t>(cta) > static_cast<int64_t>(free_max_changes) * nwarps;
+        __syncthreads();   // s_chg is rewritten at the next sweep
+        double dfacc = 0.0;
+        int nchg = 0;
+        for (int64_t b0 = 0; b0 < a.p; b0 += B) {
+            const int bw = static_cast<int>((a.p - b0) < B ? (a.p - b0) : B);
+            if (lockstep) {
+                if (threadIdx.x == 0) {
+                    constexpr uint32_t bytes = C::PACK * 4;
+                    mbar_arrive_expect_tx(bar, bytes);
+                    bulk_load(tri, a.tri + (b0 / B) * C::PACK, bytes, bar);
+                }
+                const bool ok =
+                    bw == B ? rows_block<B, true, false>(a, b0, bw, tri, bar, use & 1u, i, row_ok, lane, s2, dfacc, nchg)
+                            : rows_block<B, false, false>(a, b0, bw, tri, bar, use & 1u, i, row_ok, lane, s2, dfacc,
+                                                          nchg);
+                ++use;
+                if (!ok) {
+                    set_error(a.err, ERR_TIMEOUT);
+                    s_bad = 1;
+                }
+                // every warp is done with this block's Sigma_bar before the next copy replaces it
+                __syncthreads();
+                if (s_bad) return;
+            } else if (row_ok) {
+                if (bw == B)
+                    rows_block<B, true, true>(a, b0, bw, tri, bar, 0u, i, row_ok, lane, s2, dfacc, nchg);
+                else
+                    rows_block<B, false, true>(a, b0, bw, tri, bar, 0u, i, row_ok, lane, s2, dfacc, nchg);
+            }
+        }
+        prev = nchg;
+        dfacc = warp_sum(dfacc);
+        if (row_ok) {
+            if (lane == 0) rowdf_t[static_cast<int64_t>(t - t_begin) * a.q + i] = dfacc;
+            if (sweep_codes) {
+                __syncwarp();
+                const uint8_t *src = a.codes + i * a.ldc;
+                uint8_t *dst = sweep_codes + (static_cast<int64_t>(t) * a.q + i) * a.p;
+                for (int64_t j = lane; j < a.p; j += 32) dst[j] = src[j];
+            }
+        }
+    }
+}
+
+// obj[t] = obj[t-1] + sum_i rowdf_t[t][i] for nt sweeps (fixed order); prev may be NULL (0).
+__global__ void k_obj_prefix(const double *rowdf_t, int64_t q, int nt, const double *prev, double *out) {
+    __shared__ double sw[32];
+    double run = prev ? *prev : 0.0;
+    for (int t = 0; t < nt; ++t) {
+        double acc = 0.0;
+        for (int64_t k = threadIdx.x; k < q; k += blockDim.x) acc += rowdf_t[static_cast<int64_t>(t) * q + k];
+        acc = warp_sum(acc);
+        if ((threadIdx.x & 31) == 0) sw[threadIdx.x >> 5] = acc;
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            for (int w = 0; w < (int)(blockDim.x >> 5); ++w) run += sw[w];
+            out[t] = run;
+        }
+        __syncthreads();
+    }
 }
 
 template <int B, bool FULL, bool SEQ>
@@ -477,6 +783,41 @@ cudaError_t launch_cd_block(int B, const CdArgs &a, int nsm, cudaStream_t s) {
 }
 
 int64_t packed_diag_floats(int64_t p, int B) { return ceil_div(p, B) * packed_block_floats(B); }
+
+template <int B>
+static cudaError_t launch_cd_rows_b(const CdArgs &a, int t_begin, int t_end, double *rowdf_t,
+                                   uint8_t *sweep_codes, int first_lockstep, int free_max_changes, int nsm,
+                                   cudaStream_t s) {
+    using C = CdCfg<B>;
+    cudaError_t e = cudaFuncSetAttribute(k_cd_rows_lists<B>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+    if (e != cudaSuccess) return e;
+    int64_t warps = ceil_div(a.q, nsm);
+    if (warps > C::MAX_WARPS) warps = C::MAX_WARPS;
+    if (warps < 1) warps = 1;
+    const unsigned grid = static_cast<unsigned>(ceil_div(a.q, warps));
+    k_cd_rows_lists<B><<<grid, static_cast<unsigned>(32 * warps), C::SMEM, s>>>(
+        a, t_begin, t_end, rowdf_t, sweep_codes, first_lockstep, free_max_changes);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_cd_rows_lists(int B, const CdArgs &a, int t_begin, int t_end, double *rowdf_t,
+                                 uint8_t *sweep_codes, int first_lockstep, int free_max_changes, int nsm,
+                                 cudaStream_t s) {
+    if (!a.sbar || !a.lent || !a.lcnt || a.first_sweep || t_end <= t_begin) return cudaErrorInvalidValue;
+    const int f = first_lockstep, m = free_max_changes;
+    switch (B) {
+        case 64: return launch_cd_rows_b<64>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, nsm, s);
+        case 128: return launch_cd_rows_b<128>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, nsm, s);
+        case 256: return launch_cd_rows_b<256>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, nsm, s);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
+cudaError_t launch_obj_prefix(const double *rowdf_t, int64_t q, int nt, const double *prev, double *out,
+                              cudaStream_t s) {
+    k_obj_prefix<<<1, 1024, 0, s>>>(rowdf_t, q, nt, prev, out);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_pack_diag(const __nv_bfloat16 *snt, int64_t ldn, int64_t p, int B, float *out,
                              cudaStream_t s) {
@@ -651,6 +992,13 @@ cudaError_t launch_sigma_norm(const float *S, int64_t lds, int64_t p, float *d, 
                               int64_t ldn, unsigned *err, cudaStream_t s) {
     k_sigma_diag<<<static_cast<unsigned>(ceil_div(p, 256)), 256, 0, s>>>(S, lds, p, d, err);
     k_sigma_planes<<<row_grid(p, p), 256, 0, s>>>(S, lds, p, d, snt, ldn, err);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_sigma_bar_rows(const float *S, int64_t lds, int64_t p, const float *d, float *sbar,
+                                  int64_t ld, cudaStream_t s) {
+    const dim3 grid(static_cast<unsigned>(ceil_div(ld, 32)), static_cast<unsigned>(ceil_div(p, 32)));
+    k_sigma_bar_rows<<<grid, 256, 0, s>>>(S, lds, p, d, sbar, ld);
     return cudaGetLastError();
 }
 

@@ -18,6 +18,13 @@ struct CdArgs {
     const float *part;              // split-K partials [nsplit][q][ldpart] (t-units)
     int nsplit;
     int64_t part_stride, ldpart;
+    // Change lists (rolling window): per row and column block, the changes of
+    // that block's most recent visit, entry = column offset | (int16 Delta' << 16).
+    const float *sbar;              // non-NULL: correction from the lists x fp32 Sigma_bar rows
+    int64_t lds;                    // leading dimension of sbar
+    int nblk;                       // column blocks per row
+    int *lcnt;                      // [q][nblk] entry counts
+    uint32_t *lent;                 // [q][nblk][B] entries; non-NULL: record this visit's changes
     const float *tri;               // packed diagonal blocks of Sigma_bar (launch_pack_diag)
     const float *scale, *zero;
     const float *d;                 // Sigma_jj (objective change of each decision)
@@ -29,7 +36,7 @@ struct CdArgs {
     int64_t ldc;
     __nv_bfloat16 *qf;              // out: C - z
     int64_t ldq;
-    __nv_bfloat16 *dp;              // out: Delta' hi plane (mid / lo planes dp_plane_rows apart)
+    __nv_bfloat16 *dp;              // out: Delta' hi plane (mid / lo planes dp_plane_rows apart), or NULL
     int64_t ldd, dp_plane_rows;
     unsigned *err;
 };
@@ -53,6 +60,9 @@ cudaError_t launch_grid(const void *W, int w_bf16, int64_t ldw, const float *H, 
                         int64_t p, int bits, float *scale, float *zero, unsigned *err, cudaStream_t s);
 cudaError_t launch_sigma_norm(const float *S, int64_t lds, int64_t p, float *d, __nv_bfloat16 *snt,
                               int64_t ldn, unsigned *err, cudaStream_t s);
+// fp32 Sigma_bar, row k = the coupling of column k to every column (ld columns, zero-padded).
+cudaError_t launch_sigma_bar_rows(const float *S, int64_t lds, int64_t p, const float *d, float *sbar,
+                                  int64_t ld, cudaStream_t s);
 cudaError_t launch_make_planes(const void *W, int w_bf16, int64_t ldw, int64_t q, int64_t p,
                                int split, __nv_bfloat16 *out, int64_t ldo, cudaStream_t s);
 cudaError_t launch_init_residual(const void *W, int w_bf16, int64_t ldw, const float *H, int64_t ldh,
@@ -63,6 +73,18 @@ cudaError_t launch_obj_step(double *rowdf, int64_t q, const double *prev, double
 cudaError_t launch_codes_to_qf(const uint8_t *codes, int64_t ldc, const float *zero, int64_t q,
                                int64_t p, __nv_bfloat16 *qf, int64_t ldq, cudaStream_t s);
 cudaError_t launch_cd_block(int B, const CdArgs &a, int nsm, cudaStream_t s);
+// Sweeps [t_begin, t_end) with the change-list correction in one persistent launch
+// (a.sbar, a.lcnt, a.lent set; a.b0 / a.bw / a.part unused); the objective change of
+// sweep t and row i goes to rowdf_t[(t - t_begin) q + i]; sweep_codes (optional) gets
+// the codes after each sweep at [t][q][p].  A CTA runs a sweep in the free mode when
+// its rows made at most free_max_changes changes each (on average) in the previous
+// sweep; first_lockstep forces the lockstep mode for the first sweep.
+cudaError_t launch_cd_rows_lists(int B, const CdArgs &a, int t_begin, int t_end, double *rowdf_t,
+                                 uint8_t *sweep_codes, int first_lockstep, int free_max_changes, int nsm,
+                                 cudaStream_t s);
+// obj[t] = obj[t-1] + sum_i rowdf_t[t][i] for t < nt, starting from *prev (or 0).
+cudaError_t launch_obj_prefix(const double *rowdf_t, int64_t q, int nt, const double *prev, double *out,
+                              cudaStream_t s);
 int64_t packed_diag_floats(int64_t p, int B);
 cudaError_t launch_pack_diag(const __nv_bfloat16 *snt, int64_t ldn, int64_t p, int B, float *out,
                              cudaStream_t s);

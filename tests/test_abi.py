@@ -38,8 +38,9 @@ def test_status_strings_and_version(lib):
 
 
 def test_opts_struct_matches_header():
-    # 4 ints, 4 pointers, 1 size_t, 1 pointer on LP64
-    assert ctypes.sizeof(qe.QEOpts) == 4 * 4 + 4 * 8 + 8 + 8
+    # 5 ints (padded to 8-byte alignment), 4 pointers, 1 size_t, 1 pointer on LP64
+    assert ctypes.sizeof(qe.QEOpts) == 6 * 4 + 4 * 8 + 8 + 8
+    assert qe.QEOpts.init_codes.offset == 24
 
 
 def _fake(n=1):
@@ -70,6 +71,10 @@ def test_invalid_arguments_rejected_synchronously(lib):
     assert L.qe_quantize_layer(_fake(), qe.QE_F32, 4, 4, 4, _fake(2), 3, 1, ctypes.byref(o), _fake(3),
                                _fake(4), _fake(5), _fake(6), None) == qe.QE_ERR_UNSUPPORTED
     o = qe.QEOpts()
+    o.dense_sweeps = -1
+    assert L.qe_quantize_layer(_fake(), qe.QE_F32, 4, 4, 4, _fake(2), 3, 1, ctypes.byref(o), _fake(3),
+                               _fake(4), _fake(5), _fake(6), None) == qe.QE_ERR_INVALID_ARG
+    o = qe.QEOpts()
     o.block_width = 48
     assert L.qe_quantize_layer(_fake(), qe.QE_F32, 4, 4, 4, _fake(2), 3, 1, ctypes.byref(o), _fake(3),
                                _fake(4), _fake(5), _fake(6), None) == qe.QE_ERR_UNSUPPORTED
@@ -94,5 +99,8 @@ def test_invalid_arguments_rejected_synchronously(lib):
 def test_workspace_size_grows_with_shape(lib):
     a = qe.qe_workspace_size(256, 256)
     b = qe.qe_workspace_size(512, 1024)
-    c = qe.qe_workspace_size(512, 1024, outlier=True)
-    assert 0 < a < b < c
+    c = qe.qe_workspace_size(256, 256, outlier=True)
+    d = qe.qe_workspace_size(512, 1024, outlier=True)
+    assert 0 < a < b and 0 < c < d
+    # the plain layer holds at least Sigma_bar as 3 bf16 planes and in fp32, P and R
+    assert b >= 1024 * 1024 * (3 * 2 + 4) + 2 * 512 * 1024 * 4

@@ -142,6 +142,41 @@ def test_layer_parity_multi_tile_ragged(block_width):
     _check_layer(W, Sg, out, 3, 3, free_running=False)
 
 
+@pytest.mark.parametrize("dense_sweeps", [1, 2, 100])
+@pytest.mark.parametrize("block_width,corr_rank", [(64, 8), (256, 0)])
+def test_layer_correction_forms(dense_sweeps, block_width, corr_rank):
+    """The cross-block term from the dense tensor-core GEMM (sweeps <= dense_sweeps)
+    and from the per-row change lists (later sweeps) both meet the parity bar:
+    lists from sweep 2, from sweep 3, and never.  p = 520 leaves a ragged last
+    block (8 columns at B = 64, 8 at B = 256)."""
+    iters = 6
+    W = inputs.layer_weights(260, 520, dtype=torch.bfloat16, seed=61, device="cuda")
+    X = inputs.calib_inputs(520, 4096, dtype=torch.bfloat16, seed=61, device="cuda",
+                            heavy_frac=0.01, heavy_mult=30.0, corr_rank=corr_rank)
+    Sg = qe.qe_build_sigma(X)
+    out = qe.qe_quantize_layer(W, Sg, 3, iters, record_sweeps=True, want_norm=True,
+                               block_width=block_width, dense_sweeps=dense_sweeps)
+    assert qe.qe_sync_status() == qe.QE_OK
+    _check_layer(W, Sg, out, 3, iters, free_running=corr_rank == 0)
+    obj = out["obj"].cpu().numpy()
+    assert np.all(np.diff(obj) <= 1e-6 * obj[:-1])
+
+
+def test_layer_lists_agree_with_dense():
+    """Both forms of the cross-block term reach the same codes and objective
+    (uncorrelated inputs, where no near-midpoint cascade is expected)."""
+    W = inputs.layer_weights(384, 640, dtype=torch.bfloat16, seed=62, device="cuda")
+    X = inputs.calib_inputs(640, 8192, dtype=torch.bfloat16, seed=62, device="cuda",
+                            heavy_frac=0.01, heavy_mult=30.0)
+    Sg = qe.qe_build_sigma(X)
+    a = qe.qe_quantize_layer(W, Sg, 4, 8, dense_sweeps=100)
+    b = qe.qe_quantize_layer(W, Sg, 4, 8, dense_sweeps=1)
+    assert qe.qe_sync_status() == qe.QE_OK
+    parity.check_obj(b["obj"].cpu().numpy(), a["obj"].cpu().numpy(), what="lists vs dense")
+    m = parity.code_match(a["codes"].cpu().numpy(), b["codes"].cpu().numpy())
+    assert m >= parity.CODE_MATCH, f"codes match {m:.5f}"
+
+
 def test_layer_dead_columns_round_to_nearest():
     dead = (5, 77, 130)
     W, X, Sg, out = _layer_case(96, 160, 1024, torch.float32, 4, 3, seed=12, zero_rows=dead)
