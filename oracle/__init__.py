@@ -68,6 +68,12 @@ class Oracle:
         lib.qo_quantease_alg1.argtypes = [_f64p, _i64, _i64, _f64p, _f32p, _f32p, _int, _int,
                                           _u8p, _u8p, _u8p, _f64p, _u8p, _f64p]
         lib.qo_quantease_alg1.restype = _int
+        lib.qo_quantease_alg1_f32.argtypes = [_f64p, _i64, _i64, _f32p, _f32p, _f32p, _int, _int,
+                                              _u8p, _u8p, _u8p, _f64p, _u8p, _f64p]
+        lib.qo_quantease_alg1_f32.restype = _int
+        lib.qo_sigma_pairs_bf16.argtypes = [ctypes.POINTER(ctypes.c_uint16), _i64, _i64, _i64p, _i64p,
+                                            _i64, _f64p]
+        lib.qo_sigma_pairs_bf16.restype = None
         lib.qo_quantease_alg3.argtypes = [_f64p, _i64, _i64, _f64p, _f32p, _f32p, _int, _int,
                                           _u8p, _f64p]
         lib.qo_quantease_alg3.restype = _int
@@ -108,6 +114,18 @@ class Oracle:
         self.lib.qo_sigma(_ptr(X, _f64p), p, n, _ptr(S, _f64p))
         return S
 
+    def sigma_pairs_bf16(self, Xbits, a, b):
+        """Sigma_ab = sum_k X_ak X_bk in binary64 for index arrays a, b; Xbits is the
+        p x n matrix of bfloat16 bit patterns (uint16)."""
+        X = np.ascontiguousarray(Xbits, np.uint16)
+        a = np.ascontiguousarray(a, np.int64)
+        b = np.ascontiguousarray(b, np.int64)
+        out = np.empty(a.size, np.float64)
+        self.lib.qo_sigma_pairs_bf16(X.ctypes.data_as(ctypes.POINTER(ctypes.c_uint16)), X.shape[1],
+                                     X.shape[1], _ptr(a, _i64p), _ptr(b, _i64p), a.size,
+                                     _ptr(out, _f64p))
+        return out
+
     def objective_rows(self, W, codes, scale, zero, S, H=None):
         W = _f64(W)
         q, p = W.shape
@@ -124,9 +142,12 @@ class Oracle:
     def alg1(self, W, S, scale, zero, bits, iters, init_codes=None, forced=None,
              record=False, want_beta=False):
         """Algorithm 1.  Returns dict(codes, obj_rows[iters, q], obj[iters],
-        sweep_codes[iters, q, p] if record, beta[iters, q, p] if want_beta)."""
+        sweep_codes[iters, q, p] if record, beta[iters, q, p] if want_beta).
+        A float32 S is read as is and promoted exactly row by row (same binary64
+        arithmetic, half the host memory); anything else is converted to float64."""
         W = _f64(W)
-        S = _f64(S)
+        f32 = isinstance(S, np.ndarray) and S.dtype == np.float32
+        S = np.ascontiguousarray(S) if f32 else _f64(S)
         q, p = W.shape
         codes = np.empty((q, p), np.uint8)
         obj_rows = np.empty((iters, q), np.float64)
@@ -134,8 +155,9 @@ class Oracle:
         beta = np.empty((iters, q, p), np.float64) if want_beta else None
         ic = None if init_codes is None else np.ascontiguousarray(init_codes, np.uint8)
         fc = None if forced is None else np.ascontiguousarray(forced, np.uint8)
-        rc = self.lib.qo_quantease_alg1(
-            _ptr(W, _f64p), q, p, _ptr(S, _f64p),
+        fn = self.lib.qo_quantease_alg1_f32 if f32 else self.lib.qo_quantease_alg1
+        rc = fn(
+            _ptr(W, _f64p), q, p, _ptr(S, _f32p if f32 else _f64p),
             _ptr(np.ascontiguousarray(scale, np.float32), _f32p),
             _ptr(np.ascontiguousarray(zero, np.float32), _f32p), bits, iters,
             _ptr(ic, _u8p), _ptr(fc, _u8p), _ptr(codes, _u8p), _ptr(obj_rows, _f64p),

@@ -110,16 +110,72 @@ void qo_sigma(const double *X, int64_t p, int64_t n, double *S)
     }
 }
 
+/* A bfloat16 bit pattern is the upper half of a binary32: promote it exactly. */
+static double qo_bf16(uint16_t h)
+{
+    const uint32_t u = (uint32_t)h << 16;
+    float f;
+    memcpy(&f, &u, sizeof f);
+    return (double)f;
+}
+
+/*
+ * Selected entries of Sigma = X X^T (Lemma 1): out[m] = sum_k X[a[m]][k] X[b[m]][k]
+ * for X given as bfloat16 bit patterns, row-major with leading dimension ldx.
+ * For checking a Sigma too large to form here entry by entry.
+ */
+void qo_sigma_pairs_bf16(const uint16_t *X, int64_t n, int64_t ldx, const int64_t *a,
+                         const int64_t *b, int64_t npairs, double *out)
+{
+#pragma omp parallel for schedule(dynamic)
+    for (int64_t m = 0; m < npairs; ++m) {
+        const uint16_t *xa = X + a[m] * ldx, *xb = X + b[m] * ldx;
+        double acc = 0.0;
+        for (int64_t k = 0; k < n; ++k)
+            acc += qo_bf16(xa[k]) * qo_bf16(xb[k]);
+        out[m] = acc;
+    }
+}
+
+/*
+ * Sigma as the CD routines read it: binary64, or binary32 promoted exactly row
+ * by row (for layers whose binary64 Sigma would not fit in host memory).  The
+ * arithmetic is binary64 either way.
+ */
+typedef struct {
+    const double *d;
+    const float *f;
+    int64_t p;
+} qo_sig;
+
+/* Row j of Sigma in binary64: a pointer into S->d, or buf filled from S->f. */
+static const double *qo_srow(const qo_sig *S, int64_t j, double *buf)
+{
+    if (S->d)
+        return S->d + j * S->p;
+    const float *r = S->f + j * S->p;
+    for (int64_t k = 0; k < S->p; ++k)
+        buf[k] = (double)r[k];
+    return buf;
+}
+
+/* Scratch row for qo_srow (only a binary32 Sigma needs one). */
+static double *qo_sbuf(const qo_sig *S)
+{
+    return S->d ? NULL : (double *)malloc((size_t)S->p * sizeof(double));
+}
+
 /* d^T Sigma d for one row d (the per-row term of f = tr(D Sigma D^T), proof of Lemma 1). */
-static double qo_quad(const double *d, const double *S, int64_t p)
+static double qo_quad(const double *d, const qo_sig *S, int64_t p, double *buf)
 {
     double f = 0.0;
     for (int64_t a = 0; a < p; ++a) {
         if (d[a] == 0.0)
             continue;
+        const double *Sa = qo_srow(S, a, buf);
         double t = 0.0;
         for (int64_t b = 0; b < p; ++b)
-            t += S[a * p + b] * d[b];
+            t += Sa[b] * d[b];
         f += d[a] * t;
     }
     return f;
@@ -134,6 +190,7 @@ void qo_objective_rows(const double *W, const double *H, const uint8_t *codes,
                        const float *scale, const float *zero, int64_t q, int64_t p,
                        const double *S, double *rows_out)
 {
+    const qo_sig Sg = {S, NULL, p};
 #pragma omp parallel for schedule(dynamic)
     for (int64_t i = 0; i < q; ++i) {
         double *d = (double *)malloc((size_t)p * sizeof(double));
@@ -141,7 +198,7 @@ void qo_objective_rows(const double *W, const double *H, const uint8_t *codes,
             double wh = qo_level(codes[i * p + j], scale[i], zero[i]);
             d[j] = W[i * p + j] - wh - (H ? H[i * p + j] : 0.0);
         }
-        rows_out[i] = qo_quad(d, S, p);
+        rows_out[i] = qo_quad(d, &Sg, p, NULL);
         free(d);
     }
 }
@@ -165,12 +222,12 @@ void qo_objective_rows(const double *W, const double *H, const uint8_t *codes,
  * forced (p codes, may be NULL): use these codes instead of q_i(-u) (teacher
  * forcing; beta~ is still recorded).  beta (p, may be NULL) receives beta~.
  */
-static void qo_sweep_row(const double *S, int64_t p, double s, double z, int maxq,
+static void qo_sweep_row(const qo_sig *S, int64_t p, double s, double z, int maxq,
                          const double *tgt, const double *TS, double *Wh, double *WS,
-                         const uint8_t *forced, uint8_t *codes, double *beta)
+                         const uint8_t *forced, uint8_t *codes, double *beta, double *buf)
 {
     for (int64_t j = 0; j < p; ++j) {
-        const double *Sj = S + j * p;
+        const double *Sj = qo_srow(S, j, buf);
         const double djj = Sj[j];
         int c;
         if (djj > 0.0) {
@@ -194,14 +251,14 @@ static void qo_sweep_row(const double *S, int64_t p, double s, double z, int max
 }
 
 /* y = x Sigma for a row vector x. */
-static void qo_row_times_sigma(const double *x, const double *S, int64_t p, double *y)
+static void qo_row_times_sigma(const double *x, const qo_sig *S, int64_t p, double *y, double *buf)
 {
     for (int64_t k = 0; k < p; ++k)
         y[k] = 0.0;
     for (int64_t l = 0; l < p; ++l) {
         if (x[l] == 0.0)
             continue;
-        const double *Sl = S + l * p;
+        const double *Sl = qo_srow(S, l, buf);
         for (int64_t k = 0; k < p; ++k)
             y[k] += x[l] * Sl[k];
     }
@@ -215,11 +272,11 @@ static void qo_row_times_sigma(const double *x, const double *S, int64_t p, doub
  *   forced      iters*q*p in (may be NULL): teacher-forced codes per sweep
  *   beta        iters*q*p out (may be NULL): beta~ of every update
  */
-int qo_quantease_alg1(const double *W, int64_t q, int64_t p, const double *S,
-                      const float *scale, const float *zero, int bits, int iters,
-                      const uint8_t *init_codes, const uint8_t *forced,
-                      uint8_t *codes, double *obj_rows, uint8_t *sweep_codes,
-                      double *beta)
+static int qo_alg1_core(const double *W, int64_t q, int64_t p, const qo_sig *S,
+                        const float *scale, const float *zero, int bits, int iters,
+                        const uint8_t *init_codes, const uint8_t *forced,
+                        uint8_t *codes, double *obj_rows, uint8_t *sweep_codes,
+                        double *beta)
 {
     const int maxq = (1 << bits) - 1;
     int err = 0;
@@ -229,32 +286,56 @@ int qo_quantease_alg1(const double *W, int64_t q, int64_t p, const double *S,
         double *WS = (double *)malloc((size_t)p * sizeof(double));
         double *TS = (double *)malloc((size_t)p * sizeof(double));
         double *d = (double *)malloc((size_t)p * sizeof(double));
-        if (!Wh || !WS || !TS || !d) {
+        double *buf = qo_sbuf(S);
+        if (!Wh || !WS || !TS || !d || (!S->d && !buf)) {
             err = 1;
         } else {
             const double *Wi = W + i * p;
             const double s = scale[i], z = zero[i];
             for (int64_t j = 0; j < p; ++j)
                 Wh[j] = init_codes ? qo_level(init_codes[i * p + j], s, z) : Wi[j];
-            qo_row_times_sigma(Wh, S, p, WS);
-            qo_row_times_sigma(Wi, S, p, TS);
+            qo_row_times_sigma(Wh, S, p, WS, buf);
+            qo_row_times_sigma(Wi, S, p, TS, buf);
             for (int t = 0; t < iters; ++t) {
                 const size_t off = ((size_t)t * (size_t)q + (size_t)i) * (size_t)p;
                 qo_sweep_row(S, p, s, z, maxq, Wi, TS, Wh, WS,
                              forced ? forced + off : NULL, codes + i * p,
-                             beta ? beta + off : NULL);
+                             beta ? beta + off : NULL, buf);
                 if (sweep_codes)
                     memcpy(sweep_codes + off, codes + i * p, (size_t)p);
                 if (obj_rows) {
                     for (int64_t j = 0; j < p; ++j)
                         d[j] = Wi[j] - Wh[j];
-                    obj_rows[(size_t)t * (size_t)q + (size_t)i] = qo_quad(d, S, p);
+                    obj_rows[(size_t)t * (size_t)q + (size_t)i] = qo_quad(d, S, p, buf);
                 }
             }
         }
-        free(Wh); free(WS); free(TS); free(d);
+        free(Wh); free(WS); free(TS); free(d); free(buf);
     }
     return err;
+}
+
+int qo_quantease_alg1(const double *W, int64_t q, int64_t p, const double *S,
+                      const float *scale, const float *zero, int bits, int iters,
+                      const uint8_t *init_codes, const uint8_t *forced,
+                      uint8_t *codes, double *obj_rows, uint8_t *sweep_codes,
+                      double *beta)
+{
+    const qo_sig Sg = {S, NULL, p};
+    return qo_alg1_core(W, q, p, &Sg, scale, zero, bits, iters, init_codes, forced, codes,
+                        obj_rows, sweep_codes, beta);
+}
+
+/* Algorithm 1 with Sigma given in binary32 (promoted exactly; same arithmetic). */
+int qo_quantease_alg1_f32(const double *W, int64_t q, int64_t p, const float *S,
+                          const float *scale, const float *zero, int bits, int iters,
+                          const uint8_t *init_codes, const uint8_t *forced,
+                          uint8_t *codes, double *obj_rows, uint8_t *sweep_codes,
+                          double *beta)
+{
+    const qo_sig Sg = {NULL, S, p};
+    return qo_alg1_core(W, q, p, &Sg, scale, zero, bits, iters, init_codes, forced, codes,
+                        obj_rows, sweep_codes, beta);
 }
 
 /* ------------------------------------------------------------------------- */
@@ -275,6 +356,7 @@ int qo_quantease_alg3(const double *W, int64_t q, int64_t p, const double *S,
                       uint8_t *codes, double *obj_rows)
 {
     const int maxq = (1 << bits) - 1;
+    const qo_sig Sg = {S, NULL, p};
     double *Sn = (double *)malloc((size_t)p * (size_t)p * sizeof(double));
     if (!Sn)
         return 1;
@@ -333,7 +415,7 @@ int qo_quantease_alg3(const double *W, int64_t q, int64_t p, const double *S,
                     double *d = Ph; /* reuse */
                     for (int64_t j = 0; j < p; ++j)
                         d[j] = Wi[j] - Wh[j];
-                    obj_rows[(size_t)t * (size_t)q + (size_t)i] = qo_quad(d, S, p);
+                    obj_rows[(size_t)t * (size_t)q + (size_t)i] = qo_quad(d, &Sg, p, NULL);
                 }
             }
         }
@@ -452,6 +534,7 @@ int qo_quantease_outlier(const double *W, int64_t q, int64_t p, const double *S,
 {
     const int maxq = (1 << bits) - 1;
     const int64_t N = q * p;
+    const qo_sig Sg = {S, NULL, p};
     int64_t *idx = (int64_t *)malloc((size_t)(s_budget > 0 ? s_budget : 1) * sizeof(int64_t));
     uint8_t *excl = (uint8_t *)calloc((size_t)N, 1);
     double *Wh = (double *)malloc((size_t)N * sizeof(double));
@@ -485,10 +568,10 @@ int qo_quantease_outlier(const double *W, int64_t q, int64_t p, const double *S,
             double *WS = (double *)malloc((size_t)p * sizeof(double));
             for (int64_t j = 0; j < p; ++j)
                 tgt[j] = W[i * p + j] - H[i * p + j];
-            qo_row_times_sigma(tgt, S, p, TS);
-            qo_row_times_sigma(Wh + i * p, S, p, WS);
-            qo_sweep_row(S, p, scale[i], zero[i], maxq, tgt, TS, Wh + i * p, WS,
-                         NULL, codes + i * p, NULL);
+            qo_row_times_sigma(tgt, &Sg, p, TS, NULL);
+            qo_row_times_sigma(Wh + i * p, &Sg, p, WS, NULL);
+            qo_sweep_row(&Sg, p, scale[i], zero[i], maxq, tgt, TS, Wh + i * p, WS,
+                         NULL, codes + i * p, NULL, NULL);
             free(tgt); free(TS); free(WS);
         }
         qo_objective_rows(W, H, codes, scale, zero, q, p, S, rows);
@@ -505,7 +588,7 @@ int qo_quantease_outlier(const double *W, int64_t q, int64_t p, const double *S,
             double *G = (double *)malloc((size_t)p * sizeof(double));
             for (int64_t j = 0; j < p; ++j)
                 D[j] = H[i * p + j] + Wh[i * p + j] - W[i * p + j];
-            qo_row_times_sigma(D, S, p, G);          /* G/2 = (H + What - W) Sigma */
+            qo_row_times_sigma(D, &Sg, p, G, NULL);  /* G/2 = (H + What - W) Sigma */
             for (int64_t j = 0; j < p; ++j)
                 T[i * p + j] = H[i * p + j] - eta * 2.0 * G[j];
             free(D); free(G);

@@ -28,7 +28,7 @@ MUTANTS = [
     ("alg3_P_after_zero_diag", "acc += Wi[k] * Sn[k * p + j];", "if (k != j) acc += Wi[k] * Sn[k * p + j];"),
     ("alg3_drop_last_term", "for (int64_t k = 0; k < j; ++k)   /* k = j adds Sn_jj = 0 */",
      "for (int64_t k = 0; k + 1 < j; ++k)"),
-    ("objective_wrong_index", "t += S[a * p + b] * d[b];", "t += S[a * p + b] * d[a];"),
+    ("objective_wrong_index", "t += Sa[b] * d[b];", "t += Sa[b] * d[a];"),
     ("topk_reversed_ties", "if (x->idx < y->idx) return -1;      /* tie: smaller linear index first */",
      "if (x->idx < y->idx) return 1;"),
     ("iht_wrong_step_sign", "T[i * p + j] = H[i * p + j] - eta * 2.0 * G[j];",

@@ -231,6 +231,41 @@ def test_sigma_properties():
     assert np.allclose(S @ v, X @ (X.T @ v), rtol=1e-10)
 
 
+def test_sigma_pairs_from_bf16_bits():
+    """Selected Sigma entries from bfloat16 bit patterns: the bit decoding on
+    hand-picked patterns, then every entry against a numpy binary64 X X^T."""
+    pat = np.array([[0x3F80, 0xC000, 0x3E80, 0x0000, 0x8000, 0x4049]], np.uint16)
+    vals = np.array([1.0, -2.0, 0.25, 0.0, -0.0, 3.140625])
+    got = O.sigma_pairs_bf16(pat, np.zeros(1, np.int64), np.zeros(1, np.int64))
+    assert got[0] == float(np.sum(vals * vals))
+    rng = np.random.default_rng(8)
+    X = rng.normal(size=(40, 300)).astype(np.float32)
+    X[5] *= 30.0
+    bits = (X.view(np.uint32) >> 16).astype(np.uint16)          # truncate to bfloat16
+    Xb = (bits.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    a = rng.integers(0, 40, size=500)
+    b = rng.integers(0, 40, size=500)
+    a[:40] = np.arange(40)
+    b[:40] = np.arange(40)                                       # the diagonal
+    ref = np.einsum("ij,ij->i", Xb[a], Xb[b])
+    out = O.sigma_pairs_bf16(bits, a, b)
+    assert np.allclose(out, ref, rtol=1e-13, atol=1e-13 * np.abs(ref).max())
+    assert np.array_equal(out[:40], np.diag(O.sigma(Xb)))       # same sums, same order
+
+
+def test_alg1_reads_binary32_sigma_exactly():
+    """A binary32 Sigma is promoted exactly: the same run as with its binary64 copy."""
+    rng = np.random.default_rng(9)
+    W, X = _rand_layer(rng, 9, 40, 200, heavy=(3,), corr=True)
+    S32 = O.sigma(X).astype(np.float32)
+    s, z = O.grid(W, 3)
+    a = O.alg1(W, S32, s, z, 3, 3, want_beta=True)
+    b = O.alg1(W, S32.astype(np.float64), s, z, 3, 3, want_beta=True)
+    assert np.array_equal(a["codes"], b["codes"])
+    assert np.array_equal(a["obj_rows"], b["obj_rows"])
+    assert np.array_equal(a["beta"], b["beta"])
+
+
 # --------------------------------------------------------------------------
 # invariances: scaling X, permuting / sub-setting rows (Sec. 3.2, rows independent)
 # --------------------------------------------------------------------------
