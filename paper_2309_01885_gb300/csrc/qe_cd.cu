@@ -283,25 +283,30 @@ __device__ __forceinline__ bool list_correction(const CdArgs &a, int64_t b0, int
             for (int e0 = 0; e0 < c; e0 += 32) {
                 const uint32_t mine = (e0 + lane < c) ? seg[e0 + lane] : 0u;
                 const int ne = (c - e0) < 32 ? (c - e0) : 32;
+                // four changes in flight per step (the gather is bound by loads in flight);
+                // the sum still runs over the changes in list order
                 int u = 0;
-                for (; u + 2 <= ne; u += 2) {
-                    const uint32_t e1 = __shfl_sync(0xffffffffu, mine, u);
-                    const uint32_t e2 = __shfl_sync(0xffffffffu, mine, u + 1);
-                    const float *r1 = sbk + static_cast<int64_t>(e1 & 0xffffu) * a.lds;
-                    const float *r2 = sbk + static_cast<int64_t>(e2 & 0xffffu) * a.lds;
-                    const float d1 = static_cast<float>(static_cast<int16_t>(e1 >> 16));
-                    const float d2 = static_cast<float>(static_cast<int16_t>(e2 >> 16));
-                    float v1[CPL], v2[CPL];
+                for (; u + 4 <= ne; u += 4) {
+                    const float *r[4];
+                    float dv[4];
 #pragma unroll
-                    for (int h = 0; h < CPL; ++h) {
-                        const bool ok = FULL || 32 * h + lane < bw;
-                        v1[h] = ok ? __ldg(r1 + 32 * h) : 0.0f;
-                        v2[h] = ok ? __ldg(r2 + 32 * h) : 0.0f;
+                    for (int e = 0; e < 4; ++e) {
+                        const uint32_t ev = __shfl_sync(0xffffffffu, mine, u + e);
+                        r[e] = sbk + static_cast<int64_t>(ev & 0xffffu) * a.lds;
+                        dv[e] = static_cast<float>(static_cast<int16_t>(ev >> 16));
                     }
+                    float v[4][CPL];
 #pragma unroll
-                    for (int h = 0; h < CPL; ++h) ps[h] = fmaf(d2, v2[h], fmaf(d1, v1[h], ps[h]));
+                    for (int e = 0; e < 4; ++e)
+#pragma unroll
+                        for (int h = 0; h < CPL; ++h)
+                            v[e][h] = (FULL || 32 * h + lane < bw) ? __ldg(r[e] + 32 * h) : 0.0f;
+#pragma unroll
+                    for (int h = 0; h < CPL; ++h)
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) ps[h] = fmaf(dv[e], v[e][h], ps[h]);
                 }
-                if (u < ne) {
+                for (; u < ne; ++u) {
                     const uint32_t e1 = __shfl_sync(0xffffffffu, mine, u);
                     const float *r1 = sbk + static_cast<int64_t>(e1 & 0xffffu) * a.lds;
                     const float d1 = static_cast<float>(static_cast<int16_t>(e1 >> 16));
@@ -604,18 +609,18 @@ __device__ __forceinline__ bool rows_block(const CdArgs &a, int64_t b0, int bw_,
     constexpr int CPL = B / 32;
     const int bw = FULL ? B : bw_;
     const int64_t ii = row_ok ? i : 0;
-    float r_[CPL], ps[CPL], st[CPL], t[CPL];
+    float ps[CPL], st[CPL], t[CPL];
+#pragma unroll
+    for (int h = 0; h < CPL; ++h) ps[h] = 0.0f;
+    // the gathers first (they hold the registers), then the block's base and codes
+    const bool changed = list_correction<B, FULL>(a, b0, bw, ii, row_ok, lane, ps);
 #pragma unroll
     for (int h = 0; h < CPL; ++h) {
         const int l = 32 * h + lane;
         const bool ok = row_ok && (FULL || l < bw);
-        r_[h] = ok ? a.R[ii * a.ldr + b0 + l] : 0.0f;
+        t[h] = (ok ? a.R[ii * a.ldr + b0 + l] : 0.0f) + ps[h];
         st[h] = ok ? static_cast<float>(a.codes[ii * a.ldc + b0 + l]) : 0.0f;
-        ps[h] = 0.0f;
     }
-    const bool changed = list_correction<B, FULL>(a, b0, bw, ii, row_ok, lane, ps);
-#pragma unroll
-    for (int h = 0; h < CPL; ++h) t[h] = r_[h] + ps[h];
     if (changed) {
 #pragma unroll
         for (int h = 0; h < CPL; ++h) {
@@ -644,13 +649,17 @@ __device__ __forceinline__ bool rows_block(const CdArgs &a, int64_t b0, int bw_,
 //     (many in-block changes per row: early sweeps);
 //   free: every warp runs through the blocks on its own and reads the coupling
 //     row of each in-block change from the fp32 Sigma_bar in global memory
-//     (few changes: no block barriers, no copies).
+//     (few changes: no block barriers, no copies).  A CTA that goes free stays
+//     free for its remaining sweeps (correct at any density), so its warps no
+//     longer meet between sweeps, and a row at a fixed point skips its sweeps.
 // first_lockstep forces lockstep for the first sweep (its lists are empty
 // after a residual refresh although many codes are about to change).
 // Per sweep and row the objective change goes to rowdf_t[t - t_begin][i]; with
 // sweep_codes the row's codes after each sweep are copied out.
+constexpr int kRowsMaxWarps = 28;   // rows per CTA of the persistent kernel (896 threads: 72 registers)
+
 template <int B>
-__global__ void __launch_bounds__(1024, 1) k_cd_rows_lists(const CdArgs a, int t_begin, int t_end,
+__global__ void __launch_bounds__(32 * kRowsMaxWarps, 1) k_cd_rows_lists(const CdArgs a, int t_begin, int t_end,
                                                            double *rowdf_t, uint8_t *sweep_codes,
                                                            int first_lockstep, int free_max_changes) {
     using C = CdCfg<B>;
@@ -658,7 +667,7 @@ __global__ void __launch_bounds__(1024, 1) k_cd_rows_lists(const CdArgs a, int t
     float *tri = cd_smem;
     uint64_t *bar = reinterpret_cast<uint64_t *>(cd_smem + C::PACK);
     __shared__ int s_bad;
-    __shared__ int s_chg[C::MAX_WARPS];
+    __shared__ int s_chg[kRowsMaxWarps];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nwarps = static_cast<int>(blockDim.x >> 5);
     const int64_t i = static_cast<int64_t>(blockIdx.x) * nwarps + warp;
@@ -681,28 +690,45 @@ __global__ void __launch_bounds__(1024, 1) k_cd_rows_lists(const CdArgs a, int t
         }
     }
     uint32_t use = 0;
+    bool free_run = false;   // CTA-uniform; once set, the warps run their remaining sweeps alone
     for (int t = t_begin; t < t_end; ++t) {
-        if (lane == 0) s_chg[warp] = prev;
-        __syncthreads();
-        int cta = 0;
-        for (int w = 0; w < nwarps; ++w) cta += s_chg[w];
-        const bool lockstep = (first_lockstep && t == t_begin) ||
-                              static_cast<int64_t>(cta) > static_cast<int64_t>(free_max_changes) * nwarps;
-        __syncthreads();   // s_chg is rewritten at the next sweep
+        const bool forced_lockstep = first_lockstep && t == t_begin;
+        if (!free_run) {
+            if (lane == 0) s_chg[warp] = prev;
+            __syncthreads();
+            int cta = 0;
+            for (int w = 0; w < nwarps; ++w) cta += s_chg[w];
+            free_run = !forced_lockstep &&
+                       static_cast<int64_t>(cta) <= static_cast<int64_t>(free_max_changes) * nwarps;
+            __syncthreads();   // s_chg is rewritten at the next sweep
+        }
         double dfacc = 0.0;
         int nchg = 0;
-        for (int64_t b0 = 0; b0 < a.p; b0 += B) {
-            const int bw = static_cast<int>((a.p - b0) < B ? (a.p - b0) : B);
-            if (lockstep) {
+        if (free_run) {
+            // A row whose previous sweep changed nothing is at a fixed point: its window
+            // is empty, so every block stages the values it decided on last time.
+            if (row_ok && prev > 0) {
+                for (int64_t b0 = 0; b0 < a.p; b0 += B) {
+                    const int bw = static_cast<int>((a.p - b0) < B ? (a.p - b0) : B);
+                    if (bw == B)
+                        rows_block<B, true, true>(a, b0, bw, tri, bar, 0u, i, row_ok, lane, s2, dfacc, nchg);
+                    else
+                        rows_block<B, false, true>(a, b0, bw, tri, bar, 0u, i, row_ok, lane, s2, dfacc, nchg);
+                }
+            }
+        } else {
+            for (int64_t b0 = 0; b0 < a.p; b0 += B) {
+                const int bw = static_cast<int>((a.p - b0) < B ? (a.p - b0) : B);
                 if (threadIdx.x == 0) {
                     constexpr uint32_t bytes = C::PACK * 4;
                     mbar_arrive_expect_tx(bar, bytes);
                     bulk_load(tri, a.tri + (b0 / B) * C::PACK, bytes, bar);
                 }
                 const bool ok =
-                    bw == B ? rows_block<B, true, false>(a, b0, bw, tri, bar, use & 1u, i, row_ok, lane, s2, dfacc, nchg)
-                            : rows_block<B, false, false>(a, b0, bw, tri, bar, use & 1u, i, row_ok, lane, s2, dfacc,
-                                                          nchg);
+                    bw == B
+                        ? rows_block<B, true, false>(a, b0, bw, tri, bar, use & 1u, i, row_ok, lane, s2, dfacc, nchg)
+                        : rows_block<B, false, false>(a, b0, bw, tri, bar, use & 1u, i, row_ok, lane, s2, dfacc,
+                                                      nchg);
                 ++use;
                 if (!ok) {
                     set_error(a.err, ERR_TIMEOUT);
@@ -711,11 +737,6 @@ __global__ void __launch_bounds__(1024, 1) k_cd_rows_lists(const CdArgs a, int t
                 // every warp is done with this block's Sigma_bar before the next copy replaces it
                 __syncthreads();
                 if (s_bad) return;
-            } else if (row_ok) {
-                if (bw == B)
-                    rows_block<B, true, true>(a, b0, bw, tri, bar, 0u, i, row_ok, lane, s2, dfacc, nchg);
-                else
-                    rows_block<B, false, true>(a, b0, bw, tri, bar, 0u, i, row_ok, lane, s2, dfacc, nchg);
             }
         }
         prev = nchg;
@@ -792,7 +813,7 @@ static cudaError_t launch_cd_rows_b(const CdArgs &a, int t_begin, int t_end, dou
     cudaError_t e = cudaFuncSetAttribute(k_cd_rows_lists<B>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
     if (e != cudaSuccess) return e;
     int64_t warps = ceil_div(a.q, nsm);
-    if (warps > C::MAX_WARPS) warps = C::MAX_WARPS;
+    if (warps > kRowsMaxWarps) warps = kRowsMaxWarps;
     if (warps < 1) warps = 1;
     const unsigned grid = static_cast<unsigned>(ceil_div(a.q, warps));
     k_cd_rows_lists<B><<<grid, static_cast<unsigned>(32 * warps), C::SMEM, s>>>(

@@ -44,11 +44,12 @@ def check_obj(obj_gpu, obj_oracle, rtol=OBJ_RTOL, what="objective", atol=0.0):
     return float(rel.max())
 
 
-def teacher_forced(W64, S64, scale, zero, bits, sweep_codes_gpu, init_codes=None):
+def teacher_forced(W64, S64, scale, zero, bits, sweep_codes_gpu, init_codes=None, want_run=False):
     """Replay the GPU trajectory through Algorithm 1 with its own codes forced:
     every GPU code must be the nearest level of the fp64 beta~ unless beta~
     sits within MIDPOINT_TOL (in grid steps) of a rounding midpoint.
-    Returns (number of near-midpoint disagreements, number of checks)."""
+    Returns (number of near-midpoint disagreements, number of checks), plus the
+    oracle's replay (objective of the GPU's codes after each sweep) with want_run."""
     O = oracle.get()
     iters = sweep_codes_gpu.shape[0]
     r = O.alg1(W64, S64, scale, zero, bits, iters, init_codes=init_codes,
@@ -67,6 +68,9 @@ def teacher_forced(W64, S64, scale, zero, bits, sweep_codes_gpu, init_codes=None
         ok = near & neighbour
         assert np.all(ok), (f"{np.sum(~ok)} GPU codes are not the nearest level and not near a "
                             f"midpoint; worst |frac-0.5| = {np.min(np.abs(frac[~ok] - 0.5)):.3e}")
+    if want_run:
+        del r["beta"]
+        return int(bad.sum()), int(bad.size), r
     return int(bad.sum()), int(bad.size)
 
 
