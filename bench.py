@@ -121,9 +121,9 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
-def traffic_per_launch(kernel: str):
-    """DRAM bytes per launch of `kernel` from the committed ncu summary, if the
-    kernel sources are unchanged since it was taken (else None)."""
+def traffic_per_launch(kernel: str, launches_per_step: int):
+    """DRAM bytes per launch from the committed ncu summary (bytes of all launches of
+    one bench step), if the kernel sources are unchanged since it was taken (else None)."""
     import hashlib
     path = os.path.join(ROOT, "profiles", "roofline_traffic.json")
     try:
@@ -137,25 +137,45 @@ def traffic_per_launch(kernel: str):
         with open(os.path.join(csrc, name), "rb") as fh:
             h.update(name.encode() + b"\0" + fh.read())
     entry = rec.get(kernel)
-    if not entry or entry.get("csrc_sha256") != h.hexdigest():
+    if not entry or entry.get("csrc_sha256") != h.hexdigest() or not launches_per_step:
         return None
-    return entry.get("dram_bytes_per_launch")
+    return entry.get("dram_bytes_per_step") / launches_per_step
 
 
-def roofline_entry(launches, total_ms, total_flops, expected_launches, pk):
-    """The dominant kernel (per-block trailing GEMM) against the bf16 tensor roofline.
-    achieved = algorithmic flops (2 per deferred column update) / measured time; the
-    kernel executes 3 bf16 MMAs per product (hi/mid/lo planes of Sigma_bar)."""
-    if launches == 0 or total_ms <= 0:
+def gemm_tiles_sigma(p):
+    """Tiles of the Sigma GEMM that run (128 x 256, on or above the diagonal)."""
+    return sum(1 for m0 in range(0, p, 128) for n0 in range(0, p, 256) if n0 + 256 > m0)
+
+
+def roofline_gemm(flops, exec_flops, ms, launches, pk):
+    """k_tc_gemm<256> (Sigma, P, residual refresh, sweep-1 trailing corrections) over one
+    step against the bf16 tensor roofline: achieved = algorithmic flops / measured time.
+    The CD GEMMs execute 3 (or 6) bf16 products per algorithmic product (the hi / mid / lo
+    planes that carry fp32 accuracy), so `executed_tflops` is reported beside it."""
+    if ms <= 0 or launches <= 0:
         return None
-    achieved = total_flops * (launches / expected_launches) / (total_ms / 1e3) / 1e12
-    return {"bound": "tensor", "kernel": "k_tc_gemm<256> trailing block correction",
+    achieved = flops / (ms / 1e3) / 1e12
+    traffic = traffic_per_launch("k_tc_gemm_step", launches)
+    return {"bound": "tensor", "kernel": "k_tc_gemm<256> (Sigma, P, residual, sweep-1 trailing)",
             "achieved": achieved, "peak": pk["bf16_sustained"], "unit": "TFLOP/s",
-            "frac": achieved / pk["bf16_sustained"],
-            "traffic": traffic_per_launch("trail_gemm"),
-            "launches_timed": launches, "avg_launch_us": 1e3 * total_ms / launches,
-            "executed_tflops": 3 * achieved, "split_products": 3,
+            "frac": achieved / pk["bf16_sustained"], "traffic": traffic,
+            "launches_per_step": launches, "avg_launch_us": 1e3 * ms / launches,
+            "executed_tflops": exec_flops / (ms / 1e3) / 1e12,
             "peak_source": f"{pk['source']} bf16 dense sustained (MEASURED_PEAKS.json)"}
+
+
+def roofline_lists(bytes_per_launch, ms, launches, pk):
+    """The persistent change-list CD kernel against the HBM roofline.  Algorithmic bytes
+    of one list sweep: the residual R (4 q p), the codes (q p) and fp32 Sigma_bar (4 p^2)
+    read once; the gathers of Sigma_bar rows re-read it from L2 and are not counted."""
+    if ms <= 0 or launches <= 0:
+        return None
+    achieved = bytes_per_launch / (ms / launches / 1e3) / 1e9
+    return {"bound": "hbm", "kernel": "k_cd_rows_lists<256>", "achieved": achieved, "peak": pk["hbm"],
+            "unit": "GB/s", "frac": achieved / pk["hbm"],
+            "traffic": traffic_per_launch("k_cd_rows_lists_step", launches),
+            "launches_per_step": launches, "avg_launch_us": 1e3 * ms / launches,
+            "peak_source": f"{pk['source']} HBM copy bandwidth (MEASURED_PEAKS.json)"}
 
 
 def cpu_oracle_sample(W64, S64, bits, rows, sweeps):
@@ -281,10 +301,13 @@ def main():
         dist.barrier()
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
-    # the dominant kernel (the per-block trailing GEMM) is timed by CUDA events that the
-    # library records around each of its launches on this stream
+    # the kernels are timed by CUDA events that the library records around each of its
+    # launches on this stream (the Sigma GEMM by the step's own events around qe_build_sigma,
+    # whose only launch it is)
     nblk = (p + 255) // 256                    # default column block width 256
-    dom = qe.Timer([qe.QE_KERNEL_TRAIL_GEMM], capacity=args.steps * nb * cfg.iters * nblk + 16)
+    kinds = [qe.QE_KERNEL_PINIT_GEMM, qe.QE_KERNEL_RESIDUAL_GEMM, qe.QE_KERNEL_TRAIL_GEMM,
+             qe.QE_KERNEL_CD_BLOCK, qe.QE_KERNEL_CD_LISTS]
+    dom = qe.Timer(kinds, capacity=args.steps * nb * (8 + 2 * nblk * (cfg.iters + 1)) + 16)
     t_start.record(stream)
     outs = None
     for k in range(args.steps):
@@ -303,7 +326,7 @@ def main():
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         ms = float(t.item())
 
-    dom_launches, dom_ms = dom.read(qe.QE_KERNEL_TRAIL_GEMM)
+    timed = {k: dom.read(k) for k in kinds}
     dom.close()
 
     # algorithmic flops of the trailing GEMMs of one quantize call (block width 256):
@@ -338,13 +361,26 @@ def main():
               "sigma_dense_equiv_tflops": 2 * p * p * n / (sigma_avg / 1e3) / 1e12,
               "cd_ms": {str(b): v for b, v in zip(cfg.bits, cd_avg)},
               "cd_updates_per_s": q * p * p * cfg.iters * nb / (sum(cd_avg) / 1e3),
-              "roofline": roofline_entry(dom_launches, dom_ms, trail_flops * nb * args.steps,
-                                         trail_launches * nb * args.steps, pk),
               "clocks": clk}
+    # k_tc_gemm<256> over one step: algorithmic and executed flops, measured time
+    gemm_ms = sigma_avg + sum(timed[k][1] for k in kinds[:3]) / args.steps
+    gemm_launches = 1 + sum(timed[k][0] for k in kinds[:3]) // args.steps
+    qpad, ppad = -(-q // 128) * 128, -(-p // 256) * 256
+    gemm_flops = sig_flops + nb * (2 * 2 * q * p * p + trail_flops)
+    gemm_exec = (gemm_tiles_sigma(p) * 2 * 128 * 256 * n
+                 + nb * (2 * 3 * 2 * qpad * ppad * (-(-p // 64) * 64)
+                         + 6 * tri_flops + 3 * (trail_flops - tri_flops)))   # 6 products in sweep 1
+    result["roofline"] = roofline_gemm(gemm_flops, gemm_exec, gemm_ms, gemm_launches, pk)
+    # the persistent change-list kernel: one launch per layer (per 32 list sweeps)
+    list_launches, list_ms = timed[qe.QE_KERNEL_CD_LISTS]
+    n_list = max(cfg.iters - dense, 0)
+    n_chunks = -(-n_list // 32)
+    list_bytes = n_list * (4 * q * p + q * p + 4 * p * p) / n_chunks if n_chunks else 0
+    result["roofline_cd"] = roofline_lists(list_bytes, list_ms / args.steps, list_launches // args.steps, pk)
+
 
     # per-class breakdown of one extra, untimed step (events around every launch)
-    brk = qe.Timer([qe.QE_KERNEL_PINIT_GEMM, qe.QE_KERNEL_RESIDUAL_GEMM, qe.QE_KERNEL_TRAIL_GEMM,
-                    qe.QE_KERNEL_CD_BLOCK], capacity=nb * (2 + cfg.iters * (2 * nblk + 1)) + 16)
+    brk = qe.Timer(kinds, capacity=nb * (8 + 2 * nblk * (cfg.iters + 1)) + 16)
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(stream)
@@ -354,7 +390,8 @@ def main():
         qe.qe_quantize_layer(W, Sigma, b, cfg.iters, workspace=ws, timer=brk, dense_sweeps=args.dense_sweeps)
     torch.cuda.synchronize()
     names = {qe.QE_KERNEL_PINIT_GEMM: "pinit_gemm", qe.QE_KERNEL_RESIDUAL_GEMM: "residual_gemm",
-             qe.QE_KERNEL_TRAIL_GEMM: "trail_gemm", qe.QE_KERNEL_CD_BLOCK: "cd_block"}
+             qe.QE_KERNEL_TRAIL_GEMM: "trail_gemm", qe.QE_KERNEL_CD_BLOCK: "cd_block",
+             qe.QE_KERNEL_CD_LISTS: "cd_lists"}
     breakdown = {"sigma_gemm": {"launches": 1, "ms": e0.elapsed_time(e1)}}
     for k, nm in names.items():
         n_, ms_ = brk.read(k)
@@ -379,12 +416,26 @@ def main():
     if not args.no_e2e:
         Xh = X.cpu().pin_memory()
         Wh = W.cpu().pin_memory()
-        Xd = torch.empty_like(X)
         Wd = torch.empty_like(W)
+        # X stays on the host: qe_build_sigma_host streams it in token chunks through
+        # device buffers, one per chunk, so the next step's copies run while this step's
+        # CD computes (the copy link, ~210 GB/s here, is slower than the Sigma GEMM)
+        chunk = 65536
+        staging = qe.sigma_host_staging(p, chunk, nbuf=-(-n // chunk))
         host_out = [dict(codes=torch.empty(q, p, dtype=torch.uint8).pin_memory(),
                          scales=torch.empty(q).pin_memory(), zeros=torch.empty(q).pin_memory(),
                          obj=torch.empty(cfg.iters, dtype=torch.float64).pin_memory())
                     for _ in cfg.bits]
+        def e2e_step():
+            Wd.copy_(Wh, non_blocking=True)
+            qe.qe_build_sigma_host(Xh, Sigma, staging, chunk)
+            for k, b in enumerate(cfg.bits):
+                o = qe.qe_quantize_layer(Wd, Sigma, b, cfg.iters, workspace=ws,
+                                         dense_sweeps=args.dense_sweeps)
+                for key in ("codes", "scales", "zeros", "obj"):
+                    host_out[k][key].copy_(o[key], non_blocking=True)
+
+        e2e_step()                     # untimed: creates the copy stream and its events
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
         torch.cuda.synchronize()
@@ -392,14 +443,7 @@ def main():
             dist.barrier()
         e0.record(stream)
         for _ in range(args.steps):
-            Xd.copy_(Xh, non_blocking=True)
-            Wd.copy_(Wh, non_blocking=True)
-            qe.qe_build_sigma(Xd, Sigma=Sigma)
-            for k, b in enumerate(cfg.bits):
-                o = qe.qe_quantize_layer(Wd, Sigma, b, cfg.iters, workspace=ws,
-                                         dense_sweeps=args.dense_sweeps)
-                for key in ("codes", "scales", "zeros", "obj"):
-                    host_out[k][key].copy_(o[key], non_blocking=True)
+            e2e_step()
         e1.record(stream)
         torch.cuda.synchronize()
         e2e_ms = e0.elapsed_time(e1) / args.steps

@@ -60,7 +60,8 @@ typedef enum {
     QE_KERNEL_RESIDUAL_GEMM = 1,  /* R = P - What Sigma_bar (+ the fused objective) */
     QE_KERNEL_TRAIL_GEMM = 2,     /* per column block: Delta' Sigma_bar correction (split-K) */
     QE_KERNEL_CD_BLOCK = 3,       /* per column block: the in-block coordinate updates */
-    QE_KERNEL_COUNT = 4
+    QE_KERNEL_CD_LISTS = 4,       /* the sweeps driven by change lists (one persistent launch) */
+    QE_KERNEL_COUNT = 5
 } qe_kernel;
 
 /* Opaque set of CUDA event pairs; see qe_timer_create. */
@@ -159,6 +160,35 @@ qe_status qe_quantize_layer_outlier(const void *W, qe_dtype w_dtype, int64_t q,
                                     float *scales, float *zeros, float *H_val,
                                     int64_t *H_idx, int64_t *H_nnz, double *obj,
                                     double *obj_cd, qe_stream_t stream);
+
+/*
+ * Sigma = X X^T (Lemma 1) for bf16 X held in HOST memory, streamed to the GPU
+ * in chunks of tokens.  (Beyond Lemma 1 the paper has no counterpart: this is
+ * how calibration activations that live on the host reach the GPU.)
+ *   X          host, bf16, feature-major p x n, leading dimension ldx >= n
+ *              (elements).  Page-locked memory (cudaHostAlloc/Register) lets
+ *              the copies run asynchronously; pageable memory is still correct.
+ *   Sigma      device, fp32 p x p as in qe_build_sigma; accumulate as there.
+ *   staging    device, 16-byte aligned, holding nbuf = staging_bytes /
+ *              (p * chunk * 2) chunk buffers, at least 2 (at most 64 are used).
+ *              Caller-owned; it may be reused across calls.
+ *   chunk      tokens per copy, a positive multiple of 64 (wide chunks copy
+ *              faster: rows of chunk * 2 bytes are the copy's unit).
+ * Chunk c is copied on an internal per-device copy stream into buffer c % nbuf
+ * while earlier chunks accumulate on `stream`; a buffer is refilled only after
+ * the GEMM that read it (also one of an earlier call) has finished, so the
+ * copies of one call overlap work queued on `stream` before it (with nbuf >=
+ * the number of chunks, all of them can arrive during that work).  The call
+ * returns once all work is enqueued; X must stay unchanged and allocated until
+ * Sigma is complete on `stream`.  Calls are serialized per device while they
+ * enqueue (the copy stream and its events are shared).
+ * Errors: QE_ERR_INVALID_ARG for bad sizes or pointers, a chunk that is not a
+ * positive multiple of 64, or a staging area that is too small or misaligned
+ * (before anything is enqueued); QE_ERR_CUDA when a copy, event or launch fails.
+ */
+qe_status qe_build_sigma_host(const void *X, int64_t p, int64_t n, int64_t ldx, float *Sigma,
+                              int accumulate, void *staging, size_t staging_bytes, int64_t chunk,
+                              qe_stream_t stream);
 
 /*
  * Sigma = X X^T like qe_build_sigma, but the call never allocates device

@@ -309,6 +309,7 @@ static qe_status prepare(Ctx &c, const void *W, int wbf16, int64_t ldw, const fl
     GemmArgs g = gemm_args(c, static_cast<int>(q), static_cast<int>(p), static_cast<int>(ceil_div(p, 64)),
                            EPI_PINIT);
     set_prods(g, c.wa_planes);
+    g.m_fast = 1;
     g.a_plane_rows = static_cast<int>(q);
     g.b_plane_rows = static_cast<int>(p);
     g.out = Pout;
@@ -341,6 +342,7 @@ static qe_status residual(Ctx &c, const float *scales, const ObjFuse *f = nullpt
     GemmArgs g = gemm_args(c, static_cast<int>(q), static_cast<int>(p), static_cast<int>(ceil_div(p, 64)),
                            EPI_RFULL);
     set_prods(g, 1);
+    g.m_fast = 1;
     g.a_plane_rows = static_cast<int>(q);
     g.b_plane_rows = static_cast<int>(p);
     g.out = c.R;
@@ -751,7 +753,7 @@ qe_status qe_quantize_layer(const void *W, qe_dtype w_dtype, int64_t q, int64_t 
         const int te = (iters - t) < kSweepChunk ? iters : t + kSweepChunk;
         CdArgs a = list_args(c, codes, scales, zeros, bits);
         {
-            Timed tm(c.timer, QE_KERNEL_CD_BLOCK, c.s);
+            Timed tm(c.timer, QE_KERNEL_CD_LISTS, c.s);
             // the lists are empty at the window start (t0): that sweep steps in lockstep
             QE_CK(launch_cd_rows_lists(pl.B, a, t, te, c.rowdft, opts ? opts->sweep_codes : nullptr, t == t0,
                                        kFreeMaxChanges, c.nsm, c.s));

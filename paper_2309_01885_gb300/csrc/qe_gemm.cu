@@ -205,8 +205,10 @@ __global__ void __launch_bounds__(320, 1)
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    const int m0 = blockIdx.y * C::BM;
-    const int n0 = blockIdx.x * BN;
+    // m_fast: consecutive CTAs walk down M, so a wave shares a few B column
+    // slices (each read once from DRAM) instead of sweeping all of B
+    const int m0 = (g.m_fast ? blockIdx.x : blockIdx.y) * C::BM;
+    const int n0 = (g.m_fast ? blockIdx.y : blockIdx.x) * BN;
     // Sigma: a tile whose every element lies strictly below the diagonal is
     // produced by the mirror of its transpose (uniform exit, before any barrier).
     if (g.mode == EPI_SIGMA && n0 + BN <= m0) return;
@@ -389,8 +391,8 @@ static cudaError_t launch_bn(const CUtensorMap &ta, const CUtensorMap &tb, const
     cudaError_t e = cudaFuncSetAttribute(k_tc_gemm<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          C::SMEM_BYTES);
     if (e != cudaSuccess) return e;
-    dim3 grid(static_cast<unsigned>(ceil_div(g.N, BN)), static_cast<unsigned>(ceil_div(g.M, C::BM)),
-              static_cast<unsigned>(splits));
+    const unsigned nt = static_cast<unsigned>(ceil_div(g.N, BN)), mt = static_cast<unsigned>(ceil_div(g.M, C::BM));
+    dim3 grid(g.m_fast ? mt : nt, g.m_fast ? nt : mt, static_cast<unsigned>(splits));
     k_tc_gemm<BN><<<grid, C::THREADS, C::SMEM_BYTES, s>>>(ta, tb, g);
     return cudaGetLastError();
 }
@@ -399,7 +401,7 @@ cudaError_t launch_tc_gemm(int BN, const CUtensorMap &ta, const CUtensorMap &tb,
                            int splits, cudaStream_t s) {
     if (g.M <= 0 || g.N <= 0 || splits < 1 || g.n_prod < 1 || g.n_prod > 6)
         return cudaErrorInvalidValue;
-    if (ceil_div(g.M, 128) > 65535 || splits > 65535) return cudaErrorInvalidValue;
+    if ((g.m_fast ? ceil_div(g.N, BN) : ceil_div(g.M, 128)) > 65535 || splits > 65535) return cudaErrorInvalidValue;
     switch (BN) {
         case 64: return launch_bn<64>(ta, tb, g, splits, s);
         case 128: return launch_bn<128>(ta, tb, g, splits, s);

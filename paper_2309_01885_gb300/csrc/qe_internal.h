@@ -24,6 +24,7 @@ struct GemmArgs {
     int a_plane_rows, b_plane_rows;  // row distance between stacked planes in the maps
     int a_row0, b_row0;       // row offsets of the operand windows
     int mode;
+    int m_fast;               // grid x runs over M tiles (B slices shared within a wave)
     float *out;
     int64_t ldo;
     int64_t split_stride;     // EPI_TRAIL: elements between split slices

@@ -23,9 +23,9 @@ QE_FEATURE_MAJOR, QE_TOKEN_MAJOR = 0, 1
 EXPORTED = ("qe_build_sigma", "qe_quantize_layer", "qe_quantize_layer_outlier",
             "qe_workspace_size", "qe_sync_status", "qe_status_string", "qe_version",
             "qe_build_sigma_static", "qe_timer_create", "qe_timer_read", "qe_timer_reset",
-            "qe_timer_destroy")
+            "qe_timer_destroy", "qe_build_sigma_host")
 QE_KERNEL_PINIT_GEMM, QE_KERNEL_RESIDUAL_GEMM, QE_KERNEL_TRAIL_GEMM, QE_KERNEL_CD_BLOCK, \
-    QE_KERNEL_COUNT = range(5)
+    QE_KERNEL_CD_LISTS, QE_KERNEL_COUNT = range(6)
 
 
 class QEError(RuntimeError):
@@ -76,6 +76,8 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     L.qe_version.restype = ctypes.c_int
     L.qe_build_sigma_static.argtypes = [vp, i32, i32, i64, i64, i64, vp, i32, vp]
     L.qe_build_sigma_static.restype = st
+    L.qe_build_sigma_host.argtypes = [vp, i64, i64, i64, vp, i32, vp, ctypes.c_size_t, i64, vp]
+    L.qe_build_sigma_host.restype = st
     L.qe_timer_create.argtypes = [ctypes.c_uint, i32, ctypes.POINTER(vp)]
     L.qe_timer_create.restype = st
     L.qe_timer_read.argtypes = [vp, i32, ctypes.POINTER(ctypes.c_int), ctypes.POINTER(ctypes.c_double)]
@@ -144,6 +146,24 @@ def qe_build_sigma(X: torch.Tensor, layout: int = QE_FEATURE_MAJOR, Sigma: torch
         Sigma = torch.empty(p, p, dtype=torch.float32, device=X.device)
     _check(load().qe_build_sigma(_ptr(X), _dtype(X), layout, p, n, ld, _ptr(Sigma), int(accumulate),
                                  _stream(stream)), "qe_build_sigma")
+    return Sigma
+
+
+def sigma_host_staging(p: int, chunk: int, nbuf: int = 2, device="cuda") -> torch.Tensor:
+    """A device staging area for qe_build_sigma_host (nbuf >= 2 chunk buffers)."""
+    return torch.empty(nbuf * p * chunk * 2, dtype=torch.uint8, device=device)
+
+
+def qe_build_sigma_host(X: torch.Tensor, Sigma: torch.Tensor, staging: torch.Tensor, chunk: int,
+                        accumulate: bool = False, stream=None) -> torch.Tensor:
+    """Sigma = X X^T for bf16 X (p x n feature-major) in host memory (pin it for the
+    copies to overlap), streamed through `staging` in chunks of `chunk` tokens."""
+    if X.device.type != "cpu" or X.dtype != torch.bfloat16:
+        raise ValueError("qe_build_sigma_host takes a bf16 tensor in host memory")
+    p, n = X.shape
+    _check(load().qe_build_sigma_host(X.data_ptr(), p, n, _rowmajor_ld(X), _ptr(Sigma), int(accumulate),
+                                      _ptr(staging), staging.numel() * staging.element_size(), int(chunk),
+                                      _stream(stream)), "qe_build_sigma_host")
     return Sigma
 
 

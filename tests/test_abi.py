@@ -96,6 +96,21 @@ def test_invalid_arguments_rejected_synchronously(lib):
                             None) == qe.QE_ERR_INVALID_ARG
 
 
+def test_sigma_host_rejects_bad_arguments(lib):
+    L = lib
+    # chunk not a multiple of 64, staging too small, misaligned staging, NULL X, ldx < n
+    assert L.qe_build_sigma_host(_fake(), 8, 100, 100, _fake(2), 0, _fake(3), 1 << 20, 100,
+                                 None) == qe.QE_ERR_INVALID_ARG
+    assert L.qe_build_sigma_host(_fake(), 8, 100, 100, _fake(2), 0, _fake(3), 2 * 8 * 64 * 2 - 2, 64,
+                                 None) == qe.QE_ERR_INVALID_ARG
+    assert L.qe_build_sigma_host(_fake(), 8, 100, 100, _fake(2), 0, ctypes.c_void_p(0x1008), 1 << 20, 64,
+                                 None) == qe.QE_ERR_INVALID_ARG
+    assert L.qe_build_sigma_host(None, 8, 100, 100, _fake(2), 0, _fake(3), 1 << 20, 64,
+                                 None) == qe.QE_ERR_INVALID_ARG
+    assert L.qe_build_sigma_host(_fake(), 8, 100, 99, _fake(2), 0, _fake(3), 1 << 20, 64,
+                                 None) == qe.QE_ERR_INVALID_ARG
+
+
 def test_workspace_size_grows_with_shape(lib):
     a = qe.qe_workspace_size(256, 256)
     b = qe.qe_workspace_size(512, 1024)

@@ -62,6 +62,31 @@ def test_sigma_bf16_token_major_and_accumulate():
     _sigma_check(S2, parity.f64(X))
 
 
+def test_sigma_host_streamed():
+    """Sigma from pinned host X streamed in token chunks (ragged last chunk), the
+    staging area reused by the next calls, and accumulation over two token ranges
+    given as strided views of the host array."""
+    p, n, chunk = 384, 5000, 1024
+    X = inputs.calib_inputs(p, n, dtype=torch.bfloat16, seed=4, device="cuda", heavy_frac=0.02,
+                            heavy_mult=30.0)
+    Xh = X.cpu().pin_memory()
+    staging = qe.sigma_host_staging(p, chunk)
+    S = torch.empty(p, p, dtype=torch.float32, device="cuda")
+    qe.qe_build_sigma_host(Xh, S, staging, chunk)
+    S2 = torch.empty_like(S)
+    qe.qe_build_sigma_host(Xh[:, :2000], S2, staging, chunk)
+    qe.qe_build_sigma_host(Xh[:, 2000:], S2, staging, chunk, accumulate=True)
+    torch.cuda.synchronize()
+    assert qe.qe_sync_status() == qe.QE_OK
+    X64 = parity.f64(X)
+    _sigma_check(S, X64)
+    _sigma_check(S2, X64)
+    Sd = qe.qe_build_sigma(X)
+    torch.cuda.synchronize()
+    rel = (S.double() - Sd.double()).abs().max() / Sd.double().abs().max()
+    assert rel.item() < 1e-6
+
+
 @pytest.mark.parametrize("layout", [qe.QE_FEATURE_MAJOR, qe.QE_TOKEN_MAJOR])
 def test_sigma_fp32(layout):
     p, n = 150, 777
