@@ -82,7 +82,9 @@ class Oracle:
         lib.qo_topk.argtypes = [_f64p, _i64, _i64, _i64p]
         lib.qo_topk.restype = _i64
         lib.qo_quantease_outlier.argtypes = [_f64p, _i64, _i64, _f64p, _int, _int, _i64, _int,
-                                             _u8p, _f32p, _f32p, _f64p, _f64p, _f64p, _f64p, _i64p]
+                                             _u8p, _f32p, _f32p, _f64p, _f64p, _f64p, _f64p, _i64p, _int]
+        lib.qo_topk_columns.argtypes = [_f64p, _i64, _i64, _i64, _i64p]
+        lib.qo_topk_columns.restype = _i64
         lib.qo_quantease_outlier.restype = _int
         self.lib = lib
 
@@ -197,7 +199,14 @@ class Oracle:
         cnt = self.lib.qo_topk(_ptr(T, _f64p), T.size, int(s), _ptr(idx, _i64p))
         return idx[:cnt].copy()
 
-    def outlier(self, W, S, bits, iters, s_budget, power_iters):
+    def topk_columns(self, T, k):
+        """Indices (ascending) of the k columns of T with the largest l2 norms."""
+        T = _f64(T)
+        idx = np.empty(max(T.shape[1], 1), np.int64)
+        cnt = self.lib.qo_topk_columns(_ptr(T, _f64p), T.shape[0], T.shape[1], int(k), _ptr(idx, _i64p))
+        return idx[:cnt].copy()
+
+    def outlier(self, W, S, bits, iters, s_budget, power_iters, structured=False):
         W = _f64(W)
         S = _f64(S)
         q, p = W.shape
@@ -212,7 +221,7 @@ class Oracle:
         rc = self.lib.qo_quantease_outlier(
             _ptr(W, _f64p), q, p, _ptr(S, _f64p), bits, iters, int(s_budget), power_iters,
             _ptr(codes, _u8p), _ptr(scale, _f32p), _ptr(zero, _f32p), _ptr(H, _f64p),
-            _ptr(obj, _f64p), _ptr(obj_cd, _f64p), _ptr(eta, _f64p), _ptr(nnz, _i64p))
+            _ptr(obj, _f64p), _ptr(obj_cd, _f64p), _ptr(eta, _f64p), _ptr(nnz, _i64p), int(structured))
         if rc:
             raise MemoryError("oracle outlier allocation failed")
         return dict(codes=codes, scale=scale, zero=zero, H=H, obj=obj, obj_cd=obj_cd,

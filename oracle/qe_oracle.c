@@ -517,6 +517,42 @@ int64_t qo_topk(const double *T, int64_t N, int64_t s, int64_t *idx_out)
 }
 
 /*
+ * Structured outliers (Sec. 4.3, "Structured Outliers"): in place of the s
+ * largest entries, keep whole columns of T: those with the floor(s / q) largest
+ * l2 norms, which is the Euclidean projection onto matrices with at most that
+ * many nonzero columns.  Ties go to the smaller column index and a column of
+ * zeros is never kept (the rules of P_s, applied to the squared column norms,
+ * summed over the rows in order).  idx_out receives the kept column indices,
+ * ascending; the return value is their number.
+ */
+int64_t qo_topk_columns(const double *T, int64_t q, int64_t p, int64_t k, int64_t *idx_out)
+{
+    double *norm2 = (double *)calloc((size_t)(p > 0 ? p : 1), sizeof(double));
+    for (int64_t i = 0; i < q; ++i)
+        for (int64_t j = 0; j < p; ++j)
+            norm2[j] += T[i * p + j] * T[i * p + j];
+    const int64_t cnt = qo_topk(norm2, p, k, idx_out);
+    free(norm2);
+    return cnt;
+}
+
+/*
+ * The kept entries of T as ascending linear indices: P_s (the s largest |T|),
+ * or with `structured` every entry of the kept columns (zeros included).
+ */
+static int64_t qo_select(const double *T, int64_t q, int64_t p, int64_t s_budget, int structured,
+                         int64_t *idx, int64_t *cols)
+{
+    if (!structured)
+        return qo_topk(T, q * p, s_budget, idx);
+    const int64_t nc = qo_topk_columns(T, q, p, s_budget / q, cols);
+    for (int64_t i = 0; i < q; ++i)
+        for (int64_t r = 0; r < nc; ++r)
+            idx[i * nc + r] = i * p + cols[r];
+    return q * nc;
+}
+
+/*
  * Algorithm 4 (outlier-aware QuantEase), block coordinate descent between What
  * and H (Sec. 4.3):
  *   H = P_s(W); grid from W without the support of H; What = W - H;
@@ -524,27 +560,30 @@ int64_t qo_topk(const double *T, int64_t N, int64_t s, int64_t *idx_out)
  *   per iteration t:
  *     one sweep of Algorithm 1 on every row with target W - H;   obj_cd[t] = g
  *     G = 2 (H + What - W) Sigma;  H = P_s(H - eta G);           obj[t]    = g
+ * With `structured`, P_s is the column selection of qo_topk_columns, both for
+ * the start H and in the IHT step, and the grid leaves out the start columns.
  * Outputs: codes, scale, zero, dense H (q*p), obj, obj_cd (iters each), eta.
  */
 int qo_quantease_outlier(const double *W, int64_t q, int64_t p, const double *S,
                          int bits, int iters, int64_t s_budget, int power_iters,
                          uint8_t *codes, float *scale, float *zero, double *H,
                          double *obj, double *obj_cd, double *eta_out,
-                         int64_t *nnz_out)
+                         int64_t *nnz_out, int structured)
 {
     const int maxq = (1 << bits) - 1;
     const int64_t N = q * p;
     const qo_sig Sg = {S, NULL, p};
     int64_t *idx = (int64_t *)malloc((size_t)(s_budget > 0 ? s_budget : 1) * sizeof(int64_t));
+    int64_t *cols = (int64_t *)malloc((size_t)(p > 0 ? p : 1) * sizeof(int64_t));
     uint8_t *excl = (uint8_t *)calloc((size_t)N, 1);
     double *Wh = (double *)malloc((size_t)N * sizeof(double));
     double *T = (double *)malloc((size_t)N * sizeof(double));
     double *rows = (double *)malloc((size_t)q * sizeof(double));
-    if (!idx || !excl || !Wh || !T || !rows)
+    if (!idx || !cols || !excl || !Wh || !T || !rows)
         return 1;
 
     /* H = P_s(W), grid without the support of H, What = W - H */
-    int64_t nnz = qo_topk(W, N, s_budget, idx);
+    int64_t nnz = qo_select(W, q, p, s_budget, structured, idx, cols);
     memset(H, 0, (size_t)N * sizeof(double));
     for (int64_t k = 0; k < nnz; ++k) {
         H[idx[k]] = W[idx[k]];
@@ -593,7 +632,7 @@ int qo_quantease_outlier(const double *W, int64_t q, int64_t p, const double *S,
                 T[i * p + j] = H[i * p + j] - eta * 2.0 * G[j];
             free(D); free(G);
         }
-        nnz = qo_topk(T, N, s_budget, idx);
+        nnz = qo_select(T, q, p, s_budget, structured, idx, cols);
         memset(H, 0, (size_t)N * sizeof(double));
         for (int64_t k = 0; k < nnz; ++k)
             H[idx[k]] = T[idx[k]];
@@ -607,6 +646,6 @@ int qo_quantease_outlier(const double *W, int64_t q, int64_t p, const double *S,
     }
     if (nnz_out)
         *nnz_out = nnz;
-    free(idx); free(excl); free(Wh); free(T); free(rows);
+    free(idx); free(cols); free(excl); free(Wh); free(T); free(rows);
     return 0;
 }

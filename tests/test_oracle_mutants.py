@@ -34,6 +34,7 @@ MUTANTS = [
     ("iht_wrong_step_sign", "T[i * p + j] = H[i * p + j] - eta * 2.0 * G[j];",
      "T[i * p + j] = H[i * p + j] + eta * 2.0 * G[j];"),
     ("power_wrong_rayleigh", "lam += v[a] * w[a];", "lam += w[a] * w[a];"),
+    ("column_norm_not_squared", "norm2[j] += T[i * p + j] * T[i * p + j];", "norm2[j] += T[i * p + j];"),
 ]
 
 PINS = [
@@ -49,6 +50,8 @@ PINS = [
     pins.test_power_lambda_matches_eigvalsh,
     pins.test_topk_matches_full_sort_with_ties,
     pins.test_outlier_iht_descent_and_budget,
+    pins.test_column_selection_is_the_projection,
+    pins.test_structured_outlier_descent_budget_and_columns,
     golden.test_hand_worked_two_feature_layer,
 ]
 

@@ -359,3 +359,70 @@ def test_outlier_with_zero_budget_reduces_to_algorithm1():
     assert np.array_equal(r["codes"], a1["codes"])
     assert np.allclose(r["obj"], a1["obj"], rtol=1e-12) and np.allclose(r["obj_cd"], a1["obj"], rtol=1e-12)
     assert not np.any(r["H"])
+
+
+# --------------------------------------------------------------------------
+# structured outliers (Sec. 4.3, "Structured Outliers"): whole columns
+# --------------------------------------------------------------------------
+def test_column_selection_is_the_projection():
+    """Keeping the k columns of largest l2 norm is the Euclidean projection onto
+    matrices with at most k nonzero columns: brute force over every subset of k
+    columns, with planted ties (smaller index wins) and a zero column (never kept)."""
+    rng = np.random.default_rng(15)
+    q, p = 5, 7
+    for trial in range(30):
+        T = rng.normal(size=(q, p))
+        T[:, 2] = T[:, 4]                  # equal norms: column 2 ranks first
+        T[:, 6] = 0.0
+        for k in (1, 2, 3):
+            sel = O.topk_columns(T, k)
+            assert np.all(np.diff(sel) > 0) and 6 not in sel and sel.size == k
+            # the kept columns leave the least residual ||T - H||_F^2 (up to rounding:
+            # the planted tie makes two subsets equal in exact arithmetic)
+            res = lambda c: np.sum(np.delete(T, list(c), axis=1) ** 2)
+            best = min(res(c) for c in itertools.combinations(range(p), k))
+            assert res(sel) <= best * (1 + 1e-12)
+            if (2 in sel) != (4 in sel):
+                assert 2 in sel                      # the tie goes to the smaller index
+        norms = np.sum(T * T, axis=0)
+        order = np.lexsort((np.arange(p), -norms))
+        assert np.array_equal(O.topk_columns(T, 4), np.sort(order[:4]))
+    # fewer nonzero columns than k: only those are kept
+    T = np.zeros((q, p))
+    T[:, 3] = 1.0
+    assert np.array_equal(O.topk_columns(T, 3), [3])
+
+
+def test_structured_outlier_descent_budget_and_columns():
+    rng = np.random.default_rng(16)
+    q, p, n = 10, 24, 90
+    W, X = _rand_layer(rng, q, p, n, heavy=(5,), heavy_mult=10.0, corr=True)
+    W[:, [3, 17]] += rng.normal(0, 0.3, size=(q, 2))        # two outlier columns
+    S = O.sigma(X)
+    s_budget = 3 * q + 4                                     # floor(s / q) = 3 columns
+    r = O.outlier(W, S, 3, 8, s_budget, 600, structured=True)
+    cols = np.nonzero(np.any(r["H"] != 0, axis=0))[0]
+    assert cols.size <= 3 and r["nnz"] == q * 3
+    # Lemma 3 carries over (the column selection is a projection): IHT halves never increase g
+    assert np.all(r["obj"] <= r["obj_cd"] * (1 + 1e-10))
+    assert np.all(r["obj_cd"][1:] <= r["obj"][:-1] * (1 + 1e-10))
+    # the grid leaves out the starting columns, those of W with the largest norms
+    start = O.topk_columns(W, 3)
+    assert set(start) >= {3, 17}
+    excl = np.zeros((q, p), np.uint8)
+    excl[:, start] = 1
+    s_, z_ = O.grid(W, 3, excl)
+    assert np.array_equal(s_, r["scale"]) and np.array_equal(z_, r["zero"])
+    What = levels(r["codes"], r["scale"], r["zero"])
+    assert np.isclose(r["obj"][-1], _f_direct(W, What + r["H"], X), rtol=1e-10)
+
+
+def test_structured_outlier_below_one_column_reduces_to_algorithm1():
+    rng = np.random.default_rng(17)
+    W, X = _rand_layer(rng, 8, 20, 50, corr=True)
+    S = O.sigma(X)
+    r = O.outlier(W, S, 3, 4, 7, 50, structured=True)        # s < q: no column fits
+    s, z = O.grid(W, 3)
+    a1 = O.alg1(W, S, s, z, 3, iters=4)
+    assert np.array_equal(r["codes"], a1["codes"]) and not np.any(r["H"])
+    assert np.allclose(r["obj"], a1["obj"], rtol=1e-12)
