@@ -72,7 +72,9 @@ typedef struct {
     int block_width;
     /* Relax heuristic of Sec. 3.2 (skip quantization every R-th sweep): must be 0. */
     int relax_period;
-    /* Structured (column) outliers of Sec. 4.3: must be 0. */
+    /* Structured outliers (Sec. 4.3): 1 = H keeps whole columns, the floor(s/q)
+     * of largest l2 norm, in place of the s largest entries (outlier variant
+     * only; must be 0 for qe_quantize_layer). */
     int structured_outliers;
     /* Outlier variant: power-method iterations for lambda_max(Sigma), 0 = default 64. */
     int power_iters;
@@ -146,9 +148,14 @@ qe_status qe_quantize_layer(const void *W, qe_dtype w_dtype, int64_t q, int64_t 
  *   lambda_max from opts->power_iters power-method steps (Sec. 4.3).
  *   P_s keeps the s_budget largest |entries|; ties go to the smaller
  *   row-major index i*p + j; exact zeros are never kept.
+ *   With opts->structured_outliers = 1 (Sec. 4.3, "Structured Outliers") P_s
+ *   keeps instead the floor(s_budget / q) columns of largest l2 norm (ties:
+ *   smaller column index; a column of zeros is never kept), and the grid
+ *   leaves out the starting columns; every entry of a kept column is kept.
  *   H_val, H_idx  out, device s_budget floats / int64: the kept values and
  *                 their linear indices i*p + j in ascending order.
- *   H_nnz         out, device int64: number of kept entries (<= s_budget).
+ *   H_nnz         out, device int64: number of kept entries (<= s_budget;
+ *                 q x the kept columns when structured).
  *   obj           out, device iters doubles: g after the IHT step of each iteration.
  *   obj_cd        out (may be NULL), device iters doubles: g after the CD sweep.
  * Other arguments as qe_quantize_layer.

@@ -62,7 +62,7 @@ struct Plan {
            rowdf = 0, objbase = 0, sbar = 0, lcnt = 0, lent = 0, rowdft = 0;
     int64_t nblk = 0;
     size_t PW = 0, H = 0, T = 0, st = 0, cg = 0, ce = 0, sb = 0, eb = 0, y0 = 0, y1 = 0, lam = 0,
-           eta = 0, rowptr = 0;
+           eta = 0, rowptr = 0, cpart = 0, cnorm = 0, ccols = 0, cval = 0, cn = 0;
     size_t total = 0;
 };
 
@@ -122,6 +122,12 @@ static Plan make_plan(int64_t q, int64_t p, int B, bool outlier, int wpl_planes,
         pl.lam = take(cur, 8);
         pl.eta = take(cur, 8);
         pl.rowptr = take(cur, (q + 1) * 8);
+        // structured outliers: column norms and the kept columns
+        pl.cpart = take(cur, static_cast<size_t>(colnorm_chunks(q)) * p * 8);
+        pl.cnorm = take(cur, p * 4);
+        pl.ccols = take(cur, p * 8);
+        pl.cval = take(cur, p * 4);
+        pl.cn = take(cur, 8);
     }
     pl.total = cur;
     return pl;
@@ -181,6 +187,9 @@ struct Ctx {
     unsigned *cg = nullptr, *ce = nullptr, *sb = nullptr, *eb = nullptr;
     double *lam = nullptr, *eta = nullptr;
     int64_t *rowptr = nullptr;
+    double *cpart = nullptr;
+    float *cnorm = nullptr, *cval = nullptr;
+    int64_t *ccols = nullptr, *cn = nullptr;
     CUtensorMap tm_snt256, tm_snt64, tm_snt128, tm_qf, tm_dp, tm_wa;
     int wa_planes = 1;
 
@@ -247,6 +256,11 @@ static qe_status setup_ctx(Ctx &c, const Plan &pl, const qe_opts *o, cudaStream_
         c.lam = at<double>(w, pl.lam);
         c.eta = at<double>(w, pl.eta);
         c.rowptr = at<int64_t>(w, pl.rowptr);
+        c.cpart = at<double>(w, pl.cpart);
+        c.cnorm = at<float>(w, pl.cnorm);
+        c.ccols = at<int64_t>(w, pl.ccols);
+        c.cval = at<float>(w, pl.cval);
+        c.cn = at<int64_t>(w, pl.cn);
     }
     const uint64_t q = pl.q, p = pl.p, ld = pl.ld;
     if (!make_tmap_bf16(&c.tm_snt256, c.snt, 3 * p, p, ld, 256) ||
@@ -501,9 +515,11 @@ static int dense_sweeps(const qe_opts *o) {
     return (o && o->dense_sweeps) ? o->dense_sweeps : kDefaultDenseSweeps;
 }
 
-static qe_status check_opts(const qe_opts *o) {
+// structured: the call accepts structured_outliers = 1 (the outlier variant)
+static qe_status check_opts(const qe_opts *o, bool structured = false) {
     if (!o) return QE_OK;
-    if (o->relax_period != 0 || o->structured_outliers != 0) return QE_ERR_UNSUPPORTED;
+    if (o->relax_period != 0) return QE_ERR_UNSUPPORTED;
+    if (o->structured_outliers != 0 && !(structured && o->structured_outliers == 1)) return QE_ERR_UNSUPPORTED;
     if (o->block_width != 0 && o->block_width != 64 && o->block_width != 128 && o->block_width != 256)
         return QE_ERR_UNSUPPORTED;
     if (o->power_iters < 0 || o->dense_sweeps < 0) return QE_ERR_INVALID_ARG;
@@ -617,7 +633,7 @@ qe_status qe_sync_status(qe_stream_t stream) {
 
 qe_status qe_workspace_size(int64_t q, int64_t p, int outlier, const qe_opts *opts, size_t *bytes) {
     if (!bytes || q < 1 || p < 1) return QE_ERR_INVALID_ARG;
-    const qe_status st = check_opts(opts);
+    const qe_status st = check_opts(opts, outlier != 0);
     if (st != QE_OK) return st;
     const Plan pl = make_plan(q, p, block_width(opts), outlier != 0, 3, sm_count());
     *bytes = pl.total;
@@ -771,7 +787,8 @@ qe_status qe_quantize_layer_outlier(const void *W, qe_dtype w_dtype, int64_t q, 
                                     double *obj_cd, qe_stream_t stream) {
     qe_status st = check_layer(W, w_dtype, q, p, ldw, Sigma, bits, iters, codes, scales, zeros, obj);
     if (st != QE_OK) return st;
-    if ((st = check_opts(opts)) != QE_OK) return st;
+    if ((st = check_opts(opts, true)) != QE_OK) return st;
+    const bool structured = opts && opts->structured_outliers == 1;
     const int64_t N = q * p;
     if (s_budget < 0 || s_budget > N || N >= (1ll << 32) || !H_nnz) return QE_ERR_INVALID_ARG;
     if (s_budget > 0 && (!H_val || !H_idx)) return QE_ERR_INVALID_ARG;
@@ -783,9 +800,17 @@ qe_status qe_quantize_layer_outlier(const void *W, qe_dtype w_dtype, int64_t q, 
     if ((st = setup_ctx(c, pl, opts, reinterpret_cast<cudaStream_t>(stream))) != QE_OK) return st;
     const int64_t ld = pl.ld;
 
+    // P_s: the s largest |T|, or with structured outliers the floor(s/q) columns of
+    // largest l2 norm (Sec. 4.3, "Structured Outliers")
+    auto select = [&](const float *T) -> cudaError_t {
+        if (structured)
+            return launch_topk_columns(T, q, p, s_budget / q, c.st, c.cg, c.ce, c.sb, c.eb, c.cpart, c.cnorm,
+                                       c.ccols, c.cval, c.cn, H_idx, H_val, H_nnz, c.nsm, c.s);
+        return launch_topk(T, N, s_budget, c.st, c.cg, c.ce, c.sb, c.eb, H_idx, H_val, H_nnz, c.nsm, c.s);
+    };
     // H = P_s(W); the grid ignores those entries (Sec. 4.3)
     QE_CK(launch_flat_copy(W, wbf16, ldw, q, p, c.T, c.s));
-    QE_CK(launch_topk(c.T, N, s_budget, c.st, c.cg, c.ce, c.sb, c.eb, H_idx, H_val, H_nnz, c.nsm, c.s));
+    QE_CK(select(c.T));
     QE_CK(cudaMemsetAsync(c.H, 0, static_cast<size_t>(q) * ld * 4, c.s));
     QE_CK(launch_scatter_rowptr(H_idx, H_val, H_nnz, s_budget, q, p, c.H, ld, c.rowptr, c.s));
     QE_CK(launch_grid(W, wbf16, ldw, c.H, ld, q, p, bits, scales, zeros, c.err, c.s));
@@ -811,7 +836,7 @@ qe_status qe_quantize_layer_outlier(const void *W, qe_dtype w_dtype, int64_t q, 
         if ((st = residual(c, scales, obj_cd ? &f : nullptr)) != QE_OK) return st;
         // IHT step: T = H + 2 eta d (R - What); H = P_s(T)
         QE_CK(launch_iht_target(c.H, c.R, ld, codes, p, scales, zeros, c.d, c.eta, q, p, c.T, c.s));
-        QE_CK(launch_topk(c.T, N, s_budget, c.st, c.cg, c.ce, c.sb, c.eb, H_idx, H_val, H_nnz, c.nsm, c.s));
+        QE_CK(select(c.T));
         QE_CK(cudaMemsetAsync(c.H, 0, static_cast<size_t>(q) * ld * 4, c.s));
         QE_CK(launch_scatter_rowptr(H_idx, H_val, H_nnz, s_budget, q, p, c.H, ld, c.rowptr, c.s));
         // P = P_W - H (I + Sigma_bar); R += P_new - P_old  (R = P - What Sigma_bar stays current)

@@ -267,6 +267,46 @@ __global__ void __launch_bounds__(256) k_topk_emit(const float *T, int64_t N, co
     }
 }
 
+// ---- structured outliers (Sec. 4.3): keep whole columns -----------------------
+// Squared column norms of the flat q x p matrix T, summed in fp64 over row
+// chunks (part[rc][j]) and then over the chunks in order, rounded to fp32 keys
+// for the radix select.
+__global__ void __launch_bounds__(256) k_colnorm_partial(const float *T, int64_t q, int64_t p, int64_t rows_per,
+                                                         double *part) {
+    const int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+    if (j >= p) return;
+    const int64_t i0 = blockIdx.y * rows_per;
+    const int64_t i1 = (i0 + rows_per) < q ? (i0 + rows_per) : q;
+    double acc = 0.0;
+    for (int64_t i = i0; i < i1; ++i) {
+        const double v = T[i * p + j];
+        acc += v * v;
+    }
+    part[blockIdx.y * p + j] = acc;
+}
+
+__global__ void k_colnorm_final(const double *part, int nrc, int64_t p, float *norm2) {
+    const int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+    if (j >= p) return;
+    double acc = 0.0;
+    for (int rc = 0; rc < nrc; ++rc) acc += part[rc * p + j];
+    norm2[j] = static_cast<float>(acc);
+}
+
+// Every entry of the kept columns, as ascending linear indices: row i, kept
+// column r -> slot i * ncols + r (the kept columns are ascending).
+__global__ void k_col_emit(const float *T, int64_t q, int64_t p, const int64_t *cols, const int64_t *ncols_p,
+                           int64_t *H_idx, float *H_val, int64_t *H_nnz) {
+    const int64_t nc = *ncols_p;
+    const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+    if (t == 0) *H_nnz = q * nc;
+    if (nc == 0 || t >= q * nc) return;
+    const int64_t i = t / nc, r = t % nc;
+    const int64_t e = i * p + cols[r];
+    H_idx[t] = e;
+    H_val[t] = T[e];
+}
+
 // Dense H from the kept entries (H zeroed before).
 __global__ void k_scatter(const int64_t *H_idx, const float *H_val, const int64_t *nnz, int64_t cap,
                           int64_t p, float *H, int64_t ld) {
@@ -384,6 +424,25 @@ cudaError_t launch_topk(const float *T, int64_t N, int64_t s_budget, TopkState *
     k_topk_count<<<static_cast<unsigned>(nch), 256, 0, s>>>(T, N, st, cnt_gt, cnt_eq);
     k_topk_scan<<<1, 1024, 0, s>>>(cnt_gt, cnt_eq, static_cast<int>(nch), st, sel_base, eq_base, nnz);
     k_topk_emit<<<static_cast<unsigned>(nch), 256, 0, s>>>(T, N, st, sel_base, eq_base, H_idx, H_val);
+    return cudaGetLastError();
+}
+
+int colnorm_chunks(int64_t q) { return static_cast<int>(q < 64 * 64 ? ceil_div(q, 64) : 64); }
+
+cudaError_t launch_topk_columns(const float *T, int64_t q, int64_t p, int64_t k, TopkState *st, unsigned *cnt_gt,
+                                unsigned *cnt_eq, unsigned *sel_base, unsigned *eq_base, double *part,
+                                float *norm2, int64_t *cols, float *colval, int64_t *ncols, int64_t *H_idx,
+                                float *H_val, int64_t *nnz, int nsm, cudaStream_t s) {
+    const int nrc = colnorm_chunks(q);
+    const int64_t rows_per = ceil_div(q, nrc);
+    const dim3 g1(static_cast<unsigned>(ceil_div(p, 256)), static_cast<unsigned>(nrc));
+    k_colnorm_partial<<<g1, 256, 0, s>>>(T, q, p, rows_per, part);
+    k_colnorm_final<<<static_cast<unsigned>(ceil_div(p, 256)), 256, 0, s>>>(part, nrc, p, norm2);
+    cudaError_t e = launch_topk(norm2, p, k, st, cnt_gt, cnt_eq, sel_base, eq_base, cols, colval, ncols, nsm, s);
+    if (e != cudaSuccess) return e;
+    const int64_t cap = q * k;
+    k_col_emit<<<static_cast<unsigned>(ceil_div(cap > 0 ? cap : 1, 256)), 256, 0, s>>>(T, q, p, cols, ncols, H_idx,
+                                                                                     H_val, nnz);
     return cudaGetLastError();
 }
 

@@ -29,6 +29,15 @@ int64_t topk_chunks(int64_t N);
 cudaError_t launch_topk(const float *T, int64_t N, int64_t s_budget, TopkState *st, unsigned *cnt_gt,
                         unsigned *cnt_eq, unsigned *sel_base, unsigned *eq_base, int64_t *H_idx,
                         float *H_val, int64_t *nnz, int nsm, cudaStream_t s);
+// Structured outliers (Sec. 4.3): the k columns of T with the largest l2 norm
+// (ties: smaller index; zero columns never kept), emitted as every entry of those
+// columns in ascending linear order (nnz = q x kept columns).  part: colnorm_chunks(q)
+// x p doubles; norm2, colval: p floats; cols: p indices; ncols: one.
+int colnorm_chunks(int64_t q);
+cudaError_t launch_topk_columns(const float *T, int64_t q, int64_t p, int64_t k, TopkState *st, unsigned *cnt_gt,
+                                unsigned *cnt_eq, unsigned *sel_base, unsigned *eq_base, double *part,
+                                float *norm2, int64_t *cols, float *colval, int64_t *ncols, int64_t *H_idx,
+                                float *H_val, int64_t *nnz, int nsm, cudaStream_t s);
 cudaError_t launch_scatter_rowptr(const int64_t *H_idx, const float *H_val, const int64_t *nnz,
                                   int64_t cap, int64_t q, int64_t p, float *H, int64_t ld,
                                   int64_t *rowptr, cudaStream_t s);

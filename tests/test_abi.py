@@ -71,6 +71,14 @@ def test_invalid_arguments_rejected_synchronously(lib):
     assert L.qe_quantize_layer(_fake(), qe.QE_F32, 4, 4, 4, _fake(2), 3, 1, ctypes.byref(o), _fake(3),
                                _fake(4), _fake(5), _fake(6), None) == qe.QE_ERR_UNSUPPORTED
     o = qe.QEOpts()
+    o.structured_outliers = 1     # only the outlier variant takes it
+    assert L.qe_quantize_layer(_fake(), qe.QE_F32, 4, 4, 4, _fake(2), 3, 1, ctypes.byref(o), _fake(3),
+                               _fake(4), _fake(5), _fake(6), None) == qe.QE_ERR_UNSUPPORTED
+    o.structured_outliers = 2
+    assert L.qe_quantize_layer_outlier(_fake(), qe.QE_F32, 4, 4, 4, _fake(2), 3, 1, 4, ctypes.byref(o),
+                                       _fake(3), _fake(4), _fake(5), _fake(7), _fake(8), _fake(9), _fake(6),
+                                       None, None) == qe.QE_ERR_UNSUPPORTED
+    o = qe.QEOpts()
     o.dense_sweeps = -1
     assert L.qe_quantize_layer(_fake(), qe.QE_F32, 4, 4, 4, _fake(2), 3, 1, ctypes.byref(o), _fake(3),
                                _fake(4), _fake(5), _fake(6), None) == qe.QE_ERR_INVALID_ARG

@@ -130,7 +130,8 @@ def test_fullsize_layer_sampled_rows(name, nrows, free_run, full_obj):
         torch.cuda.empty_cache()
 
 
-def test_fullsize_outlier_properties():
+@pytest.mark.parametrize("structured", [False, True], ids=["entries", "columns"])
+def test_fullsize_outlier_properties(structured):
     """The outlier-aware workload at full size.  The IHT support is a global
     top-s (Eq. iht-update), so rows are not independent here: the sampled-row
     check covers the grid (W without the initial support P_s(W), Sec. 4.3);
@@ -144,10 +145,13 @@ def test_fullsize_outlier_properties():
     Sg = qe.qe_build_sigma(X)
     del X
     bits = cfg.bits[0]
-    out = qe.qe_quantize_layer_outlier(W, Sg, bits, cfg.iters, cfg.s_budget)
+    out = qe.qe_quantize_layer_outlier(W, Sg, bits, cfg.iters, cfg.s_budget, structured=structured)
     assert qe.qe_sync_status() == qe.QE_OK
     nnz = int(out["H_nnz"].item())
     assert 0 < nnz <= cfg.s_budget
+    if structured:   # whole columns, floor(s / q) of them
+        assert nnz == q * (cfg.s_budget // q)
+        assert np.unique(out["H_idx"][:nnz].cpu().numpy() % p).size == cfg.s_budget // q
     idx = out["H_idx"][:nnz].cpu().numpy()
     assert np.all(np.diff(idx) > 0) and idx[0] >= 0 and idx[-1] < q * p
     obj, obj_cd = out["obj"].cpu().numpy(), out["obj_cd"].cpu().numpy()
@@ -155,9 +159,11 @@ def test_fullsize_outlier_properties():
     assert np.all(np.diff(obj[1:]) <= 1e-6 * obj[1:-1])
     # grid on sampled rows, from W without P_s(W)
     W64 = W.double().cpu().numpy()
-    sel = O.topk(W64, cfg.s_budget)
     excl = np.zeros(q * p, np.uint8)
-    excl[sel] = 1
+    if structured:
+        excl.reshape(q, p)[:, O.topk_columns(W64, cfg.s_budget // q)] = 1
+    else:
+        excl[O.topk(W64, cfg.s_budget)] = 1
     rows = np.random.default_rng(5).choice(q, size=64, replace=False)
     s, z = O.grid(W64[rows], bits, excl.reshape(q, p)[rows])
     rows_t = torch.from_numpy(rows).cuda()

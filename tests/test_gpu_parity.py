@@ -310,6 +310,60 @@ def test_outlier_parity_small(q, p, bits, frac):
     assert np.all(out["obj"].cpu().numpy() <= out["obj_cd"].cpu().numpy() * (1 + 1e-6))
 
 
+def _planted_columns(W, cols, std, seed):
+    g = torch.Generator().manual_seed(seed)
+    noise = torch.randn(W.shape[0], len(cols), generator=g) * std
+    W[:, cols] = (W[:, cols].float() + noise.to(W.device)).to(W.dtype)
+    return W
+
+
+@pytest.mark.parametrize("q,p,bits,ncols", [(96, 192, 3, 3), (130, 260, 2, 5)])
+def test_structured_outlier_parity_small(q, p, bits, ncols):
+    """Whole-column outliers (Sec. 4.3): the kept columns, grid, objectives, codes
+    and H values against the oracle."""
+    iters, power_iters = 4, 200
+    W = inputs.layer_weights(q, p, dtype=torch.bfloat16, seed=43, device="cuda")
+    W = _planted_columns(W, [5, 40, 77, 121, 150][:ncols], 0.3, 43)
+    X = inputs.calib_inputs(p, 2048, dtype=torch.bfloat16, seed=43, device="cuda", heavy_frac=0.02,
+                            heavy_mult=30.0)
+    Sg = qe.qe_build_sigma(X)
+    s_budget = ncols * q + 7
+    out = qe.qe_quantize_layer_outlier(W, Sg, bits, iters, s_budget, power_iters=power_iters,
+                                       structured=True)
+    assert qe.qe_sync_status() == qe.QE_OK
+    W64, S64 = parity.f64(W), parity.f64(Sg)
+    ref = O.outlier(W64, S64, bits, iters, s_budget, power_iters, structured=True)
+    assert np.array_equal(out["scales"].cpu().numpy(), ref["scale"])
+    assert np.array_equal(out["zeros"].cpu().numpy(), ref["zero"])
+    parity.check_obj(out["obj_cd"].cpu().numpy(), ref["obj_cd"], what="g after CD")
+    parity.check_obj(out["obj"].cpu().numpy(), ref["obj"], what="g after IHT")
+    m = parity.code_match(out["codes"].cpu().numpy(), ref["codes"])
+    assert m >= parity.CODE_MATCH, f"codes match {m:.5f}"
+    nnz = int(out["H_nnz"].item())
+    assert nnz == ref["nnz"] == q * ncols
+    idx = out["H_idx"][:nnz].cpu().numpy()
+    assert np.all(np.diff(idx) > 0)
+    gpu_cols = np.unique(idx % p)
+    ref_cols = np.nonzero(np.any(ref["H"] != 0, axis=0))[0]
+    assert np.array_equal(gpu_cols, ref_cols)
+    Hd = np.zeros(q * p)
+    Hd[idx] = out["H_val"][:nnz].cpu().numpy()
+    assert np.allclose(Hd, ref["H"].ravel(), rtol=1e-3, atol=1e-6)
+    assert np.all(out["obj"].cpu().numpy() <= out["obj_cd"].cpu().numpy() * (1 + 1e-6))
+
+
+def test_structured_outlier_below_one_column_matches_plain_layer():
+    q, p, bits, iters = 64, 128, 3, 3
+    W = inputs.layer_weights(q, p, dtype=torch.bfloat16, seed=52, device="cuda")
+    X = inputs.calib_inputs(p, 1024, dtype=torch.bfloat16, seed=52, device="cuda", corr_rank=4)
+    Sg = qe.qe_build_sigma(X)
+    a = qe.qe_quantize_layer_outlier(W, Sg, bits, iters, 0)
+    b = qe.qe_quantize_layer_outlier(W, Sg, bits, iters, q - 1, structured=True)
+    torch.cuda.synchronize()
+    assert torch.equal(a["codes"], b["codes"]) and int(b["H_nnz"].item()) == 0
+    assert np.array_equal(a["obj"].cpu().numpy(), b["obj"].cpu().numpy())
+
+
 def test_outlier_zero_budget_matches_plain_layer():
     q, p, bits, iters = 64, 128, 3, 3
     W = inputs.layer_weights(q, p, dtype=torch.bfloat16, seed=51, device="cuda")
