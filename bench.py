@@ -45,6 +45,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-rows", type=int, default=4096, help="oracle rows in the CPU sample")
+    ap.add_argument("--structured", action="store_true",
+                    help="outlier workloads: keep whole columns (Sec. 4.3, structured outliers)")
     ap.add_argument("--dense-sweeps", type=int, default=0,
                     help="sweeps whose cross-block term uses the tensor-core GEMM (0 = library default)")
     ap.add_argument("--tokens", type=int, default=0,
@@ -259,16 +261,23 @@ def main():
     qe.load()
 
     cfg = inputs.CONFIGS[args.config]
+    import dataclasses
     if args.tokens:
-        import dataclasses
         cfg = dataclasses.replace(cfg, n=args.tokens)
     q, p, n = cfg.q, cfg.p, cfg.n
-    seed = cfg.seed + rank                        # each rank owns a different layer
-    W = inputs.layer_weights(q, p, dtype=cfg.w_dtype, seed=seed, device="cuda")
-    X = inputs.calib_inputs(p, n, dtype=cfg.x_dtype, seed=seed, device="cuda",
-                            heavy_frac=cfg.heavy_frac, heavy_mult=cfg.heavy_mult)
+    cfg_r = dataclasses.replace(cfg, seed=cfg.seed + rank)   # each rank owns a different layer
+    W = cfg_r.weights("cuda")
+    X = cfg_r.inputs("cuda")
     Sigma = torch.empty(p, p, dtype=torch.float32, device="cuda")
-    ws = torch.empty(qe.qe_workspace_size(q, p), dtype=torch.uint8, device="cuda")
+    outlier = cfg.s_budget > 0                    # the outlier-aware workload (Algorithm 4)
+    ws = torch.empty(qe.qe_workspace_size(q, p, outlier=outlier), dtype=torch.uint8, device="cuda")
+
+    def quantize(Wt, b, timer=None):
+        if outlier:
+            return qe.qe_quantize_layer_outlier(Wt, Sigma, b, cfg.iters, cfg.s_budget, workspace=ws,
+                                                structured=args.structured, timer=timer)
+        return qe.qe_quantize_layer(Wt, Sigma, b, cfg.iters, workspace=ws, timer=timer,
+                                    dense_sweeps=args.dense_sweeps)
     stream = torch.cuda.current_stream()
     nb = len(cfg.bits)
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(nb + 2)]
@@ -282,8 +291,7 @@ def main():
             events[1].record(stream)
         outs = []
         for k, b in enumerate(cfg.bits):
-            outs.append(qe.qe_quantize_layer(W, Sigma, b, cfg.iters, workspace=ws, timer=timer,
-                                             dense_sweeps=args.dense_sweeps))
+            outs.append(quantize(W, b, timer))
             if events:
                 events[2 + k].record(stream)
         return outs
@@ -335,12 +343,15 @@ def main():
     blocks = [(b0, min(256, p - b0)) for b0 in range(0, p, 256)]
     tri_flops = sum(2 * q * bw * b0 for b0, bw in blocks)
     win_flops = sum(2 * q * bw * p for b0, bw in blocks)
-    dense = args.dense_sweeps or DEFAULT_DENSE_SWEEPS
+    dense = cfg.iters if outlier else (args.dense_sweeps or DEFAULT_DENSE_SWEEPS)
     trail_flops, trail_launches = tri_flops, nblk - 1
     for t in range(1, cfg.iters):
-        if t < dense:   # later sweeps take the cross-block term from the change lists
+        if outlier:     # Algorithm 4: sweeps after the first take the change lists
+            continue
+        elif t < dense:   # later sweeps take the cross-block term from the change lists
             trail_flops += tri_flops if t == 1 else win_flops
             trail_launches += nblk - 1 if t == 1 else nblk
+    refreshes = cfg.iters if outlier else 1         # residual GEMMs per layer
 
     units_per_step = q * p * p * cfg.iters * nb           # column updates per rank per step
     value = units_per_step * world / (ms / 1e3)
@@ -354,7 +365,9 @@ def main():
               "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
               "config": {"workload": cfg.name, "q": q, "p": p, "n": n, "bits": list(cfg.bits),
                          "sweeps": cfg.iters, "parallelism": f"layer-replicas x{world}",
-                         "l2": "inputs larger than L2 (X is %.2f GiB)" % (p * n * 2 / 2**30)},
+                         "l2": "inputs larger than L2 (X is %.2f GiB)" % (p * n * 2 / 2**30),
+                         **({"s_budget": cfg.s_budget,
+                             "outliers": "columns" if args.structured else "entries"} if outlier else {})},
               "layer_quantize_ms": ms,
               "sigma_ms": sigma_avg,
               "sigma_tflops": sig_flops / (sigma_avg / 1e3) / 1e12,
@@ -366,9 +379,9 @@ def main():
     gemm_ms = sigma_avg + sum(timed[k][1] for k in kinds[:3]) / args.steps
     gemm_launches = 1 + sum(timed[k][0] for k in kinds[:3]) // args.steps
     qpad, ppad = -(-q // 128) * 128, -(-p // 256) * 256
-    gemm_flops = sig_flops + nb * (2 * 2 * q * p * p + trail_flops)
+    gemm_flops = sig_flops + nb * (2 * q * p * p * (1 + refreshes) + trail_flops)
     gemm_exec = (gemm_tiles_sigma(p) * 2 * 128 * 256 * n
-                 + nb * (2 * 3 * 2 * qpad * ppad * (-(-p // 64) * 64)
+                 + nb * ((1 + refreshes) * 3 * 2 * qpad * ppad * (-(-p // 64) * 64)
                          + 6 * tri_flops + 3 * (trail_flops - tri_flops)))   # 6 products in sweep 1
     result["roofline"] = roofline_gemm(gemm_flops, gemm_exec, gemm_ms, gemm_launches, pk)
     # the persistent change-list kernel: one launch per layer (per 32 list sweeps)
@@ -376,7 +389,8 @@ def main():
     n_list = max(cfg.iters - dense, 0)
     n_chunks = -(-n_list // 32)
     list_bytes = n_list * (4 * q * p + q * p + 4 * p * p) / n_chunks if n_chunks else 0
-    result["roofline_cd"] = roofline_lists(list_bytes, list_ms / args.steps, list_launches // args.steps, pk)
+    if not outlier:
+        result["roofline_cd"] = roofline_lists(list_bytes, list_ms / args.steps, list_launches // args.steps, pk)
 
 
     # per-class breakdown of one extra, untimed step (events around every launch)
@@ -387,7 +401,7 @@ def main():
     qe.qe_build_sigma(X, Sigma=Sigma)
     e1.record(stream)
     for b in cfg.bits:
-        qe.qe_quantize_layer(W, Sigma, b, cfg.iters, workspace=ws, timer=brk, dense_sweeps=args.dense_sweeps)
+        quantize(W, b, brk)
     torch.cuda.synchronize()
     names = {qe.QE_KERNEL_PINIT_GEMM: "pinit_gemm", qe.QE_KERNEL_RESIDUAL_GEMM: "residual_gemm",
              qe.QE_KERNEL_TRAIL_GEMM: "trail_gemm", qe.QE_KERNEL_CD_BLOCK: "cd_block",
@@ -410,6 +424,16 @@ def main():
     for t in range(1, min(dense, cfg.iters)):
         per_layer += (nblk - 1 if t == 1 else nblk) + nblk + 1
     per_layer += 2 * -(-max(cfg.iters - max(dense, 1), 0) // 32)
+    if outlier:
+        # selection (P_s: 4 radix passes x 2 + count, scan, emit; columns: + 2 norm
+        # kernels + emit), start: copy, selection, scatter + row pointers, grid,
+        # Sigma_bar set-up (5) + [W planes] + P, 64 power steps (+ fill, last, final),
+        # SpMM refresh, initial residual; sweep 1 blocked (2 nblk - 1), later sweeps one
+        # change-list launch; per iteration: residual GEMM + objective sum, IHT target,
+        # selection, scatter + row pointers, SpMM, objective (2)
+        sel = 14 if args.structured else 11
+        per_layer = (1 + sel + 2 + 1 + 6 + w_planes + 67 + 1 + 1 + (2 * nblk - 1) + (cfg.iters - 1)
+                     + cfg.iters * (2 + 1 + sel + 2 + 1 + 2))
     result["gpu_launches"] = args.steps * (1 + nb * per_layer)
 
     # end to end through the C ABI with host buffers
@@ -430,8 +454,7 @@ def main():
             Wd.copy_(Wh, non_blocking=True)
             qe.qe_build_sigma_host(Xh, Sigma, staging, chunk)
             for k, b in enumerate(cfg.bits):
-                o = qe.qe_quantize_layer(Wd, Sigma, b, cfg.iters, workspace=ws,
-                                         dense_sweeps=args.dense_sweeps)
+                o = quantize(Wd, b)
                 for key in ("codes", "scales", "zeros", "obj"):
                     host_out[k][key].copy_(o[key], non_blocking=True)
 

@@ -100,7 +100,7 @@ static Plan make_plan(int64_t q, int64_t p, int B, bool outlier, int wpl_planes,
                                                                                     : objective_blocks(q)) * 8);
     pl.rowdf = take(cur, static_cast<size_t>(q) * 8);
     pl.objbase = take(cur, 8);
-    if (!outlier) {   // change lists and fp32 Sigma_bar rows of the rolling-window sweeps
+    {   // change lists and fp32 Sigma_bar rows of the change-list sweeps
         pl.sbar = take(cur, static_cast<size_t>(p) * pl.ld * 4);
         pl.lcnt = take(cur, static_cast<size_t>(q) * pl.nblk * 4);
         pl.lent = take(cur, static_cast<size_t>(q) * pl.nblk * B * 4);
@@ -831,7 +831,19 @@ qe_status qe_quantize_layer_outlier(const void *W, qe_dtype w_dtype, int64_t q, 
         QE_CK(launch_init_residual(W, wbf16, ldw, c.H, ld, q, p, scales, zeros, c.R, ld, c.s));
     }
     for (int t = 0; t < iters; ++t) {
-        if ((st = sweep(c, codes, scales, zeros, bits, t == 0 && !warm, 0)) != QE_OK) return st;
+        if (t == 0 && !warm) {
+            if ((st = sweep(c, codes, scales, zeros, bits, true, 0)) != QE_OK) return st;
+        } else {
+            // R is fresh and the target W - H stays fixed during the sweep: one
+            // change-list sweep whose window starts empty (each block corrected by
+            // this sweep's changes left of it); it keeps C - z current for the
+            // residual GEMM below
+            QE_CK(cudaMemsetAsync(c.lcnt, 0, static_cast<size_t>(q) * pl.nblk * 4, c.s));
+            CdArgs a = list_args(c, codes, scales, zeros, bits);
+            a.write_qf = 1;
+            Timed tm(c.timer, QE_KERNEL_CD_LISTS, c.s);
+            QE_CK(launch_cd_rows_lists(pl.B, a, t, t + 1, c.rowdft, nullptr, 1, kFreeMaxChanges, c.nsm, c.s));
+        }
         const ObjFuse f{obj_cd ? obj_cd + t : nullptr, W, wbf16, ldw, codes, zeros, c.H};
         if ((st = residual(c, scales, obj_cd ? &f : nullptr)) != QE_OK) return st;
         // IHT step: T = H + 2 eta d (R - What); H = P_s(T)

@@ -121,12 +121,14 @@ __device__ __forceinline__ void epilogue_row(const GemmArgs &g, int r, int c0, c
                 // f = sum D_ij d_j s (R'_ij - C_ij)
                 const float z = zz;
                 float part = 0.0f;
-                const bool vec = full && g.w_is_bf16 && (g.ldw % 8) == 0 && (g.ldc % 16) == 0 && g.Hd == nullptr;
+                const bool vec = full && g.w_is_bf16 && (g.ldw % 8) == 0 && (g.ldc % 16) == 0 &&
+                                 (g.Hd == nullptr || (g.ldh % 4) == 0);
                 if (vec) {
                     const uint4 *wp = reinterpret_cast<const uint4 *>(
                         reinterpret_cast<const __nv_bfloat16 *>(g.W) + rr * g.ldw + c0);
                     const uint4 *cp = reinterpret_cast<const uint4 *>(g.codes + rr * g.ldc + c0);
                     const float4 *dp = reinterpret_cast<const float4 *>(g.dvec + c0);
+                    const float4 *hp = g.Hd ? reinterpret_cast<const float4 *>(g.Hd + rr * g.ldh + c0) : nullptr;
 #pragma unroll
                     for (int h = 0; h < 2; ++h) {
                         union { uint4 v; uint8_t b[16]; } cu;
@@ -139,12 +141,14 @@ __device__ __forceinline__ void epilogue_row(const GemmArgs &g, int r, int c0, c
                             for (int q4 = 0; q4 < 2; ++q4) {
                                 const float4 d4 = dp[4 * h + 2 * w8 + q4];
                                 const float dd[4] = {d4.x, d4.y, d4.z, d4.w};
+                                const float4 h4 = hp ? hp[4 * h + 2 * w8 + q4] : make_float4(0.f, 0.f, 0.f, 0.f);
+                                const float hh[4] = {h4.x, h4.y, h4.z, h4.w};
 #pragma unroll
                                 for (int e = 0; e < 4; ++e) {
                                     const int i = 16 * h + 8 * w8 + 4 * q4 + e;
                                     const float cj = static_cast<float>(cu.b[i - 16 * h]);
                                     const float wh = s * (cj - z);
-                                    const float t = __bfloat162float(wu.e[4 * q4 + e]) - wh;
+                                    const float t = (__bfloat162float(wu.e[4 * q4 + e]) - wh) - hh[e];
                                     const float dj = dd[e] > 0.0f ? dd[e] : 0.0f;
                                     part += t * dj * (s * (o[i] - cj));
                                 }

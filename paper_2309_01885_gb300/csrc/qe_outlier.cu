@@ -49,7 +49,10 @@ __device__ __forceinline__ unsigned block_excl_scan(unsigned v, unsigned *sh, un
 }
 
 // ---- power method (Sec. 4.3: lambda_max(X X^T) "by iterative power method") --
-// y_out = Sigma (y_in / ||y_in||); every CTA recomputes ||y_in||.
+// y_out = Sigma (y_in / ||y_in||); every CTA recomputes ||y_in||.  One warp per
+// row of Sigma; eight independent partial sums keep eight loads in flight per
+// lane (a dependent chain of single loads made this step latency-bound), and
+// 16-byte loads are used when the rows are 16-byte aligned.
 __global__ void __launch_bounds__(256) k_power_step(const float *S, int64_t lds, int64_t p,
                                                     const float *y_in, float *y_out) {
     __shared__ double sh[8];
@@ -58,12 +61,39 @@ __global__ void __launch_bounds__(256) k_power_step(const float *S, int64_t lds,
     n2 = block_sum(n2, sh);
     const float inv = n2 > 0.0 ? static_cast<float>(1.0 / sqrt(n2)) : 0.0f;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const bool vec = (lds % 4 == 0) && ((reinterpret_cast<uintptr_t>(S) & 15u) == 0) &&
+                     ((reinterpret_cast<uintptr_t>(y_in) & 15u) == 0);
     for (int64_t a = (int64_t)blockIdx.x * 8 + warp; a < p; a += (int64_t)gridDim.x * 8) {
-        float acc = 0.0f;
-        for (int64_t b = lane; b < p; b += 32) acc = fmaf(S[a * lds + b], y_in[b], acc);
+        const float *row = S + a * lds;
+        float acc[8];
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-        if (lane == 0) y_out[a] = acc * inv;
+        for (int u = 0; u < 8; ++u) acc[u] = 0.0f;
+        int64_t b0 = 0;
+        if (vec) {
+            const int64_t n4 = p / 4;
+            const float4 *r4 = reinterpret_cast<const float4 *>(row);
+            const float4 *y4 = reinterpret_cast<const float4 *>(y_in);
+            for (int64_t b = lane; b < n4; b += 64) {
+                const float4 x0 = r4[b], v0 = y4[b];
+                const bool two = b + 32 < n4;
+                const float4 x1 = two ? r4[b + 32] : make_float4(0.f, 0.f, 0.f, 0.f);
+                const float4 v1 = two ? y4[b + 32] : make_float4(0.f, 0.f, 0.f, 0.f);
+                acc[0] = fmaf(x0.x, v0.x, acc[0]);
+                acc[1] = fmaf(x0.y, v0.y, acc[1]);
+                acc[2] = fmaf(x0.z, v0.z, acc[2]);
+                acc[3] = fmaf(x0.w, v0.w, acc[3]);
+                acc[4] = fmaf(x1.x, v1.x, acc[4]);
+                acc[5] = fmaf(x1.y, v1.y, acc[5]);
+                acc[6] = fmaf(x1.z, v1.z, acc[6]);
+                acc[7] = fmaf(x1.w, v1.w, acc[7]);
+            }
+            b0 = n4 * 4;
+        }
+        for (int64_t b = b0 + lane; b < p; b += 32) acc[0] = fmaf(row[b], y_in[b], acc[0]);
+        float t = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+        if (lane == 0) y_out[a] = t * inv;
     }
 }
 
@@ -333,29 +363,56 @@ __global__ void k_rowptr(const int64_t *H_idx, const int64_t *nnz, int64_t q, in
 
 // P_new = P_W - H (I + Sigma_bar) for row i (Sigma_bar_kj = Sigma_kj / d_j off
 // the diagonal, 0 for dead columns); R += (P_new - P_old) / s_i when update_r
-// (R in grid-step units); P = P_new.
+// (R in grid-step units); P = P_new.  One CTA per (row, tile of kSpmmCols
+// columns): each thread keeps kSpmmPer columns in registers and walks the row's
+// kept entries, so every entry issues kSpmmPer independent coalesced loads of its
+// Sigma row.
+constexpr int kSpmmPer = 16;
+constexpr int kSpmmCols = 256 * kSpmmPer;
+
 __global__ void __launch_bounds__(256) k_spmm_refresh(const float *PW, float *P, float *R, int64_t ld,
                                                       const float *S, int64_t lds, const float *d,
                                                       const float *dinv, const int64_t *H_idx,
                                                       const float *H_val, const int64_t *rowptr,
                                                       int64_t p, int update_r, const float *scale) {
     const int64_t i = blockIdx.x;
+    const int64_t j0 = static_cast<int64_t>(blockIdx.y) * kSpmmCols + threadIdx.x;
     const float s = update_r ? scale[i] : 1.0f;
     const int64_t e0 = rowptr[i], e1 = rowptr[i + 1];
-    for (int64_t j = threadIdx.x; j < p; j += blockDim.x) {
-        float acc = PW[i * ld + j];
-        const float dj = d[j];
-        const float ij = dinv[j];
-        for (int64_t e = e0; e < e1; ++e) {
-            const int64_t k = H_idx[e] - i * p;
-            const float v = H_val[e];
-            float sb;
-            if (k == j) sb = 1.0f;
-            else sb = (dj > 0.0f && d[k] > 0.0f) ? S[k * lds + j] * ij : 0.0f;
-            acc = fmaf(-v, sb, acc);
+    float acc[kSpmmPer], ij[kSpmmPer];
+    bool alive[kSpmmPer];
+#pragma unroll
+    for (int u = 0; u < kSpmmPer; ++u) {
+        const int64_t j = j0 + 256 * u;
+        const bool ok = j < p;
+        acc[u] = ok ? __ldcs(PW + i * ld + j) : 0.0f;   // streamed: keep L2 for Sigma's rows
+        ij[u] = ok ? dinv[j] : 0.0f;
+        alive[u] = ok && d[j] > 0.0f;
+    }
+    for (int64_t e = e0; e < e1; ++e) {
+        const int64_t k = H_idx[e] - i * p;
+        const float v = H_val[e];
+        const bool kalive = d[k] > 0.0f;
+        const float *srow = S + k * lds;
+        float sv[kSpmmPer];
+#pragma unroll
+        for (int u = 0; u < kSpmmPer; ++u) {
+            const int64_t j = j0 + 256 * u;
+            sv[u] = (j < p && kalive) ? srow[j] : 0.0f;
         }
-        if (update_r) R[i * ld + j] += __fdiv_rn(acc - P[i * ld + j], s);
-        P[i * ld + j] = acc;
+#pragma unroll
+        for (int u = 0; u < kSpmmPer; ++u) {
+            const int64_t j = j0 + 256 * u;
+            const float sb = (k == j) ? 1.0f : (alive[u] ? sv[u] * ij[u] : 0.0f);
+            acc[u] = fmaf(-v, sb, acc[u]);
+        }
+    }
+#pragma unroll
+    for (int u = 0; u < kSpmmPer; ++u) {
+        const int64_t j = j0 + 256 * u;
+        if (j >= p) continue;
+        if (update_r) __stcs(R + i * ld + j, __ldcs(R + i * ld + j) + __fdiv_rn(acc[u] - __ldcs(P + i * ld + j), s));
+        __stcs(P + i * ld + j, acc[u]);
     }
 }
 
@@ -460,8 +517,8 @@ cudaError_t launch_spmm_refresh(const float *PW, float *P, float *R, int64_t ld,
                                 int64_t lds, const float *d, const float *dinv, const int64_t *H_idx,
                                 const float *H_val, const int64_t *rowptr, int64_t q, int64_t p,
                                 int update_r, const float *scale, cudaStream_t s) {
-    k_spmm_refresh<<<static_cast<unsigned>(q), 256, 0, s>>>(PW, P, R, ld, S, lds, d, dinv, H_idx, H_val,
-                                                            rowptr, p, update_r, scale);
+    const dim3 grid(static_cast<unsigned>(q), static_cast<unsigned>(ceil_div(p, kSpmmCols)));
+    k_spmm_refresh<<<grid, 256, 0, s>>>(PW, P, R, ld, S, lds, d, dinv, H_idx, H_val, rowptr, p, update_r, scale);
     return cudaGetLastError();
 }
 
