@@ -38,6 +38,7 @@ struct GemmCfg {
     static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + 256;
     static_assert(BN == 64 || BN == 128 || BN == 256, "BN");
     static_assert(SMEM_BYTES <= 232448, "smem");
+    static_assert(8 * 32 * (HALF + 4) * 4 <= STAGES * STAGE_BYTES, "epilogue staging fits the ring");
 };
 
 // Virtual K steps (k-block x operand-plane product) accumulated in one TMEM
@@ -194,6 +195,136 @@ __device__ __forceinline__ void epilogue_row(const GemmArgs &g, int r, int c0, c
     }
 }
 
+template <int N>
+__device__ __forceinline__ void ld_fv(const float *p, float *v) {
+    if constexpr (N == 4) {
+        const float4 t = *reinterpret_cast<const float4 *>(p);
+        v[0] = t.x; v[1] = t.y; v[2] = t.z; v[3] = t.w;
+    } else if constexpr (N == 2) {
+        const float2 t = *reinterpret_cast<const float2 *>(p);
+        v[0] = t.x; v[1] = t.y;
+    } else {
+        v[0] = *p;
+    }
+}
+
+template <int N>
+__device__ __forceinline__ void st_fv(float *p, const float *v) {
+    if constexpr (N == 4) *reinterpret_cast<float4 *>(p) = make_float4(v[0], v[1], v[2], v[3]);
+    else if constexpr (N == 2) *reinterpret_cast<float2 *>(p) = make_float2(v[0], v[1]);
+    else *p = v[0];
+}
+
+// Epilogue of the P, residual and trailing GEMMs.  Each epilogue thread holds one
+// row of the tile, so writing from registers would touch 32 rows per warp
+// access; instead the warp's 32 rows x HALF columns go through shared memory
+// (the operand ring is idle once the last chunk has been folded) and are then
+// processed row by row with the lanes across the columns: every global load and
+// store becomes one contiguous access.  `objacc` collects the fused objective of
+// EPI_RFULL (when requested).
+template <int HALF>
+__device__ __forceinline__ void epilogue_rows(const GemmArgs &g, float *stg, int r0, int c0, int lane,
+                                              const float (&acc)[HALF], int split, double &objacc) {
+    constexpr int LD = HALF + 4;          // padded row: spreads the column-wise writes over the banks
+    constexpr int VEC = HALF / 32;        // columns per lane
+#pragma unroll
+    for (int i = 0; i < HALF; i += 4)
+        *reinterpret_cast<float4 *>(stg + lane * LD + i) = make_float4(acc[i], acc[i + 1], acc[i + 2], acc[i + 3]);
+    __syncwarp();
+    const int cl = c0 + VEC * lane;
+    const bool full = cl + VEC <= g.N;
+    for (int rr = 0; rr < 32; ++rr) {
+        const int r = r0 + rr;
+        if (r >= g.M) break;
+        const int64_t rw = r;
+        float v[VEC];
+        ld_fv<VEC>(stg + rr * LD + VEC * lane, v);
+        if (g.mode == EPI_TRAIL) {
+            float *orow = g.out + static_cast<int64_t>(split) * g.split_stride + rw * g.ldo;
+            if (full) st_fv<VEC>(orow + cl, v);
+            else
+#pragma unroll
+                for (int e = 0; e < VEC; ++e)
+                    if (cl + e < g.N) orow[cl + e] = v[e];
+        } else if (g.mode == EPI_PINIT) {
+            float *orow = g.out + rw * g.ldo;
+            float o[VEC];
+#pragma unroll
+            for (int e = 0; e < VEC; ++e) o[e] = (cl + e < g.N) ? load_w(g, rw, cl + e) + v[e] : 0.0f;
+            if (full) st_fv<VEC>(orow + cl, o);
+            else
+#pragma unroll
+                for (int e = 0; e < VEC; ++e)
+                    if (cl + e < g.N) orow[cl + e] = o[e];
+        } else {   // EPI_RFULL: R in grid-step units, P / s - acc + z
+            const float sc = g.scale[r];
+            const float zz = g.zero[r];
+            const float *prow = g.P + rw * g.ldp;
+            float *orow = g.out + rw * g.ldo;
+            float pv[VEC], o[VEC];
+            if (full) ld_fv<VEC>(prow + cl, pv);
+            else
+#pragma unroll
+                for (int e = 0; e < VEC; ++e) pv[e] = (cl + e < g.N) ? prow[cl + e] : 0.0f;
+#pragma unroll
+            for (int e = 0; e < VEC; ++e) o[e] = (__fdiv_rn(pv[e], sc) - v[e]) + zz;
+            if (full) st_fv<VEC>(orow + cl, o);
+            else
+#pragma unroll
+                for (int e = 0; e < VEC; ++e)
+                    if (cl + e < g.N) orow[cl + e] = o[e];
+            if (g.obj_part) {
+                // (D Sigma)_ij = d_j (R_ij - What_ij) = d_j s (R'_ij - C_ij) with R' = R / s + z:
+                // f = sum D_ij d_j s (R'_ij - C_ij), D = W - What (- H)
+                float part = 0.0f;
+                if constexpr (VEC == 4) {
+                    // 4 columns per lane: W as 4 bf16 (8 bytes), codes as one word, d and H as float4
+                    const bool vec = full && g.w_is_bf16 && (g.ldw % 4) == 0 && (g.ldc % 4) == 0 &&
+                                     ((reinterpret_cast<uintptr_t>(g.W) & 7u) == 0) &&
+                                     ((reinterpret_cast<uintptr_t>(g.codes) & 3u) == 0) &&
+                                     (g.Hd == nullptr || (g.ldh % 4) == 0);
+                    if (vec) {
+                        const uint2 wraw = *reinterpret_cast<const uint2 *>(
+                            reinterpret_cast<const __nv_bfloat16 *>(g.W) + rw * g.ldw + cl);
+                        const uint32_t craw = *reinterpret_cast<const uint32_t *>(g.codes + rw * g.ldc + cl);
+                        float dv[4], hv[4] = {0.f, 0.f, 0.f, 0.f};
+                        ld_fv<4>(g.dvec + cl, dv);
+                        if (g.Hd) ld_fv<4>(g.Hd + rw * g.ldh + cl, hv);
+                        const __nv_bfloat162 w01 = *reinterpret_cast<const __nv_bfloat162 *>(&wraw.x);
+                        const __nv_bfloat162 w23 = *reinterpret_cast<const __nv_bfloat162 *>(&wraw.y);
+                        const float wv[4] = {__low2float(w01), __high2float(w01), __low2float(w23), __high2float(w23)};
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            const float cj = static_cast<float>((craw >> (8 * e)) & 0xffu);
+                            const float wh = sc * (cj - zz);
+                            const float t = (wv[e] - wh) - hv[e];
+                            const float dj = dv[e] > 0.0f ? dv[e] : 0.0f;
+                            part += t * dj * (sc * (o[e] - cj));
+                        }
+                        objacc += static_cast<double>(part);
+                        continue;
+                    }
+                }
+#pragma unroll
+                for (int e = 0; e < VEC; ++e) {
+                    const int c = cl + e;
+                    if (c < g.N) {
+                        const float dj = g.dvec[c];
+                        if (dj > 0.0f) {
+                            const float cj = static_cast<float>(g.codes[rw * g.ldc + c]);
+                            const float wh = sc * (cj - zz);
+                            float t = load_w(g, rw, c) - wh;
+                            if (g.Hd) t -= g.Hd[rw * g.ldh + c];
+                            part += t * dj * (sc * (o[e] - cj));
+                        }
+                    }
+                }
+                objacc += static_cast<double>(part);
+            }
+        }
+    }
+}
+
 template <int BN>
 __global__ void __launch_bounds__(320, 1)
     k_tc_gemm(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb,
@@ -335,16 +466,26 @@ __global__ void __launch_bounds__(320, 1)
         }
         double objacc = 0.0;
         if (ok && *abort_flag == 0) {
-            const int r = m0 + quad * 32 + lane;
+            // Sigma (mirrored writes) and the residual refresh (already vectorized along the
+            // thread's row, and its fused objective reads several arrays per element) write
+            // from registers; P and the trailing partials go row-wise through shared memory
+            if (g.mode == EPI_SIGMA || g.mode == EPI_RFULL) {
+                const int r = m0 + quad * 32 + lane;
 #pragma unroll
-            for (int q = 0; q < C::HALF / 32; ++q) {
-                const int c0 = n0 + half * C::HALF + q * 32;
-                if (c0 < g.N) {
-                    float v[32];
+                for (int q = 0; q < C::HALF / 32; ++q) {
+                    const int c0 = n0 + half * C::HALF + q * 32;
+                    if (c0 < g.N) {
+                        float v[32];
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) v[i] = acc[q * 32 + i];
-                    epilogue_row(g, r, c0, v, split, objacc);
+                        for (int i = 0; i < 32; ++i) v[i] = acc[q * 32 + i];
+                        epilogue_row(g, r, c0, v, split, objacc);
+                    }
                 }
+            } else {
+                // every MMA has completed (the last chunk was folded), so the operand
+                // ring is free: 8 warps x 32 rows x (HALF + 4) floats fit in it
+                float *stg = reinterpret_cast<float *>(smem) + (warp - 2) * 32 * (C::HALF + 4);
+                epilogue_rows<C::HALF>(g, stg, m0 + quad * 32, n0 + half * C::HALF, lane, acc, split, objacc);
             }
         }
         if (g.obj_part) {   // one fp64 partial per epilogue warp, reduced later in a fixed order
