@@ -80,25 +80,69 @@ __global__ void k_sigma_diag(const float *S, int64_t lds, int64_t p, float *d, u
     d[j] = v;
 }
 
-__global__ void k_sigma_planes(const float *S, int64_t lds, int64_t p, const float *d,
-                               __nv_bfloat16 *snt, int64_t ldn, unsigned *err) {
+// The hi/mid/lo split of one binary32 value.
+__device__ __forceinline__ void split3(float x, __nv_bfloat16 &h, __nv_bfloat16 &m, __nv_bfloat16 &l) {
+    h = __float2bfloat16_rn(x);
+    const float r1 = x - __bfloat162float(h);
+    m = __float2bfloat16_rn(r1);
+    l = __float2bfloat16_rn(r1 - __bfloat162float(m));
+}
+
+// One CTA per row j of Sigma (grid.y), 4 consecutive columns k per thread:
+// 16-byte reads of Sigma and d, 8-byte writes of each plane.
+__global__ void __launch_bounds__(256) k_sigma_planes(const float *S, int64_t lds, int64_t p, const float *d,
+                                                      __nv_bfloat16 *snt, int64_t ldn, unsigned *err) {
     bool bad = false;
+    const bool vec = (lds % 4 == 0) && ((reinterpret_cast<uintptr_t>(S) & 15u) == 0);
     for (int64_t j = blockIdx.y; j < p; j += gridDim.y) {
         const float dj = d[j];
         const bool jalive = dj > 0.0f;
-        for (int64_t k = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; k < p;
-             k += (int64_t)gridDim.x * blockDim.x) {
-            const float sv = S[j * lds + k];
-            if (!isfinite(sv)) bad = true;
-            float x = 0.0f;
-            if (jalive && k != j && d[k] > 0.0f) x = __fdiv_rn(sv, dj);
-            const __nv_bfloat16 h = __float2bfloat16_rn(x);
-            const float r1 = x - __bfloat162float(h);
-            const __nv_bfloat16 m = __float2bfloat16_rn(r1);
-            const __nv_bfloat16 l = __float2bfloat16_rn(r1 - __bfloat162float(m));
-            snt[j * ldn + k] = h;
-            snt[(p + j) * ldn + k] = m;
-            snt[(2 * p + j) * ldn + k] = l;
+        for (int64_t k0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) * 4; k0 < p;
+             k0 += (int64_t)gridDim.x * blockDim.x * 4) {
+            float sv[4], dk[4];
+            if (vec && k0 + 4 <= p) {
+                const float4 a = *reinterpret_cast<const float4 *>(S + j * lds + k0);
+                const float4 b = *reinterpret_cast<const float4 *>(d + k0);
+                sv[0] = a.x; sv[1] = a.y; sv[2] = a.z; sv[3] = a.w;
+                dk[0] = b.x; dk[1] = b.y; dk[2] = b.z; dk[3] = b.w;
+            } else {
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    sv[e] = (k0 + e < p) ? S[j * lds + k0 + e] : 0.0f;
+                    dk[e] = (k0 + e < p) ? d[k0 + e] : 0.0f;
+                }
+            }
+            __nv_bfloat16 h[4], m[4], l[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const int64_t k = k0 + e;
+                if (k < p && !isfinite(sv[e])) bad = true;
+                float x = 0.0f;
+                if (k < p && jalive && k != j && dk[e] > 0.0f) x = __fdiv_rn(sv[e], dj);
+                split3(x, h[e], m[e], l[e]);
+            }
+            __nv_bfloat16 *r0 = snt + j * ldn + k0;
+            __nv_bfloat16 *r1 = snt + (p + j) * ldn + k0;
+            __nv_bfloat16 *r2 = snt + (2 * p + j) * ldn + k0;
+            if (k0 + 4 <= p) {   // ldn is a multiple of 64, k0 of 4: 8-byte aligned
+                *reinterpret_cast<uint2 *>(r0) = make_uint2(
+                    (uint32_t)__bfloat16_as_ushort(h[0]) | ((uint32_t)__bfloat16_as_ushort(h[1]) << 16),
+                    (uint32_t)__bfloat16_as_ushort(h[2]) | ((uint32_t)__bfloat16_as_ushort(h[3]) << 16));
+                *reinterpret_cast<uint2 *>(r1) = make_uint2(
+                    (uint32_t)__bfloat16_as_ushort(m[0]) | ((uint32_t)__bfloat16_as_ushort(m[1]) << 16),
+                    (uint32_t)__bfloat16_as_ushort(m[2]) | ((uint32_t)__bfloat16_as_ushort(m[3]) << 16));
+                *reinterpret_cast<uint2 *>(r2) = make_uint2(
+                    (uint32_t)__bfloat16_as_ushort(l[0]) | ((uint32_t)__bfloat16_as_ushort(l[1]) << 16),
+                    (uint32_t)__bfloat16_as_ushort(l[2]) | ((uint32_t)__bfloat16_as_ushort(l[3]) << 16));
+            } else {
+#pragma unroll
+                for (int e = 0; e < 4; ++e)
+                    if (k0 + e < p) {
+                        r0[e] = h[e];
+                        r1[e] = m[e];
+                        r2[e] = l[e];
+                    }
+            }
         }
     }
     if (bad) set_error(err, ERR_NUMERIC);
@@ -164,11 +208,25 @@ __global__ void k_init_residual(const void *W, int w_bf16, int64_t ldw, const fl
                                 int64_t ldr) {
     for (int64_t i = blockIdx.y; i < q; i += gridDim.y) {
         const float s = scale[i], z = zero[i];
-        for (int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; j < p;
-             j += (int64_t)gridDim.x * blockDim.x) {
-            float w = load_elem(W, w_bf16, i * ldw + j);
-            if (H) w -= H[i * ldh + j];
-            R[i * ldr + j] = __fdiv_rn(w, s) + z;
+        for (int64_t j0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) * 4; j0 < p;
+             j0 += (int64_t)gridDim.x * blockDim.x * 4) {
+            float o[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const int64_t j = j0 + e;
+                float w = 0.0f;
+                if (j < p) {
+                    w = load_elem(W, w_bf16, i * ldw + j);
+                    if (H) w -= H[i * ldh + j];
+                }
+                o[e] = __fdiv_rn(w, s) + z;
+            }
+            float *rr = R + i * ldr + j0;
+            if (j0 + 4 <= p) *reinterpret_cast<float4 *>(rr) = make_float4(o[0], o[1], o[2], o[3]);   // ldr % 64 == 0
+            else
+#pragma unroll
+                for (int e = 0; e < 4; ++e)
+                    if (j0 + e < p) rr[e] = o[e];
         }
     }
 }
@@ -753,21 +811,25 @@ __global__ void __launch_bounds__(32 * kRowsMaxWarps, 1) k_cd_rows_lists(const C
     }
 }
 
-// obj[t] = obj[t-1] + sum_i rowdf_t[t][i] for nt sweeps (fixed order); prev may be NULL (0).
+// obj[t] = obj[t-1] + sum_i rowdf_t[t][i] for nt <= 32 sweeps; prev may be NULL (0).
+// Warp t sums sweep t (lane-strided, then a fixed butterfly: a fixed order); one
+// thread then runs the prefix over the sweeps.
 __global__ void k_obj_prefix(const double *rowdf_t, int64_t q, int nt, const double *prev, double *out) {
     __shared__ double sw[32];
-    double run = prev ? *prev : 0.0;
-    for (int t = 0; t < nt; ++t) {
+    const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (w < nt) {
         double acc = 0.0;
-        for (int64_t k = threadIdx.x; k < q; k += blockDim.x) acc += rowdf_t[static_cast<int64_t>(t) * q + k];
+        for (int64_t k = lane; k < q; k += 32) acc += rowdf_t[static_cast<int64_t>(w) * q + k];
         acc = warp_sum(acc);
-        if ((threadIdx.x & 31) == 0) sw[threadIdx.x >> 5] = acc;
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            for (int w = 0; w < (int)(blockDim.x >> 5); ++w) run += sw[w];
+        if (lane == 0) sw[w] = acc;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double run = prev ? *prev : 0.0;
+        for (int t = 0; t < nt; ++t) {
+            run += sw[t];
             out[t] = run;
         }
-        __syncthreads();
     }
 }
 
@@ -836,7 +898,8 @@ cudaError_t launch_cd_rows_lists(int B, const CdArgs &a, int t_begin, int t_end,
 
 cudaError_t launch_obj_prefix(const double *rowdf_t, int64_t q, int nt, const double *prev, double *out,
                               cudaStream_t s) {
-    k_obj_prefix<<<1, 1024, 0, s>>>(rowdf_t, q, nt, prev, out);
+    if (nt < 1 || nt > 32) return cudaErrorInvalidValue;
+    k_obj_prefix<<<1, 32 * nt, 0, s>>>(rowdf_t, q, nt, prev, out);
     return cudaGetLastError();
 }
 
@@ -1001,6 +1064,9 @@ static inline dim3 row_grid(int64_t rows, int64_t cols) {
     return dim3(static_cast<unsigned>(bx > 0 ? bx : 1), static_cast<unsigned>(rows < 65535 ? rows : 65535));
 }
 
+// for kernels that take 4 consecutive columns per thread
+static inline dim3 row_grid4(int64_t rows, int64_t cols) { return row_grid(rows, ceil_div(cols, 4)); }
+
 cudaError_t launch_grid(const void *W, int w_bf16, int64_t ldw, const float *H, int64_t ldh, int64_t q,
                         int64_t p, int bits, float *scale, float *zero, unsigned *err, cudaStream_t s) {
     k_grid<<<static_cast<unsigned>(q), 256, 0, s>>>(W, w_bf16, ldw, H, ldh, p,
@@ -1012,7 +1078,7 @@ cudaError_t launch_grid(const void *W, int w_bf16, int64_t ldw, const float *H, 
 cudaError_t launch_sigma_norm(const float *S, int64_t lds, int64_t p, float *d, __nv_bfloat16 *snt,
                               int64_t ldn, unsigned *err, cudaStream_t s) {
     k_sigma_diag<<<static_cast<unsigned>(ceil_div(p, 256)), 256, 0, s>>>(S, lds, p, d, err);
-    k_sigma_planes<<<row_grid(p, p), 256, 0, s>>>(S, lds, p, d, snt, ldn, err);
+    k_sigma_planes<<<row_grid4(p, p), 256, 0, s>>>(S, lds, p, d, snt, ldn, err);
     return cudaGetLastError();
 }
 
@@ -1032,7 +1098,7 @@ cudaError_t launch_make_planes(const void *W, int w_bf16, int64_t ldw, int64_t q
 cudaError_t launch_init_residual(const void *W, int w_bf16, int64_t ldw, const float *H, int64_t ldh,
                                  int64_t q, int64_t p, const float *scale, const float *zero, float *R,
                                  int64_t ldr, cudaStream_t s) {
-    k_init_residual<<<row_grid(q, p), 256, 0, s>>>(W, w_bf16, ldw, H, ldh, q, p, scale, zero, R, ldr);
+    k_init_residual<<<row_grid4(q, p), 256, 0, s>>>(W, w_bf16, ldw, H, ldh, q, p, scale, zero, R, ldr);
     return cudaGetLastError();
 }
 
