@@ -52,7 +52,7 @@ constexpr int kDefaultBlock = 256;
 constexpr int kDefaultPowerIters = 64;
 constexpr int kDefaultDenseSweeps = 1;
 constexpr int kSweepChunk = 32;          // list-mode sweeps per persistent launch
-constexpr int kFreeMaxChanges = 16;      // changes per row in the previous sweep below which a CTA runs free
+constexpr int kFreeMaxChanges = 64;      // changes per row in the previous sweep below which a CTA runs free
 
 // ---- workspace layout -----------------------------------------------------------
 struct Plan {

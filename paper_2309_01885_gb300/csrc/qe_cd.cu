@@ -319,7 +319,7 @@ struct CdCfg {
 // Delta'_ik Sigma_bar[k][block] to the row; Sigma_bar rows are fp32 and
 // contiguous over the block, so each change is one coalesced read of B floats
 // per warp.  Returns whether the row had any change in the window.
-template <int B, bool FULL>
+template <int B, bool FULL, int U = 4>
 __device__ __forceinline__ bool list_correction(const CdArgs &a, int64_t b0, int bw_, int64_t ii, bool row_ok,
                                                 int lane, float (&ps)[B / 32]) {
     constexpr int CPL = B / 32;
@@ -341,28 +341,28 @@ __device__ __forceinline__ bool list_correction(const CdArgs &a, int64_t b0, int
             for (int e0 = 0; e0 < c; e0 += 32) {
                 const uint32_t mine = (e0 + lane < c) ? seg[e0 + lane] : 0u;
                 const int ne = (c - e0) < 32 ? (c - e0) : 32;
-                // four changes in flight per step (the gather is bound by loads in flight);
+                // U changes in flight per step (the gather is bound by loads in flight);
                 // the sum still runs over the changes in list order
                 int u = 0;
-                for (; u + 4 <= ne; u += 4) {
-                    const float *r[4];
-                    float dv[4];
+                for (; u + U <= ne; u += U) {
+                    const float *r[U];
+                    float dv[U];
 #pragma unroll
-                    for (int e = 0; e < 4; ++e) {
+                    for (int e = 0; e < U; ++e) {
                         const uint32_t ev = __shfl_sync(0xffffffffu, mine, u + e);
                         r[e] = sbk + static_cast<int64_t>(ev & 0xffffu) * a.lds;
                         dv[e] = static_cast<float>(static_cast<int16_t>(ev >> 16));
                     }
-                    float v[4][CPL];
+                    float v[U][CPL];
 #pragma unroll
-                    for (int e = 0; e < 4; ++e)
+                    for (int e = 0; e < U; ++e)
 #pragma unroll
                         for (int h = 0; h < CPL; ++h)
                             v[e][h] = (FULL || 32 * h + lane < bw) ? __ldg(r[e] + 32 * h) : 0.0f;
 #pragma unroll
                     for (int h = 0; h < CPL; ++h)
 #pragma unroll
-                        for (int e = 0; e < 4; ++e) ps[h] = fmaf(dv[e], v[e][h], ps[h]);
+                        for (int e = 0; e < U; ++e) ps[h] = fmaf(dv[e], v[e][h], ps[h]);
                 }
                 for (; u < ne; ++u) {
                     const uint32_t e1 = __shfl_sync(0xffffffffu, mine, u);
@@ -656,7 +656,8 @@ __global__ void __launch_bounds__(1024, 1) k_cd_block_chg(const CdArgs a) {
         cd_epilogue<B, FULL, false>(a, a.b0, a.bw, i, lane, code, dlt, true);
 }
 
-// One block of one row in the persistent list kernel: stage t = R + the
+// One block of one row in the persistent list kernel (R and the codes stream with
+// evict-first hints, so that L2 keeps the Sigma_bar rows the gathers re-read): stage t = R + the
 // change-list correction (storing it back as the block's base when the window
 // held a change), wait for the block's packed Sigma_bar, decide, write back.
 // Returns false when the wait gave up.
@@ -670,20 +671,36 @@ __device__ __forceinline__ bool rows_block(const CdArgs &a, int64_t b0, int bw_,
     float ps[CPL], st[CPL], t[CPL];
 #pragma unroll
     for (int h = 0; h < CPL; ++h) ps[h] = 0.0f;
-    // the gathers first (they hold the registers), then the block's base and codes
-    const bool changed = list_correction<B, FULL>(a, b0, bw, ii, row_ok, lane, ps);
+    bool changed;
+    if (LATE) {
+        // few listed changes: issue the block's base and codes first, so their
+        // latency overlaps the count / entry / gather chain
 #pragma unroll
-    for (int h = 0; h < CPL; ++h) {
-        const int l = 32 * h + lane;
-        const bool ok = row_ok && (FULL || l < bw);
-        t[h] = (ok ? a.R[ii * a.ldr + b0 + l] : 0.0f) + ps[h];
-        st[h] = ok ? static_cast<float>(a.codes[ii * a.ldc + b0 + l]) : 0.0f;
+        for (int h = 0; h < CPL; ++h) {
+            const int l = 32 * h + lane;
+            const bool ok = row_ok && (FULL || l < bw);
+            t[h] = ok ? __ldcs(a.R + ii * a.ldr + b0 + l) : 0.0f;
+            st[h] = ok ? static_cast<float>(__ldcs(a.codes + ii * a.ldc + b0 + l)) : 0.0f;
+        }
+        changed = list_correction<B, FULL, 2>(a, b0, bw, ii, row_ok, lane, ps);
+#pragma unroll
+        for (int h = 0; h < CPL; ++h) t[h] += ps[h];
+    } else {
+        // the gathers first (many changes: they hold the registers), then base and codes
+        changed = list_correction<B, FULL>(a, b0, bw, ii, row_ok, lane, ps);
+#pragma unroll
+        for (int h = 0; h < CPL; ++h) {
+            const int l = 32 * h + lane;
+            const bool ok = row_ok && (FULL || l < bw);
+            t[h] = (ok ? __ldcs(a.R + ii * a.ldr + b0 + l) : 0.0f) + ps[h];
+            st[h] = ok ? static_cast<float>(__ldcs(a.codes + ii * a.ldc + b0 + l)) : 0.0f;
+        }
     }
     if (changed) {
 #pragma unroll
         for (int h = 0; h < CPL; ++h) {
             const int l = 32 * h + lane;
-            if (row_ok && (FULL || l < bw)) a.R[ii * a.ldr + b0 + l] = t[h];
+            if (row_ok && (FULL || l < bw)) __stcs(a.R + ii * a.ldr + b0 + l, t[h]);
         }
     }
     if (!LATE && !mbar_wait_bounded(bar, parity, nullptr)) return false;
