@@ -62,6 +62,34 @@ def test_sigma_bf16_token_major_and_accumulate():
     _sigma_check(S2, parity.f64(X))
 
 
+@pytest.mark.parametrize("accumulate", [False, True])
+def test_sigma_two_waves(accumulate):
+    """p = 3584 has 210 tiles on or above the diagonal, more than one wave on 152 SMs,
+    with heavy features; direct and accumulated over two token halves.  Sampled
+    entries against binary64 dot products of the same bf16 X (Lemma 1), exact
+    symmetry, every diagonal entry."""
+    p, n = 3584, 1536
+    X = inputs.calib_inputs(p, n, dtype=torch.bfloat16, seed=5, device="cuda", heavy_frac=0.02,
+                            heavy_mult=30.0)
+    if accumulate:
+        Sg = qe.qe_build_sigma(X[:, :768].contiguous())
+        qe.qe_build_sigma(X[:, 768:].contiguous(), Sigma=Sg, accumulate=True)
+    else:
+        Sg = qe.qe_build_sigma(X)
+    torch.cuda.synchronize()
+    assert qe.qe_sync_status() == qe.QE_OK
+    assert torch.equal(Sg, Sg.t())
+    rng = np.random.default_rng(6)
+    bits = X.contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+    a = np.concatenate([np.arange(p), rng.integers(0, p, 6000), np.arange(p - 300, p)])
+    b = np.concatenate([np.arange(p), rng.integers(0, p, 6000), rng.integers(0, p, 300)])
+    ref = O.sigma_pairs_bf16(bits, a, b)
+    got = Sg[torch.from_numpy(a).cuda(), torch.from_numpy(b).cuda()].double().cpu().numpy()
+    d = ref[:p]
+    tol = 1e-5 * np.sqrt(d[a] * d[b])
+    assert np.all(np.abs(got - ref) <= tol), f"max err/tol {np.max(np.abs(got - ref) / tol):.3f}"
+
+
 def test_sigma_host_streamed():
     """Sigma from pinned host X streamed in token chunks (ragged last chunk), the
     staging area reused by the next calls, and accumulation over two token ranges
