@@ -87,6 +87,13 @@ typedef struct {
      * dense form throughout;
      * negative is QE_ERR_INVALID_ARG.  Ignored by the outlier variant. */
     int dense_sweeps;
+    /* List sweeps: the rows of a CTA step through the column blocks together
+     * (sharing each packed Sigma_bar block) while they made more than this many
+     * changes per row in the previous sweep, then each row runs on its own.
+     * Both modes take the same decisions in the same order; only the speed
+     * differs.  0 = default (64); -1 = always together; below -1 is
+     * QE_ERR_INVALID_ARG.  Ignored by the outlier variant. */
+    int free_changes;
     /* Optional warm start (Sec. 3.1, "initialized with ... any other algorithm"):
      * q x p codes (leading dimension p) on the grid this call computes.  NULL = start at W. */
     const uint8_t *init_codes;

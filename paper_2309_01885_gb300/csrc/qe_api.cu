@@ -515,6 +515,10 @@ static int dense_sweeps(const qe_opts *o) {
     return (o && o->dense_sweeps) ? o->dense_sweeps : kDefaultDenseSweeps;
 }
 
+static int free_changes(const qe_opts *o) {
+    return (o && o->free_changes) ? o->free_changes : kFreeMaxChanges;
+}
+
 // structured: the call accepts structured_outliers = 1 (the outlier variant)
 static qe_status check_opts(const qe_opts *o, bool structured = false) {
     if (!o) return QE_OK;
@@ -522,7 +526,7 @@ static qe_status check_opts(const qe_opts *o, bool structured = false) {
     if (o->structured_outliers != 0 && !(structured && o->structured_outliers == 1)) return QE_ERR_UNSUPPORTED;
     if (o->block_width != 0 && o->block_width != 64 && o->block_width != 128 && o->block_width != 256)
         return QE_ERR_UNSUPPORTED;
-    if (o->power_iters < 0 || o->dense_sweeps < 0) return QE_ERR_INVALID_ARG;
+    if (o->power_iters < 0 || o->dense_sweeps < 0 || o->free_changes < -1) return QE_ERR_INVALID_ARG;
     if (o->workspace && o->workspace_bytes == 0) return QE_ERR_INVALID_ARG;
     return QE_OK;
 }
@@ -772,7 +776,7 @@ qe_status qe_quantize_layer(const void *W, qe_dtype w_dtype, int64_t q, int64_t 
             Timed tm(c.timer, QE_KERNEL_CD_LISTS, c.s);
             // the lists are empty at the window start (t0): that sweep steps in lockstep
             QE_CK(launch_cd_rows_lists(pl.B, a, t, te, c.rowdft, opts ? opts->sweep_codes : nullptr, t == t0,
-                                       kFreeMaxChanges, c.nsm, c.s));
+                                       free_changes(opts), c.nsm, c.s));
         }
         QE_CK(launch_obj_prefix(c.rowdft, q, te - t, t == 0 ? c.objbase : obj + t - 1, obj + t, c.s));
         t = te;

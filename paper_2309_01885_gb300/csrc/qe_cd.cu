@@ -712,6 +712,158 @@ __device__ __forceinline__ bool rows_block(const CdArgs &a, int64_t b0, int bw_,
     return true;
 }
 
+// Free-mode shared memory of one warp of the persistent list kernel: the row's
+// window (kWinCap entries) and a staging area for the Sigma_bar row segments of
+// the correction, filled by cp.async so that many segments are in flight
+// without holding registers.
+constexpr int kFreeWarpBytes = 8192;
+constexpr int kWinCap = 128;
+constexpr int kStageFloats = (kFreeWarpBytes - 4 * kWinCap) / 4;
+
+// Window of one row: the entries of all its change lists (the changes of every
+// block's most recent visit) in ascending global column, each as
+// column | Delta' << 16 (p <= 65536).  All lists of 32 blocks are read in one
+// gather.  Returns the number of entries, or -1 when there are more than
+// kWinCap (the lists in global memory serve then).
+template <int B>
+__device__ __forceinline__ int build_window(const CdArgs &a, int64_t i, int lane, uint32_t *win) {
+    const int64_t rb = i * a.nblk;
+    int wn = 0;
+    for (int c0 = 0; c0 < a.nblk; c0 += 32) {
+        const int cnt = (c0 + lane < a.nblk) ? a.lcnt[rb + c0 + lane] : 0;
+        int incl = cnt;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int v = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += v;
+        }
+        const int tot = __shfl_sync(0xffffffffu, incl, 31);
+        if (tot == 0) continue;
+        if (wn + tot > kWinCap) return -1;
+        uint32_t e[kWinCap / 32];
+#pragma unroll
+        for (int k = 0; k < kWinCap / 32; ++k) {
+            const int x = 32 * k + lane;   // entry number within the chunk
+            // its block: how many blocks have an inclusive count <= x
+            int pos = 0;
+#pragma unroll
+            for (int st = 16; st > 0; st >>= 1) {
+                const int v = __shfl_sync(0xffffffffu, incl, pos + st - 1);
+                if (v <= x) pos += st;
+            }
+            const int excl = __shfl_sync(0xffffffffu, incl - cnt, pos);
+            e[k] = 0u;
+            if (x < tot) {
+                const uint32_t raw = a.lent[(rb + c0 + pos) * B + (x - excl)];
+                e[k] = (static_cast<uint32_t>((c0 + pos) * B) + (raw & 0xffffu)) | (raw & 0xffff0000u);
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < kWinCap / 32; ++k)
+            if (32 * k + lane < tot) win[wn + 32 * k + lane] = e[k];
+        wn += tot;
+    }
+    __syncwarp();
+    return wn;
+}
+
+// One block of one row in the free mode with the shared-memory window: the same
+// steps as rows_block (the correction adds the same changes in the same order,
+// so the same sums), then this block's entries in the window are replaced by
+// the changes just made.  The lists in global memory are written as well, so a
+// window that outgrows kWinCap (wn = -1) hands over to them.
+template <int B, bool FULL>
+__device__ __forceinline__ void rows_block_win(const CdArgs &a, int64_t b0, int bw_, int64_t i, int lane, float s2,
+                                               double &dfacc, int &nchg, uint32_t *win, float *stg, int &wn) {
+    constexpr int CPL = B / 32;
+    constexpr int NST = kStageFloats / B;       // segments per staged batch
+    constexpr int SEG16 = B / 4;                // 16-byte pieces per segment
+    const int bw = FULL ? B : bw_;
+    float ps[CPL], st[CPL], t[CPL];
+#pragma unroll
+    for (int h = 0; h < CPL; ++h) {
+        const int l = 32 * h + lane;
+        const bool ok = FULL || l < bw;
+        t[h] = ok ? __ldcs(a.R + i * a.ldr + b0 + l) : 0.0f;
+        st[h] = ok ? static_cast<float>(__ldcs(a.codes + i * a.ldc + b0 + l)) : 0.0f;
+        ps[h] = 0.0f;
+    }
+    const float *sb = a.sbar + b0;
+    for (int u0 = 0; u0 < wn; u0 += NST) {
+        const int nb = (wn - u0) < NST ? (wn - u0) : NST;
+        for (int x = lane; x < nb * SEG16; x += 32) {
+            const int e = x / SEG16, c = x % SEG16;
+            if (FULL || 4 * c < bw)
+                cp_async16(stg + e * B + 4 * c, sb + static_cast<int64_t>(win[u0 + e] & 0xffffu) * a.lds + 4 * c);
+        }
+        cp_async_wait_all();
+        __syncwarp();
+        for (int e = 0; e < nb; ++e) {
+            const float dv = static_cast<float>(static_cast<int16_t>(win[u0 + e] >> 16));
+#pragma unroll
+            for (int h = 0; h < CPL; ++h)
+                if (FULL || 32 * h + lane < bw) ps[h] = fmaf(dv, stg[e * B + 32 * h + lane], ps[h]);
+        }
+        __syncwarp();
+    }
+#pragma unroll
+    for (int h = 0; h < CPL; ++h) t[h] += ps[h];
+    if (wn > 0) {
+#pragma unroll
+        for (int h = 0; h < CPL; ++h) {
+            const int l = 32 * h + lane;
+            if (FULL || l < bw) __stcs(a.R + i * a.ldr + b0 + l, t[h]);
+        }
+    }
+    float code[CPL], dlt[CPL];
+    nchg += chg_decide<B, FULL, true>(nullptr, a.d + b0, bw, a.maxq, s2, true, lane, t, st, code, dlt, dfacc,
+                                      a.sbar + b0 * a.lds + b0, a.lds);
+    cd_epilogue<B, FULL, true>(a, b0, bw, i, lane, code, dlt, true);
+    // window = [entries left of the block (k1)] [this visit's changes (nn)] [entries right of it]
+    int k1 = 0, k2 = 0;
+#pragma unroll
+    for (int k = 0; k < kWinCap / 32; ++k) {
+        const int x = 32 * k + lane;
+        const int64_t col = x < wn ? static_cast<int64_t>(win[x] & 0xffffu) : INT64_MAX;
+        k1 += __popc(__ballot_sync(0xffffffffu, col < b0));
+        k2 += __popc(__ballot_sync(0xffffffffu, col < b0 + bw));
+    }
+    int nn = 0;
+#pragma unroll
+    for (int h = 0; h < CPL; ++h)
+        nn += __popc(__ballot_sync(0xffffffffu, (FULL || 32 * h + lane < bw) && dlt[h] != 0.0f));
+    const int wn2 = k1 + nn + (wn - k2);
+    if (wn2 > kWinCap) {
+        wn = -1;
+        return;
+    }
+    uint32_t tail[kWinCap / 32];
+#pragma unroll
+    for (int k = 0; k < kWinCap / 32; ++k) {
+        const int x = k2 + 32 * k + lane;
+        tail[k] = x < wn ? win[x] : 0u;
+    }
+    __syncwarp();
+#pragma unroll
+    for (int k = 0; k < kWinCap / 32; ++k)
+        if (k2 + 32 * k + lane < wn) win[k1 + nn + 32 * k + lane] = tail[k];
+    int r = 0;
+#pragma unroll
+    for (int h = 0; h < CPL; ++h) {
+        const int l = 32 * h + lane;
+        const bool ch = (FULL || l < bw) && dlt[h] != 0.0f;
+        const unsigned m = __ballot_sync(0xffffffffu, ch);
+        if (ch) {
+            const int16_t dv = static_cast<int16_t>(__float2int_rn(dlt[h]));
+            win[k1 + r + __popc(m & ((1u << lane) - 1u))] =
+                static_cast<uint32_t>(b0 + l) | (static_cast<uint32_t>(static_cast<uint16_t>(dv)) << 16);
+        }
+        r += __popc(m);
+    }
+    __syncwarp();
+    wn = wn2;
+}
+
 // Rolling-window sweeps t_begin .. t_end-1 with the change-list correction,
 // persistent over column blocks and sweeps.  With the correction taken from
 // each row's own change lists, rows need nothing from one another (rows are
@@ -775,6 +927,8 @@ __global__ void __launch_bounds__(32 * kRowsMaxWarps, 1) k_cd_rows_lists(const C
             for (int w = 0; w < nwarps; ++w) cta += s_chg[w];
             free_run = !forced_lockstep &&
                        static_cast<int64_t>(cta) <= static_cast<int64_t>(free_max_changes) * nwarps;
+            // the free mode reuses the shared memory of the packed block and its barrier
+            if (free_run && threadIdx.x == 0) mbar_inval(bar);
             __syncthreads();   // s_chg is rewritten at the next sweep
         }
         double dfacc = 0.0;
@@ -782,13 +936,24 @@ __global__ void __launch_bounds__(32 * kRowsMaxWarps, 1) k_cd_rows_lists(const C
         if (free_run) {
             // A row whose previous sweep changed nothing is at a fixed point: its window
             // is empty, so every block stages the values it decided on last time.
+            // With at most kWinCap changes the window lives in the warp's shared memory
+            // (the packed block is no longer needed once the CTA runs free).
             if (row_ok && prev > 0) {
+                uint32_t *win = reinterpret_cast<uint32_t *>(reinterpret_cast<char *>(cd_smem) + warp * kFreeWarpBytes);
+                float *stg = reinterpret_cast<float *>(win + kWinCap);
+                int wn = (prev <= kWinCap && a.p <= 65536) ? build_window<B>(a, i, lane, win) : -1;
                 for (int64_t b0 = 0; b0 < a.p; b0 += B) {
                     const int bw = static_cast<int>((a.p - b0) < B ? (a.p - b0) : B);
-                    if (bw == B)
+                    if (wn >= 0) {
+                        if (bw == B)
+                            rows_block_win<B, true>(a, b0, bw, i, lane, s2, dfacc, nchg, win, stg, wn);
+                        else
+                            rows_block_win<B, false>(a, b0, bw, i, lane, s2, dfacc, nchg, win, stg, wn);
+                    } else if (bw == B) {
                         rows_block<B, true, true>(a, b0, bw, tri, bar, 0u, i, row_ok, lane, s2, dfacc, nchg);
-                    else
+                    } else {
                         rows_block<B, false, true>(a, b0, bw, tri, bar, 0u, i, row_ok, lane, s2, dfacc, nchg);
+                    }
                 }
             }
         } else {
@@ -889,13 +1054,15 @@ static cudaError_t launch_cd_rows_b(const CdArgs &a, int t_begin, int t_end, dou
                                    uint8_t *sweep_codes, int first_lockstep, int free_max_changes, int nsm,
                                    cudaStream_t s) {
     using C = CdCfg<B>;
-    cudaError_t e = cudaFuncSetAttribute(k_cd_rows_lists<B>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
-    if (e != cudaSuccess) return e;
     int64_t warps = ceil_div(a.q, nsm);
     if (warps > kRowsMaxWarps) warps = kRowsMaxWarps;
     if (warps < 1) warps = 1;
+    // the packed block (lockstep) or one free-mode area per warp, whichever is larger
+    const int smem = static_cast<int>(warps * kFreeWarpBytes > C::SMEM ? warps * kFreeWarpBytes : C::SMEM);
+    cudaError_t e = cudaFuncSetAttribute(k_cd_rows_lists<B>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
     const unsigned grid = static_cast<unsigned>(ceil_div(a.q, warps));
-    k_cd_rows_lists<B><<<grid, static_cast<unsigned>(32 * warps), C::SMEM, s>>>(
+    k_cd_rows_lists<B><<<grid, static_cast<unsigned>(32 * warps), smem, s>>>(
         a, t_begin, t_end, rowdf_t, sweep_codes, first_lockstep, free_max_changes);
     return cudaGetLastError();
 }

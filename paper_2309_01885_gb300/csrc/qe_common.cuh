@@ -71,6 +71,23 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint64_t *bar, uint32_t parity
     }
 }
 
+__device__ __forceinline__ void mbar_inval(uint64_t *bar) {
+    asm volatile("mbarrier.inval.shared::cta.b64 [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+// ---- cp.async (per-thread asynchronous copies into shared memory) -------------
+// 16 bytes global -> shared, cached in L2 only; both addresses 16-byte aligned.
+__device__ __forceinline__ void cp_async16(void *dst, const void *src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)),
+                 "l"(static_cast<unsigned long long>(__cvta_generic_to_global(src)))
+                 : "memory");
+}
+
+// Wait for all of this thread's cp.async copies (they always complete).
+__device__ __forceinline__ void cp_async_wait_all() {
+    asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+}
+
 // ---- TMA --------------------------------------------------------------------
 // 2-D tiled bulk tensor load into shared memory, completion counted in bytes on
 // `bar`.  c0 is the innermost (contiguous) coordinate; callers keep

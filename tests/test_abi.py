@@ -83,6 +83,10 @@ def test_invalid_arguments_rejected_synchronously(lib):
     assert L.qe_quantize_layer(_fake(), qe.QE_F32, 4, 4, 4, _fake(2), 3, 1, ctypes.byref(o), _fake(3),
                                _fake(4), _fake(5), _fake(6), None) == qe.QE_ERR_INVALID_ARG
     o = qe.QEOpts()
+    o.free_changes = -2
+    assert L.qe_quantize_layer(_fake(), qe.QE_F32, 4, 4, 4, _fake(2), 3, 1, ctypes.byref(o), _fake(3),
+                               _fake(4), _fake(5), _fake(6), None) == qe.QE_ERR_INVALID_ARG
+    o = qe.QEOpts()
     o.block_width = 48
     assert L.qe_quantize_layer(_fake(), qe.QE_F32, 4, 4, 4, _fake(2), 3, 1, ctypes.byref(o), _fake(3),
                                _fake(4), _fake(5), _fake(6), None) == qe.QE_ERR_UNSUPPORTED
