@@ -66,16 +66,16 @@ class Oracle:
         lib.qo_objective_rows.argtypes = [_f64p, _f64p, _u8p, _f32p, _f32p, _i64, _i64, _f64p, _f64p]
         lib.qo_objective_rows.restype = None
         lib.qo_quantease_alg1.argtypes = [_f64p, _i64, _i64, _f64p, _f32p, _f32p, _int, _int,
-                                          _u8p, _u8p, _u8p, _f64p, _u8p, _f64p]
+                                          _u8p, _u8p, _u8p, _f64p, _u8p, _f64p, _int]
         lib.qo_quantease_alg1.restype = _int
         lib.qo_quantease_alg1_f32.argtypes = [_f64p, _i64, _i64, _f32p, _f32p, _f32p, _int, _int,
-                                              _u8p, _u8p, _u8p, _f64p, _u8p, _f64p]
+                                              _u8p, _u8p, _u8p, _f64p, _u8p, _f64p, _int]
         lib.qo_quantease_alg1_f32.restype = _int
         lib.qo_sigma_pairs_bf16.argtypes = [ctypes.POINTER(ctypes.c_uint16), _i64, _i64, _i64p, _i64p,
                                             _i64, _f64p]
         lib.qo_sigma_pairs_bf16.restype = None
         lib.qo_quantease_alg3.argtypes = [_f64p, _i64, _i64, _f64p, _f32p, _f32p, _int, _int,
-                                          _u8p, _f64p]
+                                          _u8p, _f64p, _int]
         lib.qo_quantease_alg3.restype = _int
         lib.qo_power_lambda.argtypes = [_f64p, _i64, _int]
         lib.qo_power_lambda.restype = ctypes.c_double
@@ -142,9 +142,11 @@ class Oracle:
 
     # -- Algorithm 1 / 3 ----------------------------------------------------
     def alg1(self, W, S, scale, zero, bits, iters, init_codes=None, forced=None,
-             record=False, want_beta=False):
+             record=False, want_beta=False, relax_period=0):
         """Algorithm 1.  Returns dict(codes, obj_rows[iters, q], obj[iters],
         sweep_codes[iters, q, p] if record, beta[iters, q, p] if want_beta).
+        relax_period > 0: sweeps t (from 1) with t mod relax_period = 0 and t < iters
+        keep beta~ unquantized (the relax heuristic of Sec. 3.2).
         A float32 S is read as is and promoted exactly row by row (same binary64
         arithmetic, half the host memory); anything else is converted to float64."""
         W = _f64(W)
@@ -163,7 +165,7 @@ class Oracle:
             _ptr(np.ascontiguousarray(scale, np.float32), _f32p),
             _ptr(np.ascontiguousarray(zero, np.float32), _f32p), bits, iters,
             _ptr(ic, _u8p), _ptr(fc, _u8p), _ptr(codes, _u8p), _ptr(obj_rows, _f64p),
-            _ptr(sweep, _u8p), _ptr(beta, _f64p))
+            _ptr(sweep, _u8p), _ptr(beta, _f64p), relax_period)
         if rc:
             raise MemoryError("oracle alg1 allocation failed")
         out = dict(codes=codes, obj_rows=obj_rows, obj=obj_rows.sum(axis=1))
@@ -173,7 +175,7 @@ class Oracle:
             out["beta"] = beta
         return out
 
-    def alg3(self, W, S, scale, zero, bits, iters):
+    def alg3(self, W, S, scale, zero, bits, iters, relax_period=0):
         W = _f64(W)
         S = _f64(S)
         q, p = W.shape
@@ -183,7 +185,7 @@ class Oracle:
             _ptr(W, _f64p), q, p, _ptr(S, _f64p),
             _ptr(np.ascontiguousarray(scale, np.float32), _f32p),
             _ptr(np.ascontiguousarray(zero, np.float32), _f32p), bits, iters,
-            _ptr(codes, _u8p), _ptr(obj_rows, _f64p))
+            _ptr(codes, _u8p), _ptr(obj_rows, _f64p), relax_period)
         if rc:
             raise MemoryError("oracle alg3 allocation failed")
         return dict(codes=codes, obj_rows=obj_rows, obj=obj_rows.sum(axis=1))

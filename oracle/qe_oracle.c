@@ -18,8 +18,8 @@
  * (brute-force 1-D argmin, exhaustive search on tiny layers, monotone
  * objective, Algorithm 1 == Algorithm 3, diagonal Sigma == round-to-nearest,
  * direct ||WX - W^X||^2, eigvalsh for lambda_max, a full sort for P_s, and
- * the IHT descent of Lemma 3).  The relax-every-third-iteration heuristic of
- * Sec. 3.2 is not implemented here (parity unpinned, not on the hot path).
+ * the IHT descent of Lemma 3, and for the relax heuristic one Gauss-Seidel
+ * step of the normal equations per relaxed sweep).
  */
 #include <math.h>
 #include <stdint.h>
@@ -221,10 +221,14 @@ void qo_objective_rows(const double *W, const double *H, const uint8_t *codes,
  * of the objective; it is set to the nearest level of the target and fixed.
  * forced (p codes, may be NULL): use these codes instead of q_i(-u) (teacher
  * forcing; beta~ is still recorded).  beta (p, may be NULL) receives beta~.
+ * relax != 0: the relax heuristic of Sec. 3.2, What_ij = beta~ itself (no
+ * quantization, forced ignored); codes[j] then records q_i(beta~), the nearest
+ * level, as a view of the relaxed row.  Dead columns stay on their level.
  */
 static void qo_sweep_row(const qo_sig *S, int64_t p, double s, double z, int maxq,
                          const double *tgt, const double *TS, double *Wh, double *WS,
-                         const uint8_t *forced, uint8_t *codes, double *beta, double *buf)
+                         const uint8_t *forced, uint8_t *codes, double *beta, double *buf,
+                         int relax)
 {
     for (int64_t j = 0; j < p; ++j) {
         const double *Sj = qo_srow(S, j, buf);
@@ -236,8 +240,13 @@ static void qo_sweep_row(const qo_sig *S, int64_t p, double s, double z, int max
             double old = Wh[j];
             for (int64_t k = 0; k < p; ++k)          /* part (A) */
                 WS[k] -= old * Sj[k];
-            c = forced ? (int)forced[j] : qo_code(b, s, z, maxq);
-            Wh[j] = qo_level(c, s, z);
+            if (relax) {
+                c = qo_code(b, s, z, maxq);
+                Wh[j] = b;
+            } else {
+                c = forced ? (int)forced[j] : qo_code(b, s, z, maxq);
+                Wh[j] = qo_level(c, s, z);
+            }
             for (int64_t k = 0; k < p; ++k)          /* part (B) */
                 WS[k] += Wh[j] * Sj[k];
             if (beta) beta[j] = b;
@@ -265,18 +274,30 @@ static void qo_row_times_sigma(const double *x, const qo_sig *S, int64_t p, doub
 }
 
 /*
+ * Relax heuristic of Sec. 3.2 (a reading of "every other third iteration"):
+ * with period R > 0, sweep t (counted from 1) is relaxed when t mod R = 0 and
+ * t < iters, so the last sweep always quantizes.  R = 0: never.
+ */
+static int qo_relaxed(int relax_period, int t1, int iters)
+{
+    return relax_period > 0 && t1 % relax_period == 0 && t1 < iters;
+}
+
+/*
  * Algorithm 1.  Start: What = W (Sec. 3.1), or the levels of init_codes.
  *   codes       q*p   out: codes after the last sweep
  *   obj_rows    iters*q out (may be NULL): f_i after each sweep
  *   sweep_codes iters*q*p out (may be NULL): codes after each sweep
  *   forced      iters*q*p in (may be NULL): teacher-forced codes per sweep
- *   beta        iters*q*p out (may be NULL): beta~ of every update
+ *   beta        iters*q*p out (may be NULL): beta~ of every update (in a relaxed
+ *               sweep, the relaxed row itself)
+ *   relax_period  the relax heuristic (qo_relaxed); 0 = off
  */
 static int qo_alg1_core(const double *W, int64_t q, int64_t p, const qo_sig *S,
                         const float *scale, const float *zero, int bits, int iters,
                         const uint8_t *init_codes, const uint8_t *forced,
                         uint8_t *codes, double *obj_rows, uint8_t *sweep_codes,
-                        double *beta)
+                        double *beta, int relax_period)
 {
     const int maxq = (1 << bits) - 1;
     int err = 0;
@@ -300,7 +321,8 @@ static int qo_alg1_core(const double *W, int64_t q, int64_t p, const qo_sig *S,
                 const size_t off = ((size_t)t * (size_t)q + (size_t)i) * (size_t)p;
                 qo_sweep_row(S, p, s, z, maxq, Wi, TS, Wh, WS,
                              forced ? forced + off : NULL, codes + i * p,
-                             beta ? beta + off : NULL, buf);
+                             beta ? beta + off : NULL, buf,
+                             qo_relaxed(relax_period, t + 1, iters));
                 if (sweep_codes)
                     memcpy(sweep_codes + off, codes + i * p, (size_t)p);
                 if (obj_rows) {
@@ -319,11 +341,11 @@ int qo_quantease_alg1(const double *W, int64_t q, int64_t p, const double *S,
                       const float *scale, const float *zero, int bits, int iters,
                       const uint8_t *init_codes, const uint8_t *forced,
                       uint8_t *codes, double *obj_rows, uint8_t *sweep_codes,
-                      double *beta)
+                      double *beta, int relax_period)
 {
     const qo_sig Sg = {S, NULL, p};
     return qo_alg1_core(W, q, p, &Sg, scale, zero, bits, iters, init_codes, forced, codes,
-                        obj_rows, sweep_codes, beta);
+                        obj_rows, sweep_codes, beta, relax_period);
 }
 
 /* Algorithm 1 with Sigma given in binary32 (promoted exactly; same arithmetic). */
@@ -331,11 +353,11 @@ int qo_quantease_alg1_f32(const double *W, int64_t q, int64_t p, const float *S,
                           const float *scale, const float *zero, int bits, int iters,
                           const uint8_t *init_codes, const uint8_t *forced,
                           uint8_t *codes, double *obj_rows, uint8_t *sweep_codes,
-                          double *beta)
+                          double *beta, int relax_period)
 {
     const qo_sig Sg = {NULL, S, p};
     return qo_alg1_core(W, q, p, &Sg, scale, zero, bits, iters, init_codes, forced, codes,
-                        obj_rows, sweep_codes, beta);
+                        obj_rows, sweep_codes, beta, relax_period);
 }
 
 /* ------------------------------------------------------------------------- */
@@ -350,10 +372,11 @@ int qo_quantease_alg1_f32(const double *W, int64_t q, int64_t p, const float *S,
  *     per column j: beta = P_:,j - Ph_:,j + dW_:,1:j Sn_1:j,j;  What_:,j = q(beta);
  *                   dW_:,j -= What_:,j.
  * Dead columns (Sigma_jj <= 0) are set to the nearest level of W and fixed.
+ * In a relaxed sweep (qo_relaxed) What_:,j = beta itself, as in Algorithm 1.
  */
 int qo_quantease_alg3(const double *W, int64_t q, int64_t p, const double *S,
                       const float *scale, const float *zero, int bits, int iters,
-                      uint8_t *codes, double *obj_rows)
+                      uint8_t *codes, double *obj_rows, int relax_period)
 {
     const int maxq = (1 << bits) - 1;
     const qo_sig Sg = {S, NULL, p};
@@ -387,6 +410,7 @@ int qo_quantease_alg3(const double *W, int64_t q, int64_t p, const double *S,
             for (int64_t j = 0; j < p; ++j)
                 Wh[j] = Wi[j];
             for (int t = 0; t < iters; ++t) {
+                const int relax = qo_relaxed(relax_period, t + 1, iters);
                 for (int64_t j = 0; j < p; ++j)
                     dW[j] = Wh[j];
                 /* Ph = What Sn with Sn_jj = 0 */
@@ -399,15 +423,17 @@ int qo_quantease_alg3(const double *W, int64_t q, int64_t p, const double *S,
                 }
                 for (int64_t j = 0; j < p; ++j) {
                     int c;
-                    if (S[j * p + j] > 0.0) {
-                        double b = P[j] - Ph[j];
+                    double b = 0.0;
+                    const int live = S[j * p + j] > 0.0;
+                    if (live) {
+                        b = P[j] - Ph[j];
                         for (int64_t k = 0; k < j; ++k)   /* k = j adds Sn_jj = 0 */
                             b += dW[k] * Sn[k * p + j];
                         c = qo_code(b, s, z, maxq);
                     } else {
                         c = qo_code(Wi[j], s, z, maxq);
                     }
-                    Wh[j] = qo_level(c, s, z);
+                    Wh[j] = (relax && live) ? b : qo_level(c, s, z);
                     dW[j] -= Wh[j];
                     codes[i * p + j] = (uint8_t)c;
                 }
@@ -610,7 +636,7 @@ int qo_quantease_outlier(const double *W, int64_t q, int64_t p, const double *S,
             qo_row_times_sigma(tgt, &Sg, p, TS, NULL);
             qo_row_times_sigma(Wh + i * p, &Sg, p, WS, NULL);
             qo_sweep_row(&Sg, p, scale[i], zero[i], maxq, tgt, TS, Wh + i * p, WS,
-                         NULL, codes + i * p, NULL, NULL);
+                         NULL, codes + i * p, NULL, NULL, 0);
             free(tgt); free(TS); free(WS);
         }
         qo_objective_rows(W, H, codes, scale, zero, q, p, S, rows);

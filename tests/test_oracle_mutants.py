@@ -35,6 +35,8 @@ MUTANTS = [
      "T[i * p + j] = H[i * p + j] + eta * 2.0 * G[j];"),
     ("power_wrong_rayleigh", "lam += v[a] * w[a];", "lam += w[a] * w[a];"),
     ("column_norm_not_squared", "norm2[j] += T[i * p + j] * T[i * p + j];", "norm2[j] += T[i * p + j];"),
+    ("relax_keeps_level", "                Wh[j] = b;\n", "                Wh[j] = qo_level(c, s, z);\n"),
+    ("relax_last_sweep_too", "t1 % relax_period == 0 && t1 < iters;", "t1 % relax_period == 0 && t1 <= iters;"),
 ]
 
 PINS = [
@@ -43,7 +45,7 @@ PINS = [
     lambda: pins.test_every_update_is_bruteforce_argmin(3),
     lambda: pins.test_exhaustive_tiny_layer_cw_minimum(3),
     lambda: pins.test_objective_non_increasing(1, True),
-    lambda: pins.test_algorithm1_equals_algorithm3(4),
+    lambda: pins.test_algorithm1_equals_algorithm3(4, 0),
     pins.test_diagonal_sigma_gives_round_to_nearest,
     pins.test_objective_matches_direct_residual,
     pins.test_sigma_properties,
@@ -52,6 +54,9 @@ PINS = [
     pins.test_outlier_iht_descent_and_budget,
     pins.test_column_selection_is_the_projection,
     pins.test_structured_outlier_descent_budget_and_columns,
+    lambda: pins.test_relaxed_sweep_is_one_gauss_seidel_step(3),
+    pins.test_relaxed_sweeps_converge_to_w,
+    pins.test_relax_period_not_below_iters_is_plain_algorithm1,
     golden.test_hand_worked_two_feature_layer,
 ]
 

@@ -168,16 +168,100 @@ def test_objective_non_increasing(seed, corr):
 # --------------------------------------------------------------------------
 # Algorithm 1 == Algorithm 3 (Sec. 3.2: an exact reassociation)
 # --------------------------------------------------------------------------
-@pytest.mark.parametrize("bits", [3, 4])
-def test_algorithm1_equals_algorithm3(bits):
+@pytest.mark.parametrize("bits,relax", [(3, 0), (4, 0), (3, 2), (4, 3)])
+def test_algorithm1_equals_algorithm3(bits, relax):
     rng = np.random.default_rng(400 + bits)
     W, X = _rand_layer(rng, 24, 40, 160, heavy=(1,), heavy_mult=30.0, zero_rows=(7,), corr=True)
     S = O.sigma(X)
     s, z = O.grid(W, bits)
-    a1 = O.alg1(W, S, s, z, bits, iters=5)
-    a3 = O.alg3(W, S, s, z, bits, iters=5)
+    a1 = O.alg1(W, S, s, z, bits, iters=5, relax_period=relax)
+    a3 = O.alg3(W, S, s, z, bits, iters=5, relax_period=relax)
     assert np.array_equal(a1["codes"], a3["codes"])
     assert np.allclose(a1["obj_rows"], a3["obj_rows"], rtol=1e-10, atol=0)
+
+
+# --------------------------------------------------------------------------
+# relax heuristic (Sec. 3.2): a relaxed sweep takes beta~ itself, i.e. exact
+# coordinate minimization of the convex quadratic f over all reals.  One such
+# sweep over j = 1..p is one Gauss-Seidel step for the normal equations
+# What Sigma = W Sigma (Lemma 1), so it is pinned by the textbook splitting
+# Sigma = L + D + U:  (D + L) x_new = Sigma w - U x_old  (rows of W are
+# independent, Sec. 3.2).
+# --------------------------------------------------------------------------
+def _gauss_seidel_step(S, w, x_old):
+    from scipy.linalg import solve_triangular
+    return solve_triangular(np.tril(S), S @ w - np.triu(S, 1) @ x_old, lower=True)
+
+
+@pytest.mark.parametrize("bits", [2, 3])
+def test_relaxed_sweep_is_one_gauss_seidel_step(bits):
+    rng = np.random.default_rng(700 + bits)
+    W, X = _rand_layer(rng, 8, 28, 120, heavy=(2, 9), heavy_mult=12.0, corr=True)
+    S = O.sigma(X)
+    s, z = O.grid(W, bits)
+    r = O.alg1(W, S, s, z, bits, iters=3, record=True, want_beta=True, relax_period=2)
+    x_old = levels(r["sweep_codes"][0], s, z)          # state after sweep 1 (quantized)
+    for i in range(W.shape[0]):
+        x_new = _gauss_seidel_step(S, W[i], x_old[i])
+        assert np.allclose(r["beta"][1][i], x_new, rtol=1e-9, atol=1e-12)
+        f_new = float((W[i] - x_new) @ S @ (W[i] - x_new))
+        assert np.isclose(r["obj_rows"][1][i], f_new, rtol=1e-9, atol=1e-18)
+    # exact minimization along every coordinate: the relaxed sweep never increases f
+    assert np.all(r["obj_rows"][1] <= r["obj_rows"][0] * (1 + 1e-12))
+    # its code record is the nearest level of the relaxed values; sweep 3 quantizes again
+    s32, z32 = s.astype(np.float64), z.astype(np.float64)
+    near = np.clip(np.rint(r["beta"][1] / s32[:, None] + z32[:, None]), 0, 2 ** bits - 1)
+    assert np.array_equal(r["sweep_codes"][1], near.astype(np.uint8))
+
+
+def test_relaxed_sweep_with_diagonal_sigma_reaches_w():
+    """Orthogonal input channels: beta~ = W_ij whatever the state (up to the rounding
+    of (W_ij Sigma_jj) / Sigma_jj), so a relaxed sweep gives f = 0 and the following
+    quantized sweep is round-to-nearest."""
+    rng = np.random.default_rng(8)
+    q, p, n = 6, 20, 48
+    Qm, _ = np.linalg.qr(rng.normal(size=(n, p)))
+    X = Qm.T * rng.uniform(0.5, 3.0, size=(p, 1))
+    W = rng.normal(0, 0.02, size=(q, p))
+    S = np.diag(np.diag(X @ X.T))
+    s, z = O.grid(W, 3)
+    rtn = O.rtn(W, s, z, 3)
+    r = O.alg1(W, S, s, z, 3, iters=3, record=True, init_codes=np.zeros((q, p), np.uint8),
+               relax_period=1)
+    scale = (W * W) @ np.diag(S)                      # f of What = 0, per row
+    assert np.all(r["obj_rows"][:2] <= 1e-24 * scale)
+    assert np.array_equal(r["codes"], rtn)
+
+
+def test_relaxed_sweeps_converge_to_w():
+    """Gauss-Seidel on a positive definite Sigma converges: from round-to-nearest
+    codes, relaxed sweeps (period 1: all but the last) drive What to W and f to 0
+    (down to rounding), never increasing f on the way."""
+    rng = np.random.default_rng(9)
+    W, X = _rand_layer(rng, 5, 16, 400, heavy=(3,), heavy_mult=4.0)
+    S = O.sigma(X)
+    s, z = O.grid(W, 3)
+    rtn = O.rtn(W, s, z, 3)
+    f0 = O.alg1(W, S, s, z, 3, iters=1, init_codes=rtn, forced=rtn[None])["obj"][0]
+    r = O.alg1(W, S, s, z, 3, iters=40, init_codes=rtn, want_beta=True, relax_period=1)
+    obj = r["obj"][:-1]
+    big = obj > 1e-20 * f0
+    assert np.all(np.diff(obj)[big[:-1]] <= 1e-12 * obj[:-1][big[:-1]])
+    assert obj[-1] <= 1e-20 * f0
+    assert np.allclose(r["beta"][-2], W, rtol=0, atol=1e-12 * np.abs(W).max())
+
+
+def test_relax_period_not_below_iters_is_plain_algorithm1():
+    rng = np.random.default_rng(10)
+    W, X = _rand_layer(rng, 6, 24, 100, corr=True)
+    S = O.sigma(X)
+    s, z = O.grid(W, 4)
+    a = O.alg1(W, S, s, z, 4, iters=4, record=True)
+    b = O.alg1(W, S, s, z, 4, iters=4, record=True, relax_period=4)
+    assert np.array_equal(a["sweep_codes"], b["sweep_codes"])
+    assert np.array_equal(a["obj_rows"], b["obj_rows"])
+    c = O.alg1(W, S, s, z, 4, iters=4, record=True, relax_period=3)
+    assert not np.array_equal(a["obj_rows"][2], c["obj_rows"][2])
 
 
 # --------------------------------------------------------------------------
