@@ -70,7 +70,13 @@ typedef struct qe_timer qe_timer;
 typedef struct {
     /* Column block width B of the blocked CD sweep: 0 = default (256); 64, 128 or 256. */
     int block_width;
-    /* Relax heuristic of Sec. 3.2 (skip quantization every R-th sweep): must be 0. */
+    /* Relax heuristic of Sec. 3.2: with R > 0, sweep t (counted from 1) with
+     * t mod R = 0 and t < iters keeps every live coordinate at beta~ of Lemma 1
+     * unquantized (a column with Sigma_jj <= 0 stays on its level); the last
+     * sweep always quantizes.  obj[t] of a relaxed sweep is f of the relaxed
+     * weights, and its sweep_codes record their nearest levels.  0 = off;
+     * negative is QE_ERR_INVALID_ARG; the outlier variant returns
+     * QE_ERR_UNSUPPORTED for R != 0. */
     int relax_period;
     /* Structured outliers (Sec. 4.3): 1 = H keeps whole columns, the floor(s/q)
      * of largest l2 norm, in place of the s largest entries (outlier variant

@@ -347,11 +347,10 @@ struct ObjFuse {
     int wbf16;
     int64_t ldw;
     const uint8_t *codes;
-    const float *zeros;
     const float *H;
 };
 
-static qe_status residual(Ctx &c, const float *scales, const ObjFuse *f = nullptr) {
+static qe_status residual(Ctx &c, const float *scales, const float *zeros, const ObjFuse *f = nullptr) {
     const int64_t q = c.pl.q, p = c.pl.p, ld = c.pl.ld;
     GemmArgs g = gemm_args(c, static_cast<int>(q), static_cast<int>(p), static_cast<int>(ceil_div(p, 64)),
                            EPI_RFULL);
@@ -364,6 +363,7 @@ static qe_status residual(Ctx &c, const float *scales, const ObjFuse *f = nullpt
     g.P = c.P;
     g.ldp = ld;
     g.scale = scales;
+    g.zero = zeros;   // R is kept in grid-step units: the epilogue adds z
     if (f) {
         g.obj_part = c.objp;
         g.W = f->W;
@@ -371,7 +371,6 @@ static qe_status residual(Ctx &c, const float *scales, const ObjFuse *f = nullpt
         g.ldw = f->ldw;
         g.codes = f->codes;
         g.ldc = p;
-        g.zero = f->zeros;
         g.dvec = c.d;
         g.Hd = f->H;
         g.ldh = ld;
@@ -396,10 +395,21 @@ static qe_status residual(Ctx &c, const float *scales, const ObjFuse *f = nullpt
 //       means the first window sweep after a residual refresh: only columns < b0.
 //       Every window visit also records its changes in the block's change list,
 //       from which the later sweeps (k_cd_rows_lists) take the correction.
+// src: where What at the sweep start comes from: W itself (the first sweep, R
+// then holds it), the codes, or the real values a relaxed sweep left (kept in
+// the change-list entry buffer, unused while such sweeps run).  relax: the
+// relax heuristic of Sec. 3.2 (the sweep keeps beta~ unquantized).  When the
+// changes are real-valued (src != SRC_CODES or relax) they take three bf16
+// planes and the in-block sequential kernel.
+enum { SRC_W = 0, SRC_CODES = 1, SRC_V = 2 };
+
+static float *relaxed_values(const Ctx &c) { return reinterpret_cast<float *>(c.lent); }
+
 static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float *zeros, int bits,
-                       bool first, int window) {
+                       int src, bool relax, int window) {
     const int64_t q = c.pl.q, p = c.pl.p, ld = c.pl.ld;
     const int B = c.pl.B;
+    const bool frac = src != SRC_CODES || relax;
     for (int64_t b0 = 0; b0 < p; b0 += B) {
         const int bw = static_cast<int>((p - b0) < B ? (p - b0) : B);
         const int64_t kcols = (window > 0) ? p : b0;
@@ -408,7 +418,7 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
             const int kb = static_cast<int>(ceil_div(kcols, 64));
             const int S = kb < c.pl.smax ? kb : c.pl.smax;
             GemmArgs g = gemm_args(c, static_cast<int>(q), bw, kb, EPI_TRAIL);
-            set_prods(g, first ? 3 : 1);
+            set_prods(g, frac ? 3 : 1);
             g.a_plane_rows = static_cast<int>(q);
             g.b_plane_rows = static_cast<int>(p);
             g.b_row0 = static_cast<int>(b0);
@@ -439,7 +449,11 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
         a.d = c.d;
         a.rowdf = window != 0 ? c.rowdf : nullptr;
         a.maxq = static_cast<float>((1 << bits) - 1);
-        a.first_sweep = first ? 1 : 0;
+        a.first_sweep = src == SRC_W ? 1 : 0;
+        a.frac = frac ? 1 : 0;
+        a.vstart = src == SRC_V ? relaxed_values(c) : nullptr;
+        a.vout = relax ? relaxed_values(c) : nullptr;
+        a.ldv = ld;
         a.write_qf = window != 0 ? 0 : 1;
         a.codes = codes;
         a.ldc = p;
@@ -448,7 +462,7 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
         a.dp = c.dp;
         a.nblk = static_cast<int>(c.pl.nblk);
         a.lcnt = c.lcnt;
-        if (window != 0) a.lent = c.lent;
+        if (window != 0 && !frac) a.lent = c.lent;
         a.ldd = ld;
         a.dp_plane_rows = q;
         a.err = c.err;
@@ -515,14 +529,18 @@ static int dense_sweeps(const qe_opts *o) {
     return (o && o->dense_sweeps) ? o->dense_sweeps : kDefaultDenseSweeps;
 }
 
+static int relax_period(const qe_opts *o) { return o ? o->relax_period : 0; }
+
 static int free_changes(const qe_opts *o) {
     return (o && o->free_changes) ? o->free_changes : kFreeMaxChanges;
 }
 
-// structured: the call accepts structured_outliers = 1 (the outlier variant)
+// structured: the call accepts structured_outliers = 1 (the outlier variant,
+// which has no relax heuristic)
 static qe_status check_opts(const qe_opts *o, bool structured = false) {
     if (!o) return QE_OK;
-    if (o->relax_period != 0) return QE_ERR_UNSUPPORTED;
+    if (o->relax_period < 0) return QE_ERR_INVALID_ARG;
+    if (o->relax_period != 0 && structured) return QE_ERR_UNSUPPORTED;
     if (o->structured_outliers != 0 && !(structured && o->structured_outliers == 1)) return QE_ERR_UNSUPPORTED;
     if (o->block_width != 0 && o->block_width != 64 && o->block_width != 128 && o->block_width != 256)
         return QE_ERR_UNSUPPORTED;
@@ -736,50 +754,103 @@ qe_status qe_quantize_layer(const void *W, qe_dtype w_dtype, int64_t q, int64_t 
     // Sweep 1 starts at What = W (Sec. 3.1) and changes every coordinate by a
     // real amount: the classic schedule with a residual refresh (which also
     // yields obj[0]).  Later sweeps change few codes, by integers: the rolling
-    // window schedule with the objective updated decision by decision.
+    // window schedule with the objective updated decision by decision.  A
+    // relaxed sweep (relax heuristic, Sec. 3.2) and the sweep after it move
+    // every coordinate by a real amount again: they run as sequential in-block
+    // sweeps between two residual refreshes.
     const bool warm = opts && opts->init_codes;
+    const int rp = relax_period(opts);
+    auto relaxed = [&](int t) { return rp > 0 && (t + 1) % rp == 0 && t + 1 < iters; };
     const size_t plane0 = static_cast<size_t>(q) * pl.ld * 2;
-    int t0 = 0;
-    if (warm) {
-        QE_CK(cudaMemcpyAsync(codes, opts->init_codes, static_cast<size_t>(q) * p, cudaMemcpyDeviceToDevice, c.s));
+    // after a residual refresh R holds every change so far: empty window, no list entries
+    auto restart = [&](int planes) -> qe_status {
+        QE_CK(cudaMemsetAsync(c.dp, 0, plane0 * planes, c.s));
+        QE_CK(cudaMemsetAsync(c.lcnt, 0, static_cast<size_t>(q) * pl.nblk * 4, c.s));
+        QE_CK(cudaMemsetAsync(c.rowdf, 0, static_cast<size_t>(q) * 8, c.s));
+        return QE_OK;
+    };
+    auto refresh = [&]() -> qe_status {
         QE_CK(launch_codes_to_qf(codes, p, zeros, q, p, c.qf, pl.ld, c.s));
-        const ObjFuse f{c.objbase, W, wbf16, ldw, codes, zeros, nullptr};
-        if ((st = residual(c, scales, &f)) != QE_OK) return st;
-    } else {
-        QE_CK(launch_init_residual(W, wbf16, ldw, nullptr, 0, q, p, scales, zeros, c.R, pl.ld, c.s));
-        if ((st = sweep(c, codes, scales, zeros, bits, true, 0)) != QE_OK) return st;
-        const ObjFuse f{obj, W, wbf16, ldw, codes, zeros, nullptr};
-        if ((st = residual(c, scales, &f)) != QE_OK) return st;
-        if (opts && opts->sweep_codes)
-            QE_CK(cudaMemcpyAsync(opts->sweep_codes, codes, static_cast<size_t>(q) * p, cudaMemcpyDeviceToDevice, c.s));
-        t0 = 1;
-    }
-    // the refreshed residual already holds every change so far: start the window empty
-    QE_CK(cudaMemsetAsync(c.dp, 0, plane0, c.s));
-    QE_CK(cudaMemsetAsync(c.lcnt, 0, static_cast<size_t>(q) * pl.nblk * 4, c.s));
-    QE_CK(cudaMemsetAsync(c.rowdf, 0, static_cast<size_t>(q) * 8, c.s));
-    // sweeps 1 .. dense use the tensor-core correction, one launch pair per block
-    const int dense = dense_sweeps(opts);
-    int t = t0;
-    for (; t < iters && t < dense; ++t) {
-        if ((st = sweep(c, codes, scales, zeros, bits, false, t == t0 ? -1 : 1)) != QE_OK) return st;
-        QE_CK(launch_obj_step(c.rowdf, q, t == 0 ? c.objbase : obj + t - 1, obj + t, c.s));
+        return residual(c, scales, zeros);
+    };
+    auto record = [&](int t) -> qe_status {
         if (opts && opts->sweep_codes)
             QE_CK(cudaMemcpyAsync(opts->sweep_codes + static_cast<size_t>(t) * q * p, codes,
                                   static_cast<size_t>(q) * p, cudaMemcpyDeviceToDevice, c.s));
-    }
-    // later sweeps: the change lists, persistent over blocks and sweeps
-    while (t < iters) {
-        const int te = (iters - t) < kSweepChunk ? iters : t + kSweepChunk;
-        CdArgs a = list_args(c, codes, scales, zeros, bits);
-        {
-            Timed tm(c.timer, QE_KERNEL_CD_LISTS, c.s);
-            // the lists are empty at the window start (t0): that sweep steps in lockstep
-            QE_CK(launch_cd_rows_lists(pl.B, a, t, te, c.rowdft, opts ? opts->sweep_codes : nullptr, t == t0,
-                                       free_changes(opts), c.nsm, c.s));
+        return QE_OK;
+    };
+    int t = 0, src = SRC_CODES;
+    if (warm) {
+        QE_CK(cudaMemcpyAsync(codes, opts->init_codes, static_cast<size_t>(q) * p, cudaMemcpyDeviceToDevice, c.s));
+        QE_CK(launch_codes_to_qf(codes, p, zeros, q, p, c.qf, pl.ld, c.s));
+        const ObjFuse f{c.objbase, W, wbf16, ldw, codes, nullptr};
+        if ((st = residual(c, scales, zeros, &f)) != QE_OK) return st;
+    } else {
+        QE_CK(launch_init_residual(W, wbf16, ldw, nullptr, 0, q, p, scales, zeros, c.R, pl.ld, c.s));
+        QE_CK(cudaMemsetAsync(c.objbase, 0, 8, c.s));   // f(W) = 0
+        src = SRC_W;
+        if (!relaxed(0)) {
+            if ((st = sweep(c, codes, scales, zeros, bits, SRC_W, false, 0)) != QE_OK) return st;
+            const ObjFuse f{obj, W, wbf16, ldw, codes, nullptr};
+            if ((st = residual(c, scales, zeros, &f)) != QE_OK) return st;
+            if ((st = record(0)) != QE_OK) return st;
+            t = 1;
+            src = SRC_CODES;
         }
-        QE_CK(launch_obj_prefix(c.rowdft, q, te - t, t == 0 ? c.objbase : obj + t - 1, obj + t, c.s));
-        t = te;
+    }
+    if ((st = restart(src == SRC_CODES ? 1 : 3)) != QE_OK) return st;
+    bool exact = true;   // R is the residual of the current What and no list has entries
+    bool chain = false;  // the last sweep was a sequential one (its three-plane changes are in dp)
+    const int dense = dense_sweeps(opts);
+    while (t < iters) {
+        const bool rx = relaxed(t);
+        if (rx || src != SRC_CODES) {
+            if (!exact && !chain) {   // from the change lists: refresh R from the codes
+                if ((st = refresh()) != QE_OK) return st;
+                if ((st = restart(3)) != QE_OK) return st;
+                exact = true;
+            }
+            if ((st = sweep(c, codes, scales, zeros, bits, src, rx, exact ? -1 : 1)) != QE_OK) return st;
+            QE_CK(launch_obj_step(c.rowdf, q, t == 0 ? c.objbase : obj + t - 1, obj + t, c.s));
+            if ((st = record(t)) != QE_OK) return st;
+            ++t;
+            src = rx ? SRC_V : SRC_CODES;
+            exact = false;
+            chain = true;
+            if (src == SRC_CODES && t < iters) {   // back on the grid
+                if ((st = refresh()) != QE_OK) return st;
+                if ((st = restart(1)) != QE_OK) return st;
+                exact = true;
+                chain = false;
+            }
+            continue;
+        }
+        // quantized sweeps up to the next relaxed one: sweeps 1 .. dense use the
+        // tensor-core correction (one launch pair per block), later ones the change
+        // lists, persistent over blocks and sweeps
+        int tend = t;
+        while (tend < iters && !relaxed(tend)) ++tend;
+        for (; t < tend && t < dense; ++t) {
+            if ((st = sweep(c, codes, scales, zeros, bits, SRC_CODES, false, exact ? -1 : 1)) != QE_OK) return st;
+            QE_CK(launch_obj_step(c.rowdf, q, t == 0 ? c.objbase : obj + t - 1, obj + t, c.s));
+            if ((st = record(t)) != QE_OK) return st;
+            exact = false;
+            chain = false;
+        }
+        while (t < tend) {
+            const int te = (tend - t) < kSweepChunk ? tend : t + kSweepChunk;
+            CdArgs a = list_args(c, codes, scales, zeros, bits);
+            {
+                Timed tm(c.timer, QE_KERNEL_CD_LISTS, c.s);
+                // with empty lists (after a refresh) the first sweep steps in lockstep
+                QE_CK(launch_cd_rows_lists(pl.B, a, t, te, c.rowdft, opts ? opts->sweep_codes : nullptr,
+                                           exact ? 1 : 0, free_changes(opts), c.nsm, c.s));
+            }
+            QE_CK(launch_obj_prefix(c.rowdft, q, te - t, t == 0 ? c.objbase : obj + t - 1, obj + t, c.s));
+            t = te;
+            exact = false;
+            chain = false;
+        }
     }
     return QE_OK;
 }
@@ -830,13 +901,13 @@ qe_status qe_quantize_layer_outlier(const void *W, qe_dtype w_dtype, int64_t q, 
     if (warm) {
         QE_CK(cudaMemcpyAsync(codes, opts->init_codes, static_cast<size_t>(q) * p, cudaMemcpyDeviceToDevice, c.s));
         QE_CK(launch_codes_to_qf(codes, p, zeros, q, p, c.qf, ld, c.s));
-        if ((st = residual(c, scales)) != QE_OK) return st;
+        if ((st = residual(c, scales, zeros)) != QE_OK) return st;
     } else {
         QE_CK(launch_init_residual(W, wbf16, ldw, c.H, ld, q, p, scales, zeros, c.R, ld, c.s));
     }
     for (int t = 0; t < iters; ++t) {
         if (t == 0 && !warm) {
-            if ((st = sweep(c, codes, scales, zeros, bits, true, 0)) != QE_OK) return st;
+            if ((st = sweep(c, codes, scales, zeros, bits, SRC_W, false, 0)) != QE_OK) return st;
         } else {
             // R is fresh and the target W - H stays fixed during the sweep: one
             // change-list sweep whose window starts empty (each block corrected by
@@ -848,8 +919,8 @@ qe_status qe_quantize_layer_outlier(const void *W, qe_dtype w_dtype, int64_t q, 
             Timed tm(c.timer, QE_KERNEL_CD_LISTS, c.s);
             QE_CK(launch_cd_rows_lists(pl.B, a, t, t + 1, c.rowdft, nullptr, 1, kFreeMaxChanges, c.nsm, c.s));
         }
-        const ObjFuse f{obj_cd ? obj_cd + t : nullptr, W, wbf16, ldw, codes, zeros, c.H};
-        if ((st = residual(c, scales, obj_cd ? &f : nullptr)) != QE_OK) return st;
+        const ObjFuse f{obj_cd ? obj_cd + t : nullptr, W, wbf16, ldw, codes, c.H};
+        if ((st = residual(c, scales, zeros, obj_cd ? &f : nullptr)) != QE_OK) return st;
         // IHT step: T = H + 2 eta d (R - What); H = P_s(T)
         QE_CK(launch_iht_target(c.H, c.R, ld, codes, p, scales, zeros, c.d, c.eta, q, p, c.T, c.s));
         QE_CK(select(c.T));

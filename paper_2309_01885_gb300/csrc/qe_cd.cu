@@ -408,7 +408,7 @@ __device__ __forceinline__ bool cd_prologue(const CdArgs &a, float *tri, uint64_
         const int l = 32 * h + lane;
         const bool ok = row_ok && (FULL || l < bw);
         r_[h] = ok ? a.R[ii * a.ldr + b0 + l] : 0.0f;
-        cd_[h] = (ok && !a.first_sweep) ? a.codes[ii * a.ldc + b0 + l] : 0u;
+        cd_[h] = (ok && !a.first_sweep && !a.vstart) ? a.codes[ii * a.ldc + b0 + l] : 0u;
         ps[h] = 0.0f;
     }
 #pragma unroll
@@ -422,7 +422,10 @@ __device__ __forceinline__ bool cd_prologue(const CdArgs &a, float *tri, uint64_
     const bool changed = a.nsplit > 0;
 #pragma unroll
     for (int h = 0; h < CPL; ++h) {
-        st[h] = a.first_sweep ? r_[h] : static_cast<float>(cd_[h]);
+        st[h] = a.first_sweep ? r_[h]
+                : (a.vstart ? ((row_ok && (FULL || 32 * h + lane < bw)) ? a.vstart[ii * a.ldv + b0 + 32 * h + lane]
+                                                                         : 0.0f)
+                            : static_cast<float>(cd_[h]));
         t[h] = r_[h] + ps[h];
     }
     if (a.store_base && changed) {
@@ -453,14 +456,17 @@ __device__ __forceinline__ void cd_epilogue(const CdArgs &a, int64_t b0, int bw_
         const int l = 32 * h + lane;
         if (!FULL && l >= bw) continue;
         const int64_t col = b0 + l;
-        if (!skip_same || dlt[h] != 0.0f) {
+        if (a.vout) {   // relaxed: the value itself, and its nearest level as the code
+            a.vout[i * a.ldv + col] = code[h];
+            a.codes[i * a.ldc + col] = static_cast<uint8_t>(rintf(fminf(fmaxf(code[h], 0.0f), a.maxq)));
+        } else if (!skip_same || dlt[h] != 0.0f) {
             a.codes[i * a.ldc + col] = static_cast<uint8_t>(code[h]);
             if (a.write_qf) a.qf[i * a.ldq + col] = __float2bfloat16_rn(code[h] - z);
         }
         if (!a.dp) continue;
         const __nv_bfloat16 hi = __float2bfloat16_rn(dlt[h]);
         a.dp[i * a.ldd + col] = hi;
-        if (a.first_sweep) {   // Delta' is not an integer in the first sweep: three planes
+        if (a.frac) {   // Delta' is not an integer: three planes
             const float r1 = dlt[h] - __bfloat162float(hi);
             const __nv_bfloat16 mid = __float2bfloat16_rn(r1);
             a.dp[(a.dp_plane_rows + i) * a.ldd + col] = mid;
@@ -488,13 +494,24 @@ __device__ __forceinline__ void cd_epilogue(const CdArgs &a, int64_t b0, int bw_
     }
 }
 
-// Sequential in-block kernel (the first sweep, where every column changes).
+__device__ __forceinline__ double warp_sum(double x) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+    return x;
+}
+
+// Sequential in-block kernel (sweeps where every column moves by a real
+// amount: the first sweep, a relaxed sweep and the sweep after one).
 // One warp per row; column j = 32 h + jj is decided by lane jj, which keeps
 // its code and change Delta'; the change (db, the same in every lane after the
 // shuffle) times Sigma_bar[j][l] is added to every later column l.  Lanes whose
 // column is already decided (l <= j) absorb harmless updates, so no lane test
 // is needed; an unchanged column (db == 0) skips the updates.
-template <int B, bool FULL>
+// RELAX: the relax heuristic (Sec. 3.2): a live column (Sigma_jj > 0) takes
+// beta~ itself instead of its nearest level; a dead one stays on its level.
+// DF: the objective change of each decision (Lemma 1 along one coordinate)
+// goes to rowdf, as in the change-driven kernels.
+template <int B, bool FULL, bool RELAX, bool DF>
 __global__ void __launch_bounds__(1024) k_cd_block_seq(const CdArgs a) {
     using C = CdCfg<B>;
     constexpr int CPL = C::CPL;
@@ -509,6 +526,18 @@ __global__ void __launch_bounds__(1024) k_cd_block_seq(const CdArgs a) {
     if (!row_ok) return;
     const int bw = FULL ? B : a.bw;
     const float maxq = a.maxq;
+    uint32_t live = 0u;   // bit h: this lane's column 32 h + lane has Sigma_jj > 0
+    if (RELAX) {
+#pragma unroll
+        for (int h = 0; h < CPL; ++h)
+            if ((FULL || 32 * h + lane < bw) && a.d[a.b0 + 32 * h + lane] > 0.0f) live |= 1u << h;
+    }
+    float s2 = 0.0f;
+    double dfacc = 0.0;
+    if (DF) {
+        const float sc = a.scale[i];
+        s2 = sc * sc;
+    }
     float code[CPL], dlt[CPL];
 #pragma unroll
     for (int h = 0; h < CPL; ++h) {
@@ -521,11 +550,19 @@ __global__ void __launch_bounds__(1024) k_cd_block_seq(const CdArgs a) {
         for (int jj = 0; jj < 32; ++jj) {
             const int j = 32 * h + jj;
             if (!FULL && j >= bw) break;
-            const float c = rintf(fminf(fmaxf(t[h], 0.0f), maxq));
+            const float cq = rintf(fminf(fmaxf(t[h], 0.0f), maxq));
+            const float c = (RELAX && ((live >> h) & 1u)) ? t[h] : cq;
             const float dl = st[h] - c;
             if (lane == jj) {
                 code[h] = c;
                 dlt[h] = dl;
+                if (DF) {
+                    const float dj = a.d[a.b0 + j];
+                    if (dj > 0.0f) {
+                        const float e1 = c - t[h], e0 = st[h] - t[h];
+                        dfacc += static_cast<double>(dj * s2 * (e1 * e1 - e0 * e0));
+                    }
+                }
             }
             const float db = __shfl_sync(0xffffffffu, dl, jj);
             if (db != 0.0f) {
@@ -534,6 +571,10 @@ __global__ void __launch_bounds__(1024) k_cd_block_seq(const CdArgs a) {
                 for (int g = h; g < CPL; ++g) t[g] = fmaf(db, row[32 * g + lane], t[g]);
             }
         }
+    }
+    if (DF) {
+        dfacc = warp_sum(dfacc);
+        if (lane == 0) a.rowdf[i] += dfacc;
     }
     cd_epilogue<B, FULL, false>(a, a.b0, a.bw, i, lane, code, dlt, false);
 }
@@ -617,12 +658,6 @@ __device__ __forceinline__ int chg_decide(const float *tri, const float *d_blk, 
         ++nchg;
     }
     return nchg;
-}
-
-__device__ __forceinline__ double warp_sum(double x) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
-    return x;
 }
 
 // Change-driven in-block kernel (every sweep after the first), exactly
@@ -1015,11 +1050,11 @@ __global__ void k_obj_prefix(const double *rowdf_t, int64_t q, int nt, const dou
     }
 }
 
-template <int B, bool FULL, bool SEQ>
+template <int B, bool FULL, bool SEQ, bool RELAX = false, bool DF = false>
 static cudaError_t launch_cd_block_b(const CdArgs &a, int nsm, cudaStream_t s) {
     using C = CdCfg<B>;
     if (a.nsplit > C::MAX_SPLITS) return cudaErrorInvalidValue;
-    auto kern = SEQ ? k_cd_block_seq<B, FULL> : k_cd_block_chg<B, FULL>;
+    auto kern = SEQ ? k_cd_block_seq<B, FULL, RELAX, DF> : k_cd_block_chg<B, FULL>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
     if (e != cudaSuccess) return e;
     // one CTA per SM when the rows allow it (the packed block is shared by the CTA's rows)
@@ -1031,11 +1066,17 @@ static cudaError_t launch_cd_block_b(const CdArgs &a, int nsm, cudaStream_t s) {
     return cudaGetLastError();
 }
 
+template <int B, bool FULL>
+static cudaError_t launch_cd_block_f(const CdArgs &a, int nsm, cudaStream_t s) {
+    if (!a.frac) return launch_cd_block_b<B, FULL, false>(a, nsm, s);
+    if (a.vout) return a.rowdf ? launch_cd_block_b<B, FULL, true, true, true>(a, nsm, s) : cudaErrorInvalidValue;
+    return a.rowdf ? launch_cd_block_b<B, FULL, true, false, true>(a, nsm, s)
+                   : launch_cd_block_b<B, FULL, true, false, false>(a, nsm, s);
+}
+
 template <int B>
 static cudaError_t launch_cd_block_w(const CdArgs &a, int nsm, cudaStream_t s) {
-    const bool full = a.bw == B, seq = a.first_sweep != 0;
-    if (full) return seq ? launch_cd_block_b<B, true, true>(a, nsm, s) : launch_cd_block_b<B, true, false>(a, nsm, s);
-    return seq ? launch_cd_block_b<B, false, true>(a, nsm, s) : launch_cd_block_b<B, false, false>(a, nsm, s);
+    return a.bw == B ? launch_cd_block_f<B, true>(a, nsm, s) : launch_cd_block_f<B, false>(a, nsm, s);
 }
 
 cudaError_t launch_cd_block(int B, const CdArgs &a, int nsm, cudaStream_t s) {

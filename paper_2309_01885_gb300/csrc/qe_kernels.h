@@ -31,6 +31,13 @@ struct CdArgs {
     double *rowdf;                  // per-row objective change accumulator, or NULL
     float maxq;
     int first_sweep;                // What_start is R itself (not on the grid)
+    int frac;                       // Delta' real-valued (every coordinate moves): three planes, in-block
+                                    // sequential kernel
+    const float *vstart;            // non-NULL: What_start in grid units, leading dimension ldv (the
+                                    // values a relaxed sweep left)
+    float *vout;                    // non-NULL: relaxed sweep (relax heuristic, Sec. 3.2): a live column
+                                    // takes beta~ itself, written here; codes get its nearest level
+    int64_t ldv;
     int write_qf;                   // also write C - z (needed by the residual GEMM)
     uint8_t *codes;                 // in: codes at sweep start (unless first_sweep); out: new codes
     int64_t ldc;

@@ -215,8 +215,9 @@ class Timer:
 
 
 def _opts(block_width=0, power_iters=0, init_codes=None, sweep_codes=None, wx_norm2=None,
-          workspace=None, timer=None, dense_sweeps=0, free_changes=0) -> QEOpts:
+          workspace=None, timer=None, dense_sweeps=0, free_changes=0, relax_period=0) -> QEOpts:
     o = QEOpts()
+    o.relax_period = relax_period
     o.timer = None if timer is None else timer.handle.value
     o.block_width = block_width
     o.power_iters = power_iters
@@ -235,11 +236,14 @@ def qe_quantize_layer(W: torch.Tensor, Sigma: torch.Tensor, bits: int, iters: in
                       init_codes: torch.Tensor | None = None, record_sweeps: bool = False,
                       want_norm: bool = False, block_width: int = 0,
                       workspace: torch.Tensor | None = None, timer: Timer | None = None,
-                      dense_sweeps: int = 0, free_changes: int = 0, stream=None) -> dict:
+                      dense_sweeps: int = 0, free_changes: int = 0, relax_period: int = 0,
+                      stream=None) -> dict:
     """QuantEase on one layer; returns codes (u8 q x p), scales, zeros, obj (fp64 per sweep),
     and optionally sweep_codes (iters x q x p) and wx_norm2.  dense_sweeps: sweeps whose
     cross-block term uses the tensor-core GEMM before the change lists take over (0 = default);
-    free_changes: changes per row below which list sweeps run row by row (0 = default, -1 = never)."""
+    free_changes: changes per row below which list sweeps run row by row (0 = default, -1 = never);
+    relax_period: the relax heuristic of Sec. 3.2 (sweep t from 1 with t mod R = 0 and t < iters
+    keeps beta~ unquantized; 0 = off)."""
     q, p = W.shape
     dev = W.device
     codes = torch.empty(q, p, dtype=torch.uint8, device=dev)
@@ -248,7 +252,8 @@ def qe_quantize_layer(W: torch.Tensor, Sigma: torch.Tensor, bits: int, iters: in
     obj = torch.empty(iters, dtype=torch.float64, device=dev)
     sweep = torch.empty(iters, q, p, dtype=torch.uint8, device=dev) if record_sweeps else None
     norm = torch.empty(1, dtype=torch.float64, device=dev) if want_norm else None
-    o = _opts(block_width, 0, init_codes, sweep, norm, workspace, timer, dense_sweeps, free_changes)
+    o = _opts(block_width, 0, init_codes, sweep, norm, workspace, timer, dense_sweeps, free_changes,
+              relax_period)
     _check(load().qe_quantize_layer(_ptr(W), _dtype(W), q, p, _rowmajor_ld(W), _ptr(Sigma), bits, iters,
                                     ctypes.byref(o), _ptr(codes), _ptr(scales), _ptr(zeros), _ptr(obj),
                                     _stream(stream)), "qe_quantize_layer")

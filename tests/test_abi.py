@@ -65,11 +65,16 @@ def test_invalid_arguments_rejected_synchronously(lib):
     # iters = 0
     assert L.qe_quantize_layer(_fake(), qe.QE_BF16, 4, 4, 4, _fake(2), 3, 0, opts, _fake(3), _fake(4),
                                _fake(5), _fake(6), None) == qe.QE_ERR_INVALID_ARG
-    # unsupported options
+    # unsupported / invalid options
     o = qe.QEOpts()
-    o.relax_period = 3
+    o.relax_period = -1
     assert L.qe_quantize_layer(_fake(), qe.QE_F32, 4, 4, 4, _fake(2), 3, 1, ctypes.byref(o), _fake(3),
-                               _fake(4), _fake(5), _fake(6), None) == qe.QE_ERR_UNSUPPORTED
+                               _fake(4), _fake(5), _fake(6), None) == qe.QE_ERR_INVALID_ARG
+    o = qe.QEOpts()
+    o.relax_period = 3            # the outlier variant has no relax heuristic
+    assert L.qe_quantize_layer_outlier(_fake(), qe.QE_F32, 4, 4, 4, _fake(2), 3, 1, 4, ctypes.byref(o),
+                                       _fake(3), _fake(4), _fake(5), _fake(7), _fake(8), _fake(9), _fake(6),
+                                       None, None) == qe.QE_ERR_UNSUPPORTED
     o = qe.QEOpts()
     o.structured_outliers = 1     # only the outlier variant takes it
     assert L.qe_quantize_layer(_fake(), qe.QE_F32, 4, 4, 4, _fake(2), 3, 1, ctypes.byref(o), _fake(3),

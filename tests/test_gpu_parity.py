@@ -4,6 +4,8 @@ Sizes here run in seconds on the oracle and span several GEMM tiles, several
 64-column CD blocks and ragged tails.  Full-size workloads are in
 test_gpu_fullsize.py.
 """
+import ctypes
+
 import numpy as np
 import pytest
 import torch
@@ -255,6 +257,47 @@ def test_layer_list_modes_identical(p):
     assert int(late.max()) <= 32
 
 
+@pytest.mark.parametrize("relax,w_dtype,zero_rows", [(3, torch.bfloat16, ()), (2, torch.float32, (5,)),
+                                                     (1, torch.bfloat16, ())])
+def test_layer_relax_heuristic(relax, w_dtype, zero_rows):
+    """The relax heuristic of Sec. 3.2 against the oracle's Algorithm 1 with the same
+    period: the objective after every sweep (relaxed ones: f of the real-valued
+    weights), the codes after every sweep (relaxed ones: their nearest levels) and
+    the final codes.  A relaxed sweep minimizes f exactly along each coordinate, so
+    it never increases f.  p = 300 ends on a ragged block; a zero row of X makes a
+    dead column, which stays on its level."""
+    q, p, n, bits, iters = 160, 300, 2048, 3, 7
+    W = inputs.layer_weights(q, p, dtype=w_dtype, seed=64 + relax, device="cuda")
+    X = inputs.calib_inputs(p, n, dtype=torch.bfloat16, seed=64 + relax, device="cuda",
+                            heavy_frac=0.01, heavy_mult=30.0, zero_rows=zero_rows)
+    Sg = qe.qe_build_sigma(X)
+    out = qe.qe_quantize_layer(W, Sg, bits, iters, record_sweeps=True, want_norm=True, relax_period=relax)
+    assert qe.qe_sync_status() == qe.QE_OK
+    W64, S64 = parity.f64(W), parity.f64(Sg)
+    wx = float(np.einsum("ij,jk,ik->", W64, S64, W64))
+    s, z = parity.check_grid(out["scales"], out["zeros"], W64, bits)
+    ref = O.alg1(W64, S64, s, z, bits, iters, record=True, relax_period=relax)
+    obj = out["obj"].cpu().numpy()
+    parity.check_obj(obj, ref["obj"], what="objective with relaxed sweeps", atol=1e-7 * wx)
+    sweep = out["sweep_codes"].cpu().numpy()
+    for t in range(iters):
+        m = parity.code_match(sweep[t], ref["sweep_codes"][t])
+        assert m >= 0.995, f"sweep {t + 1}: codes match {m:.5f}"
+    m = parity.code_match(out["codes"].cpu().numpy(), ref["codes"])
+    assert m >= parity.CODE_MATCH, f"codes match {m:.5f}"
+    for t in range(1, iters - 1):
+        if (t + 1) % relax == 0:
+            assert obj[t] <= obj[t - 1] * (1 + 1e-6) + 1e-9 * wx, f"relaxed sweep {t + 1} increased f"
+
+
+def test_layer_relax_period_not_below_iters_is_plain():
+    W, X, Sg, out = _layer_case(96, 200, 1024, torch.bfloat16, 4, 5, seed=65)
+    r = qe.qe_quantize_layer(W, Sg, 4, 5, record_sweeps=True, relax_period=5)
+    assert qe.qe_sync_status() == qe.QE_OK
+    assert torch.equal(r["sweep_codes"], out["sweep_codes"])
+    assert torch.equal(r["obj"], out["obj"])
+
+
 def test_layer_dead_columns_round_to_nearest():
     dead = (5, 77, 130)
     W, X, Sg, out = _layer_case(96, 160, 1024, torch.float32, 4, 3, seed=12, zero_rows=dead)
@@ -415,6 +458,53 @@ def test_structured_outlier_below_one_column_matches_plain_layer():
     torch.cuda.synchronize()
     assert torch.equal(a["codes"], b["codes"]) and int(b["H_nnz"].item()) == 0
     assert np.array_equal(a["obj"].cpu().numpy(), b["obj"].cpu().numpy())
+
+
+def test_outlier_warm_start_and_without_obj_cd():
+    """A warm start (init_codes) and a call without obj_cd refresh R from the codes
+    with no fused objective.  The run stays valid: the IHT half never increases g
+    (Lemma 3), g never increases (Lemma 2 from a feasible start), and g of the final
+    state recomputed in fp64 matches; without obj_cd the objective is the same."""
+    q, p, bits, iters, frac = 96, 192, 3, 4, 0.01
+    W = inputs.layer_weights(q, p, dtype=torch.bfloat16, seed=43, device="cuda", planted_frac=frac,
+                             planted_std=0.3)
+    X = inputs.calib_inputs(p, 2048, dtype=torch.bfloat16, seed=43, device="cuda", heavy_frac=0.02,
+                            heavy_mult=30.0)
+    Sg = qe.qe_build_sigma(X)
+    s_budget = int(round(frac * q * p))
+    first = qe.qe_quantize_layer_outlier(W, Sg, bits, iters, s_budget, power_iters=200)
+    out = qe.qe_quantize_layer_outlier(W, Sg, bits, iters, s_budget, power_iters=200,
+                                       init_codes=first["codes"])
+    assert qe.qe_sync_status() == qe.QE_OK
+    obj, obj_cd = out["obj"].cpu().numpy(), out["obj_cd"].cpu().numpy()
+    assert np.all(obj <= obj_cd * (1 + 1e-6)), "IHT step increased g (Lemma 3)"
+    assert np.all(np.diff(obj) <= 1e-6 * obj[:-1])
+    nnz = int(out["H_nnz"].item())
+    H = torch.zeros(q * p, dtype=torch.float64, device="cuda")
+    H[out["H_idx"][:nnz]] = out["H_val"][:nnz].double()
+    What = out["scales"].double()[:, None] * (out["codes"].double() - out["zeros"].double()[:, None])
+    D = W.double() - What - H.view(q, p)
+    g = float(torch.sum((D @ Sg.double()) * D).item())
+    parity.check_obj(obj[-1], g, what="g of the final state (fp64)")
+    # the same call through the C ABI with obj_cd = NULL
+    L = qe.load()
+    codes = torch.empty(q, p, dtype=torch.uint8, device="cuda")
+    sc = torch.empty(q, dtype=torch.float32, device="cuda")
+    zp = torch.empty(q, dtype=torch.float32, device="cuda")
+    ob = torch.empty(iters, dtype=torch.float64, device="cuda")
+    hv = torch.empty(s_budget, dtype=torch.float32, device="cuda")
+    hi = torch.empty(s_budget, dtype=torch.int64, device="cuda")
+    hn = torch.zeros(1, dtype=torch.int64, device="cuda")
+    o = qe.QEOpts()
+    o.power_iters = 200
+    o.init_codes = first["codes"].data_ptr()
+    st = L.qe_quantize_layer_outlier(W.data_ptr(), qe.QE_BF16, q, p, p, Sg.data_ptr(), bits, iters, s_budget,
+                                     ctypes.byref(o), codes.data_ptr(), sc.data_ptr(), zp.data_ptr(),
+                                     hv.data_ptr(), hi.data_ptr(), hn.data_ptr(), ob.data_ptr(), None,
+                                     ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
+    assert st == qe.QE_OK
+    assert qe.qe_sync_status() == qe.QE_OK
+    assert torch.equal(ob, out["obj"]) and torch.equal(codes, out["codes"])
 
 
 def test_outlier_zero_budget_matches_plain_layer():
