@@ -49,9 +49,54 @@ def parse():
                     help="outlier workloads: keep whole columns (Sec. 4.3, structured outliers)")
     ap.add_argument("--dense-sweeps", type=int, default=0,
                     help="sweeps whose cross-block term uses the tensor-core GEMM (0 = library default)")
+    ap.add_argument("--relax", type=int, default=0,
+                    help="relax heuristic period R (Sec. 3.2): sweeps t with t mod R = 0, t < iters, unquantized")
     ap.add_argument("--tokens", type=int, default=0,
                     help="override n (calibration tokens), for small profiling captures only")
     return ap.parse_args()
+
+
+def plan_sweeps(iters, relax, dense):
+    """The sweep schedule of qe_quantize_layer, mirrored: per sweep its kind and
+    window ("first": classic sweep 1 + a residual refresh with the objective; "seq":
+    a relaxed sweep or the one after it, three-plane changes; "dense": tensor-core
+    window sweep; "list": change-list sweep), the residual refreshes without the
+    objective, and the change-list launches (one per run of list sweeps, per 32)."""
+    def relaxed(t):
+        return relax > 0 and (t + 1) % relax == 0 and t + 1 < iters
+    sweeps, refreshes, list_runs = [], 0, []
+    t, src = 0, "w"
+    if not relaxed(0):
+        sweeps.append(("first", 0))
+        t, src = 1, "codes"
+    exact, chain = True, False
+    while t < iters:
+        if relaxed(t) or src != "codes":
+            if not exact and not chain:
+                refreshes += 1
+                exact = True
+            sweeps.append(("seq", -1 if exact else 1))
+            src = "v" if relaxed(t) else "codes"
+            t += 1
+            exact, chain = False, True
+            if src == "codes" and t < iters:
+                refreshes += 1
+                exact, chain = True, False
+            continue
+        tend = t
+        while tend < iters and not relaxed(tend):
+            tend += 1
+        while t < tend and t < dense:
+            sweeps.append(("dense", -1 if exact else 1))
+            t += 1
+            exact, chain = False, False
+        while t < tend:
+            te = min(tend, t + 32)
+            list_runs.append(te - t)
+            sweeps += [("list", 0)] * (te - t)
+            t = te
+            exact, chain = False, False
+    return sweeps, refreshes, list_runs
 
 
 def peaks():
@@ -277,7 +322,7 @@ def main():
             return qe.qe_quantize_layer_outlier(Wt, Sigma, b, cfg.iters, cfg.s_budget, workspace=ws,
                                                 structured=args.structured, timer=timer)
         return qe.qe_quantize_layer(Wt, Sigma, b, cfg.iters, workspace=ws, timer=timer,
-                                    dense_sweeps=args.dense_sweeps)
+                                    dense_sweeps=args.dense_sweeps, relax_period=args.relax)
     stream = torch.cuda.current_stream()
     nb = len(cfg.bits)
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(nb + 2)]
@@ -344,14 +389,18 @@ def main():
     tri_flops = sum(2 * q * bw * b0 for b0, bw in blocks)
     win_flops = sum(2 * q * bw * p for b0, bw in blocks)
     dense = cfg.iters if outlier else (args.dense_sweeps or DEFAULT_DENSE_SWEEPS)
-    trail_flops, trail_launches = tri_flops, nblk - 1
-    for t in range(1, cfg.iters):
-        if outlier:     # Algorithm 4: sweeps after the first take the change lists
-            continue
-        elif t < dense:   # later sweeps take the cross-block term from the change lists
-            trail_flops += tri_flops if t == 1 else win_flops
-            trail_launches += nblk - 1 if t == 1 else nblk
-    refreshes = cfg.iters if outlier else 1         # residual GEMMs per layer
+    if outlier:     # Algorithm 4: sweep 1 blocked, later sweeps take the change lists
+        plan, extra_refreshes, list_runs = [("first", 0)] + [("list", 0)] * (cfg.iters - 1), 0, []
+    else:
+        plan, extra_refreshes, list_runs = plan_sweeps(cfg.iters, args.relax, dense)
+    trail_flops = trail_exec = 0
+    for kind, window in plan:
+        if kind in ("first", "seq", "dense"):
+            f = win_flops if window == 1 else tri_flops
+            trail_flops += f
+            trail_exec += (3 if kind == "dense" else 6) * f   # three-plane changes: 6 products
+    # residual GEMMs per layer (besides P): after sweep 1 (or every iteration, Algorithm 4)
+    refreshes = cfg.iters if outlier else (1 if plan[0][0] == "first" else 0) + extra_refreshes
 
     units_per_step = q * p * p * cfg.iters * nb           # column updates per rank per step
     value = units_per_step * world / (ms / 1e3)
@@ -365,6 +414,7 @@ def main():
               "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
               "config": {"workload": cfg.name, "q": q, "p": p, "n": n, "bits": list(cfg.bits),
                          "sweeps": cfg.iters, "parallelism": f"layer-replicas x{world}",
+                         **({"relax_period": args.relax} if args.relax else {}),
                          "l2": "inputs larger than L2 (X is %.2f GiB)" % (p * n * 2 / 2**30),
                          **({"s_budget": cfg.s_budget,
                              "outliers": "columns" if args.structured else "entries"} if outlier else {})},
@@ -381,13 +431,12 @@ def main():
     qpad, ppad = -(-q // 128) * 128, -(-p // 256) * 256
     gemm_flops = sig_flops + nb * (2 * q * p * p * (1 + refreshes) + trail_flops)
     gemm_exec = (gemm_tiles_sigma(p) * 2 * 128 * 256 * n
-                 + nb * ((1 + refreshes) * 3 * 2 * qpad * ppad * (-(-p // 64) * 64)
-                         + 6 * tri_flops + 3 * (trail_flops - tri_flops)))   # 6 products in sweep 1
+                 + nb * ((1 + refreshes) * 3 * 2 * qpad * ppad * (-(-p // 64) * 64) + trail_exec))
     result["roofline"] = roofline_gemm(gemm_flops, gemm_exec, gemm_ms, gemm_launches, pk)
     # the persistent change-list kernel: one launch per layer (per 32 list sweeps)
     list_launches, list_ms = timed[qe.QE_KERNEL_CD_LISTS]
-    n_list = max(cfg.iters - dense, 0)
-    n_chunks = -(-n_list // 32)
+    n_list = sum(1 for kind, _ in plan if kind == "list")
+    n_chunks = len(list_runs)
     list_bytes = n_list * (4 * q * p + q * p + 4 * p * p) / n_chunks if n_chunks else 0
     if not outlier:
         result["roofline_cd"] = roofline_lists(list_bytes, list_ms / args.steps, list_launches // args.steps, pk)
@@ -420,10 +469,14 @@ def main():
     # residual GEMM + objective sum; dense window sweeps: trailing GEMMs (nblk - 1 in the
     # first) + nblk in-block + objective step; list sweeps: one persistent launch and one
     # objective prefix per 32 sweeps
-    per_layer = 8 + w_planes + (nblk - 1) + nblk + 2
-    for t in range(1, min(dense, cfg.iters)):
-        per_layer += (nblk - 1 if t == 1 else nblk) + nblk + 1
-    per_layer += 2 * -(-max(cfg.iters - max(dense, 1), 0) // 32)
+    # seq / dense sweeps: trailing GEMMs (nblk - 1 with window -1) + nblk in-block +
+    # objective step; an extra refresh: codes -> C - z + residual GEMM
+    per_layer = 8 + w_planes + 2 * extra_refreshes + 2 * len(list_runs)
+    for kind, window in plan:
+        if kind == "first":
+            per_layer += (nblk - 1) + nblk + 2
+        elif kind in ("seq", "dense"):
+            per_layer += (nblk if window == 1 else nblk - 1) + nblk + 1
     if outlier:
         # selection (P_s: 4 radix passes x 2 + count, scan, emit; columns: + 2 norm
         # kernels + emit), start: copy, selection, scatter + row pointers, grid,

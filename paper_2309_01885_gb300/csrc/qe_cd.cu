@@ -510,7 +510,10 @@ __device__ __forceinline__ double warp_sum(double x) {
 // RELAX: the relax heuristic (Sec. 3.2): a live column (Sigma_jj > 0) takes
 // beta~ itself instead of its nearest level; a dead one stays on its level.
 // DF: the objective change of each decision (Lemma 1 along one coordinate)
-// goes to rowdf, as in the change-driven kernels.
+// goes to rowdf, as in the change-driven kernels: the deciding lane only stores
+// beta~ of its column (in grid units) to the warp's row of shared memory, and
+// the changes are formed after the sweep over the block, so the sequential
+// chain waits on no load.
 template <int B, bool FULL, bool RELAX, bool DF>
 __global__ void __launch_bounds__(1024) k_cd_block_seq(const CdArgs a) {
     using C = CdCfg<B>;
@@ -519,6 +522,7 @@ __global__ void __launch_bounds__(1024) k_cd_block_seq(const CdArgs a) {
     float *tri = cd_smem;
     uint64_t *bar = reinterpret_cast<uint64_t *>(cd_smem + C::PACK);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    float *tdec = cd_smem + C::PACK + 4 + warp * B;   // DF: beta~ at each decision (after the barrier)
     const int64_t i = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + warp;
     const bool row_ok = i < a.q;
     float t[CPL], st[CPL];
@@ -531,12 +535,6 @@ __global__ void __launch_bounds__(1024) k_cd_block_seq(const CdArgs a) {
 #pragma unroll
         for (int h = 0; h < CPL; ++h)
             if ((FULL || 32 * h + lane < bw) && a.d[a.b0 + 32 * h + lane] > 0.0f) live |= 1u << h;
-    }
-    float s2 = 0.0f;
-    double dfacc = 0.0;
-    if (DF) {
-        const float sc = a.scale[i];
-        s2 = sc * sc;
     }
     float code[CPL], dlt[CPL];
 #pragma unroll
@@ -556,13 +554,7 @@ __global__ void __launch_bounds__(1024) k_cd_block_seq(const CdArgs a) {
             if (lane == jj) {
                 code[h] = c;
                 dlt[h] = dl;
-                if (DF) {
-                    const float dj = a.d[a.b0 + j];
-                    if (dj > 0.0f) {
-                        const float e1 = c - t[h], e0 = st[h] - t[h];
-                        dfacc += static_cast<double>(dj * s2 * (e1 * e1 - e0 * e0));
-                    }
-                }
+                if (DF) tdec[j] = t[h];
             }
             const float db = __shfl_sync(0xffffffffu, dl, jj);
             if (db != 0.0f) {
@@ -573,6 +565,21 @@ __global__ void __launch_bounds__(1024) k_cd_block_seq(const CdArgs a) {
         }
     }
     if (DF) {
+        __syncwarp();
+        const float sc = a.scale[i];
+        const float s2 = sc * sc;
+        double dfacc = 0.0;
+#pragma unroll
+        for (int h = 0; h < CPL; ++h) {
+            const int l = 32 * h + lane;
+            if (!FULL && l >= bw) continue;
+            const float dj = a.d[a.b0 + l];
+            if (dj > 0.0f) {
+                const float tv = tdec[l];
+                const float e1 = code[h] - tv, e0 = st[h] - tv;
+                dfacc += static_cast<double>(dj * s2 * (e1 * e1 - e0 * e0));
+            }
+        }
         dfacc = warp_sum(dfacc);
         if (lane == 0) a.rowdf[i] += dfacc;
     }
@@ -1055,14 +1062,16 @@ static cudaError_t launch_cd_block_b(const CdArgs &a, int nsm, cudaStream_t s) {
     using C = CdCfg<B>;
     if (a.nsplit > C::MAX_SPLITS) return cudaErrorInvalidValue;
     auto kern = SEQ ? k_cd_block_seq<B, FULL, RELAX, DF> : k_cd_block_chg<B, FULL>;
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
-    if (e != cudaSuccess) return e;
     // one CTA per SM when the rows allow it (the packed block is shared by the CTA's rows)
     int64_t warps = ceil_div(a.q, nsm);
     if (warps > C::MAX_WARPS) warps = C::MAX_WARPS;
     if (warps < 1) warps = 1;
+    // the sequential kernel with DF keeps one row of beta~ per warp after the packed block
+    const int smem = (SEQ && DF) ? (C::PACK + 4) * 4 + static_cast<int>(warps) * B * 4 : C::SMEM;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
     const unsigned grid = static_cast<unsigned>(ceil_div(a.q, warps));
-    kern<<<grid, static_cast<unsigned>(32 * warps), C::SMEM, s>>>(a);
+    kern<<<grid, static_cast<unsigned>(32 * warps), smem, s>>>(a);
     return cudaGetLastError();
 }
 

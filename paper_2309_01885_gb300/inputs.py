@@ -113,9 +113,10 @@ class LayerConfig:
                             heavy_frac=self.heavy_frac, heavy_mult=self.heavy_mult)
 
 
-# The five synthetic workloads: an OPT-125m-sized layer (oracle-sized), a
-# LLaMA-7B attention projection, the LLaMA-7B MLP pair, the Falcon-180B QKV and
-# down projections, and the outlier-aware variant of the LLaMA-7B projection.
+# The synthetic workloads: an OPT-125m-sized layer (oracle-sized), a LLaMA-7B
+# attention projection, the LLaMA-7B MLP pair, the Falcon-180B QKV and down
+# projections, and the outlier-aware variant of the LLaMA-7B projection at 3 bits
+# with 1% outliers and at 2 bits with 2%.
 CONFIGS = {
     "opt125m_768x768": LayerConfig("opt125m_768x768", 768, 768, 4096, torch.float32,
                                    torch.float32, (4,), 5, heavy_frac=0.01, heavy_mult=20.0,
@@ -139,4 +140,9 @@ CONFIGS = {
                                                   262144, torch.bfloat16, torch.bfloat16, (3,), 20,
                                                   heavy_frac=0.005, planted_frac=0.01,
                                                   planted_std=0.3, outlier_budget_frac=0.01),
+    # the 2-bit regime of Sec. 5 (2 bits with 2% outliers): the same path at b = 2, twice the budget
+    "llama7b_proj_outlier2b_4096x4096": LayerConfig("llama7b_proj_outlier2b_4096x4096", 4096, 4096,
+                                                    262144, torch.bfloat16, torch.bfloat16, (2,), 20,
+                                                    heavy_frac=0.005, planted_frac=0.02,
+                                                    planted_std=0.3, outlier_budget_frac=0.02),
 }

@@ -130,15 +130,18 @@ def test_fullsize_layer_sampled_rows(name, nrows, free_run, full_obj):
         torch.cuda.empty_cache()
 
 
-@pytest.mark.parametrize("structured", [False, True], ids=["entries", "columns"])
-def test_fullsize_outlier_properties(structured):
+@pytest.mark.parametrize("name,structured", [("llama7b_proj_outlier_4096x4096", False),
+                                             ("llama7b_proj_outlier_4096x4096", True),
+                                             ("llama7b_proj_outlier2b_4096x4096", False)],
+                         ids=["3bit-entries", "3bit-columns", "2bit-entries"])
+def test_fullsize_outlier_properties(name, structured):
     """The outlier-aware workload at full size.  The IHT support is a global
     top-s (Eq. iht-update), so rows are not independent here: the sampled-row
     check covers the grid (W without the initial support P_s(W), Sec. 4.3);
     the rest are properties: the budget, sorted unique indices, Lemma 3 (the
     IHT half never increases g), a non-increasing g, and g of the final state
     recomputed in fp64."""
-    cfg = inputs.CONFIGS["llama7b_proj_outlier_4096x4096"]
+    cfg = inputs.CONFIGS[name]
     q, p = cfg.q, cfg.p
     W = cfg.weights("cuda")
     X = cfg.inputs("cuda")
