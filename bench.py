@@ -168,23 +168,32 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
+# The sources the bench step's kernels are compiled from and launched by (the
+# layer schedule, the CD kernels, the tensor-core GEMM and their shared headers).
+TRAFFIC_SOURCES = ("qe_api.cu", "qe_cd.cu", "qe_common.cuh", "qe_gemm.cu", "qe_internal.h", "qe_kernels.h")
+
+
+def traffic_sources_sha256() -> str:
+    import hashlib
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2309_01885_gb300", "csrc")
+    for name in TRAFFIC_SOURCES:
+        with open(os.path.join(csrc, name), "rb") as fh:
+            h.update(name.encode() + b"\0" + fh.read())
+    return h.hexdigest()
+
+
 def traffic_per_launch(kernel: str, launches_per_step: int):
     """DRAM bytes per launch from the committed ncu summary (bytes of all launches of
     one bench step), if the kernel sources are unchanged since it was taken (else None)."""
-    import hashlib
     path = os.path.join(ROOT, "profiles", "roofline_traffic.json")
     try:
         with open(path) as fh:
             rec = json.load(fh)
     except (OSError, ValueError):
         return None
-    h = hashlib.sha256()
-    csrc = os.path.join(ROOT, "paper_2309_01885_gb300", "csrc")
-    for name in sorted(os.listdir(csrc)):
-        with open(os.path.join(csrc, name), "rb") as fh:
-            h.update(name.encode() + b"\0" + fh.read())
     entry = rec.get(kernel)
-    if not entry or entry.get("csrc_sha256") != h.hexdigest() or not launches_per_step:
+    if not entry or entry.get("sources_sha256") != traffic_sources_sha256() or not launches_per_step:
         return None
     return entry.get("dram_bytes_per_step") / launches_per_step
 

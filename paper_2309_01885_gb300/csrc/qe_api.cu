@@ -892,7 +892,7 @@ qe_status qe_quantize_layer_outlier(const void *W, qe_dtype w_dtype, int64_t q, 
     // P_W = W (I + Sigma_bar), eta = 1 / (2 lambda_max), P = P_W - H (I + Sigma_bar)
     if ((st = prepare(c, W, wbf16, ldw, Sigma, c.PW)) != QE_OK) return st;
     QE_CK(launch_power_lambda(Sigma, p, p, power_iters, c.y0, c.y1, c.lam, c.eta, c.nsm, c.s));
-    QE_CK(launch_spmm_refresh(c.PW, c.P, c.R, ld, Sigma, p, c.d, c.dinv, H_idx, H_val, c.rowptr, q, p, 0, scales,
+    QE_CK(launch_spmm_refresh(c.PW, c.P, c.R, ld, c.sbar, ld, H_idx, H_val, c.rowptr, q, p, 0, scales,
                               c.s));
     if (opts && opts->wx_norm2)
         if ((st = objective(c, W, wbf16, ldw, c.H, nullptr, nullptr, nullptr, c.P, opts->wx_norm2)) != QE_OK)
@@ -927,7 +927,7 @@ qe_status qe_quantize_layer_outlier(const void *W, qe_dtype w_dtype, int64_t q, 
         QE_CK(cudaMemsetAsync(c.H, 0, static_cast<size_t>(q) * ld * 4, c.s));
         QE_CK(launch_scatter_rowptr(H_idx, H_val, H_nnz, s_budget, q, p, c.H, ld, c.rowptr, c.s));
         // P = P_W - H (I + Sigma_bar); R += P_new - P_old  (R = P - What Sigma_bar stays current)
-        QE_CK(launch_spmm_refresh(c.PW, c.P, c.R, ld, Sigma, p, c.d, c.dinv, H_idx, H_val, c.rowptr, q, p, 1, scales,
+        QE_CK(launch_spmm_refresh(c.PW, c.P, c.R, ld, c.sbar, ld, H_idx, H_val, c.rowptr, q, p, 1, scales,
                                   c.s));
         if ((st = objective(c, W, wbf16, ldw, c.H, codes, scales, zeros, c.R, obj + t)) != QE_OK) return st;
         if (opts && opts->sweep_codes)

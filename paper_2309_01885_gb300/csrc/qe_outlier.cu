@@ -361,52 +361,79 @@ __global__ void k_rowptr(const int64_t *H_idx, const int64_t *nnz, int64_t q, in
     rowptr[i] = lo;
 }
 
-// P_new = P_W - H (I + Sigma_bar) for row i (Sigma_bar_kj = Sigma_kj / d_j off
-// the diagonal, 0 for dead columns); R += (P_new - P_old) / s_i when update_r
-// (R in grid-step units); P = P_new.  One CTA per (row, tile of kSpmmCols
-// columns): each thread keeps kSpmmPer columns in registers and walks the row's
-// kept entries, so every entry issues kSpmmPer independent coalesced loads of its
-// Sigma row.
+// P_new = P_W - H (I + Sigma_bar) for row i; R += (P_new - P_old) / s_i when
+// update_r (R in grid-step units); P = P_new.  Sigma_bar comes as fp32 rows
+// (sbar[k][j] = Sigma_jk / d_j, zero on the diagonal and for dead columns: the
+// binary32 values the tensor-core planes split), so the identity adds 1 at
+// j = k.  One CTA per (row, tile of kSpmmCols columns); each thread keeps
+// kSpmmPer columns in registers.  The row's kept entries are staged in shared
+// memory kSpmmChunk at a time, and the rows of kSpmmU entries are in flight
+// together, so no index load sits in the gather chain; the entries are still
+// added one after another in their sorted order.
 constexpr int kSpmmPer = 16;
 constexpr int kSpmmCols = 256 * kSpmmPer;
+constexpr int kSpmmChunk = 256;
+constexpr int kSpmmU = 2;
 
 __global__ void __launch_bounds__(256) k_spmm_refresh(const float *PW, float *P, float *R, int64_t ld,
-                                                      const float *S, int64_t lds, const float *d,
-                                                      const float *dinv, const int64_t *H_idx,
-                                                      const float *H_val, const int64_t *rowptr,
-                                                      int64_t p, int update_r, const float *scale) {
+                                                      const float *sbar, int64_t lds, const int64_t *H_idx,
+                                                      const float *H_val, const int64_t *rowptr, int64_t p,
+                                                      int update_r, const float *scale) {
+    __shared__ int sk[kSpmmChunk];
+    __shared__ float sv[kSpmmChunk];
     const int64_t i = blockIdx.x;
     const int64_t j0 = static_cast<int64_t>(blockIdx.y) * kSpmmCols + threadIdx.x;
-    const float s = update_r ? scale[i] : 1.0f;
     const int64_t e0 = rowptr[i], e1 = rowptr[i + 1];
-    float acc[kSpmmPer], ij[kSpmmPer];
-    bool alive[kSpmmPer];
+    float acc[kSpmmPer];
 #pragma unroll
     for (int u = 0; u < kSpmmPer; ++u) {
         const int64_t j = j0 + 256 * u;
-        const bool ok = j < p;
-        acc[u] = ok ? __ldcs(PW + i * ld + j) : 0.0f;   // streamed: keep L2 for Sigma's rows
-        ij[u] = ok ? dinv[j] : 0.0f;
-        alive[u] = ok && d[j] > 0.0f;
+        acc[u] = j < p ? __ldcs(PW + i * ld + j) : 0.0f;   // streamed: keep L2 for Sigma_bar's rows
     }
-    for (int64_t e = e0; e < e1; ++e) {
-        const int64_t k = H_idx[e] - i * p;
-        const float v = H_val[e];
-        const bool kalive = d[k] > 0.0f;
-        const float *srow = S + k * lds;
-        float sv[kSpmmPer];
-#pragma unroll
-        for (int u = 0; u < kSpmmPer; ++u) {
-            const int64_t j = j0 + 256 * u;
-            sv[u] = (j < p && kalive) ? srow[j] : 0.0f;
+    for (int64_t c0 = e0; c0 < e1; c0 += kSpmmChunk) {
+        const int n = static_cast<int>((e1 - c0) < kSpmmChunk ? (e1 - c0) : kSpmmChunk);
+        __syncthreads();   // the previous chunk is consumed
+        if (static_cast<int>(threadIdx.x) < n) {
+            sk[threadIdx.x] = static_cast<int>(H_idx[c0 + threadIdx.x] - i * p);
+            sv[threadIdx.x] = H_val[c0 + threadIdx.x];
         }
+        __syncthreads();
+        int e = 0;
+        for (; e + kSpmmU <= n; e += kSpmmU) {
+            int k[kSpmmU];
+            float v[kSpmmU][kSpmmPer];
 #pragma unroll
-        for (int u = 0; u < kSpmmPer; ++u) {
-            const int64_t j = j0 + 256 * u;
-            const float sb = (k == j) ? 1.0f : (alive[u] ? sv[u] * ij[u] : 0.0f);
-            acc[u] = fmaf(-v, sb, acc[u]);
+            for (int x = 0; x < kSpmmU; ++x) {
+                k[x] = sk[e + x];
+                const float *srow = sbar + static_cast<int64_t>(k[x]) * lds;
+#pragma unroll
+                for (int u = 0; u < kSpmmPer; ++u) {
+                    const int64_t j = j0 + 256 * u;
+                    v[x][u] = j < p ? __ldg(srow + j) : 0.0f;
+                }
+            }
+#pragma unroll
+            for (int x = 0; x < kSpmmU; ++x) {
+                const float hv = sv[e + x];
+#pragma unroll
+                for (int u = 0; u < kSpmmPer; ++u) {
+                    const int64_t j = j0 + 256 * u;
+                    acc[u] = fmaf(-hv, (j == k[x]) ? 1.0f : v[x][u], acc[u]);
+                }
+            }
+        }
+        for (; e < n; ++e) {
+            const int kk = sk[e];
+            const float hv = sv[e];
+            const float *srow = sbar + static_cast<int64_t>(kk) * lds;
+#pragma unroll
+            for (int u = 0; u < kSpmmPer; ++u) {
+                const int64_t j = j0 + 256 * u;
+                if (j < p) acc[u] = fmaf(-hv, (j == kk) ? 1.0f : __ldg(srow + j), acc[u]);
+            }
         }
     }
+    const float s = update_r ? scale[i] : 1.0f;
 #pragma unroll
     for (int u = 0; u < kSpmmPer; ++u) {
         const int64_t j = j0 + 256 * u;
@@ -513,12 +540,11 @@ cudaError_t launch_scatter_rowptr(const int64_t *H_idx, const float *H_val, cons
     return cudaGetLastError();
 }
 
-cudaError_t launch_spmm_refresh(const float *PW, float *P, float *R, int64_t ld, const float *S,
-                                int64_t lds, const float *d, const float *dinv, const int64_t *H_idx,
-                                const float *H_val, const int64_t *rowptr, int64_t q, int64_t p,
-                                int update_r, const float *scale, cudaStream_t s) {
+cudaError_t launch_spmm_refresh(const float *PW, float *P, float *R, int64_t ld, const float *sbar,
+                                int64_t lds, const int64_t *H_idx, const float *H_val, const int64_t *rowptr,
+                                int64_t q, int64_t p, int update_r, const float *scale, cudaStream_t s) {
     const dim3 grid(static_cast<unsigned>(q), static_cast<unsigned>(ceil_div(p, kSpmmCols)));
-    k_spmm_refresh<<<grid, 256, 0, s>>>(PW, P, R, ld, S, lds, d, dinv, H_idx, H_val, rowptr, p, update_r, scale);
+    k_spmm_refresh<<<grid, 256, 0, s>>>(PW, P, R, ld, sbar, lds, H_idx, H_val, rowptr, p, update_r, scale);
     return cudaGetLastError();
 }
 

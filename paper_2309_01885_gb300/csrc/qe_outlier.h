@@ -41,10 +41,9 @@ cudaError_t launch_topk_columns(const float *T, int64_t q, int64_t p, int64_t k,
 cudaError_t launch_scatter_rowptr(const int64_t *H_idx, const float *H_val, const int64_t *nnz,
                                   int64_t cap, int64_t q, int64_t p, float *H, int64_t ld,
                                   int64_t *rowptr, cudaStream_t s);
-cudaError_t launch_spmm_refresh(const float *PW, float *P, float *R, int64_t ld, const float *S,
-                                int64_t lds, const float *d, const float *dinv, const int64_t *H_idx,
-                                const float *H_val, const int64_t *rowptr, int64_t q, int64_t p,
-                                int update_r, const float *scale, cudaStream_t s);
+cudaError_t launch_spmm_refresh(const float *PW, float *P, float *R, int64_t ld, const float *sbar,
+                                int64_t lds, const int64_t *H_idx, const float *H_val, const int64_t *rowptr,
+                                int64_t q, int64_t p, int update_r, const float *scale, cudaStream_t s);
 cudaError_t launch_dinv(const float *d, int64_t p, float *dinv, cudaStream_t s);
 
 }  // namespace qe
