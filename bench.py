@@ -409,7 +409,7 @@ def main():
             trail_flops += f
             trail_exec += (3 if kind == "dense" else 6) * f   # three-plane changes: 6 products
     # residual GEMMs per layer (besides P): after sweep 1 (or every iteration, Algorithm 4)
-    refreshes = cfg.iters if outlier else (1 if plan[0][0] == "first" else 0) + extra_refreshes
+    refreshes = (1 if plan[0][0] == "first" else 0) + extra_refreshes
 
     units_per_step = q * p * p * cfg.iters * nb           # column updates per rank per step
     value = units_per_step * world / (ms / 1e3)
@@ -491,11 +491,12 @@ def main():
         # kernels + emit), start: copy, selection, scatter + row pointers, grid,
         # Sigma_bar set-up (5) + [W planes] + P, 64 power steps (+ fill, last, final),
         # SpMM refresh, initial residual; sweep 1 blocked (2 nblk - 1), later sweeps one
-        # change-list launch; per iteration: residual GEMM + objective sum, IHT target,
-        # selection, scatter + row pointers, SpMM, objective (2)
+        # change-list launch (ending with the flush of its window into R) and an
+        # objective prefix, sweep 1 a residual GEMM + objective sum; per iteration: IHT
+        # target, selection, scatter + row pointers, SpMM, objective (2)
         sel = 14 if args.structured else 11
-        per_layer = (1 + sel + 2 + 1 + 6 + w_planes + 67 + 1 + 1 + (2 * nblk - 1) + (cfg.iters - 1)
-                     + cfg.iters * (2 + 1 + sel + 2 + 1 + 2))
+        per_layer = (1 + sel + 2 + 1 + 6 + w_planes + 67 + 1 + 1 + (2 * nblk - 1) + 2 * (cfg.iters - 1) + 2
+                     + cfg.iters * (1 + sel + 2 + 1 + 2))
     result["gpu_launches"] = args.steps * (1 + nb * per_layer)
 
     # end to end through the C ABI with host buffers

@@ -844,7 +844,7 @@ qe_status qe_quantize_layer(const void *W, qe_dtype w_dtype, int64_t q, int64_t 
                 Timed tm(c.timer, QE_KERNEL_CD_LISTS, c.s);
                 // with empty lists (after a refresh) the first sweep steps in lockstep
                 QE_CK(launch_cd_rows_lists(pl.B, a, t, te, c.rowdft, opts ? opts->sweep_codes : nullptr,
-                                           exact ? 1 : 0, free_changes(opts), c.nsm, c.s));
+                                           exact ? 1 : 0, free_changes(opts), 0, c.nsm, c.s));
             }
             QE_CK(launch_obj_prefix(c.rowdft, q, te - t, t == 0 ? c.objbase : obj + t - 1, obj + t, c.s));
             t = te;
@@ -905,22 +905,30 @@ qe_status qe_quantize_layer_outlier(const void *W, qe_dtype w_dtype, int64_t q, 
     } else {
         QE_CK(launch_init_residual(W, wbf16, ldw, c.H, ld, q, p, scales, zeros, c.R, ld, c.s));
     }
+    // g of a warm start, the base of the first sweep's objective changes
+    if (warm && obj_cd)
+        if ((st = objective(c, W, wbf16, ldw, c.H, codes, scales, zeros, c.R, c.objbase)) != QE_OK) return st;
     for (int t = 0; t < iters; ++t) {
         if (t == 0 && !warm) {
+            // sweep 1 from What = W: the blocked classic sweep, then the residual GEMM
+            // (with g fused)
             if ((st = sweep(c, codes, scales, zeros, bits, SRC_W, false, 0)) != QE_OK) return st;
+            const ObjFuse f{obj_cd ? obj_cd + t : nullptr, W, wbf16, ldw, codes, c.H};
+            if ((st = residual(c, scales, zeros, obj_cd ? &f : nullptr)) != QE_OK) return st;
         } else {
-            // R is fresh and the target W - H stays fixed during the sweep: one
+            // R is exact and the target W - H stays fixed during the sweep: one
             // change-list sweep whose window starts empty (each block corrected by
-            // this sweep's changes left of it); it keeps C - z current for the
-            // residual GEMM below
+            // this sweep's changes left of it), which ends by flushing the window into
+            // R; g after it = g before + the objective changes of its decisions
             QE_CK(cudaMemsetAsync(c.lcnt, 0, static_cast<size_t>(q) * pl.nblk * 4, c.s));
             CdArgs a = list_args(c, codes, scales, zeros, bits);
-            a.write_qf = 1;
-            Timed tm(c.timer, QE_KERNEL_CD_LISTS, c.s);
-            QE_CK(launch_cd_rows_lists(pl.B, a, t, t + 1, c.rowdft, nullptr, 1, kFreeMaxChanges, c.nsm, c.s));
+            {
+                Timed tm(c.timer, QE_KERNEL_CD_LISTS, c.s);
+                QE_CK(launch_cd_rows_lists(pl.B, a, t, t + 1, c.rowdft, nullptr, 1, kFreeMaxChanges, 1, c.nsm,
+                                           c.s));
+            }
+            if (obj_cd) QE_CK(launch_obj_prefix(c.rowdft, q, 1, t == 0 ? c.objbase : obj + t - 1, obj_cd + t, c.s));
         }
-        const ObjFuse f{obj_cd ? obj_cd + t : nullptr, W, wbf16, ldw, codes, c.H};
-        if ((st = residual(c, scales, zeros, obj_cd ? &f : nullptr)) != QE_OK) return st;
         // IHT step: T = H + 2 eta d (R - What); H = P_s(T)
         QE_CK(launch_iht_target(c.H, c.R, ld, codes, p, scales, zeros, c.d, c.eta, q, p, c.T, c.s));
         QE_CK(select(c.T));

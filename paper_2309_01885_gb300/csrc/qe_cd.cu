@@ -318,17 +318,18 @@ struct CdCfg {
 // (this one included) the changes of its most recent visit, each adding
 // Delta'_ik Sigma_bar[k][block] to the row; Sigma_bar rows are fp32 and
 // contiguous over the block, so each change is one coalesced read of B floats
-// per warp.  Returns whether the row had any change in the window.
+// per warp.  Returns whether the row had any change in the window.  Lists of
+// blocks below bmin are left out.
 template <int B, bool FULL, int U = 4>
 __device__ __forceinline__ bool list_correction(const CdArgs &a, int64_t b0, int bw_, int64_t ii, bool row_ok,
-                                                int lane, float (&ps)[B / 32]) {
+                                                int lane, float (&ps)[B / 32], int bmin = 0) {
     constexpr int CPL = B / 32;
     const int bw = FULL ? B : bw_;
     const int64_t rb = ii * a.nblk;
     const float *sb0 = a.sbar + b0 + lane;
     bool any = false;
     for (int c0 = 0; c0 < a.nblk; c0 += 32) {
-        const int cnt = (row_ok && c0 + lane < a.nblk) ? a.lcnt[rb + c0 + lane] : 0;
+        const int cnt = (row_ok && c0 + lane < a.nblk && c0 + lane >= bmin) ? a.lcnt[rb + c0 + lane] : 0;
         unsigned m = __ballot_sync(0xffffffffu, cnt > 0);
         any = any || m != 0u;
         while (m != 0u) {
@@ -924,13 +925,16 @@ __device__ __forceinline__ void rows_block_win(const CdArgs &a, int64_t b0, int 
 // first_lockstep forces lockstep for the first sweep (its lists are empty
 // after a residual refresh although many codes are about to change).
 // Per sweep and row the objective change goes to rowdf_t[t - t_begin][i]; with
-// sweep_codes the row's codes after each sweep are copied out.
+// sweep_codes the row's codes after each sweep are copied out.  flush: after the
+// last sweep every block's base takes the changes of the lists of its own and
+// later blocks (the ones its last visit did not see), so R is the exact residual
+// of the final codes.
 constexpr int kRowsMaxWarps = 28;   // rows per CTA of the persistent kernel (896 threads: 72 registers)
 
 template <int B>
 __global__ void __launch_bounds__(32 * kRowsMaxWarps, 1) k_cd_rows_lists(const CdArgs a, int t_begin, int t_end,
                                                            double *rowdf_t, uint8_t *sweep_codes,
-                                                           int first_lockstep, int free_max_changes) {
+                                                           int first_lockstep, int free_max_changes, int flush) {
     using C = CdCfg<B>;
     extern __shared__ __align__(16) float cd_smem[];
     float *tri = cd_smem;
@@ -1033,6 +1037,25 @@ __global__ void __launch_bounds__(32 * kRowsMaxWarps, 1) k_cd_rows_lists(const C
             }
         }
     }
+    if (flush && row_ok) {
+        constexpr int CPL = B / 32;
+        __syncwarp();
+        for (int64_t b0 = 0; b0 < a.p; b0 += B) {
+            const int bw = static_cast<int>((a.p - b0) < B ? (a.p - b0) : B);
+            float ps[CPL];
+#pragma unroll
+            for (int h = 0; h < CPL; ++h) ps[h] = 0.0f;
+            const int bmin = static_cast<int>(b0 / B);
+            const bool any = bw == B ? list_correction<B, true>(a, b0, bw, i, true, lane, ps, bmin)
+                                     : list_correction<B, false>(a, b0, bw, i, true, lane, ps, bmin);
+            if (!any) continue;
+#pragma unroll
+            for (int h = 0; h < CPL; ++h) {
+                const int l = 32 * h + lane;
+                if (l < bw) a.R[i * a.ldr + b0 + l] += ps[h];
+            }
+        }
+    }
 }
 
 // obj[t] = obj[t-1] + sum_i rowdf_t[t][i] for nt <= 32 sweeps; prev may be NULL (0).
@@ -1101,8 +1124,8 @@ int64_t packed_diag_floats(int64_t p, int B) { return ceil_div(p, B) * packed_bl
 
 template <int B>
 static cudaError_t launch_cd_rows_b(const CdArgs &a, int t_begin, int t_end, double *rowdf_t,
-                                   uint8_t *sweep_codes, int first_lockstep, int free_max_changes, int nsm,
-                                   cudaStream_t s) {
+                                   uint8_t *sweep_codes, int first_lockstep, int free_max_changes, int flush,
+                                   int nsm, cudaStream_t s) {
     using C = CdCfg<B>;
     int64_t warps = ceil_div(a.q, nsm);
     if (warps > kRowsMaxWarps) warps = kRowsMaxWarps;
@@ -1113,19 +1136,19 @@ static cudaError_t launch_cd_rows_b(const CdArgs &a, int t_begin, int t_end, dou
     if (e != cudaSuccess) return e;
     const unsigned grid = static_cast<unsigned>(ceil_div(a.q, warps));
     k_cd_rows_lists<B><<<grid, static_cast<unsigned>(32 * warps), smem, s>>>(
-        a, t_begin, t_end, rowdf_t, sweep_codes, first_lockstep, free_max_changes);
+        a, t_begin, t_end, rowdf_t, sweep_codes, first_lockstep, free_max_changes, flush);
     return cudaGetLastError();
 }
 
 cudaError_t launch_cd_rows_lists(int B, const CdArgs &a, int t_begin, int t_end, double *rowdf_t,
-                                 uint8_t *sweep_codes, int first_lockstep, int free_max_changes, int nsm,
-                                 cudaStream_t s) {
+                                 uint8_t *sweep_codes, int first_lockstep, int free_max_changes, int flush,
+                                 int nsm, cudaStream_t s) {
     if (!a.sbar || !a.lent || !a.lcnt || a.first_sweep || t_end <= t_begin) return cudaErrorInvalidValue;
-    const int f = first_lockstep, m = free_max_changes;
+    const int f = first_lockstep, m = free_max_changes, fl = flush;
     switch (B) {
-        case 64: return launch_cd_rows_b<64>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, nsm, s);
-        case 128: return launch_cd_rows_b<128>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, nsm, s);
-        case 256: return launch_cd_rows_b<256>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, nsm, s);
+        case 64: return launch_cd_rows_b<64>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, fl, nsm, s);
+        case 128: return launch_cd_rows_b<128>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, fl, nsm, s);
+        case 256: return launch_cd_rows_b<256>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, fl, nsm, s);
         default: return cudaErrorInvalidValue;
     }
 }

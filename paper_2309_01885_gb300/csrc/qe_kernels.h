@@ -85,10 +85,12 @@ cudaError_t launch_cd_block(int B, const CdArgs &a, int nsm, cudaStream_t s);
 // sweep t and row i goes to rowdf_t[(t - t_begin) q + i]; sweep_codes (optional) gets
 // the codes after each sweep at [t][q][p].  A CTA runs a sweep in the free mode when
 // its rows made at most free_max_changes changes each (on average) in the previous
-// sweep; first_lockstep forces the lockstep mode for the first sweep.
+// sweep; first_lockstep forces the lockstep mode for the first sweep.  flush: end
+// with R the exact residual of the final codes (each block's base takes the changes
+// its last visit did not see).
 cudaError_t launch_cd_rows_lists(int B, const CdArgs &a, int t_begin, int t_end, double *rowdf_t,
-                                 uint8_t *sweep_codes, int first_lockstep, int free_max_changes, int nsm,
-                                 cudaStream_t s);
+                                 uint8_t *sweep_codes, int first_lockstep, int free_max_changes, int flush,
+                                 int nsm, cudaStream_t s);
 // obj[t] = obj[t-1] + sum_i rowdf_t[t][i] for t < nt, starting from *prev (or 0).
 cudaError_t launch_obj_prefix(const double *rowdf_t, int64_t q, int nt, const double *prev, double *out,
                               cudaStream_t s);
