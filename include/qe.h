@@ -194,11 +194,14 @@ qe_status qe_quantize_layer_outlier(const void *W, qe_dtype w_dtype, int64_t q,
  *              Caller-owned; it may be reused across calls.
  *   chunk      tokens per copy, a positive multiple of 64 (wide chunks copy
  *              faster: rows of chunk * 2 bytes are the copy's unit).
- * Chunk c is copied on an internal per-device copy stream into buffer c % nbuf
- * while earlier chunks accumulate on `stream`; a buffer is refilled only after
- * the GEMM that read it (also one of an earlier call) has finished, so the
- * copies of one call overlap work queued on `stream` before it (with nbuf >=
- * the number of chunks, all of them can arrive during that work).  The call
+ * Chunks are copied on an internal per-device copy stream into the nbuf
+ * buffers in turn, the turn carrying over from one call to the next, while
+ * earlier chunks accumulate on `stream`; a buffer is refilled only after the
+ * GEMM that read it (also one of an earlier call) has finished.  So the copies
+ * of one call overlap work queued on `stream` before it: with nbuf >= the
+ * chunks of one call they all arrive during that work, and with nbuf >= twice
+ * that (e.g. chunk = n, two buffers) consecutive calls' copies run back to
+ * back, each call's while the previous one computes.  The call
  * returns once all work is enqueued; X must stay unchanged and allocated until
  * Sigma is complete on `stream`.  Calls are serialized per device while they
  * enqueue (the copy stream and its events are shared).

@@ -17,9 +17,13 @@ constexpr int kMaxBuffers = 64;
 
 // Per-device copy stream and the events that hand the chunk buffers back and forth:
 // copied[b]: buffer b holds its chunk; freed[b]: the GEMM that read buffer b is done.
+// next: the buffer the next chunk goes to; the rotation carries over from call to
+// call, so with more buffers than chunks per call a call's copies go to buffers that
+// an earlier call's GEMMs released long before, and the copy stream never waits.
 struct CopyState {
     cudaStream_t copy = nullptr;
     int nev = 0;
+    int next = 0;
     cudaEvent_t copied[kMaxBuffers] = {};
     cudaEvent_t freed[kMaxBuffers] = {};
 };
@@ -90,9 +94,9 @@ extern "C" qe_status qe_build_sigma_host(const void *X, int64_t p, int64_t n, in
     g.ldo = p;
     g.err = err;
     const __nv_bfloat16 *Xh = static_cast<const __nv_bfloat16 *>(X);
-    int c = 0;
-    for (int64_t n0 = 0; n0 < n; n0 += chunk, ++c) {
-        const int b = c % nbuf;
+    for (int64_t n0 = 0; n0 < n; n0 += chunk) {
+        const int b = cs->next % nbuf;
+        cs->next = (b + 1) % nbuf;
         uint8_t *buf = static_cast<uint8_t *>(staging) + static_cast<size_t>(b) * buf_bytes;
         CUtensorMap ta, tb;
         if (!make_tmap_bf16(&ta, buf, p, chunk, chunk, 128) || !make_tmap_bf16(&tb, buf, p, chunk, chunk, 256))

@@ -117,6 +117,24 @@ def test_sigma_host_streamed():
     assert rel.item() < 1e-6
 
 
+def test_sigma_host_buffers_rotate_across_calls():
+    """One chunk per call and two buffers: consecutive calls copy into the buffers in
+    turn (the next call's copy overlaps this call's GEMM), with no synchronization in
+    between; each Sigma is that of its own X."""
+    p, n = 256, 4096
+    Xs = [inputs.calib_inputs(p, n, dtype=torch.bfloat16, seed=40 + k, device="cuda", heavy_frac=0.02,
+                              heavy_mult=30.0) for k in range(3)]
+    hosts = [X.cpu().pin_memory() for X in Xs]
+    staging = qe.sigma_host_staging(p, n, nbuf=2)
+    outs = [torch.empty(p, p, dtype=torch.float32, device="cuda") for _ in Xs]
+    for Xh, S in zip(hosts, outs):
+        qe.qe_build_sigma_host(Xh, S, staging, n)
+    torch.cuda.synchronize()
+    assert qe.qe_sync_status() == qe.QE_OK
+    for X, S in zip(Xs, outs):
+        assert torch.equal(S, qe.qe_build_sigma(X))
+
+
 @pytest.mark.parametrize("layout", [qe.QE_FEATURE_MAJOR, qe.QE_TOKEN_MAJOR])
 def test_sigma_fp32(layout):
     p, n = 150, 777
