@@ -262,6 +262,25 @@ qe_status qe_timer_read(qe_timer *timer, int kernel, int *launches, double *tota
 qe_status qe_timer_reset(qe_timer *timer);
 qe_status qe_timer_destroy(qe_timer *timer);
 
+/*
+ * Bit-packed codes, the storage form of a quantized layer (the paper fixes the
+ * codes as integers 0 .. 2^b - 1, Sec. 2.1, and leaves their storage open).
+ * Row i of `out` is a little-endian bit stream: code j occupies bits
+ * [j bits, (j + 1) bits), least significant bit first, of the row's
+ * ceil(p bits / 8) bytes; the padding bits of the last byte are zero.
+ *   codes  device, q x p uint8, leading dimension ldc >= p; only the low `bits`
+ *          bits of each code are stored (qe_quantize_layer's codes fit).
+ *   out    device, q rows of ldo >= ceil(p bits / 8) bytes (bytes beyond that
+ *          are not written).
+ * qe_unpack_codes is the inverse.  Both are stream-ordered; QE_ERR_INVALID_ARG
+ * for NULL pointers, q or p < 1, bits outside 1 .. 8 or a short leading
+ * dimension (before anything is enqueued); QE_ERR_CUDA when the launch fails.
+ */
+qe_status qe_pack_codes(const uint8_t *codes, int64_t q, int64_t p, int64_t ldc, int bits, uint8_t *out,
+                        int64_t ldo, qe_stream_t stream);
+qe_status qe_unpack_codes(const uint8_t *packed, int64_t q, int64_t p, int64_t ldp, int bits, uint8_t *codes,
+                          int64_t ldc, qe_stream_t stream);
+
 /* Waits for `stream`, then returns and clears the error latched on the current
  * device (QE_ERR_NUMERIC / QE_ERR_TIMEOUT), or QE_ERR_CUDA if the stream failed. */
 qe_status qe_sync_status(qe_stream_t stream);

@@ -245,3 +245,19 @@ def levels(codes, scale, zero):
     """Dequantised values s_i (c - z_i) in binary64."""
     return np.asarray(scale, np.float64)[:, None] * (np.asarray(codes, np.float64)
                                                      - np.asarray(zero, np.float64)[:, None])
+
+
+# -- storage of the codes (Sec. 2.1 fixes them as integers 0 .. 2^b - 1) ------
+def pack_codes(codes, bits: int) -> np.ndarray:
+    """Each row as a little-endian bit stream, written out from its definition: bit
+    k of code j is bit j * bits + k of the row; byte m holds bits 8m .. 8m + 7 (bit 8m
+    the least significant); the padding bits of the last byte are zero."""
+    codes = np.ascontiguousarray(codes, np.uint8)
+    q, p = codes.shape
+    bitv = (codes[:, :, None] >> np.arange(bits, dtype=np.uint8)[None, None, :]) & 1
+    nbytes = (p * bits + 7) // 8
+    stream = np.zeros((q, nbytes * 8), np.uint16)
+    stream[:, :p * bits] = bitv.reshape(q, p * bits)
+    weight = (1 << np.arange(8)).astype(np.uint16)
+    return (stream.reshape(q, nbytes, 8) * weight).sum(axis=2).astype(np.uint8)
+

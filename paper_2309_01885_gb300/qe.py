@@ -23,7 +23,7 @@ QE_FEATURE_MAJOR, QE_TOKEN_MAJOR = 0, 1
 EXPORTED = ("qe_build_sigma", "qe_quantize_layer", "qe_quantize_layer_outlier",
             "qe_workspace_size", "qe_sync_status", "qe_status_string", "qe_version",
             "qe_build_sigma_static", "qe_timer_create", "qe_timer_read", "qe_timer_reset",
-            "qe_timer_destroy", "qe_build_sigma_host")
+            "qe_timer_destroy", "qe_build_sigma_host", "qe_pack_codes", "qe_unpack_codes")
 QE_KERNEL_PINIT_GEMM, QE_KERNEL_RESIDUAL_GEMM, QE_KERNEL_TRAIL_GEMM, QE_KERNEL_CD_BLOCK, \
     QE_KERNEL_CD_LISTS, QE_KERNEL_COUNT = range(6)
 
@@ -78,6 +78,10 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     L.qe_build_sigma_static.restype = st
     L.qe_build_sigma_host.argtypes = [vp, i64, i64, i64, vp, i32, vp, ctypes.c_size_t, i64, vp]
     L.qe_build_sigma_host.restype = st
+    L.qe_pack_codes.argtypes = [vp, i64, i64, i64, i32, vp, i64, vp]
+    L.qe_pack_codes.restype = st
+    L.qe_unpack_codes.argtypes = [vp, i64, i64, i64, i32, vp, i64, vp]
+    L.qe_unpack_codes.restype = st
     L.qe_timer_create.argtypes = [ctypes.c_uint, i32, ctypes.POINTER(vp)]
     L.qe_timer_create.restype = st
     L.qe_timer_read.argtypes = [vp, i32, ctypes.POINTER(ctypes.c_int), ctypes.POINTER(ctypes.c_double)]
@@ -230,6 +234,24 @@ def _opts(block_width=0, power_iters=0, init_codes=None, sweep_codes=None, wx_no
         o.workspace = workspace.data_ptr()
         o.workspace_bytes = workspace.numel() * workspace.element_size()
     return o
+
+
+def qe_pack_codes(codes: torch.Tensor, bits: int, stream=None) -> torch.Tensor:
+    """q x p uint8 codes -> q x ceil(p bits / 8) bytes, each row a little-endian bit stream."""
+    q, p = codes.shape
+    out = torch.empty(q, (p * bits + 7) // 8, dtype=torch.uint8, device=codes.device)
+    _check(load().qe_pack_codes(_ptr(codes), q, p, _rowmajor_ld(codes), bits, _ptr(out), out.shape[1],
+                                _stream(stream)), "qe_pack_codes")
+    return out
+
+
+def qe_unpack_codes(packed: torch.Tensor, p: int, bits: int, stream=None) -> torch.Tensor:
+    """The inverse of qe_pack_codes: q x p uint8 codes."""
+    q = packed.shape[0]
+    codes = torch.empty(q, p, dtype=torch.uint8, device=packed.device)
+    _check(load().qe_unpack_codes(_ptr(packed), q, p, _rowmajor_ld(packed), bits, _ptr(codes), p,
+                                  _stream(stream)), "qe_unpack_codes")
+    return codes
 
 
 def qe_quantize_layer(W: torch.Tensor, Sigma: torch.Tensor, bits: int, iters: int, *,

@@ -128,6 +128,18 @@ def test_sigma_host_rejects_bad_arguments(lib):
                                  None) == qe.QE_ERR_INVALID_ARG
 
 
+def test_pack_codes_rejects_bad_arguments(lib):
+    L = lib
+    for fn in (L.qe_pack_codes, L.qe_unpack_codes):
+        # bits outside 1 .. 8, a stream row shorter than ceil(p bits / 8), ldc < p, NULL, p < 1
+        assert fn(_fake(), 4, 10, 10, 0, _fake(2), 10, None) == qe.QE_ERR_INVALID_ARG
+        assert fn(_fake(), 4, 10, 10, 9, _fake(2), 10, None) == qe.QE_ERR_INVALID_ARG
+        assert fn(_fake(), 4, 10, 10, 3, _fake(2), 3, None) == qe.QE_ERR_INVALID_ARG
+        assert fn(_fake(), 4, 10, 9, 3, _fake(2), 4, None) == qe.QE_ERR_INVALID_ARG
+        assert fn(None, 4, 10, 10, 3, _fake(2), 4, None) == qe.QE_ERR_INVALID_ARG
+        assert fn(_fake(), 4, 0, 10, 3, _fake(2), 4, None) == qe.QE_ERR_INVALID_ARG
+
+
 def test_workspace_size_grows_with_shape(lib):
     a = qe.qe_workspace_size(256, 256)
     b = qe.qe_workspace_size(512, 1024)

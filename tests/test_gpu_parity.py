@@ -316,6 +316,23 @@ def test_layer_relax_period_not_below_iters_is_plain():
     assert torch.equal(r["obj"], out["obj"])
 
 
+@pytest.mark.parametrize("bits", [1, 2, 3, 4, 5, 7, 8])
+def test_pack_codes_bit_exact(bits):
+    """Packed codes equal the oracle's bit stream byte for byte (ragged rows: p = 1001),
+    and unpacking gives the codes back; also for the codes of a quantized layer."""
+    q, p = 37, 1001
+    g = torch.Generator(device="cuda").manual_seed(bits)
+    codes = torch.randint(0, 2 ** bits, (q, p), dtype=torch.uint8, device="cuda", generator=g)
+    packed = qe.qe_pack_codes(codes, bits)
+    assert np.array_equal(packed.cpu().numpy(), oracle.pack_codes(codes.cpu().numpy(), bits))
+    assert torch.equal(qe.qe_unpack_codes(packed, p, bits), codes)
+    if bits in (2, 3, 4):
+        W, X, Sg, out = _layer_case(64, 300, 1024, torch.bfloat16, bits, 2, seed=66)
+        pk = qe.qe_pack_codes(out["codes"], bits)
+        assert np.array_equal(pk.cpu().numpy(), oracle.pack_codes(out["codes"].cpu().numpy(), bits))
+        assert torch.equal(qe.qe_unpack_codes(pk, 300, bits), out["codes"])
+
+
 def test_layer_dead_columns_round_to_nearest():
     dead = (5, 77, 130)
     W, X, Sg, out = _layer_case(96, 160, 1024, torch.float32, 4, 3, seed=12, zero_rows=dead)

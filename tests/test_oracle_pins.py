@@ -510,3 +510,31 @@ def test_structured_outlier_below_one_column_reduces_to_algorithm1():
     a1 = O.alg1(W, S, s, z, 3, iters=4)
     assert np.array_equal(r["codes"], a1["codes"]) and not np.any(r["H"])
     assert np.allclose(r["obj"], a1["obj"], rtol=1e-12)
+
+
+# --------------------------------------------------------------------------
+# bit-packed storage of the codes (integers 0 .. 2^b - 1, Sec. 2.1)
+# --------------------------------------------------------------------------
+def test_pack_codes_hand_example():
+    """3-bit codes 5, 3, 7, 1 -> bit stream 101 110 111 100 (each code least significant
+    bit first) = bytes 0b11011101 = 221 and 0b0011 = 3 (zero padding)."""
+    assert oracle.pack_codes(np.array([[5, 3, 7, 1]]), 3).tolist() == [[221, 3]]
+    # 8 bits: the codes themselves; 1 bit: eight codes per byte
+    c = np.array([[0, 255, 17, 128]], np.uint8)
+    assert np.array_equal(oracle.pack_codes(c, 8), c)
+    assert oracle.pack_codes(np.array([[1, 0, 1, 1, 0, 0, 0, 1, 1]]), 1).tolist() == [[0b10001101, 1]]
+
+
+@pytest.mark.parametrize("bits", [1, 2, 3, 4, 5, 7, 8])
+def test_pack_codes_matches_packbits_and_unpacks(bits):
+    rng = np.random.default_rng(bits)
+    codes = rng.integers(0, 2 ** bits, size=(7, 101), dtype=np.uint8)
+    packed = oracle.pack_codes(codes, bits)
+    assert packed.shape == (7, (101 * bits + 7) // 8)
+    # numpy's own little-endian bit packing of the same stream
+    stream = np.unpackbits(codes[:, :, None], axis=2, bitorder="little")[:, :, :bits].reshape(7, -1)
+    assert np.array_equal(packed, np.packbits(stream, axis=1, bitorder="little"))
+    # read back code j from bits j * bits .. j * bits + bits - 1
+    bitsarr = np.unpackbits(packed, axis=1, bitorder="little")
+    back = sum(bitsarr[:, k::bits][:, :101].astype(np.int64) << k for k in range(bits))
+    assert np.array_equal(back, codes)
