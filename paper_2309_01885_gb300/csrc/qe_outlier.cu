@@ -361,35 +361,77 @@ __global__ void k_rowptr(const int64_t *H_idx, const int64_t *nnz, int64_t q, in
     rowptr[i] = lo;
 }
 
+// Close this thread's current group of cp.async copies / wait until at most N of
+// its committed groups are still in flight (the copies always complete).
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait_group() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+// 4 bytes global -> shared (the columns of a piece cut by p).
+__device__ __forceinline__ void cp_async4(void *dst, const void *src) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(dst)),
+                 "l"(static_cast<unsigned long long>(__cvta_generic_to_global(src)))
+                 : "memory");
+}
+
 // P_new = P_W - H (I + Sigma_bar) for row i; R += (P_new - P_old) / s_i when
 // update_r (R in grid-step units); P = P_new.  Sigma_bar comes as fp32 rows
 // (sbar[k][j] = Sigma_jk / d_j, zero on the diagonal and for dead columns: the
 // binary32 values the tensor-core planes split), so the identity adds 1 at
-// j = k.  One CTA per (row, tile of kSpmmCols columns); each thread keeps
-// kSpmmPer columns in registers.  The row's kept entries are staged in shared
-// memory kSpmmChunk at a time, and the rows of kSpmmU entries are in flight
-// together, so no index load sits in the gather chain; the entries are still
-// added one after another in their sorted order.
-constexpr int kSpmmPer = 16;
-constexpr int kSpmmCols = 256 * kSpmmPer;
+// j = k.  One CTA per (row, tile of kSpmmCols columns); thread t owns
+// kSpmmPieces pieces of 4 columns, piece u at u * 4 * kSpmmThreads + 4 t (so a
+// warp's piece is 512 contiguous bytes: coalesced, and free of shared-memory
+// bank conflicts).  The row's kept entries are staged in shared memory
+// kSpmmChunk at a time; each thread copies its own pieces of the next
+// kSpmmDepth - 1 entries' Sigma_bar rows into a ring in shared memory by
+// cp.async (many rows in flight without registers, no thread waits for
+// another) and adds the entries one after another in their sorted order.
+// Rows are 16-byte aligned (ld, lds multiples of 4); a piece cut by p goes
+// column by column.
+constexpr int kSpmmThreads = 256;
+constexpr int kSpmmPieces = 4;
+constexpr int kSpmmPer = 4 * kSpmmPieces;
+constexpr int kSpmmCols = kSpmmThreads * kSpmmPer;
 constexpr int kSpmmChunk = 256;
-constexpr int kSpmmU = 2;
+constexpr int kSpmmDepth = 4;
+constexpr int kSpmmSmem = kSpmmDepth * kSpmmCols * 4;
 
-__global__ void __launch_bounds__(256) k_spmm_refresh(const float *PW, float *P, float *R, int64_t ld,
-                                                      const float *sbar, int64_t lds, const int64_t *H_idx,
-                                                      const float *H_val, const int64_t *rowptr, int64_t p,
-                                                      int update_r, const float *scale) {
+__global__ void __launch_bounds__(kSpmmThreads) k_spmm_refresh(const float *PW, float *P, float *R, int64_t ld,
+                                                               const float *sbar, int64_t lds,
+                                                               const int64_t *H_idx, const float *H_val,
+                                                               const int64_t *rowptr, int64_t p, int update_r,
+                                                               const float *scale) {
     __shared__ int sk[kSpmmChunk];
     __shared__ float sv[kSpmmChunk];
+    extern __shared__ __align__(16) float ring[];   // [kSpmmDepth][kSpmmPieces][kSpmmThreads][4]
     const int64_t i = blockIdx.x;
-    const int64_t j0 = static_cast<int64_t>(blockIdx.y) * kSpmmCols + threadIdx.x;
+    const int64_t j0 = static_cast<int64_t>(blockIdx.y) * kSpmmCols + 4 * threadIdx.x;
+    int ncol[kSpmmPieces];   // columns of piece u inside the layer (0 .. 4)
+#pragma unroll
+    for (int u = 0; u < kSpmmPieces; ++u) {
+        const int64_t j = j0 + u * 4 * kSpmmThreads;
+        ncol[u] = j >= p ? 0 : static_cast<int>((p - j) < 4 ? (p - j) : 4);
+    }
     const int64_t e0 = rowptr[i], e1 = rowptr[i + 1];
     float acc[kSpmmPer];
 #pragma unroll
-    for (int u = 0; u < kSpmmPer; ++u) {
-        const int64_t j = j0 + 256 * u;
-        acc[u] = j < p ? __ldcs(PW + i * ld + j) : 0.0f;   // streamed: keep L2 for Sigma_bar's rows
+    for (int u = 0; u < kSpmmPieces; ++u) {
+        const int64_t j = j0 + u * 4 * kSpmmThreads;
+        float4 v = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+        if (ncol[u] == 4) {
+            v = __ldcs(reinterpret_cast<const float4 *>(PW + i * ld + j));   // streamed
+        } else {
+            if (ncol[u] > 0) v.x = __ldcs(PW + i * ld + j);
+            if (ncol[u] > 1) v.y = __ldcs(PW + i * ld + j + 1);
+            if (ncol[u] > 2) v.z = __ldcs(PW + i * ld + j + 2);
+        }
+        acc[4 * u] = v.x;
+        acc[4 * u + 1] = v.y;
+        acc[4 * u + 2] = v.z;
+        acc[4 * u + 3] = v.w;
     }
+    float *mine = ring + 4 * threadIdx.x;
     for (int64_t c0 = e0; c0 < e1; c0 += kSpmmChunk) {
         const int n = static_cast<int>((e1 - c0) < kSpmmChunk ? (e1 - c0) : kSpmmChunk);
         __syncthreads();   // the previous chunk is consumed
@@ -398,48 +440,75 @@ __global__ void __launch_bounds__(256) k_spmm_refresh(const float *PW, float *P,
             sv[threadIdx.x] = H_val[c0 + threadIdx.x];
         }
         __syncthreads();
-        int e = 0;
-        for (; e + kSpmmU <= n; e += kSpmmU) {
-            int k[kSpmmU];
-            float v[kSpmmU][kSpmmPer];
+        // entry e goes to slot e % kSpmmDepth; one commit group per entry (empty past n)
+        auto issue = [&](int e) {
+            if (e < n) {
+                const float *src = sbar + static_cast<int64_t>(sk[e]) * lds + j0;
+                float *dst = mine + (e % kSpmmDepth) * kSpmmCols;
 #pragma unroll
-            for (int x = 0; x < kSpmmU; ++x) {
-                k[x] = sk[e + x];
-                const float *srow = sbar + static_cast<int64_t>(k[x]) * lds;
+                for (int u = 0; u < kSpmmPieces; ++u) {
+                    const int off = u * 4 * kSpmmThreads;
+                    if (ncol[u] == 4) {
+                        cp_async16(dst + off, src + off);
+                    } else {
 #pragma unroll
-                for (int u = 0; u < kSpmmPer; ++u) {
-                    const int64_t j = j0 + 256 * u;
-                    v[x][u] = j < p ? __ldg(srow + j) : 0.0f;
+                        for (int x = 0; x < 3; ++x)
+                            if (x < ncol[u]) cp_async4(dst + off + x, src + off + x);
+                    }
                 }
             }
+            cp_async_commit();
+        };
 #pragma unroll
-            for (int x = 0; x < kSpmmU; ++x) {
-                const float hv = sv[e + x];
-#pragma unroll
-                for (int u = 0; u < kSpmmPer; ++u) {
-                    const int64_t j = j0 + 256 * u;
-                    acc[u] = fmaf(-hv, (j == k[x]) ? 1.0f : v[x][u], acc[u]);
-                }
-            }
-        }
-        for (; e < n; ++e) {
-            const int kk = sk[e];
+        for (int e = 0; e < kSpmmDepth - 1; ++e) issue(e);
+        for (int e = 0; e < n; ++e) {
+            issue(e + kSpmmDepth - 1);
+            cp_async_wait_group<kSpmmDepth - 1>();   // entry e has landed
+            const int k = sk[e];
             const float hv = sv[e];
-            const float *srow = sbar + static_cast<int64_t>(kk) * lds;
+            const float *seg = mine + (e % kSpmmDepth) * kSpmmCols;
 #pragma unroll
-            for (int u = 0; u < kSpmmPer; ++u) {
-                const int64_t j = j0 + 256 * u;
-                if (j < p) acc[u] = fmaf(-hv, (j == kk) ? 1.0f : __ldg(srow + j), acc[u]);
+            for (int u = 0; u < kSpmmPieces; ++u) {
+                const int off = u * 4 * kSpmmThreads;
+                const float4 v = *reinterpret_cast<const float4 *>(seg + off);
+                const float w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+                for (int x = 0; x < 4; ++x) {
+                    if (x >= ncol[u]) break;
+                    const int64_t j = j0 + off + x;
+                    acc[4 * u + x] = fmaf(-hv, (j == k) ? 1.0f : w[x], acc[4 * u + x]);
+                }
             }
         }
+        cp_async_wait_group<0>();
     }
     const float s = update_r ? scale[i] : 1.0f;
 #pragma unroll
-    for (int u = 0; u < kSpmmPer; ++u) {
-        const int64_t j = j0 + 256 * u;
-        if (j >= p) continue;
-        if (update_r) __stcs(R + i * ld + j, __ldcs(R + i * ld + j) + __fdiv_rn(acc[u] - __ldcs(P + i * ld + j), s));
-        __stcs(P + i * ld + j, acc[u]);
+    for (int u = 0; u < kSpmmPieces; ++u) {
+        const int64_t j = j0 + u * 4 * kSpmmThreads;
+        if (ncol[u] == 4) {
+            float4 *pp = reinterpret_cast<float4 *>(P + i * ld + j);
+            const float4 pn = make_float4(acc[4 * u], acc[4 * u + 1], acc[4 * u + 2], acc[4 * u + 3]);
+            if (update_r) {
+                float4 *rp = reinterpret_cast<float4 *>(R + i * ld + j);
+                const float4 po = __ldcs(pp);
+                float4 r = __ldcs(rp);
+                r.x += __fdiv_rn(pn.x - po.x, s);
+                r.y += __fdiv_rn(pn.y - po.y, s);
+                r.z += __fdiv_rn(pn.z - po.z, s);
+                r.w += __fdiv_rn(pn.w - po.w, s);
+                __stcs(rp, r);
+            }
+            __stcs(pp, pn);
+        } else {
+#pragma unroll
+            for (int x = 0; x < 3; ++x) {
+                if (x >= ncol[u]) break;
+                float *pp = P + i * ld + j + x;
+                if (update_r) __stcs(R + i * ld + j + x, __ldcs(R + i * ld + j + x) + __fdiv_rn(acc[4 * u + x] - __ldcs(pp), s));
+                __stcs(pp, acc[4 * u + x]);
+            }
+        }
     }
 }
 
@@ -543,8 +612,12 @@ cudaError_t launch_scatter_rowptr(const int64_t *H_idx, const float *H_val, cons
 cudaError_t launch_spmm_refresh(const float *PW, float *P, float *R, int64_t ld, const float *sbar,
                                 int64_t lds, const int64_t *H_idx, const float *H_val, const int64_t *rowptr,
                                 int64_t q, int64_t p, int update_r, const float *scale, cudaStream_t s) {
+    if (ld % 4 != 0 || lds % 4 != 0) return cudaErrorInvalidValue;
+    cudaError_t e = cudaFuncSetAttribute(k_spmm_refresh, cudaFuncAttributeMaxDynamicSharedMemorySize, kSpmmSmem);
+    if (e != cudaSuccess) return e;
     const dim3 grid(static_cast<unsigned>(q), static_cast<unsigned>(ceil_div(p, kSpmmCols)));
-    k_spmm_refresh<<<grid, 256, 0, s>>>(PW, P, R, ld, sbar, lds, H_idx, H_val, rowptr, p, update_r, scale);
+    k_spmm_refresh<<<grid, kSpmmThreads, kSpmmSmem, s>>>(PW, P, R, ld, sbar, lds, H_idx, H_val, rowptr, p,
+                                                         update_r, scale);
     return cudaGetLastError();
 }
 

@@ -406,7 +406,8 @@ def test_nonfinite_input_is_reported():
 # ---------------------------------------------------------------------------
 # qe_quantize_layer_outlier
 # ---------------------------------------------------------------------------
-@pytest.mark.parametrize("q,p,bits,frac", [(96, 192, 3, 0.01), (130, 260, 2, 0.02)])
+@pytest.mark.parametrize("q,p,bits,frac", [(96, 192, 3, 0.01), (130, 260, 2, 0.02), (70, 203, 3, 0.01),
+                                         (8, 4200, 3, 0.01)])
 def test_outlier_parity_small(q, p, bits, frac):
     iters, power_iters = 4, 200
     W = inputs.layer_weights(q, p, dtype=torch.bfloat16, seed=41, device="cuda", planted_frac=frac,
