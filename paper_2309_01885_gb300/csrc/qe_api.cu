@@ -62,7 +62,7 @@ struct Plan {
            rowdf = 0, objbase = 0, sbar = 0, lcnt = 0, lent = 0, rowdft = 0;
     int64_t nblk = 0;
     size_t PW = 0, H = 0, T = 0, st = 0, cg = 0, ce = 0, sb = 0, eb = 0, y0 = 0, y1 = 0, lam = 0,
-           eta = 0, rowptr = 0, cpart = 0, cnorm = 0, ccols = 0, cval = 0, cn = 0;
+           eta = 0, rowptr = 0, cpart = 0, cnorm = 0, ccols = 0, cval = 0, cn = 0, ppart = 0;
     size_t total = 0;
 };
 
@@ -120,6 +120,7 @@ static Plan make_plan(int64_t q, int64_t p, int B, bool outlier, int wpl_planes,
         pl.y0 = take(cur, p * 4);
         pl.y1 = take(cur, p * 4);
         pl.lam = take(cur, 8);
+        pl.ppart = take(cur, 2 * kPowerMaxBlocks * 8);
         pl.eta = take(cur, 8);
         pl.rowptr = take(cur, (q + 1) * 8);
         // structured outliers: column norms and the kept columns
@@ -185,7 +186,7 @@ struct Ctx {
     float *PW = nullptr, *H = nullptr, *T = nullptr, *y0 = nullptr, *y1 = nullptr;
     TopkState *st = nullptr;
     unsigned *cg = nullptr, *ce = nullptr, *sb = nullptr, *eb = nullptr;
-    double *lam = nullptr, *eta = nullptr;
+    double *lam = nullptr, *eta = nullptr, *ppart = nullptr;
     int64_t *rowptr = nullptr;
     double *cpart = nullptr;
     float *cnorm = nullptr, *cval = nullptr;
@@ -254,6 +255,7 @@ static qe_status setup_ctx(Ctx &c, const Plan &pl, const qe_opts *o, cudaStream_
         c.y0 = at<float>(w, pl.y0);
         c.y1 = at<float>(w, pl.y1);
         c.lam = at<double>(w, pl.lam);
+        c.ppart = at<double>(w, pl.ppart);
         c.eta = at<double>(w, pl.eta);
         c.rowptr = at<int64_t>(w, pl.rowptr);
         c.cpart = at<double>(w, pl.cpart);
@@ -891,7 +893,7 @@ qe_status qe_quantize_layer_outlier(const void *W, qe_dtype w_dtype, int64_t q, 
     QE_CK(launch_grid(W, wbf16, ldw, c.H, ld, q, p, bits, scales, zeros, c.err, c.s));
     // P_W = W (I + Sigma_bar), eta = 1 / (2 lambda_max), P = P_W - H (I + Sigma_bar)
     if ((st = prepare(c, W, wbf16, ldw, Sigma, c.PW)) != QE_OK) return st;
-    QE_CK(launch_power_lambda(Sigma, p, p, power_iters, c.y0, c.y1, c.lam, c.eta, c.nsm, c.s));
+    QE_CK(launch_power_lambda(Sigma, p, p, power_iters, c.y0, c.y1, c.ppart, c.lam, c.eta, c.nsm, c.s));
     QE_CK(launch_spmm_refresh(c.PW, c.P, c.R, ld, c.sbar, ld, H_idx, H_val, c.rowptr, q, p, 0, scales,
                               c.s));
     if (opts && opts->wx_norm2)

@@ -49,20 +49,30 @@ __device__ __forceinline__ unsigned block_excl_scan(unsigned v, unsigned *sh, un
 }
 
 // ---- power method (Sec. 4.3: lambda_max(X X^T) "by iterative power method") --
-// y_out = Sigma (y_in / ||y_in||); every CTA recomputes ||y_in||.  One warp per
-// row of Sigma; eight independent partial sums keep eight loads in flight per
-// lane (a dependent chain of single loads made this step latency-bound), and
-// 16-byte loads are used when the rows are 16-byte aligned.
+// y_out = Sigma (y_in / ||y_in||).  ||y_in||^2 is the sum of the per-CTA
+// partials the previous step left in part_in (nparts of them, added in a fixed
+// order, so the result is reproducible), or is computed here when part_in is
+// NULL (the first step); each CTA leaves the sum of the squares of the y_out
+// values it wrote in part_out[blockIdx.x].  One warp per row of Sigma; eight
+// independent partial sums keep eight loads in flight per lane (a dependent
+// chain of single loads made this step latency-bound), and 16-byte loads are
+// used when the rows are 16-byte aligned.
 __global__ void __launch_bounds__(256) k_power_step(const float *S, int64_t lds, int64_t p,
-                                                    const float *y_in, float *y_out) {
+                                                    const float *y_in, const double *part_in, int nparts,
+                                                    float *y_out, double *part_out) {
     __shared__ double sh[8];
     double n2 = 0.0;
-    for (int64_t k = threadIdx.x; k < p; k += blockDim.x) n2 += (double)y_in[k] * y_in[k];
+    if (part_in) {
+        for (int k = threadIdx.x; k < nparts; k += blockDim.x) n2 += part_in[k];
+    } else {
+        for (int64_t k = threadIdx.x; k < p; k += blockDim.x) n2 += (double)y_in[k] * y_in[k];
+    }
     n2 = block_sum(n2, sh);
     const float inv = n2 > 0.0 ? static_cast<float>(1.0 / sqrt(n2)) : 0.0f;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const bool vec = (lds % 4 == 0) && ((reinterpret_cast<uintptr_t>(S) & 15u) == 0) &&
                      ((reinterpret_cast<uintptr_t>(y_in) & 15u) == 0);
+    double own2 = 0.0;
     for (int64_t a = (int64_t)blockIdx.x * 8 + warp; a < p; a += (int64_t)gridDim.x * 8) {
         const float *row = S + a * lds;
         float acc[8];
@@ -93,11 +103,16 @@ __global__ void __launch_bounds__(256) k_power_step(const float *S, int64_t lds,
         float t = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
-        if (lane == 0) y_out[a] = t * inv;
+        if (lane == 0) {
+            const float ya = t * inv;
+            y_out[a] = ya;
+            own2 += (double)ya * ya;
+        }
     }
+    own2 = block_sum(own2, sh);
+    if (threadIdx.x == 0) part_out[blockIdx.x] = own2;
 }
 
-// lambda = (y/||y||) . z with z = Sigma (y/||y||); eta = 1 / (2 lambda).
 __global__ void __launch_bounds__(256) k_power_final(const float *y, const float *z, int64_t p,
                                                      double *lam, double *eta) {
     __shared__ double sh[8];
@@ -526,17 +541,23 @@ static inline dim3 rows_grid(int64_t rows, int64_t cols) {
 }
 
 cudaError_t launch_power_lambda(const float *S, int64_t lds, int64_t p, int iters, float *y0, float *y1,
-                                double *lam, double *eta, int nsm, cudaStream_t s) {
+                                double *part, double *lam, double *eta, int nsm, cudaStream_t s) {
     k_fill<<<static_cast<unsigned>(ceil_div(p, 256)), 256, 0, s>>>(y0, p, 1.0f);
     int64_t blocks = ceil_div(p, 8);
     if (blocks > nsm * 4) blocks = nsm * 4;
+    if (blocks > kPowerMaxBlocks) blocks = kPowerMaxBlocks;
     float *a = y0, *b = y1;
+    const double *pin = nullptr;
+    double *pout = part;
     for (int it = 0; it <= iters; ++it) {
-        k_power_step<<<static_cast<unsigned>(blocks), 256, 0, s>>>(S, lds, p, a, b);
+        k_power_step<<<static_cast<unsigned>(blocks), 256, 0, s>>>(S, lds, p, a, pin, static_cast<int>(blocks), b,
+                                                                   pout);
         if (it < iters) {
             float *t = a;
             a = b;
             b = t;
+            pin = pout;
+            pout = (pout == part) ? part + kPowerMaxBlocks : part;
         }
     }
     // a = y_iters, b = Sigma (y_iters / ||y_iters||)

@@ -18,8 +18,10 @@ struct TopkState {
     unsigned pad;
 };
 
+// part: 2 * kPowerMaxBlocks doubles (the per-CTA partial norms carried between steps).
+constexpr int kPowerMaxBlocks = 1024;
 cudaError_t launch_power_lambda(const float *S, int64_t lds, int64_t p, int iters, float *y0, float *y1,
-                                double *lam, double *eta, int nsm, cudaStream_t s);
+                                double *part, double *lam, double *eta, int nsm, cudaStream_t s);
 cudaError_t launch_iht_target(const float *H, const float *R, int64_t ld, const uint8_t *codes,
                               int64_t ldc, const float *scale, const float *zero, const float *d,
                               const double *eta, int64_t q, int64_t p, float *T, cudaStream_t s);
