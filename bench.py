@@ -234,18 +234,23 @@ def roofline_lists(bytes_per_launch, ms, launches, pk):
             "peak_source": f"{pk['source']} HBM copy bandwidth (MEASURED_PEAKS.json)"}
 
 
-def cpu_oracle_sample(W64, S64, bits, rows, sweeps):
-    """Time Algorithm 1 of the fp64 oracle on a row sample; returns (units/s, seconds, threads)."""
+def cpu_oracle_sample(W64, S64, bits, rows, sweeps, threads=0):
+    """Time Algorithm 1 of the fp64 oracle on a row sample (on `threads` host threads,
+    0 = all); returns (units/s, seconds, threads used)."""
     import numpy as np
     import oracle
     O = oracle.get()
     s, z = O.grid(W64[:rows], bits)
-    t0 = time.perf_counter()
-    O.alg1(np.ascontiguousarray(W64[:rows]), S64, s, z, bits, sweeps)
-    dt = time.perf_counter() - t0
+    old = O.threads(threads)
+    used = O.threads(0)
+    try:
+        t0 = time.perf_counter()
+        O.alg1(np.ascontiguousarray(W64[:rows]), S64, s, z, bits, sweeps)
+        dt = time.perf_counter() - t0
+    finally:
+        O.threads(old)
     p = W64.shape[1]
-    threads = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
-    return rows * p * p * sweeps / dt, dt, threads
+    return rows * p * p * sweeps / dt, dt, used
 
 
 def run_reference(args):
@@ -277,7 +282,7 @@ def run_reference(args):
     units = rows * cfg.p * cfg.p * len(cfg.bits)
     ms = 1e3 * sum(times) / len(times)
     value = units / (ms / 1e3)
-    threads = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    threads = O.threads(0)   # the OpenMP threads the oracle's row loops use
     sample = (f"Algorithm 1 (fp64 oracle) on {rows} of {cfg.q} rows, 1 sweep per bit-width "
               f"{list(cfg.bits)}, p={cfg.p}, Sigma from {n_ref} tokens; rows are independent given Sigma")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
@@ -442,6 +447,17 @@ def main():
     gemm_exec = (gemm_tiles_sigma(p) * 2 * 128 * 256 * n
                  + nb * ((1 + refreshes) * 3 * 2 * qpad * ppad * (-(-p // 64) * 64) + trail_exec))
     result["roofline"] = roofline_gemm(gemm_flops, gemm_exec, gemm_ms, gemm_launches, pk)
+    # ideal step: per phase max(algorithmic flops / tensor peak, algorithmic bytes / HBM), summed
+    peak_tf, hbm = pk["bf16_sustained"] * 1e12, pk["hbm"] * 1e9
+    cd_flops, cd_bytes = 2.0 * q * p * p * cfg.iters, 15.0 * q * p * cfg.iters   # ~15 B per coordinate per sweep
+    ideal_s = (max(sig_flops / peak_tf, 2.0 * p * n / hbm)
+               + nb * (max(2.0 * q * p * p * (1 + refreshes) / peak_tf, 12.0 * q * p * (1 + refreshes) / hbm)
+                       + max(cd_flops / peak_tf, cd_bytes / hbm)))
+    result["ideal"] = {"ms_per_step": ideal_s * 1e3, "frac": ideal_s * 1e3 / ms,
+                       "model": ("per phase max(algorithmic flops / measured sustained bf16, algorithmic bytes / "
+                                 "measured HBM): Sigma p(p+1)n flops vs X read once; per layer P and residual "
+                                 "refreshes 2qp^2 flops each; CD 2qp^2 flops per sweep vs ~15 bytes per "
+                                 "coordinate per sweep")}
     # the persistent change-list kernel: one launch per layer (per 32 list sweeps)
     list_launches, list_ms = timed[qe.QE_KERNEL_CD_LISTS]
     n_list = sum(1 for kind, _ in plan if kind == "list")
@@ -559,11 +575,15 @@ def main():
         S64 = Sigma.double().cpu().numpy()
         rows = max(1, min(q, args.cpu_rows))
         rate, dt, threads = cpu_oracle_sample(W64, S64, cfg.bits[0], rows, 1)
+        rows1 = max(1, rows // 16)
+        rate1, dt1, _ = cpu_oracle_sample(W64, S64, cfg.bits[0], rows1, 1, threads=1)
         result["cpu_baseline"] = {
             "value": rate, "unit": "q·p² column-updates/s (CD only)", "cores": threads,
             "kind": "oracle",
             "sample": (f"Algorithm 1 (fp64 oracle) on {rows} of {q} rows x 1 sweep, {cfg.bits[0]}-bit, "
-                       f"given this layer's Sigma; {dt:.1f} s")}
+                       f"given this layer's Sigma; {dt:.1f} s"),
+            "single_core": {"value": rate1, "cores": 1,
+                            "sample": f"the same on {rows1} rows and one host thread; {dt1:.1f} s"}}
         result["obj_last"] = {str(b): float(o["obj"][-1].item()) for b, o in zip(cfg.bits, outs)}
 
     if rank == 0:

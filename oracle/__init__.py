@@ -77,6 +77,8 @@ class Oracle:
         lib.qo_quantease_alg3.argtypes = [_f64p, _i64, _i64, _f64p, _f32p, _f32p, _int, _int,
                                           _u8p, _f64p, _int]
         lib.qo_quantease_alg3.restype = _int
+        lib.qo_threads.argtypes = [_int]
+        lib.qo_threads.restype = _int
         lib.qo_power_lambda.argtypes = [_f64p, _i64, _int]
         lib.qo_power_lambda.restype = ctypes.c_double
         lib.qo_topk.argtypes = [_f64p, _i64, _i64, _i64p]
@@ -139,6 +141,11 @@ class Oracle:
                                    _ptr(np.ascontiguousarray(zero, np.float32), _f32p),
                                    q, p, _ptr(_f64(S), _f64p), _ptr(out, _f64p))
         return out
+
+    def threads(self, n: int = 0) -> int:
+        """Host threads of the row loops (timing only): n > 0 sets them; returns the
+        count in effect before the call."""
+        return int(self.lib.qo_threads(n))
 
     # -- Algorithm 1 / 3 ----------------------------------------------------
     def alg1(self, W, S, scale, zero, bits, iters, init_codes=None, forced=None,

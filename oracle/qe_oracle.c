@@ -25,6 +25,24 @@
 #include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+/* Host threads of the OpenMP row loops (for timing only): n > 0 sets the count;
+ * returns the count in effect before the call. */
+int qo_threads(int n)
+{
+#ifdef _OPENMP
+    const int old = omp_get_max_threads();
+    if (n > 0)
+        omp_set_num_threads(n);
+    return old;
+#else
+    (void)n;
+    return 1;
+#endif
+}
 
 /* ------------------------------------------------------------------------- */
 /* Quantization grid and operator                                            */
