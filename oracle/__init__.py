@@ -59,6 +59,16 @@ class Oracle:
         lib = ctypes.CDLL(self.path)
         lib.qo_grid.argtypes = [_f64p, _i64, _i64, _int, _u8p, _f32p, _f32p]
         lib.qo_grid.restype = None
+        lib.qo_grid_groups.argtypes = [_f64p, _i64, _i64, _i64, _int, _u8p, _f32p, _f32p]
+        lib.qo_grid_groups.restype = None
+        lib.qo_rtn_groups.argtypes = [_f64p, _i64, _i64, _i64, _f32p, _f32p, _int, _u8p]
+        lib.qo_rtn_groups.restype = None
+        lib.qo_objective_rows_groups.argtypes = [_f64p, _f64p, _u8p, _f32p, _f32p, _i64, _i64, _i64, _f64p,
+                                                 _f64p]
+        lib.qo_objective_rows_groups.restype = None
+        lib.qo_quantease_alg1_groups.argtypes = [_f64p, _i64, _i64, _f64p, _i64, _f32p, _f32p, _int, _int,
+                                                 _u8p, _u8p, _u8p, _f64p, _u8p, _f64p, _int]
+        lib.qo_quantease_alg1_groups.restype = _int
         lib.qo_rtn.argtypes = [_f64p, _i64, _i64, _f32p, _f32p, _int, _u8p]
         lib.qo_rtn.restype = None
         lib.qo_sigma.argtypes = [_f64p, _i64, _i64, _f64p]
@@ -91,23 +101,32 @@ class Oracle:
         self.lib = lib
 
     # -- grid ---------------------------------------------------------------
-    def grid(self, W, bits, excl=None):
-        """Per-row (scale, zero) of the asymmetric min/max grid (binary32)."""
+    def grid(self, W, bits, excl=None, group_size=0):
+        """(scale, zero) of the asymmetric min/max grid (binary32): per row, or with
+        group_size > 0 per row and group of group_size columns (arrays q x groups)."""
         W = _f64(W)
         q, p = W.shape
+        ex = None if excl is None else np.ascontiguousarray(excl, dtype=np.uint8)
+        if group_size:
+            ng = -(-p // group_size)
+            scale = np.empty((q, ng), np.float32)
+            zero = np.empty((q, ng), np.float32)
+            self.lib.qo_grid_groups(_ptr(W, _f64p), q, p, group_size, bits, _ptr(ex, _u8p),
+                                    _ptr(scale, _f32p), _ptr(zero, _f32p))
+            return scale, zero
         scale = np.empty(q, np.float32)
         zero = np.empty(q, np.float32)
-        ex = None if excl is None else np.ascontiguousarray(excl, dtype=np.uint8)
         self.lib.qo_grid(_ptr(W, _f64p), q, p, bits, _ptr(ex, _u8p),
                          _ptr(scale, _f32p), _ptr(zero, _f32p))
         return scale, zero
 
-    def rtn(self, W, scale, zero, bits):
+    def rtn(self, W, scale, zero, bits, group_size=0):
         W = _f64(W)
         q, p = W.shape
         codes = np.empty((q, p), np.uint8)
-        self.lib.qo_rtn(_ptr(W, _f64p), q, p, _ptr(np.ascontiguousarray(scale, np.float32), _f32p),
-                        _ptr(np.ascontiguousarray(zero, np.float32), _f32p), bits, _ptr(codes, _u8p))
+        self.lib.qo_rtn_groups(_ptr(W, _f64p), q, p, group_size or p,
+                               _ptr(np.ascontiguousarray(scale, np.float32), _f32p),
+                               _ptr(np.ascontiguousarray(zero, np.float32), _f32p), bits, _ptr(codes, _u8p))
         return codes
 
     # -- Sigma / objective --------------------------------------------------
@@ -130,16 +149,16 @@ class Oracle:
                                      _ptr(out, _f64p))
         return out
 
-    def objective_rows(self, W, codes, scale, zero, S, H=None):
+    def objective_rows(self, W, codes, scale, zero, S, H=None, group_size=0):
         W = _f64(W)
         q, p = W.shape
         out = np.empty(q, np.float64)
         Hc = None if H is None else _f64(H)
-        self.lib.qo_objective_rows(_ptr(W, _f64p), _ptr(Hc, _f64p),
-                                   _ptr(np.ascontiguousarray(codes, np.uint8), _u8p),
-                                   _ptr(np.ascontiguousarray(scale, np.float32), _f32p),
-                                   _ptr(np.ascontiguousarray(zero, np.float32), _f32p),
-                                   q, p, _ptr(_f64(S), _f64p), _ptr(out, _f64p))
+        self.lib.qo_objective_rows_groups(_ptr(W, _f64p), _ptr(Hc, _f64p),
+                                          _ptr(np.ascontiguousarray(codes, np.uint8), _u8p),
+                                          _ptr(np.ascontiguousarray(scale, np.float32), _f32p),
+                                          _ptr(np.ascontiguousarray(zero, np.float32), _f32p),
+                                          q, p, group_size or p, _ptr(_f64(S), _f64p), _ptr(out, _f64p))
         return out
 
     def threads(self, n: int = 0) -> int:
@@ -149,11 +168,12 @@ class Oracle:
 
     # -- Algorithm 1 / 3 ----------------------------------------------------
     def alg1(self, W, S, scale, zero, bits, iters, init_codes=None, forced=None,
-             record=False, want_beta=False, relax_period=0):
+             record=False, want_beta=False, relax_period=0, group_size=0):
         """Algorithm 1.  Returns dict(codes, obj_rows[iters, q], obj[iters],
         sweep_codes[iters, q, p] if record, beta[iters, q, p] if want_beta).
         relax_period > 0: sweeps t (from 1) with t mod relax_period = 0 and t < iters
-        keep beta~ unquantized (the relax heuristic of Sec. 3.2).
+        keep beta~ unquantized (the relax heuristic of Sec. 3.2).  group_size > 0: grouped
+        grids, scale / zero q x groups (from grid(..., group_size)); binary64 S only.
         A float32 S is read as is and promoted exactly row by row (same binary64
         arithmetic, half the host memory); anything else is converted to float64."""
         W = _f64(W)
@@ -166,13 +186,21 @@ class Oracle:
         beta = np.empty((iters, q, p), np.float64) if want_beta else None
         ic = None if init_codes is None else np.ascontiguousarray(init_codes, np.uint8)
         fc = None if forced is None else np.ascontiguousarray(forced, np.uint8)
-        fn = self.lib.qo_quantease_alg1_f32 if f32 else self.lib.qo_quantease_alg1
-        rc = fn(
-            _ptr(W, _f64p), q, p, _ptr(S, _f32p if f32 else _f64p),
-            _ptr(np.ascontiguousarray(scale, np.float32), _f32p),
-            _ptr(np.ascontiguousarray(zero, np.float32), _f32p), bits, iters,
-            _ptr(ic, _u8p), _ptr(fc, _u8p), _ptr(codes, _u8p), _ptr(obj_rows, _f64p),
-            _ptr(sweep, _u8p), _ptr(beta, _f64p), relax_period)
+        sc = _ptr(np.ascontiguousarray(scale, np.float32), _f32p)
+        zc = _ptr(np.ascontiguousarray(zero, np.float32), _f32p)
+        if group_size:
+            if f32:
+                S = S.astype(np.float64)
+            rc = self.lib.qo_quantease_alg1_groups(
+                _ptr(W, _f64p), q, p, _ptr(S, _f64p), group_size, sc, zc, bits, iters,
+                _ptr(ic, _u8p), _ptr(fc, _u8p), _ptr(codes, _u8p), _ptr(obj_rows, _f64p),
+                _ptr(sweep, _u8p), _ptr(beta, _f64p), relax_period)
+        else:
+            fn = self.lib.qo_quantease_alg1_f32 if f32 else self.lib.qo_quantease_alg1
+            rc = fn(
+                _ptr(W, _f64p), q, p, _ptr(S, _f32p if f32 else _f64p), sc, zc, bits, iters,
+                _ptr(ic, _u8p), _ptr(fc, _u8p), _ptr(codes, _u8p), _ptr(obj_rows, _f64p),
+                _ptr(sweep, _u8p), _ptr(beta, _f64p), relax_period)
         if rc:
             raise MemoryError("oracle alg1 allocation failed")
         out = dict(codes=codes, obj_rows=obj_rows, obj=obj_rows.sum(axis=1))

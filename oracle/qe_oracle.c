@@ -55,29 +55,42 @@ int qo_threads(int n)
  * excl (q*p bytes, may be NULL) removes entries from the pool; with 0 always in
  * the range this is the same as setting them to 0 (Sec. 4.3, outliers removed
  * from the quantization pool).  Evaluated in binary32 (see file header).
+ * Grouped grids (a grid per row and group of gsize consecutive columns, the
+ * grouping the paper notes can be incorporated): the same rule over each
+ * group's columns; scale / zero are q x ceil(p / gsize), row-major.  gsize = p
+ * is the per-row grid.
  */
+void qo_grid_groups(const double *W, int64_t q, int64_t p, int64_t gsize, int bits,
+                    const uint8_t *excl, float *scale, float *zero)
+{
+    const float maxq = (float)((1 << bits) - 1);
+    const int64_t ng = (p + gsize - 1) / gsize;
+    for (int64_t i = 0; i < q; ++i)
+        for (int64_t g = 0; g < ng; ++g) {
+            float lo = 0.0f, hi = 0.0f;
+            const int64_t j1 = (g + 1) * gsize < p ? (g + 1) * gsize : p;
+            for (int64_t j = g * gsize; j < j1; ++j) {
+                if (excl && excl[i * p + j])
+                    continue;
+                float w = (float)W[i * p + j];
+                if (w < lo) lo = w;
+                if (w > hi) hi = w;
+            }
+            if (lo == 0.0f && hi == 0.0f) {
+                lo = -1.0f;
+                hi = 1.0f;
+            }
+            float s = (hi - lo) / maxq;
+            float z = nearbyintf(-lo / s);
+            scale[i * ng + g] = s;
+            zero[i * ng + g] = z;
+        }
+}
+
 void qo_grid(const double *W, int64_t q, int64_t p, int bits,
              const uint8_t *excl, float *scale, float *zero)
 {
-    const float maxq = (float)((1 << bits) - 1);
-    for (int64_t i = 0; i < q; ++i) {
-        float lo = 0.0f, hi = 0.0f;
-        for (int64_t j = 0; j < p; ++j) {
-            if (excl && excl[i * p + j])
-                continue;
-            float w = (float)W[i * p + j];
-            if (w < lo) lo = w;
-            if (w > hi) hi = w;
-        }
-        if (lo == 0.0f && hi == 0.0f) {
-            lo = -1.0f;
-            hi = 1.0f;
-        }
-        float s = (hi - lo) / maxq;
-        float z = nearbyintf(-lo / s);
-        scale[i] = s;
-        zero[i] = z;
-    }
+    qo_grid_groups(W, q, p, p, bits, excl, scale, zero);
 }
 
 /*
@@ -99,14 +112,22 @@ static double qo_level(int c, double s, double z)
     return s * ((double)c - z);
 }
 
-/* Round-to-nearest of a whole matrix on the grid (used for dead columns). */
+/* Round-to-nearest of a whole matrix on the (grouped) grid. */
+void qo_rtn_groups(const double *W, int64_t q, int64_t p, int64_t gsize, const float *scale,
+                   const float *zero, int bits, uint8_t *codes)
+{
+    const int maxq = (1 << bits) - 1;
+    const int64_t ng = (p + gsize - 1) / gsize;
+    for (int64_t i = 0; i < q; ++i)
+        for (int64_t j = 0; j < p; ++j)
+            codes[i * p + j] = (uint8_t)qo_code(W[i * p + j], scale[i * ng + j / gsize],
+                                                zero[i * ng + j / gsize], maxq);
+}
+
 void qo_rtn(const double *W, int64_t q, int64_t p, const float *scale,
             const float *zero, int bits, uint8_t *codes)
 {
-    const int maxq = (1 << bits) - 1;
-    for (int64_t i = 0; i < q; ++i)
-        for (int64_t j = 0; j < p; ++j)
-            codes[i * p + j] = (uint8_t)qo_code(W[i * p + j], scale[i], zero[i], maxq);
+    qo_rtn_groups(W, q, p, p, scale, zero, bits, codes);
 }
 
 /* ------------------------------------------------------------------------- */
@@ -204,21 +225,29 @@ static double qo_quad(const double *d, const qo_sig *S, int64_t p, double *buf)
  * (layerwise-main), What = s (codes - z) plus the optional dense H (Eq.
  * main-outlier: g = ||W X - (What + H) X||^2).  rows_out[i] = f_i.
  */
-void qo_objective_rows(const double *W, const double *H, const uint8_t *codes,
-                       const float *scale, const float *zero, int64_t q, int64_t p,
-                       const double *S, double *rows_out)
+void qo_objective_rows_groups(const double *W, const double *H, const uint8_t *codes,
+                              const float *scale, const float *zero, int64_t q, int64_t p,
+                              int64_t gsize, const double *S, double *rows_out)
 {
     const qo_sig Sg = {S, NULL, p};
+    const int64_t ng = (p + gsize - 1) / gsize;
 #pragma omp parallel for schedule(dynamic)
     for (int64_t i = 0; i < q; ++i) {
         double *d = (double *)malloc((size_t)p * sizeof(double));
         for (int64_t j = 0; j < p; ++j) {
-            double wh = qo_level(codes[i * p + j], scale[i], zero[i]);
+            double wh = qo_level(codes[i * p + j], scale[i * ng + j / gsize], zero[i * ng + j / gsize]);
             d[j] = W[i * p + j] - wh - (H ? H[i * p + j] : 0.0);
         }
         rows_out[i] = qo_quad(d, &Sg, p, NULL);
         free(d);
     }
+}
+
+void qo_objective_rows(const double *W, const double *H, const uint8_t *codes,
+                       const float *scale, const float *zero, int64_t q, int64_t p,
+                       const double *S, double *rows_out)
+{
+    qo_objective_rows_groups(W, H, codes, scale, zero, q, p, p, S, rows_out);
 }
 
 /* ------------------------------------------------------------------------- */
@@ -243,12 +272,13 @@ void qo_objective_rows(const double *W, const double *H, const uint8_t *codes,
  * quantization, forced ignored); codes[j] then records q_i(beta~), the nearest
  * level, as a view of the relaxed row.  Dead columns stay on their level.
  */
-static void qo_sweep_row(const qo_sig *S, int64_t p, double s, double z, int maxq,
-                         const double *tgt, const double *TS, double *Wh, double *WS,
+static void qo_sweep_row(const qo_sig *S, int64_t p, const float *srow, const float *zrow, int64_t gsize,
+                         int maxq, const double *tgt, const double *TS, double *Wh, double *WS,
                          const uint8_t *forced, uint8_t *codes, double *beta, double *buf,
                          int relax)
 {
     for (int64_t j = 0; j < p; ++j) {
+        const double s = srow[j / gsize], z = zrow[j / gsize];
         const double *Sj = qo_srow(S, j, buf);
         const double djj = Sj[j];
         int c;
@@ -312,12 +342,13 @@ static int qo_relaxed(int relax_period, int t1, int iters)
  *   relax_period  the relax heuristic (qo_relaxed); 0 = off
  */
 static int qo_alg1_core(const double *W, int64_t q, int64_t p, const qo_sig *S,
-                        const float *scale, const float *zero, int bits, int iters,
+                        const float *scale, const float *zero, int64_t gsize, int bits, int iters,
                         const uint8_t *init_codes, const uint8_t *forced,
                         uint8_t *codes, double *obj_rows, uint8_t *sweep_codes,
                         double *beta, int relax_period)
 {
     const int maxq = (1 << bits) - 1;
+    const int64_t ng = (p + gsize - 1) / gsize;
     int err = 0;
 #pragma omp parallel for schedule(dynamic)
     for (int64_t i = 0; i < q; ++i) {
@@ -330,14 +361,14 @@ static int qo_alg1_core(const double *W, int64_t q, int64_t p, const qo_sig *S,
             err = 1;
         } else {
             const double *Wi = W + i * p;
-            const double s = scale[i], z = zero[i];
+            const float *srow = scale + i * ng, *zrow = zero + i * ng;
             for (int64_t j = 0; j < p; ++j)
-                Wh[j] = init_codes ? qo_level(init_codes[i * p + j], s, z) : Wi[j];
+                Wh[j] = init_codes ? qo_level(init_codes[i * p + j], srow[j / gsize], zrow[j / gsize]) : Wi[j];
             qo_row_times_sigma(Wh, S, p, WS, buf);
             qo_row_times_sigma(Wi, S, p, TS, buf);
             for (int t = 0; t < iters; ++t) {
                 const size_t off = ((size_t)t * (size_t)q + (size_t)i) * (size_t)p;
-                qo_sweep_row(S, p, s, z, maxq, Wi, TS, Wh, WS,
+                qo_sweep_row(S, p, srow, zrow, gsize, maxq, Wi, TS, Wh, WS,
                              forced ? forced + off : NULL, codes + i * p,
                              beta ? beta + off : NULL, buf,
                              qo_relaxed(relax_period, t + 1, iters));
@@ -362,7 +393,19 @@ int qo_quantease_alg1(const double *W, int64_t q, int64_t p, const double *S,
                       double *beta, int relax_period)
 {
     const qo_sig Sg = {S, NULL, p};
-    return qo_alg1_core(W, q, p, &Sg, scale, zero, bits, iters, init_codes, forced, codes,
+    return qo_alg1_core(W, q, p, &Sg, scale, zero, p, bits, iters, init_codes, forced, codes,
+                        obj_rows, sweep_codes, beta, relax_period);
+}
+
+/* Algorithm 1 on grouped grids: scale / zero are q x ceil(p / gsize) (qo_grid_groups). */
+int qo_quantease_alg1_groups(const double *W, int64_t q, int64_t p, const double *S, int64_t gsize,
+                             const float *scale, const float *zero, int bits, int iters,
+                             const uint8_t *init_codes, const uint8_t *forced,
+                             uint8_t *codes, double *obj_rows, uint8_t *sweep_codes,
+                             double *beta, int relax_period)
+{
+    const qo_sig Sg = {S, NULL, p};
+    return qo_alg1_core(W, q, p, &Sg, scale, zero, gsize, bits, iters, init_codes, forced, codes,
                         obj_rows, sweep_codes, beta, relax_period);
 }
 
@@ -374,7 +417,7 @@ int qo_quantease_alg1_f32(const double *W, int64_t q, int64_t p, const float *S,
                           double *beta, int relax_period)
 {
     const qo_sig Sg = {NULL, S, p};
-    return qo_alg1_core(W, q, p, &Sg, scale, zero, bits, iters, init_codes, forced, codes,
+    return qo_alg1_core(W, q, p, &Sg, scale, zero, p, bits, iters, init_codes, forced, codes,
                         obj_rows, sweep_codes, beta, relax_period);
 }
 
@@ -653,7 +696,7 @@ int qo_quantease_outlier(const double *W, int64_t q, int64_t p, const double *S,
                 tgt[j] = W[i * p + j] - H[i * p + j];
             qo_row_times_sigma(tgt, &Sg, p, TS, NULL);
             qo_row_times_sigma(Wh + i * p, &Sg, p, WS, NULL);
-            qo_sweep_row(&Sg, p, scale[i], zero[i], maxq, tgt, TS, Wh + i * p, WS,
+            qo_sweep_row(&Sg, p, scale + i, zero + i, p, maxq, tgt, TS, Wh + i * p, WS,
                          NULL, codes + i * p, NULL, NULL, 0);
             free(tgt); free(TS); free(WS);
         }

@@ -37,6 +37,9 @@ MUTANTS = [
     ("column_norm_not_squared", "norm2[j] += T[i * p + j] * T[i * p + j];", "norm2[j] += T[i * p + j];"),
     ("relax_keeps_level", "                Wh[j] = b;\n", "                Wh[j] = qo_level(c, s, z);\n"),
     ("relax_last_sweep_too", "t1 % relax_period == 0 && t1 < iters;", "t1 % relax_period == 0 && t1 <= iters;"),
+    ("group_scale_of_first_group", "const double s = srow[j / gsize], z = zrow[j / gsize];",
+     "const double s = srow[0], z = zrow[0];"),
+    ("group_range_from_row_start", "for (int64_t j = g * gsize; j < j1; ++j) {", "for (int64_t j = 0; j < j1; ++j) {"),
 ]
 
 PINS = [
@@ -57,6 +60,9 @@ PINS = [
     lambda: pins.test_relaxed_sweep_is_one_gauss_seidel_step(3),
     pins.test_relaxed_sweeps_converge_to_w,
     pins.test_relax_period_not_below_iters_is_plain_algorithm1,
+    lambda: pins.test_grouped_grid_is_the_row_rule_per_group(3, 16),
+    pins.test_grouped_diagonal_sigma_gives_per_group_round_to_nearest,
+    lambda: pins.test_grouped_update_is_bruteforce_argmin_on_its_group(2),
     golden.test_hand_worked_two_feature_layer,
 ]
 

@@ -538,3 +538,104 @@ def test_pack_codes_matches_packbits_and_unpacks(bits):
     bitsarr = np.unpackbits(packed, axis=1, bitorder="little")
     back = sum(bitsarr[:, k::bits][:, :101].astype(np.int64) << k for k in range(bits))
     assert np.array_equal(back, codes)
+
+
+# --------------------------------------------------------------------------
+# grouped grids: a grid per row and group of gsize consecutive columns (the
+# grouping the paper notes can be incorporated into the per-channel grid)
+# --------------------------------------------------------------------------
+def _levels_grouped(codes, s, z, gsize):
+    g = np.arange(codes.shape[1]) // gsize
+    return s.astype(np.float64)[:, g] * (codes.astype(np.float64) - z.astype(np.float64)[:, g])
+
+
+@pytest.mark.parametrize("bits,gsize", [(2, 8), (3, 16), (4, 24)])
+def test_grouped_grid_is_the_row_rule_per_group(bits, gsize):
+    """Each group gets the row rule over its own columns, in binary32: range with 0,
+    s = (hi - lo) / (2^b - 1), z = round(-lo / s); an all-zero group gets [-1, 1]."""
+    rng = np.random.default_rng(20 + bits)
+    W = rng.normal(0, 0.02, size=(5, 70)).astype(np.float32).astype(np.float64)
+    W[1, gsize:2 * gsize] = 0.0
+    W[2, :gsize] = np.abs(W[2, :gsize])
+    s, z = O.grid(W, bits, group_size=gsize)
+    ng = -(-70 // gsize)
+    assert s.shape == (5, ng) and z.shape == (5, ng)
+    maxq = np.float32(2 ** bits - 1)
+    for i in range(5):
+        for g in range(ng):
+            w = W[i, g * gsize:(g + 1) * gsize].astype(np.float32)
+            lo, hi = min(np.float32(0), w.min()), max(np.float32(0), w.max())
+            if lo == 0 and hi == 0:
+                lo, hi = np.float32(-1), np.float32(1)
+            sg = np.float32(hi - lo) / maxq
+            assert s[i, g] == sg
+            assert z[i, g] == np.rint(np.float32(-lo) / sg)
+    # one group of p columns is the per-row grid
+    s1, z1 = O.grid(W, bits, group_size=70)
+    s0, z0 = O.grid(W, bits)
+    assert np.array_equal(s1[:, 0], s0) and np.array_equal(z1[:, 0], z0)
+
+
+def test_grouped_algorithm1_with_one_group_is_per_row_algorithm1():
+    rng = np.random.default_rng(21)
+    W, X = _rand_layer(rng, 6, 30, 120, heavy=(3,), corr=True)
+    S = O.sigma(X)
+    s, z = O.grid(W, 3)
+    a = O.alg1(W, S, s, z, 3, iters=3, record=True)
+    sg, zg = O.grid(W, 3, group_size=30)
+    b = O.alg1(W, S, sg, zg, 3, iters=3, record=True, group_size=30)
+    assert np.array_equal(a["sweep_codes"], b["sweep_codes"])
+    assert np.array_equal(a["obj_rows"], b["obj_rows"])
+
+
+def test_grouped_diagonal_sigma_gives_per_group_round_to_nearest():
+    rng = np.random.default_rng(22)
+    q, p, n, gsize = 6, 32, 64, 8
+    Qm, _ = np.linalg.qr(rng.normal(size=(n, p)))
+    X = Qm.T * rng.uniform(0.5, 3.0, size=(p, 1))
+    W = rng.normal(0, 0.02, size=(q, p))
+    W[:, 8:16] *= 5.0                       # groups of very different ranges
+    S = np.diag(np.diag(X @ X.T))
+    s, z = O.grid(W, 3, group_size=gsize)
+    r = O.alg1(W, S, s, z, 3, iters=2, record=True, group_size=gsize)
+    g = np.arange(p) // gsize
+    sf, zf = s.astype(np.float64)[:, g], z.astype(np.float64)[:, g]
+    rtn = np.clip(np.rint(W / sf + zf), 0, 7).astype(np.uint8)
+    for t in range(2):
+        assert np.array_equal(r["sweep_codes"][t], rtn)
+    assert np.array_equal(O.rtn(W, s, z, 3, group_size=gsize), rtn)
+
+
+@pytest.mark.parametrize("bits", [2, 3])
+def test_grouped_update_is_bruteforce_argmin_on_its_group(bits):
+    """Every update is the brute-force minimiser of ||W X - What X||^2 (from X itself,
+    Lemma 1) over the 2^b levels of its own column's group; the objective never
+    increases (Lemma 2) and equals the direct residual."""
+    rng = np.random.default_rng(110 + bits)
+    q, p, n, iters, gsize = 3, 9, 40, 3, 3
+    W, X = _rand_layer(rng, q, p, n, heavy=(2,), corr=True)
+    W[:, 3:6] *= 4.0
+    S = O.sigma(X)
+    s, z = O.grid(W, bits, group_size=gsize)
+    r = O.alg1(W, S, s, z, bits, iters, record=True, group_size=gsize)
+    sc = r["sweep_codes"]
+    cand = np.arange(2 ** bits)
+    for t in range(iters):
+        before = W.copy() if t == 0 else _levels_grouped(sc[t - 1], s, z, gsize)
+        after = _levels_grouped(sc[t], s, z, gsize)
+        for i in range(q):
+            for j in range(p):
+                state = np.concatenate([after[i, :j], before[i, j:]])
+                sg, zg = float(s[i, j // gsize]), float(z[i, j // gsize])
+                f = []
+                for c in cand:
+                    row = state.copy()
+                    row[j] = sg * (c - zg)
+                    f.append(_f_direct(W[i:i + 1], row[None, :], X))
+                f = np.array(f)
+                assert f[sc[t, i, j]] <= f.min() + 1e-12 * max(1.0, abs(f.min())), (t, i, j)
+    obj = r["obj"]
+    assert np.all(np.diff(obj) <= 1e-12 * obj[:-1])
+    direct = np.sum(((W - _levels_grouped(r["codes"], s, z, gsize)) @ X) ** 2, axis=1)
+    assert np.allclose(r["obj_rows"][-1], direct, rtol=1e-10)
+    assert np.allclose(O.objective_rows(W, r["codes"], s, z, S, group_size=gsize), direct, rtol=1e-10)
