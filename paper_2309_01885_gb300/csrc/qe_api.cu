@@ -58,6 +58,8 @@ constexpr int kFreeMaxChanges = 64;      // changes per row in the previous swee
 struct Plan {
     int64_t q = 0, p = 0, ld = 0;
     int B = kDefaultBlock, smax = 1;
+    int64_t gsize = 0, ngroups = 1;   // grid columns per group (p: per row), groups per row
+    bool grouped = false;
     size_t snt = 0, d = 0, dinv = 0, tri = 0, P = 0, R = 0, wpl = 0, qf = 0, dp = 0, part = 0, objp = 0,
            rowdf = 0, objbase = 0, sbar = 0, lcnt = 0, lent = 0, rowdft = 0;
     int64_t nblk = 0;
@@ -72,10 +74,13 @@ static size_t take(size_t &cur, size_t bytes) {
     return o;
 }
 
-static Plan make_plan(int64_t q, int64_t p, int B, bool outlier, int wpl_planes, int nsm) {
+static Plan make_plan(int64_t q, int64_t p, int B, bool outlier, int wpl_planes, int nsm, int64_t group = 0) {
     Plan pl;
     pl.q = q;
     pl.p = p;
+    pl.grouped = group > 0 && group < p;
+    pl.gsize = pl.grouped ? group : p;
+    pl.ngroups = ceil_div(p, pl.gsize);
     pl.ld = round_up(p, 64);
     pl.B = B;
     pl.nblk = ceil_div(p, B);
@@ -93,7 +98,7 @@ static Plan make_plan(int64_t q, int64_t p, int B, bool outlier, int wpl_planes,
     pl.P = take(cur, qld * 4);
     pl.R = take(cur, qld * 4);
     pl.wpl = take(cur, wpl_planes > 0 ? qld * 2 * wpl_planes : 0);
-    pl.qf = take(cur, qld * 2);
+    pl.qf = take(cur, qld * 2 * (pl.grouped ? 3 : 1));   // grouped: s_g (C - z_g) in three planes
     pl.dp = take(cur, qld * 2 * 3);
     pl.part = take(cur, static_cast<size_t>(pl.smax) * q * B * 4);
     pl.objp = take(cur, static_cast<size_t>(rfull_partials(q, p) > objective_blocks(q) ? rfull_partials(q, p)
@@ -268,7 +273,7 @@ static qe_status setup_ctx(Ctx &c, const Plan &pl, const qe_opts *o, cudaStream_
     if (!make_tmap_bf16(&c.tm_snt256, c.snt, 3 * p, p, ld, 256) ||
         !make_tmap_bf16(&c.tm_snt64, c.snt, 3 * p, p, ld, 64) ||
         !make_tmap_bf16(&c.tm_snt128, c.snt, 3 * p, p, ld, 128) ||
-        !make_tmap_bf16(&c.tm_qf, c.qf, q, p, ld, 128) ||
+        !make_tmap_bf16(&c.tm_qf, c.qf, pl.grouped ? 3 * q : q, p, ld, 128) ||
         !make_tmap_bf16(&c.tm_dp, c.dp, 3 * q, p, ld, 128))
         return QE_ERR_CUDA;
     return QE_OK;
@@ -356,7 +361,10 @@ static qe_status residual(Ctx &c, const float *scales, const float *zeros, const
     const int64_t q = c.pl.q, p = c.pl.p, ld = c.pl.ld;
     GemmArgs g = gemm_args(c, static_cast<int>(q), static_cast<int>(p), static_cast<int>(ceil_div(p, 64)),
                            EPI_RFULL);
-    set_prods(g, 1);
+    set_prods(g, c.pl.grouped ? 3 : 1);
+    g.gsize = c.pl.gsize;
+    g.ngroups = c.pl.ngroups;
+    g.absolute = c.pl.grouped ? 1 : 0;
     g.m_fast = 1;
     g.a_plane_rows = static_cast<int>(q);
     g.b_plane_rows = static_cast<int>(p);
@@ -420,7 +428,7 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
             const int kb = static_cast<int>(ceil_div(kcols, 64));
             const int S = kb < c.pl.smax ? kb : c.pl.smax;
             GemmArgs g = gemm_args(c, static_cast<int>(q), bw, kb, EPI_TRAIL);
-            set_prods(g, frac ? 3 : 1);
+            set_prods(g, (frac || c.pl.grouped) ? 3 : 1);
             g.a_plane_rows = static_cast<int>(q);
             g.b_plane_rows = static_cast<int>(p);
             g.b_row0 = static_cast<int>(b0);
@@ -448,6 +456,9 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
         a.tri = c.tri;
         a.scale = scales;
         a.zero = zeros;
+        a.gsize = c.pl.gsize;
+        a.ngroups = c.pl.ngroups;
+        a.grouped = c.pl.grouped ? 1 : 0;
         a.d = c.d;
         a.rowdf = window != 0 ? c.rowdf : nullptr;
         a.maxq = static_cast<float>((1 << bits) - 1);
@@ -485,6 +496,9 @@ static CdArgs list_args(const Ctx &c, uint8_t *codes, const float *scales, const
     a.tri = c.tri;
     a.scale = scales;
     a.zero = zeros;
+    a.gsize = c.pl.gsize;
+    a.ngroups = c.pl.ngroups;
+    a.grouped = c.pl.grouped ? 1 : 0;
     a.d = c.d;
     a.maxq = static_cast<float>((1 << bits) - 1);
     a.codes = codes;
@@ -546,10 +560,18 @@ static qe_status check_opts(const qe_opts *o, bool structured = false) {
     if (o->structured_outliers != 0 && !(structured && o->structured_outliers == 1)) return QE_ERR_UNSUPPORTED;
     if (o->block_width != 0 && o->block_width != 64 && o->block_width != 128 && o->block_width != 256)
         return QE_ERR_UNSUPPORTED;
-    if (o->power_iters < 0 || o->dense_sweeps < 0 || o->free_changes < -1) return QE_ERR_INVALID_ARG;
+    if (o->power_iters < 0 || o->dense_sweeps < 0 || o->free_changes < -1 || o->group_size < 0)
+        return QE_ERR_INVALID_ARG;
     if (o->workspace && o->workspace_bytes == 0) return QE_ERR_INVALID_ARG;
+    if (o->group_size > 0) {
+        // groups hold whole column blocks; no relax heuristic, no outlier variant with groups
+        if (o->group_size % block_width(o) != 0) return QE_ERR_INVALID_ARG;
+        if (structured || o->relax_period != 0) return QE_ERR_UNSUPPORTED;
+    }
     return QE_OK;
 }
+
+static int64_t group_size(const qe_opts *o) { return o ? o->group_size : 0; }
 
 static qe_status check_layer(const void *W, qe_dtype wt, int64_t q, int64_t p, int64_t ldw,
                              const float *Sigma, int bits, int iters, const uint8_t *codes,
@@ -659,7 +681,7 @@ qe_status qe_workspace_size(int64_t q, int64_t p, int outlier, const qe_opts *op
     if (!bytes || q < 1 || p < 1) return QE_ERR_INVALID_ARG;
     const qe_status st = check_opts(opts, outlier != 0);
     if (st != QE_OK) return st;
-    const Plan pl = make_plan(q, p, block_width(opts), outlier != 0, 3, sm_count());
+    const Plan pl = make_plan(q, p, block_width(opts), outlier != 0, 3, sm_count(), group_size(opts));
     *bytes = pl.total;
     return QE_OK;
 }
@@ -745,10 +767,10 @@ qe_status qe_quantize_layer(const void *W, qe_dtype w_dtype, int64_t q, int64_t 
     const int wbf16 = (w_dtype == QE_BF16);
     Ctx c;
     c.nsm = sm_count();
-    const Plan pl = make_plan(q, p, block_width(opts), false, wbf16 ? 1 : 3, c.nsm);
+    const Plan pl = make_plan(q, p, block_width(opts), false, wbf16 ? 1 : 3, c.nsm, group_size(opts));
     if ((st = setup_ctx(c, pl, opts, reinterpret_cast<cudaStream_t>(stream))) != QE_OK) return st;
 
-    QE_CK(launch_grid(W, wbf16, ldw, nullptr, 0, q, p, bits, scales, zeros, c.err, c.s));
+    QE_CK(launch_grid(W, wbf16, ldw, nullptr, 0, q, p, pl.gsize, bits, scales, zeros, c.err, c.s));
     if ((st = prepare(c, W, wbf16, ldw, Sigma, c.P)) != QE_OK) return st;
     if (opts && opts->wx_norm2)
         if ((st = objective(c, W, wbf16, ldw, nullptr, nullptr, nullptr, nullptr, c.P, opts->wx_norm2)) != QE_OK)
@@ -772,7 +794,7 @@ qe_status qe_quantize_layer(const void *W, qe_dtype w_dtype, int64_t q, int64_t 
         return QE_OK;
     };
     auto refresh = [&]() -> qe_status {
-        QE_CK(launch_codes_to_qf(codes, p, zeros, q, p, c.qf, pl.ld, c.s));
+        QE_CK(launch_codes_to_qf(codes, p, scales, zeros, q, p, pl.gsize, pl.grouped, c.qf, pl.ld, c.s));
         return residual(c, scales, zeros);
     };
     auto record = [&](int t) -> qe_status {
@@ -784,11 +806,11 @@ qe_status qe_quantize_layer(const void *W, qe_dtype w_dtype, int64_t q, int64_t 
     int t = 0, src = SRC_CODES;
     if (warm) {
         QE_CK(cudaMemcpyAsync(codes, opts->init_codes, static_cast<size_t>(q) * p, cudaMemcpyDeviceToDevice, c.s));
-        QE_CK(launch_codes_to_qf(codes, p, zeros, q, p, c.qf, pl.ld, c.s));
+        QE_CK(launch_codes_to_qf(codes, p, scales, zeros, q, p, pl.gsize, pl.grouped, c.qf, pl.ld, c.s));
         const ObjFuse f{c.objbase, W, wbf16, ldw, codes, nullptr};
         if ((st = residual(c, scales, zeros, &f)) != QE_OK) return st;
     } else {
-        QE_CK(launch_init_residual(W, wbf16, ldw, nullptr, 0, q, p, scales, zeros, c.R, pl.ld, c.s));
+        QE_CK(launch_init_residual(W, wbf16, ldw, nullptr, 0, q, p, pl.gsize, scales, zeros, c.R, pl.ld, c.s));
         QE_CK(cudaMemsetAsync(c.objbase, 0, 8, c.s));   // f(W) = 0
         src = SRC_W;
         if (!relaxed(0)) {
@@ -803,7 +825,9 @@ qe_status qe_quantize_layer(const void *W, qe_dtype w_dtype, int64_t q, int64_t 
     if ((st = restart(src == SRC_CODES ? 1 : 3)) != QE_OK) return st;
     bool exact = true;   // R is the residual of the current What and no list has entries
     bool chain = false;  // the last sweep was a sequential one (its three-plane changes are in dp)
-    const int dense = dense_sweeps(opts);
+    // grouped grids: the change lists assume one scale per row, so every sweep takes the
+    // tensor-core form of the window
+    const int dense = pl.grouped ? iters : dense_sweeps(opts);
     while (t < iters) {
         const bool rx = relaxed(t);
         if (rx || src != SRC_CODES) {
@@ -890,7 +914,7 @@ qe_status qe_quantize_layer_outlier(const void *W, qe_dtype w_dtype, int64_t q, 
     QE_CK(select(c.T));
     QE_CK(cudaMemsetAsync(c.H, 0, static_cast<size_t>(q) * ld * 4, c.s));
     QE_CK(launch_scatter_rowptr(H_idx, H_val, H_nnz, s_budget, q, p, c.H, ld, c.rowptr, c.s));
-    QE_CK(launch_grid(W, wbf16, ldw, c.H, ld, q, p, bits, scales, zeros, c.err, c.s));
+    QE_CK(launch_grid(W, wbf16, ldw, c.H, ld, q, p, p, bits, scales, zeros, c.err, c.s));
     // P_W = W (I + Sigma_bar), eta = 1 / (2 lambda_max), P = P_W - H (I + Sigma_bar)
     if ((st = prepare(c, W, wbf16, ldw, Sigma, c.PW)) != QE_OK) return st;
     QE_CK(launch_power_lambda(Sigma, p, p, power_iters, c.y0, c.y1, c.ppart, c.lam, c.eta, c.nsm, c.s));
@@ -902,10 +926,10 @@ qe_status qe_quantize_layer_outlier(const void *W, qe_dtype w_dtype, int64_t q, 
     const bool warm = opts && opts->init_codes;
     if (warm) {
         QE_CK(cudaMemcpyAsync(codes, opts->init_codes, static_cast<size_t>(q) * p, cudaMemcpyDeviceToDevice, c.s));
-        QE_CK(launch_codes_to_qf(codes, p, zeros, q, p, c.qf, ld, c.s));
+        QE_CK(launch_codes_to_qf(codes, p, scales, zeros, q, p, p, 0, c.qf, ld, c.s));
         if ((st = residual(c, scales, zeros)) != QE_OK) return st;
     } else {
-        QE_CK(launch_init_residual(W, wbf16, ldw, c.H, ld, q, p, scales, zeros, c.R, ld, c.s));
+        QE_CK(launch_init_residual(W, wbf16, ldw, c.H, ld, q, p, p, scales, zeros, c.R, ld, c.s));
     }
     // g of a warm start, the base of the first sweep's objective changes
     if (warm && obj_cd)

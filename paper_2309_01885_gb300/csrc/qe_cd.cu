@@ -19,13 +19,17 @@ __device__ __forceinline__ float load_elem(const void *base, int is_bf16, int64_
 // that the entries held by H (exactly equal to W there) leave the pool
 // (Sec. 4.3).  Non-finite entries latch ERR_NUMERIC.
 // ---------------------------------------------------------------------------
+// Grouped grids: CTA (i, g) takes the columns of group g only and writes entry
+// i * gridDim.y + g.
 __global__ void __launch_bounds__(256) k_grid(const void *W, int w_bf16, int64_t ldw, const float *H,
-                                              int64_t ldh, int64_t p, float maxq, float *scale,
+                                              int64_t ldh, int64_t p, int64_t gsize, float maxq, float *scale,
                                               float *zero, unsigned *err) {
     const int64_t i = blockIdx.x;
+    const int64_t j0 = static_cast<int64_t>(blockIdx.y) * gsize;
+    const int64_t j1 = (j0 + gsize) < p ? (j0 + gsize) : p;
     float lo = 0.0f, hi = 0.0f;
     bool bad = false;
-    for (int64_t j = threadIdx.x; j < p; j += blockDim.x) {
+    for (int64_t j = j0 + threadIdx.x; j < j1; j += blockDim.x) {
         float w = load_elem(W, w_bf16, i * ldw + j);
         if (!isfinite(w)) bad = true;
         if (H) w = w - H[i * ldh + j];
@@ -58,8 +62,8 @@ __global__ void __launch_bounds__(256) k_grid(const void *W, int w_bf16, int64_t
         }
         const float s = __fdiv_rn(__fsub_rn(hi, lo), maxq);
         const float z = rintf(__fdiv_rn(-lo, s));
-        scale[i] = s;
-        zero[i] = z;
+        scale[i * gridDim.y + blockIdx.y] = s;
+        zero[i * gridDim.y + blockIdx.y] = z;
         if (sbad) set_error(err, ERR_NUMERIC);
     }
 }
@@ -204,12 +208,13 @@ __global__ void k_make_planes(const void *W, int w_bf16, int64_t ldw, int64_t q,
 // What = W - H, P - What Sigma_bar = (W - H)(I + Sigma_bar) - (W - H) Sigma_bar
 // = W - H, stored as (W - H) / s + z.
 __global__ void k_init_residual(const void *W, int w_bf16, int64_t ldw, const float *H, int64_t ldh,
-                                int64_t q, int64_t p, const float *scale, const float *zero, float *R,
-                                int64_t ldr) {
+                                int64_t q, int64_t p, int64_t gsize, const float *scale, const float *zero,
+                                float *R, int64_t ldr) {
+    const int64_t ng = ceil_div(p, gsize);   // the 4 columns of a thread lie in one group (gsize = p or % 64 == 0)
     for (int64_t i = blockIdx.y; i < q; i += gridDim.y) {
-        const float s = scale[i], z = zero[i];
         for (int64_t j0 = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) * 4; j0 < p;
              j0 += (int64_t)gridDim.x * blockDim.x * 4) {
+            const float s = scale[i * ng + j0 / gsize], z = zero[i * ng + j0 / gsize];
             float o[4];
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
@@ -251,13 +256,24 @@ __global__ void k_obj_step(double *rowdf, int64_t q, const double *prev, double 
 }
 
 // (C - z) as bf16 (exact: |C - z| <= 255) for the R = P - s (C - z) Sigma_bar GEMM.
-__global__ void k_codes_to_qf(const uint8_t *codes, int64_t ldc, const float *zero, int64_t q,
-                              int64_t p, __nv_bfloat16 *qf, int64_t ldq) {
+__global__ void k_codes_to_qf(const uint8_t *codes, int64_t ldc, const float *scale, const float *zero,
+                              int64_t q, int64_t p, int64_t gsize, int grouped, __nv_bfloat16 *qf, int64_t ldq) {
+    const int64_t ng = ceil_div(p, gsize);
     for (int64_t i = blockIdx.y; i < q; i += gridDim.y) {
-        const float z = zero[i];
         for (int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; j < p;
-             j += (int64_t)gridDim.x * blockDim.x)
-            qf[i * ldq + j] = __float2bfloat16_rn(static_cast<float>(codes[i * ldc + j]) - z);
+             j += (int64_t)gridDim.x * blockDim.x) {
+            const int64_t gi = i * ng + j / gsize;
+            const float cz = static_cast<float>(codes[i * ldc + j]) - zero[gi];
+            if (!grouped) {
+                qf[i * ldq + j] = __float2bfloat16_rn(cz);
+            } else {
+                __nv_bfloat16 h, m, l;
+                split3(scale[gi] * cz, h, m, l);
+                qf[i * ldq + j] = h;
+                qf[(q + i) * ldq + j] = m;
+                qf[(2 * q + i) * ldq + j] = l;
+            }
+        }
     }
 }
 
@@ -421,6 +437,11 @@ __device__ __forceinline__ bool cd_prologue(const CdArgs &a, float *tri, uint64_
             if (row_ok && (FULL || 32 * h + lane < bw)) ps[h] += prow[32 * h + lane];
     }
     const bool changed = a.nsplit > 0;
+    if (a.grouped && changed) {   // absolute partials: into the grid units of the block's group
+        const float sg = a.scale[ii * a.ngroups + b0 / a.gsize];
+#pragma unroll
+        for (int h = 0; h < CPL; ++h) ps[h] = __fdiv_rn(ps[h], sg);
+    }
 #pragma unroll
     for (int h = 0; h < CPL; ++h) {
         st[h] = a.first_sweep ? r_[h]
@@ -451,7 +472,9 @@ __device__ __forceinline__ void cd_epilogue(const CdArgs &a, int64_t b0, int bw_
                                             bool skip_same) {
     constexpr int CPL = B / 32;
     const int bw = FULL ? B : bw_;
-    const float z = a.zero[i];
+    const int64_t gi = i * a.ngroups + b0 / a.gsize;   // the block lies in one group
+    const float z = a.zero[gi];
+    const float sg = a.grouped ? a.scale[gi] : 1.0f;
 #pragma unroll
     for (int h = 0; h < CPL; ++h) {
         const int l = 32 * h + lane;
@@ -462,13 +485,26 @@ __device__ __forceinline__ void cd_epilogue(const CdArgs &a, int64_t b0, int bw_
             a.codes[i * a.ldc + col] = static_cast<uint8_t>(rintf(fminf(fmaxf(code[h], 0.0f), a.maxq)));
         } else if (!skip_same || dlt[h] != 0.0f) {
             a.codes[i * a.ldc + col] = static_cast<uint8_t>(code[h]);
-            if (a.write_qf) a.qf[i * a.ldq + col] = __float2bfloat16_rn(code[h] - z);
+            if (a.write_qf) {
+                if (!a.grouped) {
+                    a.qf[i * a.ldq + col] = __float2bfloat16_rn(code[h] - z);
+                } else {   // the residual GEMM takes s_g (C - z_g), three planes
+                    __nv_bfloat16 qh, qm, ql;
+                    split3(sg * (code[h] - z), qh, qm, ql);
+                    a.qf[i * a.ldq + col] = qh;
+                    a.qf[(a.q + i) * a.ldq + col] = qm;
+                    a.qf[(2 * a.q + i) * a.ldq + col] = ql;
+                }
+            }
         }
         if (!a.dp) continue;
-        const __nv_bfloat16 hi = __float2bfloat16_rn(dlt[h]);
+        // grouped: the trailing GEMM sums changes of several groups, so it takes them
+        // absolute (s_g Delta'), which is not an integer: three planes
+        const float dv = a.grouped ? sg * dlt[h] : dlt[h];
+        const __nv_bfloat16 hi = __float2bfloat16_rn(dv);
         a.dp[i * a.ldd + col] = hi;
-        if (a.frac) {   // Delta' is not an integer: three planes
-            const float r1 = dlt[h] - __bfloat162float(hi);
+        if (a.frac || a.grouped) {   // Delta' is not an integer: three planes
+            const float r1 = dv - __bfloat162float(hi);
             const __nv_bfloat16 mid = __float2bfloat16_rn(r1);
             a.dp[(a.dp_plane_rows + i) * a.ldd + col] = mid;
             a.dp[(2 * a.dp_plane_rows + i) * a.ldd + col] = __float2bfloat16_rn(r1 - __bfloat162float(mid));
@@ -567,7 +603,7 @@ __global__ void __launch_bounds__(1024) k_cd_block_seq(const CdArgs a) {
     }
     if (DF) {
         __syncwarp();
-        const float sc = a.scale[i];
+        const float sc = a.scale[i * a.ngroups + a.b0 / a.gsize];
         const float s2 = sc * sc;
         double dfacc = 0.0;
 #pragma unroll
@@ -686,7 +722,7 @@ __global__ void __launch_bounds__(1024, 1) k_cd_block_chg(const CdArgs a) {
     if (!cd_prologue<B, FULL>(a, tri, bar, i, row_ok, lane, t, st)) return;
     if (!row_ok) return;
     float code[CPL], dlt[CPL];
-    const float s = a.scale[i];
+    const float s = a.scale[i * a.ngroups + a.b0 / a.gsize];
     double dfacc = 0.0;
     chg_decide<B, FULL>(tri, a.d + a.b0, a.bw, a.maxq, s * s, a.rowdf != nullptr, lane, t, st, code, dlt, dfacc);
     if (a.rowdf) {
@@ -1325,10 +1361,11 @@ static inline dim3 row_grid(int64_t rows, int64_t cols) {
 static inline dim3 row_grid4(int64_t rows, int64_t cols) { return row_grid(rows, ceil_div(cols, 4)); }
 
 cudaError_t launch_grid(const void *W, int w_bf16, int64_t ldw, const float *H, int64_t ldh, int64_t q,
-                        int64_t p, int bits, float *scale, float *zero, unsigned *err, cudaStream_t s) {
-    k_grid<<<static_cast<unsigned>(q), 256, 0, s>>>(W, w_bf16, ldw, H, ldh, p,
-                                                    static_cast<float>((1 << bits) - 1), scale, zero,
-                                                    err);
+                        int64_t p, int64_t gsize, int bits, float *scale, float *zero, unsigned *err,
+                        cudaStream_t s) {
+    const dim3 grid(static_cast<unsigned>(q), static_cast<unsigned>(ceil_div(p, gsize)));
+    k_grid<<<grid, 256, 0, s>>>(W, w_bf16, ldw, H, ldh, p, gsize, static_cast<float>((1 << bits) - 1), scale,
+                                zero, err);
     return cudaGetLastError();
 }
 
@@ -1353,9 +1390,9 @@ cudaError_t launch_make_planes(const void *W, int w_bf16, int64_t ldw, int64_t q
 }
 
 cudaError_t launch_init_residual(const void *W, int w_bf16, int64_t ldw, const float *H, int64_t ldh,
-                                 int64_t q, int64_t p, const float *scale, const float *zero, float *R,
-                                 int64_t ldr, cudaStream_t s) {
-    k_init_residual<<<row_grid4(q, p), 256, 0, s>>>(W, w_bf16, ldw, H, ldh, q, p, scale, zero, R, ldr);
+                                 int64_t q, int64_t p, int64_t gsize, const float *scale, const float *zero,
+                                 float *R, int64_t ldr, cudaStream_t s) {
+    k_init_residual<<<row_grid4(q, p), 256, 0, s>>>(W, w_bf16, ldw, H, ldh, q, p, gsize, scale, zero, R, ldr);
     return cudaGetLastError();
 }
 
@@ -1364,9 +1401,10 @@ cudaError_t launch_obj_step(double *rowdf, int64_t q, const double *prev, double
     return cudaGetLastError();
 }
 
-cudaError_t launch_codes_to_qf(const uint8_t *codes, int64_t ldc, const float *zero, int64_t q,
-                               int64_t p, __nv_bfloat16 *qf, int64_t ldq, cudaStream_t s) {
-    k_codes_to_qf<<<row_grid(q, p), 256, 0, s>>>(codes, ldc, zero, q, p, qf, ldq);
+cudaError_t launch_codes_to_qf(const uint8_t *codes, int64_t ldc, const float *scale, const float *zero,
+                               int64_t q, int64_t p, int64_t gsize, int grouped, __nv_bfloat16 *qf,
+                               int64_t ldq, cudaStream_t s) {
+    k_codes_to_qf<<<row_grid(q, p), 256, 0, s>>>(codes, ldc, scale, zero, q, p, gsize, grouped, qf, ldq);
     return cudaGetLastError();
 }
 

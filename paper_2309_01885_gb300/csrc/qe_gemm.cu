@@ -92,14 +92,24 @@ __device__ __forceinline__ void epilogue_row(const GemmArgs &g, int r, int c0, c
             break;
         }
         case EPI_RFULL: {
-            // R in grid-step units: (P - s (C - z) Sigma_bar) / s + z = P / s - acc + z
-            const float s = g.scale[r];
-            const float zz = g.zero[r];
+            // R in grid-step units: (P - s (C - z) Sigma_bar) / s + z = P / s - acc + z; with
+            // grouped grids (absolute) acc = s_g (C - z_g) Sigma_bar, R = (P - acc) / s_g + z_g
+            // (the 32 columns lie in one group)
+            const int64_t gi = g.ngroups > 1 ? rr * g.ngroups + c0 / g.gsize : rr;
+            const float s = g.scale[gi];
+            const float zz = g.zero[gi];
             const float *prow = g.P + rr * g.ldp;
             float *orow = g.out + rr * g.ldo;
             float o[32];
             const bool full = c0 + 32 <= g.N;
-            if (full && ((g.ldo | g.ldp) & 3) == 0) {
+            if (g.absolute) {
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    const int c = c0 + i;
+                    o[i] = 0.0f;
+                    if (c < g.N) orow[c] = o[i] = __fdiv_rn(prow[c] - v[i], s) + zz;
+                }
+            } else if (full && ((g.ldo | g.ldp) & 3) == 0) {
 #pragma unroll
                 for (int i = 0; i < 32; i += 4) {
                     const float4 pv = *reinterpret_cast<const float4 *>(prow + c0 + i);

@@ -42,6 +42,11 @@ struct GemmArgs {
     const uint8_t *codes;
     int64_t ldc;
     const float *zero;
+    // EPI_RFULL with grouped grids: scale / zero per row and group of gsize columns
+    // ([r * ngroups + c / gsize]; ngroups = 1: per row), and absolute = 1: the A operand
+    // is s_g (C - z_g), so R = (P - acc) / s_g + z_g
+    int64_t gsize, ngroups;
+    int absolute;
     const float *dvec;
     const float *Hd;
     int64_t ldh;

@@ -26,7 +26,10 @@ struct CdArgs {
     int *lcnt;                      // [q][nblk] entry counts
     uint32_t *lent;                 // [q][nblk][B] entries; non-NULL: record this visit's changes
     const float *tri;               // packed diagonal blocks of Sigma_bar (launch_pack_diag)
-    const float *scale, *zero;
+    const float *scale, *zero;      // per row, or per row and group: [i * ngroups + column / gsize]
+    int64_t gsize, ngroups;         // columns per group (p when not grouped) and groups per row
+    int grouped;                    // grouped grids: the Delta' planes carry s_g Delta' (absolute) and
+                                    // the split partials are absolute (divided by the block's scale)
     const float *d;                 // Sigma_jj (objective change of each decision)
     double *rowdf;                  // per-row objective change accumulator, or NULL
     float maxq;
@@ -63,8 +66,10 @@ struct ObjArgs {
     int64_t ldr;
 };
 
+// Per row (gsize = p) or per row and group of gsize columns: scale / zero [q][ceil(p / gsize)].
 cudaError_t launch_grid(const void *W, int w_bf16, int64_t ldw, const float *H, int64_t ldh, int64_t q,
-                        int64_t p, int bits, float *scale, float *zero, unsigned *err, cudaStream_t s);
+                        int64_t p, int64_t gsize, int bits, float *scale, float *zero, unsigned *err,
+                        cudaStream_t s);
 cudaError_t launch_sigma_norm(const float *S, int64_t lds, int64_t p, float *d, __nv_bfloat16 *snt,
                               int64_t ldn, unsigned *err, cudaStream_t s);
 // fp32 Sigma_bar, row k = the coupling of column k to every column (ld columns, zero-padded).
@@ -73,12 +78,15 @@ cudaError_t launch_sigma_bar_rows(const float *S, int64_t lds, int64_t p, const 
 cudaError_t launch_make_planes(const void *W, int w_bf16, int64_t ldw, int64_t q, int64_t p,
                                int split, __nv_bfloat16 *out, int64_t ldo, cudaStream_t s);
 cudaError_t launch_init_residual(const void *W, int w_bf16, int64_t ldw, const float *H, int64_t ldh,
-                                 int64_t q, int64_t p, const float *scale, const float *zero, float *R,
-                                 int64_t ldr, cudaStream_t s);
+                                 int64_t q, int64_t p, int64_t gsize, const float *scale, const float *zero,
+                                 float *R, int64_t ldr, cudaStream_t s);
 // obj[out] = obj[prev] + sum_i rowdf[i]; rowdf is zeroed.  prev may be NULL (0).
 cudaError_t launch_obj_step(double *rowdf, int64_t q, const double *prev, double *out, cudaStream_t s);
-cudaError_t launch_codes_to_qf(const uint8_t *codes, int64_t ldc, const float *zero, int64_t q,
-                               int64_t p, __nv_bfloat16 *qf, int64_t ldq, cudaStream_t s);
+// C - z (one exact bf16 plane), or with grouped grids s_g (C - z_g) in three planes
+// (rows [0, q), [q, 2q), [2q, 3q)); gsize = p: per-row grids.
+cudaError_t launch_codes_to_qf(const uint8_t *codes, int64_t ldc, const float *scale, const float *zero,
+                               int64_t q, int64_t p, int64_t gsize, int grouped, __nv_bfloat16 *qf,
+                               int64_t ldq, cudaStream_t s);
 cudaError_t launch_cd_block(int B, const CdArgs &a, int nsm, cudaStream_t s);
 // Sweeps [t_begin, t_end) with the change-list correction in one persistent launch
 // (a.sbar, a.lcnt, a.lent set; a.b0 / a.bw / a.part unused); the objective change of

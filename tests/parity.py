@@ -44,18 +44,26 @@ def check_obj(obj_gpu, obj_oracle, rtol=OBJ_RTOL, what="objective", atol=0.0):
     return float(rel.max())
 
 
-def teacher_forced(W64, S64, scale, zero, bits, sweep_codes_gpu, init_codes=None, want_run=False):
+def teacher_forced(W64, S64, scale, zero, bits, sweep_codes_gpu, init_codes=None, want_run=False,
+                   group_size=0):
     """Replay the GPU trajectory through Algorithm 1 with its own codes forced:
     every GPU code must be the nearest level of the fp64 beta~ unless beta~
     sits within MIDPOINT_TOL (in grid steps) of a rounding midpoint.
     Returns (number of near-midpoint disagreements, number of checks), plus the
-    oracle's replay (objective of the GPU's codes after each sweep) with want_run."""
+    oracle's replay (objective of the GPU's codes after each sweep) with want_run.
+    group_size > 0: grouped grids (scale / zero q x groups)."""
     O = oracle.get()
     iters = sweep_codes_gpu.shape[0]
     r = O.alg1(W64, S64, scale, zero, bits, iters, init_codes=init_codes,
-               forced=sweep_codes_gpu, want_beta=True)
+               forced=sweep_codes_gpu, want_beta=True, group_size=group_size)
     maxq = 2 ** bits - 1
-    t = r["beta"] / scale.astype(np.float64)[None, :, None] + zero.astype(np.float64)[None, :, None]
+    p = W64.shape[1]
+    if group_size:
+        g = np.arange(p) // group_size
+        sc, zc = scale.astype(np.float64)[:, g], zero.astype(np.float64)[:, g]
+    else:
+        sc, zc = scale.astype(np.float64)[:, None], zero.astype(np.float64)[:, None]
+    t = r["beta"] / sc[None] + zc[None]
     ideal = np.clip(np.rint(t), 0, maxq)
     got = sweep_codes_gpu.astype(np.float64)
     bad = got != ideal

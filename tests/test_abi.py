@@ -37,10 +37,21 @@ def test_status_strings_and_version(lib):
     assert qe.qe_status_string(99) == "unknown status"
 
 
-def test_opts_struct_matches_header():
-    # 5 ints (padded to 8-byte alignment), 4 pointers, 1 size_t, 1 pointer on LP64
-    assert ctypes.sizeof(qe.QEOpts) == 6 * 4 + 4 * 8 + 8 + 8
-    assert qe.QEOpts.init_codes.offset == 24
+def test_opts_struct_matches_header(tmp_path):
+    """The ctypes mirror of qe_opts has the size and field offsets the C compiler
+    gives the header's struct."""
+    import subprocess
+    fields = [f[0] for f in qe.QEOpts._fields_]
+    src = tmp_path / "opts.c"
+    src.write_text('#include "qe.h"\n#include <stdio.h>\n#include <stddef.h>\nint main(void) {\n'
+                   '    printf("%zu\\n", sizeof(qe_opts));\n'
+                   + "".join(f'    printf("%zu\\n", offsetof(qe_opts, {f}));\n' for f in fields)
+                   + "    return 0;\n}\n")
+    exe = tmp_path / "opts"
+    subprocess.check_call(["gcc", "-std=c11", f"-I{os.path.join(ROOT, 'include')}", "-o", str(exe), str(src)])
+    out = [int(x) for x in subprocess.check_output([str(exe)], text=True).split()]
+    assert out[0] == ctypes.sizeof(qe.QEOpts)
+    assert out[1:] == [getattr(qe.QEOpts, f).offset for f in fields]
 
 
 def _fake(n=1):
@@ -91,6 +102,18 @@ def test_invalid_arguments_rejected_synchronously(lib):
     o.free_changes = -2
     assert L.qe_quantize_layer(_fake(), qe.QE_F32, 4, 4, 4, _fake(2), 3, 1, ctypes.byref(o), _fake(3),
                                _fake(4), _fake(5), _fake(6), None) == qe.QE_ERR_INVALID_ARG
+    o = qe.QEOpts()
+    o.group_size = 100            # not a multiple of the block width (256)
+    assert L.qe_quantize_layer(_fake(), qe.QE_F32, 4, 4, 4, _fake(2), 3, 1, ctypes.byref(o), _fake(3),
+                               _fake(4), _fake(5), _fake(6), None) == qe.QE_ERR_INVALID_ARG
+    o.group_size = 256
+    o.relax_period = 3            # groups and the relax heuristic do not combine
+    assert L.qe_quantize_layer(_fake(), qe.QE_F32, 4, 4, 4, _fake(2), 3, 1, ctypes.byref(o), _fake(3),
+                               _fake(4), _fake(5), _fake(6), None) == qe.QE_ERR_UNSUPPORTED
+    o.relax_period = 0            # nor groups and the outlier variant
+    assert L.qe_quantize_layer_outlier(_fake(), qe.QE_F32, 4, 4, 4, _fake(2), 3, 1, 4, ctypes.byref(o),
+                                       _fake(3), _fake(4), _fake(5), _fake(7), _fake(8), _fake(9), _fake(6),
+                                       None, None) == qe.QE_ERR_UNSUPPORTED
     o = qe.QEOpts()
     o.block_width = 48
     assert L.qe_quantize_layer(_fake(), qe.QE_F32, 4, 4, 4, _fake(2), 3, 1, ctypes.byref(o), _fake(3),

@@ -333,6 +333,47 @@ def test_pack_codes_bit_exact(bits):
         assert torch.equal(qe.qe_unpack_codes(pk, 300, bits), out["codes"])
 
 
+@pytest.mark.parametrize("block_width,group_size", [(256, 256), (128, 128), (128, 256)])
+def test_layer_grouped_grids(block_width, group_size):
+    """Grouped grids (one grid per row and group of columns) against the oracle's
+    grouped Algorithm 1: the per-group scales and zero-points bit for bit,
+    teacher-forced decisions, the objective of the GPU's own state and the
+    free-running objective and codes.  Groups differ in range by a factor 6; p =
+    704 ends on a ragged group."""
+    q, p, bits, iters = 160, 704, 3, 4
+    W = inputs.layer_weights(q, p, dtype=torch.bfloat16, seed=67, device="cuda")
+    W[:, 256:384] *= 6.0
+    X = inputs.calib_inputs(p, 4096, dtype=torch.bfloat16, seed=67, device="cuda", heavy_frac=0.01,
+                            heavy_mult=30.0)
+    Sg = qe.qe_build_sigma(X)
+    out = qe.qe_quantize_layer(W, Sg, bits, iters, record_sweeps=True, block_width=block_width,
+                               group_size=group_size)
+    assert qe.qe_sync_status() == qe.QE_OK
+    W64, S64 = parity.f64(W), parity.f64(Sg)
+    wx = float(np.einsum("ij,jk,ik->", W64, S64, W64))
+    s, z = O.grid(W64, bits, group_size=group_size)
+    assert out["scales"].shape == (q, -(-p // group_size))
+    assert np.array_equal(out["scales"].cpu().numpy(), s) and np.array_equal(out["zeros"].cpu().numpy(), z)
+    sweep = out["sweep_codes"].cpu().numpy()
+    parity.teacher_forced(W64, S64, s, z, bits, sweep, group_size=group_size)
+    forced = O.alg1(W64, S64, s, z, bits, iters, forced=sweep, group_size=group_size)
+    parity.check_obj(out["obj"].cpu().numpy(), forced["obj"], what="objective (GPU state, groups)",
+                     atol=1e-7 * wx)
+    ref = O.alg1(W64, S64, s, z, bits, iters, group_size=group_size)
+    parity.check_obj(out["obj"].cpu().numpy(), ref["obj"], what="objective (free-running, groups)",
+                     atol=1e-7 * wx)
+    m = parity.code_match(out["codes"].cpu().numpy(), ref["codes"])
+    assert m >= parity.CODE_MATCH, f"codes match {m:.5f}"
+
+
+def test_layer_group_of_all_columns_is_the_plain_layer():
+    W, X, Sg, out = _layer_case(96, 300, 1024, torch.bfloat16, 4, 3, seed=68)
+    r = qe.qe_quantize_layer(W, Sg, 4, 3, record_sweeps=True, group_size=512)
+    assert qe.qe_sync_status() == qe.QE_OK
+    assert r["scales"].shape == (96,)
+    assert torch.equal(r["sweep_codes"], out["sweep_codes"]) and torch.equal(r["obj"], out["obj"])
+
+
 def test_layer_dead_columns_round_to_nearest():
     dead = (5, 77, 130)
     W, X, Sg, out = _layer_case(96, 160, 1024, torch.float32, 4, 3, seed=12, zero_rows=dead)
