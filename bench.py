@@ -49,6 +49,8 @@ def parse():
                     help="outlier workloads: keep whole columns (Sec. 4.3, structured outliers)")
     ap.add_argument("--dense-sweeps", type=int, default=0,
                     help="sweeps whose cross-block term uses the tensor-core GEMM (0 = library default)")
+    ap.add_argument("--group-size", type=int, default=0,
+                    help="grouped grids: a scale and zero-point per row and group of this many columns")
     ap.add_argument("--relax", type=int, default=0,
                     help="relax heuristic period R (Sec. 3.2): sweeps t with t mod R = 0, t < iters, unquantized")
     ap.add_argument("--tokens", type=int, default=0,
@@ -329,14 +331,17 @@ def main():
     X = cfg_r.inputs("cuda")
     Sigma = torch.empty(p, p, dtype=torch.float32, device="cuda")
     outlier = cfg.s_budget > 0                    # the outlier-aware workload (Algorithm 4)
-    ws = torch.empty(qe.qe_workspace_size(q, p, outlier=outlier), dtype=torch.uint8, device="cuda")
+    grouped = 0 < args.group_size < p
+    ws = torch.empty(qe.qe_workspace_size(q, p, outlier=outlier, group_size=args.group_size), dtype=torch.uint8,
+                     device="cuda")
 
     def quantize(Wt, b, timer=None):
         if outlier:
             return qe.qe_quantize_layer_outlier(Wt, Sigma, b, cfg.iters, cfg.s_budget, workspace=ws,
                                                 structured=args.structured, timer=timer)
         return qe.qe_quantize_layer(Wt, Sigma, b, cfg.iters, workspace=ws, timer=timer,
-                                    dense_sweeps=args.dense_sweeps, relax_period=args.relax)
+                                    dense_sweeps=args.dense_sweeps, relax_period=args.relax,
+                                    group_size=args.group_size)
     stream = torch.cuda.current_stream()
     nb = len(cfg.bits)
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(nb + 2)]
@@ -402,7 +407,7 @@ def main():
     blocks = [(b0, min(256, p - b0)) for b0 in range(0, p, 256)]
     tri_flops = sum(2 * q * bw * b0 for b0, bw in blocks)
     win_flops = sum(2 * q * bw * p for b0, bw in blocks)
-    dense = cfg.iters if outlier else (args.dense_sweeps or DEFAULT_DENSE_SWEEPS)
+    dense = cfg.iters if (outlier or grouped) else (args.dense_sweeps or DEFAULT_DENSE_SWEEPS)
     if outlier:     # Algorithm 4: sweep 1 blocked, later sweeps take the change lists
         plan, extra_refreshes, list_runs = [("first", 0)] + [("list", 0)] * (cfg.iters - 1), 0, []
     else:
@@ -412,7 +417,7 @@ def main():
         if kind in ("first", "seq", "dense"):
             f = win_flops if window == 1 else tri_flops
             trail_flops += f
-            trail_exec += (3 if kind == "dense" else 6) * f   # three-plane changes: 6 products
+            trail_exec += (3 if kind == "dense" and not grouped else 6) * f   # three-plane changes: 6 products
     # residual GEMMs per layer (besides P): after sweep 1 (or every iteration, Algorithm 4)
     refreshes = (1 if plan[0][0] == "first" else 0) + extra_refreshes
 
@@ -429,6 +434,7 @@ def main():
               "config": {"workload": cfg.name, "q": q, "p": p, "n": n, "bits": list(cfg.bits),
                          "sweeps": cfg.iters, "parallelism": f"layer-replicas x{world}",
                          **({"relax_period": args.relax} if args.relax else {}),
+                         **({"group_size": args.group_size} if grouped else {}),
                          "l2": "inputs larger than L2 (X is %.2f GiB)" % (p * n * 2 / 2**30),
                          **({"s_budget": cfg.s_budget,
                              "outliers": "columns" if args.structured else "entries"} if outlier else {})},
@@ -445,7 +451,8 @@ def main():
     qpad, ppad = -(-q // 128) * 128, -(-p // 256) * 256
     gemm_flops = sig_flops + nb * (2 * q * p * p * (1 + refreshes) + trail_flops)
     gemm_exec = (gemm_tiles_sigma(p) * 2 * 128 * 256 * n
-                 + nb * ((1 + refreshes) * 3 * 2 * qpad * ppad * (-(-p // 64) * 64) + trail_exec))
+                 + nb * ((3 + (6 if grouped else 3) * refreshes) * 2 * qpad * ppad * (-(-p // 64) * 64)
+                         + trail_exec))
     result["roofline"] = roofline_gemm(gemm_flops, gemm_exec, gemm_ms, gemm_launches, pk)
     # ideal step: per phase max(algorithmic flops / tensor peak, algorithmic bytes / HBM), summed
     peak_tf, hbm = pk["bf16_sustained"] * 1e12, pk["hbm"] * 1e9

@@ -136,9 +136,11 @@ def qe_sync_status(stream=None) -> int:
     return load().qe_sync_status(_stream(stream))
 
 
-def qe_workspace_size(q: int, p: int, outlier: bool = False) -> int:
+def qe_workspace_size(q: int, p: int, outlier: bool = False, group_size: int = 0,
+                      block_width: int = 0) -> int:
     out = ctypes.c_size_t(0)
-    _check(load().qe_workspace_size(q, p, int(outlier), None, ctypes.byref(out)), "qe_workspace_size")
+    o = _opts(block_width, group_size=group_size)
+    _check(load().qe_workspace_size(q, p, int(outlier), ctypes.byref(o), ctypes.byref(out)), "qe_workspace_size")
     return out.value
 
 

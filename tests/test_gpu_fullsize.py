@@ -130,6 +130,43 @@ def test_fullsize_layer_sampled_rows(name, nrows, free_run, full_obj):
         torch.cuda.empty_cache()
 
 
+def test_fullsize_grouped_grids():
+    """Grouped grids (groups of 256 columns) on the 4096 x 4096 projection in the bench
+    configuration: per-group grids bit for bit on sampled rows, teacher-forced
+    decisions and the sampled rows' objective against the oracle's grouped
+    Algorithm 1 (fed the GPU's Sigma), a non-increasing objective, and the objective
+    of the final codes recomputed in fp64."""
+    cfg = inputs.CONFIGS["llama7b_proj_4096x4096"]
+    q, p, G, bits = cfg.q, cfg.p, 256, 3
+    rng = np.random.default_rng(2310)
+    W = inputs.layer_weights(q, p, dtype=cfg.w_dtype, seed=cfg.seed, device="cuda")
+    X = inputs.calib_inputs(p, cfg.n, dtype=cfg.x_dtype, seed=cfg.seed, device="cuda",
+                            heavy_frac=cfg.heavy_frac, heavy_mult=cfg.heavy_mult)
+    Sg = qe.qe_build_sigma(X)
+    del X
+    out = qe.qe_quantize_layer(W, Sg, bits, cfg.iters, record_sweeps=True, group_size=G)
+    assert qe.qe_sync_status() == qe.QE_OK
+    obj = out["obj"].cpu().numpy()
+    assert np.all(np.diff(obj) <= 1e-6 * obj[:-1]), "objective not monotone"
+    rows = np.sort(rng.choice(q, size=24, replace=False))
+    rows_t = torch.from_numpy(rows).cuda()
+    W64 = W[rows_t].double().cpu().numpy()
+    S64 = Sg.double().cpu().numpy()
+    s, z = O.grid(W64, bits, group_size=G)
+    assert np.array_equal(out["scales"][rows_t].cpu().numpy(), s)
+    assert np.array_equal(out["zeros"][rows_t].cpu().numpy(), z)
+    sweep = out["sweep_codes"][:, rows_t, :].cpu().numpy()
+    _, _, forced = parity.teacher_forced(W64, S64, s, z, bits, sweep, want_run=True, group_size=G)
+    ref = O.alg1(W64, S64, s, z, bits, cfg.iters, group_size=G)
+    parity.check_obj(forced["obj"], ref["obj"], what="sampled-row objective (groups)")
+    # the whole objective of the final codes in fp64
+    g = torch.arange(p, device="cuda") // G
+    sc, zc = out["scales"].double()[:, g], out["zeros"].double()[:, g]
+    D = W.double() - sc * (out["codes"].double() - zc)
+    f = sum(float(torch.sum((D[r0:r0 + 2048] @ Sg.double()) * D[r0:r0 + 2048]).item()) for r0 in range(0, q, 2048))
+    parity.check_obj(obj[-1], f, what="objective of the final codes (fp64, groups)")
+
+
 @pytest.mark.parametrize("name,structured", [("llama7b_proj_outlier_4096x4096", False),
                                              ("llama7b_proj_outlier_4096x4096", True),
                                              ("llama7b_proj_outlier2b_4096x4096", False)],
