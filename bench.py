@@ -407,7 +407,7 @@ def main():
     blocks = [(b0, min(256, p - b0)) for b0 in range(0, p, 256)]
     tri_flops = sum(2 * q * bw * b0 for b0, bw in blocks)
     win_flops = sum(2 * q * bw * p for b0, bw in blocks)
-    dense = cfg.iters if (outlier or grouped) else (args.dense_sweeps or DEFAULT_DENSE_SWEEPS)
+    dense = cfg.iters if outlier else (args.dense_sweeps or DEFAULT_DENSE_SWEEPS)
     if outlier:     # Algorithm 4: sweep 1 blocked, later sweeps take the change lists
         plan, extra_refreshes, list_runs = [("first", 0)] + [("list", 0)] * (cfg.iters - 1), 0, []
     else:

@@ -105,9 +105,8 @@ typedef struct {
      * zero-point per group of G consecutive columns, and the call's `scales` /
      * `zeros` hold q x ceil(p / G) values, row-major ([i * groups + j / G]).
      * 0 (or G >= p) = one grid per row.  G must be a multiple of the block width
-     * (QE_ERR_INVALID_ARG otherwise); with G < p every sweep after the first takes
-     * the tensor-core form of the cross-block term (dense_sweeps has no effect),
-     * and relax_period != 0 or the outlier variant return QE_ERR_UNSUPPORTED. */
+     * (QE_ERR_INVALID_ARG otherwise); relax_period != 0 or the outlier variant
+     * return QE_ERR_UNSUPPORTED with G < p. */
     int group_size;
     /* Optional warm start (Sec. 3.1, "initialized with ... any other algorithm"):
      * q x p codes (leading dimension p) on the grid this call computes.  NULL = start at W. */

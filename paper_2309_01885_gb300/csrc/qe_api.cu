@@ -825,9 +825,7 @@ qe_status qe_quantize_layer(const void *W, qe_dtype w_dtype, int64_t q, int64_t 
     if ((st = restart(src == SRC_CODES ? 1 : 3)) != QE_OK) return st;
     bool exact = true;   // R is the residual of the current What and no list has entries
     bool chain = false;  // the last sweep was a sequential one (its three-plane changes are in dp)
-    // grouped grids: the change lists assume one scale per row, so every sweep takes the
-    // tensor-core form of the window
-    const int dense = pl.grouped ? iters : dense_sweeps(opts);
+    const int dense = dense_sweeps(opts);
     while (t < iters) {
         const bool rx = relaxed(t);
         if (rx || src != SRC_CODES) {

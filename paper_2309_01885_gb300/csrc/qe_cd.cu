@@ -336,7 +336,7 @@ struct CdCfg {
 // contiguous over the block, so each change is one coalesced read of B floats
 // per warp.  Returns whether the row had any change in the window.  Lists of
 // blocks below bmin are left out.
-template <int B, bool FULL, int U = 4>
+template <int B, bool FULL, int U = 4, bool GR = false>
 __device__ __forceinline__ bool list_correction(const CdArgs &a, int64_t b0, int bw_, int64_t ii, bool row_ok,
                                                 int lane, float (&ps)[B / 32], int bmin = 0) {
     constexpr int CPL = B / 32;
@@ -355,6 +355,9 @@ __device__ __forceinline__ bool list_correction(const CdArgs &a, int64_t b0, int
             const int64_t blk2 = c0 + sl;
             const uint32_t *seg = a.lent + (rb + blk2) * B;
             const float *sbk = sb0 + blk2 * B * a.lds;
+            // grouped grids: the listed changes are in the grid units of their own group
+            float fac = 1.0f;
+            if (GR) fac = __fdiv_rn(a.scale[ii * a.ngroups + blk2 * B / a.gsize], a.scale[ii * a.ngroups + b0 / a.gsize]);
             for (int e0 = 0; e0 < c; e0 += 32) {
                 const uint32_t mine = (e0 + lane < c) ? seg[e0 + lane] : 0u;
                 const int ne = (c - e0) < 32 ? (c - e0) : 32;
@@ -368,7 +371,7 @@ __device__ __forceinline__ bool list_correction(const CdArgs &a, int64_t b0, int
                     for (int e = 0; e < U; ++e) {
                         const uint32_t ev = __shfl_sync(0xffffffffu, mine, u + e);
                         r[e] = sbk + static_cast<int64_t>(ev & 0xffffu) * a.lds;
-                        dv[e] = static_cast<float>(static_cast<int16_t>(ev >> 16));
+                        dv[e] = static_cast<float>(static_cast<int16_t>(ev >> 16)) * fac;
                     }
                     float v[U][CPL];
 #pragma unroll
@@ -384,7 +387,7 @@ __device__ __forceinline__ bool list_correction(const CdArgs &a, int64_t b0, int
                 for (; u < ne; ++u) {
                     const uint32_t e1 = __shfl_sync(0xffffffffu, mine, u);
                     const float *r1 = sbk + static_cast<int64_t>(e1 & 0xffffu) * a.lds;
-                    const float d1 = static_cast<float>(static_cast<int16_t>(e1 >> 16));
+                    const float d1 = static_cast<float>(static_cast<int16_t>(e1 >> 16)) * fac;
 #pragma unroll
                     for (int h = 0; h < CPL; ++h)
                         if (FULL || 32 * h + lane < bw) ps[h] = fmaf(d1, __ldg(r1 + 32 * h), ps[h]);
@@ -465,16 +468,18 @@ __device__ __forceinline__ bool cd_prologue(const CdArgs &a, float *tri, uint64_
 }
 
 // Common epilogue: codes, C - z (both skipped for unchanged columns when
-// skip_same) and the Delta' plane(s).
-template <int B, bool FULL, bool RECORD>
+// skip_same) and the Delta' plane(s).  G = false: never grouped grids (one
+// scale per row, no group logic compiled in); G = true: as a.grouped says.
+template <int B, bool FULL, bool RECORD, bool G = true>
 __device__ __forceinline__ void cd_epilogue(const CdArgs &a, int64_t b0, int bw_, int64_t i, int lane,
                                             const float (&code)[B / 32], const float (&dlt)[B / 32],
                                             bool skip_same) {
     constexpr int CPL = B / 32;
     const int bw = FULL ? B : bw_;
-    const int64_t gi = i * a.ngroups + b0 / a.gsize;   // the block lies in one group
+    const bool grouped = G && a.grouped;
+    const int64_t gi = G ? i * a.ngroups + b0 / a.gsize : i;   // the block lies in one group
     const float z = a.zero[gi];
-    const float sg = a.grouped ? a.scale[gi] : 1.0f;
+    const float sg = grouped ? a.scale[gi] : 1.0f;
 #pragma unroll
     for (int h = 0; h < CPL; ++h) {
         const int l = 32 * h + lane;
@@ -486,7 +491,7 @@ __device__ __forceinline__ void cd_epilogue(const CdArgs &a, int64_t b0, int bw_
         } else if (!skip_same || dlt[h] != 0.0f) {
             a.codes[i * a.ldc + col] = static_cast<uint8_t>(code[h]);
             if (a.write_qf) {
-                if (!a.grouped) {
+                if (!grouped) {
                     a.qf[i * a.ldq + col] = __float2bfloat16_rn(code[h] - z);
                 } else {   // the residual GEMM takes s_g (C - z_g), three planes
                     __nv_bfloat16 qh, qm, ql;
@@ -500,10 +505,10 @@ __device__ __forceinline__ void cd_epilogue(const CdArgs &a, int64_t b0, int bw_
         if (!a.dp) continue;
         // grouped: the trailing GEMM sums changes of several groups, so it takes them
         // absolute (s_g Delta'), which is not an integer: three planes
-        const float dv = a.grouped ? sg * dlt[h] : dlt[h];
+        const float dv = grouped ? sg * dlt[h] : dlt[h];
         const __nv_bfloat16 hi = __float2bfloat16_rn(dv);
         a.dp[i * a.ldd + col] = hi;
-        if (a.frac || a.grouped) {   // Delta' is not an integer: three planes
+        if (a.frac || grouped) {   // Delta' is not an integer: three planes
             const float r1 = dv - __bfloat162float(hi);
             const __nv_bfloat16 mid = __float2bfloat16_rn(r1);
             a.dp[(a.dp_plane_rows + i) * a.ldd + col] = mid;
@@ -740,13 +745,18 @@ __global__ void __launch_bounds__(1024, 1) k_cd_block_chg(const CdArgs a) {
 // change-list correction (storing it back as the block's base when the window
 // held a change), wait for the block's packed Sigma_bar, decide, write back.
 // Returns false when the wait gave up.
-template <int B, bool FULL, bool LATE>
+template <int B, bool FULL, bool LATE, bool GR = false>
 __device__ __forceinline__ bool rows_block(const CdArgs &a, int64_t b0, int bw_, const float *tri, uint64_t *bar,
-                                           uint32_t parity, int64_t i, bool row_ok, int lane, float s2,
+                                           uint32_t parity, int64_t i, bool row_ok, int lane, float s2_row,
                                            double &dfacc, int &nchg) {
     constexpr int CPL = B / 32;
     const int bw = FULL ? B : bw_;
     const int64_t ii = row_ok ? i : 0;
+    float s2 = s2_row;   // grouped grids: the scale of the block's group
+    if (GR) {
+        const float sb = a.scale[ii * a.ngroups + b0 / a.gsize];
+        s2 = sb * sb;
+    }
     float ps[CPL], st[CPL], t[CPL];
 #pragma unroll
     for (int h = 0; h < CPL; ++h) ps[h] = 0.0f;
@@ -761,12 +771,12 @@ __device__ __forceinline__ bool rows_block(const CdArgs &a, int64_t b0, int bw_,
             t[h] = ok ? __ldcs(a.R + ii * a.ldr + b0 + l) : 0.0f;
             st[h] = ok ? static_cast<float>(__ldcs(a.codes + ii * a.ldc + b0 + l)) : 0.0f;
         }
-        changed = list_correction<B, FULL, 2>(a, b0, bw, ii, row_ok, lane, ps);
+        changed = list_correction<B, FULL, 2, GR>(a, b0, bw, ii, row_ok, lane, ps);
 #pragma unroll
         for (int h = 0; h < CPL; ++h) t[h] += ps[h];
     } else {
         // the gathers first (many changes: they hold the registers), then base and codes
-        changed = list_correction<B, FULL>(a, b0, bw, ii, row_ok, lane, ps);
+        changed = list_correction<B, FULL, 4, GR>(a, b0, bw, ii, row_ok, lane, ps);
 #pragma unroll
         for (int h = 0; h < CPL; ++h) {
             const int l = 32 * h + lane;
@@ -787,7 +797,7 @@ __device__ __forceinline__ bool rows_block(const CdArgs &a, int64_t b0, int bw_,
     float code[CPL], dlt[CPL];
     nchg += chg_decide<B, FULL, LATE>(tri, a.d + b0, bw, a.maxq, s2, true, lane, t, st, code, dlt, dfacc,
                                       a.sbar + b0 * a.lds + b0, a.lds);
-    cd_epilogue<B, FULL, true>(a, b0, bw, i, lane, code, dlt, true);
+    cd_epilogue<B, FULL, true, GR>(a, b0, bw, i, lane, code, dlt, true);
     return true;
 }
 
@@ -851,13 +861,19 @@ __device__ __forceinline__ int build_window(const CdArgs &a, int64_t i, int lane
 // so the same sums), then this block's entries in the window are replaced by
 // the changes just made.  The lists in global memory are written as well, so a
 // window that outgrows kWinCap (wn = -1) hands over to them.
-template <int B, bool FULL>
-__device__ __forceinline__ void rows_block_win(const CdArgs &a, int64_t b0, int bw_, int64_t i, int lane, float s2,
-                                               double &dfacc, int &nchg, uint32_t *win, float *stg, int &wn) {
+template <int B, bool FULL, bool GR = false>
+__device__ __forceinline__ void rows_block_win(const CdArgs &a, int64_t b0, int bw_, int64_t i, int lane,
+                                               float s2_row, double &dfacc, int &nchg, uint32_t *win, float *stg,
+                                               int &wn) {
     constexpr int CPL = B / 32;
     constexpr int NST = kStageFloats / B;       // segments per staged batch
     constexpr int SEG16 = B / 4;                // 16-byte pieces per segment
     const int bw = FULL ? B : bw_;
+    float s2 = s2_row, sblk = 1.0f;   // grouped grids: the scale of the block's group
+    if (GR) {
+        sblk = a.scale[i * a.ngroups + b0 / a.gsize];
+        s2 = sblk * sblk;
+    }
     float ps[CPL], st[CPL], t[CPL];
 #pragma unroll
     for (int h = 0; h < CPL; ++h) {
@@ -878,7 +894,11 @@ __device__ __forceinline__ void rows_block_win(const CdArgs &a, int64_t b0, int 
         cp_async_wait_all();
         __syncwarp();
         for (int e = 0; e < nb; ++e) {
-            const float dv = static_cast<float>(static_cast<int16_t>(win[u0 + e] >> 16));
+            // grouped grids: the change is in the grid units of its own group (the same
+            // factor list_correction applies per list)
+            float fac = 1.0f;
+            if (GR) fac = __fdiv_rn(a.scale[i * a.ngroups + (win[u0 + e] & 0xffffu) / a.gsize], sblk);
+            const float dv = static_cast<float>(static_cast<int16_t>(win[u0 + e] >> 16)) * fac;
 #pragma unroll
             for (int h = 0; h < CPL; ++h)
                 if (FULL || 32 * h + lane < bw) ps[h] = fmaf(dv, stg[e * B + 32 * h + lane], ps[h]);
@@ -897,7 +917,7 @@ __device__ __forceinline__ void rows_block_win(const CdArgs &a, int64_t b0, int 
     float code[CPL], dlt[CPL];
     nchg += chg_decide<B, FULL, true>(nullptr, a.d + b0, bw, a.maxq, s2, true, lane, t, st, code, dlt, dfacc,
                                       a.sbar + b0 * a.lds + b0, a.lds);
-    cd_epilogue<B, FULL, true>(a, b0, bw, i, lane, code, dlt, true);
+    cd_epilogue<B, FULL, true, GR>(a, b0, bw, i, lane, code, dlt, true);
     // window = [entries left of the block (k1)] [this visit's changes (nn)] [entries right of it]
     int k1 = 0, k2 = 0;
 #pragma unroll
@@ -967,7 +987,7 @@ __device__ __forceinline__ void rows_block_win(const CdArgs &a, int64_t b0, int 
 // of the final codes.
 constexpr int kRowsMaxWarps = 28;   // rows per CTA of the persistent kernel (896 threads: 72 registers)
 
-template <int B>
+template <int B, bool GR>
 __global__ void __launch_bounds__(32 * kRowsMaxWarps, 1) k_cd_rows_lists(const CdArgs a, int t_begin, int t_end,
                                                            double *rowdf_t, uint8_t *sweep_codes,
                                                            int first_lockstep, int free_max_changes, int flush) {
@@ -1028,13 +1048,13 @@ __global__ void __launch_bounds__(32 * kRowsMaxWarps, 1) k_cd_rows_lists(const C
                     const int bw = static_cast<int>((a.p - b0) < B ? (a.p - b0) : B);
                     if (wn >= 0) {
                         if (bw == B)
-                            rows_block_win<B, true>(a, b0, bw, i, lane, s2, dfacc, nchg, win, stg, wn);
+                            rows_block_win<B, true, GR>(a, b0, bw, i, lane, s2, dfacc, nchg, win, stg, wn);
                         else
-                            rows_block_win<B, false>(a, b0, bw, i, lane, s2, dfacc, nchg, win, stg, wn);
+                            rows_block_win<B, false, GR>(a, b0, bw, i, lane, s2, dfacc, nchg, win, stg, wn);
                     } else if (bw == B) {
-                        rows_block<B, true, true>(a, b0, bw, tri, bar, 0u, i, row_ok, lane, s2, dfacc, nchg);
+                        rows_block<B, true, true, GR>(a, b0, bw, tri, bar, 0u, i, row_ok, lane, s2, dfacc, nchg);
                     } else {
-                        rows_block<B, false, true>(a, b0, bw, tri, bar, 0u, i, row_ok, lane, s2, dfacc, nchg);
+                        rows_block<B, false, true, GR>(a, b0, bw, tri, bar, 0u, i, row_ok, lane, s2, dfacc, nchg);
                     }
                 }
             }
@@ -1048,8 +1068,8 @@ __global__ void __launch_bounds__(32 * kRowsMaxWarps, 1) k_cd_rows_lists(const C
                 }
                 const bool ok =
                     bw == B
-                        ? rows_block<B, true, false>(a, b0, bw, tri, bar, use & 1u, i, row_ok, lane, s2, dfacc, nchg)
-                        : rows_block<B, false, false>(a, b0, bw, tri, bar, use & 1u, i, row_ok, lane, s2, dfacc,
+                        ? rows_block<B, true, false, GR>(a, b0, bw, tri, bar, use & 1u, i, row_ok, lane, s2, dfacc, nchg)
+                        : rows_block<B, false, false, GR>(a, b0, bw, tri, bar, use & 1u, i, row_ok, lane, s2, dfacc,
                                                       nchg);
                 ++use;
                 if (!ok) {
@@ -1082,8 +1102,8 @@ __global__ void __launch_bounds__(32 * kRowsMaxWarps, 1) k_cd_rows_lists(const C
 #pragma unroll
             for (int h = 0; h < CPL; ++h) ps[h] = 0.0f;
             const int bmin = static_cast<int>(b0 / B);
-            const bool any = bw == B ? list_correction<B, true>(a, b0, bw, i, true, lane, ps, bmin)
-                                     : list_correction<B, false>(a, b0, bw, i, true, lane, ps, bmin);
+            const bool any = bw == B ? list_correction<B, true, 4, GR>(a, b0, bw, i, true, lane, ps, bmin)
+                                     : list_correction<B, false, 4, GR>(a, b0, bw, i, true, lane, ps, bmin);
             if (!any) continue;
 #pragma unroll
             for (int h = 0; h < CPL; ++h) {
@@ -1158,7 +1178,7 @@ cudaError_t launch_cd_block(int B, const CdArgs &a, int nsm, cudaStream_t s) {
 
 int64_t packed_diag_floats(int64_t p, int B) { return ceil_div(p, B) * packed_block_floats(B); }
 
-template <int B>
+template <int B, bool GR>
 static cudaError_t launch_cd_rows_b(const CdArgs &a, int t_begin, int t_end, double *rowdf_t,
                                    uint8_t *sweep_codes, int first_lockstep, int free_max_changes, int flush,
                                    int nsm, cudaStream_t s) {
@@ -1168,10 +1188,10 @@ static cudaError_t launch_cd_rows_b(const CdArgs &a, int t_begin, int t_end, dou
     if (warps < 1) warps = 1;
     // the packed block (lockstep) or one free-mode area per warp, whichever is larger
     const int smem = static_cast<int>(warps * kFreeWarpBytes > C::SMEM ? warps * kFreeWarpBytes : C::SMEM);
-    cudaError_t e = cudaFuncSetAttribute(k_cd_rows_lists<B>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaError_t e = cudaFuncSetAttribute(k_cd_rows_lists<B, GR>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     const unsigned grid = static_cast<unsigned>(ceil_div(a.q, warps));
-    k_cd_rows_lists<B><<<grid, static_cast<unsigned>(32 * warps), smem, s>>>(
+    k_cd_rows_lists<B, GR><<<grid, static_cast<unsigned>(32 * warps), smem, s>>>(
         a, t_begin, t_end, rowdf_t, sweep_codes, first_lockstep, free_max_changes, flush);
     return cudaGetLastError();
 }
@@ -1182,9 +1202,15 @@ cudaError_t launch_cd_rows_lists(int B, const CdArgs &a, int t_begin, int t_end,
     if (!a.sbar || !a.lent || !a.lcnt || a.first_sweep || t_end <= t_begin) return cudaErrorInvalidValue;
     const int f = first_lockstep, m = free_max_changes, fl = flush;
     switch (B) {
-        case 64: return launch_cd_rows_b<64>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, fl, nsm, s);
-        case 128: return launch_cd_rows_b<128>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, fl, nsm, s);
-        case 256: return launch_cd_rows_b<256>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, fl, nsm, s);
+        case 64:
+            return a.grouped ? launch_cd_rows_b<64, true>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, fl, nsm, s)
+                             : launch_cd_rows_b<64, false>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, fl, nsm, s);
+        case 128:
+            return a.grouped ? launch_cd_rows_b<128, true>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, fl, nsm, s)
+                             : launch_cd_rows_b<128, false>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, fl, nsm, s);
+        case 256:
+            return a.grouped ? launch_cd_rows_b<256, true>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, fl, nsm, s)
+                             : launch_cd_rows_b<256, false>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, fl, nsm, s);
         default: return cudaErrorInvalidValue;
     }
 }

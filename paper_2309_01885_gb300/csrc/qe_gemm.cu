@@ -59,6 +59,9 @@ __device__ __forceinline__ float load_w(const GemmArgs &g, int64_t r, int64_t c)
 
 // Epilogue for one thread: output row r, columns [c0, c0 + 32) of the window.
 // `objacc` collects the fused objective terms of EPI_RFULL (when requested).
+// GR: grouped grids possible (per-group scales, the absolute residual form); the
+// per-row kernel is compiled without them.
+template <bool GR>
 __device__ __forceinline__ void epilogue_row(const GemmArgs &g, int r, int c0, const float (&v)[32],
                                              int split, double &objacc) {
     if (r >= g.M) return;
@@ -95,14 +98,14 @@ __device__ __forceinline__ void epilogue_row(const GemmArgs &g, int r, int c0, c
             // R in grid-step units: (P - s (C - z) Sigma_bar) / s + z = P / s - acc + z; with
             // grouped grids (absolute) acc = s_g (C - z_g) Sigma_bar, R = (P - acc) / s_g + z_g
             // (the 32 columns lie in one group)
-            const int64_t gi = g.ngroups > 1 ? rr * g.ngroups + c0 / g.gsize : rr;
+            const int64_t gi = (GR && g.ngroups > 1) ? rr * g.ngroups + c0 / g.gsize : rr;
             const float s = g.scale[gi];
             const float zz = g.zero[gi];
             const float *prow = g.P + rr * g.ldp;
             float *orow = g.out + rr * g.ldo;
             float o[32];
             const bool full = c0 + 32 <= g.N;
-            if (g.absolute) {
+            if (GR && g.absolute) {
 #pragma unroll
                 for (int i = 0; i < 32; ++i) {
                     const int c = c0 + i;
@@ -335,7 +338,7 @@ __device__ __forceinline__ void epilogue_rows(const GemmArgs &g, float *stg, int
     }
 }
 
-template <int BN>
+template <int BN, bool GR>
 __global__ void __launch_bounds__(320, 1)
     k_tc_gemm(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb,
               const GemmArgs g) {
@@ -488,7 +491,7 @@ __global__ void __launch_bounds__(320, 1)
                         float v[32];
 #pragma unroll
                         for (int i = 0; i < 32; ++i) v[i] = acc[q * 32 + i];
-                        epilogue_row(g, r, c0, v, split, objacc);
+                        epilogue_row<GR>(g, r, c0, v, split, objacc);
                     }
                 }
             } else {
@@ -541,16 +544,16 @@ bool make_tmap_bf16(CUtensorMap *map, const void *base, uint64_t rows, uint64_t 
     return r == CUDA_SUCCESS;
 }
 
-template <int BN>
+template <int BN, bool GR>
 static cudaError_t launch_bn(const CUtensorMap &ta, const CUtensorMap &tb, const GemmArgs &g,
                              int splits, cudaStream_t s) {
     using C = GemmCfg<BN>;
-    cudaError_t e = cudaFuncSetAttribute(k_tc_gemm<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(k_tc_gemm<BN, GR>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          C::SMEM_BYTES);
     if (e != cudaSuccess) return e;
     const unsigned nt = static_cast<unsigned>(ceil_div(g.N, BN)), mt = static_cast<unsigned>(ceil_div(g.M, C::BM));
     dim3 grid(g.m_fast ? mt : nt, g.m_fast ? nt : mt, static_cast<unsigned>(splits));
-    k_tc_gemm<BN><<<grid, C::THREADS, C::SMEM_BYTES, s>>>(ta, tb, g);
+    k_tc_gemm<BN, GR><<<grid, C::THREADS, C::SMEM_BYTES, s>>>(ta, tb, g);
     return cudaGetLastError();
 }
 
@@ -560,9 +563,11 @@ cudaError_t launch_tc_gemm(int BN, const CUtensorMap &ta, const CUtensorMap &tb,
         return cudaErrorInvalidValue;
     if ((g.m_fast ? ceil_div(g.N, BN) : ceil_div(g.M, 128)) > 65535 || splits > 65535) return cudaErrorInvalidValue;
     switch (BN) {
-        case 64: return launch_bn<64>(ta, tb, g, splits, s);
-        case 128: return launch_bn<128>(ta, tb, g, splits, s);
-        case 256: return launch_bn<256>(ta, tb, g, splits, s);
+        case 64: return launch_bn<64, false>(ta, tb, g, splits, s);
+        case 128: return launch_bn<128, false>(ta, tb, g, splits, s);
+        case 256:   // grouped grids only reach the residual GEMM, which runs 128 x 256 tiles
+            return (g.ngroups > 1 || g.absolute) ? launch_bn<256, true>(ta, tb, g, splits, s)
+                                                 : launch_bn<256, false>(ta, tb, g, splits, s);
         default: return cudaErrorInvalidValue;
     }
 }
