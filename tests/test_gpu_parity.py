@@ -250,19 +250,21 @@ def test_layer_lists_agree_with_dense():
     assert m >= parity.CODE_MATCH, f"codes match {m:.5f}"
 
 
-@pytest.mark.parametrize("p", [640, 1000])
-def test_layer_list_modes_identical(p):
+@pytest.mark.parametrize("p,group_size", [(640, 0), (1000, 0), (1000, 256)])
+def test_layer_list_modes_identical(p, group_size):
     """The list sweeps in lockstep (shared packed Sigma_bar block, lists read from
     global memory) and row by row (coupling rows from global Sigma_bar, the window
     held in registers while it fits one entry per lane) take the same decisions in
     the same order: codes, every sweep's codes and the objective are identical.
-    p = 1000 ends on a ragged block."""
+    p = 1000 ends on a ragged block; with grouped grids every change is scaled into
+    the block's group the same way in both modes."""
     q = 512
     W = inputs.layer_weights(q, p, dtype=torch.bfloat16, seed=63, device="cuda")
     X = inputs.calib_inputs(p, 8192, dtype=torch.bfloat16, seed=63, device="cuda",
                             heavy_frac=0.01, heavy_mult=30.0)
     Sg = qe.qe_build_sigma(X)
-    runs = [qe.qe_quantize_layer(W, Sg, 3, 12, record_sweeps=True, free_changes=f) for f in (-1, 0, 100000)]
+    runs = [qe.qe_quantize_layer(W, Sg, 3, 12, record_sweeps=True, free_changes=f, group_size=group_size)
+            for f in (-1, 0, 100000)]
     assert qe.qe_sync_status() == qe.QE_OK
     ref = runs[0]
     for r in runs[1:]:
