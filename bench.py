@@ -510,14 +510,14 @@ def main():
         elif kind in ("seq", "dense"):
             per_layer += (nblk if window == 1 else nblk - 1) + nblk + 1
     if outlier:
-        # selection (P_s: 4 radix passes x 2 + count, scan, emit; columns: + 2 norm
+        # selection (P_s: 3 radix digit passes + count, scan, emit; columns: + 2 norm
         # kernels + emit), start: copy, selection, scatter + row pointers, grid,
         # Sigma_bar set-up (5) + [W planes] + P, 64 power steps (+ fill, last, final),
         # SpMM refresh, initial residual; sweep 1 blocked (2 nblk - 1), later sweeps one
         # change-list launch (ending with the flush of its window into R) and an
         # objective prefix, sweep 1 a residual GEMM + objective sum; per iteration: IHT
         # target, selection, scatter + row pointers, SpMM, objective (2)
-        sel = 14 if args.structured else 11
+        sel = 9 if args.structured else 6
         per_layer = (1 + sel + 2 + 1 + 6 + w_planes + 67 + 1 + 1 + (2 * nblk - 1) + 2 * (cfg.iters - 1) + 2
                      + cfg.iters * (1 + sel + 2 + 1 + 2))
     result["gpu_launches"] = args.steps * (1 + nb * per_layer)

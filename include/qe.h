@@ -289,6 +289,26 @@ qe_status qe_pack_codes(const uint8_t *codes, int64_t q, int64_t p, int64_t ldc,
 qe_status qe_unpack_codes(const uint8_t *packed, int64_t q, int64_t p, int64_t ldp, int bits, uint8_t *codes,
                           int64_t ldc, qe_stream_t stream);
 
+/*
+ * P_s of the IHT step (Sec. 4.3, Eq. iht-update) on its own: of the N entries
+ * of T, keep the s of largest magnitude.  Exact zeros are never kept; among
+ * entries of equal magnitude at the threshold the smaller index goes first.
+ * The operator qe_quantize_layer_outlier applies once per iteration.
+ *   T          device, N fp32 values (any alignment; 16-byte aligned is faster).
+ *   s          0 <= s <= N.
+ *   idx, val   device, s int64 / s fp32 (may be NULL when s = 0): the kept
+ *              indices in ascending order and their values T[idx[k]].
+ *   nnz        device, one int64: the number kept (min(s, nonzeros of T)).
+ *   workspace  device scratch of qe_hard_threshold_workspace(N) bytes,
+ *              256-byte aligned, owned by the caller, not used across calls.
+ * Stream-ordered.  QE_ERR_INVALID_ARG for NULL pointers, N < 1 or N >= 2^32,
+ * s outside 0 .. N, or a short or misaligned workspace (before anything is
+ * enqueued); QE_ERR_CUDA when a launch fails.
+ */
+qe_status qe_hard_threshold_workspace(int64_t N, size_t *bytes);
+qe_status qe_hard_threshold(const float *T, int64_t N, int64_t s, int64_t *idx, float *val, int64_t *nnz,
+                            void *workspace, size_t workspace_bytes, qe_stream_t stream);
+
 /* Waits for `stream`, then returns and clears the error latched on the current
  * device (QE_ERR_NUMERIC / QE_ERR_TIMEOUT), or QE_ERR_CUDA if the stream failed. */
 qe_status qe_sync_status(qe_stream_t stream);

@@ -21,7 +21,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 OUT_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(OUT_DIR, "libqe.so")
-SOURCES = ["qe_api.cu", "qe_gemm.cu", "qe_cd.cu", "qe_outlier.cu", "qe_noalloc.cu", "qe_stream.cu", "qe_pack.cu"]
+SOURCES = ["qe_api.cu", "qe_gemm.cu", "qe_cd.cu", "qe_outlier.cu", "qe_noalloc.cu", "qe_stream.cu", "qe_pack.cu", "qe_select.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
               f"-I{os.path.join(ROOT, 'include')}", f"-I{CSRC}"]

@@ -48,7 +48,7 @@ __device__ __forceinline__ unsigned block_excl_scan(unsigned v, unsigned *sh, un
     return warp_base + x - v;
 }
 
-// ---- power method (Sec. 4.3: lambda_max(X X^T) "by iterative power method") --
+// ---- power method (Sec. 4.3: lambda_max(X X^T) by power iteration) ----------
 // y_out = Sigma (y_in / ||y_in||).  ||y_in||^2 is the sum of the per-CTA
 // partials the previous step left in part_in (nparts of them, added in a fixed
 // order, so the result is reproducible), or is computed here when part_in is
@@ -168,68 +168,151 @@ __global__ void k_flat_copy(const void *W, int w_bf16, int64_t ldw, int64_t q, i
 
 // ---- P_s: radix select of the s-th largest nonzero |T| ----------------------
 // Keys are the binary32 magnitudes (sign bit cleared): for non-negative floats
-// the unsigned bit pattern orders like the value.  Four 8-bit digit passes find
-// kstar; then exactly count_gt keys are > kstar and need_eq keys == kstar are
-// taken in ascending linear index (the tie rule).
+// the unsigned bit pattern orders like the value.  Three digit passes (bits
+// 30..20, 19..9, 8..0) find kstar; then exactly count_gt keys are > kstar and
+// need_eq keys == kstar are taken in ascending linear index (the tie rule).
 __device__ __forceinline__ unsigned mag_key(float v) { return __float_as_uint(v) & 0x7fffffffu; }
 
-__global__ void __launch_bounds__(256) k_topk_hist(const float *T, int64_t N, TopkState *st, int shift,
-                                                   unsigned mask_hi) {
-    __shared__ unsigned h[256];
-    h[threadIdx.x] = 0;
-    __syncthreads();
-    const unsigned prefix = st->prefix;
-    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < N; e += stride) {
-        const unsigned k = mag_key(T[e]);
-        if (k == 0u || ((k ^ prefix) & mask_hi) != 0u) continue;
-        atomicAdd(&h[(k >> shift) & 255u], 1u);
-    }
-    __syncthreads();
-    if (h[threadIdx.x]) atomicAdd(&st->hist[threadIdx.x], h[threadIdx.x]);
-}
+constexpr int kHistThreads = 256;
+__host__ __device__ constexpr int topk_shift(int pass) { return pass == 0 ? 20 : (pass == 1 ? 9 : 0); }
+__host__ __device__ constexpr int topk_bins(int pass) { return pass == 2 ? 512 : kTopkBins; }
+// Key bits fixed before the pass.
+__host__ __device__ constexpr unsigned topk_fixed(int pass) { return pass == 0 ? 0u : (pass == 1 ? 0x7ff00000u : 0x7ffffe00u); }
 
-__global__ void k_topk_pick(TopkState *st, int shift, int64_t s_budget, int first) {
-    if (threadIdx.x != 0) return;
-    if (first) {
-        unsigned long long total = 0;
-        for (int b = 0; b < 256; ++b) total += st->hist[b];
-        st->count_gt = 0;
-        st->prefix = 0;
-        const unsigned long long want = (unsigned long long)s_budget < total ? (unsigned long long)s_budget : total;
-        st->remaining = static_cast<unsigned>(want);
-        st->empty = (want == 0) ? 1u : 0u;
-    }
-    if (!st->empty) {
-        unsigned cum = 0;
-        int b = 255;
-        for (; b > 0; --b) {
-            if (cum + st->hist[b] >= st->remaining) break;
-            cum += st->hist[b];
+// One digit pass.  Each CTA histograms its grid-stride share of T (16-byte loads
+// when T is 16-byte aligned) in shared memory and adds it to st->hist[PASS]; the
+// CTA that finishes last (ticket) picks the digit of the s-th largest key: the
+// digit bins are scanned from the top, each thread owning a run of R consecutive
+// bins, and the one thread whose run holds the crossing fixes the digit.
+template <int PASS>
+__global__ void __launch_bounds__(kHistThreads) k_topk_hist(const float *T, int64_t N, TopkState *st,
+                                                            int64_t s_budget) {
+    constexpr int kShift = topk_shift(PASS), kBins = topk_bins(PASS), R = kBins / kHistThreads;
+    constexpr unsigned kFixed = topk_fixed(PASS), kMask = static_cast<unsigned>(kBins - 1);
+    __shared__ unsigned h[kBins];
+    __shared__ unsigned sh[32];
+    __shared__ unsigned last;
+#pragma unroll
+    for (int j = 0; j < R; ++j) h[threadIdx.x + j * kHistThreads] = 0;
+    __syncthreads();
+    const unsigned prefix = PASS == 0 ? 0u : st->prefix;
+    const int64_t stride = (int64_t)gridDim.x * kHistThreads;
+    const int64_t t0 = blockIdx.x * (int64_t)kHistThreads + threadIdx.x;
+    int64_t tail = 0;
+    if ((reinterpret_cast<uintptr_t>(T) & 15u) == 0) {
+        const int64_t N4 = N >> 2;
+        const float4 *T4 = reinterpret_cast<const float4 *>(T);
+#pragma unroll 4
+        for (int64_t e = t0; e < N4; e += stride) {
+            const float4 v = T4[e];
+            const unsigned k[4] = {mag_key(v.x), mag_key(v.y), mag_key(v.z), mag_key(v.w)};
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+                if (k[u] != 0u && ((k[u] ^ prefix) & kFixed) == 0u) atomicAdd(&h[(k[u] >> kShift) & kMask], 1u);
         }
-        st->prefix |= static_cast<unsigned>(b) << shift;
-        st->count_gt += cum;
-        st->remaining -= cum;
+        tail = N4 << 2;
     }
-    for (int b = 0; b < 256; ++b) st->hist[b] = 0;
-    if (shift == 0) {
-        st->kstar = st->empty ? 0xffffffffu : st->prefix;
-        st->need_eq = st->empty ? 0u : st->remaining;
+    for (int64_t e = tail + t0; e < N; e += stride) {
+        const unsigned k = mag_key(T[e]);
+        if (k != 0u && ((k ^ prefix) & kFixed) == 0u) atomicAdd(&h[(k >> kShift) & kMask], 1u);
+    }
+    __syncthreads();
+    unsigned *gh = st->hist[PASS];
+#pragma unroll
+    for (int j = 0; j < R; ++j) {
+        const int b = threadIdx.x + j * kHistThreads;
+        if (h[b]) atomicAdd(&gh[b], h[b]);
+    }
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) last = (atomicAdd(&st->ticket[PASS], 1u) == gridDim.x - 1) ? 1u : 0u;
+    __syncthreads();
+    if (!last) return;
+    __threadfence();
+    // The last CTA: thread t owns the bins of descending rank [t R, t R + R).
+    unsigned c[R];
+    unsigned mine = 0;
+#pragma unroll
+    for (int j = 0; j < R; ++j) {
+        c[j] = __ldcg(&gh[kBins - 1 - (threadIdx.x * R + j)]);
+        mine += c[j];
+    }
+    unsigned total;
+    const unsigned before = block_excl_scan(mine, sh, &total);
+    unsigned remaining, empty;
+    if (PASS == 0) {
+        const unsigned long long want = (unsigned long long)s_budget < total ? (unsigned long long)s_budget : total;
+        remaining = static_cast<unsigned>(want);
+        empty = want == 0 ? 1u : 0u;
+        if (threadIdx.x == 0) st->empty = empty;
+    } else {
+        remaining = st->remaining;
+        empty = st->empty;
+    }
+    __syncthreads();
+    if (empty) {
+        if (threadIdx.x == 0 && PASS == 2) {
+            st->kstar = 0xffffffffu;
+            st->need_eq = 0u;
+        }
+        return;
+    }
+    if (before < remaining && before + mine >= remaining) {
+        unsigned cum = before, run = before;
+        int jj = R - 1;
+        bool found = false;
+#pragma unroll
+        for (int j = 0; j < R; ++j) {   // the first bin of the run at which the running sum reaches remaining
+            if (!found && run + c[j] >= remaining) {
+                jj = j;
+                cum = run;
+                found = true;
+            }
+            run += c[j];
+        }
+        const unsigned digit = static_cast<unsigned>(kBins - 1 - (threadIdx.x * R + jj));
+        const unsigned pre = prefix | (digit << kShift);
+        st->prefix = pre;
+        st->count_gt += cum;
+        st->remaining = remaining - cum;
+        if (PASS == 2) {
+            st->kstar = pre;
+            st->need_eq = remaining - cum;
+        }
     }
 }
 
 constexpr int kChunk = 4096;   // elements per CTA in the compaction (256 threads x 16)
 
+// The 16 consecutive keys of thread threadIdx.x in chunk blockIdx.x (0 past N).
+__device__ __forceinline__ void chunk_keys(const float *T, int64_t N, bool vec, float v[16]) {
+    const int64_t base = (int64_t)blockIdx.x * kChunk + threadIdx.x * 16;
+    if (vec && base + 16 <= N) {
+        const float4 *p4 = reinterpret_cast<const float4 *>(T + base);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const float4 x = p4[u];
+            v[4 * u] = x.x;
+            v[4 * u + 1] = x.y;
+            v[4 * u + 2] = x.z;
+            v[4 * u + 3] = x.w;
+        }
+    } else {
+#pragma unroll
+        for (int u = 0; u < 16; ++u) v[u] = (base + u < N) ? T[base + u] : 0.0f;
+    }
+}
+
 __global__ void __launch_bounds__(256) k_topk_count(const float *T, int64_t N, const TopkState *st,
                                                     unsigned *cnt_gt, unsigned *cnt_eq) {
     __shared__ unsigned sh[32];
     const unsigned kstar = st->kstar;
-    const int64_t base = (int64_t)blockIdx.x * kChunk + threadIdx.x * 16;
+    float v[16];
+    chunk_keys(T, N, (reinterpret_cast<uintptr_t>(T) & 15u) == 0, v);
     unsigned g = 0, q = 0;
+#pragma unroll
     for (int u = 0; u < 16; ++u) {
-        const int64_t e = base + u;
-        if (e >= N) break;
-        const unsigned k = mag_key(T[e]);
+        const unsigned k = mag_key(v[u]);
         if (k == 0u) continue;
         g += (k > kstar) ? 1u : 0u;
         q += (k == kstar) ? 1u : 0u;
@@ -278,12 +361,12 @@ __global__ void __launch_bounds__(256) k_topk_emit(const float *T, int64_t N, co
                                                    int64_t *H_idx, float *H_val) {
     __shared__ unsigned sh[32];
     const unsigned kstar = st->kstar, need = st->need_eq;
-    const int64_t base = (int64_t)blockIdx.x * kChunk + threadIdx.x * 16;
+    float v[16];
+    chunk_keys(T, N, (reinterpret_cast<uintptr_t>(T) & 15u) == 0, v);
     unsigned ng = 0, nq = 0;
+#pragma unroll
     for (int u = 0; u < 16; ++u) {
-        const int64_t e = base + u;
-        if (e >= N) break;
-        const unsigned k = mag_key(T[e]);
+        const unsigned k = mag_key(v[u]);
         if (k == 0u) continue;
         ng += (k > kstar) ? 1u : 0u;
         nq += (k == kstar) ? 1u : 0u;
@@ -292,12 +375,12 @@ __global__ void __launch_bounds__(256) k_topk_emit(const float *T, int64_t N, co
     unsigned take = 0;
     if (need > eq0) take = (need - eq0) < nq ? (need - eq0) : nq;
     unsigned out = sel_base[blockIdx.x] + block_excl_scan(ng + take, sh, nullptr);
+    if (ng + take == 0u) return;
+    const int64_t base = (int64_t)blockIdx.x * kChunk + threadIdx.x * 16;
     unsigned eqseen = 0;
+#pragma unroll
     for (int u = 0; u < 16; ++u) {
-        const int64_t e = base + u;
-        if (e >= N) break;
-        const float v = T[e];
-        const unsigned k = mag_key(v);
+        const unsigned k = mag_key(v[u]);
         if (k == 0u) continue;
         bool keep = k > kstar;
         if (k == kstar) {
@@ -305,8 +388,8 @@ __global__ void __launch_bounds__(256) k_topk_emit(const float *T, int64_t N, co
             ++eqseen;
         }
         if (keep) {
-            H_idx[out] = e;
-            H_val[out] = v;
+            H_idx[out] = base + u;
+            H_val[out] = v[u];
             ++out;
         }
     }
@@ -585,15 +668,12 @@ cudaError_t launch_topk(const float *T, int64_t N, int64_t s_budget, TopkState *
                         float *H_val, int64_t *nnz, int nsm, cudaStream_t s) {
     cudaError_t e = cudaMemsetAsync(st, 0, sizeof(TopkState), s);
     if (e != cudaSuccess) return e;
-    int64_t hb = ceil_div(N, 256 * 8);
-    if (hb > nsm * 8) hb = nsm * 8;
+    int64_t hb = ceil_div(N, 256 * 16);
+    if (hb > nsm * 4) hb = nsm * 4;
     if (hb < 1) hb = 1;
-    const unsigned masks[4] = {0x00000000u, 0xff000000u, 0xffff0000u, 0xffffff00u};
-    for (int pass = 0; pass < 4; ++pass) {
-        const int shift = 24 - 8 * pass;
-        k_topk_hist<<<static_cast<unsigned>(hb), 256, 0, s>>>(T, N, st, shift, masks[pass]);
-        k_topk_pick<<<1, 32, 0, s>>>(st, shift, s_budget, pass == 0);
-    }
+    k_topk_hist<0><<<static_cast<unsigned>(hb), kHistThreads, 0, s>>>(T, N, st, s_budget);
+    k_topk_hist<1><<<static_cast<unsigned>(hb), kHistThreads, 0, s>>>(T, N, st, s_budget);
+    k_topk_hist<2><<<static_cast<unsigned>(hb), kHistThreads, 0, s>>>(T, N, st, s_budget);
     const int64_t nch = topk_chunks(N);
     k_topk_count<<<static_cast<unsigned>(nch), 256, 0, s>>>(T, N, st, cnt_gt, cnt_eq);
     k_topk_scan<<<1, 1024, 0, s>>>(cnt_gt, cnt_eq, static_cast<int>(nch), st, sel_base, eq_base, nnz);

@@ -7,15 +7,16 @@
 namespace qe {
 
 // Device-side state of the radix select behind P_s.
+constexpr int kTopkBins = 2048;   // digit bins of the first two passes (the third has 512)
 struct TopkState {
-    unsigned hist[256];
-    unsigned prefix;
-    unsigned remaining;
+    unsigned hist[3][kTopkBins];   // per digit pass (zeroed by the launcher)
+    unsigned ticket[3];            // CTAs done with each pass
+    unsigned prefix;               // key bits fixed so far
+    unsigned remaining;            // keys still to take from the current bucket
+    unsigned empty;
     unsigned long long count_gt;
     unsigned kstar;      // the s-th largest nonzero key (0xffffffff: nothing kept)
     unsigned need_eq;    // keys == kstar to keep, in ascending linear index
-    unsigned empty;
-    unsigned pad;
 };
 
 // part: 2 * kPowerMaxBlocks doubles (the per-CTA partial norms carried between steps).

@@ -23,7 +23,8 @@ QE_FEATURE_MAJOR, QE_TOKEN_MAJOR = 0, 1
 EXPORTED = ("qe_build_sigma", "qe_quantize_layer", "qe_quantize_layer_outlier",
             "qe_workspace_size", "qe_sync_status", "qe_status_string", "qe_version",
             "qe_build_sigma_static", "qe_timer_create", "qe_timer_read", "qe_timer_reset",
-            "qe_timer_destroy", "qe_build_sigma_host", "qe_pack_codes", "qe_unpack_codes")
+            "qe_timer_destroy", "qe_build_sigma_host", "qe_pack_codes", "qe_unpack_codes",
+            "qe_hard_threshold", "qe_hard_threshold_workspace")
 QE_KERNEL_PINIT_GEMM, QE_KERNEL_RESIDUAL_GEMM, QE_KERNEL_TRAIL_GEMM, QE_KERNEL_CD_BLOCK, \
     QE_KERNEL_CD_LISTS, QE_KERNEL_COUNT = range(6)
 
@@ -83,6 +84,10 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     L.qe_pack_codes.restype = st
     L.qe_unpack_codes.argtypes = [vp, i64, i64, i64, i32, vp, i64, vp]
     L.qe_unpack_codes.restype = st
+    L.qe_hard_threshold_workspace.argtypes = [i64, ctypes.POINTER(ctypes.c_size_t)]
+    L.qe_hard_threshold_workspace.restype = st
+    L.qe_hard_threshold.argtypes = [vp, i64, i64, vp, vp, vp, vp, ctypes.c_size_t, vp]
+    L.qe_hard_threshold.restype = st
     L.qe_timer_create.argtypes = [ctypes.c_uint, i32, ctypes.POINTER(vp)]
     L.qe_timer_create.restype = st
     L.qe_timer_read.argtypes = [vp, i32, ctypes.POINTER(ctypes.c_int), ctypes.POINTER(ctypes.c_double)]
@@ -257,6 +262,29 @@ def qe_unpack_codes(packed: torch.Tensor, p: int, bits: int, stream=None) -> tor
     _check(load().qe_unpack_codes(_ptr(packed), q, p, _rowmajor_ld(packed), bits, _ptr(codes), p,
                                   _stream(stream)), "qe_unpack_codes")
     return codes
+
+
+def qe_hard_threshold_workspace(N: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(load().qe_hard_threshold_workspace(N, ctypes.byref(n)), "qe_hard_threshold_workspace")
+    return n.value
+
+
+def qe_hard_threshold(T: torch.Tensor, s: int, stream=None) -> tuple:
+    """P_s of the IHT step on the flat fp32 tensor T: (indices ascending, values), the s entries
+    of largest magnitude (zeros never kept; ties to the smaller index)."""
+    if T.dtype != torch.float32 or not T.is_contiguous():
+        raise ValueError("expected a contiguous fp32 tensor")
+    N = T.numel()
+    dev = T.device
+    idx = torch.empty(max(s, 1), dtype=torch.int64, device=dev)
+    val = torch.empty(max(s, 1), dtype=torch.float32, device=dev)
+    nnz = torch.empty(1, dtype=torch.int64, device=dev)
+    ws = torch.empty(qe_hard_threshold_workspace(N), dtype=torch.uint8, device=dev)
+    _check(load().qe_hard_threshold(_ptr(T), N, s, _ptr(idx), _ptr(val), _ptr(nnz), _ptr(ws),
+                                    ws.numel(), _stream(stream)), "qe_hard_threshold")
+    k = int(nnz.item())
+    return idx[:k], val[:k]
 
 
 def qe_quantize_layer(W: torch.Tensor, Sigma: torch.Tensor, bits: int, iters: int, *,

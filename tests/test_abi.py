@@ -163,6 +163,27 @@ def test_pack_codes_rejects_bad_arguments(lib):
         assert fn(_fake(), 4, 0, 10, 3, _fake(2), 4, None) == qe.QE_ERR_INVALID_ARG
 
 
+def test_hard_threshold_rejects_bad_arguments(lib):
+    L = lib
+    ws = qe.qe_hard_threshold_workspace(1000)
+    assert ws >= 3 * 2048 * 4    # the three digit histograms at least
+    ok = dict(T=_fake(), N=1000, s=10, idx=_fake(2), val=_fake(3), nnz=_fake(4), w=ctypes.c_void_p(0x100000), wb=ws)
+
+    def call(**kw):
+        a = {**ok, **kw}
+        return L.qe_hard_threshold(a["T"], a["N"], a["s"], a["idx"], a["val"], a["nnz"], a["w"], a["wb"], None)
+    # NULL T / nnz / workspace, N < 1, s outside 0 .. N, NULL outputs with s > 0,
+    # a short or misaligned workspace
+    for bad in (dict(T=None), dict(nnz=None), dict(w=None), dict(N=0), dict(s=-1), dict(s=1001),
+                dict(idx=None), dict(val=None), dict(wb=ws - 1), dict(w=ctypes.c_void_p(0x100010)),
+                dict(N=1 << 32, s=0)):
+        assert call(**bad) == qe.QE_ERR_INVALID_ARG, bad
+    n = ctypes.c_size_t(0)
+    assert L.qe_hard_threshold_workspace(0, ctypes.byref(n)) == qe.QE_ERR_INVALID_ARG
+    assert L.qe_hard_threshold_workspace(10, None) == qe.QE_ERR_INVALID_ARG
+    assert qe.qe_hard_threshold_workspace(1 << 24) > qe.qe_hard_threshold_workspace(1 << 12)
+
+
 def test_workspace_size_grows_with_shape(lib):
     a = qe.qe_workspace_size(256, 256)
     b = qe.qe_workspace_size(512, 1024)

@@ -335,6 +335,53 @@ def test_pack_codes_bit_exact(bits):
         assert torch.equal(qe.qe_unpack_codes(pk, 300, bits), out["codes"])
 
 
+def _threshold_input(kind, N, seed):
+    rng = np.random.default_rng(seed)
+    if kind == "normal":
+        return rng.standard_normal(N).astype(np.float32)
+    if kind == "ties":           # few distinct magnitudes: the threshold falls inside a tie group
+        return rng.integers(-50, 51, N).astype(np.float32)
+    if kind == "sparse":         # mostly exact zeros (and a few -0.0): s may exceed the nonzeros
+        T = rng.standard_normal(N).astype(np.float32)
+        T[rng.random(N) < 0.97] = 0.0
+        T[rng.random(N) < 0.01] = -0.0
+        return T
+    if kind == "wide":           # 70 decades, denormals included
+        return (rng.standard_normal(N) * 10.0 ** rng.uniform(-44, 26, N)).astype(np.float32)
+    raise ValueError(kind)
+
+
+@pytest.mark.parametrize("kind,N,frac", [("normal", 10007, 0.01), ("normal", 10007, 1.0), ("ties", 50001, 0.013),
+                                         ("sparse", 40000, 0.05), ("wide", 30011, 0.3),
+                                         ("ties", 3_000_003, 0.01), ("normal", (1 << 24) + 3, 0.01)])
+def test_hard_threshold_bit_exact(kind, N, frac):
+    """P_s (Eq. iht-update) on its own against the oracle's: the kept indices and values
+    bit for bit, ties at the threshold to the smaller index across many compaction
+    chunks, zeros never kept; also from a T that is not 16-byte aligned."""
+    T = _threshold_input(kind, N + 1, seed=N % 1000 + 70)
+    s = int(round(frac * N))
+    Tg = torch.from_numpy(T).cuda()
+    for view, Th in ((Tg[:N], T[:N]), (Tg[1:], T[1:])):
+        idx, val = qe.qe_hard_threshold(view, s)
+        want = O.topk(Th.astype(np.float64), s)
+        got = idx.cpu().numpy()
+        assert got.shape == want.shape and np.array_equal(got, want), kind
+        assert np.array_equal(val.cpu().numpy().view(np.uint32), Th[want].view(np.uint32))
+
+
+def test_hard_threshold_degenerate():
+    """s = 0, all-zero T, s = N, N = 1 and N = 3 (no 16-byte body)."""
+    T = torch.zeros(1000, device="cuda")
+    assert qe.qe_hard_threshold(T, 0)[0].numel() == 0
+    assert qe.qe_hard_threshold(T, 1000)[0].numel() == 0
+    for N in (1, 3, 17):
+        Th = np.arange(1, N + 1, dtype=np.float32)[::-1].copy() * np.float32(-1.5)
+        for s in range(N + 1):
+            idx, val = qe.qe_hard_threshold(torch.from_numpy(Th).cuda(), s)
+            assert np.array_equal(idx.cpu().numpy(), O.topk(Th.astype(np.float64), s))
+            assert np.array_equal(val.cpu().numpy(), Th[idx.cpu().numpy()])
+
+
 @pytest.mark.parametrize("block_width,group_size", [(256, 256), (128, 128), (128, 256)])
 def test_layer_grouped_grids(block_width, group_size):
     """Grouped grids (one grid per row and group of columns) against the oracle's
