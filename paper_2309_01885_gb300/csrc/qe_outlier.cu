@@ -154,6 +154,34 @@ __global__ void k_iht_target(const float *H, const float *R, int64_t ld, const u
     }
 }
 
+// The same with 4 consecutive columns per thread (16-byte loads of H, R, d and T,
+// 4-byte loads of the codes; p, ld and ldc multiples of 4 and aligned rows), a CTA
+// covering 1024 columns of gridDim.y-strided rows.
+__global__ void __launch_bounds__(256) k_iht_target4(const float *H, const float *R, int64_t ld,
+                                                     const uint8_t *codes, int64_t ldc, const float *scale,
+                                                     const float *d, const double *eta, int64_t q, int64_t p,
+                                                     float *T) {
+    const int64_t j = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) * 4;
+    if (j >= p) return;
+    const float e2 = static_cast<float>(2.0 * (*eta));
+    const float4 dv = *reinterpret_cast<const float4 *>(d + j);
+    const float dj[4] = {dv.x > 0.0f ? dv.x : 0.0f, dv.y > 0.0f ? dv.y : 0.0f, dv.z > 0.0f ? dv.z : 0.0f,
+                         dv.w > 0.0f ? dv.w : 0.0f};
+#pragma unroll 2
+    for (int64_t i = blockIdx.y; i < q; i += gridDim.y) {
+        const float s = scale[i];
+        const float4 h = *reinterpret_cast<const float4 *>(H + i * ld + j);
+        const float4 r = *reinterpret_cast<const float4 *>(R + i * ld + j);
+        const uchar4 c = *reinterpret_cast<const uchar4 *>(codes + i * ldc + j);
+        float4 o;
+        o.x = h.x + e2 * dj[0] * (s * (r.x - static_cast<float>(c.x)));
+        o.y = h.y + e2 * dj[1] * (s * (r.y - static_cast<float>(c.y)));
+        o.z = h.z + e2 * dj[2] * (s * (r.z - static_cast<float>(c.z)));
+        o.w = h.w + e2 * dj[3] * (s * (r.w - static_cast<float>(c.w)));
+        *reinterpret_cast<float4 *>(T + i * p + j) = o;
+    }
+}
+
 // Flat copy of a q x p matrix (bf16 / fp32, leading dimension ldw) into T (ld = p).
 __global__ void k_flat_copy(const void *W, int w_bf16, int64_t ldw, int64_t q, int64_t p, float *T) {
     for (int64_t i = blockIdx.y; i < q; i += gridDim.y) {
@@ -616,6 +644,8 @@ __global__ void k_dinv(const float *d, int64_t p, float *dinv) {
 }
 
 // ---- launchers --------------------------------------------------------------
+static inline bool aligned16(const void *ptr) { return (reinterpret_cast<uintptr_t>(ptr) & 15u) == 0; }
+
 static inline dim3 rows_grid(int64_t rows, int64_t cols) {
     int64_t bx = ceil_div(cols, 256);
     if (bx > 16) bx = 16;
@@ -651,7 +681,14 @@ cudaError_t launch_power_lambda(const float *S, int64_t lds, int64_t p, int iter
 cudaError_t launch_iht_target(const float *H, const float *R, int64_t ld, const uint8_t *codes,
                               int64_t ldc, const float *scale, const float *zero, const float *d,
                               const double *eta, int64_t q, int64_t p, float *T, cudaStream_t s) {
-    k_iht_target<<<rows_grid(q, p), 256, 0, s>>>(H, R, ld, codes, ldc, scale, zero, d, eta, q, p, T);
+    const bool vec = p % 4 == 0 && ld % 4 == 0 && ldc % 4 == 0 && aligned16(H) && aligned16(R) && aligned16(T) &&
+                     aligned16(d) && (reinterpret_cast<uintptr_t>(codes) & 3u) == 0;
+    if (vec) {
+        const dim3 grid(static_cast<unsigned>(ceil_div(p, 1024)), static_cast<unsigned>(q < 1024 ? q : 1024));
+        k_iht_target4<<<grid, 256, 0, s>>>(H, R, ld, codes, ldc, scale, d, eta, q, p, T);
+    } else {
+        k_iht_target<<<rows_grid(q, p), 256, 0, s>>>(H, R, ld, codes, ldc, scale, zero, d, eta, q, p, T);
+    }
     return cudaGetLastError();
 }
 
