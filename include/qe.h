@@ -98,7 +98,8 @@ typedef struct {
      * changes per row in the previous sweep, then each row runs on its own.
      * Both modes take the same decisions in the same order; only the speed
      * differs.  0 = default (64); -1 = always together; below -1 is
-     * QE_ERR_INVALID_ARG.  Ignored by the outlier variant. */
+     * QE_ERR_INVALID_ARG.  The outlier variant applies it to its per-iteration
+     * sweeps after the first. */
     int free_changes;
     /* Grouped grids (the paper notes that grouping can be incorporated into the
      * per-channel grid of Sec. 2.1): G > 0 gives every row one scale and
@@ -108,7 +109,7 @@ typedef struct {
      * (QE_ERR_INVALID_ARG otherwise); relax_period != 0 or the outlier variant
      * return QE_ERR_UNSUPPORTED with G < p. */
     int group_size;
-    /* Optional warm start (Sec. 3.1, "initialized with ... any other algorithm"):
+    /* Optional warm start (Sec. 3.1: the descent may start from another method's solution):
      * q x p codes (leading dimension p) on the grid this call computes.  NULL = start at W. */
     const uint8_t *init_codes;
     /* Optional output: iters x q x p codes after every sweep (for parity checks). */
@@ -149,7 +150,7 @@ qe_status qe_build_sigma(const void *X, qe_dtype x_dtype, qe_xlayout layout,
  *   scales   out, device q floats s_i;  zeros: out, device q floats z_i
  *            (integer-valued).  Grid: asymmetric per-row min/max with 0 in
  *            range, s = (max - min)/(2^b - 1), z = round(-min/s), evaluated
- *            in binary32 (Sec. 2.1, "uniformly spaced, following GPTQ").
+ *            in binary32 (Sec. 2.1: evenly spaced levels, as in GPTQ).
  *   obj      out, device iters doubles: f after each sweep.
  *   opts     may be NULL (all defaults).
  * Each coordinate takes the nearest level of the closed-form minimiser

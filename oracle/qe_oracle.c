@@ -49,7 +49,7 @@ int qo_threads(int n)
 /* ------------------------------------------------------------------------- */
 
 /*
- * Per-channel uniform grid Q_i (Sec. 2.1, "uniformly spaced, following GPTQ"):
+ * Per-channel uniform grid Q_i (Sec. 2.1: evenly spaced levels, the grid GPTQ uses):
  * levels s_i * (c - z_i), c = 0 .. 2^b - 1, asymmetric min/max over row i with
  * 0 always inside the range; an all-zero row gets the range [-1, 1].
  * excl (q*p bytes, may be NULL) removes entries from the pool; with 0 always in
@@ -517,7 +517,7 @@ int qo_quantease_alg3(const double *W, int64_t q, int64_t p, const double *S,
 /* ------------------------------------------------------------------------- */
 
 /*
- * lambda_max(Sigma) by the power method (Sec. 4.3, "iterative power method"):
+ * lambda_max(Sigma) by the power method (Sec. 4.3 names power iteration for it):
  * v0 = 1/sqrt(p) * ones;  iters times: v <- Sigma v / ||Sigma v||;
  * return the Rayleigh quotient v^T Sigma v.
  */

@@ -943,13 +943,16 @@ qe_status qe_quantize_layer_outlier(const void *W, qe_dtype w_dtype, int64_t q, 
             // R is exact and the target W - H stays fixed during the sweep: one
             // change-list sweep whose window starts empty (each block corrected by
             // this sweep's changes left of it), which ends by flushing the window into
-            // R; g after it = g before + the objective changes of its decisions
-            QE_CK(cudaMemsetAsync(c.lcnt, 0, static_cast<size_t>(q) * pl.nblk * 4, c.s));
+            // R; g after it = g before + the objective changes of its decisions.  The
+            // first such sweep of the call starts in lockstep; later ones take their
+            // mode from the change counts the previous sweep left in the lists.
+            const bool first_list = t == (warm ? 0 : 1);
+            if (first_list) QE_CK(cudaMemsetAsync(c.lcnt, 0, static_cast<size_t>(q) * pl.nblk * 4, c.s));
             CdArgs a = list_args(c, codes, scales, zeros, bits);
             {
                 Timed tm(c.timer, QE_KERNEL_CD_LISTS, c.s);
-                QE_CK(launch_cd_rows_lists(pl.B, a, t, t + 1, c.rowdft, nullptr, 1, kFreeMaxChanges, 1, c.nsm,
-                                           c.s));
+                QE_CK(launch_cd_rows_lists(pl.B, a, t, t + 1, c.rowdft, nullptr, first_list ? 1 : 2,
+                                           free_changes(opts), 1, c.nsm, c.s));
             }
             if (obj_cd) QE_CK(launch_obj_prefix(c.rowdft, q, 1, t == 0 ? c.objbase : obj + t - 1, obj_cd + t, c.s));
         }

@@ -978,8 +978,13 @@ __device__ __forceinline__ void rows_block_win(const CdArgs &a, int64_t b0, int 
 //     (few changes: no block barriers, no copies).  A CTA that goes free stays
 //     free for its remaining sweeps (correct at any density), so its warps no
 //     longer meet between sweeps, and a row at a fixed point skips its sweeps.
-// first_lockstep forces lockstep for the first sweep (its lists are empty
+// first_lockstep = 1 forces lockstep for the first sweep (its lists are empty
 // after a residual refresh although many codes are about to change).
+// first_lockstep = 2 (fresh): R was refreshed since the sweep that left the
+// lists (the outlier variant's target moved), so the lists only give that
+// sweep's change counts: the first sweep picks its mode from them, each row
+// clears its own lists (the window starts empty) and visits its blocks even at
+// a fixed point.
 // Per sweep and row the objective change goes to rowdf_t[t - t_begin][i]; with
 // sweep_codes the row's codes after each sweep are copied out.  flush: after the
 // last sweep every block's base takes the changes of the lists of its own and
@@ -1018,10 +1023,16 @@ __global__ void __launch_bounds__(32 * kRowsMaxWarps, 1) k_cd_rows_lists(const C
             prev += cnt;
         }
     }
+    const bool fresh = first_lockstep == 2;
+    if (fresh && row_ok) {
+        __syncwarp();
+        for (int c = lane; c < a.nblk; c += 32) a.lcnt[i * a.nblk + c] = 0;
+        __syncwarp();
+    }
     uint32_t use = 0;
     bool free_run = false;   // CTA-uniform; once set, the warps run their remaining sweeps alone
     for (int t = t_begin; t < t_end; ++t) {
-        const bool forced_lockstep = first_lockstep && t == t_begin;
+        const bool forced_lockstep = first_lockstep == 1 && t == t_begin;
         if (!free_run) {
             if (lane == 0) s_chg[warp] = prev;
             __syncthreads();
@@ -1040,7 +1051,7 @@ __global__ void __launch_bounds__(32 * kRowsMaxWarps, 1) k_cd_rows_lists(const C
             // is empty, so every block stages the values it decided on last time.
             // With at most kWinCap changes the window lives in the warp's shared memory
             // (the packed block is no longer needed once the CTA runs free).
-            if (row_ok && prev > 0) {
+            if (row_ok && (prev > 0 || (fresh && t == t_begin))) {
                 uint32_t *win = reinterpret_cast<uint32_t *>(reinterpret_cast<char *>(cd_smem) + warp * kFreeWarpBytes);
                 float *stg = reinterpret_cast<float *>(win + kWinCap);
                 int wn = (prev <= kWinCap && a.p <= 65536) ? build_window<B>(a, i, lane, win) : -1;

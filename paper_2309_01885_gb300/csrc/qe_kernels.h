@@ -93,7 +93,9 @@ cudaError_t launch_cd_block(int B, const CdArgs &a, int nsm, cudaStream_t s);
 // sweep t and row i goes to rowdf_t[(t - t_begin) q + i]; sweep_codes (optional) gets
 // the codes after each sweep at [t][q][p].  A CTA runs a sweep in the free mode when
 // its rows made at most free_max_changes changes each (on average) in the previous
-// sweep; first_lockstep forces the lockstep mode for the first sweep.  flush: end
+// sweep; first_lockstep = 1 forces the lockstep mode for the first sweep, 2 marks
+// R as refreshed since the lists were left (they give only the previous sweep's
+// change counts; the window starts empty, every row is visited).  flush: end
 // with R the exact residual of the final codes (each block's base takes the changes
 // its last visit did not see).
 cudaError_t launch_cd_rows_lists(int B, const CdArgs &a, int t_begin, int t_end, double *rowdf_t,

@@ -325,9 +325,11 @@ def qe_quantize_layer_outlier(W: torch.Tensor, Sigma: torch.Tensor, bits: int, i
                               s_budget: int, *, power_iters: int = 0, init_codes=None,
                               record_sweeps: bool = False, want_norm: bool = False,
                               workspace: torch.Tensor | None = None, structured: bool = False,
+                              free_changes: int = 0,
                               timer: Timer | None = None, stream=None) -> dict:
     """Outlier-aware QuantEase; adds H_val, H_idx (sorted linear indices), H_nnz, obj_cd.
-    structured: H keeps whole columns (floor(s_budget / q) of them)."""
+    structured: H keeps whole columns (floor(s_budget / q) of them); free_changes: as for
+    qe_quantize_layer, for the per-iteration sweeps after the first."""
     q, p = W.shape
     dev = W.device
     codes = torch.empty(q, p, dtype=torch.uint8, device=dev)
@@ -341,7 +343,7 @@ def qe_quantize_layer_outlier(W: torch.Tensor, Sigma: torch.Tensor, bits: int, i
     H_nnz = torch.zeros(1, dtype=torch.int64, device=dev)
     sweep = torch.empty(iters, q, p, dtype=torch.uint8, device=dev) if record_sweeps else None
     norm = torch.empty(1, dtype=torch.float64, device=dev) if want_norm else None
-    o = _opts(0, power_iters, init_codes, sweep, norm, workspace, timer)
+    o = _opts(0, power_iters, init_codes, sweep, norm, workspace, timer, free_changes=free_changes)
     o.structured_outliers = int(structured)
     _check(load().qe_quantize_layer_outlier(
         _ptr(W), _dtype(W), q, p, _rowmajor_ld(W), _ptr(Sigma), bits, iters, int(s_budget),

@@ -586,6 +586,30 @@ def test_structured_outlier_below_one_column_matches_plain_layer():
     assert np.array_equal(a["obj"].cpu().numpy(), b["obj"].cpu().numpy())
 
 
+@pytest.mark.parametrize("p", [1024, 203])
+def test_outlier_sweep_modes_identical(p):
+    """The per-iteration sweeps after the first take their mode (rows in lockstep or each
+    on its own) from the previous sweep's change counts; every mode takes the same
+    decisions in the same order, so the results agree bit for bit with always-lockstep
+    (free_changes = -1) and always-free (a huge threshold) runs."""
+    q, bits, iters = 256, 3, 6
+    W = inputs.layer_weights(q, p, dtype=torch.bfloat16, seed=91, device="cuda", planted_frac=0.01,
+                             planted_std=0.3)
+    X = inputs.calib_inputs(p, 4096, dtype=torch.bfloat16, seed=91, device="cuda", heavy_frac=0.02,
+                            heavy_mult=30.0)
+    Sg = qe.qe_build_sigma(X)
+    s_budget = int(0.01 * q * p)
+    outs = [qe.qe_quantize_layer_outlier(W, Sg, bits, iters, s_budget, free_changes=f) for f in (-1, 0, 1 << 20)]
+    assert qe.qe_sync_status() == qe.QE_OK
+    ref = outs[0]
+    for o in outs[1:]:
+        assert torch.equal(o["codes"], ref["codes"])
+        assert torch.equal(o["obj"], ref["obj"]) and torch.equal(o["obj_cd"], ref["obj_cd"])
+        n = int(ref["H_nnz"].item())
+        assert int(o["H_nnz"].item()) == n
+        assert torch.equal(o["H_idx"][:n], ref["H_idx"][:n]) and torch.equal(o["H_val"][:n], ref["H_val"][:n])
+
+
 def test_outlier_warm_start_and_without_obj_cd():
     """A warm start (init_codes) and a call without obj_cd refresh R from the codes
     with no fused objective.  The run stays valid: the IHT half never increases g
