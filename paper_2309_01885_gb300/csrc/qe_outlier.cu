@@ -54,9 +54,9 @@ __device__ __forceinline__ unsigned block_excl_scan(unsigned v, unsigned *sh, un
 // order, so the result is reproducible), or is computed here when part_in is
 // NULL (the first step); each CTA leaves the sum of the squares of the y_out
 // values it wrote in part_out[blockIdx.x].  One warp per row of Sigma; eight
-// independent partial sums keep eight loads in flight per lane (a dependent
-// chain of single loads made this step latency-bound), and 16-byte loads are
-// used when the rows are 16-byte aligned.
+// independent partial sums and four 16-byte row loads in flight per lane (a
+// dependent chain of single loads made this step latency-bound) when the rows
+// are 16-byte aligned.
 __global__ void __launch_bounds__(256) k_power_step(const float *S, int64_t lds, int64_t p,
                                                     const float *y_in, const double *part_in, int nparts,
                                                     float *y_out, double *part_out) {
@@ -83,19 +83,24 @@ __global__ void __launch_bounds__(256) k_power_step(const float *S, int64_t lds,
             const int64_t n4 = p / 4;
             const float4 *r4 = reinterpret_cast<const float4 *>(row);
             const float4 *y4 = reinterpret_cast<const float4 *>(y_in);
-            for (int64_t b = lane; b < n4; b += 64) {
-                const float4 x0 = r4[b], v0 = y4[b];
-                const bool two = b + 32 < n4;
-                const float4 x1 = two ? r4[b + 32] : make_float4(0.f, 0.f, 0.f, 0.f);
-                const float4 v1 = two ? y4[b + 32] : make_float4(0.f, 0.f, 0.f, 0.f);
-                acc[0] = fmaf(x0.x, v0.x, acc[0]);
-                acc[1] = fmaf(x0.y, v0.y, acc[1]);
-                acc[2] = fmaf(x0.z, v0.z, acc[2]);
-                acc[3] = fmaf(x0.w, v0.w, acc[3]);
-                acc[4] = fmaf(x1.x, v1.x, acc[4]);
-                acc[5] = fmaf(x1.y, v1.y, acc[5]);
-                acc[6] = fmaf(x1.z, v1.z, acc[6]);
-                acc[7] = fmaf(x1.w, v1.w, acc[7]);
+            // four 16-byte loads of the row in flight per lane; accumulators 0-3 take pieces
+            // lane, lane + 64, ... and 4-7 pieces lane + 32, lane + 96, ..., in order
+            for (int64_t b = lane; b < n4; b += 128) {
+                float4 x[4], v[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const bool in = b + 32 * u < n4;
+                    x[u] = in ? r4[b + 32 * u] : make_float4(0.f, 0.f, 0.f, 0.f);
+                    v[u] = in ? y4[b + 32 * u] : make_float4(0.f, 0.f, 0.f, 0.f);
+                }
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int k = 4 * (u & 1);
+                    acc[k] = fmaf(x[u].x, v[u].x, acc[k]);
+                    acc[k + 1] = fmaf(x[u].y, v[u].y, acc[k + 1]);
+                    acc[k + 2] = fmaf(x[u].z, v[u].z, acc[k + 2]);
+                    acc[k + 3] = fmaf(x[u].w, v[u].w, acc[k + 3]);
+                }
             }
             b0 = n4 * 4;
         }
@@ -530,6 +535,7 @@ __global__ void __launch_bounds__(kSpmmThreads) k_spmm_refresh(const float *PW, 
                                                                const float *scale) {
     __shared__ int sk[kSpmmChunk];
     __shared__ float sv[kSpmmChunk];
+    __shared__ int so[kSpmmChunk];   // owner thread << 4 | slot of column k in this tile, or -1
     extern __shared__ __align__(16) float ring[];   // [kSpmmDepth][kSpmmPieces][kSpmmThreads][4]
     const int64_t i = blockIdx.x;
     const int64_t j0 = static_cast<int64_t>(blockIdx.y) * kSpmmCols + 4 * threadIdx.x;
@@ -562,8 +568,16 @@ __global__ void __launch_bounds__(kSpmmThreads) k_spmm_refresh(const float *PW, 
         const int n = static_cast<int>((e1 - c0) < kSpmmChunk ? (e1 - c0) : kSpmmChunk);
         __syncthreads();   // the previous chunk is consumed
         if (static_cast<int>(threadIdx.x) < n) {
-            sk[threadIdx.x] = static_cast<int>(H_idx[c0 + threadIdx.x] - i * p);
+            const int k = static_cast<int>(H_idx[c0 + threadIdx.x] - i * p);
+            sk[threadIdx.x] = k;
             sv[threadIdx.x] = H_val[c0 + threadIdx.x];
+            const int64_t kk = k - static_cast<int64_t>(blockIdx.y) * kSpmmCols;
+            int own = -1;
+            if (kk >= 0 && kk < kSpmmCols) {
+                const int u = static_cast<int>(kk) / (4 * kSpmmThreads), w = static_cast<int>(kk) % (4 * kSpmmThreads);
+                own = ((w >> 2) << 4) | (4 * u + (w & 3));
+            }
+            so[threadIdx.x] = own;
         }
         __syncthreads();
         // entry e goes to slot e % kSpmmDepth; one commit group per entry (empty past n)
@@ -590,19 +604,26 @@ __global__ void __launch_bounds__(kSpmmThreads) k_spmm_refresh(const float *PW, 
         for (int e = 0; e < n; ++e) {
             issue(e + kSpmmDepth - 1);
             cp_async_wait_group<kSpmmDepth - 1>();   // entry e has landed
-            const int k = sk[e];
             const float hv = sv[e];
             const float *seg = mine + (e % kSpmmDepth) * kSpmmCols;
+            // every column adds -h Sigma_bar[k][j] (columns past p take values never
+            // stored); Sigma_bar[k][k] = 0, so the identity's -h at column k follows as one
+            // more step of the same chain, in the thread that owns the column
 #pragma unroll
             for (int u = 0; u < kSpmmPieces; ++u) {
-                const int off = u * 4 * kSpmmThreads;
-                const float4 v = *reinterpret_cast<const float4 *>(seg + off);
-                const float w[4] = {v.x, v.y, v.z, v.w};
+                const float4 v = *reinterpret_cast<const float4 *>(seg + u * 4 * kSpmmThreads);
+                acc[4 * u] = fmaf(-hv, v.x, acc[4 * u]);
+                acc[4 * u + 1] = fmaf(-hv, v.y, acc[4 * u + 1]);
+                acc[4 * u + 2] = fmaf(-hv, v.z, acc[4 * u + 2]);
+                acc[4 * u + 3] = fmaf(-hv, v.w, acc[4 * u + 3]);
+            }
+            const int own = so[e];
+            if ((own >> 4) == static_cast<int>(threadIdx.x)) {
+                const int sl = own & 15;
 #pragma unroll
-                for (int x = 0; x < 4; ++x) {
-                    if (x >= ncol[u]) break;
-                    const int64_t j = j0 + off + x;
-                    acc[4 * u + x] = fmaf(-hv, (j == k) ? 1.0f : w[x], acc[4 * u + x]);
+                for (int z = 0; z < kSpmmPer; ++z) {
+                    const float y = fmaf(-hv, 1.0f, acc[z]);
+                    acc[z] = (z == sl) ? y : acc[z];
                 }
             }
         }
