@@ -35,6 +35,24 @@ UNIT = "q·p² column-updates/s"
 DEFAULT_DENSE_SWEEPS = 1      # the library's default for qe_opts.dense_sweeps
 
 
+def max_over_ranks(x: float, device) -> float:
+    """The slowest rank's value of x (the job ends when its last replica ends); x itself on
+    one rank or outside a process group."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(units_per_rank: float, world: int, ms: float) -> float:
+    """Whole-job units per second: every rank processes units_per_rank per step (weak
+    scaling, independent layers) and the step takes the slowest rank's ms."""
+    return units_per_rank * world / (ms / 1e3)
+
+
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -392,11 +410,7 @@ def main():
     total_ms = t_start.elapsed_time(t_end)
     sigma_ms = [e[0].elapsed_time(e[1]) for e in ev]
     cd_ms = [[e[1 + k].elapsed_time(e[2 + k]) for e in ev] for k in range(nb)]
-    ms = total_ms / args.steps
-    if world > 1:
-        t = torch.tensor([ms], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(total_ms / args.steps, "cuda")
 
     timed = {k: dom.read(k) for k in kinds}
     dom.close()
@@ -422,7 +436,7 @@ def main():
     refreshes = (1 if plan[0][0] == "first" else 0) + extra_refreshes
 
     units_per_step = q * p * p * cfg.iters * nb           # column updates per rank per step
-    value = units_per_step * world / (ms / 1e3)
+    value = job_throughput(units_per_step, world, ms)
     sig_flops = p * (p + 1) * n                            # symmetric half of X X^T
     sigma_avg = statistics.mean(sigma_ms)
     cd_avg = [statistics.mean(x) for x in cd_ms]
@@ -561,14 +575,10 @@ def main():
             e2e_step()
         e1.record(stream)
         torch.cuda.synchronize()
-        e2e_ms = e0.elapsed_time(e1) / e2e_steps
-        if world > 1:
-            t = torch.tensor([e2e_ms], dtype=torch.float64, device="cuda")
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            e2e_ms = float(t.item())
+        e2e_ms = max_over_ranks(e0.elapsed_time(e1) / e2e_steps, "cuda")
         h2d = X.numel() * X.element_size() + W.numel() * W.element_size()
         d2h = nb * (q * p + 4 * q + 4 * q + 8 * cfg.iters)
-        result["e2e"] = {"value": units_per_step * world / (e2e_ms / 1e3), "unit": UNIT,
+        result["e2e"] = {"value": job_throughput(units_per_step, world, e2e_ms), "unit": UNIT,
                          "ms_per_step": e2e_ms, "steps": e2e_steps, "h2d_bytes_per_step": h2d,
                          "d2h_bytes_per_step": d2h}
 
