@@ -89,8 +89,9 @@ typedef struct {
      * Eq. cd-update-closed-2).  Sweeps 1 .. dense_sweeps multiply the dense
      * change matrix on the tensor cores; later sweeps, where few codes change,
      * walk per-row lists of the changed columns and add their fp32 Sigma_bar
-     * rows.  0 = default (1: lists from sweep 2 on); a value >= iters keeps the
-     * dense form throughout;
+     * rows.  0 = default: the adaptive schedule of switch_below; n > 0: sweeps
+     * 1 .. n dense, lists from sweep n + 1; a value >= iters keeps the dense
+     * form throughout;
      * negative is QE_ERR_INVALID_ARG.  Ignored by the outlier variant. */
     int dense_sweeps;
     /* List sweeps: the rows of a CTA step through the column blocks together
@@ -122,6 +123,25 @@ typedef struct {
     size_t workspace_bytes;
     /* Optional: record CUDA events around the launches of the timed kernel classes. */
     qe_timer *timer;
+    /* Adaptive sweep schedule, used when dense_sweeps = 0 (no paper counterpart:
+     * it only picks which of the two forms above computes each sweep's sums).
+     * The sweeps after the first take the dense tensor-core form until a sweep
+     * changes fewer than switch_below codes; the change lists take the rest.
+     * The choice is made on the device from the change counts, so the call
+     * stays asynchronous: both forms of such a sweep are enqueued and the one
+     * not chosen returns at once.  0 = automatic: when the fp32 Sigma_bar rows
+     * (4 p^2 bytes) fit in three quarters of the GPU's L2, lists from sweep 2
+     * (their gathers hit L2); otherwise the threshold of a cost model (a dense
+     * sweep's 6 q p^2 flops of plane products against a gather of 4 p bytes
+     * from DRAM per change, the next sweep changing about 0.7 times as many
+     * codes).  > 0 forces the adaptive schedule with this threshold; negative is
+     * QE_ERR_INVALID_ARG.  Ignored by the outlier variant. */
+    int64_t switch_below;
+    /* Optional output (device, iters bytes): how each sweep of qe_quantize_layer
+     * formed its cross-block sums: 0 = the sequential form (sweep 1, a relaxed
+     * sweep and the sweep after one), 1 = the dense tensor-core form, 2 = the
+     * change lists.  NULL = not recorded.  Ignored by the outlier variant. */
+    uint8_t *sweep_forms;
 } qe_opts;
 
 /*

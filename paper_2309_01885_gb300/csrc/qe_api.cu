@@ -53,6 +53,33 @@ constexpr int kDefaultPowerIters = 64;
 constexpr int kDefaultDenseSweeps = 1;
 constexpr int kSweepChunk = 32;          // list-mode sweeps per persistent launch
 constexpr int kFreeMaxChanges = 64;      // changes per row in the previous sweep below which a CTA runs free
+constexpr int kMaxSplits = 16;           // split-K pieces of a trailing GEMM (partial buffers)
+constexpr int kMinStepsPerSplit = 48;    // k-steps (k-blocks x plane products) per split-K piece
+
+// Split-K pieces of a trailing GEMM with mt tile rows and kb k-blocks of nprod
+// products: the count whose CTAs (one per SM) fill their waves best, less a
+// small charge per piece for the partial sums it writes and the in-block
+// prologue reads back; every piece keeps at least kMinStepsPerSplit k-steps.
+// (A wide layer with 116 tile rows on 152 SMs runs 5 pieces in 4 full waves
+// instead of one wave three quarters full.)
+static int choose_splits(int64_t mt, int kb, int nprod, int nsm) {
+    int cap = (kb * nprod) / kMinStepsPerSplit;
+    if (cap > kb) cap = kb;
+    if (cap > kMaxSplits) cap = kMaxSplits;
+    if (cap < 1) cap = 1;
+    int best = 1;
+    double bv = -1.0;
+    for (int S = 1; S <= cap; ++S) {
+        const int64_t ctas = S * mt;
+        const int64_t waves = ceil_div(ctas, nsm);
+        const double v = static_cast<double>(ctas) / static_cast<double>(waves * nsm) - 0.01 * S;
+        if (v > bv + 1e-12) {
+            bv = v;
+            best = S;
+        }
+    }
+    return best;
+}
 
 // ---- workspace layout -----------------------------------------------------------
 struct Plan {
@@ -61,7 +88,7 @@ struct Plan {
     int64_t gsize = 0, ngroups = 1;   // grid columns per group (p: per row), groups per row
     bool grouped = false;
     size_t snt = 0, d = 0, dinv = 0, tri = 0, P = 0, R = 0, wpl = 0, qf = 0, dp = 0, part = 0, objp = 0,
-           rowdf = 0, objbase = 0, sbar = 0, lcnt = 0, lent = 0, rowdft = 0;
+           rowdf = 0, objbase = 0, sbar = 0, lcnt = 0, lent = 0, rowdft = 0, sw = 0;
     int64_t nblk = 0;
     size_t PW = 0, H = 0, T = 0, st = 0, cg = 0, ce = 0, sb = 0, eb = 0, y0 = 0, y1 = 0, lam = 0,
            eta = 0, rowptr = 0, cpart = 0, cnorm = 0, ccols = 0, cval = 0, cn = 0, ppart = 0;
@@ -84,11 +111,8 @@ static Plan make_plan(int64_t q, int64_t p, int B, bool outlier, int wpl_planes,
     pl.ld = round_up(p, 64);
     pl.B = B;
     pl.nblk = ceil_div(p, B);
-    const int64_t mtiles = ceil_div(q, 128);
-    int64_t smax = nsm / mtiles;
-    if (smax < 1) smax = 1;
-    if (smax > 16) smax = 16;
-    pl.smax = static_cast<int>(smax);
+    (void)nsm;
+    pl.smax = kMaxSplits;
     const size_t qld = static_cast<size_t>(q) * pl.ld;
     size_t cur = 0;
     pl.snt = take(cur, static_cast<size_t>(3 * p) * pl.ld * 2);
@@ -110,6 +134,7 @@ static Plan make_plan(int64_t q, int64_t p, int B, bool outlier, int wpl_planes,
         pl.lcnt = take(cur, static_cast<size_t>(q) * pl.nblk * 4);
         pl.lent = take(cur, static_cast<size_t>(q) * pl.nblk * B * 4);
         pl.rowdft = take(cur, static_cast<size_t>(q) * kSweepChunk * 8);
+        pl.sw = take(cur, 16);   // adaptive schedule: switch flag (int) and change counter (u64)
     }
     if (outlier) {
         const int64_t N = q * p;
@@ -188,6 +213,8 @@ struct Ctx {
     int *lcnt = nullptr;
     uint32_t *lent = nullptr;
     double *rowdft = nullptr;
+    int *swflag = nullptr;
+    unsigned long long *swcount = nullptr;
     float *PW = nullptr, *H = nullptr, *T = nullptr, *y0 = nullptr, *y1 = nullptr;
     TopkState *st = nullptr;
     unsigned *cg = nullptr, *ce = nullptr, *sb = nullptr, *eb = nullptr;
@@ -247,6 +274,8 @@ static qe_status setup_ctx(Ctx &c, const Plan &pl, const qe_opts *o, cudaStream_
         c.lcnt = at<int>(w, pl.lcnt);
         c.lent = at<uint32_t>(w, pl.lent);
         c.rowdft = at<double>(w, pl.rowdft);
+        c.swflag = at<int>(w, pl.sw);
+        c.swcount = at<unsigned long long>(w, pl.sw + 8);
     }
     if (pl.PW) {
         c.PW = at<float>(w, pl.PW);
@@ -416,7 +445,7 @@ enum { SRC_W = 0, SRC_CODES = 1, SRC_V = 2 };
 static float *relaxed_values(const Ctx &c) { return reinterpret_cast<float *>(c.lent); }
 
 static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float *zeros, int bits,
-                       int src, bool relax, int window) {
+                       int src, bool relax, int window, const int *gate = nullptr) {
     const int64_t q = c.pl.q, p = c.pl.p, ld = c.pl.ld;
     const int B = c.pl.B;
     const bool frac = src != SRC_CODES || relax;
@@ -426,15 +455,17 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
         int nsplit = 0;
         if (kcols > 0) {
             const int kb = static_cast<int>(ceil_div(kcols, 64));
-            const int S = kb < c.pl.smax ? kb : c.pl.smax;
             GemmArgs g = gemm_args(c, static_cast<int>(q), bw, kb, EPI_TRAIL);
             set_prods(g, (frac || c.pl.grouped) ? 3 : 1);
+            int S = choose_splits(ceil_div(q, 128), kb, g.n_prod, c.nsm);
+            if (S > c.pl.smax) S = c.pl.smax;
             g.a_plane_rows = static_cast<int>(q);
             g.b_plane_rows = static_cast<int>(p);
             g.b_row0 = static_cast<int>(b0);
             g.out = c.part;
             g.ldo = B;
             g.split_stride = q * B;
+            g.gate = gate;
             Timed tm(c.timer, QE_KERNEL_TRAIL_GEMM, c.s);
             QE_CK(launch_tc_gemm(B, c.tm_dp, B == 64 ? c.tm_snt64 : (B == 128 ? c.tm_snt128 : c.tm_snt256), g,
                                  S, c.s));
@@ -479,6 +510,7 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
         a.ldd = ld;
         a.dp_plane_rows = q;
         a.err = c.err;
+        a.gate = gate;
         Timed tm(c.timer, QE_KERNEL_CD_BLOCK, c.s);
         QE_CK(launch_cd_block(B, a, c.nsm, c.s));
     }
@@ -547,6 +579,32 @@ static int dense_sweeps(const qe_opts *o) {
 
 static int relax_period(const qe_opts *o) { return o ? o->relax_period : 0; }
 
+// Whether the fp32 Sigma_bar rows that the list sweeps gather (4 p ld bytes) fit
+// in three quarters of this GPU's L2.
+static bool sbar_rows_fit_l2(int64_t p, int64_t ld) {
+    int dev = 0, l2 = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&l2, cudaDevAttrL2CacheSize, dev) != cudaSuccess ||
+        l2 <= 0) {
+        cudaGetLastError();
+        l2 = 128 << 20;
+    }
+    return 4.0 * static_cast<double>(p) * static_cast<double>(ld) <= 0.75 * static_cast<double>(l2);
+}
+
+// The adaptive schedule's switch threshold for layers whose Sigma_bar rows exceed
+// L2: a dense sweep costs its 6 q p^2 flops of bf16 plane products (~1.3 PFLOP/s
+// on 152 SMs, as measured for the trailing GEMMs) plus an in-block pass (~42 ps
+// per coordinate); a list sweep gathers one Sigma_bar row of 4 p bytes per change
+// (~8 TB/s from DRAM and L2 together, measured on the 14848 x 59392 layer); the
+// next sweep makes about 0.7 times the changes of the one just finished.
+static int64_t switch_below_model(int64_t q, int64_t p, int nsm) {
+    const double qd = static_cast<double>(q), pd = static_cast<double>(p);
+    const double t_dense = 6.0 * qd * pd * pd / (1.3e15 * nsm / 152.0) + 4.2e-11 * qd * pd;
+    const double t_change = 4.0 * pd / 8.0e12;
+    const double below = t_dense / t_change / 0.7;
+    return below > 9.0e18 ? static_cast<int64_t>(9.0e18) : static_cast<int64_t>(below);
+}
+
 static int free_changes(const qe_opts *o) {
     return (o && o->free_changes) ? o->free_changes : kFreeMaxChanges;
 }
@@ -560,7 +618,8 @@ static qe_status check_opts(const qe_opts *o, bool structured = false) {
     if (o->structured_outliers != 0 && !(structured && o->structured_outliers == 1)) return QE_ERR_UNSUPPORTED;
     if (o->block_width != 0 && o->block_width != 64 && o->block_width != 128 && o->block_width != 256)
         return QE_ERR_UNSUPPORTED;
-    if (o->power_iters < 0 || o->dense_sweeps < 0 || o->free_changes < -1 || o->group_size < 0)
+    if (o->power_iters < 0 || o->dense_sweeps < 0 || o->free_changes < -1 || o->group_size < 0 ||
+        o->switch_below < 0)
         return QE_ERR_INVALID_ARG;
     if (o->workspace && o->workspace_bytes == 0) return QE_ERR_INVALID_ARG;
     if (o->group_size > 0) {
@@ -803,6 +862,11 @@ qe_status qe_quantize_layer(const void *W, qe_dtype w_dtype, int64_t q, int64_t 
                                   static_cast<size_t>(q) * p, cudaMemcpyDeviceToDevice, c.s));
         return QE_OK;
     };
+    // sweep_forms[t0 .. t0 + n) = form (0 sequential, 1 dense, 2 lists)
+    auto form = [&](int t0, int n, int f) -> qe_status {
+        if (opts && opts->sweep_forms && n > 0) QE_CK(cudaMemsetAsync(opts->sweep_forms + t0, f, n, c.s));
+        return QE_OK;
+    };
     int t = 0, src = SRC_CODES;
     if (warm) {
         QE_CK(cudaMemcpyAsync(codes, opts->init_codes, static_cast<size_t>(q) * p, cudaMemcpyDeviceToDevice, c.s));
@@ -818,6 +882,7 @@ qe_status qe_quantize_layer(const void *W, qe_dtype w_dtype, int64_t q, int64_t 
             const ObjFuse f{obj, W, wbf16, ldw, codes, nullptr};
             if ((st = residual(c, scales, zeros, &f)) != QE_OK) return st;
             if ((st = record(0)) != QE_OK) return st;
+            if ((st = form(0, 1, 0)) != QE_OK) return st;
             t = 1;
             src = SRC_CODES;
         }
@@ -826,6 +891,19 @@ qe_status qe_quantize_layer(const void *W, qe_dtype w_dtype, int64_t q, int64_t 
     bool exact = true;   // R is the residual of the current What and no list has entries
     bool chain = false;  // the last sweep was a sequential one (its three-plane changes are in dp)
     const int dense = dense_sweeps(opts);
+    // adaptive schedule (dense_sweeps = 0): dense sweeps until one changes fewer than
+    // `below` codes, decided on the device after each sweep
+    bool adaptive = false;
+    int64_t below = 0;
+    if (!(opts && opts->dense_sweeps > 0)) {
+        if (opts && opts->switch_below > 0) {
+            adaptive = true;
+            below = opts->switch_below;
+        } else if (!sbar_rows_fit_l2(p, pl.ld)) {
+            adaptive = true;
+            below = switch_below_model(q, p, c.nsm);
+        }
+    }
     while (t < iters) {
         const bool rx = relaxed(t);
         if (rx || src != SRC_CODES) {
@@ -837,6 +915,7 @@ qe_status qe_quantize_layer(const void *W, qe_dtype w_dtype, int64_t q, int64_t 
             if ((st = sweep(c, codes, scales, zeros, bits, src, rx, exact ? -1 : 1)) != QE_OK) return st;
             QE_CK(launch_obj_step(c.rowdf, q, t == 0 ? c.objbase : obj + t - 1, obj + t, c.s));
             if ((st = record(t)) != QE_OK) return st;
+            if ((st = form(t, 1, 0)) != QE_OK) return st;
             ++t;
             src = rx ? SRC_V : SRC_CODES;
             exact = false;
@@ -854,10 +933,38 @@ qe_status qe_quantize_layer(const void *W, qe_dtype w_dtype, int64_t q, int64_t 
         // lists, persistent over blocks and sweeps
         int tend = t;
         while (tend < iters && !relaxed(tend)) ++tend;
+        if (adaptive && t < tend) {
+            // both forms of every sweep are enqueued; the flag (reset here, where the
+            // lists are empty or hold one sweep's changes) runs the dense form until
+            // the switch sets it, then the list form (one launch per sweep)
+            QE_CK(cudaMemsetAsync(c.swflag, 0, 16, c.s));   // flag and change counter
+            for (; t < tend; ++t) {
+                const double *prev_obj = t == 0 ? c.objbase : obj + t - 1;
+                if ((st = sweep(c, codes, scales, zeros, bits, SRC_CODES, false, exact ? -1 : 1, c.swflag)) != QE_OK)
+                    return st;
+                QE_CK(launch_obj_step(c.rowdf, q, prev_obj, obj + t, c.s, c.swflag, 0));
+                CdArgs a = list_args(c, codes, scales, zeros, bits);
+                a.gate = c.swflag;
+                a.gate_run = 1;
+                {
+                    Timed tm(c.timer, QE_KERNEL_CD_LISTS, c.s);
+                    QE_CK(launch_cd_rows_lists(pl.B, a, t, t + 1, c.rowdft, nullptr, 0, free_changes(opts), 0, c.nsm,
+                                               c.s));
+                }
+                QE_CK(launch_obj_prefix(c.rowdft, q, 1, prev_obj, obj + t, c.s, c.swflag, 1));
+                if ((st = record(t)) != QE_OK) return st;
+                if (opts && opts->sweep_forms) QE_CK(launch_record_form(c.swflag, opts->sweep_forms + t, c.s));
+                if (t + 1 < tend) QE_CK(launch_list_switch(c.lcnt, q * pl.nblk, below, c.swcount, c.swflag, c.s));
+                exact = false;
+                chain = false;
+            }
+            continue;
+        }
         for (; t < tend && t < dense; ++t) {
             if ((st = sweep(c, codes, scales, zeros, bits, SRC_CODES, false, exact ? -1 : 1)) != QE_OK) return st;
             QE_CK(launch_obj_step(c.rowdf, q, t == 0 ? c.objbase : obj + t - 1, obj + t, c.s));
             if ((st = record(t)) != QE_OK) return st;
+            if ((st = form(t, 1, 1)) != QE_OK) return st;
             exact = false;
             chain = false;
         }
@@ -871,6 +978,7 @@ qe_status qe_quantize_layer(const void *W, qe_dtype w_dtype, int64_t q, int64_t 
                                            exact ? 1 : 0, free_changes(opts), 0, c.nsm, c.s));
             }
             QE_CK(launch_obj_prefix(c.rowdft, q, te - t, t == 0 ? c.objbase : obj + t - 1, obj + t, c.s));
+            if ((st = form(t, te - t, 2)) != QE_OK) return st;
             t = te;
             exact = false;
             chain = false;

@@ -237,7 +237,9 @@ __global__ void k_init_residual(const void *W, int w_bf16, int64_t ldw, const fl
 }
 
 // obj_out = obj_prev + sum_i rowdf[i] (fixed order); rowdf is cleared.
-__global__ void k_obj_step(double *rowdf, int64_t q, const double *prev, double *out) {
+__global__ void k_obj_step(double *rowdf, int64_t q, const double *prev, double *out, const int *gate,
+                           int gate_run) {
+    if (gate && *gate != gate_run) return;
     __shared__ double sw[32];
     double acc = 0.0;
     for (int64_t k = threadIdx.x; k < q; k += blockDim.x) {
@@ -715,6 +717,7 @@ __device__ __forceinline__ int chg_decide(const float *tri, const float *d_blk, 
 // data-parallel passes (chg_decide).
 template <int B, bool FULL>
 __global__ void __launch_bounds__(1024, 1) k_cd_block_chg(const CdArgs a) {
+    if (a.gate && *a.gate != a.gate_run) return;   // uniform: the list form of the sweep runs
     using C = CdCfg<B>;
     constexpr int CPL = C::CPL;
     extern __shared__ __align__(16) float cd_smem[];
@@ -996,6 +999,7 @@ template <int B, bool GR>
 __global__ void __launch_bounds__(32 * kRowsMaxWarps, 1) k_cd_rows_lists(const CdArgs a, int t_begin, int t_end,
                                                            double *rowdf_t, uint8_t *sweep_codes,
                                                            int first_lockstep, int free_max_changes, int flush) {
+    if (a.gate && *a.gate != a.gate_run) return;   // uniform: the dense form of the sweep runs
     using C = CdCfg<B>;
     extern __shared__ __align__(16) float cd_smem[];
     float *tri = cd_smem;
@@ -1128,7 +1132,9 @@ __global__ void __launch_bounds__(32 * kRowsMaxWarps, 1) k_cd_rows_lists(const C
 // obj[t] = obj[t-1] + sum_i rowdf_t[t][i] for nt <= 32 sweeps; prev may be NULL (0).
 // Warp t sums sweep t (lane-strided, then a fixed butterfly: a fixed order); one
 // thread then runs the prefix over the sweeps.
-__global__ void k_obj_prefix(const double *rowdf_t, int64_t q, int nt, const double *prev, double *out) {
+__global__ void k_obj_prefix(const double *rowdf_t, int64_t q, int nt, const double *prev, double *out,
+                             const int *gate, int gate_run) {
+    if (gate && *gate != gate_run) return;
     __shared__ double sw[32];
     const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (w < nt) {
@@ -1227,9 +1233,52 @@ cudaError_t launch_cd_rows_lists(int B, const CdArgs &a, int t_begin, int t_end,
 }
 
 cudaError_t launch_obj_prefix(const double *rowdf_t, int64_t q, int nt, const double *prev, double *out,
-                              cudaStream_t s) {
+                              cudaStream_t s, const int *gate, int gate_run) {
     if (nt < 1 || nt > 32) return cudaErrorInvalidValue;
-    k_obj_prefix<<<1, 32 * nt, 0, s>>>(rowdf_t, q, nt, prev, out);
+    k_obj_prefix<<<1, 32 * nt, 0, s>>>(rowdf_t, q, nt, prev, out, gate, gate_run);
+    return cudaGetLastError();
+}
+
+// Sum of the list entry counts (the changes of the sweep just finished), per CTA
+// then one 64-bit atomic add per CTA (integer sums: the order does not matter).
+__global__ void __launch_bounds__(256) k_count_changes(const int *lcnt, int64_t n, const int *flag,
+                                                       unsigned long long *counter) {
+    if (*flag) return;
+    __shared__ unsigned long long sw[8];
+    unsigned long long acc = 0;
+    for (int64_t k = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; k < n;
+         k += static_cast<int64_t>(gridDim.x) * blockDim.x)
+        acc += static_cast<unsigned long long>(lcnt[k]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if ((threadIdx.x & 31) == 0) sw[threadIdx.x >> 5] = acc;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        unsigned long long t = 0;
+        for (int w = 0; w < 8; ++w) t += sw[w];
+        if (t) atomicAdd(counter, t);
+    }
+}
+
+__global__ void k_switch_decide(unsigned long long *counter, long long below, int *flag) {
+    if (*flag == 0 && *counter < static_cast<unsigned long long>(below)) *flag = 1;
+    *counter = 0ull;
+}
+
+__global__ void k_record_form(const int *flag, uint8_t *form) { *form = *flag ? 2 : 1; }
+
+cudaError_t launch_record_form(const int *flag, uint8_t *form, cudaStream_t s) {
+    k_record_form<<<1, 1, 0, s>>>(flag, form);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_list_switch(const int *lcnt, int64_t n, int64_t below, unsigned long long *counter, int *flag,
+                               cudaStream_t s) {
+    if (n < 1 || below < 0) return cudaErrorInvalidValue;
+    int64_t blocks = ceil_div(n, 256 * 16);
+    if (blocks > 1024) blocks = 1024;
+    k_count_changes<<<static_cast<unsigned>(blocks), 256, 0, s>>>(lcnt, n, flag, counter);
+    k_switch_decide<<<1, 1, 0, s>>>(counter, static_cast<long long>(below), flag);
     return cudaGetLastError();
 }
 
@@ -1503,8 +1552,9 @@ cudaError_t launch_init_residual(const void *W, int w_bf16, int64_t ldw, const f
     return cudaGetLastError();
 }
 
-cudaError_t launch_obj_step(double *rowdf, int64_t q, const double *prev, double *out, cudaStream_t s) {
-    k_obj_step<<<1, 1024, 0, s>>>(rowdf, q, prev, out);
+cudaError_t launch_obj_step(double *rowdf, int64_t q, const double *prev, double *out, cudaStream_t s,
+                            const int *gate, int gate_run) {
+    k_obj_step<<<1, 1024, 0, s>>>(rowdf, q, prev, out, gate, gate_run);
     return cudaGetLastError();
 }
 

@@ -51,6 +51,47 @@ struct GemmCfg {
 // traffic; every 8 steps gains ~1% more for twice the bias.
 constexpr int kChunkSteps = 4;
 
+// Sigma's tile order.  Only the tiles on or above the diagonal run (the mirror
+// writes the rest).  They are taken in groups of kSigmaGroupM consecutive tile
+// rows; inside a group the tile row runs fastest, then the tile column, from the
+// first column that reaches the group's diagonal.  A wave of CTAs then covers a
+// compact patch of tiles: at a given k-step it reads a few hundred kilobytes of
+// distinct rows of X, where row-by-row order (one tile row against 152 tile
+// columns) read several megabytes per k-step and left the GEMM waiting on DRAM
+// for wide layers.
+constexpr int kSigmaGroupM = 8;
+
+// Tiles of group gi (tile rows [gi * kSigmaGroupM, ...)), counting from the
+// first tile column whose BN columns reach the group's first row.
+__host__ __device__ __forceinline__ int64_t sigma_group_tiles(int gi, int mt, int nt, int BN) {
+    const int mlo = gi * kSigmaGroupM;
+    const int gm = (mt - mlo) < kSigmaGroupM ? (mt - mlo) : kSigmaGroupM;
+    const int ns = static_cast<int>((static_cast<int64_t>(mlo) * 128) / BN);
+    return static_cast<int64_t>(gm) * (nt - ns);
+}
+
+__host__ __device__ __forceinline__ int64_t sigma_tiles(int mt, int nt, int BN) {
+    int64_t t = 0;
+    for (int gi = 0; gi * kSigmaGroupM < mt; ++gi) t += sigma_group_tiles(gi, mt, nt, BN);
+    return t;
+}
+
+// Linear tile id -> (tile row, tile column) in the grouped order.
+__host__ __device__ __forceinline__ void sigma_tile(int64_t id, int mt, int nt, int BN, int &m, int &n) {
+    int gi = 0;
+    for (;;) {
+        const int64_t t = sigma_group_tiles(gi, mt, nt, BN);
+        if (id < t || (gi + 1) * kSigmaGroupM >= mt) break;
+        id -= t;
+        ++gi;
+    }
+    const int mlo = gi * kSigmaGroupM;
+    const int gm = (mt - mlo) < kSigmaGroupM ? (mt - mlo) : kSigmaGroupM;
+    const int ns = static_cast<int>((static_cast<int64_t>(mlo) * 128) / BN);
+    m = mlo + static_cast<int>(id % gm);
+    n = ns + static_cast<int>(id / gm);
+}
+
 __device__ __forceinline__ float load_w(const GemmArgs &g, int64_t r, int64_t c) {
     if (g.w_is_bf16)
         return __bfloat162float(reinterpret_cast<const __nv_bfloat16 *>(g.W)[r * g.ldw + c]);
@@ -343,6 +384,7 @@ __global__ void __launch_bounds__(320, 1)
     k_tc_gemm(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb,
               const GemmArgs g) {
     using C = GemmCfg<BN>;
+    if (g.gate && *g.gate != g.gate_run) return;   // uniform: the other form of the sweep runs
     extern __shared__ uint8_t smem_raw[];
     const uint32_t pad = (1024u - (smem_u32(smem_raw) & 1023u)) & 1023u;
     uint8_t *smem = smem_raw + pad;
@@ -356,9 +398,20 @@ __global__ void __launch_bounds__(320, 1)
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
     // m_fast: consecutive CTAs walk down M, so a wave shares a few B column
-    // slices (each read once from DRAM) instead of sweeping all of B
-    const int m0 = (g.m_fast ? blockIdx.x : blockIdx.y) * C::BM;
-    const int n0 = (g.m_fast ? blockIdx.y : blockIdx.x) * BN;
+    // slices (each read once from DRAM) instead of sweeping all of B.  Sigma:
+    // the 1-D grid runs over the tiles on or above the diagonal in groups of
+    // kSigmaGroupM tile rows (sigma_tile).
+    int m0, n0;
+    if (g.mode == EPI_SIGMA) {
+        int mt_, nt_;
+        sigma_tile(static_cast<int64_t>(blockIdx.x), static_cast<int>(ceil_div(g.M, C::BM)),
+                   static_cast<int>(ceil_div(g.N, BN)), BN, mt_, nt_);
+        m0 = mt_ * C::BM;
+        n0 = nt_ * BN;
+    } else {
+        m0 = (g.m_fast ? blockIdx.x : blockIdx.y) * C::BM;
+        n0 = (g.m_fast ? blockIdx.y : blockIdx.x) * BN;
+    }
     // Sigma: a tile whose every element lies strictly below the diagonal is
     // produced by the mirror of its transpose (uniform exit, before any barrier).
     if (g.mode == EPI_SIGMA && n0 + BN <= m0) return;
@@ -553,6 +606,11 @@ static cudaError_t launch_bn(const CUtensorMap &ta, const CUtensorMap &tb, const
     if (e != cudaSuccess) return e;
     const unsigned nt = static_cast<unsigned>(ceil_div(g.N, BN)), mt = static_cast<unsigned>(ceil_div(g.M, C::BM));
     dim3 grid(g.m_fast ? mt : nt, g.m_fast ? nt : mt, static_cast<unsigned>(splits));
+    if (g.mode == EPI_SIGMA) {
+        const int64_t tiles = sigma_tiles(static_cast<int>(mt), static_cast<int>(nt), BN);
+        if (tiles > 0x7fffffffll) return cudaErrorInvalidValue;
+        grid = dim3(static_cast<unsigned>(tiles), 1, static_cast<unsigned>(splits));
+    }
     k_tc_gemm<BN, GR><<<grid, C::THREADS, C::SMEM_BYTES, s>>>(ta, tb, g);
     return cudaGetLastError();
 }
@@ -561,7 +619,8 @@ cudaError_t launch_tc_gemm(int BN, const CUtensorMap &ta, const CUtensorMap &tb,
                            int splits, cudaStream_t s) {
     if (g.M <= 0 || g.N <= 0 || splits < 1 || g.n_prod < 1 || g.n_prod > 6)
         return cudaErrorInvalidValue;
-    if ((g.m_fast ? ceil_div(g.N, BN) : ceil_div(g.M, 128)) > 65535 || splits > 65535) return cudaErrorInvalidValue;
+    if (g.mode != EPI_SIGMA && (g.m_fast ? ceil_div(g.N, BN) : ceil_div(g.M, 128)) > 65535) return cudaErrorInvalidValue;
+    if (splits > 65535) return cudaErrorInvalidValue;
     switch (BN) {
         case 64: return launch_bn<64, false>(ta, tb, g, splits, s);
         case 128: return launch_bn<128, false>(ta, tb, g, splits, s);

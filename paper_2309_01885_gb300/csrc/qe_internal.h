@@ -51,6 +51,10 @@ struct GemmArgs {
     const float *Hd;
     int64_t ldh;
     unsigned *err;
+    // optional gate: the launch does its work only when *gate == gate_run (the
+    // adaptive sweep schedule enqueues both forms of a sweep and runs one)
+    const int *gate;
+    int gate_run;
 };
 
 // The per-device error word that qe_sync_status reads and clears.

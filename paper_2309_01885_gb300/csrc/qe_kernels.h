@@ -49,6 +49,10 @@ struct CdArgs {
     __nv_bfloat16 *dp;              // out: Delta' hi plane (mid / lo planes dp_plane_rows apart), or NULL
     int64_t ldd, dp_plane_rows;
     unsigned *err;
+    // optional gate: the launch does its work only when *gate == gate_run (the
+    // adaptive sweep schedule enqueues both forms of a sweep and runs one)
+    const int *gate;
+    int gate_run;
 };
 
 // Objective / reference-norm reduction.
@@ -80,8 +84,18 @@ cudaError_t launch_make_planes(const void *W, int w_bf16, int64_t ldw, int64_t q
 cudaError_t launch_init_residual(const void *W, int w_bf16, int64_t ldw, const float *H, int64_t ldh,
                                  int64_t q, int64_t p, int64_t gsize, const float *scale, const float *zero,
                                  float *R, int64_t ldr, cudaStream_t s);
-// obj[out] = obj[prev] + sum_i rowdf[i]; rowdf is zeroed.  prev may be NULL (0).
-cudaError_t launch_obj_step(double *rowdf, int64_t q, const double *prev, double *out, cudaStream_t s);
+// obj[out] = obj[prev] + sum_i rowdf[i]; rowdf is zeroed.  prev may be NULL (0).  With a
+// gate, only when *gate == gate_run.
+cudaError_t launch_obj_step(double *rowdf, int64_t q, const double *prev, double *out, cudaStream_t s,
+                            const int *gate = nullptr, int gate_run = 0);
+// The adaptive sweep schedule's switch: counts the entries of the change lists
+// (the changes of the sweep just finished, n = q * nblk counts) and sets *flag = 1
+// when they are fewer than `below`; a set flag stays set (no work then).  counter:
+// one 8-byte device word of scratch.
+// *form = *flag ? 2 : 1 (which form of the adaptive schedule ran the sweep just enqueued).
+cudaError_t launch_record_form(const int *flag, uint8_t *form, cudaStream_t s);
+cudaError_t launch_list_switch(const int *lcnt, int64_t n, int64_t below, unsigned long long *counter, int *flag,
+                               cudaStream_t s);
 // C - z (one exact bf16 plane), or with grouped grids s_g (C - z_g) in three planes
 // (rows [0, q), [q, 2q), [2q, 3q)); gsize = p: per-row grids.
 cudaError_t launch_codes_to_qf(const uint8_t *codes, int64_t ldc, const float *scale, const float *zero,
@@ -101,9 +115,10 @@ cudaError_t launch_cd_block(int B, const CdArgs &a, int nsm, cudaStream_t s);
 cudaError_t launch_cd_rows_lists(int B, const CdArgs &a, int t_begin, int t_end, double *rowdf_t,
                                  uint8_t *sweep_codes, int first_lockstep, int free_max_changes, int flush,
                                  int nsm, cudaStream_t s);
-// obj[t] = obj[t-1] + sum_i rowdf_t[t][i] for t < nt, starting from *prev (or 0).
+// obj[t] = obj[t-1] + sum_i rowdf_t[t][i] for t < nt, starting from *prev (or 0).  With a
+// gate, only when *gate == gate_run.
 cudaError_t launch_obj_prefix(const double *rowdf_t, int64_t q, int nt, const double *prev, double *out,
-                              cudaStream_t s);
+                              cudaStream_t s, const int *gate = nullptr, int gate_run = 0);
 int64_t packed_diag_floats(int64_t p, int B);
 cudaError_t launch_pack_diag(const __nv_bfloat16 *snt, int64_t ldn, int64_t p, int B, float *out,
                              cudaStream_t s);

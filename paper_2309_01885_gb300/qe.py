@@ -42,7 +42,8 @@ class QEOpts(ctypes.Structure):
                 ("dense_sweeps", ctypes.c_int), ("free_changes", ctypes.c_int), ("group_size", ctypes.c_int),
                 ("init_codes", ctypes.c_void_p), ("sweep_codes", ctypes.c_void_p),
                 ("wx_norm2", ctypes.c_void_p), ("workspace", ctypes.c_void_p),
-                ("workspace_bytes", ctypes.c_size_t), ("timer", ctypes.c_void_p)]
+                ("workspace_bytes", ctypes.c_size_t), ("timer", ctypes.c_void_p),
+                ("switch_below", ctypes.c_int64), ("sweep_forms", ctypes.c_void_p)]
 
 
 _lib = None
@@ -228,8 +229,9 @@ class Timer:
 
 def _opts(block_width=0, power_iters=0, init_codes=None, sweep_codes=None, wx_norm2=None,
           workspace=None, timer=None, dense_sweeps=0, free_changes=0, relax_period=0,
-          group_size=0) -> QEOpts:
+          group_size=0, switch_below=0) -> QEOpts:
     o = QEOpts()
+    o.switch_below = switch_below
     o.group_size = group_size
     o.relax_period = relax_period
     o.timer = None if timer is None else timer.handle.value
@@ -292,13 +294,16 @@ def qe_quantize_layer(W: torch.Tensor, Sigma: torch.Tensor, bits: int, iters: in
                       want_norm: bool = False, block_width: int = 0,
                       workspace: torch.Tensor | None = None, timer: Timer | None = None,
                       dense_sweeps: int = 0, free_changes: int = 0, relax_period: int = 0,
-                      group_size: int = 0, stream=None) -> dict:
+                      group_size: int = 0, switch_below: int = 0, record_forms: bool = False,
+                      stream=None) -> dict:
     """QuantEase on one layer; returns codes (u8 q x p), scales, zeros, obj (fp64 per sweep),
     and optionally sweep_codes (iters x q x p) and wx_norm2.  dense_sweeps: sweeps whose
-    cross-block term uses the tensor-core GEMM before the change lists take over (0 = default);
+    cross-block term uses the tensor-core GEMM before the change lists take over (0 = the
+    adaptive schedule: dense until a sweep changes fewer than switch_below codes, 0 = automatic);
     free_changes: changes per row below which list sweeps run row by row (0 = default, -1 = never);
     relax_period: the relax heuristic of Sec. 3.2 (sweep t from 1 with t mod R = 0 and t < iters
-    keeps beta~ unquantized; 0 = off); group_size: grouped grids (scales / zeros q x groups)."""
+    keeps beta~ unquantized; 0 = off); group_size: grouped grids (scales / zeros q x groups);
+    record_forms: also return sweep_forms (uint8 per sweep: 0 sequential, 1 dense, 2 lists)."""
     q, p = W.shape
     dev = W.device
     codes = torch.empty(q, p, dtype=torch.uint8, device=dev)
@@ -309,7 +314,9 @@ def qe_quantize_layer(W: torch.Tensor, Sigma: torch.Tensor, bits: int, iters: in
     sweep = torch.empty(iters, q, p, dtype=torch.uint8, device=dev) if record_sweeps else None
     norm = torch.empty(1, dtype=torch.float64, device=dev) if want_norm else None
     o = _opts(block_width, 0, init_codes, sweep, norm, workspace, timer, dense_sweeps, free_changes,
-              relax_period, group_size)
+              relax_period, group_size, switch_below)
+    forms = torch.full((iters,), 255, dtype=torch.uint8, device=dev) if record_forms else None
+    o.sweep_forms = None if forms is None else forms.data_ptr()
     _check(load().qe_quantize_layer(_ptr(W), _dtype(W), q, p, _rowmajor_ld(W), _ptr(Sigma), bits, iters,
                                     ctypes.byref(o), _ptr(codes), _ptr(scales), _ptr(zeros), _ptr(obj),
                                     _stream(stream)), "qe_quantize_layer")
@@ -318,6 +325,8 @@ def qe_quantize_layer(W: torch.Tensor, Sigma: torch.Tensor, bits: int, iters: in
         out["sweep_codes"] = sweep
     if want_norm:
         out["wx_norm2"] = norm
+    if record_forms:
+        out["sweep_forms"] = forms
     return out
 
 

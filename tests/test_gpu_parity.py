@@ -250,6 +250,57 @@ def test_layer_lists_agree_with_dense():
     assert m >= parity.CODE_MATCH, f"codes match {m:.5f}"
 
 
+@pytest.mark.parametrize("group_size", [0, 256])
+def test_layer_adaptive_schedule(group_size):
+    """The adaptive sweep schedule (dense form until a sweep changes fewer than
+    switch_below codes, then the change lists, chosen on the device): with a
+    threshold no sweep reaches it is the all-dense schedule bit for bit; with one
+    every sweep reaches it switches after sweep 2 and is the dense_sweeps = 2
+    schedule bit for bit (one list launch per sweep against one for all); with a
+    threshold between the two it switches mid-way and meets the parity bar
+    against the oracle (teacher-forced decisions, objectives, codes).  p = 1000
+    leaves a ragged last block."""
+    q, p, iters, bits = 200, 1000, 8, 3
+    W = inputs.layer_weights(q, p, dtype=torch.bfloat16, seed=63, device="cuda")
+    X = inputs.calib_inputs(p, 8192, dtype=torch.bfloat16, seed=63, device="cuda",
+                            heavy_frac=0.01, heavy_mult=30.0)
+    Sg = qe.qe_build_sigma(X)
+    kw = dict(record_sweeps=True, group_size=group_size, record_forms=True)
+    dense_all = qe.qe_quantize_layer(W, Sg, bits, iters, dense_sweeps=100, **kw)
+    never = qe.qe_quantize_layer(W, Sg, bits, iters, switch_below=1, **kw)
+    dense2 = qe.qe_quantize_layer(W, Sg, bits, iters, dense_sweeps=2, **kw)
+    always = qe.qe_quantize_layer(W, Sg, bits, iters, switch_below=q * p, **kw)
+    assert qe.qe_sync_status() == qe.QE_OK
+    changes = [int((dense_all["sweep_codes"][t] != dense_all["sweep_codes"][t - 1]).sum().item())
+               for t in range(1, iters)]
+    assert all(c > 0 for c in changes), changes      # switch_below = 1 never switches
+    for x, y in ((never, dense_all), (always, dense2)):
+        for key in ("codes", "obj", "sweep_codes", "sweep_forms"):
+            assert torch.equal(x[key], y[key]), key
+    assert dense_all["sweep_forms"].tolist() == [0] + [1] * (iters - 1)
+    assert dense2["sweep_forms"].tolist() == [0, 1] + [2] * (iters - 2)
+    # the fourth sweep's count as the threshold: dense at least through sweep 5, lists
+    # from the sweep after the first one that changes fewer codes
+    mid = changes[2]
+    out = qe.qe_quantize_layer(W, Sg, bits, iters, switch_below=mid, want_norm=True, **kw)
+    assert qe.qe_sync_status() == qe.QE_OK
+    forms = out["sweep_forms"].tolist()
+    assert forms[:5] == [0, 1, 1, 1, 1] and forms == sorted(forms), forms
+    if group_size:
+        W64 = parity.f64(W)
+        S64 = parity.f64(Sg)
+        s, z = O.grid(W64, bits, group_size=group_size)
+        assert np.array_equal(out["scales"].cpu().numpy(), s)
+        sweep = out["sweep_codes"].cpu().numpy()
+        parity.teacher_forced(W64, S64, s, z, bits, sweep, group_size=group_size)
+        ref = O.alg1(W64, S64, s, z, bits, iters, group_size=group_size)
+        parity.check_obj(out["obj"].cpu().numpy(), ref["obj"], what="adaptive, groups")
+    else:
+        _check_layer(W, Sg, out, bits, iters, free_running=True)
+    obj = out["obj"].cpu().numpy()
+    assert np.all(np.diff(obj) <= 1e-6 * obj[:-1])
+
+
 @pytest.mark.parametrize("p,group_size", [(640, 0), (1000, 0), (1000, 256)])
 def test_layer_list_modes_identical(p, group_size):
     """The list sweeps in lockstep (shared packed Sigma_bar block, lists read from
