@@ -78,6 +78,9 @@ class Oracle:
         lib.qo_quantease_alg1.argtypes = [_f64p, _i64, _i64, _f64p, _f32p, _f32p, _int, _int,
                                           _u8p, _u8p, _u8p, _f64p, _u8p, _f64p, _int]
         lib.qo_quantease_alg1.restype = _int
+        lib.qo_iht_step.argtypes = [_f64p, _i64, _i64, _f64p, _u8p, _f32p, _f32p, _f64p, ctypes.c_double,
+                                    _i64, _int, _f64p, _i64p]
+        lib.qo_iht_step.restype = _i64
         lib.qo_quantease_alg1_f32.argtypes = [_f64p, _i64, _i64, _f32p, _f32p, _f32p, _int, _int,
                                               _u8p, _u8p, _u8p, _f64p, _u8p, _f64p, _int]
         lib.qo_quantease_alg1_f32.restype = _int
@@ -242,6 +245,26 @@ class Oracle:
         idx = np.empty(max(T.shape[1], 1), np.int64)
         cnt = self.lib.qo_topk_columns(_ptr(T, _f64p), T.shape[0], T.shape[1], int(k), _ptr(idx, _i64p))
         return idx[:cnt].copy()
+
+    def iht_step(self, W, S, codes, scale, zero, H, eta, s_budget, structured=False):
+        """One IHT half-step of Algorithm 4 from the state (codes on the grid, H):
+        returns (T, support) with T = H - 2 eta (H + What - W) Sigma and the support of
+        P_s(T) (ascending linear indices; the column selection with structured)."""
+        W = _f64(W)
+        S = _f64(S)
+        q, p = W.shape
+        H = _f64(H)
+        T = np.empty((q, p), np.float64)
+        idx = np.empty(max(int(s_budget), 1), np.int64)
+        cnt = self.lib.qo_iht_step(_ptr(W, _f64p), q, p, _ptr(S, _f64p),
+                                   _ptr(np.ascontiguousarray(codes, np.uint8), _u8p),
+                                   _ptr(np.ascontiguousarray(scale, np.float32), _f32p),
+                                   _ptr(np.ascontiguousarray(zero, np.float32), _f32p),
+                                   _ptr(H, _f64p), float(eta), int(s_budget), int(structured),
+                                   _ptr(T, _f64p), _ptr(idx, _i64p))
+        if cnt < 0:
+            raise MemoryError("oracle iht_step allocation failed")
+        return T, idx[:cnt].copy()
 
     def outlier(self, W, S, bits, iters, s_budget, power_iters, structured=False):
         W = _f64(W)

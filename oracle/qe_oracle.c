@@ -736,3 +736,37 @@ int qo_quantease_outlier(const double *W, int64_t q, int64_t p, const double *S,
     free(idx); free(cols); free(excl); free(Wh); free(T); free(rows);
     return 0;
 }
+
+/*
+ * One IHT half-step of Algorithm 4 entered from a given state: the codes on the
+ * grid (scale, zero) give What, H is the current outlier matrix (dense q*p), and
+ *   G = 2 (H + What - W) Sigma,   T = H - eta G,   H_new = P_s(T)
+ * (the column selection of qo_topk_columns with `structured`).  Writes T (q*p)
+ * and the support of H_new (ascending linear indices, at most s_budget entries;
+ * H_new = T there) and returns its size.  These are the steps of the IHT half of
+ * qo_quantease_outlier; a test uses them to replay another implementation's
+ * iterations one at a time from that implementation's own state.
+ */
+int64_t qo_iht_step(const double *W, int64_t q, int64_t p, const double *S, const uint8_t *codes,
+                    const float *scale, const float *zero, const double *H, double eta,
+                    int64_t s_budget, int structured, double *T, int64_t *idx)
+{
+    const qo_sig Sg = {S, NULL, p};
+    int64_t *cols = (int64_t *)malloc((size_t)(p > 0 ? p : 1) * sizeof(int64_t));
+    if (!cols)
+        return -1;
+#pragma omp parallel for schedule(dynamic)
+    for (int64_t i = 0; i < q; ++i) {
+        double *D = (double *)malloc((size_t)p * sizeof(double));
+        double *G = (double *)malloc((size_t)p * sizeof(double));
+        for (int64_t j = 0; j < p; ++j)
+            D[j] = H[i * p + j] + qo_level(codes[i * p + j], scale[i], zero[i]) - W[i * p + j];
+        qo_row_times_sigma(D, &Sg, p, G, NULL);  /* G/2 = (H + What - W) Sigma */
+        for (int64_t j = 0; j < p; ++j)
+            T[i * p + j] = H[i * p + j] - 2.0 * eta * G[j];   /* 2 eta = eta 2 exactly */
+        free(D); free(G);
+    }
+    const int64_t nnz = qo_select(T, q, p, s_budget, structured, idx, cols);
+    free(cols);
+    return nnz;
+}

@@ -33,6 +33,10 @@ MUTANTS = [
      "if (x->idx < y->idx) return 1;"),
     ("iht_wrong_step_sign", "T[i * p + j] = H[i * p + j] - eta * 2.0 * G[j];",
      "T[i * p + j] = H[i * p + j] + eta * 2.0 * G[j];"),
+    ("iht_step_wrong_sign", "T[i * p + j] = H[i * p + j] - 2.0 * eta * G[j];",
+     "T[i * p + j] = H[i * p + j] + 2.0 * eta * G[j];"),
+    ("iht_step_target_not_level", "D[j] = H[i * p + j] + qo_level(codes[i * p + j], scale[i], zero[i]) - W[i * p + j];",
+     "D[j] = H[i * p + j] + W[i * p + j] - W[i * p + j];"),
     ("power_wrong_rayleigh", "lam += v[a] * w[a];", "lam += w[a] * w[a];"),
     ("column_norm_not_squared", "norm2[j] += T[i * p + j] * T[i * p + j];", "norm2[j] += T[i * p + j];"),
     ("relax_keeps_level", "                Wh[j] = b;\n", "                Wh[j] = qo_level(c, s, z);\n"),
@@ -64,6 +68,8 @@ PINS = [
     pins.test_grouped_diagonal_sigma_gives_per_group_round_to_nearest,
     lambda: pins.test_grouped_update_is_bruteforce_argmin_on_its_group(2),
     golden.test_hand_worked_two_feature_layer,
+    lambda: pins.test_iht_step_gradient_and_projection(False),
+    pins.test_iht_step_replays_algorithm4,
 ]
 
 

@@ -433,6 +433,69 @@ def test_outlier_iht_descent_and_budget():
     assert np.isclose(r["obj"][-1], _f_direct(W, What + r["H"], X), rtol=1e-10)
 
 
+@pytest.mark.parametrize("structured", [False, True])
+def test_iht_step_gradient_and_projection(structured):
+    """The IHT half-step entered from outside state (used to replay the GPU's
+    iterations): with a budget that keeps everything, (H - T) / eta is the gradient
+    of g(H) = ||(W - What - H) X||^2 (Eq. main-outlier), checked by central
+    differences of g computed from X itself; with a small budget the support is the
+    s largest |T| (a full sort) or the columns of largest norm (brute force over
+    column subsets), and the step never increases g (Lemma 3)."""
+    rng = np.random.default_rng(31)
+    q, p, n, bits = 4, 6, 30, 3
+    W, X = _rand_layer(rng, q, p, n, heavy=(2,), heavy_mult=6.0)
+    S = O.sigma(X)
+    s_, z_ = O.grid(W, bits)
+    codes = O.rtn(W, s_, z_, bits)
+    What = levels(codes, s_, z_)
+    H = np.zeros((q, p))
+    H[rng.integers(0, q, 5), rng.integers(0, p, 5)] = rng.normal(0, 0.1, 5)
+    eta = 1.0 / (2.0 * np.linalg.eigvalsh(S)[-1])
+    T, sup = O.iht_step(W, S, codes, s_, z_, H, eta, q * p, structured)
+    grad = (H - T) / eta
+    eps = 1e-6
+    for i in range(q):
+        for j in range(p):
+            E = np.zeros((q, p))
+            E[i, j] = eps
+            fd = (_f_direct(W - H - E, What, X) - _f_direct(W - H + E, What, X)) / (2 * eps)
+            assert abs(fd - grad[i, j]) <= 1e-5 * max(1.0, abs(fd)), (i, j, fd, grad[i, j])
+    # projection and descent with a small budget
+    s_budget = 8 if not structured else 2 * q
+    T, sup = O.iht_step(W, S, codes, s_, z_, H, eta, s_budget, structured)
+    if structured:
+        norms = np.sum(T * T, axis=0)
+        best = max(itertools.combinations(range(p), s_budget // q), key=lambda c: norms[list(c)].sum())
+        assert sorted({int(k) % p for k in sup}) == sorted(best)
+        assert sup.size == s_budget
+    else:
+        order = np.argsort(-np.abs(T).ravel(), kind="stable")
+        assert np.array_equal(np.sort(order[:s_budget]), sup)
+    Hn = np.zeros(q * p)
+    Hn[sup] = T.ravel()[sup]
+    Hn = Hn.reshape(q, p)
+    assert _f_direct(W - Hn, What, X) <= _f_direct(W - H, What, X) * (1 + 1e-12)
+
+
+def test_iht_step_replays_algorithm4():
+    """From the state one oracle iteration of Algorithm 4 leaves behind (the start
+    H = P_s(W) and the codes of the first sweep), the IHT step gives that
+    iteration's H bit for bit."""
+    rng = np.random.default_rng(32)
+    q, p, n, s_budget = 10, 20, 60, 15
+    W, X = _rand_layer(rng, q, p, n, heavy=(3,), heavy_mult=10.0)
+    W[rng.integers(0, q, 6), rng.integers(0, p, 6)] += rng.normal(0, 0.3, 6)
+    S = O.sigma(X)
+    r = O.outlier(W, S, 3, 1, s_budget, 200)
+    H0 = np.zeros(q * p)
+    k0 = O.topk(W, s_budget)
+    H0[k0] = W.ravel()[k0]
+    T, sup = O.iht_step(W, S, r["codes"], r["scale"], r["zero"], H0.reshape(q, p), r["eta"], s_budget)
+    Hn = np.zeros(q * p)
+    Hn[sup] = T.ravel()[sup]
+    assert np.array_equal(Hn.reshape(q, p), r["H"])
+
+
 def test_outlier_with_zero_budget_reduces_to_algorithm1():
     rng = np.random.default_rng(14)
     W, X = _rand_layer(rng, 8, 20, 50, corr=True)
