@@ -142,6 +142,23 @@ typedef struct {
      * sweep and the sweep after one), 1 = the dense tensor-core form, 2 = the
      * change lists.  NULL = not recorded.  Ignored by the outlier variant. */
     uint8_t *sweep_forms;
+    /* Test hook of the failure path (no paper counterpart): 1 = qe_quantize_layer
+     * (without init_codes; ignored by the outlier variant) runs up to its first
+     * in-block kernel, which issues no copy of its packed
+     * Sigma_bar block and waits for it with a 5 ms limit.  The wait gives up,
+     * QE_ERR_TIMEOUT is latched for qe_sync_status, and the call returns QE_OK
+     * without further work (codes, scales, zeros and obj are not all written).
+     * Nothing is left in flight, so the next call runs normally.  0 = off. */
+    int wait_test;
+    /* Near-tie refinement (no paper counterpart: it makes the binary32 kernels
+     * take the decisions exact arithmetic takes).  A coordinate update rounds
+     * beta~ / s + z (Lemma 1) to the nearest level; where that binary32 value
+     * lies within tie_eps grid steps of a midpoint between two levels, the
+     * decision is taken again from beta~ recomputed in binary64 from the row's
+     * current codes, W (and H) and Sigma.  0 = default (2e-5, about ten times the
+     * largest binary32 error measured on the benchmark layers); negative = off.
+     * Not applied in relaxed sweeps or the sweep after one. */
+    float tie_eps;
 } qe_opts;
 
 /*
@@ -261,7 +278,10 @@ qe_status qe_build_sigma_host(const void *X, int64_t p, int64_t n, int64_t ldx, 
  *   8 MiB); larger p returns QE_ERR_INVALID_ARG before anything is enqueued.
  *   First call per device: looks up the array's device address (with that
  *   device current) and caches it; make that first call before any stream
- *   capture.
+ *   capture.  The cached address is not looked up again: resetting the device
+ *   (cudaDeviceReset) after the first call and then calling again is not
+ *   supported (the same holds for the device error word every entry point
+ *   caches, see qe_sync_status).
  *   Every call shares the array: calls that overlap on the GPU (other streams,
  *   other host threads) race.  Each call clears the part of the array it relies
  *   on being zero.
@@ -331,7 +351,10 @@ qe_status qe_hard_threshold(const float *T, int64_t N, int64_t s, int64_t *idx, 
                             void *workspace, size_t workspace_bytes, qe_stream_t stream);
 
 /* Waits for `stream`, then returns and clears the error latched on the current
- * device (QE_ERR_NUMERIC / QE_ERR_TIMEOUT), or QE_ERR_CUDA if the stream failed. */
+ * device (QE_ERR_NUMERIC / QE_ERR_TIMEOUT), or QE_ERR_CUDA if the stream failed.
+ * The error word is a file-scope device variable whose address the library looks
+ * up once per device and caches; calling the library on a device after a
+ * cudaDeviceReset of that device is not supported. */
 qe_status qe_sync_status(qe_stream_t stream);
 
 /* Static description of a status code. */

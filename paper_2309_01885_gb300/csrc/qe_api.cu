@@ -225,6 +225,13 @@ struct Ctx {
     int64_t *ccols = nullptr, *cn = nullptr;
     CUtensorMap tm_snt256, tm_snt64, tm_snt128, tm_qf, tm_dp, tm_wa;
     int wa_planes = 1;
+    // near-tie refinement: the layer's inputs as given (and H for the outlier variant)
+    float tie_eps = 0.0f;
+    const float *Sig = nullptr;
+    const void *Wl = nullptr;
+    int wbf16 = 0;
+    int64_t ldw = 0;
+    const float *Hr = nullptr;
 
     ~Ctx() {
         if (own && ws) cudaFreeAsync(ws, s);
@@ -440,12 +447,24 @@ static qe_status residual(Ctx &c, const float *scales, const float *zeros, const
 // relax heuristic of Sec. 3.2 (the sweep keeps beta~ unquantized).  When the
 // changes are real-valued (src != SRC_CODES or relax) they take three bf16
 // planes and the in-block sequential kernel.
+// Near-tie refinement fields of a CD launch.
+static void set_tie(const Ctx &c, CdArgs &a, bool on) {
+    a.tie_eps = on ? c.tie_eps : 0.0f;
+    a.S = c.Sig;
+    a.lds_full = c.pl.p;
+    a.W = c.Wl;
+    a.w_bf16 = c.wbf16;
+    a.ldw = c.ldw;
+    a.Hd = c.Hr;
+    a.ldh = c.pl.ld;
+}
+
 enum { SRC_W = 0, SRC_CODES = 1, SRC_V = 2 };
 
 static float *relaxed_values(const Ctx &c) { return reinterpret_cast<float *>(c.lent); }
 
 static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float *zeros, int bits,
-                       int src, bool relax, int window, const int *gate = nullptr) {
+                       int src, bool relax, int window, const int *gate = nullptr, bool wait_test = false) {
     const int64_t q = c.pl.q, p = c.pl.p, ld = c.pl.ld;
     const int B = c.pl.B;
     const bool frac = src != SRC_CODES || relax;
@@ -511,6 +530,14 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
         a.dp_plane_rows = q;
         a.err = c.err;
         a.gate = gate;
+        // relaxed sweeps and the sweep after one start from real values: no refinement
+        set_tie(c, a, !relax && src != SRC_V);
+        if (wait_test) {   // the failure-path test hook: the first block waits for a copy never issued
+            a.skip_copy = 1;
+            a.wait_ns = 5000000ull;
+            QE_CK(launch_cd_block(B, a, c.nsm, c.s));
+            return QE_OK;
+        }
         Timed tm(c.timer, QE_KERNEL_CD_BLOCK, c.s);
         QE_CK(launch_cd_block(B, a, c.nsm, c.s));
     }
@@ -543,6 +570,7 @@ static CdArgs list_args(const Ctx &c, uint8_t *codes, const float *scales, const
     a.lcnt = c.lcnt;
     a.lent = c.lent;
     a.err = c.err;
+    set_tie(c, a, true);
     return a;
 }
 
@@ -578,6 +606,12 @@ static int dense_sweeps(const qe_opts *o) {
 }
 
 static int relax_period(const qe_opts *o) { return o ? o->relax_period : 0; }
+
+constexpr float kDefaultTieEps = 2e-5f;
+static float tie_eps(const qe_opts *o) {
+    if (!o || o->tie_eps == 0.0f) return kDefaultTieEps;
+    return o->tie_eps > 0.0f ? o->tie_eps : 0.0f;
+}
 
 // Whether the fp32 Sigma_bar rows that the list sweeps gather (4 p ld bytes) fit
 // in three quarters of this GPU's L2.
@@ -622,6 +656,8 @@ static qe_status check_opts(const qe_opts *o, bool structured = false) {
         o->switch_below < 0)
         return QE_ERR_INVALID_ARG;
     if (o->workspace && o->workspace_bytes == 0) return QE_ERR_INVALID_ARG;
+    if (o->wait_test < 0 || o->wait_test > 1) return QE_ERR_INVALID_ARG;
+    if (!(o->tie_eps == o->tie_eps) || o->tie_eps > 0.25f) return QE_ERR_INVALID_ARG;   // NaN or too wide
     if (o->group_size > 0) {
         // groups hold whole column blocks; no relax heuristic, no outlier variant with groups
         if (o->group_size % block_width(o) != 0) return QE_ERR_INVALID_ARG;
@@ -828,6 +864,11 @@ qe_status qe_quantize_layer(const void *W, qe_dtype w_dtype, int64_t q, int64_t 
     c.nsm = sm_count();
     const Plan pl = make_plan(q, p, block_width(opts), false, wbf16 ? 1 : 3, c.nsm, group_size(opts));
     if ((st = setup_ctx(c, pl, opts, reinterpret_cast<cudaStream_t>(stream))) != QE_OK) return st;
+    c.tie_eps = tie_eps(opts);
+    c.Sig = Sigma;
+    c.Wl = W;
+    c.wbf16 = wbf16;
+    c.ldw = ldw;
 
     QE_CK(launch_grid(W, wbf16, ldw, nullptr, 0, q, p, pl.gsize, bits, scales, zeros, c.err, c.s));
     if ((st = prepare(c, W, wbf16, ldw, Sigma, c.P)) != QE_OK) return st;
@@ -877,6 +918,7 @@ qe_status qe_quantize_layer(const void *W, qe_dtype w_dtype, int64_t q, int64_t 
         QE_CK(launch_init_residual(W, wbf16, ldw, nullptr, 0, q, p, pl.gsize, scales, zeros, c.R, pl.ld, c.s));
         QE_CK(cudaMemsetAsync(c.objbase, 0, 8, c.s));   // f(W) = 0
         src = SRC_W;
+        if (opts && opts->wait_test) return sweep(c, codes, scales, zeros, bits, SRC_W, false, 0, nullptr, true);
         if (!relaxed(0)) {
             if ((st = sweep(c, codes, scales, zeros, bits, SRC_W, false, 0)) != QE_OK) return st;
             const ObjFuse f{obj, W, wbf16, ldw, codes, nullptr};
@@ -1006,6 +1048,12 @@ qe_status qe_quantize_layer_outlier(const void *W, qe_dtype w_dtype, int64_t q, 
     const Plan pl = make_plan(q, p, block_width(opts), true, wbf16 ? 1 : 3, c.nsm);
     if ((st = setup_ctx(c, pl, opts, reinterpret_cast<cudaStream_t>(stream))) != QE_OK) return st;
     const int64_t ld = pl.ld;
+    c.tie_eps = tie_eps(opts);
+    c.Sig = Sigma;
+    c.Wl = W;
+    c.wbf16 = wbf16;
+    c.ldw = ldw;
+    c.Hr = c.H;   // the target of every sweep is W - H (dense H, leading dimension ld)
 
     // P_s: the s largest |T|, or with structured outliers the floor(s/q) columns of
     // largest l2 norm (Sec. 4.3, "Structured Outliers")

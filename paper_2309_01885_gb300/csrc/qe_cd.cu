@@ -417,7 +417,7 @@ __device__ __forceinline__ bool cd_prologue(const CdArgs &a, float *tri, uint64_
         fence_mbar_init();
     }
     __syncthreads();
-    if (threadIdx.x == 0) {
+    if (threadIdx.x == 0 && !a.skip_copy) {
         constexpr uint32_t bytes = C::PACK * 4;
         mbar_arrive_expect_tx(bar, bytes);
         bulk_load(tri, a.tri + (b0 / B) * C::PACK, bytes, bar);
@@ -462,8 +462,12 @@ __device__ __forceinline__ bool cd_prologue(const CdArgs &a, float *tri, uint64_
             if (row_ok && (FULL || l < bw)) a.R[ii * a.ldr + b0 + l] = t[h];
         }
     }
-    if (!mbar_wait_bounded(bar, 0u, nullptr)) {
+    const unsigned long long lim = a.wait_ns ? a.wait_ns : kWaitLimitNs;
+    if (!mbar_wait_bounded_ns(bar, 0u, nullptr, lim)) {
         if (lane == 0) set_error(a.err, ERR_TIMEOUT);
+        // a copy that was issued may still land: thread 0 keeps the CTA (and its
+        // shared memory) alive until it has, within one more limit
+        if (threadIdx.x == 0 && !a.skip_copy) mbar_wait_bounded_ns(bar, 0u, nullptr, lim);
         return false;
     }
     return true;
@@ -544,6 +548,147 @@ __device__ __forceinline__ double warp_sum(double x) {
     return x;
 }
 
+// ---- near-tie refinement ------------------------------------------------------
+// A decision rounds beta~ / s + z (binary32, grid units) to the nearest level; it
+// can only come out differently from exact arithmetic when that value lies within
+// the binary32 error of a midpoint between two levels.  Such decisions (within
+// a.tie_eps, far above that error) are taken again from beta~ recomputed from
+// the row's current state, Lemma 1:
+//   beta~_j = T_j + sum_{k != j} (T_k - What_k) Sigma_kj / Sigma_jj,  T = W (- H),
+// with What_k = s (c_k - z) of the code column k holds at that moment (this
+// sweep's for k < j, the previous sweep's for k > j; in the first sweep the
+// columns after j still hold T).  One warp-wide pass over the row: every term
+// exact, the sum in double-float arithmetic (about 48 significant bits), the
+// last steps in binary64, so the decision is that of exact arithmetic except
+// within about 1e-9 grid steps of a midpoint.
+
+__device__ __forceinline__ float tie_w(const CdArgs &a, int64_t i, int64_t k) {
+    return a.w_bf16 ? __bfloat162float(static_cast<const __nv_bfloat16 *>(a.W)[i * a.ldw + k])
+                    : static_cast<const float *>(a.W)[i * a.ldw + k];
+}
+
+// beta~ / s + z of column b0 + j of row i, from the row's current
+// state.  blk: the warp's shared row with the block's current codes (decided in
+// this visit before j, start codes after j; unused after j in the first sweep).
+// Warp-collective (every lane calls it; the result is the same in every lane).
+// The columns outside the block are read from global memory in 16-byte pieces,
+// several pieces per lane in flight, so a pass over a long row takes few round
+// trips.  Compiled only into the kernels' refinement variants.
+// Error-free transformations (Knuth's two-sum; the fma two-product), for the
+// refinement's sums in double-float arithmetic: about 48 significant bits on the
+// fp32 pipes (GB300's binary64 rate is a small fraction of its binary32 rate).
+__device__ __forceinline__ void ef_two_sum(float a, float b, float &s, float &e) {
+    s = __fadd_rn(a, b);
+    const float bb = __fsub_rn(s, a);
+    e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+}
+
+// (hi, lo) += (t - hs - sg (c - zg)) * sjk in double-float; t, hs, sg, zg, sjk are
+// binary32 values and c - zg an exact small integer, so every operand is exact.
+__device__ __forceinline__ void df_term(float &hi, float &lo, float t, float hs, float sg, float m, float sjk) {
+    const float w1 = __fmul_rn(sg, m);
+    const float w2 = fmaf(sg, m, -w1);            // sg m = w1 + w2 exactly
+    float u1, u2, d1, e1;
+    ef_two_sum(t, -hs, u1, u2);                   // t - hs = u1 + u2 exactly
+    ef_two_sum(u1, -w1, d1, e1);
+    const float d2 = __fadd_rn(e1, __fsub_rn(u2, w2));
+    const float p1 = __fmul_rn(d1, sjk);
+    const float p2 = fmaf(d2, sjk, fmaf(d1, sjk, -p1));
+    float s1, s2;
+    ef_two_sum(hi, p1, s1, s2);
+    s2 = __fadd_rn(s2, __fadd_rn(lo, p2));
+    hi = __fadd_rn(s1, s2);
+    lo = __fsub_rn(s2, __fsub_rn(hi, s1));
+}
+
+__device__ __forceinline__ double tie_beta(const CdArgs *ap, int64_t i, int64_t b0, int bw, int j, int lane,
+                                        const float *blk) {
+    const CdArgs &a = *ap;
+    const int64_t jg = b0 + j;
+    const float *Srow = a.S + jg * a.lds_full;
+    const int64_t kend = a.first_sweep ? b0 : a.p;   // first sweep: later columns still hold T
+    const float *sc = a.scale + i * a.ngroups;
+    const float *zc = a.zero + i * a.ngroups;
+    const bool grouped = a.ngroups > 1;
+    const uint32_t gs = static_cast<uint32_t>(a.gsize);
+    const uint8_t *crow = a.codes + i * a.ldc;
+    const float *hrow = a.Hd ? a.Hd + i * a.ldh : nullptr;
+    // Pull the row's data toward L2 first, every line at once (prefetches hold no
+    // register), so the summing loop below waits on L2 rather than on DRAM.
+    for (int64_t k = 32 * lane; k < kend; k += 32 * 32) prefetch_l2(Srow + k);
+    for (int64_t k = 128 * lane; k < kend; k += 128 * 32) prefetch_l2(crow + k);
+    if (a.w_bf16) {
+        for (int64_t k = 64 * lane; k < kend; k += 64 * 32)
+            prefetch_l2(static_cast<const __nv_bfloat16 *>(a.W) + i * a.ldw + k);
+    } else {
+        for (int64_t k = 32 * lane; k < kend; k += 32 * 32) prefetch_l2(static_cast<const float *>(a.W) + i * a.ldw + k);
+    }
+    if (hrow)
+        for (int64_t k = 32 * lane; k < kend; k += 32 * 32) prefetch_l2(hrow + k);
+    float hi = 0.0f, lo = 0.0f;   // the lane's sum, double-float
+    // the block's own columns from the shared row
+    for (int l = lane; l < bw; l += 32) {
+        if (l == j || (a.first_sweep && l > j)) continue;
+        const int64_t k = b0 + l;
+        const uint32_t g = grouped ? static_cast<uint32_t>(k) / gs : 0u;
+        df_term(hi, lo, tie_w(a, i, k), hrow ? hrow[k] : 0.0f, sc[g], blk[l] - zc[g], Srow[k]);
+    }
+    // the columns outside the block from the row's codes in global memory
+    const bool vec = (a.lds_full % 4) == 0 && (a.ldc % 4) == 0 && (a.ldw % 4) == 0 && (!hrow || (a.ldh % 4) == 0) &&
+                     ((reinterpret_cast<uintptr_t>(a.S) & 15u) == 0) &&
+                     ((reinterpret_cast<uintptr_t>(a.codes) & 3u) == 0) &&
+                     ((reinterpret_cast<uintptr_t>(a.W) & (a.w_bf16 ? 7u : 15u)) == 0) &&
+                     (!hrow || (reinterpret_cast<uintptr_t>(a.Hd) & 15u) == 0) && (b0 % 4) == 0;
+    if (vec) {
+#pragma unroll 2
+        for (int64_t k = 4 * lane; k < kend; k += 128) {
+            if (k >= b0 && k < b0 + bw) continue;   // 4-aligned pieces never straddle the block
+            const float4 s4 = *reinterpret_cast<const float4 *>(Srow + k);
+            const uint32_t c4 = *reinterpret_cast<const uint32_t *>(crow + k);
+            float wv[4];
+            if (a.w_bf16) {
+                const uint2 r = *reinterpret_cast<const uint2 *>(static_cast<const __nv_bfloat16 *>(a.W) + i * a.ldw + k);
+                const __nv_bfloat162 w01 = *reinterpret_cast<const __nv_bfloat162 *>(&r.x);
+                const __nv_bfloat162 w23 = *reinterpret_cast<const __nv_bfloat162 *>(&r.y);
+                wv[0] = __low2float(w01); wv[1] = __high2float(w01);
+                wv[2] = __low2float(w23); wv[3] = __high2float(w23);
+            } else {
+                const float4 w4 = *reinterpret_cast<const float4 *>(static_cast<const float *>(a.W) + i * a.ldw + k);
+                wv[0] = w4.x; wv[1] = w4.y; wv[2] = w4.z; wv[3] = w4.w;
+            }
+            float hv[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+            if (hrow) {
+                const float4 h4 = *reinterpret_cast<const float4 *>(hrow + k);
+                hv[0] = h4.x; hv[1] = h4.y; hv[2] = h4.z; hv[3] = h4.w;
+            }
+            const float sv[4] = {s4.x, s4.y, s4.z, s4.w};
+            const uint32_t g = grouped ? static_cast<uint32_t>(k) / gs : 0u;   // 4 columns share a group
+            const float sg = sc[g], zg = zc[g];
+#pragma unroll
+            for (int e = 0; e < 4; ++e)
+                df_term(hi, lo, wv[e], hv[e], sg, static_cast<float>((c4 >> (8 * e)) & 0xffu) - zg, sv[e]);
+        }
+    } else {
+        for (int64_t k = lane; k < kend; k += 32) {
+            if (k >= b0 && k < b0 + bw) continue;
+            const uint32_t g = grouped ? static_cast<uint32_t>(k) / gs : 0u;
+            df_term(hi, lo, tie_w(a, i, k), hrow ? hrow[k] : 0.0f, sc[g], static_cast<float>(crow[k]) - zc[g], Srow[k]);
+        }
+    }
+    const double acc = warp_sum(static_cast<double>(hi) + static_cast<double>(lo));
+    double tj = static_cast<double>(tie_w(a, i, jg));
+    if (hrow) tj -= static_cast<double>(hrow[jg]);
+    const double dj = static_cast<double>(Srow[jg]);
+    const uint32_t g = grouped ? static_cast<uint32_t>(jg) / gs : 0u;
+    const double beta = dj > 0.0 ? tj + acc / dj : tj;
+    return beta / static_cast<double>(sc[g]) + static_cast<double>(zc[g]);
+}
+
+// The level of t in binary64 (round half to even, clamped to 0 .. maxq).
+__device__ __forceinline__ float tie_code(double t, float maxq) {
+    return static_cast<float>(rint(fmin(fmax(t, 0.0), static_cast<double>(maxq))));
+}
+
 // Sequential in-block kernel (sweeps where every column moves by a real
 // amount: the first sweep, a relaxed sweep and the sweep after one).
 // One warp per row; column j = 32 h + jj is decided by lane jj, which keeps
@@ -558,8 +703,8 @@ __device__ __forceinline__ double warp_sum(double x) {
 // beta~ of its column (in grid units) to the warp's row of shared memory, and
 // the changes are formed after the sweep over the block, so the sequential
 // chain waits on no load.
-template <int B, bool FULL, bool RELAX, bool DF>
-__global__ void __launch_bounds__(1024) k_cd_block_seq(const CdArgs a) {
+template <int B, bool FULL, bool RELAX, bool DF, bool TIE = false>
+__global__ void __launch_bounds__(1024) k_cd_block_seq(const __grid_constant__ CdArgs a) {
     using C = CdCfg<B>;
     constexpr int CPL = C::CPL;
     extern __shared__ __align__(16) float cd_smem[];
@@ -567,6 +712,10 @@ __global__ void __launch_bounds__(1024) k_cd_block_seq(const CdArgs a) {
     uint64_t *bar = reinterpret_cast<uint64_t *>(cd_smem + C::PACK);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     float *tdec = cd_smem + C::PACK + 4 + warp * B;   // DF: beta~ at each decision (after the barrier)
+    // the codes decided in this visit and a snapshot of the lanes' values, for the
+    // near-tie refinement (after the DF rows)
+    float *cdec = cd_smem + C::PACK + 4 + (DF ? (blockDim.x >> 5) * B : 0) + 2 * warp * B;
+    float *snap = cdec + B;
     const int64_t i = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + warp;
     const bool row_ok = i < a.q;
     float t[CPL], st[CPL];
@@ -580,6 +729,8 @@ __global__ void __launch_bounds__(1024) k_cd_block_seq(const CdArgs a) {
         for (int h = 0; h < CPL; ++h)
             if ((FULL || 32 * h + lane < bw) && a.d[a.b0 + 32 * h + lane] > 0.0f) live |= 1u << h;
     }
+    // near-tie refinement: only in the first sweep (RELAX and a real-valued start turn it off)
+    const bool tie = TIE && !RELAX && a.tie_eps > 0.0f && a.first_sweep && !a.vstart;
     float code[CPL], dlt[CPL];
 #pragma unroll
     for (int h = 0; h < CPL; ++h) {
@@ -588,24 +739,82 @@ __global__ void __launch_bounds__(1024) k_cd_block_seq(const CdArgs a) {
     }
 #pragma unroll
     for (int h = 0; h < CPL; ++h) {
+        // The word's 32 columns in order.  The deciding lane notes whether its value
+        // sat within tie_eps of a midpoint (off the sequential chain); after the word,
+        // the first such column is decided again from the binary64 beta~: the lanes
+        // restore the values of the snapshot taken before the pass, replay the
+        // decisions before that column (the same arithmetic, so the same results),
+        // decide it exactly and resume after it.
+        int start = 0;
+        while (true) {
+            if (tie) {
 #pragma unroll
-        for (int jj = 0; jj < 32; ++jj) {
-            const int j = 32 * h + jj;
-            if (!FULL && j >= bw) break;
-            const float cq = rintf(fminf(fmaxf(t[h], 0.0f), maxq));
-            const float c = (RELAX && ((live >> h) & 1u)) ? t[h] : cq;
-            const float dl = st[h] - c;
-            if (lane == jj) {
+                for (int g = h; g < CPL; ++g) snap[32 * g + lane] = t[g];
+            }
+            bool mynear = false;
+#pragma unroll
+            for (int jj = 0; jj < 32; ++jj) {
+                if (jj < start) continue;
+                const int j = 32 * h + jj;
+                if (!FULL && j >= bw) break;
+                const float cq = rintf(fminf(fmaxf(t[h], 0.0f), maxq));
+                const float c = (RELAX && ((live >> h) & 1u)) ? t[h] : cq;
+                const float dl = st[h] - c;
+                if (lane == jj) {
+                    code[h] = c;
+                    dlt[h] = dl;
+                    if (DF) tdec[j] = t[h];
+                    if (tie) {
+                        cdec[j] = c;
+                        mynear = fabsf(fabsf(t[h] - cq) - 0.5f) < a.tie_eps;
+                    }
+                }
+                const float db = __shfl_sync(0xffffffffu, dl, jj);
+                if (db != 0.0f) {
+                    const float *row = tri + kPackPad + tri_off(B, j) - (j + 1);
+#pragma unroll
+                    for (int g = h; g < CPL; ++g) t[g] = fmaf(db, row[32 * g + lane], t[g]);
+                }
+            }
+            if (!tie) break;
+            const unsigned nb = __ballot_sync(0xffffffffu, mynear);
+            if (nb == 0u) break;
+            const int jt = __ffs(nb) - 1;
+            __syncwarp();
+#pragma unroll
+            for (int g = h; g < CPL; ++g) t[g] = snap[32 * g + lane];
+#pragma unroll
+            for (int jj = 0; jj < 32; ++jj) {   // replay the columns before jt
+                if (jj < start) continue;
+                if (jj >= jt) break;
+                const int j = 32 * h + jj;
+                const float c = rintf(fminf(fmaxf(t[h], 0.0f), maxq));
+                const float dl = st[h] - c;
+                const float db = __shfl_sync(0xffffffffu, dl, jj);
+                if (db != 0.0f) {
+                    const float *row = tri + kPackPad + tri_off(B, j) - (j + 1);
+#pragma unroll
+                    for (int g = h; g < CPL; ++g) t[g] = fmaf(db, row[32 * g + lane], t[g]);
+                }
+            }
+            // column 32 h + jt from the binary64 beta~ of the row's state
+            const int j = 32 * h + jt;
+            const double te = tie_beta(&a, i, a.b0, bw, j, lane, cdec);
+            const float c = tie_code(te, maxq);
+            const float dl = __shfl_sync(0xffffffffu, st[h], jt) - c;
+            if (lane == jt) {
                 code[h] = c;
                 dlt[h] = dl;
-                if (DF) tdec[j] = t[h];
+                if (DF) tdec[j] = static_cast<float>(te);
+                cdec[j] = c;
             }
-            const float db = __shfl_sync(0xffffffffu, dl, jj);
-            if (db != 0.0f) {
+            if (dl != 0.0f) {
                 const float *row = tri + kPackPad + tri_off(B, j) - (j + 1);
 #pragma unroll
-                for (int g = h; g < CPL; ++g) t[g] = fmaf(db, row[32 * g + lane], t[g]);
+                for (int g = h; g < CPL; ++g) t[g] = fmaf(dl, row[32 * g + lane], t[g]);
             }
+            start = jt + 1;
+            if (start >= 32 || (!FULL && 32 * h + start >= bw)) break;
         }
     }
     if (DF) {
@@ -646,22 +855,32 @@ __global__ void __launch_bounds__(1024) k_cd_block_seq(const CdArgs a) {
 //   GROWS = false: the coupling rows come from the packed triangle in shared
 //   memory; GROWS = true: from the fp32 Sigma_bar rows in global memory
 //   (`grow` = &Sigma_bar[b0][b0], leading dimension lds; the same values).
-template <int B, bool FULL, bool GROWS = false>
+// With `ax` (near-tie refinement on, ax->tie_eps > 0; row i, block start b0;
+// tie_blk: B floats of the warp's shared memory), a
+// column whose beta~ lies within tie_eps of a midpoint also stops the pass: its
+// decision is taken from the binary64 beta~ of the row's state at that point
+// (columns before it final, after it at their start codes), and the pass goes on
+// from it as from any other column.
+template <int B, bool FULL, bool GROWS = false, bool TIE = false>
 __device__ __forceinline__ int chg_decide(const float *tri, const float *d_blk, int bw_, float maxq, float s2,
                                           bool want_df, int lane, float (&t)[B / 32], const float (&st)[B / 32],
                                           float (&code)[B / 32], float (&dlt)[B / 32], double &dfacc,
-                                          const float *grow = nullptr, int64_t lds = 0) {
+                                          const float *grow = nullptr, int64_t lds = 0,
+                                          const CdArgs *ax = nullptr, int64_t i = 0, int64_t b0 = 0,
+                                          float *tie_blk = nullptr) {
     constexpr int CPL = B / 32;
     const int bw = FULL ? B : bw_;
+    const bool tie = TIE && ax != nullptr && tie_blk != nullptr && ax->tie_eps > 0.0f;
+    const float eps = tie ? ax->tie_eps : 0.0f;
 #pragma unroll
-    for (int h = 0; h < CPL; ++h) {
-        code[h] = st[h];
-        dlt[h] = 0.0f;
-    }
+    for (int h = 0; h < CPL; ++h) code[h] = st[h];
+    // dlt (= st - code, exact for these small integers) is formed once at the end, so
+    // it holds no registers during the passes
     int pos = 0;                                       // first column not yet final
     int nchg = 0;
     while (pos < bw) {
         int jstar = -1;
+        bool jtie = false;
         // values of this lane's column in the word that holds the first change
         // (captured with a compile-time h, so the arrays stay in registers)
         float v = 0.0f, tv = 0.0f, cv = 0.0f, sv = 0.0f;
@@ -671,13 +890,14 @@ __device__ __forceinline__ int chg_decide(const float *tri, const float *d_blk, 
             const bool active = l >= pos && (FULL || l < bw);
             const float c = rintf(fminf(fmaxf(t[h], 0.0f), maxq));
             const float dl = st[h] - c;
-            if (active) {
-                code[h] = c;
-                dlt[h] = dl;
-            }
-            const unsigned m = __ballot_sync(0xffffffffu, active && dl != 0.0f);
+            if (active) code[h] = c;
+            // within eps of a midpoint: |t - nearest level| within eps of 1/2 (a clamped
+            // t just beyond the end levels also passes; deciding it exactly is harmless)
+            const bool nt = tie && active && fabsf(fabsf(t[h] - c) - 0.5f) < eps;
+            const unsigned m = __ballot_sync(0xffffffffu, active && (dl != 0.0f || nt));
             if (jstar < 0 && m != 0u) {
                 jstar = 32 * h + (__ffs(m) - 1);
+                if (TIE) jtie = tie && ((__ballot_sync(0xffffffffu, nt) >> (jstar & 31)) & 1u);
                 v = dl;
                 tv = t[h];
                 cv = c;
@@ -685,6 +905,30 @@ __device__ __forceinline__ int chg_decide(const float *tri, const float *d_blk, 
             }
         }
         if (jstar < 0) break;
+        if (TIE && jtie) {
+            // binary64 beta~ of column jstar: the block's columns from this warp's shared
+            // row (final before jstar, start after), the rest from global memory
+#pragma unroll
+            for (int h = 0; h < CPL; ++h)
+                if (FULL || 32 * h + lane < bw) tie_blk[32 * h + lane] = (32 * h + lane < jstar) ? code[h] : st[h];
+            __syncwarp();
+            const double te = tie_beta(ax, i, b0, bw, jstar, lane, tie_blk);
+            __syncwarp();
+            const float ce = tie_code(te, maxq);
+            const float se = __shfl_sync(0xffffffffu, sv, jstar & 31);
+            const float de = se - ce;
+#pragma unroll
+            for (int h = 0; h < CPL; ++h)
+                if (32 * h + lane == jstar) code[h] = ce;
+            if (de == 0.0f) {   // no change: the columns after it keep their provisional decisions
+                pos = jstar + 1;
+                continue;
+            }
+            v = de;
+            tv = static_cast<float>(te);
+            cv = ce;
+            sv = se;
+        }
         if (want_df && lane == (jstar & 31)) {
             const float dj = d_blk[jstar];
             if (dj > 0.0f) {
@@ -708,15 +952,182 @@ __device__ __forceinline__ int chg_decide(const float *tri, const float *d_blk, 
         pos = jstar + 1;
         ++nchg;
     }
+#pragma unroll
+    for (int h = 0; h < CPL; ++h) dlt[h] = st[h] - code[h];
     return nchg;
+}
+
+// ---- refinement of the per-block change-driven kernel, CTA-wide -----------------
+// The rows of a CTA first decide in binary32 as usual, noting every final
+// decision whose t lies within tie_eps of a midpoint; then the whole CTA checks
+// those decisions one at a time, each against beta~ recomputed from the row's
+// state at that decision (one pass over the row by every thread of the CTA,
+// double-float sums); a row whose decision was wrong decides again from the
+// block's start with that column forced to its exact code, noting only the
+// near-ties after it, and the check repeats.  A row checks its first kMaxEv notes
+// of a visit and forces at most kMaxForced decisions (at tie_eps = 2e-5 a
+// 256-column visit has one note in about forty).
+constexpr int kMaxEv = 8;      // near-tie notes per row and block visit
+constexpr int kMaxForced = 4;  // exact decisions forced per row and block visit
+
+// chg_decide's binary32 passes with notes: columns fj[0 .. nf) take the codes
+// fc[..]; every decision after column rec_from whose t lay within eps of a
+// midpoint goes to ev (ascending), *nev counting past kMaxEv on overflow.  A
+// change here updates only the columns after it, so every column keeps the t it
+// was decided on, and the notes are taken once at the end.
+template <int B, bool FULL>
+__device__ __forceinline__ void chg_decide_rec(const float *tri, const float *d_blk, int bw_, float maxq, float s2,
+                                               bool want_df, int lane, float (&t)[B / 32], const float (&st)[B / 32],
+                                               float (&code)[B / 32], float (&dlt)[B / 32], double &dfacc, float eps,
+                                               const int *fj, const float *fc, int nf, int rec_from, int *ev,
+                                               int *nev) {
+    constexpr int CPL = B / 32;
+    const int bw = FULL ? B : bw_;
+#pragma unroll
+    for (int h = 0; h < CPL; ++h) code[h] = st[h];
+    int pos = 0;
+    while (pos < bw) {
+        int jstar = -1;
+        float v = 0.0f, tv = 0.0f, cv = 0.0f, sv = 0.0f;
+#pragma unroll
+        for (int h = 0; h < CPL; ++h) {
+            const int l = 32 * h + lane;
+            const bool active = l >= pos && (FULL || l < bw);
+            float c = rintf(fminf(fmaxf(t[h], 0.0f), maxq));
+            if (nf > 0)
+                for (int f = 0; f < nf; ++f)
+                    if (fj[f] == l) c = fc[f];
+            const float dl = st[h] - c;
+            if (active) code[h] = c;
+            const unsigned m = __ballot_sync(0xffffffffu, active && dl != 0.0f);
+            if (jstar < 0 && m != 0u) {
+                jstar = 32 * h + (__ffs(m) - 1);
+                v = dl;
+                tv = t[h];
+                cv = c;
+                sv = st[h];
+            }
+        }
+        if (jstar < 0) break;
+        if (want_df && lane == (jstar & 31)) {
+            const float dj = d_blk[jstar];
+            if (dj > 0.0f) {
+                const float e1 = cv - tv, e0 = sv - tv;
+                dfacc += static_cast<double>(dj * s2 * (e1 * e1 - e0 * e0));
+            }
+        }
+        const float db = __shfl_sync(0xffffffffu, v, jstar & 31);
+        const float *row = tri + kPackPad + tri_off(B, jstar) - (jstar + 1);
+#pragma unroll
+        for (int g = 0; g < CPL; ++g)
+            if (32 * g + lane > jstar) t[g] = fmaf(db, row[32 * g + lane], t[g]);
+        pos = jstar + 1;
+    }
+    // the notes: every column's t is the one it was decided on
+#pragma unroll
+    for (int h = 0; h < CPL; ++h) {
+        const int l = 32 * h + lane;
+        bool nt = (FULL || l < bw) && l > rec_from && fabsf(fabsf(t[h] - rintf(fminf(fmaxf(t[h], 0.0f), maxq))) - 0.5f) < eps;
+        for (int f = 0; f < nf; ++f)
+            if (fj[f] == l) nt = false;
+        unsigned mn = __ballot_sync(0xffffffffu, nt);
+        if (mn != 0u && lane == 0) {
+            int n = *nev;
+            while (mn != 0u) {
+                const int b = __ffs(mn) - 1;
+                mn &= mn - 1u;
+                if (n < kMaxEv) ev[n] = 32 * h + b;
+                ++n;
+            }
+            *nev = n;
+        }
+    }
+    __syncwarp();
+#pragma unroll
+    for (int h = 0; h < CPL; ++h) dlt[h] = st[h] - code[h];
+}
+
+// CTA-wide: beta~ / s + z of column b0 + j of row i at its decision: the block's
+// columns before j from cr (final codes), after j from sr (start codes), the rest
+// from the codes in global memory.  Every thread of the CTA calls it; red holds
+// 34 doubles of shared memory.  Returns the same value in every thread.
+__device__ __forceinline__ double coop_tie_beta(const CdArgs &a, int64_t i, int64_t b0, int bw, int j,
+                                                const float *cr, const float *sr, double *red) {
+    const int tid = threadIdx.x, nth = blockDim.x;
+    const int64_t jg = b0 + j;
+    const float *Srow = a.S + jg * a.lds_full;
+    const float *sc = a.scale + i * a.ngroups;
+    const float *zc = a.zero + i * a.ngroups;
+    const bool grouped = a.ngroups > 1;
+    const uint32_t gs = static_cast<uint32_t>(a.gsize);
+    const uint8_t *crow = a.codes + i * a.ldc;
+    const float *hrow = a.Hd ? a.Hd + i * a.ldh : nullptr;
+    float hi = 0.0f, lo = 0.0f;
+    // U columns per thread in flight: all their loads are issued before the sums
+    constexpr int U = 8;
+    for (int64_t k0 = tid; k0 < a.p; k0 += static_cast<int64_t>(nth) * U) {
+        float cv[U], wv[U], hv[U], sv[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int64_t k = k0 + static_cast<int64_t>(u) * nth;
+            cv[u] = wv[u] = hv[u] = sv[u] = 0.0f;
+            if (k < a.p) {
+                if (k >= b0 && k < b0 + bw) {
+                    const int l = static_cast<int>(k - b0);
+                    cv[u] = l < j ? cr[l] : sr[l];
+                } else {
+                    cv[u] = static_cast<float>(crow[k]);
+                }
+                wv[u] = tie_w(a, i, k);
+                if (hrow) hv[u] = hrow[k];
+                sv[u] = (k == jg) ? 0.0f : Srow[k];   // column j itself is left out
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int64_t k = k0 + static_cast<int64_t>(u) * nth;
+            if (k >= a.p) continue;
+            const uint32_t g = grouped ? static_cast<uint32_t>(k) / gs : 0u;
+            df_term(hi, lo, wv[u], hv[u], sc[g], cv[u] - zc[g], sv[u]);
+        }
+    }
+    double acc = warp_sum(static_cast<double>(hi) + static_cast<double>(lo));
+    if ((tid & 31) == 0) red[tid >> 5] = acc;
+    __syncthreads();
+    if (tid == 0) {
+        double sum = 0.0;
+        for (int w = 0; w < (nth >> 5); ++w) sum += red[w];
+        double tj = static_cast<double>(tie_w(a, i, jg));
+        if (hrow) tj -= static_cast<double>(hrow[jg]);
+        const double dj = static_cast<double>(Srow[jg]);
+        const uint32_t g = grouped ? static_cast<uint32_t>(jg) / gs : 0u;
+        const double beta = dj > 0.0 ? tj + sum / dj : tj;
+        red[32] = beta / static_cast<double>(sc[g]) + static_cast<double>(zc[g]);
+    }
+    __syncthreads();
+    return red[32];
+}
+
+// Shared memory of the refinement variant after the packed block, per warp.
+struct TieWarp {
+    int ev[kMaxEv];
+    int fj[kMaxForced];
+    float fc[kMaxForced];
+    int nev, nf, wrong_j;
+    float wrong_c;
+};
+
+template <int B>
+__host__ __device__ constexpr int tie_cta_bytes(int warps) {
+    return warps * (2 * B * 4 + static_cast<int>(sizeof(TieWarp))) + 34 * 8;
 }
 
 // Change-driven in-block kernel (every sweep after the first), exactly
 // equivalent to the sequential order: a column whose code does not change
 // alters no other column, so the cost is (number of changed columns + 1)
 // data-parallel passes (chg_decide).
-template <int B, bool FULL>
-__global__ void __launch_bounds__(1024, 1) k_cd_block_chg(const CdArgs a) {
+template <int B, bool FULL, bool TIE = false>
+__global__ void __launch_bounds__(1024, 1) k_cd_block_chg(const __grid_constant__ CdArgs a) {
     if (a.gate && *a.gate != a.gate_run) return;   // uniform: the list form of the sweep runs
     using C = CdCfg<B>;
     constexpr int CPL = C::CPL;
@@ -727,12 +1138,101 @@ __global__ void __launch_bounds__(1024, 1) k_cd_block_chg(const CdArgs a) {
     const int64_t i = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + warp;
     const bool row_ok = i < a.q;
     float t[CPL], st[CPL];
-    if (!cd_prologue<B, FULL>(a, tri, bar, i, row_ok, lane, t, st)) return;
-    if (!row_ok) return;
     float code[CPL], dlt[CPL];
-    const float s = a.scale[i * a.ngroups + a.b0 / a.gsize];
     double dfacc = 0.0;
-    chg_decide<B, FULL>(tri, a.d + a.b0, a.bw, a.maxq, s * s, a.rowdf != nullptr, lane, t, st, code, dlt, dfacc);
+    if constexpr (TIE) {
+        // refinement variant: binary32 decisions with notes, checked CTA-wide
+        const int nw = static_cast<int>(blockDim.x >> 5);
+        float *cr = cd_smem + C::PACK + 4;                  // [nw][B] final codes
+        float *sr = cr + nw * B;                            // [nw][B] start codes
+        TieWarp *tw = reinterpret_cast<TieWarp *>(sr + nw * B);
+        double *red = reinterpret_cast<double *>(tw + nw);
+        const bool ok = cd_prologue<B, FULL>(a, tri, bar, i, row_ok, lane, t, st);
+        if (__syncthreads_or(!ok)) return;   // a wait gave up somewhere: every warp leaves
+        const int bw = FULL ? B : a.bw;
+        const float s = row_ok ? a.scale[i * a.ngroups + a.b0 / a.gsize] : 1.0f;
+        TieWarp &me = tw[warp];
+        if (lane == 0) {
+            me.nev = 0;
+            me.nf = 0;
+            me.wrong_j = -1;
+        }
+        __syncwarp();
+        if (row_ok)
+            chg_decide_rec<B, FULL>(tri, a.d + a.b0, a.bw, a.maxq, s * s, a.rowdf != nullptr, lane, t, st, code, dlt,
+                                    dfacc, a.tie_eps, me.fj, me.fc, 0, -1, me.ev, &me.nev);
+#pragma unroll
+        for (int h = 0; h < CPL; ++h) {
+            cr[warp * B + 32 * h + lane] = code[h];
+            sr[warp * B + 32 * h + lane] = st[h];
+        }
+        for (int round = 0; round <= kMaxForced; ++round) {
+            __syncthreads();
+            // check the notes, row by row, in order; the first wrong one stops its row's checks
+            bool any = false;
+            for (int w = 0; w < nw; ++w) {
+                const int64_t iw = static_cast<int64_t>(blockIdx.x) * nw + w;
+                if (iw >= a.q) break;
+                // (more than kMaxEv notes: the first kMaxEv, in column order, are checked)
+                const int n = tw[w].nev < kMaxEv ? tw[w].nev : kMaxEv;
+                for (int e = 0; e < n; ++e) {
+                    const int j = tw[w].ev[e];
+                    const double te = coop_tie_beta(a, iw, a.b0, bw, j, cr + w * B, sr + w * B, red);
+                    const float ce = tie_code(te, a.maxq);
+                    const bool wrong = ce != cr[w * B + j];
+                    if (wrong) {
+                        if (threadIdx.x == 0) {
+                            tw[w].wrong_j = j;
+                            tw[w].wrong_c = ce;
+                        }
+                        any = true;
+                        break;
+                    }
+                }
+            }
+            __syncthreads();
+            if (!any) break;
+            if (lane == 0 && me.wrong_j == -1) me.nev = 0;   // this row's notes all held
+            // rows with a wrong decision decide again from the block's start (R holds it)
+            if (row_ok && me.wrong_j != -1) {
+                const int wj = me.wrong_j;
+                __syncwarp();
+#pragma unroll
+                for (int h = 0; h < CPL; ++h) {
+                    const int l = 32 * h + lane;
+                    t[h] = (FULL || l < bw) ? a.R[i * a.ldr + a.b0 + l] : 0.0f;
+                }
+                dfacc = 0.0;
+                // force the exact code (a row whose kMaxForced forced decisions are used
+                // up keeps its last decisions: in practice never reached)
+                if (lane == 0) {
+                    if (me.nf < kMaxForced) {
+                        me.fj[me.nf] = wj;
+                        me.fc[me.nf] = me.wrong_c;
+                        me.nf += 1;
+                    }
+                    me.nev = 0;
+                    me.wrong_j = -1;
+                }
+                __syncwarp();
+                chg_decide_rec<B, FULL>(tri, a.d + a.b0, a.bw, a.maxq, s * s, a.rowdf != nullptr, lane, t, st, code,
+                                        dlt, dfacc, a.tie_eps, me.fj, me.fc, me.nf, wj, me.ev, &me.nev);
+                if (round == kMaxForced && lane == 0) me.nev = 0;
+                __syncwarp();
+#pragma unroll
+                for (int h = 0; h < CPL; ++h) {
+                    cr[warp * B + 32 * h + lane] = code[h];
+                    sr[warp * B + 32 * h + lane] = st[h];
+                }
+            }
+        }
+        if (!row_ok) return;
+    } else {
+        if (!cd_prologue<B, FULL>(a, tri, bar, i, row_ok, lane, t, st)) return;
+        if (!row_ok) return;
+        const float s = a.scale[i * a.ngroups + a.b0 / a.gsize];
+        chg_decide<B, FULL>(tri, a.d + a.b0, a.bw, a.maxq, s * s, a.rowdf != nullptr, lane, t, st, code, dlt, dfacc);
+    }
     if (a.rowdf) {
         dfacc = warp_sum(dfacc);
         if (lane == 0) a.rowdf[i] += dfacc;
@@ -748,10 +1248,10 @@ __global__ void __launch_bounds__(1024, 1) k_cd_block_chg(const CdArgs a) {
 // change-list correction (storing it back as the block's base when the window
 // held a change), wait for the block's packed Sigma_bar, decide, write back.
 // Returns false when the wait gave up.
-template <int B, bool FULL, bool LATE, bool GR = false>
+template <int B, bool FULL, bool LATE, bool GR = false, bool TIE = false>
 __device__ __forceinline__ bool rows_block(const CdArgs &a, int64_t b0, int bw_, const float *tri, uint64_t *bar,
                                            uint32_t parity, int64_t i, bool row_ok, int lane, float s2_row,
-                                           double &dfacc, int &nchg) {
+                                           double &dfacc, int &nchg, float *tie_blk) {
     constexpr int CPL = B / 32;
     const int bw = FULL ? B : bw_;
     const int64_t ii = row_ok ? i : 0;
@@ -798,8 +1298,8 @@ __device__ __forceinline__ bool rows_block(const CdArgs &a, int64_t b0, int bw_,
     if (!LATE && !mbar_wait_bounded(bar, parity, nullptr)) return false;
     if (!row_ok) return true;
     float code[CPL], dlt[CPL];
-    nchg += chg_decide<B, FULL, LATE>(tri, a.d + b0, bw, a.maxq, s2, true, lane, t, st, code, dlt, dfacc,
-                                      a.sbar + b0 * a.lds + b0, a.lds);
+    nchg += chg_decide<B, FULL, LATE, TIE>(tri, a.d + b0, bw, a.maxq, s2, true, lane, t, st, code, dlt, dfacc,
+                                      a.sbar + b0 * a.lds + b0, a.lds, &a, i, b0, tie_blk);
     cd_epilogue<B, FULL, true, GR>(a, b0, bw, i, lane, code, dlt, true);
     return true;
 }
@@ -864,7 +1364,7 @@ __device__ __forceinline__ int build_window(const CdArgs &a, int64_t i, int lane
 // so the same sums), then this block's entries in the window are replaced by
 // the changes just made.  The lists in global memory are written as well, so a
 // window that outgrows kWinCap (wn = -1) hands over to them.
-template <int B, bool FULL, bool GR = false>
+template <int B, bool FULL, bool GR = false, bool TIE = false>
 __device__ __forceinline__ void rows_block_win(const CdArgs &a, int64_t b0, int bw_, int64_t i, int lane,
                                                float s2_row, double &dfacc, int &nchg, uint32_t *win, float *stg,
                                                int &wn) {
@@ -918,8 +1418,8 @@ __device__ __forceinline__ void rows_block_win(const CdArgs &a, int64_t b0, int 
         }
     }
     float code[CPL], dlt[CPL];
-    nchg += chg_decide<B, FULL, true>(nullptr, a.d + b0, bw, a.maxq, s2, true, lane, t, st, code, dlt, dfacc,
-                                      a.sbar + b0 * a.lds + b0, a.lds);
+    nchg += chg_decide<B, FULL, true, TIE>(nullptr, a.d + b0, bw, a.maxq, s2, true, lane, t, st, code, dlt, dfacc,
+                                      a.sbar + b0 * a.lds + b0, a.lds, &a, i, b0, stg);
     cd_epilogue<B, FULL, true, GR>(a, b0, bw, i, lane, code, dlt, true);
     // window = [entries left of the block (k1)] [this visit's changes (nn)] [entries right of it]
     int k1 = 0, k2 = 0;
@@ -995,8 +1495,8 @@ __device__ __forceinline__ void rows_block_win(const CdArgs &a, int64_t b0, int 
 // of the final codes.
 constexpr int kRowsMaxWarps = 28;   // rows per CTA of the persistent kernel (896 threads: 72 registers)
 
-template <int B, bool GR>
-__global__ void __launch_bounds__(32 * kRowsMaxWarps, 1) k_cd_rows_lists(const CdArgs a, int t_begin, int t_end,
+template <int B, bool GR, bool TIE = false>
+__global__ void __launch_bounds__(32 * kRowsMaxWarps, 1) k_cd_rows_lists(const __grid_constant__ CdArgs a, int t_begin, int t_end,
                                                            double *rowdf_t, uint8_t *sweep_codes,
                                                            int first_lockstep, int free_max_changes, int flush) {
     if (a.gate && *a.gate != a.gate_run) return;   // uniform: the dense form of the sweep runs
@@ -1063,13 +1563,13 @@ __global__ void __launch_bounds__(32 * kRowsMaxWarps, 1) k_cd_rows_lists(const C
                     const int bw = static_cast<int>((a.p - b0) < B ? (a.p - b0) : B);
                     if (wn >= 0) {
                         if (bw == B)
-                            rows_block_win<B, true, GR>(a, b0, bw, i, lane, s2, dfacc, nchg, win, stg, wn);
+                            rows_block_win<B, true, GR, TIE>(a, b0, bw, i, lane, s2, dfacc, nchg, win, stg, wn);
                         else
-                            rows_block_win<B, false, GR>(a, b0, bw, i, lane, s2, dfacc, nchg, win, stg, wn);
+                            rows_block_win<B, false, GR, TIE>(a, b0, bw, i, lane, s2, dfacc, nchg, win, stg, wn);
                     } else if (bw == B) {
-                        rows_block<B, true, true, GR>(a, b0, bw, tri, bar, 0u, i, row_ok, lane, s2, dfacc, nchg);
+                        rows_block<B, true, true, GR, TIE>(a, b0, bw, tri, bar, 0u, i, row_ok, lane, s2, dfacc, nchg, stg);
                     } else {
-                        rows_block<B, false, true, GR>(a, b0, bw, tri, bar, 0u, i, row_ok, lane, s2, dfacc, nchg);
+                        rows_block<B, false, true, GR, TIE>(a, b0, bw, tri, bar, 0u, i, row_ok, lane, s2, dfacc, nchg, stg);
                     }
                 }
             }
@@ -1081,11 +1581,14 @@ __global__ void __launch_bounds__(32 * kRowsMaxWarps, 1) k_cd_rows_lists(const C
                     mbar_arrive_expect_tx(bar, bytes);
                     bulk_load(tri, a.tri + (b0 / B) * C::PACK, bytes, bar);
                 }
+                // the warp's row for the near-tie refinement, after the packed block
+                float *tblk = cd_smem + C::PACK + 4 + warp * B;
                 const bool ok =
                     bw == B
-                        ? rows_block<B, true, false, GR>(a, b0, bw, tri, bar, use & 1u, i, row_ok, lane, s2, dfacc, nchg)
-                        : rows_block<B, false, false, GR>(a, b0, bw, tri, bar, use & 1u, i, row_ok, lane, s2, dfacc,
-                                                      nchg);
+                        ? rows_block<B, true, false, GR, TIE>(a, b0, bw, tri, bar, use & 1u, i, row_ok, lane, s2, dfacc, nchg,
+                                                     tblk)
+                        : rows_block<B, false, false, GR, TIE>(a, b0, bw, tri, bar, use & 1u, i, row_ok, lane, s2, dfacc,
+                                                      nchg, tblk);
                 ++use;
                 if (!ok) {
                     set_error(a.err, ERR_TIMEOUT);
@@ -1093,7 +1596,11 @@ __global__ void __launch_bounds__(32 * kRowsMaxWarps, 1) k_cd_rows_lists(const C
                 }
                 // every warp is done with this block's Sigma_bar before the next copy replaces it
                 __syncthreads();
-                if (s_bad) return;
+                if (s_bad) {
+                    // the copy may still land: keep the CTA until it has (bounded)
+                    if (threadIdx.x == 0) mbar_wait_bounded(bar, (use - 1) & 1u, nullptr);
+                    return;
+                }
             }
         }
         prev = nchg;
@@ -1153,17 +1660,22 @@ __global__ void k_obj_prefix(const double *rowdf_t, int64_t q, int nt, const dou
     }
 }
 
-template <int B, bool FULL, bool SEQ, bool RELAX = false, bool DF = false>
+template <int B, bool FULL, bool SEQ, bool RELAX = false, bool DF = false, bool TIE = false>
 static cudaError_t launch_cd_block_b(const CdArgs &a, int nsm, cudaStream_t s) {
     using C = CdCfg<B>;
     if (a.nsplit > C::MAX_SPLITS) return cudaErrorInvalidValue;
-    auto kern = SEQ ? k_cd_block_seq<B, FULL, RELAX, DF> : k_cd_block_chg<B, FULL>;
+    auto kern = SEQ ? k_cd_block_seq<B, FULL, RELAX, DF, TIE> : k_cd_block_chg<B, FULL, TIE>;
     // one CTA per SM when the rows allow it (the packed block is shared by the CTA's rows)
     int64_t warps = ceil_div(a.q, nsm);
     if (warps > C::MAX_WARPS) warps = C::MAX_WARPS;
     if (warps < 1) warps = 1;
-    // the sequential kernel with DF keeps one row of beta~ per warp after the packed block
-    const int smem = (SEQ && DF) ? (C::PACK + 4) * 4 + static_cast<int>(warps) * B * 4 : C::SMEM;
+    // the sequential kernel keeps one row of beta~ per warp (DF), and one row of the
+    // codes decided in the visit and one snapshot row (near-tie refinement), after the
+    // packed block
+    // (the change-driven kernel keeps one row per warp for the refinement)
+    const int rows = static_cast<int>(warps) * B * 4;
+    const int smem = SEQ ? (C::PACK + 4) * 4 + (DF ? rows : 0) + (TIE ? 2 * rows : 0)
+                         : (C::PACK + 4) * 4 + (TIE ? tie_cta_bytes<B>(static_cast<int>(warps)) : 0);
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     const unsigned grid = static_cast<unsigned>(ceil_div(a.q, warps));
@@ -1173,8 +1685,15 @@ static cudaError_t launch_cd_block_b(const CdArgs &a, int nsm, cudaStream_t s) {
 
 template <int B, bool FULL>
 static cudaError_t launch_cd_block_f(const CdArgs &a, int nsm, cudaStream_t s) {
-    if (!a.frac) return launch_cd_block_b<B, FULL, false>(a, nsm, s);
+    // the refinement variants: change-driven kernel, and the first sweep's sequential kernel
+    const bool tie = a.tie_eps > 0.0f;
+    if (!a.frac)
+        return tie ? launch_cd_block_b<B, FULL, false, false, false, true>(a, nsm, s)
+                   : launch_cd_block_b<B, FULL, false>(a, nsm, s);
     if (a.vout) return a.rowdf ? launch_cd_block_b<B, FULL, true, true, true>(a, nsm, s) : cudaErrorInvalidValue;
+    if (tie && a.first_sweep && !a.vstart)
+        return a.rowdf ? launch_cd_block_b<B, FULL, true, false, true, true>(a, nsm, s)
+                       : launch_cd_block_b<B, FULL, true, false, false, true>(a, nsm, s);
     return a.rowdf ? launch_cd_block_b<B, FULL, true, false, true>(a, nsm, s)
                    : launch_cd_block_b<B, FULL, true, false, false>(a, nsm, s);
 }
@@ -1195,7 +1714,7 @@ cudaError_t launch_cd_block(int B, const CdArgs &a, int nsm, cudaStream_t s) {
 
 int64_t packed_diag_floats(int64_t p, int B) { return ceil_div(p, B) * packed_block_floats(B); }
 
-template <int B, bool GR>
+template <int B, bool GR, bool TIE>
 static cudaError_t launch_cd_rows_b(const CdArgs &a, int t_begin, int t_end, double *rowdf_t,
                                    uint8_t *sweep_codes, int first_lockstep, int free_max_changes, int flush,
                                    int nsm, cudaStream_t s) {
@@ -1203,12 +1722,14 @@ static cudaError_t launch_cd_rows_b(const CdArgs &a, int t_begin, int t_end, dou
     int64_t warps = ceil_div(a.q, nsm);
     if (warps > kRowsMaxWarps) warps = kRowsMaxWarps;
     if (warps < 1) warps = 1;
-    // the packed block (lockstep) or one free-mode area per warp, whichever is larger
-    const int smem = static_cast<int>(warps * kFreeWarpBytes > C::SMEM ? warps * kFreeWarpBytes : C::SMEM);
-    cudaError_t e = cudaFuncSetAttribute(k_cd_rows_lists<B, GR>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    // the packed block and one row per warp for the near-tie refinement (lockstep), or
+    // one free-mode area per warp, whichever is larger
+    const int64_t lock = C::SMEM + (TIE ? warps * B * 4 : 0);
+    const int smem = static_cast<int>(warps * kFreeWarpBytes > lock ? warps * kFreeWarpBytes : lock);
+    cudaError_t e = cudaFuncSetAttribute(k_cd_rows_lists<B, GR, TIE>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     const unsigned grid = static_cast<unsigned>(ceil_div(a.q, warps));
-    k_cd_rows_lists<B, GR><<<grid, static_cast<unsigned>(32 * warps), smem, s>>>(
+    k_cd_rows_lists<B, GR, TIE><<<grid, static_cast<unsigned>(32 * warps), smem, s>>>(
         a, t_begin, t_end, rowdf_t, sweep_codes, first_lockstep, free_max_changes, flush);
     return cudaGetLastError();
 }
@@ -1218,18 +1739,18 @@ cudaError_t launch_cd_rows_lists(int B, const CdArgs &a, int t_begin, int t_end,
                                  int nsm, cudaStream_t s) {
     if (!a.sbar || !a.lent || !a.lcnt || a.first_sweep || t_end <= t_begin) return cudaErrorInvalidValue;
     const int f = first_lockstep, m = free_max_changes, fl = flush;
+#define QE_ROWS(BB)                                                                                            \
+    (a.grouped ? (a.tie_eps > 0.0f ? launch_cd_rows_b<BB, true, true>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, fl, nsm, s)   \
+                                   : launch_cd_rows_b<BB, true, false>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, fl, nsm, s)) \
+               : (a.tie_eps > 0.0f ? launch_cd_rows_b<BB, false, true>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, fl, nsm, s)  \
+                                   : launch_cd_rows_b<BB, false, false>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, fl, nsm, s)))
     switch (B) {
-        case 64:
-            return a.grouped ? launch_cd_rows_b<64, true>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, fl, nsm, s)
-                             : launch_cd_rows_b<64, false>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, fl, nsm, s);
-        case 128:
-            return a.grouped ? launch_cd_rows_b<128, true>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, fl, nsm, s)
-                             : launch_cd_rows_b<128, false>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, fl, nsm, s);
-        case 256:
-            return a.grouped ? launch_cd_rows_b<256, true>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, fl, nsm, s)
-                             : launch_cd_rows_b<256, false>(a, t_begin, t_end, rowdf_t, sweep_codes, f, m, fl, nsm, s);
+        case 64: return QE_ROWS(64);
+        case 128: return QE_ROWS(128);
+        case 256: return QE_ROWS(256);
         default: return cudaErrorInvalidValue;
     }
+#undef QE_ROWS
 }
 
 cudaError_t launch_obj_prefix(const double *rowdf_t, int64_t q, int nt, const double *prev, double *out,

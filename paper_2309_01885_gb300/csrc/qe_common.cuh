@@ -59,16 +59,20 @@ __device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
 }
 
 // Bounded wait for the phase with parity `parity`; false when it gave up
-// (after kWaitLimitNs) or when *abort became non-zero.
-__device__ __forceinline__ bool mbar_wait_bounded(uint64_t *bar, uint32_t parity,
-                                                  volatile int *abort) {
+// (after limit_ns) or when *abort became non-zero.
+__device__ __forceinline__ bool mbar_wait_bounded_ns(uint64_t *bar, uint32_t parity, volatile int *abort,
+                                                     unsigned long long limit_ns) {
     if (mbar_try_wait(bar, parity)) return true;
     const unsigned long long t0 = globaltimer_ns();
     while (true) {
         if (mbar_try_wait(bar, parity)) return true;
         if (abort && *abort) return false;
-        if (globaltimer_ns() - t0 > kWaitLimitNs) return false;
+        if (globaltimer_ns() - t0 > limit_ns) return false;
     }
+}
+
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t *bar, uint32_t parity, volatile int *abort) {
+    return mbar_wait_bounded_ns(bar, parity, abort, kWaitLimitNs);
 }
 
 __device__ __forceinline__ void mbar_inval(uint64_t *bar) {
@@ -86,6 +90,11 @@ __device__ __forceinline__ void cp_async16(void *dst, const void *src) {
 // Wait for all of this thread's cp.async copies (they always complete).
 __device__ __forceinline__ void cp_async_wait_all() {
     asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+}
+
+// Prefetch the 128-byte line holding p into L2 (no register or shared memory held).
+__device__ __forceinline__ void prefetch_l2(const void *p) {
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(reinterpret_cast<uint64_t>(p)));
 }
 
 // ---- TMA --------------------------------------------------------------------

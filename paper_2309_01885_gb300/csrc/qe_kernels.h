@@ -53,6 +53,24 @@ struct CdArgs {
     // adaptive sweep schedule enqueues both forms of a sweep and runs one)
     const int *gate;
     int gate_run;
+    // test hook of the failure path (in-block kernels): skip_copy = 1 issues no copy
+    // of the packed Sigma_bar block, so the bounded wait for it gives up after
+    // wait_ns (0 = the library's limit) and latches a timeout; nothing is in flight
+    int skip_copy;
+    unsigned long long wait_ns;
+    // Near-tie refinement: a decision whose beta~ (binary32, grid units) lies within
+    // tie_eps of a rounding midpoint between two levels is taken again from beta~
+    // recomputed in binary64 from the row's current state (Lemma 1):
+    //   beta~_j = T_j + sum_{k != j} (T_k - What_k) Sigma_kj / Sigma_jj,  T = W (- H).
+    // 0 = off (relaxed sweeps and the sweep after one, whose start is real-valued).
+    float tie_eps;
+    const float *S;                 // Sigma as given (p x p, leading dimension lds_full)
+    int64_t lds_full;
+    const void *W;                  // the layer (bf16 or fp32, leading dimension ldw)
+    int w_bf16;
+    int64_t ldw;
+    const float *Hd;                // outlier variant: dense H (target W - H, leading dimension ldh), or NULL
+    int64_t ldh;
 };
 
 // Objective / reference-norm reduction.

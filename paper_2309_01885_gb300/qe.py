@@ -43,7 +43,8 @@ class QEOpts(ctypes.Structure):
                 ("init_codes", ctypes.c_void_p), ("sweep_codes", ctypes.c_void_p),
                 ("wx_norm2", ctypes.c_void_p), ("workspace", ctypes.c_void_p),
                 ("workspace_bytes", ctypes.c_size_t), ("timer", ctypes.c_void_p),
-                ("switch_below", ctypes.c_int64), ("sweep_forms", ctypes.c_void_p)]
+                ("switch_below", ctypes.c_int64), ("sweep_forms", ctypes.c_void_p),
+                ("wait_test", ctypes.c_int), ("tie_eps", ctypes.c_float)]
 
 
 _lib = None
@@ -295,7 +296,7 @@ def qe_quantize_layer(W: torch.Tensor, Sigma: torch.Tensor, bits: int, iters: in
                       workspace: torch.Tensor | None = None, timer: Timer | None = None,
                       dense_sweeps: int = 0, free_changes: int = 0, relax_period: int = 0,
                       group_size: int = 0, switch_below: int = 0, record_forms: bool = False,
-                      stream=None) -> dict:
+                      wait_test: int = 0, tie_eps: float = 0.0, stream=None) -> dict:
     """QuantEase on one layer; returns codes (u8 q x p), scales, zeros, obj (fp64 per sweep),
     and optionally sweep_codes (iters x q x p) and wx_norm2.  dense_sweeps: sweeps whose
     cross-block term uses the tensor-core GEMM before the change lists take over (0 = the
@@ -303,7 +304,9 @@ def qe_quantize_layer(W: torch.Tensor, Sigma: torch.Tensor, bits: int, iters: in
     free_changes: changes per row below which list sweeps run row by row (0 = default, -1 = never);
     relax_period: the relax heuristic of Sec. 3.2 (sweep t from 1 with t mod R = 0 and t < iters
     keeps beta~ unquantized; 0 = off); group_size: grouped grids (scales / zeros q x groups);
-    record_forms: also return sweep_forms (uint8 per sweep: 0 sequential, 1 dense, 2 lists)."""
+    record_forms: also return sweep_forms (uint8 per sweep: 0 sequential, 1 dense, 2 lists);
+    wait_test: the failure-path test hook of qe_opts (a bounded device wait made to give up);
+    tie_eps: near-tie refinement threshold in grid steps (0 = default 2e-5, negative = off)."""
     q, p = W.shape
     dev = W.device
     codes = torch.empty(q, p, dtype=torch.uint8, device=dev)
@@ -315,6 +318,8 @@ def qe_quantize_layer(W: torch.Tensor, Sigma: torch.Tensor, bits: int, iters: in
     norm = torch.empty(1, dtype=torch.float64, device=dev) if want_norm else None
     o = _opts(block_width, 0, init_codes, sweep, norm, workspace, timer, dense_sweeps, free_changes,
               relax_period, group_size, switch_below)
+    o.wait_test = wait_test
+    o.tie_eps = tie_eps
     forms = torch.full((iters,), 255, dtype=torch.uint8, device=dev) if record_forms else None
     o.sweep_forms = None if forms is None else forms.data_ptr()
     _check(load().qe_quantize_layer(_ptr(W), _dtype(W), q, p, _rowmajor_ld(W), _ptr(Sigma), bits, iters,
@@ -334,7 +339,7 @@ def qe_quantize_layer_outlier(W: torch.Tensor, Sigma: torch.Tensor, bits: int, i
                               s_budget: int, *, power_iters: int = 0, init_codes=None,
                               record_sweeps: bool = False, want_norm: bool = False,
                               workspace: torch.Tensor | None = None, structured: bool = False,
-                              free_changes: int = 0,
+                              free_changes: int = 0, tie_eps: float = 0.0,
                               timer: Timer | None = None, stream=None) -> dict:
     """Outlier-aware QuantEase; adds H_val, H_idx (sorted linear indices), H_nnz, obj_cd.
     structured: H keeps whole columns (floor(s_budget / q) of them); free_changes: as for
@@ -354,6 +359,7 @@ def qe_quantize_layer_outlier(W: torch.Tensor, Sigma: torch.Tensor, bits: int, i
     norm = torch.empty(1, dtype=torch.float64, device=dev) if want_norm else None
     o = _opts(0, power_iters, init_codes, sweep, norm, workspace, timer, free_changes=free_changes)
     o.structured_outliers = int(structured)
+    o.tie_eps = tie_eps
     _check(load().qe_quantize_layer_outlier(
         _ptr(W), _dtype(W), q, p, _rowmajor_ld(W), _ptr(Sigma), bits, iters, int(s_budget),
         ctypes.byref(o), _ptr(codes), _ptr(scales), _ptr(zeros), _ptr(H_val), _ptr(H_idx),

@@ -84,3 +84,84 @@ def teacher_forced(W64, S64, scale, zero, bits, sweep_codes_gpu, init_codes=None
 
 def code_match(codes_gpu, codes_oracle):
     return float(np.mean(np.asarray(codes_gpu) == np.asarray(codes_oracle)))
+
+
+def first_divergence(sweep_gpu, ref, scale, zero, bits, group_size=0):
+    """Compare the GPU's per-sweep codes with the oracle's free-running trajectory
+    (ref: alg1 with record=True, want_beta=True) row by row.  Up to a row's first
+    differing decision both sides hold the same state, so the oracle's fp64 beta~
+    there is the teacher-forced one: that decision must lie within MIDPOINT_TOL
+    (grid steps) of a rounding midpoint, which is what starts a legitimate cascade.
+    Returns the rows that diverge, each as (row, sweep, column, |frac - 0.5|, codes
+    that differ after the last sweep)."""
+    sweep_gpu = np.asarray(sweep_gpu)
+    oc = ref["sweep_codes"]
+    iters, q, p = sweep_gpu.shape
+    if group_size:
+        g = np.arange(p) // group_size
+        sc, zc = scale.astype(np.float64)[:, g], zero.astype(np.float64)[:, g]
+    else:
+        sc = np.repeat(scale.astype(np.float64)[:, None], p, axis=1)
+        zc = np.repeat(zero.astype(np.float64)[:, None], p, axis=1)
+    out = []
+    for r in range(q):
+        diff = sweep_gpu[:, r, :] != oc[:, r, :]
+        if not diff.any():
+            continue
+        t = int(np.argmax(diff.any(axis=1)))
+        j = int(np.argmax(diff[t]))
+        x = ref["beta"][t, r, j] / sc[r, j] + zc[r, j]
+        dist = abs(x - np.floor(x) - 0.5)
+        assert dist <= MIDPOINT_TOL, (f"row {r}: first divergence at sweep {t + 1}, column {j} is not "
+                                      f"near a midpoint (beta~/s + z = {x:.9f})")
+        out.append((r, t, j, float(dist), int(diff[-1].sum())))
+    return out
+
+
+def outlier_replay(W64, S64, scale, zero, bits, sweep_gpu, H_idx_gpu, H_val_gpu, H0, eta, s_budget,
+                   structured=False, h_rtol=1e-5):
+    """Teacher-forced replay of Algorithm 4, iteration by iteration from the GPU's own
+    state.  sweep_gpu[t]: the GPU's codes after iteration t; H_idx_gpu[t] /
+    H_val_gpu[t]: its H after iteration t (support, ascending, and values); H0: the
+    start H = P_s(W).  Iteration t:
+      * CD half: Algorithm 1 for one sweep on the target W - H_{t-1}, from the GPU's
+        codes after iteration t - 1 (iteration 0 starts at the target itself), with
+        the GPU's decisions forced: each must be the nearest level of the fp64 beta~
+        unless within MIDPOINT_TOL of a midpoint;
+      * IHT half: the oracle's step from (codes_t, H_{t-1}) must keep the GPU's
+        support, except entries (columns) whose |T| (column norm) ties the threshold
+        within h_rtol, and the GPU's values must equal T there within h_rtol of max |T|.
+    Returns the number of support entries that differed at ties."""
+    q, p = W64.shape
+    iters = sweep_gpu.shape[0]
+    ties = 0
+    for t in range(iters):
+        Hprev = H0 if t == 0 else _dense(H_idx_gpu[t - 1], H_val_gpu[t - 1], q, p)
+        init = None if t == 0 else sweep_gpu[t - 1]
+        teacher_forced(W64 - Hprev, S64, scale, zero, bits, sweep_gpu[t][None], init_codes=init)
+        T, sup = oracle.get().iht_step(W64, S64, sweep_gpu[t], scale, zero, Hprev, eta, s_budget, structured)
+        gsup = np.asarray(H_idx_gpu[t])
+        Tf = T.ravel()
+        if structured:
+            norms = np.sum(T * T, axis=0)
+            oc, gc = np.unique(sup % p), np.unique(gsup % p)
+            thr = norms[oc].min() if oc.size else 0.0
+            for c in np.setxor1d(oc, gc):
+                assert abs(norms[c] - thr) <= h_rtol * thr, f"iteration {t + 1}: column {c} kept by one side only"
+                ties += 1
+        else:
+            thr = np.abs(Tf[sup]).min() if sup.size else 0.0
+            for k in np.setxor1d(sup, gsup):
+                assert abs(abs(Tf[k]) - thr) <= h_rtol * thr, f"iteration {t + 1}: entry {k} kept by one side only"
+                ties += 1
+        scale_t = np.abs(Tf).max() if Tf.size else 1.0
+        err = np.abs(np.asarray(H_val_gpu[t], np.float64) - Tf[gsup])
+        assert np.all(err <= h_rtol * scale_t), (f"iteration {t + 1}: H values off by {err.max():.3e} "
+                                                 f"(max |T| {scale_t:.3e})")
+    return ties
+
+
+def _dense(idx, val, q, p):
+    H = np.zeros(q * p)
+    H[np.asarray(idx)] = np.asarray(val, np.float64)
+    return H.reshape(q, p)

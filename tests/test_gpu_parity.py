@@ -250,6 +250,36 @@ def test_layer_lists_agree_with_dense():
     assert m >= parity.CODE_MATCH, f"codes match {m:.5f}"
 
 
+@pytest.mark.parametrize("corr_rank,group_size,dense", [(0, 0, 0), (4, 0, 0), (0, 256, 0), (4, 0, 100)],
+                         ids=["plain", "correlated", "groups", "dense-window"])
+def test_near_tie_refinement(corr_rank, group_size, dense):
+    """With the near-tie refinement (the default), every GPU decision is the nearest
+    level of the binary64 beta~ of the GPU's own state: the teacher-forced replay
+    finds no disagreement at all, not even within the 1e-4 midpoint tolerance, and
+    the trajectory matches the free-running oracle code for code.  With it off the
+    same run stays within the tolerance.  Sweep 1 (sequential kernel), the change
+    lists, the dense window and grouped grids all decide near-ties this way."""
+    q, p, bits, iters = 160, 520, 4, 6
+    W = inputs.layer_weights(q, p, dtype=torch.bfloat16, seed=81, device="cuda")
+    X = inputs.calib_inputs(p, 4096, dtype=torch.bfloat16, seed=81, device="cuda", heavy_frac=0.01,
+                            heavy_mult=30.0, corr_rank=corr_rank)
+    Sg = qe.qe_build_sigma(X)
+    kw = dict(record_sweeps=True, group_size=group_size, dense_sweeps=dense)
+    out = qe.qe_quantize_layer(W, Sg, bits, iters, **kw)
+    off = qe.qe_quantize_layer(W, Sg, bits, iters, tie_eps=-1.0, **kw)
+    assert qe.qe_sync_status() == qe.QE_OK
+    W64, S64 = parity.f64(W), parity.f64(Sg)
+    s, z = O.grid(W64, bits, group_size=group_size)
+    assert np.array_equal(out["scales"].cpu().numpy(), s)
+    sweep = out["sweep_codes"].cpu().numpy()
+    nbad, ntot = parity.teacher_forced(W64, S64, s, z, bits, sweep, group_size=group_size)
+    assert nbad == 0, f"{nbad} of {ntot} decisions off the binary64 nearest level"
+    ref = O.alg1(W64, S64, s, z, bits, iters, group_size=group_size, record=True)
+    assert np.array_equal(sweep, ref["sweep_codes"])
+    parity.check_obj(out["obj"].cpu().numpy(), ref["obj"], what="objective with refinement")
+    parity.teacher_forced(W64, S64, s, z, bits, off["sweep_codes"].cpu().numpy(), group_size=group_size)
+
+
 @pytest.mark.parametrize("group_size", [0, 256])
 def test_layer_adaptive_schedule(group_size):
     """The adaptive sweep schedule (dense form until a sweep changes fewer than
@@ -581,6 +611,37 @@ def test_outlier_parity_small(q, p, bits, frac):
     assert np.allclose(Hd[common], ref["H"].ravel()[common], rtol=1e-3, atol=1e-6)
     # Lemma 3: the IHT half never increases g
     assert np.all(out["obj"].cpu().numpy() <= out["obj_cd"].cpu().numpy() * (1 + 1e-6))
+    # teacher-forced, iteration by iteration from the GPU's own state
+    _outlier_replay(W, Sg, bits, iters, s_budget, power_iters, False, out)
+
+
+def _outlier_replay(W, Sg, bits, iters, s_budget, power_iters, structured, out):
+    """The GPU's Algorithm 4 trajectory replayed through the oracle one iteration at a
+    time from the GPU's own state (parity.outlier_replay); H after every iteration
+    comes from runs stopped there, which must be prefixes of the full run."""
+    runs = [qe.qe_quantize_layer_outlier(W, Sg, bits, k, s_budget, power_iters=power_iters,
+                                         structured=structured) for k in range(1, iters)] + [out]
+    assert qe.qe_sync_status() == qe.QE_OK
+    for o in runs[:-1]:
+        k = o["obj"].numel()
+        assert torch.equal(o["obj"], out["obj"][:k])
+    W64, S64 = parity.f64(W), parity.f64(Sg)
+    q, p = W64.shape
+    if structured:
+        cols = O.topk_columns(W64, s_budget // q)
+        H0 = np.zeros_like(W64)
+        H0[:, cols] = W64[:, cols]
+    else:
+        k0 = O.topk(W64, s_budget)
+        H0 = np.zeros(W64.size)
+        H0[k0] = W64.ravel()[k0]
+        H0 = H0.reshape(q, p)
+    eta = 1.0 / (2.0 * O.power_lambda(S64, power_iters))
+    nnz = [int(o["H_nnz"].item()) for o in runs]
+    hidx = [o["H_idx"][:m].cpu().numpy() for o, m in zip(runs, nnz)]
+    hval = [o["H_val"][:m].cpu().numpy() for o, m in zip(runs, nnz)]
+    return parity.outlier_replay(W64, S64, out["scales"].cpu().numpy(), out["zeros"].cpu().numpy(), bits,
+                                 out["sweep_codes"].cpu().numpy(), hidx, hval, H0, eta, s_budget, structured)
 
 
 def _planted_columns(W, cols, std, seed):
@@ -602,9 +663,10 @@ def test_structured_outlier_parity_small(q, p, bits, ncols):
     Sg = qe.qe_build_sigma(X)
     s_budget = ncols * q + 7
     out = qe.qe_quantize_layer_outlier(W, Sg, bits, iters, s_budget, power_iters=power_iters,
-                                       structured=True)
+                                       structured=True, record_sweeps=True)
     assert qe.qe_sync_status() == qe.QE_OK
     W64, S64 = parity.f64(W), parity.f64(Sg)
+    _outlier_replay(W, Sg, bits, iters, s_budget, power_iters, True, out)
     ref = O.outlier(W64, S64, bits, iters, s_budget, power_iters, structured=True)
     assert np.array_equal(out["scales"].cpu().numpy(), ref["scale"])
     assert np.array_equal(out["zeros"].cpu().numpy(), ref["zero"])
