@@ -79,6 +79,8 @@ def parse():
                     help="relax heuristic period R (Sec. 3.2): sweeps t with t mod R = 0, t < iters, unquantized")
     ap.add_argument("--tokens", type=int, default=0,
                     help="override n (calibration tokens), for small profiling captures only")
+    ap.add_argument("--rows", type=int, default=0,
+                    help="override q (rows of W), for small profiling captures only")
     return ap.parse_args()
 
 
@@ -383,7 +385,9 @@ def layer_schedule(q, p, iters, forms, relax, dense_opt, adaptive, grouped, outl
         if kind in ("first", "seq", "dense"):
             f = win_flops if window == 1 else tri_flops
             trail_flops += f
-            trail_exec += (3 if kind == "dense" and not grouped else 6) * f   # three-plane changes: 6 products
+            # integer changes of a window sweep: one fp16 plane x two fp16 planes of Sigma_bar
+            # (2 products); real-valued or grouped changes: three bf16 planes (6 products)
+            trail_exec += (2 if kind == "dense" and not grouped else 6) * f
     refreshes = (1 if plan[0][0] == "first" else 0) + extra
     # launches: set-up (grid, Sigma diagonal, Sigma_bar planes, 1/d, packed blocks,
     # Sigma_bar rows, [W planes], P, initial residual); sweep 1: nblk - 1 trailing GEMMs
@@ -446,6 +450,8 @@ def main():
     import dataclasses
     if args.tokens:
         cfg = dataclasses.replace(cfg, n=args.tokens)
+    if args.rows:
+        cfg = dataclasses.replace(cfg, q=args.rows)
     q, p, n = cfg.q, cfg.p, cfg.n
     cfg_r = dataclasses.replace(cfg, seed=cfg.seed + rank)   # each rank owns a different layer
     W = cfg_r.weights("cuda")
@@ -594,7 +600,8 @@ def main():
     gemm_cd_ms = sum(timed[k][1] for k in kinds[:3]) / args.steps
     gemm_cd_launches = sum(timed[k][0] for k in kinds[:3]) // args.steps
     gemm_cd_alg = sum(2 * q * p * p * (1 + sc["refreshes"]) + sc["trail_flops"] for sc in sched)
-    gemm_cd_exec = sum((3 + (6 if grouped else 3) * sc["refreshes"]) * 2 * qpad * ppad * kpad + sc["trail_exec"]
+    # P: bf16 W x three bf16 planes (3 products); residual: C - z x two fp16 planes (2), grouped: 6
+    gemm_cd_exec = sum((3 + (6 if grouped else 2) * sc["refreshes"]) * 2 * qpad * ppad * kpad + sc["trail_exec"]
                        for sc in sched)
     r_cd = roofline_tensor("CD sweep (all kernels of the quantize calls)", cd_alg, None, sum(cd_avg), None,
                            peak_tc, peak_src, None, "per-kernel traffic under the gemm and list entries",
@@ -604,8 +611,10 @@ def main():
                                     "executed_tflops": gemm_cd_exec / (gemm_cd_ms / 1e3) / 1e12 if gemm_cd_ms else None,
                                     "frac_executed": (gemm_cd_exec / (gemm_cd_ms / 1e3) / 1e12 / peak_tc)
                                     if gemm_cd_ms else None},
-                           split_factor=("3 bf16 products per fp32-accurate product (6 where both operands "
-                                         "are real-valued); ceiling of the algorithmic fraction about 1/3"))
+                           split_factor=("per algorithmic product: 2 fp16 products where one operand is an "
+                                         "exact small integer (window sweeps, residual refresh), 3 bf16 products "
+                                         "(P), 6 where both operands are real-valued (sweep 1); ceiling of the "
+                                         "algorithmic fraction about 1/2"))
     # (3) k_tc_gemm<256> over all its launches in a step (Sigma + the CD GEMMs)
     gemm_ms = sigma_avg + gemm_cd_ms
     tr, tr_note = traffic_record("k_tc_gemm_trail", cfg.name)

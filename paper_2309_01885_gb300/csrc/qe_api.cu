@@ -87,7 +87,7 @@ struct Plan {
     int B = kDefaultBlock, smax = 1;
     int64_t gsize = 0, ngroups = 1;   // grid columns per group (p: per row), groups per row
     bool grouped = false;
-    size_t snt = 0, d = 0, dinv = 0, tri = 0, P = 0, R = 0, wpl = 0, qf = 0, dp = 0, part = 0, objp = 0,
+    size_t snt = 0, snh = 0, cscale = 0, d = 0, dinv = 0, tri = 0, P = 0, R = 0, wpl = 0, qf = 0, dp = 0, part = 0, objp = 0,
            rowdf = 0, objbase = 0, sbar = 0, lcnt = 0, lent = 0, rowdft = 0, sw = 0;
     int64_t nblk = 0;
     size_t PW = 0, H = 0, T = 0, st = 0, cg = 0, ce = 0, sb = 0, eb = 0, y0 = 0, y1 = 0, lam = 0,
@@ -116,6 +116,8 @@ static Plan make_plan(int64_t q, int64_t p, int B, bool outlier, int wpl_planes,
     const size_t qld = static_cast<size_t>(q) * pl.ld;
     size_t cur = 0;
     pl.snt = take(cur, static_cast<size_t>(3 * p) * pl.ld * 2);
+    pl.snh = take(cur, static_cast<size_t>(2 * p) * pl.ld * 2);   // fp16 hi / lo, rows scaled by powers of two
+    pl.cscale = take(cur, p * 4);
     pl.d = take(cur, p * 4);
     pl.dinv = take(cur, p * 4);
     pl.tri = take(cur, static_cast<size_t>(packed_diag_floats(p, B)) * 4);
@@ -207,6 +209,8 @@ struct Ctx {
     uint8_t *ws = nullptr;
     bool own = false;
     __nv_bfloat16 *snt = nullptr, *wpl = nullptr, *qf = nullptr, *dp = nullptr;
+    __half *snh = nullptr;
+    float *cscale = nullptr;
     float *d = nullptr, *dinv = nullptr, *tri = nullptr, *P = nullptr, *R = nullptr, *part = nullptr;
     double *objp = nullptr, *rowdf = nullptr, *objbase = nullptr;
     float *sbar = nullptr;
@@ -224,6 +228,8 @@ struct Ctx {
     float *cnorm = nullptr, *cval = nullptr;
     int64_t *ccols = nullptr, *cn = nullptr;
     CUtensorMap tm_snt256, tm_snt64, tm_snt128, tm_qf, tm_dp, tm_wa;
+    // the fp16 forms: Sigma_bar^T in two planes, C - z and the integer changes Delta'
+    CUtensorMap tm_snh256, tm_snh64, tm_snh128, tm_qf16, tm_dp16;
     int wa_planes = 1;
     // near-tie refinement: the layer's inputs as given (and H for the outlier variant)
     float tie_eps = 0.0f;
@@ -264,6 +270,8 @@ static qe_status setup_ctx(Ctx &c, const Plan &pl, const qe_opts *o, cudaStream_
     }
     uint8_t *w = c.ws;
     c.snt = at<__nv_bfloat16>(w, pl.snt);
+    c.snh = at<__half>(w, pl.snh);
+    c.cscale = at<float>(w, pl.cscale);
     c.d = at<float>(w, pl.d);
     c.dinv = at<float>(w, pl.dinv);
     c.tri = at<float>(w, pl.tri);
@@ -310,7 +318,10 @@ static qe_status setup_ctx(Ctx &c, const Plan &pl, const qe_opts *o, cudaStream_
         !make_tmap_bf16(&c.tm_snt64, c.snt, 3 * p, p, ld, 64) ||
         !make_tmap_bf16(&c.tm_snt128, c.snt, 3 * p, p, ld, 128) ||
         !make_tmap_bf16(&c.tm_qf, c.qf, pl.grouped ? 3 * q : q, p, ld, 128) ||
-        !make_tmap_bf16(&c.tm_dp, c.dp, 3 * q, p, ld, 128))
+        !make_tmap_bf16(&c.tm_dp, c.dp, 3 * q, p, ld, 128) ||
+        !make_tmap_f16(&c.tm_snh256, c.snh, 2 * p, p, ld, 256) || !make_tmap_f16(&c.tm_snh64, c.snh, 2 * p, p, ld, 64) ||
+        !make_tmap_f16(&c.tm_snh128, c.snh, 2 * p, p, ld, 128) || !make_tmap_f16(&c.tm_qf16, c.qf, q, p, ld, 128) ||
+        !make_tmap_f16(&c.tm_dp16, c.dp, q, p, ld, 128))
         return QE_ERR_CUDA;
     return QE_OK;
 }
@@ -347,12 +358,24 @@ static void set_prods(GemmArgs &g, int a_planes) {
     }
 }
 
+// An exact fp16 A (C - z, or integer changes) times the two fp16 planes of Sigma_bar^T.
+static void set_prods_h2(GemmArgs &g, const Ctx &c, int64_t col0) {
+    g.n_prod = 2;
+    g.prod_a[0] = 0;
+    g.prod_b[0] = 0;
+    g.prod_a[1] = 0;
+    g.prod_b[1] = 1;
+    g.f16 = 1;
+    g.colscale = c.cscale + col0;
+}
+
 // Sigma -> d, Sigma_bar^T planes; W operand planes; P = W (I + Sigma_bar) into `Pout`.
 static qe_status prepare(Ctx &c, const void *W, int wbf16, int64_t ldw, const float *Sigma, float *Pout) {
     const int64_t q = c.pl.q, p = c.pl.p, ld = c.pl.ld;
     QE_CK(launch_sigma_norm(Sigma, p, p, c.d, c.snt, ld, c.err, c.s));
     QE_CK(launch_dinv(c.d, p, c.dinv, c.s));
     QE_CK(launch_pack_diag(c.snt, ld, p, c.pl.B, c.tri, c.s));
+    QE_CK(launch_sigma_planes_h2(Sigma, p, p, c.d, c.snh, ld, c.cscale, c.s));
     if (c.sbar) QE_CK(launch_sigma_bar_rows(Sigma, p, p, c.d, c.sbar, ld, c.s));
     const bool direct = wbf16 && ((reinterpret_cast<uintptr_t>(W) & 15u) == 0) && (ldw % 8 == 0);
     if (direct) {
@@ -397,7 +420,8 @@ static qe_status residual(Ctx &c, const float *scales, const float *zeros, const
     const int64_t q = c.pl.q, p = c.pl.p, ld = c.pl.ld;
     GemmArgs g = gemm_args(c, static_cast<int>(q), static_cast<int>(p), static_cast<int>(ceil_div(p, 64)),
                            EPI_RFULL);
-    set_prods(g, c.pl.grouped ? 3 : 1);
+    if (c.pl.grouped) set_prods(g, 3);
+    else set_prods_h2(g, c, 0);   // C - z is an exact small integer
     g.gsize = c.pl.gsize;
     g.ngroups = c.pl.ngroups;
     g.absolute = c.pl.grouped ? 1 : 0;
@@ -423,7 +447,8 @@ static qe_status residual(Ctx &c, const float *scales, const float *zeros, const
     }
     {
         Timed tm(c.timer, QE_KERNEL_RESIDUAL_GEMM, c.s);
-        QE_CK(launch_tc_gemm(256, c.tm_qf, c.tm_snt256, g, 1, c.s));
+        if (c.pl.grouped) QE_CK(launch_tc_gemm(256, c.tm_qf, c.tm_snt256, g, 1, c.s));
+        else QE_CK(launch_tc_gemm(256, c.tm_qf16, c.tm_snh256, g, 1, c.s));
     }
     if (f) QE_CK(launch_sum_partials(c.objp, static_cast<int>(rfull_partials(q, p)), f->obj, c.s));
     return QE_OK;
@@ -468,6 +493,8 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
     const int64_t q = c.pl.q, p = c.pl.p, ld = c.pl.ld;
     const int B = c.pl.B;
     const bool frac = src != SRC_CODES || relax;
+    // window sweeps over integer changes run their trailing GEMMs in fp16
+    const bool h2 = window != 0 && !frac && !c.pl.grouped;
     for (int64_t b0 = 0; b0 < p; b0 += B) {
         const int bw = static_cast<int>((p - b0) < B ? (p - b0) : B);
         const int64_t kcols = (window > 0) ? p : b0;
@@ -475,7 +502,8 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
         if (kcols > 0) {
             const int kb = static_cast<int>(ceil_div(kcols, 64));
             GemmArgs g = gemm_args(c, static_cast<int>(q), bw, kb, EPI_TRAIL);
-            set_prods(g, (frac || c.pl.grouped) ? 3 : 1);
+            if (h2) set_prods_h2(g, c, b0);   // integer changes: fp16 A, two fp16 planes of Sigma_bar^T
+            else set_prods(g, (frac || c.pl.grouped) ? 3 : 1);
             int S = choose_splits(ceil_div(q, 128), kb, g.n_prod, c.nsm);
             if (S > c.pl.smax) S = c.pl.smax;
             g.a_plane_rows = static_cast<int>(q);
@@ -486,8 +514,12 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
             g.split_stride = q * B;
             g.gate = gate;
             Timed tm(c.timer, QE_KERNEL_TRAIL_GEMM, c.s);
-            QE_CK(launch_tc_gemm(B, c.tm_dp, B == 64 ? c.tm_snt64 : (B == 128 ? c.tm_snt128 : c.tm_snt256), g,
-                                 S, c.s));
+            if (h2)
+                QE_CK(launch_tc_gemm(B, c.tm_dp16, B == 64 ? c.tm_snh64 : (B == 128 ? c.tm_snh128 : c.tm_snh256), g,
+                                     S, c.s));
+            else
+                QE_CK(launch_tc_gemm(B, c.tm_dp, B == 64 ? c.tm_snt64 : (B == 128 ? c.tm_snt128 : c.tm_snt256), g,
+                                     S, c.s));
             nsplit = S;
         }
         CdArgs a;
@@ -528,6 +560,7 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
         if (window != 0 && !frac) a.lent = c.lent;
         a.ldd = ld;
         a.dp_plane_rows = q;
+        a.dp_f16 = h2 ? 1 : 0;
         a.err = c.err;
         a.gate = gate;
         // relaxed sweeps and the sweep after one start from real values: no refinement

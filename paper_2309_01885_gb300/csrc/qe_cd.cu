@@ -4,6 +4,8 @@
 // the objective reduction, plus the fp32 SIMT Sigma and the bf16 transpose.
 #include "qe_common.cuh"
 #include "qe_internal.h"
+#include <cuda_fp16.h>
+
 #include "qe_kernels.h"
 
 namespace qe {
@@ -152,6 +154,48 @@ __global__ void __launch_bounds__(256) k_sigma_planes(const float *S, int64_t ld
     if (bad) set_error(err, ERR_NUMERIC);
 }
 
+// Sigma_bar^T in two fp16 planes for the CD GEMMs whose other operand is an
+// exact small integer (the changes Delta' of a window sweep, C - z of the
+// residual refresh): row j (Sigma_bar[:, j]) is scaled by a power of two 2^e_j
+// that brings its largest magnitude just under 2^15, then split as
+// hi = fp16(x), lo = fp16(x - hi): 22 significant bits (relative 2^-22) at one
+// product fewer than three bf16 planes; the GEMM epilogue multiplies output
+// column j by cscale[j] = 2^-e_j (exact).  x is the same binary32 value the bf16
+// planes and the fp32 rows hold.  One CTA per row j (grid-stride), two passes
+// over the row (its largest magnitude, then the planes).
+__global__ void __launch_bounds__(256) k_sigma_planes_h2(const float *S, int64_t lds, int64_t p, const float *d,
+                                                         __half *snh, int64_t ldn, float *cscale) {
+    __shared__ float red[8];
+    for (int64_t j = blockIdx.x; j < p; j += gridDim.x) {
+        const float dj = d[j];
+        const bool jalive = dj > 0.0f;
+        float mx = 0.0f;
+        for (int64_t k = threadIdx.x; k < p; k += blockDim.x)
+            if (jalive && k != j && d[k] > 0.0f) mx = fmaxf(mx, fabsf(__fdiv_rn(S[j * lds + k], dj)));
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+        if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = mx;
+        __syncthreads();
+        mx = 0.0f;
+        for (int w = 0; w < 8; ++w) mx = fmaxf(mx, red[w]);
+        __syncthreads();   // red is rewritten for the next row
+        // 2^e with mx 2^e in [2^14, 2^15) (finite mx; e = 0 for an all-zero row)
+        int e = 0;
+        if (mx > 0.0f && isfinite(mx)) e = 14 - ilogbf(mx);
+        if (e > 100) e = 100;
+        if (e < -100) e = -100;
+        if (threadIdx.x == 0) cscale[j] = ldexpf(1.0f, -e);
+        for (int64_t k = threadIdx.x; k < ldn; k += blockDim.x) {
+            float x = 0.0f;
+            if (k < p && jalive && k != j && d[k] > 0.0f) x = ldexpf(__fdiv_rn(S[j * lds + k], dj), e);
+            const __half hi = __float2half_rn(x);
+            const __half lo = __float2half_rn(x - __half2float(hi));
+            snh[j * ldn + k] = hi;
+            snh[(p + j) * ldn + k] = lo;
+        }
+    }
+}
+
 // Sigma_bar in fp32, row-major (row k, column j): Sigma_bar[k][j] =
 // Sigma[j][k] / d_j, the same binary32 value whose hi + mid + lo planes
 // k_sigma_planes writes (so the change-list correction and the tensor-core
@@ -266,8 +310,8 @@ __global__ void k_codes_to_qf(const uint8_t *codes, int64_t ldc, const float *sc
              j += (int64_t)gridDim.x * blockDim.x) {
             const int64_t gi = i * ng + j / gsize;
             const float cz = static_cast<float>(codes[i * ldc + j]) - zero[gi];
-            if (!grouped) {
-                qf[i * ldq + j] = __float2bfloat16_rn(cz);
+            if (!grouped) {   // exact in fp16: the residual GEMM takes fp16 operands
+                reinterpret_cast<__half *>(qf)[i * ldq + j] = __float2half_rn(cz);
             } else {
                 __nv_bfloat16 h, m, l;
                 split3(scale[gi] * cz, h, m, l);
@@ -497,8 +541,8 @@ __device__ __forceinline__ void cd_epilogue(const CdArgs &a, int64_t b0, int bw_
         } else if (!skip_same || dlt[h] != 0.0f) {
             a.codes[i * a.ldc + col] = static_cast<uint8_t>(code[h]);
             if (a.write_qf) {
-                if (!grouped) {
-                    a.qf[i * a.ldq + col] = __float2bfloat16_rn(code[h] - z);
+                if (!grouped) {   // exact in fp16: the residual GEMM takes fp16 operands
+                    reinterpret_cast<__half *>(a.qf)[i * a.ldq + col] = __float2half_rn(code[h] - z);
                 } else {   // the residual GEMM takes s_g (C - z_g), three planes
                     __nv_bfloat16 qh, qm, ql;
                     split3(sg * (code[h] - z), qh, qm, ql);
@@ -512,6 +556,10 @@ __device__ __forceinline__ void cd_epilogue(const CdArgs &a, int64_t b0, int bw_
         // grouped: the trailing GEMM sums changes of several groups, so it takes them
         // absolute (s_g Delta'), which is not an integer: three planes
         const float dv = grouped ? sg * dlt[h] : dlt[h];
+        if (a.dp_f16) {   // an integer change, exact in fp16, for the fp16 window GEMM
+            reinterpret_cast<__half *>(a.dp)[i * a.ldd + col] = __float2half_rn(dv);
+            continue;
+        }
         const __nv_bfloat16 hi = __float2bfloat16_rn(dv);
         a.dp[i * a.ldd + col] = hi;
         if (a.frac || grouped) {   // Delta' is not an integer: three planes
@@ -2050,6 +2098,13 @@ cudaError_t launch_sigma_norm(const float *S, int64_t lds, int64_t p, float *d, 
                               int64_t ldn, unsigned *err, cudaStream_t s) {
     k_sigma_diag<<<static_cast<unsigned>(ceil_div(p, 256)), 256, 0, s>>>(S, lds, p, d, err);
     k_sigma_planes<<<row_grid4(p, p), 256, 0, s>>>(S, lds, p, d, snt, ldn, err);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_sigma_planes_h2(const float *S, int64_t lds, int64_t p, const float *d, __half *snh, int64_t ldn,
+                                   float *cscale, cudaStream_t s) {
+    const int64_t g = p < 65535 ? p : 65535;
+    k_sigma_planes_h2<<<static_cast<unsigned>(g), 256, 0, s>>>(S, lds, p, d, snh, ldn, cscale);
     return cudaGetLastError();
 }
 

@@ -170,6 +170,13 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
            | (static_cast<uint32_t>(M >> 4) << 24);    // M >> 4
 }
 
+// Instruction descriptor, kind::f16 with fp16 A/B, fp32 D, both K-major.
+__host__ __device__ constexpr uint32_t idesc_f16_f32(int M, int N) {
+    return (1u << 4)                                   // D format: F32
+           | (static_cast<uint32_t>(N >> 3) << 17)     // N >> 3 (A, B format 0: F16)
+           | (static_cast<uint32_t>(M >> 4) << 24);    // M >> 4
+}
+
 __device__ __forceinline__ void mma_bf16_ss(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
                                             uint32_t idesc, uint32_t accumulate) {
     asm volatile(

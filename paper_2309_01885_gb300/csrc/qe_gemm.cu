@@ -293,6 +293,10 @@ __device__ __forceinline__ void epilogue_rows(const GemmArgs &g, float *stg, int
         const int64_t rw = r;
         float v[VEC];
         ld_fv<VEC>(stg + rr * LD + VEC * lane, v);
+        if (g.colscale) {
+#pragma unroll
+            for (int e = 0; e < VEC; ++e) v[e] *= (cl + e < g.N) ? g.colscale[cl + e] : 1.0f;
+        }
         if (g.mode == EPI_TRAIL) {
             float *orow = g.out + static_cast<int64_t>(split) * g.split_stride + rw * g.ldo;
             if (full) st_fv<VEC>(orow + cl, v);
@@ -477,7 +481,7 @@ __global__ void __launch_bounds__(320, 1)
     } else if (warp == 1) {
         if (lane == 0) {
             // ---- MMA issuer: chunk c accumulates into TMEM buffer c & 1 ----
-            constexpr uint32_t idesc = idesc_bf16_f32(C::BM, BN);
+            const uint32_t idesc = g.f16 ? idesc_f16_f32(C::BM, BN) : idesc_bf16_f32(C::BM, BN);
             int st = 0;
             for (int c = 0; c < nchunks && !*abort_flag; ++c) {
                 const int buf = c & 1;
@@ -556,6 +560,10 @@ __global__ void __launch_bounds__(320, 1)
                         float v[32];
 #pragma unroll
                         for (int i = 0; i < 32; ++i) v[i] = acc[q * 32 + i];
+                        if (g.colscale) {
+#pragma unroll
+                            for (int i = 0; i < 32; ++i) v[i] *= (c0 + i < g.N) ? g.colscale[c0 + i] : 1.0f;
+                        }
                         epilogue_row<GR>(g, r, c0, v, split, objacc);
                     }
                 }
@@ -604,6 +612,22 @@ bool make_tmap_bf16(CUtensorMap *map, const void *base, uint64_t rows, uint64_t 
     cuuint32_t estr[2] = {1, 1};
     const CUresult r =
         g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides,
+                 box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                 CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+bool make_tmap_f16(CUtensorMap *map, const void *base, uint64_t rows, uint64_t cols, uint64_t ld,
+                   uint32_t box_rows) {
+    if (!get_encode()) return false;
+    if ((reinterpret_cast<uintptr_t>(base) & 15u) != 0 || ((ld * 2) & 15u) != 0) return false;
+    if (rows == 0 || cols == 0 || box_rows == 0 || box_rows > 256) return false;
+    cuuint64_t dims[2] = {cols, rows};
+    cuuint64_t strides[1] = {ld * 2};
+    cuuint32_t box[2] = {64, box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    const CUresult r =
+        g_encode(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void *>(base), dims, strides,
                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;

@@ -55,6 +55,11 @@ struct GemmArgs {
     // adaptive sweep schedule enqueues both forms of a sweep and runs one)
     const int *gate;
     int gate_run;
+    // f16 = 1: both operands are fp16 (kind::f16 with f16 inputs) instead of bf16;
+    // colscale (EPI_TRAIL, EPI_RFULL; may be NULL): output column c of the window is
+    // multiplied by colscale[c] (a power of two undoing the B operand's row scaling)
+    int f16;
+    const float *colscale;
 };
 
 // The per-device error word that qe_sync_status reads and clears.
@@ -64,6 +69,9 @@ unsigned *device_error_word();
 // a box of 64 columns x box_rows rows and 128-byte swizzle.  false on failure.
 bool make_tmap_bf16(CUtensorMap *map, const void *base, uint64_t rows, uint64_t cols,
                     uint64_t ld, uint32_t box_rows);
+// The same for fp16 elements.
+bool make_tmap_f16(CUtensorMap *map, const void *base, uint64_t rows, uint64_t cols,
+                   uint64_t ld, uint32_t box_rows);
 
 // Launches the tcgen05 GEMM with BN in {64, 128, 256} output columns per CTA.
 // grid = (ceil(N / BN), ceil(M / 128), splits).

@@ -2,6 +2,7 @@
 #pragma once
 
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -48,6 +49,7 @@ struct CdArgs {
     int64_t ldq;
     __nv_bfloat16 *dp;              // out: Delta' hi plane (mid / lo planes dp_plane_rows apart), or NULL
     int64_t ldd, dp_plane_rows;
+    int dp_f16;                     // Delta' is an integer: one fp16 plane (the fp16 window GEMM)
     unsigned *err;
     // optional gate: the launch does its work only when *gate == gate_run (the
     // adaptive sweep schedule enqueues both forms of a sweep and runs one)
@@ -94,6 +96,10 @@ cudaError_t launch_grid(const void *W, int w_bf16, int64_t ldw, const float *H, 
                         cudaStream_t s);
 cudaError_t launch_sigma_norm(const float *S, int64_t lds, int64_t p, float *d, __nv_bfloat16 *snt,
                               int64_t ldn, unsigned *err, cudaStream_t s);
+// Sigma_bar^T in two fp16 planes (rows [0, p) hi, [p, 2p) lo; leading dimension ldn, zero-padded),
+// each row j scaled by a power of two; cscale[j] = the factor that undoes it.
+cudaError_t launch_sigma_planes_h2(const float *S, int64_t lds, int64_t p, const float *d, __half *snh, int64_t ldn,
+                                   float *cscale, cudaStream_t s);
 // fp32 Sigma_bar, row k = the coupling of column k to every column (ld columns, zero-padded).
 cudaError_t launch_sigma_bar_rows(const float *S, int64_t lds, int64_t p, const float *d, float *sbar,
                                   int64_t ld, cudaStream_t s);
@@ -114,7 +120,7 @@ cudaError_t launch_obj_step(double *rowdf, int64_t q, const double *prev, double
 cudaError_t launch_record_form(const int *flag, uint8_t *form, cudaStream_t s);
 cudaError_t launch_list_switch(const int *lcnt, int64_t n, int64_t below, unsigned long long *counter, int *flag,
                                cudaStream_t s);
-// C - z (one exact bf16 plane), or with grouped grids s_g (C - z_g) in three planes
+// C - z (one exact fp16 plane), or with grouped grids s_g (C - z_g) in three bf16 planes
 // (rows [0, q), [q, 2q), [2q, 3q)); gsize = p: per-row grids.
 cudaError_t launch_codes_to_qf(const uint8_t *codes, int64_t ldc, const float *scale, const float *zero,
                                int64_t q, int64_t p, int64_t gsize, int grouped, __nv_bfloat16 *qf,
