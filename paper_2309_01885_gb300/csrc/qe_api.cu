@@ -640,7 +640,7 @@ static int dense_sweeps(const qe_opts *o) {
 
 static int relax_period(const qe_opts *o) { return o ? o->relax_period : 0; }
 
-constexpr float kDefaultTieEps = 2e-5f;
+constexpr float kDefaultTieEps = 1e-5f;
 static float tie_eps(const qe_opts *o) {
     if (!o || o->tie_eps == 0.0f) return kDefaultTieEps;
     return o->tie_eps > 0.0f ? o->tie_eps : 0.0f;

@@ -1013,8 +1013,8 @@ __device__ __forceinline__ int chg_decide(const float *tri, const float *d_blk, 
 // double-float sums); a row whose decision was wrong decides again from the
 // block's start with that column forced to its exact code, noting only the
 // near-ties after it, and the check repeats.  A row checks its first kMaxEv notes
-// of a visit and forces at most kMaxForced decisions (at tie_eps = 2e-5 a
-// 256-column visit has one note in about forty).
+// of a visit and forces at most kMaxForced decisions (at tie_eps = 1e-5 a
+// 256-column visit has one note in about eighty).
 constexpr int kMaxEv = 8;      // near-tie notes per row and block visit
 constexpr int kMaxForced = 4;  // exact decisions forced per row and block visit
 
@@ -1209,11 +1209,26 @@ __global__ void __launch_bounds__(1024, 1) k_cd_block_chg(const __grid_constant_
         if (row_ok)
             chg_decide_rec<B, FULL>(tri, a.d + a.b0, a.bw, a.maxq, s * s, a.rowdf != nullptr, lane, t, st, code, dlt,
                                     dfacc, a.tie_eps, me.fj, me.fc, 0, -1, me.ev, &me.nev);
-#pragma unroll
-        for (int h = 0; h < CPL; ++h) {
-            cr[warp * B + 32 * h + lane] = code[h];
-            sr[warp * B + 32 * h + lane] = st[h];
+        // a row without notes is final: it writes its results now, without waiting
+        const bool noted = row_ok && me.nev > 0;
+        if (row_ok && !noted) {
+            if (a.rowdf) {
+                dfacc = warp_sum(dfacc);
+                if (lane == 0) a.rowdf[i] += dfacc;
+            }
+            if (a.lent)
+                cd_epilogue<B, FULL, true>(a, a.b0, a.bw, i, lane, code, dlt, true);
+            else
+                cd_epilogue<B, FULL, false>(a, a.b0, a.bw, i, lane, code, dlt, true);
         }
+        if (noted) {
+#pragma unroll
+            for (int h = 0; h < CPL; ++h) {
+                cr[warp * B + 32 * h + lane] = code[h];
+                sr[warp * B + 32 * h + lane] = st[h];
+            }
+        }
+        if (__syncthreads_count(noted && lane == 0) == 0) return;   // no notes in this CTA
         for (int round = 0; round <= kMaxForced; ++round) {
             __syncthreads();
             // check the notes, row by row, in order; the first wrong one stops its row's checks
@@ -1274,7 +1289,7 @@ __global__ void __launch_bounds__(1024, 1) k_cd_block_chg(const __grid_constant_
                 }
             }
         }
-        if (!row_ok) return;
+        if (!noted) return;   // written above
     } else {
         if (!cd_prologue<B, FULL>(a, tri, bar, i, row_ok, lane, t, st)) return;
         if (!row_ok) return;

@@ -306,7 +306,7 @@ def qe_quantize_layer(W: torch.Tensor, Sigma: torch.Tensor, bits: int, iters: in
     keeps beta~ unquantized; 0 = off); group_size: grouped grids (scales / zeros q x groups);
     record_forms: also return sweep_forms (uint8 per sweep: 0 sequential, 1 dense, 2 lists);
     wait_test: the failure-path test hook of qe_opts (a bounded device wait made to give up);
-    tie_eps: near-tie refinement threshold in grid steps (0 = default 2e-5, negative = off)."""
+    tie_eps: near-tie refinement threshold in grid steps (0 = default 1e-5, negative = off)."""
     q, p = W.shape
     dev = W.device
     codes = torch.empty(q, p, dtype=torch.uint8, device=dev)
