@@ -387,7 +387,16 @@ def layer_schedule(q, p, iters, forms, relax, dense_opt, adaptive, grouped, outl
             trail_flops += f
             # integer changes of a window sweep: one fp16 plane x two fp16 planes of Sigma_bar
             # (2 products); real-valued or grouped changes: three bf16 planes (6 products)
-            trail_exec += (2 if kind == "dense" and not grouped else 6) * f
+            # the first sweep's real changes scaled into two fp16 planes: 3 products
+            if grouped:
+                npr = 6
+            elif kind == "dense":
+                npr = 2
+            elif kind == "first":
+                npr = 3
+            else:
+                npr = 6
+            trail_exec += npr * f
     refreshes = (1 if plan[0][0] == "first" else 0) + extra
     # launches: set-up (grid, Sigma diagonal, Sigma_bar planes, 1/d, packed blocks,
     # Sigma_bar rows, [W planes], P, initial residual); sweep 1: nblk - 1 trailing GEMMs

@@ -12,6 +12,7 @@
 // qe_quantize_layer_outlier adds, per iteration (Algorithm 4 of Sec. 4.3):
 //   T = H + 2 eta d_j (R - What);  H = P_s(T);  P = P_W - H (I + Sigma_bar);
 //   R += P_new - P_old.
+#include <math.h>
 #include <stdio.h>
 #include <string.h>
 
@@ -321,7 +322,7 @@ static qe_status setup_ctx(Ctx &c, const Plan &pl, const qe_opts *o, cudaStream_
         !make_tmap_bf16(&c.tm_dp, c.dp, 3 * q, p, ld, 128) ||
         !make_tmap_f16(&c.tm_snh256, c.snh, 2 * p, p, ld, 256) || !make_tmap_f16(&c.tm_snh64, c.snh, 2 * p, p, ld, 64) ||
         !make_tmap_f16(&c.tm_snh128, c.snh, 2 * p, p, ld, 128) || !make_tmap_f16(&c.tm_qf16, c.qf, q, p, ld, 128) ||
-        !make_tmap_f16(&c.tm_dp16, c.dp, q, p, ld, 128))
+        !make_tmap_f16(&c.tm_dp16, c.dp, 2 * q, p, ld, 128))
         return QE_ERR_CUDA;
     return QE_OK;
 }
@@ -367,6 +368,21 @@ static void set_prods_h2(GemmArgs &g, const Ctx &c, int64_t col0) {
     g.prod_b[1] = 1;
     g.f16 = 1;
     g.colscale = c.cscale + col0;
+    g.ascale = 1.0f;
+}
+
+// A real A (the first sweep's changes, times 2^sh) in two fp16 planes times the two
+// fp16 planes of Sigma_bar^T: hi.hi, hi.lo, lo.hi (lo.lo is below 2^-22 relative).
+static void set_prods_h2r(GemmArgs &g, const Ctx &c, int64_t col0, int sh) {
+    static const int pa[3] = {0, 0, 1}, pb[3] = {0, 1, 0};
+    g.n_prod = 3;
+    for (int k = 0; k < 3; ++k) {
+        g.prod_a[k] = pa[k];
+        g.prod_b[k] = pb[k];
+    }
+    g.f16 = 1;
+    g.colscale = c.cscale + col0;
+    g.ascale = ldexpf(1.0f, -sh);
 }
 
 // Sigma -> d, Sigma_bar^T planes; W operand planes; P = W (I + Sigma_bar) into `Pout`.
@@ -493,8 +509,12 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
     const int64_t q = c.pl.q, p = c.pl.p, ld = c.pl.ld;
     const int B = c.pl.B;
     const bool frac = src != SRC_CODES || relax;
-    // window sweeps over integer changes run their trailing GEMMs in fp16
+    // window sweeps over integer changes run their trailing GEMMs in fp16; so does the
+    // first sweep from W, whose changes |a - c| <= 2^bits - 1 (a = W / s + z and the
+    // code both lie in [0, 2^bits - 1]) are scaled by 2^(14 - bits) into two fp16 planes
     const bool h2 = window != 0 && !frac && !c.pl.grouped;
+    const bool h2r = frac && src == SRC_W && !relax && !c.pl.grouped;
+    const int sh = 14 - bits;
     for (int64_t b0 = 0; b0 < p; b0 += B) {
         const int bw = static_cast<int>((p - b0) < B ? (p - b0) : B);
         const int64_t kcols = (window > 0) ? p : b0;
@@ -503,6 +523,7 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
             const int kb = static_cast<int>(ceil_div(kcols, 64));
             GemmArgs g = gemm_args(c, static_cast<int>(q), bw, kb, EPI_TRAIL);
             if (h2) set_prods_h2(g, c, b0);   // integer changes: fp16 A, two fp16 planes of Sigma_bar^T
+            else if (h2r) set_prods_h2r(g, c, b0, sh);
             else set_prods(g, (frac || c.pl.grouped) ? 3 : 1);
             int S = choose_splits(ceil_div(q, 128), kb, g.n_prod, c.nsm);
             if (S > c.pl.smax) S = c.pl.smax;
@@ -514,7 +535,7 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
             g.split_stride = q * B;
             g.gate = gate;
             Timed tm(c.timer, QE_KERNEL_TRAIL_GEMM, c.s);
-            if (h2)
+            if (h2 || h2r)
                 QE_CK(launch_tc_gemm(B, c.tm_dp16, B == 64 ? c.tm_snh64 : (B == 128 ? c.tm_snh128 : c.tm_snh256), g,
                                      S, c.s));
             else
@@ -560,7 +581,8 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
         if (window != 0 && !frac) a.lent = c.lent;
         a.ldd = ld;
         a.dp_plane_rows = q;
-        a.dp_f16 = h2 ? 1 : 0;
+        a.dp_f16 = h2 ? 1 : (h2r ? 2 : 0);
+        a.dp_scale = ldexpf(1.0f, sh);
         a.err = c.err;
         a.gate = gate;
         // relaxed sweeps and the sweep after one start from real values: no refinement

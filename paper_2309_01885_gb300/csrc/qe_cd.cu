@@ -556,8 +556,15 @@ __device__ __forceinline__ void cd_epilogue(const CdArgs &a, int64_t b0, int bw_
         // grouped: the trailing GEMM sums changes of several groups, so it takes them
         // absolute (s_g Delta'), which is not an integer: three planes
         const float dv = grouped ? sg * dlt[h] : dlt[h];
-        if (a.dp_f16) {   // an integer change, exact in fp16, for the fp16 window GEMM
+        if (a.dp_f16 == 1) {   // an integer change, exact in fp16, for the fp16 window GEMM
             reinterpret_cast<__half *>(a.dp)[i * a.ldd + col] = __float2half_rn(dv);
+            continue;
+        }
+        if (a.dp_f16 == 2) {   // a real change (first sweep), scaled by a power of two: fp16 hi / lo
+            const float x = dv * a.dp_scale;
+            const __half hi = __float2half_rn(x);
+            reinterpret_cast<__half *>(a.dp)[i * a.ldd + col] = hi;
+            reinterpret_cast<__half *>(a.dp)[(a.dp_plane_rows + i) * a.ldd + col] = __float2half_rn(x - __half2float(hi));
             continue;
         }
         const __nv_bfloat16 hi = __float2bfloat16_rn(dv);

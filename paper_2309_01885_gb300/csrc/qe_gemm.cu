@@ -295,7 +295,7 @@ __device__ __forceinline__ void epilogue_rows(const GemmArgs &g, float *stg, int
         ld_fv<VEC>(stg + rr * LD + VEC * lane, v);
         if (g.colscale) {
 #pragma unroll
-            for (int e = 0; e < VEC; ++e) v[e] *= (cl + e < g.N) ? g.colscale[cl + e] : 1.0f;
+            for (int e = 0; e < VEC; ++e) v[e] *= (cl + e < g.N) ? g.colscale[cl + e] * g.ascale : 1.0f;
         }
         if (g.mode == EPI_TRAIL) {
             float *orow = g.out + static_cast<int64_t>(split) * g.split_stride + rw * g.ldo;
@@ -562,7 +562,7 @@ __global__ void __launch_bounds__(320, 1)
                         for (int i = 0; i < 32; ++i) v[i] = acc[q * 32 + i];
                         if (g.colscale) {
 #pragma unroll
-                            for (int i = 0; i < 32; ++i) v[i] *= (c0 + i < g.N) ? g.colscale[c0 + i] : 1.0f;
+                            for (int i = 0; i < 32; ++i) v[i] *= (c0 + i < g.N) ? g.colscale[c0 + i] * g.ascale : 1.0f;
                         }
                         epilogue_row<GR>(g, r, c0, v, split, objacc);
                     }

@@ -60,6 +60,7 @@ struct GemmArgs {
     // multiplied by colscale[c] (a power of two undoing the B operand's row scaling)
     int f16;
     const float *colscale;
+    float ascale;             // with colscale: a further factor (a power of two) on every output
 };
 
 // The per-device error word that qe_sync_status reads and clears.

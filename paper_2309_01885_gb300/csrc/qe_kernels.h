@@ -49,7 +49,9 @@ struct CdArgs {
     int64_t ldq;
     __nv_bfloat16 *dp;              // out: Delta' hi plane (mid / lo planes dp_plane_rows apart), or NULL
     int64_t ldd, dp_plane_rows;
-    int dp_f16;                     // Delta' is an integer: one fp16 plane (the fp16 window GEMM)
+    int dp_f16;                     // 1: Delta' is an integer: one fp16 plane (the fp16 window GEMM);
+                                    // 2: real Delta' (first sweep) times dp_scale in two fp16 planes
+    float dp_scale;
     unsigned *err;
     // optional gate: the launch does its work only when *gate == gate_run (the
     // adaptive sweep schedule enqueues both forms of a sweep and runs one)
