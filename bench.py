@@ -609,9 +609,11 @@ def main():
     gemm_cd_ms = sum(timed[k][1] for k in kinds[:3]) / args.steps
     gemm_cd_launches = sum(timed[k][0] for k in kinds[:3]) // args.steps
     gemm_cd_alg = sum(2 * q * p * p * (1 + sc["refreshes"]) + sc["trail_flops"] for sc in sched)
-    # P: bf16 W x three bf16 planes (3 products); residual: C - z x two fp16 planes (2), grouped: 6
-    gemm_cd_exec = sum((3 + (6 if grouped else 2) * sc["refreshes"]) * 2 * qpad * ppad * kpad + sc["trail_exec"]
-                       for sc in sched)
+    # P: bf16 W as one fp16 plane x two fp16 planes (2 products), fp32 W in three bf16 planes x
+    # three (6); residual: C - z x two fp16 planes (2), grouped: 6
+    p_prods = 2 if cfg.w_dtype == torch.bfloat16 else 6
+    gemm_cd_exec = sum((p_prods + (6 if grouped else 2) * sc["refreshes"]) * 2 * qpad * ppad * kpad
+                       + sc["trail_exec"] for sc in sched)
     r_cd = roofline_tensor("CD sweep (all kernels of the quantize calls)", cd_alg, None, sum(cd_avg), None,
                            peak_tc, peak_src, None, "per-kernel traffic under the gemm and list entries",
                            cd_gemm={"kernel": "k_tc_gemm<256> P, residual, trailing corrections",
@@ -620,10 +622,10 @@ def main():
                                     "executed_tflops": gemm_cd_exec / (gemm_cd_ms / 1e3) / 1e12 if gemm_cd_ms else None,
                                     "frac_executed": (gemm_cd_exec / (gemm_cd_ms / 1e3) / 1e12 / peak_tc)
                                     if gemm_cd_ms else None},
-                           split_factor=("per algorithmic product: 2 fp16 products where one operand is an "
-                                         "exact small integer (window sweeps, residual refresh), 3 bf16 products "
-                                         "(P), 6 where both operands are real-valued (sweep 1); ceiling of the "
-                                         "algorithmic fraction about 1/2"))
+                           split_factor=("per algorithmic product: 2 fp16 products where one operand is exact in "
+                                         "fp16 (window sweeps' integer changes, C - z, bf16 W), 3 for the first "
+                                         "sweep's real changes, 6 bf16 products for relaxed sweeps and grouped "
+                                         "grids; ceiling of the algorithmic fraction about 1/2"))
     # (3) k_tc_gemm<256> over all its launches in a step (Sigma + the CD GEMMs)
     gemm_ms = sigma_avg + gemm_cd_ms
     tr, tr_note = traffic_record("k_tc_gemm_trail", cfg.name)

@@ -88,7 +88,7 @@ struct Plan {
     int B = kDefaultBlock, smax = 1;
     int64_t gsize = 0, ngroups = 1;   // grid columns per group (p: per row), groups per row
     bool grouped = false;
-    size_t snt = 0, snh = 0, cscale = 0, d = 0, dinv = 0, tri = 0, P = 0, R = 0, wpl = 0, qf = 0, dp = 0, part = 0, objp = 0,
+    size_t snt = 0, snh = 0, cscale = 0, wh = 0, rscale = 0, d = 0, dinv = 0, tri = 0, P = 0, R = 0, wpl = 0, qf = 0, dp = 0, part = 0, objp = 0,
            rowdf = 0, objbase = 0, sbar = 0, lcnt = 0, lent = 0, rowdft = 0, sw = 0;
     int64_t nblk = 0;
     size_t PW = 0, H = 0, T = 0, st = 0, cg = 0, ce = 0, sb = 0, eb = 0, y0 = 0, y1 = 0, lam = 0,
@@ -119,6 +119,8 @@ static Plan make_plan(int64_t q, int64_t p, int B, bool outlier, int wpl_planes,
     pl.snt = take(cur, static_cast<size_t>(3 * p) * pl.ld * 2);
     pl.snh = take(cur, static_cast<size_t>(2 * p) * pl.ld * 2);   // fp16 hi / lo, rows scaled by powers of two
     pl.cscale = take(cur, p * 4);
+    pl.wh = take(cur, qld * 2);     // bf16 W as one row-scaled fp16 plane (the P GEMM)
+    pl.rscale = take(cur, q * 4);
     pl.d = take(cur, p * 4);
     pl.dinv = take(cur, p * 4);
     pl.tri = take(cur, static_cast<size_t>(packed_diag_floats(p, B)) * 4);
@@ -210,8 +212,8 @@ struct Ctx {
     uint8_t *ws = nullptr;
     bool own = false;
     __nv_bfloat16 *snt = nullptr, *wpl = nullptr, *qf = nullptr, *dp = nullptr;
-    __half *snh = nullptr;
-    float *cscale = nullptr;
+    __half *snh = nullptr, *wh = nullptr;
+    float *cscale = nullptr, *rscale = nullptr;
     float *d = nullptr, *dinv = nullptr, *tri = nullptr, *P = nullptr, *R = nullptr, *part = nullptr;
     double *objp = nullptr, *rowdf = nullptr, *objbase = nullptr;
     float *sbar = nullptr;
@@ -273,6 +275,8 @@ static qe_status setup_ctx(Ctx &c, const Plan &pl, const qe_opts *o, cudaStream_
     c.snt = at<__nv_bfloat16>(w, pl.snt);
     c.snh = at<__half>(w, pl.snh);
     c.cscale = at<float>(w, pl.cscale);
+    c.wh = at<__half>(w, pl.wh);
+    c.rscale = at<float>(w, pl.rscale);
     c.d = at<float>(w, pl.d);
     c.dinv = at<float>(w, pl.dinv);
     c.tri = at<float>(w, pl.tri);
@@ -393,9 +397,12 @@ static qe_status prepare(Ctx &c, const void *W, int wbf16, int64_t ldw, const fl
     QE_CK(launch_pack_diag(c.snt, ld, p, c.pl.B, c.tri, c.s));
     QE_CK(launch_sigma_planes_h2(Sigma, p, p, c.d, c.snh, ld, c.cscale, c.s));
     if (c.sbar) QE_CK(launch_sigma_bar_rows(Sigma, p, p, c.d, c.sbar, ld, c.s));
-    const bool direct = wbf16 && ((reinterpret_cast<uintptr_t>(W) & 15u) == 0) && (ldw % 8 == 0);
-    if (direct) {
-        if (!make_tmap_bf16(&c.tm_wa, W, q, p, ldw, 128)) return QE_ERR_CUDA;
+    // bf16 W: one row-scaled fp16 plane against the two fp16 planes of Sigma_bar
+    // (2 products); fp32 W: three bf16 planes against three (6 products)
+    const bool h1 = wbf16 != 0;
+    if (h1) {
+        QE_CK(launch_w_plane_h1(W, ldw, q, p, c.wh, ld, c.rscale, c.s));
+        if (!make_tmap_f16(&c.tm_wa, c.wh, q, p, ld, 128)) return QE_ERR_CUDA;
         c.wa_planes = 1;
     } else {
         c.wa_planes = wbf16 ? 1 : 3;
@@ -404,7 +411,12 @@ static qe_status prepare(Ctx &c, const void *W, int wbf16, int64_t ldw, const fl
     }
     GemmArgs g = gemm_args(c, static_cast<int>(q), static_cast<int>(p), static_cast<int>(ceil_div(p, 64)),
                            EPI_PINIT);
-    set_prods(g, c.wa_planes);
+    if (h1) {
+        set_prods_h2(g, c, 0);
+        g.rowscale = c.rscale;
+    } else {
+        set_prods(g, c.wa_planes);
+    }
     g.m_fast = 1;
     g.a_plane_rows = static_cast<int>(q);
     g.b_plane_rows = static_cast<int>(p);
@@ -415,7 +427,7 @@ static qe_status prepare(Ctx &c, const void *W, int wbf16, int64_t ldw, const fl
     g.ldw = ldw;
     {
         Timed tm(c.timer, QE_KERNEL_PINIT_GEMM, c.s);
-        QE_CK(launch_tc_gemm(256, c.tm_wa, c.tm_snt256, g, 1, c.s));
+        QE_CK(launch_tc_gemm(256, c.tm_wa, h1 ? c.tm_snh256 : c.tm_snt256, g, 1, c.s));
     }
     return QE_OK;
 }

@@ -196,6 +196,42 @@ __global__ void __launch_bounds__(256) k_sigma_planes_h2(const float *S, int64_t
     }
 }
 
+// bf16 W as one fp16 plane for the P GEMM against the fp16 planes of Sigma_bar:
+// row i scaled by a power of two 2^e_i that brings its largest magnitude just
+// under 2^15 (bf16's 8 significant bits fit fp16's 11, so every entry above
+// 2^-14 of that maximum is exact); rscale[i] = 2^-e_i undoes it in the epilogue.
+// One CTA per row (grid-stride), columns [p, ld) zero.
+__global__ void __launch_bounds__(256) k_w_plane_h1(const __nv_bfloat16 *W, int64_t ldw, int64_t q, int64_t p,
+                                                    __half *wh, int64_t ld, float *rscale) {
+    __shared__ float red[8];
+    for (int64_t i = blockIdx.x; i < q; i += gridDim.x) {
+        float mx = 0.0f;
+        for (int64_t k = threadIdx.x; k < p; k += blockDim.x) mx = fmaxf(mx, fabsf(__bfloat162float(W[i * ldw + k])));
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+        if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = mx;
+        __syncthreads();
+        mx = 0.0f;
+        for (int w = 0; w < 8; ++w) mx = fmaxf(mx, red[w]);
+        __syncthreads();
+        int e = 0;
+        if (mx > 0.0f && isfinite(mx)) e = 14 - ilogbf(mx);
+        if (e > 100) e = 100;
+        if (e < -100) e = -100;
+        if (threadIdx.x == 0) rscale[i] = ldexpf(1.0f, -e);
+        for (int64_t k = threadIdx.x; k < ld; k += blockDim.x)
+            wh[i * ld + k] = __float2half_rn(k < p ? ldexpf(__bfloat162float(W[i * ldw + k]), e) : 0.0f);
+    }
+}
+
+cudaError_t launch_w_plane_h1(const void *W, int64_t ldw, int64_t q, int64_t p, __half *wh, int64_t ld, float *rscale,
+                              cudaStream_t s) {
+    const int64_t g = q < 65535 ? q : 65535;
+    k_w_plane_h1<<<static_cast<unsigned>(g), 256, 0, s>>>(static_cast<const __nv_bfloat16 *>(W), ldw, q, p, wh, ld,
+                                                          rscale);
+    return cudaGetLastError();
+}
+
 // Sigma_bar in fp32, row-major (row k, column j): Sigma_bar[k][j] =
 // Sigma[j][k] / d_j, the same binary32 value whose hi + mid + lo planes
 // k_sigma_planes writes (so the change-list correction and the tensor-core

@@ -297,6 +297,11 @@ __device__ __forceinline__ void epilogue_rows(const GemmArgs &g, float *stg, int
 #pragma unroll
             for (int e = 0; e < VEC; ++e) v[e] *= (cl + e < g.N) ? g.colscale[cl + e] * g.ascale : 1.0f;
         }
+        if (g.rowscale) {
+            const float rs = g.rowscale[rw];
+#pragma unroll
+            for (int e = 0; e < VEC; ++e) v[e] *= rs;
+        }
         if (g.mode == EPI_TRAIL) {
             float *orow = g.out + static_cast<int64_t>(split) * g.split_stride + rw * g.ldo;
             if (full) st_fv<VEC>(orow + cl, v);

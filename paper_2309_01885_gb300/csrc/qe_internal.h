@@ -61,6 +61,7 @@ struct GemmArgs {
     int f16;
     const float *colscale;
     float ascale;             // with colscale: a further factor (a power of two) on every output
+    const float *rowscale;    // EPI_PINIT (may be NULL): output row r is multiplied by rowscale[r]
 };
 
 // The per-device error word that qe_sync_status reads and clears.

@@ -102,6 +102,10 @@ cudaError_t launch_sigma_norm(const float *S, int64_t lds, int64_t p, float *d, 
 // each row j scaled by a power of two; cscale[j] = the factor that undoes it.
 cudaError_t launch_sigma_planes_h2(const float *S, int64_t lds, int64_t p, const float *d, __half *snh, int64_t ldn,
                                    float *cscale, cudaStream_t s);
+// bf16 W (q x p) as one fp16 plane (leading dimension ld), each row scaled by a power of two;
+// rscale[i] = the factor that undoes it.
+cudaError_t launch_w_plane_h1(const void *W, int64_t ldw, int64_t q, int64_t p, __half *wh, int64_t ld, float *rscale,
+                              cudaStream_t s);
 // fp32 Sigma_bar, row k = the coupling of column k to every column (ld columns, zero-padded).
 cudaError_t launch_sigma_bar_rows(const float *S, int64_t lds, int64_t p, const float *d, float *sbar,
                                   int64_t ld, cudaStream_t s);
