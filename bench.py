@@ -36,7 +36,7 @@ if ROOT not in sys.path:
 METRIC = ("layer quantize time; CD column-updates/s (q·p²/s) and Σ TFLOP/s vs roofline")
 UNIT = "q·p² column-updates/s"
 DEFAULT_CONFIG = "falcon180b_down_14848x59392"
-DTYPE = "bf16 products, fp32 accumulation (Σ: bf16 X; CD: fp32-accurate via 3 bf16 planes, binary32 decisions)"
+DTYPE = ("16-bit tensor-core products, fp32 accumulation (Σ: bf16 X x bf16 X; CD GEMMs fp32-accurate: Σ̄ in two row-scaled fp16 planes against operands exact in fp16, three bf16 planes otherwise; binary32 decisions, near-ties decided in double-float)")
 
 
 def max_over_ranks(x: float, device) -> float:
@@ -674,8 +674,12 @@ def main():
         # worth of buffers, or one whole-X copy per step) measured slower: the copied
         # bytes pass through L2 and evict the Sigma_bar rows those sweeps gather.  At
         # least four chunks per step, each at most 65536 tokens.
-        chunk = min(65536, max(8192, (n // 4) // 64 * 64))
-        staging = qe.sigma_host_staging(p, chunk, nbuf=max(2, -(-n // chunk)))
+        # fp32 X (the OPT-125m-sized layer) is copied whole and reduced on the device:
+        # the streamed form takes bf16 chunks only.
+        streamed = X.dtype == torch.bfloat16
+        chunk = min(65536, max(8192, (n // 4) // 64 * 64)) if streamed else n
+        staging = qe.sigma_host_staging(p, chunk, nbuf=max(2, -(-n // chunk))) if streamed else None
+        Xd = None if streamed else torch.empty_like(X)
         host_out = [dict(codes=torch.empty(q, p, dtype=torch.uint8).pin_memory(),
                          scales=torch.empty(q).pin_memory(), zeros=torch.empty(q).pin_memory(),
                          obj=torch.empty(cfg.iters, dtype=torch.float64).pin_memory())
@@ -683,7 +687,11 @@ def main():
 
         def e2e_step():
             Wd.copy_(Wh, non_blocking=True)
-            qe.qe_build_sigma_host(Xh, Sigma, staging, chunk)
+            if streamed:
+                qe.qe_build_sigma_host(Xh, Sigma, staging, chunk)
+            else:
+                Xd.copy_(Xh, non_blocking=True)
+                qe.qe_build_sigma(Xd, Sigma=Sigma)
             for k, b in enumerate(cfg.bits):
                 o = quantize(Wd, b)
                 for key in ("codes", "scales", "zeros", "obj"):
@@ -709,7 +717,7 @@ def main():
         result["e2e"] = {"value": job_throughput(units_per_step, world, e2e_ms), "unit": UNIT,
                          "ms_per_step": e2e_ms, "steps": e2e_steps, "h2d_bytes_per_step": h2d,
                          "d2h_bytes_per_step": d2h, "chunk_tokens": chunk}
-        del Xh, Wh, staging, host_out
+        del Xh, Wh, Xd, staging, host_out
 
     st = qe.qe_sync_status()
     if st != qe.QE_OK:
