@@ -199,7 +199,7 @@ class ClockSampler:
 # Committed DRAM-traffic figures (profiles/roofline_traffic.json): per kernel, the
 # bytes one launch moved in one ncu capture, keyed by a hash of the sources the
 # kernel is compiled from; null once those sources change.
-TRAFFIC_SOURCES = ("qe_api.cu", "qe_cd.cu", "qe_common.cuh", "qe_gemm.cu", "qe_internal.h", "qe_kernels.h")
+TRAFFIC_SOURCES = ("qe_api.cu", "qe_cd.cu", "qe_sweep.cuh", "qe_common.cuh", "qe_gemm.cu", "qe_internal.h", "qe_kernels.h")
 
 
 def traffic_sources_sha256() -> str:

@@ -2,8 +2,8 @@
 
     python -m paper_2309_01885_gb300.build        # or build_lib() from Python
 
-Each translation unit is compiled by its own nvcc process (in parallel) for
-sm_103a only, then linked into paper_2309_01885_gb300/_build/libqe.so with the
+Each translation unit is compiled by its own nvcc process (in parallel, the
+slowest first) for sm_103a only, then linked into paper_2309_01885_gb300/_build/libqe.so with the
 static CUDA runtime.  The driver API is reached through
 cudaGetDriverEntryPointByVersion, so the library has no link-time dependency on
 libcuda and loads on machines without a GPU driver.
@@ -21,7 +21,11 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 OUT_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(OUT_DIR, "libqe.so")
-SOURCES = ["qe_api.cu", "qe_gemm.cu", "qe_cd.cu", "qe_outlier.cu", "qe_noalloc.cu", "qe_stream.cu", "qe_pack.cu", "qe_select.cu"]
+# the sweep kernels' instantiations are spread over the qe_sweep_*.cu units (one
+# kernel family and block width each) so that no single unit holds up the build
+SOURCES = ["qe_sweep_seq256.cu", "qe_sweep_chg256.cu", "qe_sweep_rows256.cu", "qe_sweep_seq256r.cu",
+           "qe_sweep_chg.cu", "qe_sweep_rows.cu", "qe_sweep_seq.cu", "qe_gemm.cu", "qe_api.cu", "qe_cd.cu",
+           "qe_outlier.cu", "qe_noalloc.cu", "qe_stream.cu", "qe_pack.cu", "qe_select.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
               f"-I{os.path.join(ROOT, 'include')}", f"-I{CSRC}"]
