@@ -610,80 +610,103 @@ __device__ __forceinline__ int chg_decide(const float *tri, const float *d_blk, 
     for (int h = 0; h < CPL; ++h) code[h] = st[h];
     // dlt (= st - code, exact for these small integers) is formed once at the end, so
     // it holds no registers during the passes
-    int pos = 0;                                       // first column not yet final
     int nchg = 0;
-    while (pos < bw) {
-        int jstar = -1;
-        bool jtie = false;
-        // values of this lane's column in the word that holds the first change
-        // (captured with a compile-time h, so the arrays stay in registers)
-        float v = 0.0f, tv = 0.0f, cv = 0.0f, sv = 0.0f;
+    int pos = 0;                                       // first column not yet final
+    while (true) {
+        // Word by word (lane l of word h is column 32 h + l): a change alters only the
+        // columns after it, so once a word has no change left its decisions are final
+        // and the passes go on with the next word alone.  A near-tie column (refinement
+        // on) ends the scan; it is decided below and the scan resumes after it.
+        int jt = -1;
 #pragma unroll
         for (int h = 0; h < CPL; ++h) {
-            const int l = 32 * h + lane;
-            const bool active = l >= pos && (FULL || l < bw);
-            const float c = rintf(fminf(fmaxf(t[h], 0.0f), maxq));
-            const float dl = st[h] - c;
-            if (active) code[h] = c;
-            // within eps of a midpoint: |t - nearest level| within eps of 1/2 (a clamped
-            // t just beyond the end levels also passes; deciding it exactly is harmless)
-            const bool nt = tie && active && fabsf(fabsf(t[h] - c) - 0.5f) < eps;
-            const unsigned m = __ballot_sync(0xffffffffu, active && (dl != 0.0f || nt));
-            if (jstar < 0 && m != 0u) {
-                jstar = 32 * h + (__ffs(m) - 1);
-                if (TIE) jtie = tie && ((__ballot_sync(0xffffffffu, nt) >> (jstar & 31)) & 1u);
-                v = dl;
-                tv = t[h];
-                cv = c;
-                sv = st[h];
+            if (jt >= 0 || 32 * h + 31 < pos) continue;   // (warp-uniform)
+            const bool inb = FULL || 32 * h + lane < bw;
+            int lo = pos > 32 * h ? pos - 32 * h : 0;  // first lane of word h not yet final
+            while (true) {
+                const bool active = lane >= lo && inb;
+                const float c = rintf(fminf(fmaxf(t[h], 0.0f), maxq));
+                const float dl = st[h] - c;
+                if (active) code[h] = c;
+                // within eps of a midpoint: |t - nearest level| within eps of 1/2 (a clamped
+                // t just beyond the end levels also passes; deciding it exactly is harmless)
+                const bool nt = tie && active && fabsf(fabsf(t[h] - c) - 0.5f) < eps;
+                const unsigned m = __ballot_sync(0xffffffffu, active && (dl != 0.0f || nt));
+                if (m == 0u) break;
+                const int jl = __ffs(m) - 1;
+                const int jstar = 32 * h + jl;
+                if (TIE && ((__ballot_sync(0xffffffffu, nt) >> jl) & 1u)) {
+                    jt = jstar;
+                    break;
+                }
+                if (want_df && lane == jl) {
+                    const float dj = d_blk[jstar];
+                    if (dj > 0.0f) {
+                        const float e1 = c - t[h], e0 = st[h] - t[h];
+                        dfacc += static_cast<double>(dj * s2 * (e1 * e1 - e0 * e0));
+                    }
+                }
+                const float db = __shfl_sync(0xffffffffu, dl, jl);
+                // the change times its coupling row, added to the columns after it: the
+                // rest of this word and every later word
+                if (GROWS) {
+                    const float *row = grow + jstar * lds + lane;
+                    float rv[CPL];
+#pragma unroll
+                    for (int g = h; g < CPL; ++g)
+                        rv[g] = (FULL || 32 * g + lane < bw) && (g > h || lane > jl) ? __ldg(row + 32 * g) : 0.0f;
+                    if (lane > jl) t[h] = fmaf(db, rv[h], t[h]);
+#pragma unroll
+                    for (int g = h + 1; g < CPL; ++g) t[g] = fmaf(db, rv[g], t[g]);
+                } else {
+                    const float *row = tri + kPackPad + tri_off(B, jstar) - (jstar + 1);
+                    if (lane > jl) t[h] = fmaf(db, row[32 * h + lane], t[h]);
+#pragma unroll
+                    for (int g = h + 1; g < CPL; ++g) t[g] = fmaf(db, row[32 * g + lane], t[g]);
+                }
+                lo = jl + 1;
+                ++nchg;
             }
         }
-        if (jstar < 0) break;
-        if (TIE && jtie) {
-            // binary64 beta~ of column jstar: the block's columns from this warp's shared
-            // row (final before jstar, start after), the rest from global memory
+        if (!TIE || jt < 0) break;
+        // binary64 beta~ of the near-tie column jt: the block's columns from this warp's
+        // shared row (final before jt, start after), the rest from global memory
 #pragma unroll
-            for (int h = 0; h < CPL; ++h)
-                if (FULL || 32 * h + lane < bw) tie_blk[32 * h + lane] = (32 * h + lane < jstar) ? code[h] : st[h];
-            __syncwarp();
-            const double te = tie_beta(ax, i, b0, bw, jstar, lane, tie_blk);
-            __syncwarp();
-            const float ce = tie_code(te, maxq);
-            const float se = __shfl_sync(0xffffffffu, sv, jstar & 31);
-            const float de = se - ce;
+        for (int g = 0; g < CPL; ++g)
+            if (FULL || 32 * g + lane < bw) tie_blk[32 * g + lane] = (32 * g + lane < jt) ? code[g] : st[g];
+        __syncwarp();
+        const double te = tie_beta(ax, i, b0, bw, jt, lane, tie_blk);
+        __syncwarp();
+        const float ce = tie_code(te, maxq);
+        float se = 0.0f;
 #pragma unroll
-            for (int h = 0; h < CPL; ++h)
-                if (32 * h + lane == jstar) code[h] = ce;
-            if (de == 0.0f) {   // no change: the columns after it keep their provisional decisions
-                pos = jstar + 1;
-                continue;
-            }
-            v = de;
-            tv = static_cast<float>(te);
-            cv = ce;
-            sv = se;
-        }
-        if (want_df && lane == (jstar & 31)) {
-            const float dj = d_blk[jstar];
+        for (int g = 0; g < CPL; ++g)
+            if (g == (jt >> 5)) se = __shfl_sync(0xffffffffu, st[g], jt & 31);
+        const float de = se - ce;
+#pragma unroll
+        for (int g = 0; g < CPL; ++g)
+            if (32 * g + lane == jt) code[g] = ce;
+        pos = jt + 1;
+        if (de == 0.0f) continue;   // no change: the columns after it keep their provisional decisions
+        if (want_df && lane == (jt & 31)) {
+            const float dj = d_blk[jt];
             if (dj > 0.0f) {
-                const float e1 = cv - tv, e0 = sv - tv;
+                const float tv = static_cast<float>(te);
+                const float e1 = ce - tv, e0 = se - tv;
                 dfacc += static_cast<double>(dj * s2 * (e1 * e1 - e0 * e0));
             }
         }
-        const float db = __shfl_sync(0xffffffffu, v, jstar & 31);
         if (GROWS) {
-            const float *row = grow + jstar * lds + lane;
-            float rv[CPL];
+            const float *row = grow + jt * lds + lane;
 #pragma unroll
-            for (int g = 0; g < CPL; ++g) rv[g] = (FULL || 32 * g + lane < bw) ? __ldg(row + 32 * g) : 0.0f;
-#pragma unroll
-            for (int g = 0; g < CPL; ++g) t[g] = fmaf(db, rv[g], t[g]);
+            for (int g = 0; g < CPL; ++g)
+                if ((FULL || 32 * g + lane < bw) && 32 * g + lane > jt) t[g] = fmaf(de, __ldg(row + 32 * g), t[g]);
         } else {
-            const float *row = tri + kPackPad + tri_off(B, jstar) - (jstar + 1);
+            const float *row = tri + kPackPad + tri_off(B, jt) - (jt + 1);
 #pragma unroll
-            for (int g = 0; g < CPL; ++g) t[g] = fmaf(db, row[32 * g + lane], t[g]);
+            for (int g = 0; g < CPL; ++g)
+                if (32 * g + lane > jt) t[g] = fmaf(de, row[32 * g + lane], t[g]);
         }
-        pos = jstar + 1;
         ++nchg;
     }
 #pragma unroll
@@ -719,14 +742,14 @@ __device__ __forceinline__ void chg_decide_rec(const float *tri, const float *d_
     const int bw = FULL ? B : bw_;
 #pragma unroll
     for (int h = 0; h < CPL; ++h) code[h] = st[h];
-    int pos = 0;
-    while (pos < bw) {
-        int jstar = -1;
-        float v = 0.0f, tv = 0.0f, cv = 0.0f, sv = 0.0f;
+    // word by word, as in chg_decide: a finished word's decisions are final
 #pragma unroll
-        for (int h = 0; h < CPL; ++h) {
-            const int l = 32 * h + lane;
-            const bool active = l >= pos && (FULL || l < bw);
+    for (int h = 0; h < CPL; ++h) {
+        const int l = 32 * h + lane;
+        const bool inb = FULL || l < bw;
+        int lo = 0;
+        while (true) {
+            const bool active = lane >= lo && inb;
             float c = rintf(fminf(fmaxf(t[h], 0.0f), maxq));
             if (nf > 0)
                 for (int f = 0; f < nf; ++f)
@@ -734,28 +757,23 @@ __device__ __forceinline__ void chg_decide_rec(const float *tri, const float *d_
             const float dl = st[h] - c;
             if (active) code[h] = c;
             const unsigned m = __ballot_sync(0xffffffffu, active && dl != 0.0f);
-            if (jstar < 0 && m != 0u) {
-                jstar = 32 * h + (__ffs(m) - 1);
-                v = dl;
-                tv = t[h];
-                cv = c;
-                sv = st[h];
+            if (m == 0u) break;
+            const int jl = __ffs(m) - 1;
+            const int jstar = 32 * h + jl;
+            if (want_df && lane == jl) {
+                const float dj = d_blk[jstar];
+                if (dj > 0.0f) {
+                    const float e1 = c - t[h], e0 = st[h] - t[h];
+                    dfacc += static_cast<double>(dj * s2 * (e1 * e1 - e0 * e0));
+                }
             }
-        }
-        if (jstar < 0) break;
-        if (want_df && lane == (jstar & 31)) {
-            const float dj = d_blk[jstar];
-            if (dj > 0.0f) {
-                const float e1 = cv - tv, e0 = sv - tv;
-                dfacc += static_cast<double>(dj * s2 * (e1 * e1 - e0 * e0));
-            }
-        }
-        const float db = __shfl_sync(0xffffffffu, v, jstar & 31);
-        const float *row = tri + kPackPad + tri_off(B, jstar) - (jstar + 1);
+            const float db = __shfl_sync(0xffffffffu, dl, jl);
+            const float *row = tri + kPackPad + tri_off(B, jstar) - (jstar + 1);
+            if (lane > jl) t[h] = fmaf(db, row[32 * h + lane], t[h]);
 #pragma unroll
-        for (int g = 0; g < CPL; ++g)
-            if (32 * g + lane > jstar) t[g] = fmaf(db, row[32 * g + lane], t[g]);
-        pos = jstar + 1;
+            for (int g = h + 1; g < CPL; ++g) t[g] = fmaf(db, row[32 * g + lane], t[g]);
+            lo = jl + 1;
+        }
     }
     // the notes: every column's t is the one it was decided on
 #pragma unroll

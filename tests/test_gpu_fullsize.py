@@ -154,7 +154,9 @@ def test_fullsize_layer_sampled_rows(name, nrows):
         cascades = [dict(row=int(rows[r]), sweep=t + 1, column=j, midpoint_dist=dist, codes_differing=nd)
                     for r, t, j, dist, nd in div]
         f = _objective_full(W, out["codes"], out["scales"], out["zeros"], Sg)
-        _log(dict(test="fullsize", workload=name, bits=bits, rows=int(rows.size), code_match=m,
+        # fraction of the sampled codes that changed in each sweep after the first
+        chg = [float(np.mean(sweep[t] != sweep[t - 1])) for t in range(1, sweep.shape[0])]
+        _log(dict(test="fullsize", workload=name, bits=bits, rows=int(rows.size), code_match=m, changed=chg,
                   obj_rel_err=float(np.max(np.abs(obj_rows.sum(axis=1) - ref["obj"]) / ref["obj"])),
                   full_obj_rel_err=abs(obj[-1] - f) / f, sweep_forms=forms, cascades=cascades))
         assert m >= parity.CODE_MATCH, f"codes match {m:.5f} on {rows.size} rows; cascades {cascades}"
