@@ -668,46 +668,50 @@ __device__ __forceinline__ int chg_decide(const float *tri, const float *d_blk, 
                 ++nchg;
             }
         }
-        if (!TIE || jt < 0) break;
-        // binary64 beta~ of the near-tie column jt: the block's columns from this warp's
-        // shared row (final before jt, start after), the rest from global memory
-#pragma unroll
-        for (int g = 0; g < CPL; ++g)
-            if (FULL || 32 * g + lane < bw) tie_blk[32 * g + lane] = (32 * g + lane < jt) ? code[g] : st[g];
-        __syncwarp();
-        const double te = tie_beta(ax, i, b0, bw, jt, lane, tie_blk);
-        __syncwarp();
-        const float ce = tie_code(te, maxq);
-        float se = 0.0f;
-#pragma unroll
-        for (int g = 0; g < CPL; ++g)
-            if (g == (jt >> 5)) se = __shfl_sync(0xffffffffu, st[g], jt & 31);
-        const float de = se - ce;
-#pragma unroll
-        for (int g = 0; g < CPL; ++g)
-            if (32 * g + lane == jt) code[g] = ce;
-        pos = jt + 1;
-        if (de == 0.0f) continue;   // no change: the columns after it keep their provisional decisions
-        if (want_df && lane == (jt & 31)) {
-            const float dj = d_blk[jt];
-            if (dj > 0.0f) {
-                const float tv = static_cast<float>(te);
-                const float e1 = ce - tv, e0 = se - tv;
-                dfacc += static_cast<double>(dj * s2 * (e1 * e1 - e0 * e0));
-            }
-        }
-        if (GROWS) {
-            const float *row = grow + jt * lds + lane;
-#pragma unroll
-            for (int g = 0; g < CPL; ++g)
-                if ((FULL || 32 * g + lane < bw) && 32 * g + lane > jt) t[g] = fmaf(de, __ldg(row + 32 * g), t[g]);
+        if constexpr (!TIE) {
+            break;
         } else {
-            const float *row = tri + kPackPad + tri_off(B, jt) - (jt + 1);
+            if (jt < 0) break;
+            // binary64 beta~ of the near-tie column jt: the block's columns from this warp's
+            // shared row (final before jt, start after), the rest from global memory
 #pragma unroll
             for (int g = 0; g < CPL; ++g)
-                if (32 * g + lane > jt) t[g] = fmaf(de, row[32 * g + lane], t[g]);
+                if (FULL || 32 * g + lane < bw) tie_blk[32 * g + lane] = (32 * g + lane < jt) ? code[g] : st[g];
+            __syncwarp();
+            const double te = tie_beta(ax, i, b0, bw, jt, lane, tie_blk);
+            __syncwarp();
+            const float ce = tie_code(te, maxq);
+            float se = 0.0f;
+#pragma unroll
+            for (int g = 0; g < CPL; ++g)
+                if (g == (jt >> 5)) se = __shfl_sync(0xffffffffu, st[g], jt & 31);
+            const float de = se - ce;
+#pragma unroll
+            for (int g = 0; g < CPL; ++g)
+                if (32 * g + lane == jt) code[g] = ce;
+            pos = jt + 1;
+            if (de == 0.0f) continue;   // no change: the columns after it keep their provisional decisions
+            if (want_df && lane == (jt & 31)) {
+                const float dj = d_blk[jt];
+                if (dj > 0.0f) {
+                    const float tv = static_cast<float>(te);
+                    const float e1 = ce - tv, e0 = se - tv;
+                    dfacc += static_cast<double>(dj * s2 * (e1 * e1 - e0 * e0));
+                }
+            }
+            if (GROWS) {
+                const float *row = grow + jt * lds + lane;
+#pragma unroll
+                for (int g = 0; g < CPL; ++g)
+                    if ((FULL || 32 * g + lane < bw) && 32 * g + lane > jt) t[g] = fmaf(de, __ldg(row + 32 * g), t[g]);
+            } else {
+                const float *row = tri + kPackPad + tri_off(B, jt) - (jt + 1);
+#pragma unroll
+                for (int g = 0; g < CPL; ++g)
+                    if (32 * g + lane > jt) t[g] = fmaf(de, row[32 * g + lane], t[g]);
+            }
+            ++nchg;
         }
-        ++nchg;
     }
 #pragma unroll
     for (int h = 0; h < CPL; ++h) dlt[h] = st[h] - code[h];
