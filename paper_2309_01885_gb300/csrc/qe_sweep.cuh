@@ -335,6 +335,29 @@ __device__ __forceinline__ void df_term(float &hi, float &lo, float t, float hs,
     lo = __fsub_rn(s2, __fsub_rn(hi, s1));
 }
 
+// Pull toward L2 what an exact recompute of beta~ for row i reads (the row's codes,
+// weights and H; Sigma's row jg): every line at once, from `nth` threads of which
+// this is number `tid`.  Prefetches hold no register, so a recompute that comes
+// later waits on L2 rather than on DRAM.
+__device__ __forceinline__ void tie_prefetch_row(const CdArgs &a, int64_t i, int tid, int nth) {
+    const uint8_t *crow = a.codes + i * a.ldc;
+    for (int64_t k = 128 * static_cast<int64_t>(tid); k < a.p; k += 128 * static_cast<int64_t>(nth)) prefetch_l2(crow + k);
+    if (a.w_bf16) {
+        const __nv_bfloat16 *w = static_cast<const __nv_bfloat16 *>(a.W) + i * a.ldw;
+        for (int64_t k = 64 * static_cast<int64_t>(tid); k < a.p; k += 64 * static_cast<int64_t>(nth)) prefetch_l2(w + k);
+    } else {
+        const float *w = static_cast<const float *>(a.W) + i * a.ldw;
+        for (int64_t k = 32 * static_cast<int64_t>(tid); k < a.p; k += 32 * static_cast<int64_t>(nth)) prefetch_l2(w + k);
+    }
+    if (a.Hd)
+        for (int64_t k = 32 * static_cast<int64_t>(tid); k < a.p; k += 32 * static_cast<int64_t>(nth))
+            prefetch_l2(a.Hd + i * a.ldh + k);
+}
+__device__ __forceinline__ void tie_prefetch_srow(const CdArgs &a, int64_t jg, int tid, int nth) {
+    const float *Srow = a.S + jg * a.lds_full;
+    for (int64_t k = 32 * static_cast<int64_t>(tid); k < a.p; k += 32 * static_cast<int64_t>(nth)) prefetch_l2(Srow + k);
+}
+
 __device__ __forceinline__ double tie_beta(const CdArgs *ap, int64_t i, int64_t b0, int bw, int j, int lane,
                                         const float *blk) {
     const CdArgs &a = *ap;
@@ -930,6 +953,10 @@ __global__ void __launch_bounds__(1024, 1) k_cd_block_chg(const __grid_constant_
                 cd_epilogue<B, FULL, false>(a, a.b0, a.bw, i, lane, code, dlt, true);
         }
         if (noted) {
+            // what the CTA-wide check reads starts toward L2 while the other rows decide
+            tie_prefetch_row(a, i, lane, 32);
+            const int ne = me.nev < kMaxEv ? me.nev : kMaxEv;
+            for (int e = 0; e < ne; ++e) tie_prefetch_srow(a, a.b0 + me.ev[e], lane, 32);
 #pragma unroll
             for (int h = 0; h < CPL; ++h) {
                 cr[warp * B + 32 * h + lane] = code[h];
@@ -990,6 +1017,8 @@ __global__ void __launch_bounds__(1024, 1) k_cd_block_chg(const __grid_constant_
                                         dlt, dfacc, a.tie_eps, me.fj, me.fc, me.nf, wj, me.ev, &me.nev);
                 if (round == kMaxForced && lane == 0) me.nev = 0;
                 __syncwarp();
+                const int ne = me.nev < kMaxEv ? me.nev : kMaxEv;
+                for (int e = 0; e < ne; ++e) tie_prefetch_srow(a, a.b0 + me.ev[e], lane, 32);
 #pragma unroll
                 for (int h = 0; h < CPL; ++h) {
                     cr[warp * B + 32 * h + lane] = code[h];
