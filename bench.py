@@ -402,10 +402,11 @@ def layer_schedule(q, p, iters, forms, relax, dense_opt, adaptive, grouped, outl
     # Sigma_bar rows, [W planes], P, initial residual); sweep 1: nblk - 1 trailing GEMMs
     # + nblk in-block + residual GEMM + objective sum; a dense or sequential sweep:
     # trailing GEMMs (nblk - 1 when its window starts empty) + nblk in-block + objective
-    # step; fixed schedule: one list launch and one objective prefix per run of <= 32
-    # list sweeps; adaptive schedule: every sweep after the first enqueues both forms
-    # (trailing GEMMs, in-block, objective step, list launch, objective prefix) and all
-    # but the last the two switch kernels; an extra refresh: C - z + residual GEMM
+    # step, a dense one also nblk near-tie checks; fixed schedule: one list launch and
+    # one objective prefix per run of <= 32 list sweeps; adaptive schedule: every sweep
+    # after the first enqueues both forms (trailing GEMMs, in-block, near-tie checks,
+    # objective step, list launch, objective prefix) and all but the last the two switch
+    # kernels; an extra refresh: C - z + residual GEMM
     per = 8 + w_planes + 2 * extra
     if outlier:
         # selection (P_s: 3 radix digit passes + count, scan, emit; columns: + 2 norm
@@ -420,14 +421,14 @@ def layer_schedule(q, p, iters, forms, relax, dense_opt, adaptive, grouped, outl
     elif adaptive:
         per += (nblk - 1) + nblk + 2
         for t in range(1, iters):
-            per += (nblk - (1 if t == 1 else 0)) + nblk + 3 + (2 if t + 1 < iters else 0)
+            per += (nblk - (1 if t == 1 else 0)) + 2 * nblk + 3 + (2 if t + 1 < iters else 0)
     else:
         per += 2 * len(list_runs)
         for kind, window in plan:
             if kind == "first":
                 per += (nblk - 1) + nblk + 2
             elif kind in ("seq", "dense"):
-                per += (nblk if window == 1 else nblk - 1) + nblk + 1
+                per += (nblk if window == 1 else nblk - 1) + nblk + 1 + (nblk if kind == "dense" else 0)
     counts = {k: sum(1 for kd, _ in plan if kd == k) for k in ("first", "seq", "dense", "list")}
     return dict(trail_flops=trail_flops, trail_exec=trail_exec, refreshes=refreshes, launches=per,
                 sweeps_by_form=counts, plan=plan)

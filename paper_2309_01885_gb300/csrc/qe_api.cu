@@ -89,7 +89,7 @@ struct Plan {
     int64_t gsize = 0, ngroups = 1;   // grid columns per group (p: per row), groups per row
     bool grouped = false;
     size_t snt = 0, snh = 0, cscale = 0, wh = 0, rscale = 0, d = 0, dinv = 0, tri = 0, P = 0, R = 0, wpl = 0, qf = 0, dp = 0, part = 0, objp = 0,
-           rowdf = 0, objbase = 0, sbar = 0, lcnt = 0, lent = 0, rowdft = 0, sw = 0;
+           rowdf = 0, objbase = 0, sbar = 0, lcnt = 0, lent = 0, rowdft = 0, sw = 0, tq = 0, tqrows = 0, tqcnt = 0;
     int64_t nblk = 0;
     size_t PW = 0, H = 0, T = 0, st = 0, cg = 0, ce = 0, sb = 0, eb = 0, y0 = 0, y1 = 0, lam = 0,
            eta = 0, rowptr = 0, cpart = 0, cnorm = 0, ccols = 0, cval = 0, cn = 0, ppart = 0;
@@ -141,6 +141,10 @@ static Plan make_plan(int64_t q, int64_t p, int B, bool outlier, int wpl_planes,
         pl.rowdft = take(cur, static_cast<size_t>(q) * kSweepChunk * 8);
         pl.sw = take(cur, 16);   // adaptive schedule: switch flag (int) and change counter (u64)
     }
+    // the change-driven kernel's near-tie queue: an entry and two rows of B floats per row
+    pl.tq = take(cur, static_cast<size_t>(q) * sizeof(TieEntry));
+    pl.tqrows = take(cur, static_cast<size_t>(q) * 2 * B * 4);
+    pl.tqcnt = take(cur, 16);
     if (outlier) {
         const int64_t N = q * p;
         const int64_t nch = topk_chunks(N);
@@ -222,6 +226,9 @@ struct Ctx {
     double *rowdft = nullptr;
     int *swflag = nullptr;
     unsigned long long *swcount = nullptr;
+    TieEntry *tq = nullptr;
+    float *tqrows = nullptr;
+    unsigned *tqcnt = nullptr;
     float *PW = nullptr, *H = nullptr, *T = nullptr, *y0 = nullptr, *y1 = nullptr;
     TopkState *st = nullptr;
     unsigned *cg = nullptr, *ce = nullptr, *sb = nullptr, *eb = nullptr;
@@ -296,6 +303,15 @@ static qe_status setup_ctx(Ctx &c, const Plan &pl, const qe_opts *o, cudaStream_
         c.rowdft = at<double>(w, pl.rowdft);
         c.swflag = at<int>(w, pl.sw);
         c.swcount = at<unsigned long long>(w, pl.sw + 8);
+    }
+    c.tq = at<TieEntry>(w, pl.tq);
+    c.tqrows = at<float>(w, pl.tqrows);
+    c.tqcnt = at<unsigned>(w, pl.tqcnt);
+    // the queue's counters start at zero (every check launch leaves them so; this
+    // clears what an aborted call left)
+    if (cudaMemsetAsync(c.tqcnt, 0, 16, s) != cudaSuccess) {
+        cudaGetLastError();
+        return QE_ERR_CUDA;
     }
     if (pl.PW) {
         c.PW = at<float>(w, pl.PW);
@@ -597,6 +613,9 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
         a.dp_scale = ldexpf(1.0f, sh);
         a.err = c.err;
         a.gate = gate;
+        a.tq = c.tq;
+        a.tq_rows = c.tqrows;
+        a.tq_cnt = c.tqcnt;
         // relaxed sweeps and the sweep after one start from real values: no refinement
         set_tie(c, a, !relax && src != SRC_V);
         if (wait_test) {   // the failure-path test hook: the first block waits for a copy never issued
@@ -607,6 +626,8 @@ static qe_status sweep(Ctx &c, uint8_t *codes, const float *scales, const float 
         }
         Timed tm(c.timer, QE_KERNEL_CD_BLOCK, c.s);
         QE_CK(launch_cd_block(B, a, c.nsm, c.s));
+        // the change-driven kernel with the refinement leaves its noted rows to the check
+        if (!frac && a.tie_eps > 0.0f) QE_CK(launch_cd_tie_check(B, a, c.nsm, c.s));
     }
     return QE_OK;
 }

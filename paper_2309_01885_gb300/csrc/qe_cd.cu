@@ -404,6 +404,16 @@ static cudaError_t launch_cd_block_w(const CdArgs &a, int nsm, cudaStream_t s) {
     return full ? launch_cd_block_k<B, false, true>(a, nsm, s) : launch_cd_block_k<B, false, false>(a, nsm, s);
 }
 
+cudaError_t launch_cd_tie_check(int B, const CdArgs &a, int nsm, cudaStream_t s) {
+    const bool full = a.bw == B;
+    switch (B) {
+        case 64: return full ? launch_cd_tie_check_k<64, true>(a, nsm, s) : launch_cd_tie_check_k<64, false>(a, nsm, s);
+        case 128: return full ? launch_cd_tie_check_k<128, true>(a, nsm, s) : launch_cd_tie_check_k<128, false>(a, nsm, s);
+        case 256: return full ? launch_cd_tie_check_k<256, true>(a, nsm, s) : launch_cd_tie_check_k<256, false>(a, nsm, s);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
 cudaError_t launch_cd_block(int B, const CdArgs &a, int nsm, cudaStream_t s) {
     switch (B) {
         case 64: return launch_cd_block_w<64>(a, nsm, s);

@@ -75,6 +75,22 @@ struct CdArgs {
     int64_t ldw;
     const float *Hd;                // outlier variant: dense H (target W - H, leading dimension ldh), or NULL
     int64_t ldh;
+    // change-driven kernel with the refinement: rows with near-tie notes go to this
+    // queue (entries, then two B-float rows per entry: final and start codes) and are
+    // finished by the check kernel; tq_cnt[0] counts entries, tq_cnt[1] check CTAs done
+    // (both zero between launches: the check kernel's last CTA resets them)
+    struct TieEntry *tq;
+    float *tq_rows;
+    unsigned *tq_cnt;
+};
+
+// One queued row of the change-driven kernel's near-tie check.
+struct TieEntry {
+    int64_t i;              // the row
+    double df;              // its objective change (warp-summed)
+    int nev;                // notes (columns within tie_eps of a midpoint), ev[0 .. min(nev, 8))
+    int ev[8];
+    int pad[3];
 };
 
 // Objective / reference-norm reduction.
@@ -132,6 +148,10 @@ cudaError_t launch_codes_to_qf(const uint8_t *codes, int64_t ldc, const float *s
                                int64_t q, int64_t p, int64_t gsize, int grouped, __nv_bfloat16 *qf,
                                int64_t ldq, cudaStream_t s);
 cudaError_t launch_cd_block(int B, const CdArgs &a, int nsm, cudaStream_t s);
+// The near-tie check after a change-driven launch with the refinement (a.tq set):
+// every queued row's notes against beta~ recomputed exactly, a row with a wrong
+// decision decided again, and the queued rows' results written.
+cudaError_t launch_cd_tie_check(int B, const CdArgs &a, int nsm, cudaStream_t s);
 // Sweeps [t_begin, t_end) with the change-list correction in one persistent launch
 // (a.sbar, a.lcnt, a.lent set; a.b0 / a.bw / a.part unused); the objective change of
 // sweep t and row i goes to rowdf_t[(t - t_begin) q + i]; sweep_codes (optional) gets

@@ -887,7 +887,7 @@ __device__ __forceinline__ double coop_tie_beta(const CdArgs &a, int64_t i, int6
     return red[32];
 }
 
-// Shared memory of the refinement variant after the packed block, per warp.
+// Notes of one warp's row in shared memory (the refinement variants).
 struct TieWarp {
     int ev[kMaxEv];
     int fj[kMaxForced];
@@ -895,16 +895,23 @@ struct TieWarp {
     int nev, nf, wrong_j;
     float wrong_c;
 };
+static_assert(kMaxEv == 8, "TieEntry holds 8 notes");
 
-template <int B>
-__host__ __device__ constexpr int tie_cta_bytes(int warps) {
-    return warps * (2 * B * 4 + static_cast<int>(sizeof(TieWarp))) + 34 * 8;
+template <int B, bool FULL>
+__device__ __forceinline__ void chg_write(const CdArgs &a, int64_t i, int lane, const float (&code)[B / 32],
+                                          const float (&dlt)[B / 32]) {
+    if (a.lent)
+        cd_epilogue<B, FULL, true>(a, a.b0, a.bw, i, lane, code, dlt, true);
+    else
+        cd_epilogue<B, FULL, false>(a, a.b0, a.bw, i, lane, code, dlt, true);
 }
 
 // Change-driven in-block kernel (every sweep after the first), exactly
 // equivalent to the sequential order: a column whose code does not change
 // alters no other column, so the cost is (number of changed columns + 1)
-// data-parallel passes (chg_decide).
+// data-parallel passes (chg_decide).  With the refinement (TIE) the decisions
+// are binary32 with notes of the near ties; a row without notes writes its
+// results, a row with notes goes to the queue that k_cd_tie_check finishes.
 template <int B, bool FULL, bool TIE = false>
 __global__ void __launch_bounds__(1024, 1) k_cd_block_chg(const __grid_constant__ CdArgs a) {
     if (a.gate && *a.gate != a.gate_run) return;   // uniform: the list form of the sweep runs
@@ -919,128 +926,208 @@ __global__ void __launch_bounds__(1024, 1) k_cd_block_chg(const __grid_constant_
     float t[CPL], st[CPL];
     float code[CPL], dlt[CPL];
     double dfacc = 0.0;
+    if (!cd_prologue<B, FULL>(a, tri, bar, i, row_ok, lane, t, st)) return;
+    if (!row_ok) return;
+    const float s = a.scale[i * a.ngroups + a.b0 / a.gsize];
     if constexpr (TIE) {
-        // refinement variant: binary32 decisions with notes, checked CTA-wide
-        const int nw = static_cast<int>(blockDim.x >> 5);
-        float *cr = cd_smem + C::PACK + 4;                  // [nw][B] final codes
-        float *sr = cr + nw * B;                            // [nw][B] start codes
-        TieWarp *tw = reinterpret_cast<TieWarp *>(sr + nw * B);
-        double *red = reinterpret_cast<double *>(tw + nw);
-        const bool ok = cd_prologue<B, FULL>(a, tri, bar, i, row_ok, lane, t, st);
-        if (__syncthreads_or(!ok)) return;   // a wait gave up somewhere: every warp leaves
-        const int bw = FULL ? B : a.bw;
-        const float s = row_ok ? a.scale[i * a.ngroups + a.b0 / a.gsize] : 1.0f;
-        TieWarp &me = tw[warp];
-        if (lane == 0) {
-            me.nev = 0;
-            me.nf = 0;
-            me.wrong_j = -1;
-        }
+        TieWarp &me = reinterpret_cast<TieWarp *>(cd_smem + C::PACK + 4)[warp];
+        if (lane == 0) me.nev = 0;
         __syncwarp();
-        if (row_ok)
-            chg_decide_rec<B, FULL>(tri, a.d + a.b0, a.bw, a.maxq, s * s, a.rowdf != nullptr, lane, t, st, code, dlt,
-                                    dfacc, a.tie_eps, me.fj, me.fc, 0, -1, me.ev, &me.nev);
-        // a row without notes is final: it writes its results now, without waiting
-        const bool noted = row_ok && me.nev > 0;
-        if (row_ok && !noted) {
-            if (a.rowdf) {
-                dfacc = warp_sum(dfacc);
-                if (lane == 0) a.rowdf[i] += dfacc;
+        chg_decide_rec<B, FULL>(tri, a.d + a.b0, a.bw, a.maxq, s * s, a.rowdf != nullptr, lane, t, st, code, dlt,
+                                dfacc, a.tie_eps, me.fj, me.fc, 0, -1, me.ev, &me.nev);
+        const int nev = me.nev;
+        if (nev > 0) {
+            // the row waits for the check kernel: its notes, final and start codes to the queue,
+            // and what the check reads starts toward L2
+            int slot = 0;
+            if (lane == 0) slot = static_cast<int>(atomicAdd(a.tq_cnt, 1u));
+            slot = __shfl_sync(0xffffffffu, slot, 0);
+            const double dfw = warp_sum(dfacc);
+            TieEntry &e = a.tq[slot];
+            if (lane == 0) {
+                e.i = i;
+                e.df = dfw;
+                e.nev = nev;
             }
-            if (a.lent)
-                cd_epilogue<B, FULL, true>(a, a.b0, a.bw, i, lane, code, dlt, true);
-            else
-                cd_epilogue<B, FULL, false>(a, a.b0, a.bw, i, lane, code, dlt, true);
-        }
-        if (noted) {
-            // what the CTA-wide check reads starts toward L2 while the other rows decide
-            tie_prefetch_row(a, i, lane, 32);
-            const int ne = me.nev < kMaxEv ? me.nev : kMaxEv;
-            for (int e = 0; e < ne; ++e) tie_prefetch_srow(a, a.b0 + me.ev[e], lane, 32);
+            if (lane < kMaxEv) e.ev[lane] = me.ev[lane];
+            float *cr = a.tq_rows + static_cast<int64_t>(slot) * 2 * B, *sr = cr + B;
 #pragma unroll
             for (int h = 0; h < CPL; ++h) {
-                cr[warp * B + 32 * h + lane] = code[h];
-                sr[warp * B + 32 * h + lane] = st[h];
+                cr[32 * h + lane] = code[h];
+                sr[32 * h + lane] = st[h];
             }
+            tie_prefetch_row(a, i, lane, 32);
+            const int ne = nev < kMaxEv ? nev : kMaxEv;
+            for (int k = 0; k < ne; ++k) tie_prefetch_srow(a, a.b0 + me.ev[k], lane, 32);
+            return;
         }
-        if (__syncthreads_count(noted && lane == 0) == 0) return;   // no notes in this CTA
-        for (int round = 0; round <= kMaxForced; ++round) {
-            __syncthreads();
-            // check the notes, row by row, in order; the first wrong one stops its row's checks
-            bool any = false;
-            for (int w = 0; w < nw; ++w) {
-                const int64_t iw = static_cast<int64_t>(blockIdx.x) * nw + w;
-                if (iw >= a.q) break;
-                // (more than kMaxEv notes: the first kMaxEv, in column order, are checked)
-                const int n = tw[w].nev < kMaxEv ? tw[w].nev : kMaxEv;
-                for (int e = 0; e < n; ++e) {
-                    const int j = tw[w].ev[e];
-                    const double te = coop_tie_beta(a, iw, a.b0, bw, j, cr + w * B, sr + w * B, red);
-                    const float ce = tie_code(te, a.maxq);
-                    const bool wrong = ce != cr[w * B + j];
-                    if (wrong) {
-                        if (threadIdx.x == 0) {
-                            tw[w].wrong_j = j;
-                            tw[w].wrong_c = ce;
-                        }
-                        any = true;
-                        break;
-                    }
-                }
-            }
-            __syncthreads();
-            if (!any) break;
-            if (lane == 0 && me.wrong_j == -1) me.nev = 0;   // this row's notes all held
-            // rows with a wrong decision decide again from the block's start (R holds it)
-            if (row_ok && me.wrong_j != -1) {
-                const int wj = me.wrong_j;
-                __syncwarp();
-#pragma unroll
-                for (int h = 0; h < CPL; ++h) {
-                    const int l = 32 * h + lane;
-                    t[h] = (FULL || l < bw) ? a.R[i * a.ldr + a.b0 + l] : 0.0f;
-                }
-                dfacc = 0.0;
-                // force the exact code (a row whose kMaxForced forced decisions are used
-                // up keeps its last decisions: in practice never reached)
-                if (lane == 0) {
-                    if (me.nf < kMaxForced) {
-                        me.fj[me.nf] = wj;
-                        me.fc[me.nf] = me.wrong_c;
-                        me.nf += 1;
-                    }
-                    me.nev = 0;
-                    me.wrong_j = -1;
-                }
-                __syncwarp();
-                chg_decide_rec<B, FULL>(tri, a.d + a.b0, a.bw, a.maxq, s * s, a.rowdf != nullptr, lane, t, st, code,
-                                        dlt, dfacc, a.tie_eps, me.fj, me.fc, me.nf, wj, me.ev, &me.nev);
-                if (round == kMaxForced && lane == 0) me.nev = 0;
-                __syncwarp();
-                const int ne = me.nev < kMaxEv ? me.nev : kMaxEv;
-                for (int e = 0; e < ne; ++e) tie_prefetch_srow(a, a.b0 + me.ev[e], lane, 32);
-#pragma unroll
-                for (int h = 0; h < CPL; ++h) {
-                    cr[warp * B + 32 * h + lane] = code[h];
-                    sr[warp * B + 32 * h + lane] = st[h];
-                }
-            }
-        }
-        if (!noted) return;   // written above
     } else {
-        if (!cd_prologue<B, FULL>(a, tri, bar, i, row_ok, lane, t, st)) return;
-        if (!row_ok) return;
-        const float s = a.scale[i * a.ngroups + a.b0 / a.gsize];
         chg_decide<B, FULL>(tri, a.d + a.b0, a.bw, a.maxq, s * s, a.rowdf != nullptr, lane, t, st, code, dlt, dfacc);
     }
     if (a.rowdf) {
         dfacc = warp_sum(dfacc);
         if (lane == 0) a.rowdf[i] += dfacc;
     }
-    if (a.lent)
-        cd_epilogue<B, FULL, true>(a, a.b0, a.bw, i, lane, code, dlt, true);
-    else
-        cd_epilogue<B, FULL, false>(a, a.b0, a.bw, i, lane, code, dlt, true);
+    chg_write<B, FULL>(a, i, lane, code, dlt);
+}
+
+// Shared memory of the check kernel: the packed block (copied only when a row must
+// decide again) and its barrier, the entry's final and start codes, the forced
+// decisions and notes, the reduction slots of the CTA-wide recompute.
+template <int B>
+__host__ __device__ constexpr int tie_check_smem_bytes() {
+    return (CdCfg<B>::PACK + 4) * 4 + 2 * B * 4 + static_cast<int>(sizeof(TieWarp)) + 34 * 8;
+}
+
+// The near-tie check after a change-driven launch (same arguments): each CTA takes
+// queued rows in turn.  A row's notes are checked in column order against beta~
+// recomputed exactly by the whole CTA (coop_tie_beta, over the row's state at that
+// decision: columns before it final, after it at their start codes); at the first
+// wrong one the row decides again from the block's start (R holds it) with that
+// column forced, and its new notes are checked in the next round (at most
+// kMaxForced forced decisions; a row that uses them up keeps its last decisions, in
+// practice never reached).  Then the row's results are written.  The last CTA out
+// resets the queue's counters.
+template <int B, bool FULL>
+__global__ void __launch_bounds__(1024, 1) k_cd_tie_check(const __grid_constant__ CdArgs a) {
+    if (a.gate && *a.gate != a.gate_run) return;   // uniform: the list form of the sweep runs
+    using C = CdCfg<B>;
+    constexpr int CPL = C::CPL;
+    extern __shared__ __align__(16) float cd_smem[];
+    float *tri = cd_smem;
+    uint64_t *bar = reinterpret_cast<uint64_t *>(cd_smem + C::PACK);
+    float *cr = cd_smem + C::PACK + 4, *sr = cr + B;
+    TieWarp *me = reinterpret_cast<TieWarp *>(sr + B);
+    double *red = reinterpret_cast<double *>(me + 1);
+    __shared__ int s_copy;   // 0: block not copied, 1: copied and landed, -1: the wait gave up
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int bw = FULL ? B : a.bw;
+    const int n = static_cast<int>(a.tq_cnt[0]);
+    if (threadIdx.x == 0) {
+        s_copy = 0;
+        mbar_init(bar, 1);
+        fence_mbar_init();
+    }
+    __syncthreads();
+    const unsigned long long lim = a.wait_ns ? a.wait_ns : kWaitLimitNs;
+    for (int e = blockIdx.x; e < n && s_copy >= 0; e += gridDim.x) {
+        const TieEntry &E = a.tq[e];
+        const int64_t i = E.i;
+        const float *gcr = a.tq_rows + static_cast<int64_t>(e) * 2 * B;
+        for (int l = threadIdx.x; l < B; l += blockDim.x) {
+            cr[l] = gcr[l];
+            sr[l] = gcr[B + l];
+        }
+        if (threadIdx.x == 0) {
+            me->nev = E.nev;
+            for (int k = 0; k < kMaxEv; ++k) me->ev[k] = E.ev[k];
+            me->nf = 0;
+            me->wrong_j = -1;
+        }
+        double df = E.df;
+        __syncthreads();
+        for (int round = 0; round <= kMaxForced; ++round) {
+            // the notes in column order; the first wrong one stops the checks
+            const int ne = me->nev < kMaxEv ? me->nev : kMaxEv;
+            bool wrong = false;
+            for (int k = 0; k < ne && !wrong; ++k) {
+                const int j = me->ev[k];
+                const double te = coop_tie_beta(a, i, a.b0, bw, j, cr, sr, red);
+                const float ce = tie_code(te, a.maxq);
+                if (ce != cr[j]) {
+                    wrong = true;
+                    if (threadIdx.x == 0) {
+                        me->wrong_j = j;
+                        me->wrong_c = ce;
+                    }
+                }
+            }
+            if (!wrong) break;
+            // the packed block, once per CTA, for the rows that decide again
+            if (s_copy == 0) {
+                if (threadIdx.x == 0 && !a.skip_copy) {
+                    constexpr uint32_t bytes = C::PACK * 4;
+                    mbar_arrive_expect_tx(bar, bytes);
+                    bulk_load(tri, a.tri + (a.b0 / B) * C::PACK, bytes, bar);
+                }
+                const bool ok = mbar_wait_bounded_ns(bar, 0u, nullptr, lim);
+                __syncthreads();   // every thread has read s_copy == 0 and waited
+                if (threadIdx.x == 0) {
+                    s_copy = ok ? 1 : -1;
+                    if (!ok) set_error(a.err, ERR_TIMEOUT);
+                }
+                __syncthreads();
+                if (s_copy < 0) break;
+            }
+            if (warp == 0) {
+                __syncwarp();
+                const int wj = me->wrong_j;
+                __syncwarp();
+                if (lane == 0) {
+                    if (me->nf < kMaxForced) {
+                        me->fj[me->nf] = wj;
+                        me->fc[me->nf] = me->wrong_c;
+                        me->nf += 1;
+                    }
+                    me->nev = 0;
+                    me->wrong_j = -1;
+                }
+                __syncwarp();
+                float t[CPL], st[CPL], code[CPL], dlt[CPL];
+#pragma unroll
+                for (int h = 0; h < CPL; ++h) {
+                    const int l = 32 * h + lane;
+                    t[h] = (FULL || l < bw) ? a.R[i * a.ldr + a.b0 + l] : 0.0f;
+                    st[h] = sr[l];
+                }
+                const float s = a.scale[i * a.ngroups + a.b0 / a.gsize];
+                double dfacc = 0.0;
+                chg_decide_rec<B, FULL>(tri, a.d + a.b0, a.bw, a.maxq, s * s, a.rowdf != nullptr, lane, t, st, code,
+                                        dlt, dfacc, a.tie_eps, me->fj, me->fc, me->nf, wj, me->ev, &me->nev);
+                if (round == kMaxForced && lane == 0) me->nev = 0;
+                df = warp_sum(dfacc);
+#pragma unroll
+                for (int h = 0; h < CPL; ++h) cr[32 * h + lane] = code[h];
+                __syncwarp();
+            }
+            __syncthreads();
+        }
+        if (s_copy < 0) break;
+        // the row's results
+        if (warp == 0) {
+            float code[CPL], dlt[CPL];
+#pragma unroll
+            for (int h = 0; h < CPL; ++h) {
+                const int l = 32 * h + lane;
+                code[h] = cr[l];
+                dlt[h] = sr[l] - code[h];
+            }
+            if (a.rowdf && lane == 0) a.rowdf[i] += df;
+            chg_write<B, FULL>(a, i, lane, code, dlt);
+        }
+        __syncthreads();   // cr, sr and the notes are rewritten for the next row
+    }
+    if (threadIdx.x == 0) {
+        // an issued copy has landed before the CTA leaves (bounded once more after a
+        // wait that gave up)
+        if (s_copy < 0 && !a.skip_copy) mbar_wait_bounded_ns(bar, 0u, nullptr, lim);
+        // the last CTA out resets the queue for the next launch
+        __threadfence();
+        if (atomicAdd(a.tq_cnt + 1, 1u) == gridDim.x - 1) {
+            a.tq_cnt[0] = 0u;
+            a.tq_cnt[1] = 0u;
+            __threadfence();
+        }
+    }
+}
+
+template <int B, bool FULL>
+static cudaError_t launch_cd_tie_check_b(const CdArgs &a, int nsm, cudaStream_t s) {
+    constexpr int smem = tie_check_smem_bytes<B>();
+    cudaError_t e = cudaFuncSetAttribute(k_cd_tie_check<B, FULL>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    k_cd_tie_check<B, FULL><<<static_cast<unsigned>(nsm), 1024, smem, s>>>(a);
+    return cudaGetLastError();
 }
 
 // One block of one row in the persistent list kernel (R and the codes stream with
@@ -1447,16 +1534,22 @@ static cudaError_t launch_cd_block_b(const CdArgs &a, int nsm, cudaStream_t s) {
     if (warps < 1) warps = 1;
     // the sequential kernel keeps one row of beta~ per warp (DF), and one row of the
     // codes decided in the visit and one snapshot row (near-tie refinement), after the
-    // packed block
-    // (the change-driven kernel keeps one row per warp for the refinement)
+    // packed block; the change-driven kernel the notes of each warp's row
     const int rows = static_cast<int>(warps) * B * 4;
     const int smem = SEQ ? (C::PACK + 4) * 4 + (DF ? rows : 0) + (TIE ? 2 * rows : 0)
-                         : (C::PACK + 4) * 4 + (TIE ? tie_cta_bytes<B>(static_cast<int>(warps)) : 0);
+                         : (C::PACK + 4) * 4 + (TIE ? static_cast<int>(warps) * static_cast<int>(sizeof(TieWarp)) : 0);
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     const unsigned grid = static_cast<unsigned>(ceil_div(a.q, warps));
     kern<<<grid, static_cast<unsigned>(32 * warps), smem, s>>>(a);
     return cudaGetLastError();
+}
+
+// The near-tie check after a change-driven launch with the refinement.
+template <int B, bool FULL>
+static cudaError_t launch_cd_tie_check_f(const CdArgs &a, int nsm, cudaStream_t s) {
+    if (!a.tq || !a.tq_rows || !a.tq_cnt) return cudaErrorInvalidValue;
+    return launch_cd_tie_check_b<B, FULL>(a, nsm, s);
 }
 
 // The change-driven kernel (integer changes, !a.frac), with or without the
@@ -1488,6 +1581,12 @@ cudaError_t launch_cd_block_k(const CdArgs &a, int nsm, cudaStream_t s) {
         return launch_cd_block_seq_f<B, FULL>(a, nsm, s);
     else
         return launch_cd_block_chg_f<B, FULL>(a, nsm, s);
+}
+
+// The near-tie check at block width B (instantiated with the change-driven kernel).
+template <int B, bool FULL>
+cudaError_t launch_cd_tie_check_k(const CdArgs &a, int nsm, cudaStream_t s) {
+    return launch_cd_tie_check_f<B, FULL>(a, nsm, s);
 }
 
 template <int B, bool GR, bool TIE>
@@ -1537,6 +1636,12 @@ extern template cudaError_t launch_cd_block_k<256, false, true> QE_SWEEP_BLOCK_S
 extern template cudaError_t launch_cd_block_k<64, false, false> QE_SWEEP_BLOCK_SIG;
 extern template cudaError_t launch_cd_block_k<128, false, false> QE_SWEEP_BLOCK_SIG;
 extern template cudaError_t launch_cd_block_k<256, false, false> QE_SWEEP_BLOCK_SIG;
+extern template cudaError_t launch_cd_tie_check_k<64, true> QE_SWEEP_BLOCK_SIG;
+extern template cudaError_t launch_cd_tie_check_k<64, false> QE_SWEEP_BLOCK_SIG;
+extern template cudaError_t launch_cd_tie_check_k<128, true> QE_SWEEP_BLOCK_SIG;
+extern template cudaError_t launch_cd_tie_check_k<128, false> QE_SWEEP_BLOCK_SIG;
+extern template cudaError_t launch_cd_tie_check_k<256, true> QE_SWEEP_BLOCK_SIG;
+extern template cudaError_t launch_cd_tie_check_k<256, false> QE_SWEEP_BLOCK_SIG;
 extern template cudaError_t launch_cd_rows_k<64> QE_SWEEP_ROWS_SIG;
 extern template cudaError_t launch_cd_rows_k<128> QE_SWEEP_ROWS_SIG;
 extern template cudaError_t launch_cd_rows_k<256> QE_SWEEP_ROWS_SIG;
