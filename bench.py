@@ -198,8 +198,8 @@ class ClockSampler:
 
 # Committed DRAM-traffic figures (profiles/roofline_traffic.json): per kernel, the
 # bytes one launch moved in one ncu capture, keyed by a hash of the sources the
-# kernel is compiled from; null once those sources change.
-TRAFFIC_SOURCES = ("qe_api.cu", "qe_cd.cu", "qe_sweep.cuh", "qe_common.cuh", "qe_gemm.cu", "qe_internal.h", "qe_kernels.h")
+# tensor-core GEMM is compiled from and launched by; null once those sources change.
+TRAFFIC_SOURCES = ("qe_api.cu", "qe_common.cuh", "qe_gemm.cu", "qe_internal.h", "qe_kernels.h")
 
 
 def traffic_sources_sha256() -> str:
@@ -629,10 +629,10 @@ def main():
                                          "grids; ceiling of the algorithmic fraction about 1/2"))
     # (3) k_tc_gemm<256> over all its launches in a step (Sigma + the CD GEMMs)
     gemm_ms = sigma_avg + gemm_cd_ms
-    tr, tr_note = traffic_record("k_tc_gemm_trail", cfg.name)
+    tr, tr_note = traffic_record("k_tc_gemm_step", cfg.name)
     r_gemm = roofline_tensor("k_tc_gemm<256> (Sigma, P, residual, trailing)", sig_flops + gemm_cd_alg,
                              sig_exec + gemm_cd_exec, gemm_ms, 1 + gemm_cd_launches, peak_tc, peak_src,
-                             tr, (tr_note + "; trailing-correction launches") if tr else tr_note)
+                             tr, tr_note)
     # (4) the change-list kernel against HBM (when lists ran)
     list_launches, list_ms = timed[qe.QE_KERNEL_CD_LISTS]
     n_list = sum(sc["sweeps_by_form"]["list"] for sc in sched)

@@ -714,16 +714,17 @@ static bool sbar_rows_fit_l2(int64_t p, int64_t ld) {
 }
 
 // The adaptive schedule's switch threshold for layers whose Sigma_bar rows exceed
-// L2: a dense sweep costs its 6 q p^2 flops of bf16 plane products (~1.3 PFLOP/s
-// on 152 SMs, as measured for the trailing GEMMs) plus an in-block pass (~42 ps
-// per coordinate); a list sweep gathers one Sigma_bar row of 4 p bytes per change
-// (~8 TB/s from DRAM and L2 together, measured on the 14848 x 59392 layer); the
-// next sweep makes about 0.7 times the changes of the one just finished.
+// L2: a dense sweep costs its window GEMMs, 2 q p^2 flops of two fp16 products each
+// (~1.2 PFLOP/s on 152 SMs as measured on the 15360 x 14848 layer), plus an
+// in-block pass with its near-tie checks (~35 ps per coordinate); a list sweep
+// gathers one Sigma_bar row of 4 p bytes per change (~4.75 TB/s measured on the
+// same layer); the next sweep makes about 0.8 times the changes of the one just
+// finished.
 static int64_t switch_below_model(int64_t q, int64_t p, int nsm) {
     const double qd = static_cast<double>(q), pd = static_cast<double>(p);
-    const double t_dense = 6.0 * qd * pd * pd / (1.3e15 * nsm / 152.0) + 4.2e-11 * qd * pd;
-    const double t_change = 4.0 * pd / 8.0e12;
-    const double below = t_dense / t_change / 0.7;
+    const double t_dense = 4.0 * qd * pd * pd / (1.2e15 * nsm / 152.0) + 3.5e-11 * qd * pd;
+    const double t_change = 4.0 * pd / 4.75e12;
+    const double below = t_dense / t_change / 0.8;
     return below > 9.0e18 ? static_cast<int64_t>(9.0e18) : static_cast<int64_t>(below);
 }
 

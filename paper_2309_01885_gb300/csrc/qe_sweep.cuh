@@ -1527,7 +1527,10 @@ template <int B, bool FULL, bool SEQ, bool RELAX = false, bool DF = false, bool 
 static cudaError_t launch_cd_block_b(const CdArgs &a, int nsm, cudaStream_t s) {
     using C = CdCfg<B>;
     if (a.nsplit > C::MAX_SPLITS) return cudaErrorInvalidValue;
-    auto kern = SEQ ? k_cd_block_seq<B, FULL, RELAX, DF, TIE> : k_cd_block_chg<B, FULL, TIE>;
+    auto kern = [] {
+        if constexpr (SEQ) return k_cd_block_seq<B, FULL, RELAX, DF, TIE>;
+        else return k_cd_block_chg<B, FULL, TIE>;
+    }();
     // one CTA per SM when the rows allow it (the packed block is shared by the CTA's rows)
     int64_t warps = ceil_div(a.q, nsm);
     if (warps > C::MAX_WARPS) warps = C::MAX_WARPS;
