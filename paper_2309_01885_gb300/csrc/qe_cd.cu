@@ -162,9 +162,30 @@ __global__ void __launch_bounds__(256) k_sigma_planes_h2(const float *S, int64_t
     for (int64_t j = blockIdx.x; j < p; j += gridDim.x) {
         const float dj = d[j];
         const bool jalive = dj > 0.0f;
+        // max_k |S_jk| / d_j over the live k != j: a correctly rounded division by d_j > 0
+        // keeps the order, so the largest |S_jk| is divided once (16-byte loads where the
+        // row allows)
         float mx = 0.0f;
-        for (int64_t k = threadIdx.x; k < p; k += blockDim.x)
-            if (jalive && k != j && d[k] > 0.0f) mx = fmaxf(mx, fabsf(__fdiv_rn(S[j * lds + k], dj)));
+        if (jalive) {
+            const float *row = S + j * lds;
+            int64_t k = 0;
+            if ((lds & 3) == 0 && (reinterpret_cast<uintptr_t>(S) & 15u) == 0 &&
+                (reinterpret_cast<uintptr_t>(d) & 15u) == 0) {
+                const int64_t p4 = p >> 2;
+                for (int64_t k4 = threadIdx.x; k4 < p4; k4 += blockDim.x) {
+                    const float4 v = reinterpret_cast<const float4 *>(row)[k4];
+                    const float4 dd = reinterpret_cast<const float4 *>(d)[k4];
+                    const int64_t kb = 4 * k4;
+                    if (kb != j && dd.x > 0.0f) mx = fmaxf(mx, fabsf(v.x));
+                    if (kb + 1 != j && dd.y > 0.0f) mx = fmaxf(mx, fabsf(v.y));
+                    if (kb + 2 != j && dd.z > 0.0f) mx = fmaxf(mx, fabsf(v.z));
+                    if (kb + 3 != j && dd.w > 0.0f) mx = fmaxf(mx, fabsf(v.w));
+                }
+                k = 4 * p4;
+            }
+            for (k += threadIdx.x; k < p; k += blockDim.x)
+                if (k != j && d[k] > 0.0f) mx = fmaxf(mx, fabsf(row[k]));
+        }
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
         if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = mx;
@@ -172,19 +193,59 @@ __global__ void __launch_bounds__(256) k_sigma_planes_h2(const float *S, int64_t
         mx = 0.0f;
         for (int w = 0; w < 8; ++w) mx = fmaxf(mx, red[w]);
         __syncthreads();   // red is rewritten for the next row
+        if (jalive) mx = __fdiv_rn(mx, dj);
         // 2^e with mx 2^e in [2^14, 2^15) (finite mx; e = 0 for an all-zero row)
         int e = 0;
         if (mx > 0.0f && isfinite(mx)) e = 14 - ilogbf(mx);
         if (e > 100) e = 100;
         if (e < -100) e = -100;
         if (threadIdx.x == 0) cscale[j] = ldexpf(1.0f, -e);
-        for (int64_t k = threadIdx.x; k < ldn; k += blockDim.x) {
-            float x = 0.0f;
-            if (k < p && jalive && k != j && d[k] > 0.0f) x = ldexpf(__fdiv_rn(S[j * lds + k], dj), e);
-            const __half hi = __float2half_rn(x);
-            const __half lo = __float2half_rn(x - __half2float(hi));
-            snh[j * ldn + k] = hi;
-            snh[(p + j) * ldn + k] = lo;
+        if ((ldn & 3) == 0 && (lds & 3) == 0 && (reinterpret_cast<uintptr_t>(S) & 15u) == 0 &&
+            (reinterpret_cast<uintptr_t>(d) & 15u) == 0 && (reinterpret_cast<uintptr_t>(snh) & 7u) == 0) {
+            // four columns per thread: 16-byte loads, 8-byte stores of each plane
+            const float *row = S + j * lds;
+            for (int64_t k4 = threadIdx.x; k4 < (ldn >> 2); k4 += blockDim.x) {
+                const int64_t kb = 4 * k4;
+                float v[4] = {0.0f, 0.0f, 0.0f, 0.0f}, dd[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+                if (jalive && kb + 3 < p) {
+                    const float4 v4 = reinterpret_cast<const float4 *>(row)[k4];
+                    const float4 d4 = reinterpret_cast<const float4 *>(d)[k4];
+                    v[0] = v4.x; v[1] = v4.y; v[2] = v4.z; v[3] = v4.w;
+                    dd[0] = d4.x; dd[1] = d4.y; dd[2] = d4.z; dd[3] = d4.w;
+                } else if (jalive) {
+                    for (int u = 0; u < 4; ++u)
+                        if (kb + u < p) {
+                            v[u] = row[kb + u];
+                            dd[u] = d[kb + u];
+                        }
+                }
+                __half hi[4], lo[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    float x = 0.0f;
+                    if (kb + u < p && jalive && kb + u != j && dd[u] > 0.0f) x = ldexpf(__fdiv_rn(v[u], dj), e);
+                    hi[u] = __float2half_rn(x);
+                    lo[u] = __float2half_rn(x - __half2float(hi[u]));
+                }
+                const __half2 h01 = __halves2half2(hi[0], hi[1]), h23 = __halves2half2(hi[2], hi[3]);
+                const __half2 l01 = __halves2half2(lo[0], lo[1]), l23 = __halves2half2(lo[2], lo[3]);
+                uint2 ph, pl;
+                ph.x = *reinterpret_cast<const unsigned *>(&h01);
+                ph.y = *reinterpret_cast<const unsigned *>(&h23);
+                pl.x = *reinterpret_cast<const unsigned *>(&l01);
+                pl.y = *reinterpret_cast<const unsigned *>(&l23);
+                *reinterpret_cast<uint2 *>(snh + j * ldn + kb) = ph;
+                *reinterpret_cast<uint2 *>(snh + (p + j) * ldn + kb) = pl;
+            }
+        } else {
+            for (int64_t k = threadIdx.x; k < ldn; k += blockDim.x) {
+                float x = 0.0f;
+                if (k < p && jalive && k != j && d[k] > 0.0f) x = ldexpf(__fdiv_rn(S[j * lds + k], dj), e);
+                const __half hi = __float2half_rn(x);
+                const __half lo = __float2half_rn(x - __half2float(hi));
+                snh[j * ldn + k] = hi;
+                snh[(p + j) * ldn + k] = lo;
+            }
         }
     }
 }
