@@ -446,75 +446,6 @@ __device__ __forceinline__ float tie_code(double t, float maxq) {
     return static_cast<float>(rint(fmin(fmax(t, 0.0), static_cast<double>(maxq))));
 }
 
-// CTA-wide: beta~ / s + z of column b0 + j of row i at its decision: the block's
-// columns before j from cr (final codes), after j from sr (start codes), the rest
-// from the codes in global memory.  Every thread of the CTA calls it; red holds
-// 34 doubles of shared memory.  Returns the same value in every thread.
-template <int U = 8>
-__device__ __forceinline__ double coop_tie_beta(const CdArgs &a, int64_t i, int64_t b0, int bw, int j,
-                                                const float *cr, const float *sr, double *red) {
-    const int tid = threadIdx.x, nth = blockDim.x;
-    const int64_t jg = b0 + j;
-    const float *Srow = a.S + jg * a.lds_full;
-    const float *sc = a.scale + i * a.ngroups;
-    const float *zc = a.zero + i * a.ngroups;
-    const bool grouped = a.ngroups > 1;
-    const uint32_t gs = static_cast<uint32_t>(a.gsize);
-    const uint8_t *crow = a.codes + i * a.ldc;
-    const float *hrow = a.Hd ? a.Hd + i * a.ldh : nullptr;
-    float hi = 0.0f, lo = 0.0f;
-    // U columns per thread in flight: all their loads are issued before the sums
-    for (int64_t k0 = tid; k0 < a.p; k0 += static_cast<int64_t>(nth) * U) {
-        float cv[U], wv[U], hv[U], sv[U];
-#pragma unroll
-        for (int u = 0; u < U; ++u) {
-            const int64_t k = k0 + static_cast<int64_t>(u) * nth;
-            cv[u] = wv[u] = hv[u] = sv[u] = 0.0f;
-            // in the first sweep the columns after j (in the block and beyond it) still
-            // hold T itself and add nothing
-            bool use = k < a.p;
-            if (use) {
-                if (k >= b0 && k < b0 + bw) {
-                    const int l = static_cast<int>(k - b0);
-                    use = !(a.first_sweep && l > j);
-                    if (use) cv[u] = l < j ? cr[l] : sr[l];
-                } else {
-                    use = !a.first_sweep || k < b0;
-                    if (use) cv[u] = static_cast<float>(crow[k]);
-                }
-            }
-            if (use) {
-                wv[u] = tie_w(a, i, k);
-                if (hrow) hv[u] = hrow[k];
-                sv[u] = (k == jg) ? 0.0f : Srow[k];   // column j itself is left out
-            }
-        }
-#pragma unroll
-        for (int u = 0; u < U; ++u) {
-            const int64_t k = k0 + static_cast<int64_t>(u) * nth;
-            if (k >= a.p) continue;
-            if (sv[u] == 0.0f) continue;   // a term that adds nothing (its S is zero or left out)
-            const uint32_t g = grouped ? static_cast<uint32_t>(k) / gs : 0u;
-            df_term(hi, lo, wv[u], hv[u], sc[g], cv[u] - zc[g], sv[u]);
-        }
-    }
-    double acc = warp_sum(static_cast<double>(hi) + static_cast<double>(lo));
-    if ((tid & 31) == 0) red[tid >> 5] = acc;
-    __syncthreads();
-    if (tid == 0) {
-        double sum = 0.0;
-        for (int w = 0; w < (nth >> 5); ++w) sum += red[w];
-        double tj = static_cast<double>(tie_w(a, i, jg));
-        if (hrow) tj -= static_cast<double>(hrow[jg]);
-        const double dj = static_cast<double>(Srow[jg]);
-        const uint32_t g = grouped ? static_cast<uint32_t>(jg) / gs : 0u;
-        const double beta = dj > 0.0 ? tj + sum / dj : tj;
-        red[32] = beta / static_cast<double>(sc[g]) + static_cast<double>(zc[g]);
-    }
-    __syncthreads();
-    return red[32];
-}
-
 // Sequential in-block kernel (sweeps where every column moves by a real
 // amount: the first sweep, a relaxed sweep and the sweep after one).
 // One warp per row; column j = 32 h + jj is decided by lane jj, which keeps
@@ -542,22 +473,11 @@ __global__ void __launch_bounds__(1024) k_cd_block_seq(const __grid_constant__ C
     // near-tie refinement (after the DF rows)
     float *cdec = cd_smem + C::PACK + 4 + (DF ? (blockDim.x >> 5) * B : 0) + 2 * warp * B;
     float *snap = cdec + B;
-    const int nw = static_cast<int>(blockDim.x >> 5);
-    const int64_t i = static_cast<int64_t>(blockIdx.x) * nw + warp;
+    const int64_t i = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + warp;
     const bool row_ok = i < a.q;
-    // near-tie refinement: only in the first sweep (RELAX and a real-valued start turn it
-    // off); CTA-uniform, and then every warp of the CTA takes part in its barriers
-    const bool tie = TIE && !RELAX && a.tie_eps > 0.0f && a.first_sweep && !a.vstart;
-    __shared__ int s_jt[32];        // per warp: its first near tie of the word, or -1
-    __shared__ double s_te[32];     // beta~ / s + z of that column, recomputed exactly
-    __shared__ double s_red[34];    // reduction slots of the CTA-wide recompute
     float t[CPL], st[CPL];
-    const bool ok = cd_prologue<B, FULL>(a, tri, bar, i, row_ok, lane, t, st);
-    if (tie) {
-        if (__syncthreads_or(!ok)) return;   // a wait gave up somewhere: every warp leaves
-    } else if (!ok || !row_ok) {
-        return;
-    }
+    if (!cd_prologue<B, FULL>(a, tri, bar, i, row_ok, lane, t, st)) return;
+    if (!row_ok) return;
     const int bw = FULL ? B : a.bw;
     const float maxq = a.maxq;
     uint32_t live = 0u;   // bit h: this lane's column 32 h + lane has Sigma_jj > 0
@@ -566,6 +486,8 @@ __global__ void __launch_bounds__(1024) k_cd_block_seq(const __grid_constant__ C
         for (int h = 0; h < CPL; ++h)
             if ((FULL || 32 * h + lane < bw) && a.d[a.b0 + 32 * h + lane] > 0.0f) live |= 1u << h;
     }
+    // near-tie refinement: only in the first sweep (RELAX and a real-valued start turn it off)
+    const bool tie = TIE && !RELAX && a.tie_eps > 0.0f && a.first_sweep && !a.vstart;
     float code[CPL], dlt[CPL];
 #pragma unroll
     for (int h = 0; h < CPL; ++h) {
@@ -575,104 +497,83 @@ __global__ void __launch_bounds__(1024) k_cd_block_seq(const __grid_constant__ C
 #pragma unroll
     for (int h = 0; h < CPL; ++h) {
         // The word's 32 columns in order.  The deciding lane notes whether its value
-        // sat within tie_eps of a midpoint (off the sequential chain).  After the word
-        // the CTA meets: the first such column of every warp is decided again from
-        // beta~ recomputed exactly by the whole CTA (each note in turn); those warps
+        // sat within tie_eps of a midpoint (off the sequential chain); after the word,
+        // the first such column is decided again from the binary64 beta~: the lanes
         // restore the values of the snapshot taken before the pass, replay the
         // decisions before that column (the same arithmetic, so the same results),
-        // decide it exactly and resume after it, until no warp has a note left.
+        // decide it exactly and resume after it.
         int start = 0;
-        bool wdone = !row_ok;   // this warp's word is final
         while (true) {
-            int jt = -1;
-            if (!wdone) {
-                if (tie) {
+            if (tie) {
 #pragma unroll
-                    for (int g = h; g < CPL; ++g) snap[32 * g + lane] = t[g];
-                }
-                bool mynear = false;
-#pragma unroll
-                for (int jj = 0; jj < 32; ++jj) {
-                    if (jj < start) continue;
-                    const int j = 32 * h + jj;
-                    if (!FULL && j >= bw) break;
-                    const float cq = rintf(fminf(fmaxf(t[h], 0.0f), maxq));
-                    const float c = (RELAX && ((live >> h) & 1u)) ? t[h] : cq;
-                    const float dl = st[h] - c;
-                    if (lane == jj) {
-                        code[h] = c;
-                        dlt[h] = dl;
-                        if (DF) tdec[j] = t[h];
-                        if (tie) {
-                            cdec[j] = c;
-                            mynear = fabsf(fabsf(t[h] - cq) - 0.5f) < a.tie_eps;
-                        }
-                    }
-                    const float db = __shfl_sync(0xffffffffu, dl, jj);
-                    if (db != 0.0f) {
-                        const float *row = tri + kPackPad + tri_off(B, j) - (j + 1);
-#pragma unroll
-                        for (int g = h; g < CPL; ++g) t[g] = fmaf(db, row[32 * g + lane], t[g]);
-                    }
-                }
-                const unsigned nb = __ballot_sync(0xffffffffu, mynear);
-                if (nb == 0u) wdone = true;
-                else jt = __ffs(nb) - 1;
+                for (int g = h; g < CPL; ++g) snap[32 * g + lane] = t[g];
             }
-            if (!tie) break;
-            if (lane == 0) s_jt[warp] = jt;
-            __syncthreads();
-            bool any = false;
-            for (int w = 0; w < nw; ++w) {
-                const int jw = s_jt[w];
-                if (jw < 0) continue;
-                any = true;
-                const float *cw = cd_smem + C::PACK + 4 + (DF ? nw * B : 0) + 2 * w * B;
-                const int64_t iw = static_cast<int64_t>(blockIdx.x) * nw + w;
-                const double te = coop_tie_beta<2>(a, iw, a.b0, bw, 32 * h + jw, cw, cw, s_red);
-                if (threadIdx.x == 0) s_te[w] = te;
-            }
-            __syncthreads();   // s_te is read below; s_jt is rewritten at the next meeting
-            if (!any) break;
-            if (jt >= 0) {
+            bool mynear = false;
 #pragma unroll
-                for (int g = h; g < CPL; ++g) t[g] = snap[32 * g + lane];
-#pragma unroll
-                for (int jj = 0; jj < 32; ++jj) {   // replay the columns before jt
-                    if (jj < start) continue;
-                    if (jj >= jt) break;
-                    const int j = 32 * h + jj;
-                    const float c = rintf(fminf(fmaxf(t[h], 0.0f), maxq));
-                    const float dl = st[h] - c;
-                    const float db = __shfl_sync(0xffffffffu, dl, jj);
-                    if (db != 0.0f) {
-                        const float *row = tri + kPackPad + tri_off(B, j) - (j + 1);
-#pragma unroll
-                        for (int g = h; g < CPL; ++g) t[g] = fmaf(db, row[32 * g + lane], t[g]);
-                    }
-                }
-                // column 32 h + jt from the binary64 beta~ of the row's state
-                const int j = 32 * h + jt;
-                const double te = s_te[warp];
-                const float c = tie_code(te, maxq);
-                const float dl = __shfl_sync(0xffffffffu, st[h], jt) - c;
-                if (lane == jt) {
+            for (int jj = 0; jj < 32; ++jj) {
+                if (jj < start) continue;
+                const int j = 32 * h + jj;
+                if (!FULL && j >= bw) break;
+                const float cq = rintf(fminf(fmaxf(t[h], 0.0f), maxq));
+                const float c = (RELAX && ((live >> h) & 1u)) ? t[h] : cq;
+                const float dl = st[h] - c;
+                if (lane == jj) {
                     code[h] = c;
                     dlt[h] = dl;
-                    if (DF) tdec[j] = static_cast<float>(te);
-                    cdec[j] = c;
+                    if (DF) tdec[j] = t[h];
+                    if (tie) {
+                        cdec[j] = c;
+                        mynear = fabsf(fabsf(t[h] - cq) - 0.5f) < a.tie_eps;
+                    }
                 }
-                if (dl != 0.0f) {
+                const float db = __shfl_sync(0xffffffffu, dl, jj);
+                if (db != 0.0f) {
                     const float *row = tri + kPackPad + tri_off(B, j) - (j + 1);
 #pragma unroll
-                    for (int g = h; g < CPL; ++g) t[g] = fmaf(dl, row[32 * g + lane], t[g]);
+                    for (int g = h; g < CPL; ++g) t[g] = fmaf(db, row[32 * g + lane], t[g]);
                 }
-                start = jt + 1;
-                if (start >= 32 || (!FULL && 32 * h + start >= bw)) wdone = true;
             }
+            if (!tie) break;
+            const unsigned nb = __ballot_sync(0xffffffffu, mynear);
+            if (nb == 0u) break;
+            const int jt = __ffs(nb) - 1;
+            __syncwarp();
+#pragma unroll
+            for (int g = h; g < CPL; ++g) t[g] = snap[32 * g + lane];
+#pragma unroll
+            for (int jj = 0; jj < 32; ++jj) {   // replay the columns before jt
+                if (jj < start) continue;
+                if (jj >= jt) break;
+                const int j = 32 * h + jj;
+                const float c = rintf(fminf(fmaxf(t[h], 0.0f), maxq));
+                const float dl = st[h] - c;
+                const float db = __shfl_sync(0xffffffffu, dl, jj);
+                if (db != 0.0f) {
+                    const float *row = tri + kPackPad + tri_off(B, j) - (j + 1);
+#pragma unroll
+                    for (int g = h; g < CPL; ++g) t[g] = fmaf(db, row[32 * g + lane], t[g]);
+                }
+            }
+            // column 32 h + jt from the binary64 beta~ of the row's state
+            const int j = 32 * h + jt;
+            const double te = tie_beta(&a, i, a.b0, bw, j, lane, cdec);
+            const float c = tie_code(te, maxq);
+            const float dl = __shfl_sync(0xffffffffu, st[h], jt) - c;
+            if (lane == jt) {
+                code[h] = c;
+                dlt[h] = dl;
+                if (DF) tdec[j] = static_cast<float>(te);
+                cdec[j] = c;
+            }
+            if (dl != 0.0f) {
+                const float *row = tri + kPackPad + tri_off(B, j) - (j + 1);
+#pragma unroll
+                for (int g = h; g < CPL; ++g) t[g] = fmaf(dl, row[32 * g + lane], t[g]);
+            }
+            start = jt + 1;
+            if (start >= 32 || (!FULL && 32 * h + start >= bw)) break;
         }
     }
-    if (!row_ok) return;
     if (DF) {
         __syncwarp();
         const float sc = a.scale[i * a.ngroups + a.b0 / a.gsize];
@@ -925,6 +826,66 @@ __device__ __forceinline__ void chg_decide_rec(const float *tri, const float *d_
     for (int h = 0; h < CPL; ++h) dlt[h] = st[h] - code[h];
 }
 
+// CTA-wide: beta~ / s + z of column b0 + j of row i at its decision: the block's
+// columns before j from cr (final codes), after j from sr (start codes), the rest
+// from the codes in global memory.  Every thread of the CTA calls it; red holds
+// 34 doubles of shared memory.  Returns the same value in every thread.
+__device__ __forceinline__ double coop_tie_beta(const CdArgs &a, int64_t i, int64_t b0, int bw, int j,
+                                                const float *cr, const float *sr, double *red) {
+    const int tid = threadIdx.x, nth = blockDim.x;
+    const int64_t jg = b0 + j;
+    const float *Srow = a.S + jg * a.lds_full;
+    const float *sc = a.scale + i * a.ngroups;
+    const float *zc = a.zero + i * a.ngroups;
+    const bool grouped = a.ngroups > 1;
+    const uint32_t gs = static_cast<uint32_t>(a.gsize);
+    const uint8_t *crow = a.codes + i * a.ldc;
+    const float *hrow = a.Hd ? a.Hd + i * a.ldh : nullptr;
+    float hi = 0.0f, lo = 0.0f;
+    // U columns per thread in flight: all their loads are issued before the sums
+    constexpr int U = 8;
+    for (int64_t k0 = tid; k0 < a.p; k0 += static_cast<int64_t>(nth) * U) {
+        float cv[U], wv[U], hv[U], sv[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int64_t k = k0 + static_cast<int64_t>(u) * nth;
+            cv[u] = wv[u] = hv[u] = sv[u] = 0.0f;
+            if (k < a.p) {
+                if (k >= b0 && k < b0 + bw) {
+                    const int l = static_cast<int>(k - b0);
+                    cv[u] = l < j ? cr[l] : sr[l];
+                } else {
+                    cv[u] = static_cast<float>(crow[k]);
+                }
+                wv[u] = tie_w(a, i, k);
+                if (hrow) hv[u] = hrow[k];
+                sv[u] = (k == jg) ? 0.0f : Srow[k];   // column j itself is left out
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int64_t k = k0 + static_cast<int64_t>(u) * nth;
+            if (k >= a.p) continue;
+            const uint32_t g = grouped ? static_cast<uint32_t>(k) / gs : 0u;
+            df_term(hi, lo, wv[u], hv[u], sc[g], cv[u] - zc[g], sv[u]);
+        }
+    }
+    double acc = warp_sum(static_cast<double>(hi) + static_cast<double>(lo));
+    if ((tid & 31) == 0) red[tid >> 5] = acc;
+    __syncthreads();
+    if (tid == 0) {
+        double sum = 0.0;
+        for (int w = 0; w < (nth >> 5); ++w) sum += red[w];
+        double tj = static_cast<double>(tie_w(a, i, jg));
+        if (hrow) tj -= static_cast<double>(hrow[jg]);
+        const double dj = static_cast<double>(Srow[jg]);
+        const uint32_t g = grouped ? static_cast<uint32_t>(jg) / gs : 0u;
+        const double beta = dj > 0.0 ? tj + sum / dj : tj;
+        red[32] = beta / static_cast<double>(sc[g]) + static_cast<double>(zc[g]);
+    }
+    __syncthreads();
+    return red[32];
+}
 
 // Notes of one warp's row in shared memory (the refinement variants).
 struct TieWarp {
