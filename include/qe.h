@@ -154,9 +154,10 @@ typedef struct {
      * take the decisions exact arithmetic takes).  A coordinate update rounds
      * beta~ / s + z (Lemma 1) to the nearest level; where that binary32 value
      * lies within tie_eps grid steps of a midpoint between two levels, the
-     * decision is taken again from beta~ recomputed in binary64 from the row's
-     * current codes, W (and H) and Sigma.  0 = default (1e-5, about four times
-     * the largest binary32 error measured on the benchmark layers); negative =
+     * decision is taken again from beta~ recomputed from the row's current
+     * codes, W (and H) and Sigma: every term exact, the sum in double-float
+     * (about 48 significant bits).  0 = default (1e-5, about four times the
+     * largest binary32 error measured on the benchmark layers); negative =
      * off.
      * Not applied in relaxed sweeps or the sweep after one. */
     float tie_eps;
